@@ -1,0 +1,118 @@
+"""Float64 CPU oracle for PnP-Nystra window attention (arXiv 2506.08520).
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import this package.  The product
+path (``paper_2506_08520_gb300``) never imports, links or runs it, and the
+two share no code: the oracle is plain C in ``nystra_oracle.c`` (Algorithm 1
+with the row-max stabilisation of Sec. 2.2, in float64), wrapped here with
+ctypes.
+
+Inputs may be numpy arrays or torch tensors of any float dtype; they are
+upcast exactly to float64.  Shapes are ``[..., N, d]`` with all leading axes
+flattened into independent units (one unit = one (window, head) pair).
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` against
+properties the paper or the mathematics fixes (brute force, exact recovery,
+the iteration's residual recursion, invariances, the spectral bound).
+"""
+import ctypes
+import numpy as np
+
+from . import build as _build
+
+_lib = None
+_D = ctypes.POINTER(ctypes.c_double)
+
+
+def _load():
+    global _lib
+    if _lib is None:
+        lib = ctypes.CDLL(_build.build())
+        lib.oracle_threads.restype = ctypes.c_int
+        lib.oracle_exact_attention.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int, ctypes.c_int]
+        lib.oracle_exact_attention.restype = None
+        lib.oracle_nystra_attention.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int,
+                                                ctypes.c_int, ctypes.c_int, ctypes.c_int]
+        lib.oracle_nystra_attention.restype = ctypes.c_int
+        lib.oracle_landmarks.argtypes = [_D, ctypes.c_int, ctypes.c_int, ctypes.c_int, _D]
+        lib.oracle_landmarks.restype = None
+        lib.oracle_pinv_iteration.argtypes = [_D, ctypes.c_int, ctypes.c_int, _D]
+        lib.oracle_pinv_iteration.restype = None
+        lib.oracle_nystra_stages.argtypes = [_D, _D, _D, _D, ctypes.c_int, ctypes.c_int,
+                                             ctypes.c_int, ctypes.c_int] + [_D] * 10
+        lib.oracle_nystra_stages.restype = ctypes.c_int
+        _lib = lib
+    return _lib
+
+
+def _f64(x) -> np.ndarray:
+    if hasattr(x, "detach"):  # torch tensor: exact upcast, then to numpy
+        x = x.detach().to("cpu").double().numpy()
+    return np.ascontiguousarray(np.asarray(x, dtype=np.float64))
+
+
+def _p(a: np.ndarray):
+    return a.ctypes.data_as(_D)
+
+
+def threads() -> int:
+    """Host threads the oracle's OpenMP loops use."""
+    return int(_load().oracle_threads())
+
+
+def exact_attention(q, k, v) -> np.ndarray:
+    """Exact softmax attention, Eq. (1), per unit; float64 ``[..., N, d]``."""
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    N, d = q.shape[-2], q.shape[-1]
+    out = np.empty_like(q)
+    _load().oracle_exact_attention(_p(q), _p(k), _p(v), _p(out), q.size // (N * d), N, d)
+    return out
+
+
+def nystra_attention(q, k, v, m: int, iters: int) -> np.ndarray:
+    """PnP-Nystra output (Algorithm 1, stabilised form), float64 ``[..., N, d]``."""
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    N, d = q.shape[-2], q.shape[-1]
+    out = np.empty_like(q)
+    rc = _load().oracle_nystra_attention(_p(q), _p(k), _p(v), _p(out), q.size // (N * d),
+                                         N, d, int(m), int(iters))
+    if rc != 0:
+        raise ValueError(f"oracle: invalid m={m} for N={N} (m must divide N), iters={iters}")
+    return out
+
+
+def landmarks(x, m: int) -> np.ndarray:
+    """Segment-mean landmarks of one unit ``[N, d]`` -> ``[m, d]`` (Alg. 1 step 1)."""
+    x = _f64(x)
+    N, d = x.shape
+    out = np.empty((m, d))
+    _load().oracle_landmarks(_p(x), N, d, int(m), _p(out))
+    return out
+
+
+def pinv_iteration(A, iters: int) -> np.ndarray:
+    """Iterative pseudo-inverse of a square matrix (Alg. 1 step 4)."""
+    A = _f64(A)
+    m = A.shape[0]
+    Z = np.empty_like(A)
+    _load().oracle_pinv_iteration(_p(A), m, int(iters), _p(Z))
+    return Z
+
+
+def nystra_stages(q, k, v, m: int, iters: int) -> dict:
+    """All intermediates of one unit (``q, k, v``: ``[N, d]``)."""
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    N, d = q.shape
+    st = {
+        "qbar": np.empty((m, d)), "kbar": np.empty((m, d)), "mL": np.empty(N), "mU": np.empty(m),
+        "GLn": np.empty((N, m)), "GUn": np.empty((m, N)), "GAn": np.empty((m, m)),
+        "Z": np.empty((m, m)), "num": np.empty((N, d)), "den": np.empty(N),
+    }
+    out = np.empty((N, d))
+    order = ["qbar", "kbar", "mL", "mU", "GLn", "GUn", "GAn", "Z", "num", "den"]
+    rc = _load().oracle_nystra_stages(_p(q), _p(k), _p(v), _p(out), N, d, int(m), int(iters),
+                                      *[_p(st[n]) for n in order])
+    if rc != 0:
+        raise ValueError(f"oracle: invalid m={m} for N={N}")
+    st["out"] = out
+    return st
