@@ -1,0 +1,308 @@
+"""Benchmark of the PnP-Nystra window-attention hot path on GB300.
+
+One step = one ``nystra_attention`` call over the whole batch of the workload
+(default: SwinIR-like denoising at 256x256 -- 1024 windows of 8x8 tokens,
+6 heads, d_h = 30, m = 16 landmarks, 6 pseudo-inverse iterations, bf16 I/O).
+Prints ONE JSON line (rank 0).  Metric: tokens*heads per second.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the float64 CPU oracle, host cores
+
+Under torchrun every rank runs its own full batch (units are independent, no
+collective on the data path): weak scaling, value = all ranks' units / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2506_08520_gb300 import binding, workloads  # noqa: E402
+
+METRIC = "Nystrom attention tokens*heads/s"
+UNIT = "tokens*heads/s"
+DEFAULT_WORKLOAD = "swinir256-bf16"
+
+
+def _peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+class ClockSampler:
+    """nvidia-smi SM clock / throttle sampling while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.idx = device_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{device_index}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), parts[5:9]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, r in rows for i, x in enumerate(r) if x.lower() == "active"})
+        return {"sm_mhz": statistics.median(r[0] for r in rows), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
+    """Time the float64 oracle on a bounded sample of the workload's units."""
+    import oracle  # CPU baseline only
+    qu, ku, vu = (x.reshape(-1, wl.N, wl.d) for x in (q, k, v))
+    qd, kd, vd = (x.double().numpy() for x in (qu, ku, vu))
+    # calibrate on a few units, then size the sample to the budget
+    n0 = min(64, qd.shape[0])
+    t0 = time.perf_counter()
+    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters)
+    per_unit = max((time.perf_counter() - t0) / n0, 1e-9)
+    n = int(min(qd.shape[0], max(1, budget_s / per_unit)))
+    if max_units:
+        n = min(n, max_units)
+    t0 = time.perf_counter()
+    oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters)
+    dt = time.perf_counter() - t0
+    return n * wl.N / dt, n, dt, oracle.threads()
+
+
+def run_reference(args, wl):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    q, k, v = workloads.make_qkv(wl)
+    import oracle
+    # per-step sample sized so that warmup+steps fit in about a minute
+    per_step_budget = max(0.002, 60.0 / max(1, args.steps + args.warmup))
+    qd, kd, vd = (x.reshape(-1, wl.N, wl.d).double().numpy() for x in (q, k, v))
+    n0 = min(32, qd.shape[0])
+    t0 = time.perf_counter()
+    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters)
+    per_unit = max((time.perf_counter() - t0) / n0, 1e-9)
+    n = int(min(qd.shape[0], max(1, per_step_budget / per_unit)))
+    for _ in range(args.warmup):
+        oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters)
+    t0 = time.perf_counter()
+    for s in range(args.steps):
+        off = (s * n) % max(1, qd.shape[0] - n + 1)
+        oracle.nystra_attention(qd[off:off + n], kd[off:off + n], vd[off:off + n], wl.m, wl.iters)
+    dt = time.perf_counter() - t0
+    value = args.steps * n * wl.N / dt
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N,
+                   "d_h": wl.d, "m": wl.m, "iters": wl.iters, "io_dtype": wl.dtype},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
+                         "sample": f"{n} of {qd.shape[0]} units per step (float64 C oracle, OpenMP)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def run_cuda(args, wl):
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    binding.lib()  # fail loudly if the library is missing
+
+    q, k, v = workloads.make_qkv(wl)
+    esize = q.element_size()
+    io_bytes = 4 * q.numel() * esize
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
+    # rotate input/output sets so that one step's data is never L2-resident
+    nsets = max(2, -(-3 * l2 // io_bytes))
+    sets = []
+    for _ in range(nsets):
+        sets.append(tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),))
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    shape = (wl.n_windows, wl.heads, wl.N, wl.d)
+    dcode = {"f32": 0, "bf16": 1, "f16": 2}[wl.dtype]
+
+    def step(i, fn=binding.nystra_attention, exact=False):
+        qd, kd, vd, od = sets[i % nsets]
+        if exact:
+            rc = binding.exact_window_attention(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(),
+                                                *shape, dcode, sptr)
+        else:
+            rc = fn(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape, wl.m, wl.iters,
+                    dcode, sptr)
+        if rc != 0:
+            raise binding.NystraError(rc, "bench step")
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        step(i)
+    barrier()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        for i in range(args.steps):
+            starts[i].record(stream)
+            step(i)
+            ends[i].record(stream)
+        barrier()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    kern_ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
+    t = torch.tensor([total_ms], device=dev)
+    if ws > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    total_ms = float(t.item())
+    units_tokens = wl.n_windows * wl.heads * wl.N
+    value = ws * units_tokens * args.steps / (total_ms * 1e-3)
+
+    # exact window attention on the same inputs (the computation replaced)
+    esteps = max(3, min(args.steps, 200))
+    for i in range(3):
+        step(i, exact=True)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(esteps):
+        step(i, exact=True)
+    e1.record(stream)
+    barrier()
+    exact_ms = e0.elapsed_time(e1) / esteps
+
+    # end to end through the public API: pinned host -> device, call, device -> host
+    hq, hk, hv = (x.pin_memory() for x in (q, k, v))
+    ho = torch.empty_like(q).pin_memory()
+    dq, dk, dv, do = sets[0]
+    e2e_steps = max(3, min(args.steps, 50))
+    for _ in range(2):
+        dq.copy_(hq, non_blocking=True); dk.copy_(hk, non_blocking=True); dv.copy_(hv, non_blocking=True)
+        binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do)
+        ho.copy_(do, non_blocking=True)
+    barrier()
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        dq.copy_(hq, non_blocking=True); dk.copy_(hk, non_blocking=True); dv.copy_(hv, non_blocking=True)
+        binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do)
+        ho.copy_(do, non_blocking=True)
+    e1.record(stream)
+    barrier()
+    e2e_ms = e0.elapsed_time(e1) / e2e_steps
+    t = torch.tensor([e2e_ms], device=dev)
+    if ws > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    e2e_value = ws * units_tokens / (float(t.item()) * 1e-3)
+
+    peak, peak_kind = _peaks()
+    achieved = io_bytes / (kern_ms * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N,
+                   "d_h": wl.d, "m": wl.m, "iters": wl.iters, "io_dtype": wl.dtype,
+                   "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
+                   "parallelism": f"replica x{ws} (independent windows)"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None, "peak_kind": peak_kind,
+                     "bytes_per_launch": io_bytes, "kernel_ms": kern_ms},
+        "comparator": {"kernel": "exact_window_attention", "ms_per_step": exact_ms,
+                       "value": units_tokens / (exact_ms * 1e-3), "speedup": exact_ms / (total_ms / args.steps)},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 3 * q.numel() * esize,
+                "d2h_bytes_per_step": q.numel() * esize},
+        "gpu_launches": args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        val, n, dt, cores = _time_oracle(wl, q, k, v, budget_s=args.cpu_budget)
+        line["cpu_baseline"] = {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": f"{n} of {wl.units} units, one pass, {dt:.1f} s (float64 C oracle, OpenMP)"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="cuda", choices=["cuda", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--cpu-budget", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    wl = workloads.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_cuda(args, wl)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,128 @@
+/*
+ * nystra.h -- C ABI of the GB300 (sm_103a) PnP-Nystra window-attention library.
+ *
+ * PnP-Nystra ("Plug-and-Play Linear Attention with Provable Guarantees for
+ * Training-Free Image Restoration", arXiv 2506.08520) replaces the exact
+ * softmax attention of one (window, head) pair,
+ *     O = softmax(Q K^T / sqrt(d_h)) V                              (Eq. 1)
+ * by the Nystrom approximation of the kernel matrix G = exp(Q K^T/sqrt(d_h)),
+ *     G^ = G_L G_A^+ G_U,  O^ = (G^ V) ./ (G^ 1_N)     (Eq. 5-6, Algorithm 1)
+ * evaluated in the row-max-stabilised form of Sec. 2.2 (Eq. stable_output).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  Layout   q, k, v and out are contiguous row-major tensors of shape
+ *           [n_windows, heads, N, d_h]; one "unit" = one (window, head) pair,
+ *           whose N x d_h block starts at element (w*heads + h) * N * d_h.
+ *  Memory   every pointer is DEVICE memory owned by the caller, 16-byte
+ *           aligned, and stays valid until the work on `stream` completes.
+ *           q, k and v may alias one another; out must not overlap any input.
+ *           The library allocates no device memory per call.
+ *  dtype    element type of q, k, v and out (nystra_dtype).  Arithmetic is
+ *           fp32 (accumulation always fp32); 16-bit inputs are widened
+ *           exactly and the output is rounded to nearest-even.
+ *  Stream   `stream` is a cudaStream_t (NULL = legacy default stream).  Calls
+ *           are asynchronous: a return of NYSTRA_OK means the kernels were
+ *           enqueued; results are ready when the stream is synchronised.
+ *  Errors   invalid arguments are rejected before anything is launched and
+ *           leave `out` untouched.  No call aborts, traps or prints.
+ *  Device   the kernels are built for sm_103a (GB300) only.
+ */
+#ifndef NYSTRA_H
+#define NYSTRA_H
+
+#if defined(__GNUC__)
+#define NYSTRA_API __attribute__((visibility("default")))
+#else
+#define NYSTRA_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element type of q, k, v and out. */
+typedef enum { NYSTRA_F32 = 0, NYSTRA_BF16 = 1, NYSTRA_F16 = 2 } nystra_dtype;
+
+/* Status codes returned by every entry point (0 = success, negative = error). */
+enum {
+    NYSTRA_OK = 0,
+    NYSTRA_EINVAL = -1,   /* a size, pointer, alignment or aliasing rule is violated  */
+    NYSTRA_EDTYPE = -2,   /* dtype is not one of nystra_dtype                          */
+    NYSTRA_ELAUNCH = -3,  /* a CUDA call failed; nystra_last_cuda_error() has the code */
+    NYSTRA_ETIMEOUT = -4, /* a bounded device-side wait gave up (see nystra_status)    */
+    NYSTRA_EDEVICE = -5   /* the current device is not an sm_103 GPU                   */
+};
+
+/* Size limits of the kernels (checked on every call). */
+#define NYSTRA_MAX_N 1024     /* tokens per window                     */
+#define NYSTRA_MAX_DH 64      /* head dimension d_h                    */
+#define NYSTRA_MAX_M 64       /* landmarks per window                  */
+#define NYSTRA_MAX_ITERS 100  /* pseudo-inverse iterations             */
+
+/*
+ * nystra_attention -- PnP-Nystra attention for every (window, head) unit.
+ *
+ * Per unit, following Algorithm 1 in the stabilised form of Sec. 2.2:
+ *  1. landmarks Qbar, Kbar (m x d_h): means of m contiguous, non-overlapping
+ *     segments of N/m tokens ("average pooling over non-overlapping windows");
+ *  2-3. S_L = Q Kbar^T s, S_U = Qbar K^T s, S_A = Qbar Kbar^T s with
+ *     s = 1/sqrt(d_h); row maxima m_L (over m landmarks) and m_U (over all N
+ *     keys); G_L^n = exp(S_L - m_L), G_U^n = exp(S_U - m_U),
+ *     G_A^n = exp(S_A - m_U);
+ *  4. Z ~ (G_A^n)^+ by `iters` steps of the third-order iteration of
+ *     Razavi et al. (2014): Z_0 = A^T/(||A||_1 ||A||_inf),
+ *     Z <- Z (13I - AZ(15I - AZ(7I - AZ)))/4 with A = G_A^n;
+ *  5-7. O = (G_L^n Z G_U^n V) ./ (G_L^n Z G_U^n 1_N), evaluated as
+ *     G_L^n (Z (G_U^n [V | 1_N])) (an exact re-association of steps 5-6).
+ *
+ * Arguments
+ *  q, k, v   [n_windows, heads, N, d_h] inputs (device, caller-owned).
+ *  out       [n_windows, heads, N, d_h] output (device, caller-owned).
+ *  n_windows, heads   >= 0; n_windows*heads == 0 is a no-op returning OK.
+ *  N         tokens per window, 1..NYSTRA_MAX_N.
+ *  d_h       head dimension, 1..NYSTRA_MAX_DH.
+ *  m         landmarks, 1..min(N, NYSTRA_MAX_M), and m must divide N.
+ *  iters     pseudo-inverse iterations, 0..NYSTRA_MAX_ITERS (paper: 4-6).
+ *  dtype     nystra_dtype of q, k, v and out.
+ *  stream    cudaStream_t to enqueue on.
+ * Returns NYSTRA_OK, NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH or
+ * NYSTRA_EDEVICE.  The denominator is not guarded (Algorithm 1 step 7
+ * divides as written); a zero denominator yields inf/nan in that row.
+ */
+NYSTRA_API int nystra_attention(const void* q, const void* k, const void* v, void* out,
+                     int n_windows, int heads, int N, int d_h, int m, int iters,
+                     int dtype, void* stream);
+
+/*
+ * exact_window_attention -- exact softmax attention per unit, Eq. (1):
+ * O = softmax(Q K^T / sqrt(d_h)) V with row-max-shifted exponentials
+ * (Eq. 2).  This is the computation PnP-Nystra replaces; it serves as the
+ * in-library comparator.  Arguments and return codes as nystra_attention
+ * (no m, no iters).
+ */
+NYSTRA_API int exact_window_attention(const void* q, const void* k, const void* v, void* out,
+                           int n_windows, int heads, int N, int d_h,
+                           int dtype, void* stream);
+
+/* Human-readable text for a status code (static storage, never NULL). */
+NYSTRA_API const char* nystra_strerror(int status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+NYSTRA_API int nystra_version(void);
+
+/* cudaError_t of the most recent NYSTRA_ELAUNCH on the calling thread (0 if none). */
+NYSTRA_API int nystra_last_cuda_error(void);
+
+/*
+ * nystra_status -- synchronise `stream` and report device-side faults
+ * recorded by kernels on the current device since the previous call:
+ * NYSTRA_ETIMEOUT if a bounded wait gave up, else NYSTRA_OK (or
+ * NYSTRA_ELAUNCH if the synchronisation itself failed).  Clears the record.
+ */
+NYSTRA_API int nystra_status(void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NYSTRA_H */

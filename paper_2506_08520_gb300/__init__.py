@@ -1,0 +1,12 @@
+"""GB300-native (sm_103a) PnP-Nystra window attention.
+
+``nystra(q, k, v, m, iters)`` and ``exact(q, k, v)`` call the C-ABI CUDA
+library ``libnystra.so`` (see ``include/nystra.h``); ``workloads`` holds the
+seeded synthetic inputs.  The library is loaded on first use and every call
+fails loudly if it is missing: there is no CPU path.
+"""
+from .binding import (NystraError, exact, exact_window_attention, nystra, nystra_attention, status,
+                     strerror, version)
+
+__all__ = ["nystra", "exact", "nystra_attention", "exact_window_attention", "status", "strerror",
+           "version", "NystraError"]

@@ -1,0 +1,137 @@
+"""Thin ctypes binding of ``libnystra.so`` (C ABI in ``include/nystra.h``).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels behind the C ABI.  torch is used for device memory and streams.
+There is no CPU fallback: if the library is missing, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libnystra.so")
+
+NYSTRA_F32, NYSTRA_BF16, NYSTRA_F16 = 0, 1, 2
+NYSTRA_OK, NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH, NYSTRA_ETIMEOUT, NYSTRA_EDEVICE = 0, -1, -2, -3, -4, -5
+MAX_N, MAX_DH, MAX_M, MAX_ITERS = 1024, 64, 64, 100
+
+_DTYPE_CODE = {torch.float32: NYSTRA_F32, torch.bfloat16: NYSTRA_BF16, torch.float16: NYSTRA_F16}
+
+_lib = None
+
+
+class NystraError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = f"{where}: {strerror(status)} (status {status})"
+        if status == NYSTRA_ELAUNCH:
+            msg += f", cudaError {lib().nystra_last_cuda_error()}"
+        super().__init__(msg)
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library; raises if it has not been built (no fallback)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with "
+                               "`python -m paper_2506_08520_gb300.build` (no CPU fallback exists)")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i = ctypes.c_void_p, ctypes.c_int
+        L.nystra_attention.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp]
+        L.nystra_attention.restype = i
+        L.exact_window_attention.argtypes = [vp, vp, vp, vp, i, i, i, i, i, vp]
+        L.exact_window_attention.restype = i
+        L.nystra_strerror.argtypes = [i]
+        L.nystra_strerror.restype = ctypes.c_char_p
+        L.nystra_version.restype = i
+        L.nystra_last_cuda_error.restype = i
+        L.nystra_status.argtypes = [vp]
+        L.nystra_status.restype = i
+        _lib = L
+    return _lib
+
+
+# ---------------------------------------------------------------- raw C ABI
+def nystra_attention(q, k, v, out, n_windows, heads, N, d_h, m, iters, dtype, stream) -> int:
+    """Raw C-ABI call: pointers as ints, returns the status code."""
+    return lib().nystra_attention(q, k, v, out, n_windows, heads, N, d_h, m, iters, dtype, stream)
+
+
+def exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream) -> int:
+    return lib().exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream)
+
+
+def strerror(status: int) -> str:
+    return lib().nystra_strerror(status).decode()
+
+
+def version() -> int:
+    return lib().nystra_version()
+
+
+def status(stream=None) -> int:
+    """Synchronise ``stream`` and return the device-side fault status."""
+    return lib().nystra_status(_stream_ptr(stream))
+
+
+# ------------------------------------------------------------ torch helpers
+def _stream_ptr(stream) -> int | None:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _geometry(q: torch.Tensor):
+    if q.dim() == 4:
+        n_windows, heads, N, d = q.shape
+    elif q.dim() == 3:
+        (n_windows, N, d), heads = q.shape, 1
+    else:
+        raise ValueError("expected [n_windows, heads, N, d_h] or [units, N, d_h]")
+    return n_windows, heads, N, d
+
+
+def _check(q, k, v, out):
+    for t in (q, k, v, out):
+        if not t.is_cuda:
+            raise ValueError("tensors must be on a CUDA device (no CPU path)")
+        if not t.is_contiguous():
+            raise ValueError("tensors must be contiguous")
+        if t.shape != q.shape or t.dtype != q.dtype:
+            raise ValueError("q, k, v and out must share shape and dtype")
+    if q.dtype not in _DTYPE_CODE:
+        raise ValueError(f"unsupported dtype {q.dtype}")
+
+
+def nystra(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int = 16, iters: int = 6,
+           out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """PnP-Nystra attention of device tensors ``[n_windows, heads, N, d_h]``."""
+    out = torch.empty_like(q) if out is None else out
+    _check(q, k, v, out)
+    nw, h, N, d = _geometry(q)
+    with torch.cuda.device(q.device):
+        rc = nystra_attention(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
+                              m, iters, _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_attention")
+    return out
+
+
+def exact(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tensor | None = None,
+          stream=None) -> torch.Tensor:
+    """Exact softmax window attention (the computation PnP-Nystra replaces)."""
+    out = torch.empty_like(q) if out is None else out
+    _check(q, k, v, out)
+    nw, h, N, d = _geometry(q)
+    with torch.cuda.device(q.device):
+        rc = exact_window_attention(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
+                                    _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "exact_window_attention")
+    return out

@@ -1,0 +1,100 @@
+// C ABI of the PnP-Nystra library: argument validation and kernel dispatch.
+// Declarations and the full contract are in include/nystra.h.
+#include <stdint.h>
+
+#include "common.cuh"
+#include "nystra.h"
+
+namespace {
+
+thread_local int g_last_cuda_error = 0;
+
+int fail_cuda(cudaError_t e) {
+    g_last_cuda_error = (int)e;
+    return NYSTRA_ELAUNCH;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+bool overlaps(const void* a, const void* b, size_t bytes) {
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return x < y + bytes && y < x + bytes;
+}
+
+size_t elem_size(int dtype) { return dtype == NYSTRA_F32 ? 4 : 2; }
+
+// Shared checks of both entry points.  Returns NYSTRA_OK or an error code.
+int check_common(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                 int N, int d_h, int dtype) {
+    if (dtype != NYSTRA_F32 && dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (N < 1 || N > NYSTRA_MAX_N || d_h < 1 || d_h > NYSTRA_MAX_DH) return NYSTRA_EINVAL;
+    if ((long long)n_windows * heads == 0) return NYSTRA_OK;
+    if (!q || !k || !v || !out) return NYSTRA_EINVAL;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out)) return NYSTRA_EINVAL;
+    const size_t bytes = (size_t)n_windows * heads * N * d_h * elem_size(dtype);
+    if (overlaps(out, q, bytes) || overlaps(out, k, bytes) || overlaps(out, v, bytes)) return NYSTRA_EINVAL;
+    return NYSTRA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int nystra_attention(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                     int N, int d_h, int m, int iters, int dtype, void* stream) {
+    int rc = check_common(q, k, v, out, n_windows, heads, N, d_h, dtype);
+    if (rc != NYSTRA_OK) return rc;
+    if (m < 1 || m > N || m > NYSTRA_MAX_M || N % m != 0) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
+    const long long units = (long long)n_windows * heads;
+    if (units == 0) return NYSTRA_OK;
+    cudaError_t e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype,
+                                                       (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
+int exact_window_attention(const void* q, const void* k, const void* v, void* out, int n_windows,
+                           int heads, int N, int d_h, int dtype, void* stream) {
+    int rc = check_common(q, k, v, out, n_windows, heads, N, d_h, dtype);
+    if (rc != NYSTRA_OK) return rc;
+    const long long units = (long long)n_windows * heads;
+    if (units == 0) return NYSTRA_OK;
+    cudaError_t e = nystra_host::launch_exact_generic(q, k, v, out, units, N, d_h, dtype,
+                                                      (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
+const char* nystra_strerror(int status) {
+    switch (status) {
+        case NYSTRA_OK: return "success";
+        case NYSTRA_EINVAL: return "invalid argument (size, pointer, alignment or aliasing)";
+        case NYSTRA_EDTYPE: return "unsupported dtype";
+        case NYSTRA_ELAUNCH: return "CUDA launch or runtime error";
+        case NYSTRA_ETIMEOUT: return "a bounded device-side wait timed out";
+        case NYSTRA_EDEVICE: return "unsupported device (sm_103 required)";
+        default: return "unknown status";
+    }
+}
+
+int nystra_version(void) { return 100; }
+
+int nystra_last_cuda_error(void) { return g_last_cuda_error; }
+
+int nystra_status(void* stream) {
+    cudaError_t e = cudaSuccess;
+    const unsigned int words = nystra_host::take_fault_words((cudaStream_t)stream, &e);
+    if (e != cudaSuccess) return fail_cuda(e);
+    return (words & 1u) ? NYSTRA_ETIMEOUT : NYSTRA_OK;
+}
+
+}  // extern "C"
+
+namespace nystra_host {
+// No kernel of this build waits on a barrier yet, so there is nothing to
+// collect beyond synchronising the stream.
+unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
+    *err = cudaStreamSynchronize(stream);
+    return 0u;
+}
+}  // namespace nystra_host

@@ -1,0 +1,40 @@
+// Shared device helpers for the PnP-Nystra kernels (sm_103a).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace nystra {
+
+// Element I/O: 16-bit inputs are widened exactly; outputs are rounded to
+// nearest-even.
+__device__ __forceinline__ float to_f32(float x) { return x; }
+__device__ __forceinline__ float to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+__device__ __forceinline__ float to_f32(__half x) { return __half2float(x); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) {
+    return __float2bfloat16_rn(x);
+}
+template <> __device__ __forceinline__ __half from_f32<__half>(float x) { return __float2half_rn(x); }
+
+template <typename T> __device__ __forceinline__ float ldg_f32(const T* p) { return to_f32(p[0]); }
+template <> __device__ __forceinline__ float ldg_f32<float>(const float* p) { return __ldg(p); }
+
+}  // namespace nystra
+
+// Host-side launchers (one per kernel family), defined in their .cu files.
+// Each returns a cudaError_t of the launch.
+namespace nystra_host {
+cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, void* out,
+                                  long long n_units, int N, int d, int m, int iters, int dtype,
+                                  cudaStream_t stream);
+cudaError_t launch_exact_generic(const void* q, const void* k, const void* v, void* out,
+                                 long long n_units, int N, int d, int dtype, cudaStream_t stream);
+// Device-side fault words (bit 0: a bounded wait gave up) of the translation
+// units whose kernels wait on barriers: OR-ed together, then cleared.
+unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);
+}  // namespace nystra_host

@@ -1,0 +1,96 @@
+"""C-ABI checks that need no GPU: the library loads, exports every symbol the
+public header declares, and rejects invalid arguments before launching."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2506_08520_gb300 import build as nbuild
+from paper_2506_08520_gb300 import binding as nb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "nystra.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    nbuild.build()
+    return nb.lib()
+
+
+def declared_symbols():
+    text = open(HEADER).read()
+    return re.findall(r"NYSTRA_API\s+[\w\s\*]+?\b(\w+)\s*\(", text)
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
+                     "nystra_version", "nystra_status", "nystra_last_cuda_error"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    raw = ctypes.CDLL(nb.LIB_PATH)
+    for name in declared_symbols():
+        assert hasattr(raw, name), f"{name} declared in nystra.h but not exported"
+
+
+def test_strerror_and_version(lib):
+    for code in (0, -1, -2, -3, -4, -5, 7):
+        assert isinstance(nb.strerror(code), str) and nb.strerror(code)
+    assert nb.version() >= 100
+
+
+# Pointers that are never dereferenced: every call below must fail validation
+# (or be an empty no-op) before any CUDA call is made.
+P = 1 << 20
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(N=64, d=30, m=16, iters=6, dtype=5), nb.NYSTRA_EDTYPE),
+    (dict(N=64, d=30, m=15, iters=6), nb.NYSTRA_EINVAL),        # m does not divide N
+    (dict(N=64, d=30, m=0, iters=6), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, m=128, iters=6), nb.NYSTRA_EINVAL),       # m > N
+    (dict(N=2048, d=30, m=16, iters=6), nb.NYSTRA_EINVAL),      # N > 1024
+    (dict(N=128, d=30, m=128, iters=6), nb.NYSTRA_EINVAL),      # m > 64
+    (dict(N=64, d=65, m=16, iters=6), nb.NYSTRA_EINVAL),        # d_h > 64
+    (dict(N=64, d=0, m=16, iters=6), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, m=16, iters=-1), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, m=16, iters=101), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, m=16, iters=6, q=0), nb.NYSTRA_EINVAL),   # null pointer
+    (dict(N=64, d=30, m=16, iters=6, q=P + 8), nb.NYSTRA_EINVAL),  # misaligned
+    (dict(N=64, d=30, m=16, iters=6, out=P), nb.NYSTRA_EINVAL),    # out aliases q
+    (dict(N=64, d=30, m=16, iters=6, nw=-1), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, m=16, iters=6, nw=0), nb.NYSTRA_OK),         # empty: no-op
+    (dict(N=64, d=30, m=16, iters=6, heads=0), nb.NYSTRA_OK),
+])
+def test_nystra_argument_validation(lib, args, code):
+    q = args.get("q", P)
+    out = args.get("out", 64 * P)
+    rc = nb.nystra_attention(q, 2 * P, 3 * P, out, args.get("nw", 4), args.get("heads", 2),
+                             args["N"], args["d"], args["m"], args["iters"], args.get("dtype", 1), None)
+    assert rc == code
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(N=64, d=30, dtype=3), nb.NYSTRA_EDTYPE),
+    (dict(N=0, d=30), nb.NYSTRA_EINVAL),
+    (dict(N=1025, d=30), nb.NYSTRA_EINVAL),
+    (dict(N=64, d=30, out=3 * P + 64), nb.NYSTRA_EINVAL),     # out overlaps v
+    (dict(N=64, d=30, nw=0), nb.NYSTRA_OK),
+])
+def test_exact_argument_validation(lib, args, code):
+    rc = nb.exact_window_attention(P, 2 * P, 3 * P, args.get("out", 64 * P), args.get("nw", 4), 2,
+                                   args["N"], args["d"], args.get("dtype", 0), None)
+    assert rc == code
+
+
+def test_torch_wrappers_refuse_cpu_tensors(lib):
+    import torch
+    x = torch.zeros(1, 1, 64, 30)
+    with pytest.raises(ValueError):
+        nb.nystra(x, x, x)
+    with pytest.raises(ValueError):
+        nb.exact(x, x, x)

@@ -1,0 +1,117 @@
+"""GPU parity: the CUDA path (through the C ABI) against the float64 oracle on
+the same seeded inputs.  Bar: max over units of the relative Frobenius error
+<= 1e-4 for fp32 I/O and <= 2e-2 for bf16 / fp16 I/O (fp32 accumulation)."""
+import numpy as np
+import pytest
+import torch
+
+from paper_2506_08520_gb300 import binding, workloads
+from tests.parity import TOL, check_exact, check_nystra, sample_units
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2506_08520_gb300 import build
+    build.build()
+
+
+# Small shapes: several tiles and ragged tails, every dtype.
+SMALL = [
+    # units, N, d, m
+    (7, 64, 30, 16),
+    (9, 64, 32, 8),
+    (5, 64, 32, 32),
+    (5, 256, 32, 32),
+    (3, 256, 30, 64),
+    (2, 1024, 32, 32),
+    (2, 1024, 32, 64),
+    (4, 48, 20, 12),     # odd sizes
+    (3, 10, 3, 5),
+    (6, 128, 64, 16),    # widest head
+    (3, 96, 17, 24),
+]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
+@pytest.mark.parametrize("units,N,d,m", SMALL)
+def test_nystra_small(units, N, d, m, dtype):
+    q, k, v = workloads.random_qkv(units, N, d, dtype, seed=units * 1000 + N + d + m)
+    err, worst = check_nystra(q, k, v, m, 6)
+    assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("N,d,m,iters", [
+    (64, 30, 64, 6),     # m = N: every token is a landmark
+    (64, 30, 1, 6),      # one landmark
+    (64, 30, 16, 0),     # Z = Z_0 only
+    (64, 30, 16, 1),
+    (64, 30, 16, 12),
+    (1, 1, 1, 6),        # degenerate single token
+    (64, 1, 16, 6),      # d_h = 1
+    (32, 64, 32, 6),
+])
+def test_nystra_edge_cases(N, d, m, iters, dtype):
+    q, k, v = workloads.random_qkv(3, N, d, dtype, seed=N + d + m + iters)
+    err, worst = check_nystra(q, k, v, m, iters)
+    assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+
+
+# Full-size workloads: the GPU computes every unit, the oracle a sample.
+FULL = ["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4",
+        "large-w16-m32", "large-w16-m64", "large-w32-m32", "large-w32-m64",
+        "sr720p-w8-m16-bf16", "sr720p-w16-m16-f16", "sr720p-w32-m16-bf16", "sr720p-w8-m64-f16",
+        "sr720p-w32-m8-f16"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_nystra_workloads(name):
+    wl = workloads.WORKLOADS[name]
+    q, k, v = workloads.make_qkv(wl)
+    sample = None if wl.units <= 8192 and wl.N <= 256 else sample_units(wl.units)
+    err, worst = check_nystra(q, k, v, wl.m, wl.iters, sample)
+    print(f"{name}: max rel err {err:.3e} (unit {worst})")
+    assert err <= TOL[wl.dtype], f"{name}: max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
+@pytest.mark.parametrize("units,N,d", [(7, 64, 30), (3, 256, 32), (2, 1024, 32), (4, 48, 20), (3, 10, 64)])
+def test_exact_small(units, N, d, dtype):
+    q, k, v = workloads.random_qkv(units, N, d, dtype, seed=units + N + d)
+    err, worst = check_exact(q, k, v)
+    assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("name", ["swinir256-bf16", "large-w32-m32", "sr720p-w16-m16-bf16"])
+def test_exact_workloads(name):
+    wl = workloads.WORKLOADS[name]
+    q, k, v = workloads.make_qkv(wl)
+    err, worst = check_exact(q, k, v, sample_units(wl.units, 128))
+    assert err <= TOL[wl.dtype], f"{name}: max rel err {err:.3e} at unit {worst}"
+
+
+def test_deterministic_and_stream():
+    q, k, v = (x.cuda() for x in workloads.random_qkv(33, 64, 30, "bf16", seed=5))
+    a = binding.nystra(q, k, v, 16, 6)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        b = binding.nystra(q, k, v, 16, 6, stream=s)
+    s.synchronize()
+    assert torch.equal(a, b)
+
+
+def test_invalid_call_leaves_output_untouched():
+    q, k, v = (x.cuda() for x in workloads.random_qkv(2, 64, 30, "f32", seed=6))
+    out = torch.full_like(q, 7.0)
+    with pytest.raises(binding.NystraError):
+        binding.nystra(q, k, v, m=15, iters=6, out=out)
+    torch.cuda.synchronize()
+    assert bool((out == 7.0).all())
+
+
+def test_status_clean_after_runs():
+    q, k, v = (x.cuda() for x in workloads.random_qkv(4, 64, 30, "bf16", seed=7))
+    binding.nystra(q, k, v, 16, 6)
+    assert binding.status() == binding.NYSTRA_OK
