@@ -49,8 +49,12 @@ int nystra_attention(const void* q, const void* k, const void* v, void* out, int
     if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
-    cudaError_t e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype,
-                                                       (cudaStream_t)stream);
+    cudaError_t e;
+    if (nystra_host::nystra_w64_supports(N, d_h, m, dtype))
+        e = nystra_host::launch_nystra_w64(q, k, v, out, units, d_h, m, iters, dtype, (cudaStream_t)stream);
+    else
+        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype,
+                                               (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
@@ -91,10 +95,9 @@ int nystra_status(void* stream) {
 }  // extern "C"
 
 namespace nystra_host {
-// No kernel of this build waits on a barrier yet, so there is nothing to
-// collect beyond synchronising the stream.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
-    return 0u;
+    if (*err != cudaSuccess) return 0u;
+    return take_fault_word_w64(err);
 }
 }  // namespace nystra_host
