@@ -17,10 +17,22 @@
 //           Y = Z W, then O = (G_L^n Y_:d) / (G_L^n Y_d) (steps 5-7), written
 //           straight from registers.
 // Products with 64-token or d_h extents use mma.sync in the I/O dtype with fp32
-// accumulation; the m x m iteration and Y = Z W use split-tf32 mma.sync (three
-// tf32 products per term, close to fp32 accuracy) with fp32 accumulation.
-// Scores are kept in the log2 domain (scaled by log2(e)/sqrt(d_h)) so each
-// exponential is one ex2.
+// accumulation.  The m x m iteration and Y = Z W use split-tf32 mma.sync (three
+// tf32 products per term, close to fp32: the iteration's round-off is amplified
+// by ||A|| ||Z||, which grows with the iteration count).
+//
+// The iteration runs in registers.  Two facts make that possible:
+//  * an MMA result (C layout: lane holds columns 2t, 2t+1) feeds the next MMA's
+//    A operand unchanged if the k index is permuted consistently for both
+//    operands (k-slot t <-> column 2t, k-slot t+4 <-> column 2t+1);
+//  * X = A Z_k and every polynomial in X are symmetric (Z_0 = a A^T, and each
+//    update multiplies by a polynomial in X), so the B fragment of such a matrix
+//    is the lane's own C-layout values of its transpose.  The computed X is
+//    symmetrised, (X + X^T)/2, each step to keep this exact for X itself.
+// Z (the B operand of A Z) and X (for its transpose) go through shared memory
+// once per step; everything else stays in registers.  Scores are kept in the
+// log2 domain (scaled by log2(e)/sqrt(d_h)) so each exponential is one FFMA
+// and one ex2.
 #include "common.cuh"
 #include "ptx.cuh"
 
@@ -46,8 +58,9 @@ struct Layout64 {
     static constexpr size_t QBAR = STAGE;
     static constexpr size_t KBAR = QBAR + MP * LS * 2;
     static constexpr size_t GLF = KBAR + MP * LS * 2;
-    static constexpr size_t MATS = GLF + (N / 16) * KTL * 32 * 16;
-    static constexpr size_t WBUF = MATS + 5 * MP * SM * 4;
+    static constexpr size_t MATA = GLF + (N / 16) * KTL * 32 * 16;
+    static constexpr size_t MATZ = MATA + MP * SM * 4;
+    static constexpr size_t WBUF = MATZ + MP * SM * 4;
     static constexpr size_t YT = WBUF + MP * WS * 4;
     static constexpr size_t BAR = YT + ((NCOL * YS * 2 + 15) / 16) * 16;
     static constexpr size_t WARP_BYTES = ((BAR + 16 + 127) / 128) * 128;
@@ -57,72 +70,95 @@ template <typename T>
 __device__ __forceinline__ uint32_t ld32(const T* p) {
     return *reinterpret_cast<const uint32_t*>(p);
 }
-template <typename T>
-__device__ __forceinline__ uint16_t bits16(T x) {
-    return *reinterpret_cast<uint16_t*>(&x);
+
+// C-layout fragments of an MP x MP fp32 matrix: f[i][n][e] is row
+// 16i + g + 8(e >> 1), column 8n + 2t + (e & 1).
+template <int MT>
+using Frag = float[MT][2 * MT][4];
+
+template <int MT>
+__device__ __forceinline__ void frag_zero(Frag<MT>& f) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n) f[i][n][0] = f[i][n][1] = f[i][n][2] = f[i][n][3] = 0.f;
 }
 
-// B fragment of [V | 1 | 0...]: rows r, r+1 of column col (col == d -> ones).
-template <typename T>
-__device__ __forceinline__ uint32_t v_pair(const T* Vs, int r, int col, int d) {
-    if (col < d) {
-        return (uint32_t)bits16(Vs[r * d + col]) | ((uint32_t)bits16(Vs[(r + 1) * d + col]) << 16);
-    }
-    return col == d ? (Mma16<T>::kOne | (Mma16<T>::kOne << 16)) : 0u;
-}
-
-// Split-tf32 product term: x = hi + lo with hi, lo both tf32.  Three tf32 MMAs
-// (lo*hi, hi*lo, hi*hi, small terms first) give close to fp32 accuracy, which
-// the pseudo-inverse iteration needs: its round-off is amplified by
-// ||A|| ||Z||, which grows with the iteration count.
-struct Tf32Pair {
-    uint32_t hi, lo;
-};
-__device__ __forceinline__ Tf32Pair split_tf32(float x) {
-    const uint32_t hi = to_tf32(x);
-    return {hi, to_tf32(x - __uint_as_float(hi))};
-}
-__device__ __forceinline__ void mma_tf32x3(float (&c)[4], const Tf32Pair (&a)[4], const Tf32Pair (&b)[2]) {
-    mma_tf32(c, a[0].lo, a[1].lo, a[2].lo, a[3].lo, b[0].hi, b[1].hi);
-    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].lo, b[1].lo);
-    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].hi, b[1].hi);
-}
-
-// C = A B for MP x MP fp32 matrices in shared memory (row stride SM) on the
-// tensor cores in split-tf32; epi(r, c, v) receives each output element.
-// Column blocks are completed one at a time, so an epilogue may overwrite the
-// column block of B it has just consumed.
-template <int MT, int SM, typename Epi>
-__device__ __forceinline__ void mm_tf32(const float* A, const float* B, int g, int t, Epi epi) {
-    constexpr int MP = MT * 16;
-#pragma unroll 1
-    for (int j = 0; j < MP / 8; ++j) {
-        float acc[MT][4];
+// T = alpha I - D, in place.
+template <int MT>
+__device__ __forceinline__ void frag_shift(Frag<MT>& f, float alpha, int g, int t) {
 #pragma unroll
-        for (int i = 0; i < MT; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+    for (int i = 0; i < MT; ++i)
 #pragma unroll
-        for (int kk = 0; kk < MP / 8; ++kk) {
-            const Tf32Pair b[2] = {split_tf32(B[(8 * kk + t) * SM + 8 * j + g]),
-                                   split_tf32(B[(8 * kk + t + 4) * SM + 8 * j + g])};
+        for (int n = 0; n < 2 * MT; ++n)
 #pragma unroll
-            for (int i = 0; i < MT; ++i) {
-                const float* ar = A + (16 * i + g) * SM + 8 * kk + t;
-                const Tf32Pair a[4] = {split_tf32(ar[0]), split_tf32(ar[8 * SM]), split_tf32(ar[4]),
-                                       split_tf32(ar[8 * SM + 4])};
-                mma_tf32x3(acc[i], a, b);
+            for (int e = 0; e < 4; ++e) {
+                const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * n + (e & 1) + 2 * t);
+                f[i][n][e] = (diag ? alpha : 0.f) - f[i][n][e];
             }
-        }
-        __syncwarp();
+}
+
+// D = A B with A given as C-layout fragments (any matrix) and B as C-layout
+// fragments of a symmetric matrix, k permuted as described in the header.
+template <int MT>
+__device__ __forceinline__ void mm_frag_sym(const Frag<MT>& A, const Frag<MT>& B, Frag<MT>& D) {
+    frag_zero<MT>(D);
+#pragma unroll
+    for (int kk = 0; kk < 2 * MT; ++kk) {
+        Tf32Pair a[MT][4];
 #pragma unroll
         for (int i = 0; i < MT; ++i) {
-            const int r = 16 * i + g, c = 8 * j + 2 * t;
-            epi(r, c, acc[i][0]);
-            epi(r, c + 1, acc[i][1]);
-            epi(r + 8, c, acc[i][2]);
-            epi(r + 8, c + 1, acc[i][3]);
+            a[i][0] = split_tf32(A[i][kk][0]);
+            a[i][1] = split_tf32(A[i][kk][2]);
+            a[i][2] = split_tf32(A[i][kk][1]);
+            a[i][3] = split_tf32(A[i][kk][3]);
         }
-        __syncwarp();
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j) {
+            const Tf32Pair b[2] = {split_tf32(B[j >> 1][kk][(j & 1) * 2]),
+                                   split_tf32(B[j >> 1][kk][(j & 1) * 2 + 1])};
+#pragma unroll
+            for (int i = 0; i < MT; ++i) mma_tf32x3(D[i][j], a[i], b);
+        }
     }
+}
+
+// D = A B with both operands row-major fp32 in shared memory (stride SM).
+template <int MT, int SM>
+__device__ __forceinline__ void mm_smem(const float* As, const float* Bs, Frag<MT>& D, int g, int t) {
+    frag_zero<MT>(D);
+#pragma unroll
+    for (int kk = 0; kk < 2 * MT; ++kk) {
+        Tf32Pair a[MT][4];
+#pragma unroll
+        for (int i = 0; i < MT; ++i) {
+            const float2 p = *reinterpret_cast<const float2*>(As + (16 * i + g) * SM + 8 * kk + 2 * t);
+            const float2 r = *reinterpret_cast<const float2*>(As + (16 * i + g + 8) * SM + 8 * kk + 2 * t);
+            a[i][0] = split_tf32(p.x);
+            a[i][1] = split_tf32(r.x);
+            a[i][2] = split_tf32(p.y);
+            a[i][3] = split_tf32(r.y);
+        }
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j) {
+            const Tf32Pair b[2] = {split_tf32(Bs[(8 * kk + 2 * t) * SM + 8 * j + g]),
+                                   split_tf32(Bs[(8 * kk + 2 * t + 1) * SM + 8 * j + g])};
+#pragma unroll
+            for (int i = 0; i < MT; ++i) mma_tf32x3(D[i][j], a[i], b);
+        }
+    }
+}
+
+template <int MT, int SM>
+__device__ __forceinline__ void frag_store(const Frag<MT>& f, float* S, int g, int t) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n) {
+            const int r = 16 * i + g, c = 8 * n + 2 * t;
+            *reinterpret_cast<float2*>(S + r * SM + c) = make_float2(f[i][n][0], f[i][n][1]);
+            *reinterpret_cast<float2*>(S + (r + 8) * SM + c) = make_float2(f[i][n][2], f[i][n][3]);
+        }
 }
 
 template <typename T, int M, int NCOL, int WARPS>
@@ -146,11 +182,8 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
     T* qbar = reinterpret_cast<T*>(base + Lay::QBAR);
     T* kbar = reinterpret_cast<T*>(base + Lay::KBAR);
     unsigned char* glf = base + Lay::GLF;
-    float* mA = reinterpret_cast<float*>(base + Lay::MATS);
-    float* mZ = mA + MP * SM;
-    float* mZn = mZ + MP * SM;
-    float* mX = mZn + MP * SM;
-    float* mT = mX + MP * SM;
+    float* mA = reinterpret_cast<float*>(base + Lay::MATA);
+    float* mZ = reinterpret_cast<float*>(base + Lay::MATZ);
     float* mW = reinterpret_cast<float*>(base + Lay::WBUF);
     T* yT = reinterpret_cast<T*>(base + Lay::YT);
     uint64_t* bar = reinterpret_cast<uint64_t*>(base + Lay::BAR);
@@ -208,7 +241,17 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
         __syncwarp();
 
         // ------- front: S_U, m_U, G_U^n (registers), W = G_U^n [V | 1] -------
-        float mU[MT][2];
+        // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
+        uint32_t vb[8][NTO];
+#pragma unroll
+        for (int a = 0; a < 8; ++a)
+#pragma unroll
+            for (int b = 0; b < NTO; ++b) {
+                const int c0 = 8 * b + 2 * t;
+                const uint32_t x = c0 < d ? ld32(Vs + (8 * a + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
+                vb[a][b] = movmatrix_trans(x);
+            }
+        float mU[MT][2];  // row maxima of S_U, log2 domain
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
             uint32_t aq[2][4];
@@ -236,32 +279,28 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
             float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
             for (int nt = 0; nt < 8; ++nt) {
-#pragma unroll
-                for (int e = 0; e < 4; ++e) s[nt][e] *= sl2;
                 mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]));
                 mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]));
             }
-            mx0 = quad_max(mx0);
-            mx1 = quad_max(mx1);
+            mx0 = quad_max(mx0) * sl2;
+            mx1 = quad_max(mx1) * sl2;
             mU[mt][0] = mx0;
             mU[mt][1] = mx1;
             const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
+            auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+            auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
             float w[NTO][4];
 #pragma unroll
             for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
 #pragma unroll
             for (int kt = 0; kt < 4; ++kt) {
                 uint32_t a[4];
-                a[0] = v0 ? Op::pack(ex2(s[2 * kt][0] - mx0), ex2(s[2 * kt][1] - mx0)) : 0u;
-                a[1] = v1 ? Op::pack(ex2(s[2 * kt][2] - mx1), ex2(s[2 * kt][3] - mx1)) : 0u;
-                a[2] = v0 ? Op::pack(ex2(s[2 * kt + 1][0] - mx0), ex2(s[2 * kt + 1][1] - mx0)) : 0u;
-                a[3] = v1 ? Op::pack(ex2(s[2 * kt + 1][2] - mx1), ex2(s[2 * kt + 1][3] - mx1)) : 0u;
-                const int r0 = 16 * kt + 2 * t;
+                a[0] = v0 ? Op::pack(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : 0u;
+                a[1] = v1 ? Op::pack(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : 0u;
+                a[2] = v0 ? Op::pack(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : 0u;
+                a[3] = v1 ? Op::pack(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : 0u;
 #pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    const int col = 8 * j + g;
-                    Op::k16(w[j], a, v_pair(Vs, r0, col, d), v_pair(Vs, r0 + 8, col, d));
-                }
+                for (int j = 0; j < NTO; ++j) Op::k16(w[j], a, vb[2 * kt][j], vb[2 * kt + 1][j]);
             }
 #pragma unroll
             for (int j = 0; j < NTO; ++j) {
@@ -306,27 +345,27 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
                 float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
                 for (int j = 0; j < NTL; ++j) {
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) sl[j][e] *= sl2;
                     mx0 = fmaxf(mx0, fmaxf(sl[j][0], sl[j][1]));
                     mx1 = fmaxf(mx1, fmaxf(sl[j][2], sl[j][3]));
                 }
-                mx0 = quad_max(mx0);
-                mx1 = quad_max(mx1);
+                mx0 = quad_max(mx0) * sl2;
+                mx1 = quad_max(mx1) * sl2;
+                auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+                auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
                 if constexpr (M >= 16) {
 #pragma unroll
                     for (int kk = 0; kk < KTL; ++kk) {
                         uint4 f;
-                        f.x = Op::pack(ex2(sl[2 * kk][0] - mx0), ex2(sl[2 * kk][1] - mx0));
-                        f.y = Op::pack(ex2(sl[2 * kk][2] - mx1), ex2(sl[2 * kk][3] - mx1));
-                        f.z = Op::pack(ex2(sl[2 * kk + 1][0] - mx0), ex2(sl[2 * kk + 1][1] - mx0));
-                        f.w = Op::pack(ex2(sl[2 * kk + 1][2] - mx1), ex2(sl[2 * kk + 1][3] - mx1));
+                        f.x = Op::pack(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
+                        f.y = Op::pack(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
+                        f.z = Op::pack(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
+                        f.w = Op::pack(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
                         reinterpret_cast<uint4*>(glf)[(tm * KTL + kk) * 32 + lane] = f;
                     }
                 } else {
                     uint2 f;
-                    f.x = Op::pack(ex2(sl[0][0] - mx0), ex2(sl[0][1] - mx0));
-                    f.y = Op::pack(ex2(sl[0][2] - mx1), ex2(sl[0][3] - mx1));
+                    f.x = Op::pack(e0(sl[0][0]), e0(sl[0][1]));
+                    f.y = Op::pack(e1(sl[0][2]), e1(sl[0][3]));
                     reinterpret_cast<uint2*>(glf)[tm * 32 + lane] = f;
                 }
             }
@@ -342,99 +381,169 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
             }
         }
 
-        // ---------------- back: G_A^n, norms, Z_0 ----------------
+        // ------------- back: G_A^n (fragments), norms, Z_0 -------------
+        Frag<MT> Zc;
+        {
+            Frag<MT> Ac;
 #pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            uint32_t aq[2][4];
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk) {
-                const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-                aq[kk][0] = ld32(r0);
-                aq[kk][1] = ld32(r0 + 8 * LS);
-                aq[kk][2] = ld32(r0 + 8);
-                aq[kk][3] = ld32(r0 + 8 * LS + 8);
-            }
-#pragma unroll
-            for (int j = 0; j < MP / 8; ++j) {
-                float sa[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int mt = 0; mt < MT; ++mt) {
+                uint32_t aq[2][4];
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) {
-                    const T* kr = kbar + (8 * j + g) * LS + 16 * kk + 2 * t;
-                    Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                    const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+                    aq[kk][0] = ld32(r0);
+                    aq[kk][1] = ld32(r0 + 8 * LS);
+                    aq[kk][2] = ld32(r0 + 8);
+                    aq[kk][3] = ld32(r0 + 8 * LS + 8);
                 }
-                const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * j + 2 * t;
-                float2 x0, x1;
-                x0.x = (r0 < M && c < M) ? ex2(sa[0] * sl2 - mU[mt][0]) : 0.f;
-                x0.y = (r0 < M && c + 1 < M) ? ex2(sa[1] * sl2 - mU[mt][0]) : 0.f;
-                x1.x = (r1 < M && c < M) ? ex2(sa[2] * sl2 - mU[mt][1]) : 0.f;
-                x1.y = (r1 < M && c + 1 < M) ? ex2(sa[3] * sl2 - mU[mt][1]) : 0.f;
-                *reinterpret_cast<float2*>(mA + r0 * SM + c) = x0;
-                *reinterpret_cast<float2*>(mA + r1 * SM + c) = x1;
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n) {
+                    float sa[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                    for (int kk = 0; kk < 2; ++kk) {
+                        const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
+                        Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                    }
+                    const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
+                    Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
+                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
+                    Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
+                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+                }
             }
-        }
-        __syncwarp();
-        {
             // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
-            float rs = 0.f, cs = 0.f;
-            if (lane < M) {
-#pragma unroll 4
-                for (int c = 0; c < M; ++c) {
-                    rs += mA[lane * SM + c];
-                    cs += mA[c * SM + lane];
+            float rmax = 0.f, cmax = 0.f;
+#pragma unroll
+            for (int i = 0; i < MT; ++i) {
+                float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n) {
+                    r0 += Ac[i][n][0] + Ac[i][n][1];
+                    r1 += Ac[i][n][2] + Ac[i][n][3];
                 }
+                r0 += __shfl_xor_sync(0xffffffffu, r0, 1);
+                r0 += __shfl_xor_sync(0xffffffffu, r0, 2);
+                r1 += __shfl_xor_sync(0xffffffffu, r1, 1);
+                r1 += __shfl_xor_sync(0xffffffffu, r1, 2);
+                rmax = fmaxf(rmax, fmaxf(r0, r1));
             }
-            const float inv = 1.f / (warp_max(rs) * warp_max(cs));
-            for (int idx = lane; idx < MP * MP; idx += 32) {
-                const int i = idx / MP, j = idx - (idx / MP) * MP;
-                mZ[i * SM + j] = inv * mA[j * SM + i];
-            }
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    float c = 0.f;
+#pragma unroll
+                    for (int i = 0; i < MT; ++i) c += Ac[i][n][e] + Ac[i][n][e + 2];
+                    c += __shfl_xor_sync(0xffffffffu, c, 4);
+                    c += __shfl_xor_sync(0xffffffffu, c, 8);
+                    c += __shfl_xor_sync(0xffffffffu, c, 16);
+                    cmax = fmaxf(cmax, c);
+                }
+            const float alpha = 1.f / (warp_max(rmax) * warp_max(cmax));
+            frag_store<MT, SM>(Ac, mA, g, t);
+            __syncwarp();
+            // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                        Zc[i][n][e] = alpha * mA[c * SM + r];
+                    }
+            frag_store<MT, SM>(Zc, mZ, g, t);
+            __syncwarp();
         }
-        __syncwarp();
 
         // ---------------- back: pseudo-inverse iteration (step 4) ----------------
 #pragma unroll 1
         for (int it = 0; it < iters; ++it) {
-            mm_tf32<MT, SM>(mA, mZ, g, t, [&](int r, int c, float x) {
-                mX[r * SM + c] = x;
-                mT[r * SM + c] = (r == c ? 7.f : 0.f) - x;
-            });
-            mm_tf32<MT, SM>(mX, mT, g, t, [&](int r, int c, float x) { mT[r * SM + c] = (r == c ? 15.f : 0.f) - x; });
-            mm_tf32<MT, SM>(mX, mT, g, t, [&](int r, int c, float x) { mT[r * SM + c] = (r == c ? 13.f : 0.f) - x; });
-            mm_tf32<MT, SM>(mZ, mT, g, t, [&](int r, int c, float x) { mZn[r * SM + c] = 0.25f * x; });
-            float* tmp = mZ;
-            mZ = mZn;
-            mZn = tmp;
+            Frag<MT> X, Tm;
+            mm_smem<MT, SM>(mA, mZ, X, g, t);  // X = A Z
+            // X is symmetric in exact arithmetic; make the computed one exactly
+            // symmetric, (X + X^T)/2, so that every polynomial below is one in a
+            // single symmetric matrix.  (Without this, reading B fragments of
+            // X^T instead of X lets the antisymmetric round-off grow by up to
+            // 13/4 per step in the not-yet-converged directions.)  Z is no longer
+            // needed in shared memory, so its slot holds X for the transpose.
+            __syncwarp();
+            frag_store<MT, SM>(X, mZ, g, t);
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                        X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + r]);
+                    }
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) Tm[i][n][e] = X[i][n][e];
+            frag_shift<MT>(Tm, 7.f, g, t);          // 7I - X
+            {
+                Frag<MT> P;
+                mm_frag_sym<MT>(X, Tm, P);           // X (7I - X)
+                frag_shift<MT>(P, 15.f, g, t);       // 15I - ...
+                mm_frag_sym<MT>(X, P, Tm);           // X (15I - ...)
+            }
+            frag_shift<MT>(Tm, 13.f, g, t);         // 13I - ...
+            {
+                Frag<MT> P;
+                mm_frag_sym<MT>(Zc, Tm, P);          // Z (13I - ...)
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
+            }
+            __syncwarp();
+            frag_store<MT, SM>(Zc, mZ, g, t);
+            __syncwarp();
         }
 
         // ---------------- back: Y = Z W, Y^T as 16-bit B operand ----------------
         {
             float y[MT][NTO][4];
-            float ymax = 0.f;
 #pragma unroll
-            for (int j = 0; j < NTO; ++j) {
+            for (int i = 0; i < MT; ++i)
 #pragma unroll
-                for (int i = 0; i < MT; ++i) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
+                for (int j = 0; j < NTO; ++j) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
 #pragma unroll
-                for (int kk = 0; kk < MP / 8; ++kk) {
-                    const Tf32Pair b[2] = {split_tf32(mW[(8 * kk + t) * WS + 8 * j + g]),
-                                           split_tf32(mW[(8 * kk + t + 4) * WS + 8 * j + g])};
+            for (int kk = 0; kk < 2 * MT; ++kk) {
+                Tf32Pair a[MT][4];
 #pragma unroll
-                    for (int i = 0; i < MT; ++i) {
-                        const float* ar = mZ + (16 * i + g) * SM + 8 * kk + t;
-                        const Tf32Pair a[4] = {split_tf32(ar[0]), split_tf32(ar[8 * SM]), split_tf32(ar[4]),
-                                               split_tf32(ar[8 * SM + 4])};
-                        mma_tf32x3(y[i][j], a, b);
-                    }
+                for (int i = 0; i < MT; ++i) {
+                    a[i][0] = split_tf32(Zc[i][kk][0]);
+                    a[i][1] = split_tf32(Zc[i][kk][2]);
+                    a[i][2] = split_tf32(Zc[i][kk][1]);
+                    a[i][3] = split_tf32(Zc[i][kk][3]);
                 }
 #pragma unroll
-                for (int i = 0; i < MT; ++i)
+                for (int j = 0; j < NTO; ++j) {
+                    const Tf32Pair b[2] = {split_tf32(mW[(8 * kk + 2 * t) * WS + 8 * j + g]),
+                                           split_tf32(mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g])};
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
+                    for (int i = 0; i < MT; ++i) mma_tf32x3(y[i][j], a[i], b);
+                }
             }
             // fp16 has a narrow range: scale Y by a power of two.  Numerator and
             // denominator columns share the factor, so it cancels in step 7.
             float scale = 1.f;
             if (Op::kNarrowRange) {
+                float ymax = 0.f;
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
                 ymax = warp_max(ymax);
                 if (ymax > 0.f) scale = exp2f((float)(14 - ilogbf(ymax)));
             }
@@ -513,16 +622,20 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
                        int iters, cudaStream_t stream) {
     auto kern = nystra_w64_kernel<T, M, NCOL, WARPS>;
     const size_t smem = (size_t)WARPS * Layout64<M, NCOL>::WARP_BYTES;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    int dev = 0, sms = 0, per_sm = 0;
-    if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-    if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, WARPS * 32, smem)) != cudaSuccess)
-        return e;
-    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    static int s_blocks = 0;  // persistent grid size (device-wide), set on first use
+    if (s_blocks == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per_sm = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, WARPS * 32, smem)) != cudaSuccess)
+            return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        s_blocks = sms * per_sm;
+    }
     const long long want = (n_units + WARPS - 1) / WARPS;
-    const long long grid = want < (long long)sms * per_sm ? want : (long long)sms * per_sm;
+    const long long grid = want < s_blocks ? want : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out, n_units,
                                                       d, iters, sl2);
@@ -535,14 +648,14 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
     const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
     switch (m) {
         case 8:
-            return wide ? launch_cfg<T, 8, 40, 8>(q, k, v, out, n_units, d, iters, stream)
-                        : launch_cfg<T, 8, 32, 8>(q, k, v, out, n_units, d, iters, stream);
+            return wide ? launch_cfg<T, 8, 40, 9>(q, k, v, out, n_units, d, iters, stream)
+                        : launch_cfg<T, 8, 32, 9>(q, k, v, out, n_units, d, iters, stream);
         case 16:
-            return wide ? launch_cfg<T, 16, 40, 8>(q, k, v, out, n_units, d, iters, stream)
-                        : launch_cfg<T, 16, 32, 8>(q, k, v, out, n_units, d, iters, stream);
+            return wide ? launch_cfg<T, 16, 40, 9>(q, k, v, out, n_units, d, iters, stream)
+                        : launch_cfg<T, 16, 32, 9>(q, k, v, out, n_units, d, iters, stream);
         default:
-            return wide ? launch_cfg<T, 32, 40, 4>(q, k, v, out, n_units, d, iters, stream)
-                        : launch_cfg<T, 32, 32, 4>(q, k, v, out, n_units, d, iters, stream);
+            return wide ? launch_cfg<T, 32, 40, 5>(q, k, v, out, n_units, d, iters, stream)
+                        : launch_cfg<T, 32, 32, 5>(q, k, v, out, n_units, d, iters, stream);
     }
 }
 

@@ -75,6 +75,18 @@ __device__ __forceinline__ uint32_t to_tf32(float x) {
     asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
     return r;
 }
+// Transpose of an 8x8 matrix of 16-bit elements held one row pair per lane
+// (lane 4r + c holds row r, columns 2c and 2c+1).
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
+    uint32_t y;
+    asm("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
 __device__ __forceinline__ float warp_max(float x) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
@@ -85,6 +97,18 @@ __device__ __forceinline__ float quad_max(float x) {
     return fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 2));
 }
 
+// Split of an fp32 value into two tf32 parts by truncation: x = hi + lo + r
+// with |r| < 2^-20 |x|.  Three tf32 products (lo*hi, hi*lo, hi*hi) then give
+// a product accurate to about 2^-19, close to fp32.
+struct Tf32Pair {
+    uint32_t hi, lo;
+};
+__device__ __forceinline__ Tf32Pair split_tf32(float x) {
+    const uint32_t hi = __float_as_uint(x) & 0xffffe000u;
+    const uint32_t lo = __float_as_uint(x - __uint_as_float(hi)) & 0xffffe000u;
+    return {hi, lo};
+}
+
 // m16n8k8 tf32 MMA, fp32 accumulate: c += a (16x8, row) * b (8x8, col).
 __device__ __forceinline__ void mma_tf32(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                          uint32_t b0, uint32_t b1) {
@@ -92,6 +116,13 @@ __device__ __forceinline__ void mma_tf32(float (&c)[4], uint32_t a0, uint32_t a1
         "{%0,%1,%2,%3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// c += a * b in split-tf32 (a: 4 A-fragment registers, b: 2 B-fragment registers).
+__device__ __forceinline__ void mma_tf32x3(float (&c)[4], const Tf32Pair (&a)[4], const Tf32Pair (&b)[2]) {
+    mma_tf32(c, a[0].lo, a[1].lo, a[2].lo, a[3].lo, b[0].hi, b[1].hi);
+    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].lo, b[1].lo);
+    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].hi, b[1].hi);
 }
 
 // 16-bit MMAs (both operands of the same 16-bit type), fp32 accumulate.
