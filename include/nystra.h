@@ -6,8 +6,8 @@
  * softmax attention of one (window, head) pair,
  *     O = softmax(Q K^T / sqrt(d_h)) V                              (Eq. 1)
  * by the Nystrom approximation of the kernel matrix G = exp(Q K^T/sqrt(d_h)),
- *     G^ = G_L G_A^+ G_U,  O^ = (G^ V) ./ (G^ 1_N)     (Eq. 5-6, Algorithm 1)
- * evaluated in the row-max-stabilised form of Sec. 2.2 (Eq. stable_output).
+ *     G^ = G_L G_A^+ G_U,  O^ = (G^ V) ./ (G^ 1_N)     (Eq. 6-7, Algorithm 1)
+ * evaluated in the row-max-stabilised form of Sec. 2.2 (Eq. 8).
  *
  * Conventions shared by every entry point
  * ---------------------------------------

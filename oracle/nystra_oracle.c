@@ -164,7 +164,7 @@ void oracle_pinv_iteration(const double* A, int m, int iters, double* Z) {
 
 /* ------------------------------------------------------------------ */
 /* One unit of PnP-Nystra, Algorithm 1 in the stabilised form of       */
-/* Eq. (stable_output).  Any stage pointer may be NULL.                */
+/* Eq. 8.  Any stage pointer may be NULL.                               */
 /*   qbar, kbar : m x d   landmarks (step 1)                           */
 /*   mL  : N   row maxima of S_L = Q Kbar^T / sqrt(d)                  */
 /*   mU  : m   row maxima of S_U = Qbar K^T / sqrt(d), over all N keys */

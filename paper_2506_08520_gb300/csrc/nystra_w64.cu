@@ -98,56 +98,93 @@ __device__ __forceinline__ void frag_shift(Frag<MT>& f, float alpha, int g, int 
             }
 }
 
-// D = A B with A given as C-layout fragments (any matrix) and B as C-layout
-// fragments of a symmetric matrix, k permuted as described in the header.
 template <int MT>
-__device__ __forceinline__ void mm_frag_sym(const Frag<MT>& A, const Frag<MT>& B, Frag<MT>& D) {
-    frag_zero<MT>(D);
+using FragLo = uint32_t[MT][2 * MT][4];
+
+template <int MT>
+__device__ __forceinline__ void frag_lo(const Frag<MT>& f, FragLo<MT>& lo) {
 #pragma unroll
-    for (int kk = 0; kk < 2 * MT; ++kk) {
-        Tf32Pair a[MT][4];
+    for (int i = 0; i < MT; ++i)
 #pragma unroll
-        for (int i = 0; i < MT; ++i) {
-            a[i][0] = split_tf32(A[i][kk][0]);
-            a[i][1] = split_tf32(A[i][kk][2]);
-            a[i][2] = split_tf32(A[i][kk][1]);
-            a[i][3] = split_tf32(A[i][kk][3]);
-        }
+        for (int n = 0; n < 2 * MT; ++n)
 #pragma unroll
-        for (int j = 0; j < 2 * MT; ++j) {
-            const Tf32Pair b[2] = {split_tf32(B[j >> 1][kk][(j & 1) * 2]),
-                                   split_tf32(B[j >> 1][kk][(j & 1) * 2 + 1])};
-#pragma unroll
-            for (int i = 0; i < MT; ++i) mma_tf32x3(D[i][j], a[i], b);
-        }
-    }
+            for (int e = 0; e < 4; ++e) lo[i][n][e] = tf32_lo(f[i][n][e]);
 }
 
-// D = A B with both operands row-major fp32 in shared memory (stride SM).
-template <int MT, int SM>
-__device__ __forceinline__ void mm_smem(const float* As, const float* Bs, Frag<MT>& D, int g, int t) {
-    frag_zero<MT>(D);
+// D = A B (MP x MP, fp32 accumulate) on split-tf32 tensor cores.
+//   afrag(i, kk, hi[4], lo[4]) gives the A operand registers of m-tile i,
+//     k-step kk (k permuted as described in the header);
+//   bfrag(kk, j, y[2]) gives the B operand values of k-step kk, n-tile j.
+// Even and odd k-steps accumulate separately, halving each chain of
+// dependent MMAs.
+template <int MT, typename AF, typename BF>
+__device__ __forceinline__ void mm_tc(AF afrag, BF bfrag, Frag<MT>& D) {
+    float acc[2][MT][2 * MT][4];
+#pragma unroll
+    for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int j = 0; j < 2 * MT; ++j) acc[p][i][j][0] = acc[p][i][j][1] = acc[p][i][j][2] = acc[p][i][j][3] = 0.f;
 #pragma unroll
     for (int kk = 0; kk < 2 * MT; ++kk) {
-        Tf32Pair a[MT][4];
+        uint32_t ah[MT][4], al[MT][4];
 #pragma unroll
-        for (int i = 0; i < MT; ++i) {
-            const float2 p = *reinterpret_cast<const float2*>(As + (16 * i + g) * SM + 8 * kk + 2 * t);
-            const float2 r = *reinterpret_cast<const float2*>(As + (16 * i + g + 8) * SM + 8 * kk + 2 * t);
-            a[i][0] = split_tf32(p.x);
-            a[i][1] = split_tf32(r.x);
-            a[i][2] = split_tf32(p.y);
-            a[i][3] = split_tf32(r.y);
-        }
+        for (int i = 0; i < MT; ++i) afrag(i, kk, ah[i], al[i]);
 #pragma unroll
         for (int j = 0; j < 2 * MT; ++j) {
-            const Tf32Pair b[2] = {split_tf32(Bs[(8 * kk + 2 * t) * SM + 8 * j + g]),
-                                   split_tf32(Bs[(8 * kk + 2 * t + 1) * SM + 8 * j + g])};
+            float y[2];
+            bfrag(kk, j, y);
+            const uint32_t bh0 = __float_as_uint(y[0]), bh1 = __float_as_uint(y[1]);
+            const uint32_t bl0 = tf32_lo(y[0]), bl1 = tf32_lo(y[1]);
 #pragma unroll
-            for (int i = 0; i < MT; ++i) mma_tf32x3(D[i][j], a[i], b);
+            for (int i = 0; i < MT; ++i) {
+                float(&c)[4] = acc[kk & 1][i][j];
+                mma_tf32(c, al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
+                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
+                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
+            }
         }
     }
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) D[i][j][e] = acc[0][i][j][e] + acc[1][i][j][e];
 }
+
+// A operand (k-permuted) straight from C-layout fragments with precomputed low parts.
+template <int MT>
+struct AFromFrag {
+    const Frag<MT>& f;
+    const FragLo<MT>& lo;
+    __device__ __forceinline__ void operator()(int i, int kk, uint32_t (&h)[4], uint32_t (&l)[4]) const {
+        h[0] = __float_as_uint(f[i][kk][0]); l[0] = lo[i][kk][0];
+        h[1] = __float_as_uint(f[i][kk][2]); l[1] = lo[i][kk][2];
+        h[2] = __float_as_uint(f[i][kk][1]); l[2] = lo[i][kk][1];
+        h[3] = __float_as_uint(f[i][kk][3]); l[3] = lo[i][kk][3];
+    }
+};
+// B operand of a symmetric matrix from its own C-layout fragments.
+template <int MT>
+struct BFromSymFrag {
+    const Frag<MT>& f;
+    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
+        y[0] = f[j >> 1][kk][(j & 1) * 2];
+        y[1] = f[j >> 1][kk][(j & 1) * 2 + 1];
+    }
+};
+// B operand of a row-major fp32 matrix in shared memory (row stride S).
+template <int S>
+struct BFromSmem {
+    const float* m;
+    int g, t;
+    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
+        y[0] = m[(8 * kk + 2 * t) * S + 8 * j + g];
+        y[1] = m[(8 * kk + 2 * t + 1) * S + 8 * j + g];
+    }
+};
 
 template <int MT, int SM>
 __device__ __forceinline__ void frag_store(const Frag<MT>& f, float* S, int g, int t) {
@@ -382,9 +419,9 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
         }
 
         // ------------- back: G_A^n (fragments), norms, Z_0 -------------
-        Frag<MT> Zc;
+        Frag<MT> Zc, Ac;
+        FragLo<MT> Aclo;
         {
-            Frag<MT> Ac;
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
                 uint32_t aq[2][4];
@@ -453,14 +490,16 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
                         Zc[i][n][e] = alpha * mA[c * SM + r];
                     }
             frag_store<MT, SM>(Zc, mZ, g, t);
+            frag_lo<MT>(Ac, Aclo);
             __syncwarp();
         }
 
         // ---------------- back: pseudo-inverse iteration (step 4) ----------------
 #pragma unroll 1
         for (int it = 0; it < iters; ++it) {
-            Frag<MT> X, Tm;
-            mm_smem<MT, SM>(mA, mZ, X, g, t);  // X = A Z
+            Frag<MT> X, Tm, P;
+            FragLo<MT> Xlo;
+            mm_tc<MT>(AFromFrag<MT>{Ac, Aclo}, BFromSmem<SM>{mZ, g, t}, X);  // X = A Z
             // X is symmetric in exact arithmetic; make the computed one exactly
             // symmetric, (X + X^T)/2, so that every polynomial below is one in a
             // single symmetric matrix.  (Without this, reading B fragments of
@@ -478,31 +517,25 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
                     for (int e = 0; e < 4; ++e) {
                         const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
                         X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + r]);
+                        Tm[i][n][e] = X[i][n][e];
                     }
+            frag_lo<MT>(X, Xlo);
+            frag_shift<MT>(Tm, 7.f, g, t);                                   // 7I - X
+            mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{Tm}, P);     // X (7I - X)
+            frag_shift<MT>(P, 15.f, g, t);                                   // 15I - ...
+            mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{P}, Tm);     // X (15I - ...)
+            frag_shift<MT>(Tm, 13.f, g, t);                                  // 13I - ...
+            {
+                FragLo<MT> Zlo;
+                frag_lo<MT>(Zc, Zlo);
+                mm_tc<MT>(AFromFrag<MT>{Zc, Zlo}, BFromSymFrag<MT>{Tm}, P);  // Z (13I - ...)
+            }
 #pragma unroll
             for (int i = 0; i < MT; ++i)
 #pragma unroll
                 for (int n = 0; n < 2 * MT; ++n)
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) Tm[i][n][e] = X[i][n][e];
-            frag_shift<MT>(Tm, 7.f, g, t);          // 7I - X
-            {
-                Frag<MT> P;
-                mm_frag_sym<MT>(X, Tm, P);           // X (7I - X)
-                frag_shift<MT>(P, 15.f, g, t);       // 15I - ...
-                mm_frag_sym<MT>(X, P, Tm);           // X (15I - ...)
-            }
-            frag_shift<MT>(Tm, 13.f, g, t);         // 13I - ...
-            {
-                Frag<MT> P;
-                mm_frag_sym<MT>(Zc, Tm, P);          // Z (13I - ...)
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
-            }
+                    for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
             __syncwarp();
             frag_store<MT, SM>(Zc, mZ, g, t);
             __syncwarp();
@@ -515,22 +548,25 @@ nystra_w64_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __r
             for (int i = 0; i < MT; ++i)
 #pragma unroll
                 for (int j = 0; j < NTO; ++j) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
+            FragLo<MT> Zlo;
+            frag_lo<MT>(Zc, Zlo);
 #pragma unroll
             for (int kk = 0; kk < 2 * MT; ++kk) {
-                Tf32Pair a[MT][4];
+                uint32_t ah[MT][4], al[MT][4];
 #pragma unroll
-                for (int i = 0; i < MT; ++i) {
-                    a[i][0] = split_tf32(Zc[i][kk][0]);
-                    a[i][1] = split_tf32(Zc[i][kk][2]);
-                    a[i][2] = split_tf32(Zc[i][kk][1]);
-                    a[i][3] = split_tf32(Zc[i][kk][3]);
-                }
+                for (int i = 0; i < MT; ++i) AFromFrag<MT>{Zc, Zlo}(i, kk, ah[i], al[i]);
 #pragma unroll
                 for (int j = 0; j < NTO; ++j) {
-                    const Tf32Pair b[2] = {split_tf32(mW[(8 * kk + 2 * t) * WS + 8 * j + g]),
-                                           split_tf32(mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g])};
+                    const float y0 = mW[(8 * kk + 2 * t) * WS + 8 * j + g];
+                    const float y1 = mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g];
+                    const uint32_t bh0 = __float_as_uint(y0), bh1 = __float_as_uint(y1);
+                    const uint32_t bl0 = tf32_lo(y0), bl1 = tf32_lo(y1);
 #pragma unroll
-                    for (int i = 0; i < MT; ++i) mma_tf32x3(y[i][j], a[i], b);
+                    for (int i = 0; i < MT; ++i) {
+                        mma_tf32(y[i][j], al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
+                        mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
+                        mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
+                    }
                 }
             }
             // fp16 has a narrow range: scale Y by a power of two.  Numerator and

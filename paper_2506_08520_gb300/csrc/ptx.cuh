@@ -97,17 +97,18 @@ __device__ __forceinline__ float quad_max(float x) {
     return fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 2));
 }
 
-// Split of an fp32 value into two tf32 parts by truncation: x = hi + lo + r
-// with |r| < 2^-20 |x|.  Three tf32 products (lo*hi, hi*lo, hi*hi) then give
-// a product accurate to about 2^-19, close to fp32.
+// Split of an fp32 value into two tf32 parts: hi = x with its low 13 mantissa
+// bits cleared (the tensor core ignores those bits of a .tf32 operand, so x
+// itself is passed as hi) and lo = x - hi, exact in fp32 and again truncated
+// to tf32 by the hardware.  hi + lo equals x to within 2^-20 |x|; the three
+// products lo*hi, hi*lo and hi*hi give a product accurate to about 2^-19.
 struct Tf32Pair {
     uint32_t hi, lo;
 };
-__device__ __forceinline__ Tf32Pair split_tf32(float x) {
-    const uint32_t hi = __float_as_uint(x) & 0xffffe000u;
-    const uint32_t lo = __float_as_uint(x - __uint_as_float(hi)) & 0xffffe000u;
-    return {hi, lo};
+__device__ __forceinline__ uint32_t tf32_lo(float x) {
+    return __float_as_uint(x - __uint_as_float(__float_as_uint(x) & 0xffffe000u));
 }
+__device__ __forceinline__ Tf32Pair split_tf32(float x) { return {__float_as_uint(x), tf32_lo(x)}; }
 
 // m16n8k8 tf32 MMA, fp32 accumulate: c += a (16x8, row) * b (8x8, col).
 __device__ __forceinline__ void mma_tf32(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,

@@ -167,7 +167,7 @@ def test_iteration_converges_to_moore_penrose():
 # Steps 2-3: the kernel blocks and their stabilisation.
 # --------------------------------------------------------------------------
 def _extended(q, k, m):
-    """G~ = exp(Q~ K~^T / sqrt(d)) built directly from its definition (Eq. gtilde)."""
+    """G~ = exp(Q~ K~^T / sqrt(d)) built directly from its definition (Eq. 3)."""
     N, d = q.shape
     qb = q.reshape(m, N // m, d).mean(1)
     kb = k.reshape(m, N // m, d).mean(1)
@@ -192,7 +192,7 @@ def test_blocks_match_extended_matrix():
 
 
 def test_stable_form_equals_unnormalised_form():
-    """Eq. (stable_output) with a converged inverse equals Eq. (compact_approxattention)
+    """Eq. 8 (stabilised) with a converged inverse equals Eq. 7
     evaluated without any stabilisation, G^ = G_L G_A^+ G_U with an SVD pinv."""
     rng = _rng(21)
     N, d, m = 64, 16, 8
@@ -219,7 +219,7 @@ def test_every_token_a_landmark_is_exact_attention():
 
 
 def test_corollary_exact_recovery():
-    """Tokens constant within each segment make rank(G~) = m, so G^ = G (Corollary)."""
+    """Tokens constant within each segment make rank(G~) = m, so G^ = G (Corollary 2.2)."""
     rng = _rng(23)
     N, d, m = 64, 8, 8
     L = N // m
@@ -278,7 +278,7 @@ def test_invalid_m_rejected():
 
 
 # --------------------------------------------------------------------------
-# Lemma (spectral bound) in an explicit-constant form, and Table 6's trend.
+# Lemma 2.1 (spectral bound) in an explicit-constant form, and Table 6's trend.
 # --------------------------------------------------------------------------
 def _lemma_terms(q, k, m):
     Gt = _extended(q, k, m)
