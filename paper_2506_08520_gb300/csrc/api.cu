@@ -49,12 +49,18 @@ int nystra_attention(const void* q, const void* k, const void* v, void* out, int
     if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
+    const cudaStream_t s = (cudaStream_t)stream;
+    const bool tc = (dtype == NYSTRA_BF16 || dtype == NYSTRA_F16) && d_h % 2 == 0 && d_h <= 32 &&
+                    (m == 8 || m == 16 || m == 32);
     cudaError_t e;
-    if (nystra_host::nystra_w64_supports(N, d_h, m, dtype))
-        e = nystra_host::launch_nystra_w64(q, k, v, out, units, d_h, m, iters, dtype, (cudaStream_t)stream);
+    if (tc && N == 64)
+        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, dtype, s);
+    else if (tc && N == 256)
+        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, dtype, s);
+    else if (tc && N == 1024)
+        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, dtype, s);
     else
-        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype,
-                                               (cudaStream_t)stream);
+        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype, s);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
@@ -98,6 +104,13 @@ namespace nystra_host {
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
-    return take_fault_word_w64(err);
+    unsigned int w = 0;
+    unsigned int (*const take[3])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
+                                                   take_fault_word_tc_n1024};
+    for (auto f : take) {
+        w |= f(err);
+        if (*err != cudaSuccess) return w;
+    }
+    return w;
 }
 }  // namespace nystra_host

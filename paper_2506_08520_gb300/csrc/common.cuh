@@ -34,11 +34,17 @@ cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, v
                                   cudaStream_t stream);
 cudaError_t launch_exact_generic(const void* q, const void* k, const void* v, void* out,
                                  long long n_units, int N, int d, int dtype, cudaStream_t stream);
-// Tensor-core kernel for 64-token windows with 16-bit I/O (nystra_w64.cu).
-bool nystra_w64_supports(int N, int d, int m, int dtype);
-cudaError_t launch_nystra_w64(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                              int m, int iters, int dtype, cudaStream_t stream);
-unsigned int take_fault_word_w64(cudaError_t* err);
+// Tensor-core kernels, 16-bit I/O, windows of 64 / 256 / 1024 tokens
+// (nystra_tc_n*.cu); m in {8, 16, 32}, even d_h <= 32.
+cudaError_t launch_nystra_tc_n64(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                 int d, int m, int iters, int dtype, cudaStream_t stream);
+cudaError_t launch_nystra_tc_n256(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                  int d, int m, int iters, int dtype, cudaStream_t stream);
+cudaError_t launch_nystra_tc_n1024(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                   int d, int m, int iters, int dtype, cudaStream_t stream);
+unsigned int take_fault_word_tc_n64(cudaError_t* err);
+unsigned int take_fault_word_tc_n256(cudaError_t* err);
+unsigned int take_fault_word_tc_n1024(cudaError_t* err);
 // Device-side fault words (bit 0: a bounded wait gave up) of the translation
 // units whose kernels wait on barriers: OR-ed together, then cleared.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);

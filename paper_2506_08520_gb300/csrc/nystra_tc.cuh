@@ -1,0 +1,872 @@
+// Tensor-core PnP-Nystra kernel template, 16-bit I/O, windows of N = 64,
+// 256 or 1024 tokens (8x8, 16x16, 32x32 windows), m in {8, 16, 32}, even
+// d_h <= 32.  Included by one translation unit per N (nystra_tc_n*.cu).
+//
+// Work decomposition.  A "group" of WPU warps processes one (window, head)
+// unit at a time; a CTA holds GROUPS groups and the grid is persistent
+// (groups stride over units).  Warp r of a group owns tokens
+// [r*TPW, (r+1)*TPW) of the unit and handles them in 64-token chunks.
+//
+// Per unit:
+//   stage    each warp bulk-copies its TPW rows of Q, K and V (contiguous in
+//            HBM) into its private stage with one mbarrier; bounded wait.
+//   front    landmarks (Algorithm 1 step 1) of the segments a warp owns
+//            (segments never straddle warps: N/m <= TPW), to group memory;
+//            [P1] S_L = Q Kbar^T, G_L^n = exp(S_L - m_L) parked as MMA
+//            fragments;  S_U = Qbar K^T with a running row max across the
+//            warp's chunks, G_U^n fed straight from registers into
+//            W_r = G_U^n [V | 1], rescaled online when the max grows.
+//   combine  (WPU > 1) partial (W_r, m_r) of all warps are merged in a fixed
+//            order: m_U = max_r m_r, W = sum_r exp(m_r - m_U) W_r, which is
+//            exactly G_U^n [V | 1] with the max over all N keys.
+//            [P1] the stage is dead now: the next unit's copies are issued.
+//   core     warp 0: G_A^n = exp(Qbar Kbar^T - m_U), Z_0 = A^T/(||A||_1
+//            ||A||_inf), `iters` steps Z <- Z(13I - X(15I - X(7I - X)))/4 with
+//            X = A Z (step 4), Y = Z W, stored as a 16-bit B operand.
+//   output   every warp: O = (G_L^n Y_:d) / (G_L^n Y_d) for its tokens
+//            (steps 5-7), written from registers.  [P2] S_L and G_L^n are
+//            computed here from the still-resident Q, and the next unit's
+//            copies are issued afterwards.
+// P1 ("G_L parked") is used when the fragments fit in shared memory next to
+// the stage; otherwise P2.
+//
+// Arithmetic.  Products with token or d_h extents use mma.sync in the I/O
+// type with fp32 accumulation.  The m x m iteration and Y = Z W use
+// split-tf32 mma.sync (x = hi + lo, three tf32 products), close to fp32: the
+// iteration's round-off is amplified by ||A|| ||Z||, which grows with the
+// iteration count.  The iteration runs in registers: an MMA result feeds the
+// next A operand unchanged under a consistent k permutation (k-slot t <->
+// column 2t, t+4 <-> 2t+1); X = A Z_k and its polynomials are symmetric in
+// exact arithmetic (Z_0 = a A^T), so their B fragments are the lane's own
+// C-layout values of the transpose.  The computed X is symmetrised,
+// (X + X^T)/2, every step, which keeps the antisymmetric round-off from
+// growing by up to 13/4 per step in directions that have not converged.
+// Scores are kept in the log2 domain (scaled by log2(e)/sqrt(d_h)), so each
+// exponential is one FFMA and one ex2.
+#pragma once
+
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace nystra {
+namespace tc {
+
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
+constexpr size_t kSmemLimit = 232448;        // opt-in dynamic shared memory per CTA
+
+template <int M, int NCOL, int TPW, int WPU, bool GLS>
+struct Layout {
+    static constexpr int N = TPW * WPU;
+    static constexpr int NCH = TPW / 64;                 // 64-token chunks per warp
+    static constexpr int DS = (NCOL == 32) ? 30 : 32;    // staged row width bound (d_h <= DS)
+    static constexpr int MT = (M + 15) / 16;             // landmark m-tiles
+    static constexpr int MP = MT * 16;                   // padded landmark count
+    static constexpr int LS = 40;                        // Qbar/Kbar row stride (16-bit elements)
+    static constexpr int SM = MP + 4;                    // fp32 core-matrix row stride
+    static constexpr int WS = NCOL + 4;                  // fp32 W row stride
+    static constexpr int YS = (M < 16 ? 16 : M) + 8;     // Y^T row stride (16-bit elements)
+    static constexpr int KTL = (M >= 16) ? M / 16 : 1;   // k-steps of O = G_L^n Y
+    static constexpr int GLB = (M >= 16) ? 16 : 8;       // bytes per lane per G_L fragment
+    // per-warp private memory: stage (Q, K, V rows of the warp), G_L fragments
+    static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;
+    static constexpr size_t GLF = STAGE;
+    static constexpr size_t WARP_BYTES = ((GLF + (GLS ? (size_t)NCH * 4 * KTL * 32 * GLB : 0) + 127) / 128) * 128;
+    // A warp's partial W (fp32 MP x NCOL, then MP row maxima) lives in its
+    // stage right after the Q rows, once K and V are consumed.
+    static constexpr size_t WPART = (size_t)TPW * DS * 2;
+    static_assert((size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
+    // per-group shared memory
+    static constexpr size_t G_QBAR = 0;
+    static constexpr size_t G_KBAR = G_QBAR + MP * LS * 2;
+    static constexpr size_t G_MU = G_KBAR + MP * LS * 2;  // m_U, log2 domain
+    static constexpr size_t G_W = G_MU + MP * 4;
+    static constexpr size_t G_A = G_W + MP * WS * 4;
+    static constexpr size_t G_Z = G_A + MP * SM * 4;
+    static constexpr size_t G_YT = G_Z + MP * SM * 4;
+    static constexpr size_t G_BAR = G_YT + ((NCOL * YS * 2 + 15) / 16) * 16;
+    static constexpr size_t G_FLAG = G_BAR + 8 * WPU;
+    static constexpr size_t GROUP_BYTES = ((G_FLAG + 16 + 127) / 128) * 128;
+    static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
+};
+
+template <typename T>
+__device__ __forceinline__ uint32_t ld32(const T* p) {
+    return *reinterpret_cast<const uint32_t*>(p);
+}
+
+// C-layout fragments of an MP x MP fp32 matrix: f[i][n][e] is row
+// 16i + g + 8(e >> 1), column 8n + 2t + (e & 1).
+template <int MT>
+using Frag = float[MT][2 * MT][4];
+template <int MT>
+using FragLo = uint32_t[MT][2 * MT][4];
+
+template <int MT>
+__device__ __forceinline__ void frag_lo(const Frag<MT>& f, FragLo<MT>& lo) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) lo[i][n][e] = tf32_lo(f[i][n][e]);
+}
+
+// T = alpha I - D, in place.
+template <int MT>
+__device__ __forceinline__ void frag_shift(Frag<MT>& f, float alpha, int g, int t) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * n + (e & 1) + 2 * t);
+                f[i][n][e] = (diag ? alpha : 0.f) - f[i][n][e];
+            }
+}
+
+// D = A B (MP x MP, fp32 accumulate) on split-tf32 tensor cores.
+//   afrag(i, kk, hi[4], lo[4]) gives the A operand registers of m-tile i,
+//     k-step kk (k permuted as described in the header);
+//   bfrag(kk, j, y[2]) gives the B operand values of k-step kk, n-tile j.
+// Even and odd k-steps accumulate separately, halving each chain of
+// dependent MMAs.
+template <int MT, typename AF, typename BF>
+__device__ __forceinline__ void mm_tc(AF afrag, BF bfrag, Frag<MT>& D) {
+    float acc[2][MT][2 * MT][4];
+#pragma unroll
+    for (int p = 0; p < 2; ++p)
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int j = 0; j < 2 * MT; ++j) acc[p][i][j][0] = acc[p][i][j][1] = acc[p][i][j][2] = acc[p][i][j][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < 2 * MT; ++kk) {
+        uint32_t ah[MT][4], al[MT][4];
+#pragma unroll
+        for (int i = 0; i < MT; ++i) afrag(i, kk, ah[i], al[i]);
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j) {
+            float y[2];
+            bfrag(kk, j, y);
+            const uint32_t bh0 = __float_as_uint(y[0]), bh1 = __float_as_uint(y[1]);
+            const uint32_t bl0 = tf32_lo(y[0]), bl1 = tf32_lo(y[1]);
+#pragma unroll
+            for (int i = 0; i < MT; ++i) {
+                float(&c)[4] = acc[kk & 1][i][j];
+                mma_tf32(c, al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
+                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
+                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) D[i][j][e] = acc[0][i][j][e] + acc[1][i][j][e];
+}
+
+// A operand (k-permuted) straight from C-layout fragments with precomputed low parts.
+template <int MT>
+struct AFromFrag {
+    const Frag<MT>& f;
+    const FragLo<MT>& lo;
+    __device__ __forceinline__ void operator()(int i, int kk, uint32_t (&h)[4], uint32_t (&l)[4]) const {
+        h[0] = __float_as_uint(f[i][kk][0]); l[0] = lo[i][kk][0];
+        h[1] = __float_as_uint(f[i][kk][2]); l[1] = lo[i][kk][2];
+        h[2] = __float_as_uint(f[i][kk][1]); l[2] = lo[i][kk][1];
+        h[3] = __float_as_uint(f[i][kk][3]); l[3] = lo[i][kk][3];
+    }
+};
+// B operand of a symmetric matrix from its own C-layout fragments.
+template <int MT>
+struct BFromSymFrag {
+    const Frag<MT>& f;
+    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
+        y[0] = f[j >> 1][kk][(j & 1) * 2];
+        y[1] = f[j >> 1][kk][(j & 1) * 2 + 1];
+    }
+};
+// B operand of a row-major fp32 matrix in shared memory (row stride S).
+template <int S>
+struct BFromSmem {
+    const float* m;
+    int g, t;
+    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
+        y[0] = m[(8 * kk + 2 * t) * S + 8 * j + g];
+        y[1] = m[(8 * kk + 2 * t + 1) * S + 8 * j + g];
+    }
+};
+
+template <int MT, int SM>
+__device__ __forceinline__ void frag_store(const Frag<MT>& f, float* S, int g, int t) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n) {
+            const int r = 16 * i + g, c = 8 * n + 2 * t;
+            *reinterpret_cast<float2*>(S + r * SM + c) = make_float2(f[i][n][0], f[i][n][1]);
+            *reinterpret_cast<float2*>(S + (r + 8) * SM + c) = make_float2(f[i][n][2], f[i][n][3]);
+        }
+}
+
+// S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
+// fragments (A operand of O = G_L^n Y, k = landmarks).
+template <typename T, int M, int KTL>
+__device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g, int t, float sl2,
+                                        uint32_t (&f)[KTL][4]) {
+    using Op = Mma16<T>;
+    constexpr int NTL = M / 8, LS = 40;
+    uint32_t a[2][4];
+    const T* q1 = q0 + 8 * d;
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+        const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
+        a[kk][0] = c0 < d ? ld32(q0 + c0) : 0u;
+        a[kk][1] = c0 < d ? ld32(q1 + c0) : 0u;
+        a[kk][2] = c1 < d ? ld32(q0 + c1) : 0u;
+        a[kk][3] = c1 < d ? ld32(q1 + c1) : 0u;
+    }
+    float sl[NTL][4];
+#pragma unroll
+    for (int j = 0; j < NTL; ++j) {
+        sl[j][0] = sl[j][1] = sl[j][2] = sl[j][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const T* kr = kbar + (8 * j + g) * LS + 16 * kk + 2 * t;
+            Op::k16(sl[j], a[kk], ld32(kr), ld32(kr + 8));
+        }
+    }
+    float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < NTL; ++j) {
+        mx0 = fmaxf(mx0, fmaxf(sl[j][0], sl[j][1]));
+        mx1 = fmaxf(mx1, fmaxf(sl[j][2], sl[j][3]));
+    }
+    mx0 = quad_max(mx0) * sl2;
+    mx1 = quad_max(mx1) * sl2;
+    auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+    auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+    if constexpr (M >= 16) {
+#pragma unroll
+        for (int kk = 0; kk < KTL; ++kk) {
+            f[kk][0] = Op::pack(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
+            f[kk][1] = Op::pack(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
+            f[kk][2] = Op::pack(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
+            f[kk][3] = Op::pack(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
+        }
+    } else {
+        f[0][0] = Op::pack(e0(sl[0][0]), e0(sl[0][1]));
+        f[0][1] = Op::pack(e1(sl[0][2]), e1(sl[0][3]));
+        f[0][2] = f[0][3] = 0u;
+    }
+}
+
+template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS>
+__global__ void __launch_bounds__(GROUPS * WPU * 32, 1)
+nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
+                 T* __restrict__ out, long long n_units, int d, int iters, float sl2,
+                 unsigned int* fault) {
+    using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
+    using Op = Mma16<T>;
+    constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS, SM = Lay::SM,
+                  WS = Lay::WS, YS = Lay::YS, KTL = Lay::KTL, NTO = NCOL / 8;
+    constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
+    constexpr int LPW = TPW / L;  // landmarks owned by one warp
+    static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
+
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = warp / WPU, r = warp - grp * WPU;
+    const int g = lane >> 2, t = lane & 3;
+    unsigned char* gb = smem_raw + (size_t)grp * Lay::GROUP_BYTES;
+    unsigned char* wb = smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES + (size_t)warp * Lay::WARP_BYTES;
+    const int td = TPW * d;  // elements per staged tensor
+    T* Qs = reinterpret_cast<T*>(wb);
+    T* Ks = Qs + td;
+    T* Vs = Qs + 2 * td;
+    uint32_t* glf = reinterpret_cast<uint32_t*>(wb + Lay::GLF);
+    float* wpart = reinterpret_cast<float*>(wb + Lay::WPART);
+    T* qbar = reinterpret_cast<T*>(gb + Lay::G_QBAR);
+    T* kbar = reinterpret_cast<T*>(gb + Lay::G_KBAR);
+    float* gmu = reinterpret_cast<float*>(gb + Lay::G_MU);
+    float* mW = reinterpret_cast<float*>(gb + Lay::G_W);
+    float* mA = reinterpret_cast<float*>(gb + Lay::G_A);
+    float* mZ = reinterpret_cast<float*>(gb + Lay::G_Z);
+    T* yT = reinterpret_cast<T*>(gb + Lay::G_YT);
+    uint64_t* bar = reinterpret_cast<uint64_t*>(gb + Lay::G_BAR) + r;
+    volatile unsigned int* gflag = reinterpret_cast<volatile unsigned int*>(gb + Lay::G_FLAG);
+
+    auto gsync = [&]() {
+        if constexpr (WPU == 1) __syncwarp();
+        else named_barrier(1 + grp, WPU * 32);
+    };
+
+    const long long stride = (long long)gridDim.x * GROUPS;
+    long long u = (long long)blockIdx.x * GROUPS + grp;
+    const uint32_t tile_bytes = (uint32_t)(td * sizeof(T));
+    auto issue = [&](long long unit) {
+        const size_t off = (size_t)unit * N * d + (size_t)r * td;
+        mbar_arrive_expect_tx(bar, 3u * tile_bytes);
+        bulk_g2s(Qs, q + off, tile_bytes, bar);
+        bulk_g2s(Ks, k + off, tile_bytes, bar);
+        bulk_g2s(Vs, v + off, tile_bytes, bar);
+    };
+
+    if (lane == 0) {
+        mbar_init(bar, 1);
+        fence_mbar_init();
+        if (r == 0) *gflag = 0u;
+    }
+    gsync();
+    if (u < n_units && lane == 0) issue(u);
+    uint32_t phase = 0;
+
+    for (; u < n_units; u += stride) {
+        // ---------------- stage: bounded wait ----------------
+        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
+        if (!ok && lane == 0) {
+            atomicOr(fault, 1u);
+            *gflag = 1u;  // the whole group stops after the next barrier
+        }
+        phase ^= 1u;
+
+        // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
+        {
+            const float invL = 1.f / (float)L;
+            const int dp = d >> 1;
+            for (int idx = lane; idx < LPW * 16; idx += 32) {
+                const int jl = idx >> 4, p = idx & 15;
+                float ax = 0.f, ay = 0.f, bx = 0.f, by = 0.f;
+                if (p < dp) {
+#pragma unroll 4
+                    for (int rr = 0; rr < L; ++rr) {
+                        const int off = (jl * L + rr) * d + 2 * p;
+                        const float2 a = Op::unpack(ld32(Qs + off));
+                        const float2 b = Op::unpack(ld32(Ks + off));
+                        ax += a.x; ay += a.y; bx += b.x; by += b.y;
+                    }
+                    ax *= invL; ay *= invL; bx *= invL; by *= invL;
+                }
+                const int j = r * LPW + jl;
+                *reinterpret_cast<uint32_t*>(qbar + j * LS + 2 * p) = Op::pack(ax, ay);
+                *reinterpret_cast<uint32_t*>(kbar + j * LS + 2 * p) = Op::pack(bx, by);
+            }
+            if (M < MP && r == 0) {  // zero the padding landmark rows
+                for (int idx = lane; idx < (MP - M) * 16; idx += 32) {
+                    const int j = M + (idx >> 4), p = idx & 15;
+                    *reinterpret_cast<uint32_t*>(qbar + j * LS + 2 * p) = 0u;
+                    *reinterpret_cast<uint32_t*>(kbar + j * LS + 2 * p) = 0u;
+                }
+            }
+        }
+        gsync();
+        if (WPU == 1 ? !ok : (*gflag != 0u)) break;
+
+        // ---------------- front [P1]: S_L, G_L^n fragments ----------------
+        if constexpr (GLS) {
+#pragma unroll 1
+            for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                for (int tm = 0; tm < 4; ++tm) {
+                    uint32_t f[KTL][4];
+                    gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
+#pragma unroll
+                    for (int kk = 0; kk < KTL; ++kk) {
+                        const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
+                        if constexpr (M >= 16)
+                            reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[kk][0], f[kk][1], f[kk][2], f[kk][3]);
+                        else
+                            reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[kk][0], f[kk][1]);
+                    }
+                }
+        }
+
+        // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
+        float mU[MT][2];       // this warp's row maxima of S_U, log2 domain
+        float wall[MT][NTO][4];  // W_r rows of every m-tile (stored after the loop:
+                                 // with several warps the partial goes to the K/V stage)
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            uint32_t aq[2][4];
+#pragma unroll
+            for (int kk = 0; kk < 2; ++kk) {
+                const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+                aq[kk][0] = ld32(r0);
+                aq[kk][1] = ld32(r0 + 8 * LS);
+                aq[kk][2] = ld32(r0 + 8);
+                aq[kk][3] = ld32(r0 + 8 * LS + 8);
+            }
+            const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
+            float(&w)[NTO][4] = wall[mt];
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
+            float run0 = -INFINITY, run1 = -INFINITY;
+#pragma unroll 1
+            for (int ch = 0; ch < NCH; ++ch) {
+                const T* Kc = Ks + ch * 64 * d;
+                const T* Vc = Vs + ch * 64 * d;
+                float s[8][4];
+#pragma unroll
+                for (int nt = 0; nt < 8; ++nt) {
+                    s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+                    const T* kr = Kc + (8 * nt + g) * d;
+#pragma unroll
+                    for (int kk = 0; kk < 2; ++kk) {
+                        const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
+                        const uint32_t b0 = c0 < d ? ld32(kr + c0) : 0u;
+                        const uint32_t b1 = c1 < d ? ld32(kr + c1) : 0u;
+                        Op::k16(s[nt], aq[kk], b0, b1);
+                    }
+                }
+                float mx0 = run0, mx1 = run1;
+#pragma unroll
+                for (int nt = 0; nt < 8; ++nt) {
+                    mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
+                    mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
+                }
+                mx0 = quad_max(mx0);
+                mx1 = quad_max(mx1);
+                if (NCH > 1) {  // online rescaling of the accumulated W rows
+                    const float f0 = ex2(run0 - mx0), f1 = ex2(run1 - mx1);
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        w[j][0] *= f0; w[j][1] *= f0; w[j][2] *= f1; w[j][3] *= f1;
+                    }
+                }
+                run0 = mx0;
+                run1 = mx1;
+                auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+                auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+                // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
+#pragma unroll
+                for (int kt = 0; kt < 4; ++kt) {
+                    uint32_t a[4];
+                    a[0] = v0 ? Op::pack(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : 0u;
+                    a[1] = v1 ? Op::pack(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : 0u;
+                    a[2] = v0 ? Op::pack(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : 0u;
+                    a[3] = v1 ? Op::pack(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : 0u;
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        const int c0 = 8 * j + 2 * t;
+                        const uint32_t x0 = c0 < d ? ld32(Vc + (16 * kt + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
+                        const uint32_t x1 = c0 < d ? ld32(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
+                        Op::k16(w[j], a, movmatrix_trans(x0), movmatrix_trans(x1));
+                    }
+                }
+            }
+            mU[mt][0] = run0;
+            mU[mt][1] = run1;
+        }
+        {
+            float* dst = (WPU == 1) ? mW : wpart;
+            const int ws = (WPU == 1) ? WS : NCOL;
+            if (WPU > 1) __syncwarp();  // every lane is done reading K and V
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) {
+                    const int rr = 16 * mt + g, c = 8 * j + 2 * t;
+                    *reinterpret_cast<float2*>(dst + rr * ws + c) = make_float2(wall[mt][j][0], wall[mt][j][1]);
+                    *reinterpret_cast<float2*>(dst + (rr + 8) * ws + c) =
+                        make_float2(wall[mt][j][2], wall[mt][j][3]);
+                }
+                if (WPU > 1 && t == 0) {
+                    wpart[MP * NCOL + 16 * mt + g] = mU[mt][0];
+                    wpart[MP * NCOL + 16 * mt + g + 8] = mU[mt][1];
+                }
+            }
+        }
+
+        // ---------------- combine (WPU > 1) ----------------
+        if constexpr (WPU > 1) {
+            gsync();
+            const float* part0 = reinterpret_cast<const float*>(smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
+                                                                (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART);
+            for (int e = r * 32 + lane; e < MP * NCOL; e += WPU * 32) {
+                const int i = e / NCOL, c = e - (e / NCOL) * NCOL;
+                float mu = -INFINITY;
+#pragma unroll
+                for (int s2 = 0; s2 < WPU; ++s2)
+                    mu = fmaxf(mu, part0[(size_t)s2 * (Lay::WARP_BYTES / 4) + MP * NCOL + i]);
+                float acc = 0.f;
+#pragma unroll
+                for (int s2 = 0; s2 < WPU; ++s2) {
+                    const float* ps = part0 + (size_t)s2 * (Lay::WARP_BYTES / 4);
+                    acc = fmaf(ex2(ps[MP * NCOL + i] - mu), ps[i * NCOL + c], acc);
+                }
+                mW[i * WS + c] = acc;
+                if (c == 0) gmu[i] = mu;
+            }
+        }
+        gsync();
+
+        // [P1] Q, K, V of this unit are consumed: prefetch the next unit.
+        if constexpr (GLS) {
+            const long long un = u + stride;
+            if (un < n_units && lane == 0) {
+                fence_proxy_async_smem();
+                issue(un);
+            }
+        }
+
+        // ---------------- core (warp 0): G_A^n, Z_0, iteration, Y ----------------
+        if (r == 0) {
+            if constexpr (WPU > 1) {
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) {
+                    mU[mt][0] = gmu[16 * mt + g];
+                    mU[mt][1] = gmu[16 * mt + g + 8];
+                }
+            }
+            Frag<MT> Zc, Ac;
+            FragLo<MT> Aclo;
+            {
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) {
+                    uint32_t aq[2][4];
+#pragma unroll
+                    for (int kk = 0; kk < 2; ++kk) {
+                        const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+                        aq[kk][0] = ld32(r0);
+                        aq[kk][1] = ld32(r0 + 8 * LS);
+                        aq[kk][2] = ld32(r0 + 8);
+                        aq[kk][3] = ld32(r0 + 8 * LS + 8);
+                    }
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n) {
+                        float sa[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                        for (int kk = 0; kk < 2; ++kk) {
+                            const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
+                            Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                        }
+                        const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
+                        Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
+                        Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
+                        Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
+                        Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+                    }
+                }
+                // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
+                float rmax = 0.f, cmax = 0.f;
+#pragma unroll
+                for (int i = 0; i < MT; ++i) {
+                    float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n) {
+                        r0 += Ac[i][n][0] + Ac[i][n][1];
+                        r1 += Ac[i][n][2] + Ac[i][n][3];
+                    }
+                    r0 += __shfl_xor_sync(0xffffffffu, r0, 1);
+                    r0 += __shfl_xor_sync(0xffffffffu, r0, 2);
+                    r1 += __shfl_xor_sync(0xffffffffu, r1, 1);
+                    r1 += __shfl_xor_sync(0xffffffffu, r1, 2);
+                    rmax = fmaxf(rmax, fmaxf(r0, r1));
+                }
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e) {
+                        float c = 0.f;
+#pragma unroll
+                        for (int i = 0; i < MT; ++i) c += Ac[i][n][e] + Ac[i][n][e + 2];
+                        c += __shfl_xor_sync(0xffffffffu, c, 4);
+                        c += __shfl_xor_sync(0xffffffffu, c, 8);
+                        c += __shfl_xor_sync(0xffffffffu, c, 16);
+                        cmax = fmaxf(cmax, c);
+                    }
+                const float alpha = 1.f / (warp_max(rmax) * warp_max(cmax));
+                frag_store<MT, SM>(Ac, mA, g, t);
+                __syncwarp();
+                // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                            Zc[i][n][e] = alpha * mA[c * SM + rr];
+                        }
+                frag_store<MT, SM>(Zc, mZ, g, t);
+                frag_lo<MT>(Ac, Aclo);
+                __syncwarp();
+            }
+
+            // pseudo-inverse iteration (step 4)
+#pragma unroll 1
+            for (int it = 0; it < iters; ++it) {
+                Frag<MT> X, Tm, P;
+                FragLo<MT> Xlo;
+                mm_tc<MT>(AFromFrag<MT>{Ac, Aclo}, BFromSmem<SM>{mZ, g, t}, X);  // X = A Z
+                // exact symmetrisation (X + X^T)/2; Z's slot holds X for the transpose
+                __syncwarp();
+                frag_store<MT, SM>(X, mZ, g, t);
+                __syncwarp();
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                            X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + rr]);
+                            Tm[i][n][e] = X[i][n][e];
+                        }
+                frag_lo<MT>(X, Xlo);
+                frag_shift<MT>(Tm, 7.f, g, t);                                // 7I - X
+                mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{Tm}, P);  // X (7I - X)
+                frag_shift<MT>(P, 15.f, g, t);                                // 15I - ...
+                mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{P}, Tm);  // X (15I - ...)
+                frag_shift<MT>(Tm, 13.f, g, t);                               // 13I - ...
+                {
+                    FragLo<MT> Zlo;
+                    frag_lo<MT>(Zc, Zlo);
+                    mm_tc<MT>(AFromFrag<MT>{Zc, Zlo}, BFromSymFrag<MT>{Tm}, P);  // Z (13I - ...)
+                }
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
+                __syncwarp();
+                frag_store<MT, SM>(Zc, mZ, g, t);
+                __syncwarp();
+            }
+
+            // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
+            {
+                float y[MT][NTO][4];
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
+                FragLo<MT> Zlo;
+                frag_lo<MT>(Zc, Zlo);
+#pragma unroll
+                for (int kk = 0; kk < 2 * MT; ++kk) {
+                    uint32_t ah[MT][4], al[MT][4];
+#pragma unroll
+                    for (int i = 0; i < MT; ++i) AFromFrag<MT>{Zc, Zlo}(i, kk, ah[i], al[i]);
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        const float y0 = mW[(8 * kk + 2 * t) * WS + 8 * j + g];
+                        const float y1 = mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g];
+                        const uint32_t bh0 = __float_as_uint(y0), bh1 = __float_as_uint(y1);
+                        const uint32_t bl0 = tf32_lo(y0), bl1 = tf32_lo(y1);
+#pragma unroll
+                        for (int i = 0; i < MT; ++i) {
+                            mma_tf32(y[i][j], al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
+                            mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
+                            mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
+                        }
+                    }
+                }
+                // fp16 has a narrow range: scale Y by a power of two.  Numerator and
+                // denominator columns share the factor, so it cancels in step 7.
+                float scale = 1.f;
+                if (Op::kNarrowRange) {
+                    float ymax = 0.f;
+#pragma unroll
+                    for (int i = 0; i < MT; ++i)
+#pragma unroll
+                        for (int j = 0; j < NTO; ++j)
+#pragma unroll
+                            for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
+                    ymax = warp_max(ymax);
+                    if (ymax > 0.f) scale = exp2f((float)(14 - ilogbf(ymax)));
+                }
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        const int rr = 16 * i + g, c = 8 * j + 2 * t;
+                        yT[c * YS + rr] = from_f32<T>(y[i][j][0] * scale);
+                        yT[(c + 1) * YS + rr] = from_f32<T>(y[i][j][1] * scale);
+                        yT[c * YS + rr + 8] = from_f32<T>(y[i][j][2] * scale);
+                        yT[(c + 1) * YS + rr + 8] = from_f32<T>(y[i][j][3] * scale);
+                    }
+            }
+        }
+        gsync();
+
+        // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
+        {
+            uint32_t by[KTL][NTO][2];
+#pragma unroll
+            for (int kk = 0; kk < KTL; ++kk)
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) {
+                    const T* yr = yT + (8 * j + g) * YS + 16 * kk + 2 * t;
+                    by[kk][j][0] = ld32(yr);
+                    by[kk][j][1] = (M >= 16) ? ld32(yr + 8) : 0u;
+                }
+            const int jd = d >> 3, tdn = (d & 7) >> 1;
+            const int src = (lane & ~3) | tdn;
+            T* obase = out + (size_t)u * N * d + (size_t)r * td;
+#pragma unroll 1
+            for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                for (int tm = 0; tm < 4; ++tm) {
+                    uint32_t f[KTL][4];
+                    if constexpr (GLS) {
+#pragma unroll
+                        for (int kk = 0; kk < KTL; ++kk) {
+                            const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
+                            if constexpr (M >= 16) {
+                                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+                                f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = x.z; f[kk][3] = x.w;
+                            } else {
+                                const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
+                                f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = f[kk][3] = 0u;
+                            }
+                        }
+                    } else {
+                        gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
+                    }
+                    float o[NTO][4];
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+                    if constexpr (M >= 16) {
+#pragma unroll
+                        for (int kk = 0; kk < KTL; ++kk)
+#pragma unroll
+                            for (int j = 0; j < NTO; ++j) Op::k16(o[j], f[kk], by[kk][j][0], by[kk][j][1]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < NTO; ++j) Op::k8(o[j], f[0][0], f[0][1], by[0][j][0]);
+                    }
+                    float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j)
+                        if (j == jd) {
+                            d0 = o[j][0];
+                            d1 = o[j][2];
+                        }
+                    const float i0 = __fdividef(1.f, __shfl_sync(0xffffffffu, d0, src));
+                    const float i1 = __fdividef(1.f, __shfl_sync(0xffffffffu, d1, src));
+                    T* o0 = obase + (ch * 64 + 16 * tm + g) * d;
+                    T* o1 = o0 + 8 * d;
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        const int c = 8 * j + 2 * t;
+                        if (c < d) {
+                            *reinterpret_cast<uint32_t*>(o0 + c) = Op::pack(o[j][0] * i0, o[j][1] * i0);
+                            *reinterpret_cast<uint32_t*>(o1 + c) = Op::pack(o[j][2] * i1, o[j][3] * i1);
+                        }
+                    }
+                }
+        }
+
+        // [P2] Q was needed until now: every warp of the group is done reading
+        // the landmarks before anyone overwrites them, then prefetch.
+        if constexpr (!GLS) {
+            gsync();
+            const long long un = u + stride;
+            if (un < n_units && lane == 0) {
+                fence_proxy_async_smem();
+                issue(un);
+            }
+        }
+        __syncwarp();
+    }
+}
+
+// Largest number of groups per CTA that fits the shared-memory and register
+// budgets (M <= 16 needs about 160 registers per thread, M = 32 about 255).
+template <int M, int NCOL, int TPW, int WPU, bool GLS>
+constexpr int groups_that_fit() {
+    using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
+    const int by_smem = (int)(kSmemLimit / Lay::PER_GROUP);
+    const int by_regs = ((M <= 16) ? 12 : 8) / WPU;
+    const int n = by_smem < by_regs ? by_smem : by_regs;
+    return n > 15 ? 15 : n;
+}
+
+template <typename T, int M, int NCOL, int TPW, int WPU>
+cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                       int iters, cudaStream_t stream, unsigned int* fault) {
+    constexpr bool kGls = groups_that_fit<M, NCOL, TPW, WPU, true>() >= 1;
+    constexpr int kGroups = groups_that_fit<M, NCOL, TPW, WPU, kGls>();
+    static_assert(kGroups >= 1, "configuration does not fit on one SM");
+    using Lay = Layout<M, NCOL, TPW, WPU, kGls>;
+    auto kern = nystra_tc_kernel<T, M, NCOL, TPW, WPU, kGroups, kGls>;
+    const size_t smem = (size_t)kGroups * Lay::PER_GROUP;
+    static int s_blocks = 0;  // persistent grid size, set on first use
+    if (s_blocks == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per_sm = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGroups * WPU * 32, smem)) !=
+            cudaSuccess)
+            return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        s_blocks = sms * per_sm;
+    }
+    const long long want = (n_units + kGroups - 1) / kGroups;
+    const long long grid = want < s_blocks ? want : s_blocks;
+    const float sl2 = 1.4426950408889634f / sqrtf((float)d);
+    kern<<<(unsigned)grid, kGroups * WPU * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
+                                                              n_units, d, iters, sl2, fault);
+    return cudaGetLastError();
+}
+
+// Dispatch on m and the output-column padding for one window size.
+template <typename T, int TPW, int WPU>
+cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
+                     int iters, cudaStream_t stream, unsigned int* fault) {
+    const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
+    switch (m) {
+        case 8:
+            return wide ? launch_cfg<T, 8, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 8, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
+        case 16:
+            return wide ? launch_cfg<T, 16, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 16, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
+        default:
+            return wide ? launch_cfg<T, 32, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 32, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+}
+
+}  // namespace tc
+}  // namespace nystra
+
+// One translation unit per window size defines its fault word and entry points.
+#define NYSTRA_TC_DEFINE(NAME, TPW, WPU)                                                                     \
+    namespace nystra {                                                                                       \
+    __device__ unsigned int g_fault_tc_##NAME;                                                               \
+    }                                                                                                        \
+    namespace nystra_host {                                                                                  \
+    cudaError_t launch_nystra_tc_##NAME(const void* q, const void* k, const void* v, void* out,              \
+                                        long long n_units, int d, int m, int iters, int dtype,               \
+                                        cudaStream_t stream) {                                               \
+        static unsigned int* s_fault[64] = {};  /* device address of the fault word, per device */      \
+        int dev = 0;                                                                                         \
+        cudaError_t e = cudaGetDevice(&dev);                                                                 \
+        if (e != cudaSuccess) return e;                                                                      \
+        if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;                                             \
+        if (!s_fault[dev]) {                                                                                 \
+            e = cudaGetSymbolAddress((void**)&s_fault[dev], nystra::g_fault_tc_##NAME);                      \
+            if (e != cudaSuccess) return e;                                                                  \
+        }                                                                                                    \
+        unsigned int* fault = s_fault[dev];                                                                  \
+        if (dtype == 1)                                                                                      \
+            return nystra::tc::launch_n<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, \
+                                                                 fault);                                     \
+        return nystra::tc::launch_n<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault);    \
+    }                                                                                                        \
+    unsigned int take_fault_word_tc_##NAME(cudaError_t* err) {                                               \
+        unsigned int w = 0, zero = 0;                                                                        \
+        *err = cudaMemcpyFromSymbol(&w, nystra::g_fault_tc_##NAME, sizeof(w));                               \
+        if (*err == cudaSuccess && w != 0)                                                                   \
+            *err = cudaMemcpyToSymbol(nystra::g_fault_tc_##NAME, &zero, sizeof(zero));                       \
+        return w;                                                                                            \
+    }                                                                                                        \
+    }
