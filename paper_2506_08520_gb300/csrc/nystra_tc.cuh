@@ -31,14 +31,15 @@
 // the stage; otherwise P2.
 //
 // Arithmetic.  Products with token or d_h extents use mma.sync in the I/O
-// type with fp32 accumulation.  The m x m iteration and Y = Z W use
-// split-tf32 mma.sync (x = hi + lo, three tf32 products), close to fp32: the
-// iteration's round-off is amplified by ||A|| ||Z||, which grows with the
-// iteration count.  The iteration runs in registers: an MMA result feeds the
-// next A operand unchanged under a consistent k permutation (k-slot t <->
-// column 2t, t+4 <-> 2t+1); X = A Z_k and its polynomials are symmetric in
-// exact arithmetic (Z_0 = a A^T), so their B fragments are the lane's own
-// C-layout values of the transpose.  The computed X is symmetrised,
+// type with fp32 accumulation.  The m x m iteration needs close to fp32
+// accuracy (its round-off is amplified by ||A|| ||Z||, which grows with the
+// iteration count): it uses fp16 two-term splits (x = hi + lo, three k16
+// products lo*hi + hi*lo + hi*hi, 22 significant bits), with Z carried as
+// 2^e Z, e re-chosen every step, to stay in fp16's range.  Y = Z W uses
+// split-tf32 (W's range is not bounded).  The iteration runs in registers:
+// an MMA result is the next A operand (C layout -> A layout); X = A Z_k and
+// its polynomials are symmetric in exact arithmetic (Z_0 = a A^T), so their
+// B fragments are the lane's own C-layout values of the transpose.  The computed X is symmetrised,
 // (X + X^T)/2, every step, which keeps the antisymmetric round-off from
 // growing by up to 13/4 per step in directions that have not converged.
 // Scores are kept in the log2 domain (scaled by log2(e)/sqrt(d_h)), so each
@@ -200,6 +201,107 @@ struct BFromSmem {
     }
 };
 
+// ---- fp16 two-term split products for the m x m iteration ----
+// A operand registers (m16n8k16 row layout) of every m-tile i and k-step kk,
+// each register split into hi and lo halves.
+template <int MT>
+using HFrag = H2Pair[MT][MT][4];
+
+// A operand from C-layout fragments: k-step kk spans n-tiles 2kk and 2kk+1.
+template <int MT>
+__device__ __forceinline__ void to_hfrag(const Frag<MT>& c, HFrag<MT>& a) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int kk = 0; kk < MT; ++kk) {
+            a[i][kk][0] = split_h2(c[i][2 * kk][0], c[i][2 * kk][1]);
+            a[i][kk][1] = split_h2(c[i][2 * kk][2], c[i][2 * kk][3]);
+            a[i][kk][2] = split_h2(c[i][2 * kk + 1][0], c[i][2 * kk + 1][1]);
+            a[i][kk][3] = split_h2(c[i][2 * kk + 1][2], c[i][2 * kk + 1][3]);
+        }
+}
+
+// D = A B with A split in registers and B supplied by bfrag(kk, j, b[2]);
+// lo*hi + hi*lo and hi*hi accumulate separately (shorter dependent chains).
+template <int MT, typename BF>
+__device__ __forceinline__ void mm_h(const HFrag<MT>& A, BF bfrag, Frag<MT>& D) {
+    using H = Mma16<__half>;
+    float small[MT][2 * MT][4], big[MT][2 * MT][4];
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) small[i][j][e] = big[i][j][e] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j) {
+            H2Pair b[2];
+            bfrag(kk, j, b);
+#pragma unroll
+            for (int i = 0; i < MT; ++i) {
+                const uint32_t ahi[4] = {A[i][kk][0].hi, A[i][kk][1].hi, A[i][kk][2].hi, A[i][kk][3].hi};
+                const uint32_t alo[4] = {A[i][kk][0].lo, A[i][kk][1].lo, A[i][kk][2].lo, A[i][kk][3].lo};
+                H::k16(small[i][j], alo, b[0].hi, b[1].hi);
+                H::k16(small[i][j], ahi, b[0].lo, b[1].lo);
+                H::k16(big[i][j], ahi, b[0].hi, b[1].hi);
+            }
+        }
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) D[i][j][e] = big[i][j][e] + small[i][j][e];
+}
+
+// B operand (m16n8k16 col layout) of a symmetric matrix from its C-layout fragments.
+template <int MT>
+struct BSymH {
+    const Frag<MT>& f;
+    __device__ __forceinline__ void operator()(int kk, int j, H2Pair (&b)[2]) const {
+        const int i = j >> 1, e = (j & 1) * 2;
+        b[0] = split_h2(f[i][2 * kk][e], f[i][2 * kk][e + 1]);
+        b[1] = split_h2(f[i][2 * kk + 1][e], f[i][2 * kk + 1][e + 1]);
+    }
+};
+// B operand of a row-major fp32 matrix in shared memory (row stride S).
+template <int S>
+struct BSmemH {
+    const float* m;
+    int g, t;
+    __device__ __forceinline__ void operator()(int kk, int j, H2Pair (&b)[2]) const {
+        const float* c = m + (16 * kk + 2 * t) * S + 8 * j + g;
+        b[0] = split_h2(c[0], c[S]);
+        b[1] = split_h2(c[8 * S], c[9 * S]);
+    }
+};
+
+// Multiply fragments by 2^e with e chosen so that max |f| lands in
+// [2^10, 2^11) (fp16 headroom for the products); returns e (0 if f == 0).
+template <int MT>
+__device__ __forceinline__ int frag_normalise(Frag<MT>& f) {
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) mx = fmaxf(mx, fabsf(f[i][n][e]));
+    mx = warp_max_nonneg(mx);
+    if (!(mx > 0.f) || !(mx < INFINITY)) return 0;
+    const int e = 10 - ilogbf(mx);
+    const float s = ldexpf(1.f, e);
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int k = 0; k < 4; ++k) f[i][n][k] *= s;
+    return e;
+}
+
 template <int MT, int SM>
 __device__ __forceinline__ void frag_store(const Frag<MT>& f, float* S, int g, int t) {
 #pragma unroll
@@ -262,6 +364,54 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
         f[0][1] = Op::pack(e1(sl[0][2]), e1(sl[0][3]));
         f[0][2] = f[0][3] = 0u;
     }
+}
+
+// Landmark means of the segments one warp owns (Algorithm 1 step 1) on the
+// tensor cores: xbar = P X with the averaging matrix P (P[j][t] = 1/L when
+// token t lies in segment j; exact in 16 bits since L is a power of two) as A
+// operand and the staged tokens X (rows = tokens, k) as B operand, whose
+// fragments are 8x8 transposes of the row-major stage.  The fp32 means are
+// rounded to the I/O type and stored as rows j0.. of xbar (row stride LS);
+// columns >= d come out as zeros.
+template <typename T, int TPW, int L>
+__device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
+    using Op = Mma16<T>;
+    constexpr int LPW = TPW / L;            // segments owned by the warp
+    constexpr int MTL = (LPW + 15) / 16;    // m-tiles of landmark rows
+    constexpr int LS = 40;
+    // 1/L in the I/O type, as the low / high half of a 32-bit register
+    const uint32_t inv = Op::pack(1.f / (float)L, 0.f) & 0xffffu;
+    float c[MTL][4][4];
+#pragma unroll
+    for (int ml = 0; ml < MTL; ++ml)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) c[ml][b][0] = c[ml][b][1] = c[ml][b][2] = c[ml][b][3] = 0.f;
+#pragma unroll
+    for (int ks = 0; ks < TPW / 16; ++ks) {  // 16 tokens per k-step
+        const int ml = (16 * ks / L) / 16;   // the one m-tile these tokens feed
+        // A = P rows 16 ml + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
+        auto pv = [&](int row, int tok) -> uint32_t { return (tok / L == row) ? inv : 0u; };
+        const int r0 = 16 * ml + g, r1 = r0 + 8, k0 = 16 * ks + 2 * t;
+        const uint32_t a[4] = {pv(r0, k0) | (pv(r0, k0 + 1) << 16), pv(r1, k0) | (pv(r1, k0 + 1) << 16),
+                               pv(r0, k0 + 8) | (pv(r0, k0 + 9) << 16), pv(r1, k0 + 8) | (pv(r1, k0 + 9) << 16)};
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int c0 = 8 * b + 2 * t;
+            const uint32_t x0 = c0 < d ? ld32(X + (16 * ks + g) * d + c0) : 0u;
+            const uint32_t x1 = c0 < d ? ld32(X + (16 * ks + 8 + g) * d + c0) : 0u;
+            Op::k16(c[ml][b], a, movmatrix_trans(x0), movmatrix_trans(x1));
+        }
+    }
+#pragma unroll
+    for (int ml = 0; ml < MTL; ++ml)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int row = 16 * ml + g, col = 8 * b + 2 * t;
+            if (row < LPW)
+                *reinterpret_cast<uint32_t*>(xbar + (j0 + row) * LS + col) = Op::pack(c[ml][b][0], c[ml][b][1]);
+            if (row + 8 < LPW)
+                *reinterpret_cast<uint32_t*>(xbar + (j0 + row + 8) * LS + col) = Op::pack(c[ml][b][2], c[ml][b][3]);
+        }
 }
 
 template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS>
@@ -335,25 +485,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
 
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
         {
-            const float invL = 1.f / (float)L;
-            const int dp = d >> 1;
-            for (int idx = lane; idx < LPW * 16; idx += 32) {
-                const int jl = idx >> 4, p = idx & 15;
-                float ax = 0.f, ay = 0.f, bx = 0.f, by = 0.f;
-                if (p < dp) {
-#pragma unroll 4
-                    for (int rr = 0; rr < L; ++rr) {
-                        const int off = (jl * L + rr) * d + 2 * p;
-                        const float2 a = Op::unpack(ld32(Qs + off));
-                        const float2 b = Op::unpack(ld32(Ks + off));
-                        ax += a.x; ay += a.y; bx += b.x; by += b.y;
-                    }
-                    ax *= invL; ay *= invL; bx *= invL; by *= invL;
-                }
-                const int j = r * LPW + jl;
-                *reinterpret_cast<uint32_t*>(qbar + j * LS + 2 * p) = Op::pack(ax, ay);
-                *reinterpret_cast<uint32_t*>(kbar + j * LS + 2 * p) = Op::pack(bx, by);
-            }
+            landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
+            landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
             if (M < MP && r == 0) {  // zero the padding landmark rows
                 for (int idx = lane; idx < (MP - M) * 16; idx += 32) {
                     const int j = M + (idx >> 4), p = idx & 15;
@@ -522,7 +655,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                 }
             }
             Frag<MT> Zc, Ac;
-            FragLo<MT> Aclo;
+            HFrag<MT> Ah;   // A = G_A^n as split fp16 A operand (constant over the iteration)
+            int zexp = 0;   // Zc holds 2^zexp Z (power-of-two scaling for fp16 range)
             {
 #pragma unroll
                 for (int mt = 0; mt < MT; ++mt) {
@@ -578,7 +712,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                         c += __shfl_xor_sync(0xffffffffu, c, 16);
                         cmax = fmaxf(cmax, c);
                     }
-                const float alpha = 1.f / (warp_max(rmax) * warp_max(cmax));
+                const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
                 frag_store<MT, SM>(Ac, mA, g, t);
                 __syncwarp();
                 // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
@@ -591,19 +725,27 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                             const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
                             Zc[i][n][e] = alpha * mA[c * SM + rr];
                         }
+                zexp = frag_normalise<MT>(Zc);
                 frag_store<MT, SM>(Zc, mZ, g, t);
-                frag_lo<MT>(Ac, Aclo);
+                to_hfrag<MT>(Ac, Ah);
                 __syncwarp();
             }
 
-            // pseudo-inverse iteration (step 4)
+            // pseudo-inverse iteration (step 4), fp16 two-term split products
 #pragma unroll 1
             for (int it = 0; it < iters; ++it) {
                 Frag<MT> X, Tm, P;
-                FragLo<MT> Xlo;
-                mm_tc<MT>(AFromFrag<MT>{Ac, Aclo}, BFromSmem<SM>{mZ, g, t}, X);  // X = A Z
+                HFrag<MT> Xh;
+                mm_h<MT>(Ah, BSmemH<SM>{mZ, g, t}, X);  // X = A Z = 2^-zexp A Zc
+                const float unscale = ldexpf(1.f, -zexp);
                 // exact symmetrisation (X + X^T)/2; Z's slot holds X for the transpose
                 __syncwarp();
+#pragma unroll
+                for (int i = 0; i < MT; ++i)
+#pragma unroll
+                    for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) X[i][n][e] *= unscale;
                 frag_store<MT, SM>(X, mZ, g, t);
                 __syncwarp();
 #pragma unroll
@@ -616,16 +758,16 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                             X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + rr]);
                             Tm[i][n][e] = X[i][n][e];
                         }
-                frag_lo<MT>(X, Xlo);
-                frag_shift<MT>(Tm, 7.f, g, t);                                // 7I - X
-                mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{Tm}, P);  // X (7I - X)
-                frag_shift<MT>(P, 15.f, g, t);                                // 15I - ...
-                mm_tc<MT>(AFromFrag<MT>{X, Xlo}, BFromSymFrag<MT>{P}, Tm);  // X (15I - ...)
-                frag_shift<MT>(Tm, 13.f, g, t);                               // 13I - ...
+                to_hfrag<MT>(X, Xh);
+                frag_shift<MT>(Tm, 7.f, g, t);              // 7I - X
+                mm_h<MT>(Xh, BSymH<MT>{Tm}, P);              // X (7I - X)
+                frag_shift<MT>(P, 15.f, g, t);               // 15I - ...
+                mm_h<MT>(Xh, BSymH<MT>{P}, Tm);              // X (15I - ...)
+                frag_shift<MT>(Tm, 13.f, g, t);              // 13I - ...
                 {
-                    FragLo<MT> Zlo;
-                    frag_lo<MT>(Zc, Zlo);
-                    mm_tc<MT>(AFromFrag<MT>{Zc, Zlo}, BFromSymFrag<MT>{Tm}, P);  // Z (13I - ...)
+                    HFrag<MT> Zh;
+                    to_hfrag<MT>(Zc, Zh);
+                    mm_h<MT>(Zh, BSymH<MT>{Tm}, P);          // Zc (13I - ...)
                 }
 #pragma unroll
                 for (int i = 0; i < MT; ++i)
@@ -633,6 +775,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                     for (int n = 0; n < 2 * MT; ++n)
 #pragma unroll
                         for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
+                zexp += frag_normalise<MT>(Zc);
                 __syncwarp();
                 frag_store<MT, SM>(Zc, mZ, g, t);
                 __syncwarp();
@@ -666,9 +809,10 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                         }
                     }
                 }
-                // fp16 has a narrow range: scale Y by a power of two.  Numerator and
-                // denominator columns share the factor, so it cancels in step 7.
-                float scale = 1.f;
+                // Y = 2^-zexp (Zc W).  fp16 output has a narrow range: scale Y by a
+                // power of two instead.  Numerator and denominator columns share the
+                // factor, so it cancels in step 7.
+                float scale = ldexpf(1.f, -zexp);
                 if (Op::kNarrowRange) {
                     float ymax = 0.f;
 #pragma unroll
@@ -677,8 +821,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                         for (int j = 0; j < NTO; ++j)
 #pragma unroll
                             for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
-                    ymax = warp_max(ymax);
-                    if (ymax > 0.f) scale = exp2f((float)(14 - ilogbf(ymax)));
+                    ymax = warp_max_nonneg(ymax);
+                    if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
                 }
 #pragma unroll
                 for (int i = 0; i < MT; ++i)

@@ -98,6 +98,11 @@ __device__ __forceinline__ float warp_max(float x) {
     for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
     return x;
 }
+// Max over the warp of non-negative floats: their bit patterns order like
+// unsigned integers, so one redux.sync does it.
+__device__ __forceinline__ float warp_max_nonneg(float x) {
+    return __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(x)));
+}
 __device__ __forceinline__ float quad_max(float x) {
     x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 1));
     return fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 2));
@@ -130,6 +135,19 @@ __device__ __forceinline__ void mma_tf32x3(float (&c)[4], const Tf32Pair (&a)[4]
     mma_tf32(c, a[0].lo, a[1].lo, a[2].lo, a[3].lo, b[0].hi, b[1].hi);
     mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].lo, b[1].lo);
     mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].hi, b[1].hi);
+}
+
+// fp16 two-term split of a pair of fp32 values: hi = rn(x), lo = rn(x - hi)
+// (x - hi is exact in fp32).  hi + lo carries 22 significant bits for values
+// in fp16's normal range; callers keep operands there by power-of-two scaling.
+struct H2Pair {
+    uint32_t hi, lo;
+};
+__device__ __forceinline__ H2Pair split_h2(float x0, float x1) {
+    __half2 h = __floats2half2_rn(x0, x1);
+    const float2 hf = __half22float2(h);
+    __half2 l = __floats2half2_rn(x0 - hf.x, x1 - hf.y);
+    return {*reinterpret_cast<uint32_t*>(&h), *reinterpret_cast<uint32_t*>(&l)};
 }
 
 // 16-bit MMAs (both operands of the same 16-bit type), fp32 accumulate.
