@@ -70,8 +70,10 @@ int exact_window_attention(const void* q, const void* k, const void* v, void* ou
     if (rc != NYSTRA_OK) return rc;
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
-    cudaError_t e = nystra_host::launch_exact_generic(q, k, v, out, units, N, d_h, dtype,
-                                                      (cudaStream_t)stream);
+    cudaError_t e = nystra_host::exact_tc_supports(N, d_h, dtype)
+                        ? nystra_host::launch_exact_tc(q, k, v, out, units, N, d_h, dtype, (cudaStream_t)stream)
+                        : nystra_host::launch_exact_generic(q, k, v, out, units, N, d_h, dtype,
+                                                            (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
@@ -105,8 +107,8 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[3])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
-                                                   take_fault_word_tc_n1024};
+    unsigned int (*const take[4])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
+                                                   take_fault_word_tc_n1024, take_fault_word_exact_tc};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

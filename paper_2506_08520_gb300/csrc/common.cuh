@@ -45,6 +45,11 @@ cudaError_t launch_nystra_tc_n1024(const void* q, const void* k, const void* v, 
 unsigned int take_fault_word_tc_n64(cudaError_t* err);
 unsigned int take_fault_word_tc_n256(cudaError_t* err);
 unsigned int take_fault_word_tc_n1024(cudaError_t* err);
+// Tensor-core exact attention, 16-bit I/O, N in {64, 256, 1024}, even d_h <= 32 (exact_tc.cu).
+bool exact_tc_supports(int N, int d, int dtype);
+cudaError_t launch_exact_tc(const void* q, const void* k, const void* v, void* out, long long n_units, int N,
+                            int d, int dtype, cudaStream_t stream);
+unsigned int take_fault_word_exact_tc(cudaError_t* err);
 // Device-side fault words (bit 0: a bounded wait gave up) of the translation
 // units whose kernels wait on barriers: OR-ed together, then cleared.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);
