@@ -9,7 +9,7 @@
 //
 // Per unit:
 //   stage    each warp bulk-copies its TPW rows of Q, K and V (contiguous in
-//            HBM) into its private stage with one mbarrier; bounded wait.
+//            HBM) into its private stage; bounded waits.
 //   front    landmarks (Algorithm 1 step 1) of the segments a warp owns
 //            (segments never straddle warps: N/m <= TPW), to group memory;
 //            [P1] S_L = Q Kbar^T, G_L^n = exp(S_L - m_L) parked as MMA
@@ -19,14 +19,18 @@
 //   combine  (WPU > 1) partial (W_r, m_r) of all warps are merged in a fixed
 //            order: m_U = max_r m_r, W = sum_r exp(m_r - m_U) W_r, which is
 //            exactly G_U^n [V | 1] with the max over all N keys.
-//            [P1] the stage is dead now: the next unit's copies are issued.
 //   core     warp 0: G_A^n = exp(Qbar Kbar^T - m_U), Z_0 = A^T/(||A||_1
 //            ||A||_inf), `iters` steps Z <- Z(13I - X(15I - X(7I - X)))/4 with
 //            X = A Z (step 4), Y = Z W, stored as a 16-bit B operand.
 //   output   every warp: O = (G_L^n Y_:d) / (G_L^n Y_d) for its tokens
-//            (steps 5-7), written from registers.  [P2] S_L and G_L^n are
-//            computed here from the still-resident Q, and the next unit's
-//            copies are issued afterwards.
+//            (steps 5-7), staged row-major in its V region and written with
+//            one bulk store (whole sectors; scattered 4-byte stores of 60-byte
+//            rows touched ~11 sectors per 128 bytes).  [P2] S_L and G_L^n are
+//            computed here from the still-resident Q.
+//   copies   Q and K of the next unit are issued after the combine ([P2]: K
+//            only; Q after the output), V once the output store has read its
+//            staging, on two mbarriers, so V may land while the next unit's
+//            landmarks and S_L run.
 // P1 ("G_L parked") is used when the fragments fit in shared memory next to
 // the stage; otherwise P2.
 //
@@ -77,15 +81,25 @@ struct Layout {
     static constexpr size_t WPART = (size_t)TPW * DS * 2;
     static_assert((size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
     // per-group shared memory
+    // With one warp per unit and G_L^n parked, Y^T is written only after the
+    // core has read Qbar/Kbar for the last time and is dead before the next
+    // unit's landmarks, so it overlays them.  (With several warps a fast warp
+    // could write the next landmarks while another still reads Y^T; without
+    // parking, the output phase still reads Kbar.)  G_A^n is stored only to
+    // read Z_0 = a A^T transposed, so it uses Z's slot.
+    static constexpr bool YT_OVERLAY = (WPU == 1) && GLS;
+    static constexpr size_t QK_BYTES = 2 * MP * LS * 2;
+    static constexpr size_t YT_BYTES = ((NCOL * YS * 2 + 15) / 16) * 16;
     static constexpr size_t G_QBAR = 0;
     static constexpr size_t G_KBAR = G_QBAR + MP * LS * 2;
-    static constexpr size_t G_MU = G_KBAR + MP * LS * 2;  // m_U, log2 domain
+    static constexpr size_t G_YT = YT_OVERLAY ? G_QBAR : QK_BYTES;
+    static constexpr size_t G_MU = YT_OVERLAY ? (QK_BYTES > YT_BYTES ? QK_BYTES : YT_BYTES)
+                                              : QK_BYTES + YT_BYTES;  // m_U, log2 domain
     static constexpr size_t G_W = G_MU + MP * 4;
-    static constexpr size_t G_A = G_W + MP * WS * 4;
-    static constexpr size_t G_Z = G_A + MP * SM * 4;
-    static constexpr size_t G_YT = G_Z + MP * SM * 4;
-    static constexpr size_t G_BAR = G_YT + ((NCOL * YS * 2 + 15) / 16) * 16;
-    static constexpr size_t G_FLAG = G_BAR + 8 * WPU;
+    static constexpr size_t G_Z = G_W + MP * WS * 4;
+    static constexpr size_t G_A = G_Z;
+    static constexpr size_t G_BAR = G_Z + MP * SM * 4;
+    static constexpr size_t G_FLAG = G_BAR + 16 * WPU;  // two mbarriers per warp
     static constexpr size_t GROUP_BYTES = ((G_FLAG + 16 + 127) / 128) * 128;
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
 };
@@ -418,7 +432,7 @@ template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS>
 __global__ void __launch_bounds__(GROUPS * WPU * 32, 1)
 nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                  T* __restrict__ out, long long n_units, int d, int iters, float sl2,
-                 unsigned int* fault) {
+                 unsigned int* fault, int active) {
     using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
     using Op = Mma16<T>;
     constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS, SM = Lay::SM,
@@ -446,7 +460,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
     float* mA = reinterpret_cast<float*>(gb + Lay::G_A);
     float* mZ = reinterpret_cast<float*>(gb + Lay::G_Z);
     T* yT = reinterpret_cast<T*>(gb + Lay::G_YT);
-    uint64_t* bar = reinterpret_cast<uint64_t*>(gb + Lay::G_BAR) + r;
+    uint64_t* barQK = reinterpret_cast<uint64_t*>(gb + Lay::G_BAR) + 2 * r;  // Q and K rows
+    uint64_t* barV = barQK + 1;                                                // V rows
     volatile unsigned int* gflag = reinterpret_cast<volatile unsigned int*>(gb + Lay::G_FLAG);
 
     auto gsync = [&]() {
@@ -454,34 +469,43 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         else named_barrier(1 + grp, WPU * 32);
     };
 
-    const long long stride = (long long)gridDim.x * GROUPS;
-    long long u = (long long)blockIdx.x * GROUPS + grp;
+    // Only the first `active` groups of a CTA take units (see launch_cfg).
+    const long long stride = (long long)gridDim.x * active;
+    long long u = grp < active ? (long long)blockIdx.x * active + grp : n_units;
     const uint32_t tile_bytes = (uint32_t)(td * sizeof(T));
-    auto issue = [&](long long unit) {
-        const size_t off = (size_t)unit * N * d + (size_t)r * td;
-        mbar_arrive_expect_tx(bar, 3u * tile_bytes);
-        bulk_g2s(Qs, q + off, tile_bytes, bar);
-        bulk_g2s(Ks, k + off, tile_bytes, bar);
-        bulk_g2s(Vs, v + off, tile_bytes, bar);
+    // This warp's rows of a unit are contiguous in HBM: one bulk copy per tensor.
+    auto unit_off = [&](long long unit) { return (size_t)unit * N * d + (size_t)r * td; };
+    auto arm_qk = [&]() { mbar_arrive_expect_tx(barQK, 2u * tile_bytes); };
+    auto issue_q = [&](long long unit) { bulk_g2s(Qs, q + unit_off(unit), tile_bytes, barQK); };
+    auto issue_k = [&](long long unit) { bulk_g2s(Ks, k + unit_off(unit), tile_bytes, barQK); };
+    auto issue_v = [&](long long unit) {
+        mbar_arrive_expect_tx(barV, tile_bytes);
+        bulk_g2s(Vs, v + unit_off(unit), tile_bytes, barV);
     };
 
     if (lane == 0) {
-        mbar_init(bar, 1);
+        mbar_init(barQK, 1);
+        mbar_init(barV, 1);
         fence_mbar_init();
         if (r == 0) *gflag = 0u;
     }
     gsync();
-    if (u < n_units && lane == 0) issue(u);
-    uint32_t phase = 0;
+    if (u < n_units && lane == 0) {
+        arm_qk();
+        issue_q(u);
+        issue_k(u);
+        issue_v(u);
+    }
+    uint32_t phase_qk = 0, phase_v = 0;
 
     for (; u < n_units; u += stride) {
-        // ---------------- stage: bounded wait ----------------
-        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
+        // ---------------- stage: bounded wait for Q and K ----------------
+        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
         if (!ok && lane == 0) {
             atomicOr(fault, 1u);
             *gflag = 1u;  // the whole group stops after the next barrier
         }
-        phase ^= 1u;
+        phase_qk ^= 1u;
 
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
         {
@@ -516,6 +540,15 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                     }
                 }
         }
+
+        // ---------------- stage: bounded wait for V ----------------
+        const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
+        if (!ok_v && lane == 0) {
+            atomicOr(fault, 1u);
+            *gflag = 1u;
+        }
+        phase_v ^= 1u;
+        if (WPU == 1 && !ok_v) break;
 
         // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
         float mU[MT][2];       // this warp's row maxima of S_U, log2 domain
@@ -635,14 +668,17 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             }
         }
         gsync();
+        if (WPU > 1 && *gflag != 0u) break;
 
-        // [P1] Q, K, V of this unit are consumed: prefetch the next unit.
-        if constexpr (GLS) {
-            const long long un = u + stride;
-            if (un < n_units && lane == 0) {
-                fence_proxy_async_smem();
-                issue(un);
-            }
+        // Q and K of this unit are consumed (in P2 Q stays for the output):
+        // prefetch the next unit's rows.  V's region holds the output first.
+        const long long un = u + stride;
+        fence_proxy_async_smem();  // this lane's reads of Q/K precede the async refill
+        __syncwarp();
+        if (un < n_units && lane == 0) {
+            arm_qk();
+            if constexpr (GLS) issue_q(un);
+            issue_k(un);
         }
 
         // ---------------- core (warp 0): G_A^n, Z_0, iteration, Y ----------------
@@ -713,7 +749,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                         cmax = fmaxf(cmax, c);
                     }
                 const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
-                frag_store<MT, SM>(Ac, mA, g, t);
+                frag_store<MT, SM>(Ac, mA, g, t);  // mA is Z's slot
                 __syncwarp();
                 // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
 #pragma unroll
@@ -726,6 +762,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                             Zc[i][n][e] = alpha * mA[c * SM + rr];
                         }
                 zexp = frag_normalise<MT>(Zc);
+                __syncwarp();  // every lane has read A^T before Z overwrites the slot
                 frag_store<MT, SM>(Zc, mZ, g, t);
                 to_hfrag<MT>(Ac, Ah);
                 __syncwarp();
@@ -851,7 +888,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                 }
             const int jd = d >> 3, tdn = (d & 7) >> 1;
             const int src = (lane & ~3) | tdn;
-            T* obase = out + (size_t)u * N * d + (size_t)r * td;
+            T* obase = Vs;  // staged here, then one bulk store of the warp's rows
 #pragma unroll 1
             for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
@@ -906,18 +943,28 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                 }
         }
 
+        // The output rows are staged in V's region: one bulk store, and once it
+        // has read shared memory, the next unit's V can land there.
+        fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
+        __syncwarp();
+        if (lane == 0) {
+            bulk_s2g(out + unit_off(u), Vs, tile_bytes);
+            bulk_commit();
+            bulk_wait_read_all();
+        }
         // [P2] Q was needed until now: every warp of the group is done reading
-        // the landmarks before anyone overwrites them, then prefetch.
+        // the landmarks before anyone overwrites them.
         if constexpr (!GLS) {
+            fence_proxy_async_smem();  // reads of Q precede its refill
             gsync();
-            const long long un = u + stride;
-            if (un < n_units && lane == 0) {
-                fence_proxy_async_smem();
-                issue(un);
-            }
+        }
+        if (un < n_units && lane == 0) {
+            if constexpr (!GLS) issue_q(un);
+            issue_v(un);
         }
         __syncwarp();
     }
+    if (lane == 0) bulk_wait_all();  // outstanding output stores complete before exit
 }
 
 // Largest number of groups per CTA that fits the shared-memory and register
@@ -953,11 +1000,18 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
         s_blocks = sms * per_sm;
     }
-    const long long want = (n_units + kGroups - 1) / kGroups;
-    const long long grid = want < s_blocks ? want : s_blocks;
+    // Wave quantisation: every group processes ceil(units / groups) units, so
+    // use the fewest groups per CTA that still reach the minimal number of
+    // rounds (fewer co-resident groups contend less for the SM).
+    const long long blocks = s_blocks;
+    const long long rounds = (n_units + blocks * kGroups - 1) / (blocks * kGroups);
+    int active = (int)((n_units + blocks * rounds - 1) / (blocks * rounds));
+    active = active < 1 ? 1 : (active > kGroups ? kGroups : active);
+    const long long want = (n_units + active - 1) / active;
+    const long long grid = want < blocks ? want : blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, kGroups * WPU * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
-                                                              n_units, d, iters, sl2, fault);
+                                                              n_units, d, iters, sl2, fault, active);
     return cudaGetLastError();
 }
 
