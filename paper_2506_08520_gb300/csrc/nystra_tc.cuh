@@ -428,6 +428,394 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
         }
 }
 
+// Front, U side, for one warp's NCH chunks of 64 tokens: S_U = Qbar K^T with a
+// running row max, G_U^n = exp(S_U - m_U) fed straight from registers as the
+// A operand of W_r = G_U^n [V | 1] (B fragments of [V | 1 | 0] by 8x8
+// transposes; the ones column yields the denominator), rescaled online when
+// the max grows.  W_r (MP x NCOL) is stored at dst with row stride ws after a
+// warp sync (so every lane is done reading K and V); the row maxima (log2
+// domain) are returned in mU.
+template <typename T, int M, int NCOL, int NCH>
+__device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
+                                           float* dst, int ws, float (&mU)[(M + 15) / 16][2]) {
+    using Op = Mma16<T>;
+    constexpr int MT = (M + 15) / 16, LS = 40, NTO = NCOL / 8;
+    float wall[MT][NTO][4];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) {
+        uint32_t aq[2][4];
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+            aq[kk][0] = ld32(r0);
+            aq[kk][1] = ld32(r0 + 8 * LS);
+            aq[kk][2] = ld32(r0 + 8);
+            aq[kk][3] = ld32(r0 + 8 * LS + 8);
+        }
+        const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
+        float(&w)[NTO][4] = wall[mt];
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
+        float run0 = -INFINITY, run1 = -INFINITY;
+#pragma unroll 1
+        for (int ch = 0; ch < NCH; ++ch) {
+            const T* Kc = Ks + ch * 64 * d;
+            const T* Vc = Vs + ch * 64 * d;
+            float s[8][4];
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+                const T* kr = Kc + (8 * nt + g) * d;
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) {
+                    const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
+                    const uint32_t b0 = c0 < d ? ld32(kr + c0) : 0u;
+                    const uint32_t b1 = c1 < d ? ld32(kr + c1) : 0u;
+                    Op::k16(s[nt], aq[kk], b0, b1);
+                }
+            }
+            float mx0 = run0, mx1 = run1;
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt) {
+                mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
+                mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
+            }
+            mx0 = quad_max(mx0);
+            mx1 = quad_max(mx1);
+            if (NCH > 1) {  // online rescaling of the accumulated W rows
+                const float f0 = ex2(run0 - mx0), f1 = ex2(run1 - mx1);
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) {
+                    w[j][0] *= f0; w[j][1] *= f0; w[j][2] *= f1; w[j][3] *= f1;
+                }
+            }
+            run0 = mx0;
+            run1 = mx1;
+            auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+            auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+            // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
+#pragma unroll
+            for (int kt = 0; kt < 4; ++kt) {
+                uint32_t a[4];
+                a[0] = v0 ? Op::pack(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : 0u;
+                a[1] = v1 ? Op::pack(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : 0u;
+                a[2] = v0 ? Op::pack(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : 0u;
+                a[3] = v1 ? Op::pack(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : 0u;
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) {
+                    const int c0 = 8 * j + 2 * t;
+                    const uint32_t x0 = c0 < d ? ld32(Vc + (16 * kt + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
+                    const uint32_t x1 = c0 < d ? ld32(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
+                    Op::k16(w[j], a, movmatrix_trans(x0), movmatrix_trans(x1));
+                }
+            }
+        }
+        mU[mt][0] = run0;
+        mU[mt][1] = run1;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) {
+            const int rr = 16 * mt + g, c = 8 * j + 2 * t;
+            *reinterpret_cast<float2*>(dst + rr * ws + c) = make_float2(wall[mt][j][0], wall[mt][j][1]);
+            *reinterpret_cast<float2*>(dst + (rr + 8) * ws + c) = make_float2(wall[mt][j][2], wall[mt][j][3]);
+        }
+}
+
+// Combine (several warps per unit): the warps' partial (W_r, m_r), stored in
+// their stages at part0 + s * wstride (floats), merge in a fixed order into
+// m_U = max_r m_r and W = sum_r 2^(m_r - m_U) W_r, exactly G_U^n [V | 1] with
+// the max over all N keys.  Warp r of WPU handles every (WPU*32)-th element.
+template <int MP, int NCOL, int WS, int WPU>
+__device__ __forceinline__ void combine_partials(const float* part0, size_t wstride, float* mW, float* gmu, int r,
+                                                 int lane) {
+    for (int e = r * 32 + lane; e < MP * NCOL; e += WPU * 32) {
+        const int i = e / NCOL, c = e - (e / NCOL) * NCOL;
+        float mu = -INFINITY;
+#pragma unroll
+        for (int s2 = 0; s2 < WPU; ++s2) mu = fmaxf(mu, part0[(size_t)s2 * wstride + MP * NCOL + i]);
+        float acc = 0.f;
+#pragma unroll
+        for (int s2 = 0; s2 < WPU; ++s2) {
+            const float* ps = part0 + (size_t)s2 * wstride;
+            acc = fmaf(ex2(ps[MP * NCOL + i] - mu), ps[i * NCOL + c], acc);
+        }
+        mW[i * WS + c] = acc;
+        if (c == 0) gmu[i] = mu;
+    }
+}
+
+// Core, one warp: G_A^n = exp(Qbar Kbar^T - m_U) (mU: row maxima of this
+// lane's C-layout rows, log2 domain), Z_0 = A^T/(||A||_1 ||A||_inf), `iters`
+// steps Z <- Z (13I - X(15I - X(7I - X)))/4 with X = A Z (Algorithm 1 step 4)
+// on fp16 two-term-split MMAs in registers, and Y = Z W (split-tf32, W from
+// mW), stored as Y^T (16-bit B operand) at yT.  mZ is scratch for Z and X.
+template <typename T, int M, int NCOL>
+__device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const float (&mU)[(M + 15) / 16][2],
+                                          const float* mW, float* mZ, T* yT, int iters, float sl2, int g, int t) {
+    using Op = Mma16<T>;
+    constexpr int MT = (M + 15) / 16, MP = MT * 16, LS = 40, SM = MP + 4, WS = NCOL + 4, NTO = NCOL / 8;
+    constexpr int YS = (M < 16 ? 16 : M) + 8;
+    float* mA = mZ;  // G_A^n is stored only to read Z_0 = a A^T transposed
+    Frag<MT> Zc, Ac;
+    HFrag<MT> Ah;   // A = G_A^n as split fp16 A operand (constant over the iteration)
+    int zexp = 0;   // Zc holds 2^zexp Z (power-of-two scaling for fp16 range)
+    {
+#pragma unroll
+        for (int mt = 0; mt < MT; ++mt) {
+            uint32_t aq[2][4];
+#pragma unroll
+            for (int kk = 0; kk < 2; ++kk) {
+                const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+                aq[kk][0] = ld32(r0);
+                aq[kk][1] = ld32(r0 + 8 * LS);
+                aq[kk][2] = ld32(r0 + 8);
+                aq[kk][3] = ld32(r0 + 8 * LS + 8);
+            }
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n) {
+                float sa[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int kk = 0; kk < 2; ++kk) {
+                    const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
+                    Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                }
+                const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
+                Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
+                Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
+                Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
+                Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+            }
+        }
+        // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
+        float rmax = 0.f, cmax = 0.f;
+#pragma unroll
+        for (int i = 0; i < MT; ++i) {
+            float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n) {
+                r0 += Ac[i][n][0] + Ac[i][n][1];
+                r1 += Ac[i][n][2] + Ac[i][n][3];
+            }
+            r0 += __shfl_xor_sync(0xffffffffu, r0, 1);
+            r0 += __shfl_xor_sync(0xffffffffu, r0, 2);
+            r1 += __shfl_xor_sync(0xffffffffu, r1, 1);
+            r1 += __shfl_xor_sync(0xffffffffu, r1, 2);
+            rmax = fmaxf(rmax, fmaxf(r0, r1));
+        }
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                float c = 0.f;
+#pragma unroll
+                for (int i = 0; i < MT; ++i) c += Ac[i][n][e] + Ac[i][n][e + 2];
+                c += __shfl_xor_sync(0xffffffffu, c, 4);
+                c += __shfl_xor_sync(0xffffffffu, c, 8);
+                c += __shfl_xor_sync(0xffffffffu, c, 16);
+                cmax = fmaxf(cmax, c);
+            }
+        const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
+        frag_store<MT, SM>(Ac, mA, g, t);  // mA is Z's slot
+        __syncwarp();
+        // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                    Zc[i][n][e] = alpha * mA[c * SM + rr];
+                }
+        zexp = frag_normalise<MT>(Zc);
+        __syncwarp();  // every lane has read A^T before Z overwrites the slot
+        frag_store<MT, SM>(Zc, mZ, g, t);
+        to_hfrag<MT>(Ac, Ah);
+        __syncwarp();
+    }
+
+    // pseudo-inverse iteration (step 4), fp16 two-term split products
+#pragma unroll 1
+    for (int it = 0; it < iters; ++it) {
+        Frag<MT> X, Tm, P;
+        HFrag<MT> Xh;
+        mm_h<MT>(Ah, BSmemH<SM>{mZ, g, t}, X);  // X = A Z = 2^-zexp A Zc
+        const float unscale = ldexpf(1.f, -zexp);
+        // exact symmetrisation (X + X^T)/2; Z's slot holds X for the transpose
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) X[i][n][e] *= unscale;
+        frag_store<MT, SM>(X, mZ, g, t);
+        __syncwarp();
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                    X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + rr]);
+                    Tm[i][n][e] = X[i][n][e];
+                }
+        to_hfrag<MT>(X, Xh);
+        frag_shift<MT>(Tm, 7.f, g, t);              // 7I - X
+        mm_h<MT>(Xh, BSymH<MT>{Tm}, P);              // X (7I - X)
+        frag_shift<MT>(P, 15.f, g, t);               // 15I - ...
+        mm_h<MT>(Xh, BSymH<MT>{P}, Tm);              // X (15I - ...)
+        frag_shift<MT>(Tm, 13.f, g, t);              // 13I - ...
+        {
+            HFrag<MT> Zh;
+            to_hfrag<MT>(Zc, Zh);
+            mm_h<MT>(Zh, BSymH<MT>{Tm}, P);          // Zc (13I - ...)
+        }
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
+        zexp += frag_normalise<MT>(Zc);
+        __syncwarp();
+        frag_store<MT, SM>(Zc, mZ, g, t);
+        __syncwarp();
+    }
+
+    // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
+    {
+        float y[MT][NTO][4];
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
+        FragLo<MT> Zlo;
+        frag_lo<MT>(Zc, Zlo);
+#pragma unroll
+        for (int kk = 0; kk < 2 * MT; ++kk) {
+            uint32_t ah[MT][4], al[MT][4];
+#pragma unroll
+            for (int i = 0; i < MT; ++i) AFromFrag<MT>{Zc, Zlo}(i, kk, ah[i], al[i]);
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) {
+                const float y0 = mW[(8 * kk + 2 * t) * WS + 8 * j + g];
+                const float y1 = mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g];
+                const uint32_t bh0 = __float_as_uint(y0), bh1 = __float_as_uint(y1);
+                const uint32_t bl0 = tf32_lo(y0), bl1 = tf32_lo(y1);
+#pragma unroll
+                for (int i = 0; i < MT; ++i) {
+                    mma_tf32(y[i][j], al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
+                    mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
+                    mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
+                }
+            }
+        }
+        // Y = 2^-zexp (Zc W).  fp16 output has a narrow range: scale Y by a
+        // power of two instead.  Numerator and denominator columns share the
+        // factor, so it cancels in step 7.
+        float scale = ldexpf(1.f, -zexp);
+        if (Op::kNarrowRange) {
+            float ymax = 0.f;
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int j = 0; j < NTO; ++j)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
+            ymax = warp_max_nonneg(ymax);
+            if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
+        }
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) {
+                const int rr = 16 * i + g, c = 8 * j + 2 * t;
+                yT[c * YS + rr] = from_f32<T>(y[i][j][0] * scale);
+                yT[(c + 1) * YS + rr] = from_f32<T>(y[i][j][1] * scale);
+                yT[c * YS + rr + 8] = from_f32<T>(y[i][j][2] * scale);
+                yT[(c + 1) * YS + rr + 8] = from_f32<T>(y[i][j][3] * scale);
+            }
+    }
+        }
+
+// Output for one warp's NCH chunks: O = (G_L^n Y_:d) / (G_L^n Y_d) (steps
+// 5-7); G_L^n fragments come from glf (parked) or are recomputed from Qs and
+// Kbar; rows are written row-major to obase (N_w x d).
+template <typename T, int M, int NCOL, int NCH, bool GLS>
+__device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, const T* kbar, const T* yT,
+                                            T* obase, int d, int g, int t, int lane, float sl2) {
+    using Op = Mma16<T>;
+    constexpr int KTL = (M >= 16) ? M / 16 : 1, NTO = NCOL / 8, YS = (M < 16 ? 16 : M) + 8;
+    uint32_t by[KTL][NTO][2];
+#pragma unroll
+    for (int kk = 0; kk < KTL; ++kk)
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) {
+            const T* yr = yT + (8 * j + g) * YS + 16 * kk + 2 * t;
+            by[kk][j][0] = ld32(yr);
+            by[kk][j][1] = (M >= 16) ? ld32(yr + 8) : 0u;
+        }
+    const int jd = d >> 3, tdn = (d & 7) >> 1;
+    const int src = (lane & ~3) | tdn;
+#pragma unroll 1
+    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+        for (int tm = 0; tm < 4; ++tm) {
+            uint32_t f[KTL][4];
+            if constexpr (GLS) {
+#pragma unroll
+                for (int kk = 0; kk < KTL; ++kk) {
+                    const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
+                    if constexpr (M >= 16) {
+                        const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+                        f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = x.z; f[kk][3] = x.w;
+                    } else {
+                        const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
+                        f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = f[kk][3] = 0u;
+                    }
+                }
+            } else {
+                gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
+            }
+            float o[NTO][4];
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+            if constexpr (M >= 16) {
+#pragma unroll
+                for (int kk = 0; kk < KTL; ++kk)
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) Op::k16(o[j], f[kk], by[kk][j][0], by[kk][j][1]);
+            } else {
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) Op::k8(o[j], f[0][0], f[0][1], by[0][j][0]);
+            }
+            float d0 = 0.f, d1 = 0.f;
+#pragma unroll
+            for (int j = 0; j < NTO; ++j)
+                if (j == jd) {
+                    d0 = o[j][0];
+                    d1 = o[j][2];
+                }
+            const float i0 = __fdividef(1.f, __shfl_sync(0xffffffffu, d0, src));
+            const float i1 = __fdividef(1.f, __shfl_sync(0xffffffffu, d1, src));
+            T* o0 = obase + (ch * 64 + 16 * tm + g) * d;
+            T* o1 = o0 + 8 * d;
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) {
+                const int c = 8 * j + 2 * t;
+                if (c < d) {
+                    *reinterpret_cast<uint32_t*>(o0 + c) = Op::pack(o[j][0] * i0, o[j][1] * i0);
+                    *reinterpret_cast<uint32_t*>(o1 + c) = Op::pack(o[j][2] * i1, o[j][3] * i1);
+                }
+            }
+        }
+        }
+
 template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS>
 __global__ void __launch_bounds__(GROUPS * WPU * 32, 1)
 nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
@@ -551,121 +939,23 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         if (WPU == 1 && !ok_v) break;
 
         // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
-        float mU[MT][2];       // this warp's row maxima of S_U, log2 domain
-        float wall[MT][NTO][4];  // W_r rows of every m-tile (stored after the loop:
-                                 // with several warps the partial goes to the K/V stage)
-#pragma unroll
-        for (int mt = 0; mt < MT; ++mt) {
-            uint32_t aq[2][4];
-#pragma unroll
-            for (int kk = 0; kk < 2; ++kk) {
-                const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-                aq[kk][0] = ld32(r0);
-                aq[kk][1] = ld32(r0 + 8 * LS);
-                aq[kk][2] = ld32(r0 + 8);
-                aq[kk][3] = ld32(r0 + 8 * LS + 8);
-            }
-            const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
-            float(&w)[NTO][4] = wall[mt];
-#pragma unroll
-            for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
-            float run0 = -INFINITY, run1 = -INFINITY;
-#pragma unroll 1
-            for (int ch = 0; ch < NCH; ++ch) {
-                const T* Kc = Ks + ch * 64 * d;
-                const T* Vc = Vs + ch * 64 * d;
-                float s[8][4];
-#pragma unroll
-                for (int nt = 0; nt < 8; ++nt) {
-                    s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-                    const T* kr = Kc + (8 * nt + g) * d;
-#pragma unroll
-                    for (int kk = 0; kk < 2; ++kk) {
-                        const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-                        const uint32_t b0 = c0 < d ? ld32(kr + c0) : 0u;
-                        const uint32_t b1 = c1 < d ? ld32(kr + c1) : 0u;
-                        Op::k16(s[nt], aq[kk], b0, b1);
-                    }
-                }
-                float mx0 = run0, mx1 = run1;
-#pragma unroll
-                for (int nt = 0; nt < 8; ++nt) {
-                    mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
-                    mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
-                }
-                mx0 = quad_max(mx0);
-                mx1 = quad_max(mx1);
-                if (NCH > 1) {  // online rescaling of the accumulated W rows
-                    const float f0 = ex2(run0 - mx0), f1 = ex2(run1 - mx1);
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) {
-                        w[j][0] *= f0; w[j][1] *= f0; w[j][2] *= f1; w[j][3] *= f1;
-                    }
-                }
-                run0 = mx0;
-                run1 = mx1;
-                auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
-                auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
-                // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
-#pragma unroll
-                for (int kt = 0; kt < 4; ++kt) {
-                    uint32_t a[4];
-                    a[0] = v0 ? Op::pack(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : 0u;
-                    a[1] = v1 ? Op::pack(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : 0u;
-                    a[2] = v0 ? Op::pack(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : 0u;
-                    a[3] = v1 ? Op::pack(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : 0u;
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) {
-                        const int c0 = 8 * j + 2 * t;
-                        const uint32_t x0 = c0 < d ? ld32(Vc + (16 * kt + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                        const uint32_t x1 = c0 < d ? ld32(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                        Op::k16(w[j], a, movmatrix_trans(x0), movmatrix_trans(x1));
-                    }
-                }
-            }
-            mU[mt][0] = run0;
-            mU[mt][1] = run1;
-        }
-        {
-            float* dst = (WPU == 1) ? mW : wpart;
-            const int ws = (WPU == 1) ? WS : NCOL;
-            if (WPU > 1) __syncwarp();  // every lane is done reading K and V
+        float mU[MT][2];  // this warp's row maxima of S_U, log2 domain
+        front_su_w<T, M, NCOL, NCH>(qbar, Ks, Vs, d, g, t, sl2, WPU == 1 ? mW : wpart, WPU == 1 ? WS : NCOL, mU);
+        if (WPU > 1 && t == 0) {
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
-#pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    const int rr = 16 * mt + g, c = 8 * j + 2 * t;
-                    *reinterpret_cast<float2*>(dst + rr * ws + c) = make_float2(wall[mt][j][0], wall[mt][j][1]);
-                    *reinterpret_cast<float2*>(dst + (rr + 8) * ws + c) =
-                        make_float2(wall[mt][j][2], wall[mt][j][3]);
-                }
-                if (WPU > 1 && t == 0) {
-                    wpart[MP * NCOL + 16 * mt + g] = mU[mt][0];
-                    wpart[MP * NCOL + 16 * mt + g + 8] = mU[mt][1];
-                }
+                wpart[MP * NCOL + 16 * mt + g] = mU[mt][0];
+                wpart[MP * NCOL + 16 * mt + g + 8] = mU[mt][1];
             }
         }
 
         // ---------------- combine (WPU > 1) ----------------
         if constexpr (WPU > 1) {
             gsync();
-            const float* part0 = reinterpret_cast<const float*>(smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
-                                                                (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART);
-            for (int e = r * 32 + lane; e < MP * NCOL; e += WPU * 32) {
-                const int i = e / NCOL, c = e - (e / NCOL) * NCOL;
-                float mu = -INFINITY;
-#pragma unroll
-                for (int s2 = 0; s2 < WPU; ++s2)
-                    mu = fmaxf(mu, part0[(size_t)s2 * (Lay::WARP_BYTES / 4) + MP * NCOL + i]);
-                float acc = 0.f;
-#pragma unroll
-                for (int s2 = 0; s2 < WPU; ++s2) {
-                    const float* ps = part0 + (size_t)s2 * (Lay::WARP_BYTES / 4);
-                    acc = fmaf(ex2(ps[MP * NCOL + i] - mu), ps[i * NCOL + c], acc);
-                }
-                mW[i * WS + c] = acc;
-                if (c == 0) gmu[i] = mu;
-            }
+            combine_partials<MP, NCOL, WS, WPU>(
+                reinterpret_cast<const float*>(smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
+                                               (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART),
+                Lay::WARP_BYTES / 4, mW, gmu, r, lane);
         }
         gsync();
         if (WPU > 1 && *gflag != 0u) break;
@@ -690,258 +980,12 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                     mU[mt][1] = gmu[16 * mt + g + 8];
                 }
             }
-            Frag<MT> Zc, Ac;
-            HFrag<MT> Ah;   // A = G_A^n as split fp16 A operand (constant over the iteration)
-            int zexp = 0;   // Zc holds 2^zexp Z (power-of-two scaling for fp16 range)
-            {
-#pragma unroll
-                for (int mt = 0; mt < MT; ++mt) {
-                    uint32_t aq[2][4];
-#pragma unroll
-                    for (int kk = 0; kk < 2; ++kk) {
-                        const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-                        aq[kk][0] = ld32(r0);
-                        aq[kk][1] = ld32(r0 + 8 * LS);
-                        aq[kk][2] = ld32(r0 + 8);
-                        aq[kk][3] = ld32(r0 + 8 * LS + 8);
-                    }
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n) {
-                        float sa[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                        for (int kk = 0; kk < 2; ++kk) {
-                            const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
-                            Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
-                        }
-                        const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
-                        Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
-                        Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
-                        Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
-                        Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
-                    }
-                }
-                // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
-                float rmax = 0.f, cmax = 0.f;
-#pragma unroll
-                for (int i = 0; i < MT; ++i) {
-                    float r0 = 0.f, r1 = 0.f;
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n) {
-                        r0 += Ac[i][n][0] + Ac[i][n][1];
-                        r1 += Ac[i][n][2] + Ac[i][n][3];
-                    }
-                    r0 += __shfl_xor_sync(0xffffffffu, r0, 1);
-                    r0 += __shfl_xor_sync(0xffffffffu, r0, 2);
-                    r1 += __shfl_xor_sync(0xffffffffu, r1, 1);
-                    r1 += __shfl_xor_sync(0xffffffffu, r1, 2);
-                    rmax = fmaxf(rmax, fmaxf(r0, r1));
-                }
-#pragma unroll
-                for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        float c = 0.f;
-#pragma unroll
-                        for (int i = 0; i < MT; ++i) c += Ac[i][n][e] + Ac[i][n][e + 2];
-                        c += __shfl_xor_sync(0xffffffffu, c, 4);
-                        c += __shfl_xor_sync(0xffffffffu, c, 8);
-                        c += __shfl_xor_sync(0xffffffffu, c, 16);
-                        cmax = fmaxf(cmax, c);
-                    }
-                const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
-                frag_store<MT, SM>(Ac, mA, g, t);  // mA is Z's slot
-                __syncwarp();
-                // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
-                            Zc[i][n][e] = alpha * mA[c * SM + rr];
-                        }
-                zexp = frag_normalise<MT>(Zc);
-                __syncwarp();  // every lane has read A^T before Z overwrites the slot
-                frag_store<MT, SM>(Zc, mZ, g, t);
-                to_hfrag<MT>(Ac, Ah);
-                __syncwarp();
-            }
-
-            // pseudo-inverse iteration (step 4), fp16 two-term split products
-#pragma unroll 1
-            for (int it = 0; it < iters; ++it) {
-                Frag<MT> X, Tm, P;
-                HFrag<MT> Xh;
-                mm_h<MT>(Ah, BSmemH<SM>{mZ, g, t}, X);  // X = A Z = 2^-zexp A Zc
-                const float unscale = ldexpf(1.f, -zexp);
-                // exact symmetrisation (X + X^T)/2; Z's slot holds X for the transpose
-                __syncwarp();
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) X[i][n][e] *= unscale;
-                frag_store<MT, SM>(X, mZ, g, t);
-                __syncwarp();
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
-                            X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + rr]);
-                            Tm[i][n][e] = X[i][n][e];
-                        }
-                to_hfrag<MT>(X, Xh);
-                frag_shift<MT>(Tm, 7.f, g, t);              // 7I - X
-                mm_h<MT>(Xh, BSymH<MT>{Tm}, P);              // X (7I - X)
-                frag_shift<MT>(P, 15.f, g, t);               // 15I - ...
-                mm_h<MT>(Xh, BSymH<MT>{P}, Tm);              // X (15I - ...)
-                frag_shift<MT>(Tm, 13.f, g, t);              // 13I - ...
-                {
-                    HFrag<MT> Zh;
-                    to_hfrag<MT>(Zc, Zh);
-                    mm_h<MT>(Zh, BSymH<MT>{Tm}, P);          // Zc (13I - ...)
-                }
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
-                zexp += frag_normalise<MT>(Zc);
-                __syncwarp();
-                frag_store<MT, SM>(Zc, mZ, g, t);
-                __syncwarp();
-            }
-
-            // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
-            {
-                float y[MT][NTO][4];
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) y[i][j][0] = y[i][j][1] = y[i][j][2] = y[i][j][3] = 0.f;
-                FragLo<MT> Zlo;
-                frag_lo<MT>(Zc, Zlo);
-#pragma unroll
-                for (int kk = 0; kk < 2 * MT; ++kk) {
-                    uint32_t ah[MT][4], al[MT][4];
-#pragma unroll
-                    for (int i = 0; i < MT; ++i) AFromFrag<MT>{Zc, Zlo}(i, kk, ah[i], al[i]);
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) {
-                        const float y0 = mW[(8 * kk + 2 * t) * WS + 8 * j + g];
-                        const float y1 = mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g];
-                        const uint32_t bh0 = __float_as_uint(y0), bh1 = __float_as_uint(y1);
-                        const uint32_t bl0 = tf32_lo(y0), bl1 = tf32_lo(y1);
-#pragma unroll
-                        for (int i = 0; i < MT; ++i) {
-                            mma_tf32(y[i][j], al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
-                            mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
-                            mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
-                        }
-                    }
-                }
-                // Y = 2^-zexp (Zc W).  fp16 output has a narrow range: scale Y by a
-                // power of two instead.  Numerator and denominator columns share the
-                // factor, so it cancels in step 7.
-                float scale = ldexpf(1.f, -zexp);
-                if (Op::kNarrowRange) {
-                    float ymax = 0.f;
-#pragma unroll
-                    for (int i = 0; i < MT; ++i)
-#pragma unroll
-                        for (int j = 0; j < NTO; ++j)
-#pragma unroll
-                            for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
-                    ymax = warp_max_nonneg(ymax);
-                    if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
-                }
-#pragma unroll
-                for (int i = 0; i < MT; ++i)
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) {
-                        const int rr = 16 * i + g, c = 8 * j + 2 * t;
-                        yT[c * YS + rr] = from_f32<T>(y[i][j][0] * scale);
-                        yT[(c + 1) * YS + rr] = from_f32<T>(y[i][j][1] * scale);
-                        yT[c * YS + rr + 8] = from_f32<T>(y[i][j][2] * scale);
-                        yT[(c + 1) * YS + rr + 8] = from_f32<T>(y[i][j][3] * scale);
-                    }
-            }
+            core_warp<T, M, NCOL>(qbar, kbar, mU, mW, mZ, yT, iters, sl2, g, t);
         }
         gsync();
 
         // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
-        {
-            uint32_t by[KTL][NTO][2];
-#pragma unroll
-            for (int kk = 0; kk < KTL; ++kk)
-#pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    const T* yr = yT + (8 * j + g) * YS + 16 * kk + 2 * t;
-                    by[kk][j][0] = ld32(yr);
-                    by[kk][j][1] = (M >= 16) ? ld32(yr + 8) : 0u;
-                }
-            const int jd = d >> 3, tdn = (d & 7) >> 1;
-            const int src = (lane & ~3) | tdn;
-            T* obase = Vs;  // staged here, then one bulk store of the warp's rows
-#pragma unroll 1
-            for (int ch = 0; ch < NCH; ++ch)
-#pragma unroll
-                for (int tm = 0; tm < 4; ++tm) {
-                    uint32_t f[KTL][4];
-                    if constexpr (GLS) {
-#pragma unroll
-                        for (int kk = 0; kk < KTL; ++kk) {
-                            const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
-                            if constexpr (M >= 16) {
-                                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
-                                f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = x.z; f[kk][3] = x.w;
-                            } else {
-                                const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
-                                f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = f[kk][3] = 0u;
-                            }
-                        }
-                    } else {
-                        gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
-                    }
-                    float o[NTO][4];
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-                    if constexpr (M >= 16) {
-#pragma unroll
-                        for (int kk = 0; kk < KTL; ++kk)
-#pragma unroll
-                            for (int j = 0; j < NTO; ++j) Op::k16(o[j], f[kk], by[kk][j][0], by[kk][j][1]);
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < NTO; ++j) Op::k8(o[j], f[0][0], f[0][1], by[0][j][0]);
-                    }
-                    float d0 = 0.f, d1 = 0.f;
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j)
-                        if (j == jd) {
-                            d0 = o[j][0];
-                            d1 = o[j][2];
-                        }
-                    const float i0 = __fdividef(1.f, __shfl_sync(0xffffffffu, d0, src));
-                    const float i1 = __fdividef(1.f, __shfl_sync(0xffffffffu, d1, src));
-                    T* o0 = obase + (ch * 64 + 16 * tm + g) * d;
-                    T* o1 = o0 + 8 * d;
-#pragma unroll
-                    for (int j = 0; j < NTO; ++j) {
-                        const int c = 8 * j + 2 * t;
-                        if (c < d) {
-                            *reinterpret_cast<uint32_t*>(o0 + c) = Op::pack(o[j][0] * i0, o[j][1] * i0);
-                            *reinterpret_cast<uint32_t*>(o1 + c) = Op::pack(o[j][2] * i1, o[j][3] * i1);
-                        }
-                    }
-                }
-        }
+        output_rows<T, M, NCOL, NCH, GLS>(glf, Qs, kbar, yT, Vs, d, g, t, lane, sl2);
 
         // The output rows are staged in V's region: one bulk store, and once it
         // has read shared memory, the next unit's V can land there.
