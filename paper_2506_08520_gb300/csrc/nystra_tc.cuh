@@ -21,7 +21,8 @@
 //            exactly G_U^n [V | 1] with the max over all N keys.
 //   core     warp 0: G_A^n = exp(Qbar Kbar^T - m_U), Z_0 = A^T/(||A||_1
 //            ||A||_inf), `iters` steps Z <- Z(13I - X(15I - X(7I - X)))/4 with
-//            X = A Z (step 4), Y = Z W, stored as a 16-bit B operand.
+//            X = A Z (step 4), Y = Z W, stored as a 16-bit B operand; all in
+//            registers.
 //   output   every warp: O = (G_L^n Y_:d) / (G_L^n Y_d) for its tokens
 //            (steps 5-7), staged row-major in its V region and written with
 //            one bulk store (whole sectors; scattered 4-byte stores of 60-byte
@@ -38,14 +39,15 @@
 // type with fp32 accumulation.  The m x m iteration needs close to fp32
 // accuracy (its round-off is amplified by ||A|| ||Z||, which grows with the
 // iteration count): it uses fp16 two-term splits (x = hi + lo, three k16
-// products lo*hi + hi*lo + hi*hi, 22 significant bits), with Z carried as
-// 2^e Z, e re-chosen every step, to stay in fp16's range.  Y = Z W uses
-// split-tf32 (W's range is not bounded).  The iteration runs in registers:
-// an MMA result is the next A operand (C layout -> A layout); X = A Z_k and
-// its polynomials are symmetric in exact arithmetic (Z_0 = a A^T), so their
-// B fragments are the lane's own C-layout values of the transpose.  The computed X is symmetrised,
-// (X + X^T)/2, every step, which keeps the antisymmetric round-off from
-// growing by up to 13/4 per step in directions that have not converged.
+// products lo*hi + hi*lo + hi*hi, 22 significant bits), with Z rescaled by a
+// power of two every step to stay in fp16's range.  Y = Z W uses split-tf32
+// (W's range is not bounded).  The iteration runs in registers: it carries
+// the symmetric X = A Z_k next to Z (X_{k+1} = X_k T3/4, equal to A Z_{k+1}),
+// so every product has a symmetric or transposed right factor whose B
+// fragments are the lane's own A fragments, and X is made exactly symmetric
+// (lower triangle mirrored with 8x8 movmatrix transposes) after each update,
+// which keeps antisymmetric round-off from growing by up to 13/4 per step in
+// directions that have not converged.
 // Scores are kept in the log2 domain (scaled by log2(e)/sqrt(d_h)), so each
 // exponential is one FFMA and one ex2.
 #pragma once
@@ -67,7 +69,6 @@ struct Layout {
     static constexpr int MT = (M + 15) / 16;             // landmark m-tiles
     static constexpr int MP = MT * 16;                   // padded landmark count
     static constexpr int LS = 40;                        // Qbar/Kbar row stride (16-bit elements)
-    static constexpr int SM = MP + 4;                    // fp32 core-matrix row stride
     static constexpr int WS = NCOL + 4;                  // fp32 W row stride
     static constexpr int YS = (M < 16 ? 16 : M) + 8;     // Y^T row stride (16-bit elements)
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;   // k-steps of O = G_L^n Y
@@ -85,8 +86,7 @@ struct Layout {
     // core has read Qbar/Kbar for the last time and is dead before the next
     // unit's landmarks, so it overlays them.  (With several warps a fast warp
     // could write the next landmarks while another still reads Y^T; without
-    // parking, the output phase still reads Kbar.)  G_A^n is stored only to
-    // read Z_0 = a A^T transposed, so it uses Z's slot.
+    // parking, the output phase still reads Kbar.)
     static constexpr bool YT_OVERLAY = (WPU == 1) && GLS;
     static constexpr size_t QK_BYTES = 2 * MP * LS * 2;
     static constexpr size_t YT_BYTES = ((NCOL * YS * 2 + 15) / 16) * 16;
@@ -96,9 +96,7 @@ struct Layout {
     static constexpr size_t G_MU = YT_OVERLAY ? (QK_BYTES > YT_BYTES ? QK_BYTES : YT_BYTES)
                                               : QK_BYTES + YT_BYTES;  // m_U, log2 domain
     static constexpr size_t G_W = G_MU + MP * 4;
-    static constexpr size_t G_Z = G_W + MP * WS * 4;
-    static constexpr size_t G_A = G_Z;
-    static constexpr size_t G_BAR = G_Z + MP * SM * 4;
+    static constexpr size_t G_BAR = G_W + MP * WS * 4;
     static constexpr size_t G_FLAG = G_BAR + 16 * WPU;  // two mbarriers per warp
     static constexpr size_t GROUP_BYTES = ((G_FLAG + 16 + 127) / 128) * 128;
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
@@ -126,63 +124,6 @@ __device__ __forceinline__ void frag_lo(const Frag<MT>& f, FragLo<MT>& lo) {
             for (int e = 0; e < 4; ++e) lo[i][n][e] = tf32_lo(f[i][n][e]);
 }
 
-// T = alpha I - D, in place.
-template <int MT>
-__device__ __forceinline__ void frag_shift(Frag<MT>& f, float alpha, int g, int t) {
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * n + (e & 1) + 2 * t);
-                f[i][n][e] = (diag ? alpha : 0.f) - f[i][n][e];
-            }
-}
-
-// D = A B (MP x MP, fp32 accumulate) on split-tf32 tensor cores.
-//   afrag(i, kk, hi[4], lo[4]) gives the A operand registers of m-tile i,
-//     k-step kk (k permuted as described in the header);
-//   bfrag(kk, j, y[2]) gives the B operand values of k-step kk, n-tile j.
-// Even and odd k-steps accumulate separately, halving each chain of
-// dependent MMAs.
-template <int MT, typename AF, typename BF>
-__device__ __forceinline__ void mm_tc(AF afrag, BF bfrag, Frag<MT>& D) {
-    float acc[2][MT][2 * MT][4];
-#pragma unroll
-    for (int p = 0; p < 2; ++p)
-#pragma unroll
-        for (int i = 0; i < MT; ++i)
-#pragma unroll
-            for (int j = 0; j < 2 * MT; ++j) acc[p][i][j][0] = acc[p][i][j][1] = acc[p][i][j][2] = acc[p][i][j][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < 2 * MT; ++kk) {
-        uint32_t ah[MT][4], al[MT][4];
-#pragma unroll
-        for (int i = 0; i < MT; ++i) afrag(i, kk, ah[i], al[i]);
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j) {
-            float y[2];
-            bfrag(kk, j, y);
-            const uint32_t bh0 = __float_as_uint(y[0]), bh1 = __float_as_uint(y[1]);
-            const uint32_t bl0 = tf32_lo(y[0]), bl1 = tf32_lo(y[1]);
-#pragma unroll
-            for (int i = 0; i < MT; ++i) {
-                float(&c)[4] = acc[kk & 1][i][j];
-                mma_tf32(c, al[i][0], al[i][1], al[i][2], al[i][3], bh0, bh1);
-                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bl0, bl1);
-                mma_tf32(c, ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
-            }
-        }
-    }
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) D[i][j][e] = acc[0][i][j][e] + acc[1][i][j][e];
-}
-
 // A operand (k-permuted) straight from C-layout fragments with precomputed low parts.
 template <int MT>
 struct AFromFrag {
@@ -195,26 +136,6 @@ struct AFromFrag {
         h[3] = __float_as_uint(f[i][kk][3]); l[3] = lo[i][kk][3];
     }
 };
-// B operand of a symmetric matrix from its own C-layout fragments.
-template <int MT>
-struct BFromSymFrag {
-    const Frag<MT>& f;
-    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
-        y[0] = f[j >> 1][kk][(j & 1) * 2];
-        y[1] = f[j >> 1][kk][(j & 1) * 2 + 1];
-    }
-};
-// B operand of a row-major fp32 matrix in shared memory (row stride S).
-template <int S>
-struct BFromSmem {
-    const float* m;
-    int g, t;
-    __device__ __forceinline__ void operator()(int kk, int j, float (&y)[2]) const {
-        y[0] = m[(8 * kk + 2 * t) * S + 8 * j + g];
-        y[1] = m[(8 * kk + 2 * t + 1) * S + 8 * j + g];
-    }
-};
-
 // ---- fp16 two-term split products for the m x m iteration ----
 // A operand registers (m16n8k16 row layout) of every m-tile i and k-step kk,
 // each register split into hi and lo halves.
@@ -234,63 +155,6 @@ __device__ __forceinline__ void to_hfrag(const Frag<MT>& c, HFrag<MT>& a) {
             a[i][kk][3] = split_h2(c[i][2 * kk + 1][2], c[i][2 * kk + 1][3]);
         }
 }
-
-// D = A B with A split in registers and B supplied by bfrag(kk, j, b[2]);
-// lo*hi + hi*lo and hi*hi accumulate separately (shorter dependent chains).
-template <int MT, typename BF>
-__device__ __forceinline__ void mm_h(const HFrag<MT>& A, BF bfrag, Frag<MT>& D) {
-    using H = Mma16<__half>;
-    float small[MT][2 * MT][4], big[MT][2 * MT][4];
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) small[i][j][e] = big[i][j][e] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < MT; ++kk)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j) {
-            H2Pair b[2];
-            bfrag(kk, j, b);
-#pragma unroll
-            for (int i = 0; i < MT; ++i) {
-                const uint32_t ahi[4] = {A[i][kk][0].hi, A[i][kk][1].hi, A[i][kk][2].hi, A[i][kk][3].hi};
-                const uint32_t alo[4] = {A[i][kk][0].lo, A[i][kk][1].lo, A[i][kk][2].lo, A[i][kk][3].lo};
-                H::k16(small[i][j], alo, b[0].hi, b[1].hi);
-                H::k16(small[i][j], ahi, b[0].lo, b[1].lo);
-                H::k16(big[i][j], ahi, b[0].hi, b[1].hi);
-            }
-        }
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) D[i][j][e] = big[i][j][e] + small[i][j][e];
-}
-
-// B operand (m16n8k16 col layout) of a symmetric matrix from its C-layout fragments.
-template <int MT>
-struct BSymH {
-    const Frag<MT>& f;
-    __device__ __forceinline__ void operator()(int kk, int j, H2Pair (&b)[2]) const {
-        const int i = j >> 1, e = (j & 1) * 2;
-        b[0] = split_h2(f[i][2 * kk][e], f[i][2 * kk][e + 1]);
-        b[1] = split_h2(f[i][2 * kk + 1][e], f[i][2 * kk + 1][e + 1]);
-    }
-};
-// B operand of a row-major fp32 matrix in shared memory (row stride S).
-template <int S>
-struct BSmemH {
-    const float* m;
-    int g, t;
-    __device__ __forceinline__ void operator()(int kk, int j, H2Pair (&b)[2]) const {
-        const float* c = m + (16 * kk + 2 * t) * S + 8 * j + g;
-        b[0] = split_h2(c[0], c[S]);
-        b[1] = split_h2(c[8 * S], c[9 * S]);
-    }
-};
 
 // Multiply fragments by 2^e with e chosen so that max |f| lands in
 // [2^10, 2^11) (fp16 headroom for the products); returns e (0 if f == 0).
@@ -316,16 +180,128 @@ __device__ __forceinline__ int frag_normalise(Frag<MT>& f) {
     return e;
 }
 
-template <int MT, int SM>
-__device__ __forceinline__ void frag_store(const Frag<MT>& f, float* S, int g, int t) {
+// ---- symmetric operands in registers ----
+// A operand register r of m-tile i, k-step kk holds the 8x8 block
+// (2i + (r & 1), 2kk + (r >> 1)): row g, columns 2t and 2t + 1 of it.  The
+// B operand of P^T is P's own A operand registers: k-step kk, n-tile j uses
+// registers (j & 1) and 2 + (j & 1) of m-tile j >> 1.
+
+// prmt selector that mirrors the lower triangle of a diagonal 8x8 block:
+// element (g, 2t) keeps the lane's value when g >= 2t, else takes the
+// transpose's, element (g, 2t + 1) likewise with g >= 2t + 1.
+__device__ __forceinline__ uint32_t tril_selector(int g, int t) {
+    return ((g >= 2 * t) ? 0x10u : 0x54u) | (((g >= 2 * t + 1) ? 0x32u : 0x76u) << 8);
+}
+
+template <int MT>
+__device__ __forceinline__ H2Pair split_reg(const Frag<MT>& c, int i, int kk, int r, float s) {
+    const int n = 2 * kk + (r >> 1), e = 2 * (r & 1);
+    return split_h2(s * c[i][n][e], s * c[i][n][e + 1]);
+}
+
+// A operand of s*C split into fp16 pairs.
+template <int MT>
+__device__ __forceinline__ void to_hfrag_scaled(const Frag<MT>& c, HFrag<MT>& a, float s) {
 #pragma unroll
     for (int i = 0; i < MT; ++i)
 #pragma unroll
-        for (int n = 0; n < 2 * MT; ++n) {
-            const int r = 16 * i + g, c = 8 * n + 2 * t;
-            *reinterpret_cast<float2*>(S + r * SM + c) = make_float2(f[i][n][0], f[i][n][1]);
-            *reinterpret_cast<float2*>(S + (r + 8) * SM + c) = make_float2(f[i][n][2], f[i][n][3]);
+        for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) a[i][kk][r] = split_reg<MT>(c, i, kk, r, s);
+}
+
+// A operand of the exactly symmetric matrix defined by the lower triangle of
+// s*C: blocks below the diagonal are split from C, diagonal blocks mirror
+// their lower triangle, blocks above are transposes of their mirror blocks.
+// Taking one triangle removes the antisymmetric round-off of a product of
+// symmetric factors before it can grow.
+template <int MT>
+__device__ __forceinline__ void sym_hfrag(const Frag<MT>& c, HFrag<MT>& a, uint32_t sel, float s) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int R = 2 * i + (r & 1), C = 2 * kk + (r >> 1);
+                if (R >= C) a[i][kk][r] = split_reg<MT>(c, i, kk, r, s);
+                if (R == C) {
+                    a[i][kk][r].hi = prmt(a[i][kk][r].hi, movmatrix_trans(a[i][kk][r].hi), sel);
+                    a[i][kk][r].lo = prmt(a[i][kk][r].lo, movmatrix_trans(a[i][kk][r].lo), sel);
+                }
+            }
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int R = 2 * i + (r & 1), C = 2 * kk + (r >> 1);
+                if (R < C) {
+                    const H2Pair src = a[C >> 1][R >> 1][(C & 1) + 2 * (R & 1)];
+                    a[i][kk][r] = H2Pair{movmatrix_trans(src.hi), movmatrix_trans(src.lo)};
+                }
+            }
+}
+
+// A operand of P^T from P's A operand (8x8 block transposes).
+template <int MT>
+__device__ __forceinline__ void transpose_hfrag(const HFrag<MT>& a, HFrag<MT>& b) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int R = 2 * i + (r & 1), C = 2 * kk + (r >> 1);
+                const H2Pair src = a[C >> 1][R >> 1][(C & 1) + 2 * (R & 1)];
+                b[i][kk][r] = H2Pair{movmatrix_trans(src.hi), movmatrix_trans(src.lo)};
+            }
+}
+
+// D = s I + A P^T (+ c I P^T when CI; i7 holds the A operand register of
+// c I's diagonal blocks) with fp16 two-term split operands: lo*hi + hi*lo
+// and hi*hi accumulate separately (shorter dependent chains).
+template <int MT, bool CI>
+__device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Frag<MT>& D, float s, uint32_t i7,
+                                      int g, int t) {
+    using H = Mma16<__half>;
+    float small[MT][2 * MT][4], big[MT][2 * MT][4];
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * j + (e & 1) + 2 * t);
+                big[i][j][e] = diag ? s : 0.f;
+                small[i][j][e] = 0.f;
+            }
+#pragma unroll
+    for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j) {
+            const H2Pair b0 = P[j >> 1][kk][j & 1], b1 = P[j >> 1][kk][2 + (j & 1)];
+#pragma unroll
+            for (int i = 0; i < MT; ++i) {
+                const uint32_t ahi[4] = {A[i][kk][0].hi, A[i][kk][1].hi, A[i][kk][2].hi, A[i][kk][3].hi};
+                const uint32_t alo[4] = {A[i][kk][0].lo, A[i][kk][1].lo, A[i][kk][2].lo, A[i][kk][3].lo};
+                H::k16(small[i][j], alo, b0.hi, b1.hi);
+                H::k16(small[i][j], ahi, b0.lo, b1.lo);
+                H::k16(big[i][j], ahi, b0.hi, b1.hi);
+                if (CI && kk == i) {
+                    const uint32_t ci[4] = {i7, 0u, 0u, i7};
+                    H::k16(big[i][j], ci, b0.hi, b1.hi);
+                    H::k16(small[i][j], ci, b0.lo, b1.lo);
+                }
+            }
         }
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) D[i][j][e] = big[i][j][e] + small[i][j][e];
 }
 
 // S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
@@ -548,21 +524,32 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
 }
 
 // Core, one warp: G_A^n = exp(Qbar Kbar^T - m_U) (mU: row maxima of this
-// lane's C-layout rows, log2 domain), Z_0 = A^T/(||A||_1 ||A||_inf), `iters`
-// steps Z <- Z (13I - X(15I - X(7I - X)))/4 with X = A Z (Algorithm 1 step 4)
-// on fp16 two-term-split MMAs in registers, and Y = Z W (split-tf32, W from
-// mW), stored as Y^T (16-bit B operand) at yT.  mZ is scratch for Z and X.
+// warp's rows of S_U in the log2 domain), the iterative pseudo-inverse
+// (step 4) and Y = Z W (W = G_U^n [V | 1], fp32 row-major with stride WS at
+// mW), stored as Y^T (16-bit B operand) at yT.
+//
+// The iteration is run in registers on the symmetric X = A Z_k (Z_0 = a A^T):
+// T2 = 15I - 7X + X X, T3 = 13I - X T2, Z <- Z T3/4 and X <- X T3/4 (equal to
+// A Z_{k+1}; its factors are polynomials in X and commute).  X is kept exactly
+// symmetric (lower triangle mirrored) after every update.  Scalar factors of
+// Z (a, 1/4 per step, the power-of-two range scaling) are dropped: O is a
+// ratio of two columns of G_L^n Z W, so they cancel.
 template <typename T, int M, int NCOL>
 __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const float (&mU)[(M + 15) / 16][2],
-                                          const float* mW, float* mZ, T* yT, int iters, float sl2, int g, int t) {
+                                          const float* mW, T* yT, int iters, float sl2, int g, int t) {
     using Op = Mma16<T>;
-    constexpr int MT = (M + 15) / 16, MP = MT * 16, LS = 40, SM = MP + 4, WS = NCOL + 4, NTO = NCOL / 8;
+    constexpr int MT = (M + 15) / 16, LS = 40, WS = NCOL + 4, NTO = NCOL / 8;
     constexpr int YS = (M < 16 ? 16 : M) + 8;
-    float* mA = mZ;  // G_A^n is stored only to read Z_0 = a A^T transposed
-    Frag<MT> Zc, Ac;
-    HFrag<MT> Ah;   // A = G_A^n as split fp16 A operand (constant over the iteration)
-    int zexp = 0;   // Zc holds 2^zexp Z (power-of-two scaling for fp16 range)
+    const uint32_t sel = tril_selector(g, t);
+    uint32_t i7;  // A operand register of -7I's diagonal blocks
     {
+        const __half2 h = __floats2half2_rn(g == 2 * t ? -7.f : 0.f, g == 2 * t + 1 ? -7.f : 0.f);
+        i7 = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    Frag<MT> Zc;
+    HFrag<MT> Xh, Zh;
+    {
+        Frag<MT> Ac;
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
             uint32_t aq[2][4];
@@ -618,73 +605,44 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                 cmax = fmaxf(cmax, c);
             }
         const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
-        frag_store<MT, SM>(Ac, mA, g, t);  // mA is Z's slot
-        __syncwarp();
-        // Z_0 = alpha A^T: C-layout element (r, c) is alpha * A[c][r].
-#pragma unroll
-        for (int i = 0; i < MT; ++i)
-#pragma unroll
-            for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
-                    Zc[i][n][e] = alpha * mA[c * SM + rr];
-                }
-        zexp = frag_normalise<MT>(Zc);
-        __syncwarp();  // every lane has read A^T before Z overwrites the slot
-        frag_store<MT, SM>(Zc, mZ, g, t);
+        HFrag<MT> Ah;
         to_hfrag<MT>(Ac, Ah);
-        __syncwarp();
+        transpose_hfrag<MT>(Ah, Zh);  // Z_0 = A^T (a dropped)
+        mm_hT<MT, false>(Ah, Ah, Ac, 0.f, 0u, g, t);
+        sym_hfrag<MT>(Ac, Xh, sel, alpha);  // X_0 = a A A^T
+        if (iters == 0) {
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int kk = 0; kk < MT; ++kk)
+#pragma unroll
+                    for (int r = 0; r < 4; ++r) {
+                        const uint32_t hb = Zh[i][kk][r].hi, lb = Zh[i][kk][r].lo;
+                        const float2 h = __half22float2(*reinterpret_cast<const __half2*>(&hb));
+                        const float2 l = __half22float2(*reinterpret_cast<const __half2*>(&lb));
+                        const int n = 2 * kk + (r >> 1), e = 2 * (r & 1);
+                        Zc[i][n][e] = h.x + l.x;
+                        Zc[i][n][e + 1] = h.y + l.y;
+                    }
+        }
     }
 
-    // pseudo-inverse iteration (step 4), fp16 two-term split products
+    // pseudo-inverse iteration (step 4)
 #pragma unroll 1
     for (int it = 0; it < iters; ++it) {
-        Frag<MT> X, Tm, P;
-        HFrag<MT> Xh;
-        mm_h<MT>(Ah, BSmemH<SM>{mZ, g, t}, X);  // X = A Z = 2^-zexp A Zc
-        const float unscale = ldexpf(1.f, -zexp);
-        // exact symmetrisation (X + X^T)/2; Z's slot holds X for the transpose
-        __syncwarp();
-#pragma unroll
-        for (int i = 0; i < MT; ++i)
-#pragma unroll
-            for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) X[i][n][e] *= unscale;
-        frag_store<MT, SM>(X, mZ, g, t);
-        __syncwarp();
-#pragma unroll
-        for (int i = 0; i < MT; ++i)
-#pragma unroll
-            for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const int rr = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
-                    X[i][n][e] = 0.5f * (X[i][n][e] + mZ[c * SM + rr]);
-                    Tm[i][n][e] = X[i][n][e];
-                }
-        to_hfrag<MT>(X, Xh);
-        frag_shift<MT>(Tm, 7.f, g, t);              // 7I - X
-        mm_h<MT>(Xh, BSymH<MT>{Tm}, P);              // X (7I - X)
-        frag_shift<MT>(P, 15.f, g, t);               // 15I - ...
-        mm_h<MT>(Xh, BSymH<MT>{P}, Tm);              // X (15I - ...)
-        frag_shift<MT>(Tm, 13.f, g, t);              // 13I - ...
-        {
-            HFrag<MT> Zh;
+        Frag<MT> F;
+        HFrag<MT> Th;
+        mm_hT<MT, true>(Xh, Xh, F, 15.f, i7, g, t);  // T2 = 15I - 7X + X X
+        to_hfrag_scaled<MT>(F, Th, -0.25f);           // -T2/4
+        mm_hT<MT, false>(Xh, Th, F, 3.25f, 0u, g, t);  // T3/4 = 13/4 I - X T2/4
+        to_hfrag<MT>(F, Th);
+        mm_hT<MT, false>(Zh, Th, Zc, 0.f, 0u, g, t);   // Z T3/4
+        if (it + 1 < iters) {
+            mm_hT<MT, false>(Xh, Th, F, 0.f, 0u, g, t);  // X T3/4
+            sym_hfrag<MT>(F, Xh, sel, 1.f);
+            frag_normalise<MT>(Zc);
             to_hfrag<MT>(Zc, Zh);
-            mm_h<MT>(Zh, BSymH<MT>{Tm}, P);          // Zc (13I - ...)
         }
-#pragma unroll
-        for (int i = 0; i < MT; ++i)
-#pragma unroll
-            for (int n = 0; n < 2 * MT; ++n)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) Zc[i][n][e] = 0.25f * P[i][n][e];
-        zexp += frag_normalise<MT>(Zc);
-        __syncwarp();
-        frag_store<MT, SM>(Zc, mZ, g, t);
-        __syncwarp();
     }
 
     // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
@@ -715,10 +673,10 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                 }
             }
         }
-        // Y = 2^-zexp (Zc W).  fp16 output has a narrow range: scale Y by a
-        // power of two instead.  Numerator and denominator columns share the
-        // factor, so it cancels in step 7.
-        float scale = ldexpf(1.f, -zexp);
+        // fp16 output has a narrow range: scale Y by a power of two.
+        // Numerator and denominator columns share the factor, so it cancels
+        // in step 7.
+        float scale = 1.f;
         if (Op::kNarrowRange) {
             float ymax = 0.f;
 #pragma unroll
@@ -823,8 +781,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                  unsigned int* fault, int active) {
     using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
     using Op = Mma16<T>;
-    constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS, SM = Lay::SM,
-                  WS = Lay::WS, YS = Lay::YS, KTL = Lay::KTL, NTO = NCOL / 8;
+    constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS,
+                  WS = Lay::WS, KTL = Lay::KTL;
     constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
     constexpr int LPW = TPW / L;  // landmarks owned by one warp
     static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
@@ -845,8 +803,6 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
     T* kbar = reinterpret_cast<T*>(gb + Lay::G_KBAR);
     float* gmu = reinterpret_cast<float*>(gb + Lay::G_MU);
     float* mW = reinterpret_cast<float*>(gb + Lay::G_W);
-    float* mA = reinterpret_cast<float*>(gb + Lay::G_A);
-    float* mZ = reinterpret_cast<float*>(gb + Lay::G_Z);
     T* yT = reinterpret_cast<T*>(gb + Lay::G_YT);
     uint64_t* barQK = reinterpret_cast<uint64_t*>(gb + Lay::G_BAR) + 2 * r;  // Q and K rows
     uint64_t* barV = barQK + 1;                                                // V rows
@@ -980,7 +936,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                     mU[mt][1] = gmu[16 * mt + g + 8];
                 }
             }
-            core_warp<T, M, NCOL>(qbar, kbar, mU, mW, mZ, yT, iters, sl2, g, t);
+            core_warp<T, M, NCOL>(qbar, kbar, mU, mW, yT, iters, sl2, g, t);
         }
         gsync();
 
