@@ -688,6 +688,7 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
             ymax = warp_max_nonneg(ymax);
             if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
         }
+        __syncwarp();  // Y^T may overlay the landmarks: every lane has read them
 #pragma unroll
         for (int i = 0; i < MT; ++i)
 #pragma unroll
@@ -1015,11 +1016,24 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
     return cudaGetLastError();
 }
 
+// Stage-pool kernel for 8x8 windows (nystra_pool.cuh, N = 64 translation unit only).
+template <typename T, int M, int NCOL>
+cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                        int iters, cudaStream_t stream, unsigned int* fault);
+
 // Dispatch on m and the output-column padding for one window size.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
                      int iters, cudaStream_t stream, unsigned int* fault) {
     const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
+    if constexpr (TPW == 64 && WPU == 1) {
+        if (m == 8)
+            return wide ? launch_pool<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_pool<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (m == 16)
+            return wide ? launch_pool<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_pool<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
     switch (m) {
         case 8:
             return wide ? launch_cfg<T, 8, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)

@@ -1,5 +1,7 @@
-// Tensor-core PnP-Nystra kernels for windows of 64 tokens (see nystra_tc.cuh):
-// each unit is handled by 1 warp(s) of 64 tokens.
+// Tensor-core PnP-Nystra kernels for windows of 64 tokens: the stage-pool
+// kernel (nystra_pool.cuh) for m <= 16, the grouped kernel (nystra_tc.cuh,
+// one warp per unit) for m = 32.
 #include "nystra_tc.cuh"
+#include "nystra_pool.cuh"
 
 NYSTRA_TC_DEFINE(n64, 64, 1)
