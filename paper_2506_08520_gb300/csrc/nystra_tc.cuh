@@ -1021,6 +1021,11 @@ template <typename T, int M, int NCOL>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault);
 
+// Team kernel for 16x16 windows (nystra_team.cuh, N = 256 translation unit only).
+template <typename T, int M, int NCOL>
+cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                        int iters, cudaStream_t stream, unsigned int* fault);
+
 // Dispatch on m and the output-column padding for one window size.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
@@ -1033,6 +1038,14 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
         if (m == 16)
             return wide ? launch_pool<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_pool<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    if constexpr (TPW == 64 && WPU == 4) {
+        if (m == 8)
+            return wide ? launch_team<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_team<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (m == 16)
+            return wide ? launch_team<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_team<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
     switch (m) {
         case 8:

@@ -1,5 +1,7 @@
-// Tensor-core PnP-Nystra kernels for windows of 256 tokens (see nystra_tc.cuh):
-// each unit is handled by 4 warp(s) of 64 tokens.
+// Tensor-core PnP-Nystra kernels for windows of 256 tokens: the team kernel
+// (nystra_team.cuh) for m <= 16, the grouped kernel (nystra_tc.cuh, four
+// warps of 64 tokens per unit) for m = 32.
 #include "nystra_tc.cuh"
+#include "nystra_team.cuh"
 
 NYSTRA_TC_DEFINE(n256, 64, 4)

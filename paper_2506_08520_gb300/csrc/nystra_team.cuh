@@ -1,0 +1,300 @@
+// Team PnP-Nystra kernel for 16x16 windows (N = 256 tokens), m <= 16, even
+// d_h <= 32, 16-bit I/O.  Included by the N = 256 translation unit after
+// nystra_tc.cuh, whose per-phase device functions it reuses.
+//
+// In the grouped kernel the m x m core runs on one warp of a unit's group
+// while the group's other warps wait, so the core (a latency-bound chain of
+// small products) is exposed once per unit.  Here a team is four token warps
+// (64 tokens each, as in the grouped kernel) plus a dedicated core warp, and
+// the per-unit state handed between them is double-buffered: while the core
+// warp runs the iteration of unit k, the token warps run the front phase of
+// unit k + 1 and then the output of unit k.
+//
+// Token warp r, unit k (buffer b = k mod 2):
+//   wait Q, K rows -> landmarks -> [sync] -> S_L, G_L^n parked -> wait V ->
+//   S_U, partial W_r -> [sync] -> combine into W, m_U -> [sync] -> signal the
+//   core (mbarrier F_b) -> copy Q, K of unit k + 1 -> wait for the core of
+//   unit k - 1 (mbarrier C_{1-b}) -> output of unit k - 1 staged in the V
+//   rows and bulk-stored -> copy V of unit k + 1.
+// Core warp, unit k: wait F_b -> G_A^n, iteration, Y^T into buffer b ->
+//   signal C_b.
+// [sync] is a named barrier over the four token warps.  Every wait on an
+// mbarrier is bounded; a failed wait sets the team's flag, and the token
+// warps leave the loop together at the flag checks after a barrier.
+#pragma once
+
+#include "nystra_tc.cuh"
+
+namespace nystra {
+namespace tc {
+
+template <int M, int NCOL>
+struct TeamLayout {
+    static constexpr int NT = 4, TPW = 64, N = NT * TPW;  // token warps, tokens per token warp
+    static constexpr int DS = (NCOL == 32) ? 30 : 32;
+    static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int KTL = (M >= 16) ? M / 16 : 1;
+    static constexpr int GLB = (M >= 16) ? 16 : 8;
+    static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;  // a token warp's Q, K, V rows
+    static constexpr size_t WPART = (size_t)TPW * DS * 2;      // partial W_r after Q (K, V consumed)
+    static_assert((size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
+    // one buffer of per-unit state
+    static constexpr size_t GLF_W = 4 * KTL * 32 * GLB;  // one token warp's G_L^n fragments
+    static constexpr size_t B_QB = 0;
+    static constexpr size_t B_KB = B_QB + MP * LS * 2;
+    static constexpr size_t B_W = B_KB + MP * LS * 2;
+    static constexpr size_t B_MU = B_W + MP * WS * 4;
+    static constexpr size_t B_YT = B_MU + MP * 4;
+    static constexpr size_t B_GLF = B_YT + ((NCOL * YS * 2 + 15) / 16) * 16;
+    static constexpr size_t BUF = B_GLF + NT * GLF_W;
+    // team memory: stages, two buffers, mbarriers, flag
+    static constexpr size_t T_BUF = NT * STAGE;
+    static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // barQK[4], barV[4], F[2], C[2]
+    static constexpr size_t T_FLAG = T_BAR + 12 * 8;
+    static constexpr size_t TEAM = ((T_FLAG + 16 + 127) / 128) * 128;
+    static constexpr int TEAMS = (int)(kSmemLimit / TEAM) < 3 ? (int)(kSmemLimit / TEAM) : 3;
+    static_assert(TEAMS >= 1, "team does not fit in shared memory");
+    static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
+};
+
+template <typename T, int M, int NCOL>
+__global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
+nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
+                   T* __restrict__ out, long long n_units, int d, int iters, float sl2, unsigned int* fault) {
+    using Lay = TeamLayout<M, NCOL>;
+    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
+                  KTL = Lay::KTL, NCOLC = NCOL;
+    constexpr int L = N / M, LPW = TPW / L;
+    static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
+
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int team = warp / (NT + 1), r = warp - team * (NT + 1);  // r == NT: core warp
+    const int g = lane >> 2, t = lane & 3;
+    unsigned char* tb = smem_raw + (size_t)team * Lay::TEAM;
+    auto buf = [&](int b) { return tb + Lay::T_BUF + (size_t)b * Lay::BUF; };
+    uint64_t* bars = reinterpret_cast<uint64_t*>(tb + Lay::T_BAR);
+    uint64_t* barF = bars + 8;  // F[b]: the token warps' state for the core is ready
+    uint64_t* barC = bars + 10; // C[b]: the core's Y^T is ready
+    volatile unsigned int* flag = reinterpret_cast<volatile unsigned int*>(tb + Lay::T_FLAG);
+
+    const long long stride = (long long)gridDim.x * Lay::TEAMS;
+    const long long u0 = (long long)blockIdx.x * Lay::TEAMS + team;
+
+    if (threadIdx.x == 0) {
+        for (int tm = 0; tm < Lay::TEAMS; ++tm) {
+            uint64_t* bb = reinterpret_cast<uint64_t*>(smem_raw + (size_t)tm * Lay::TEAM + Lay::T_BAR);
+            for (int i = 0; i < 8; ++i) mbar_init(bb + i, 1);
+            mbar_init(bb + 8, NT);
+            mbar_init(bb + 9, NT);
+            mbar_init(bb + 10, 1);
+            mbar_init(bb + 11, 1);
+            *reinterpret_cast<volatile unsigned int*>(smem_raw + (size_t)tm * Lay::TEAM + Lay::T_FLAG) = 0u;
+        }
+        fence_mbar_init();
+    }
+    // padding landmark rows (m < 16) stay zero: nothing else writes them
+    if constexpr (M < MP) {
+        for (int idx = threadIdx.x; idx < Lay::TEAMS * 2 * (MP - M) * 16; idx += blockDim.x) {
+            const int tm = idx / (2 * (MP - M) * 16), rem = idx - tm * 2 * (MP - M) * 16;
+            const int b = rem / ((MP - M) * 16), e = rem - b * (MP - M) * 16;
+            unsigned char* bb = smem_raw + (size_t)tm * Lay::TEAM + Lay::T_BUF + (size_t)b * Lay::BUF;
+            const int jr = M + (e >> 4), p = e & 15;
+            *reinterpret_cast<uint32_t*>(bb + Lay::B_QB + (jr * LS + 2 * p) * 2) = 0u;
+            *reinterpret_cast<uint32_t*>(bb + Lay::B_KB + (jr * LS + 2 * p) * 2) = 0u;
+        }
+    }
+    __syncthreads();
+
+    if (r == NT) {
+        // ======================= core warp =======================
+        for (long long kk = 0;; ++kk) {
+            const long long u = u0 + kk * stride;
+            if (u >= n_units) break;
+            const int b = (int)(kk & 1);
+            const uint32_t par = (uint32_t)((kk >> 1) & 1);
+            const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, par, kWaitNs));
+            if (!ok) {
+                if (lane == 0) {
+                    atomicOr(fault, 1u);
+                    *flag = 1u;
+                }
+                break;
+            }
+            if (*flag != 0u) break;
+            unsigned char* bb = buf(b);
+            const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
+            float mU[1][2] = {{gmu[g], gmu[g + 8]}};
+            core_warp<T, M, NCOLC>(reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB),
+                                   mU, reinterpret_cast<const float*>(bb + Lay::B_W),
+                                   reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(barC + b);
+        }
+        return;
+    }
+
+    // ======================= token warp r =======================
+    T* Qs = reinterpret_cast<T*>(tb + (size_t)r * Lay::STAGE);
+    const int td = TPW * d;
+    T* Ks = Qs + td;
+    T* Vs = Qs + 2 * td;
+    float* wpart = reinterpret_cast<float*>(tb + (size_t)r * Lay::STAGE + Lay::WPART);
+    uint64_t* barQK = bars + r;
+    uint64_t* barV = bars + 4 + r;
+    const uint32_t tile_bytes = (uint32_t)(td * sizeof(T));
+    auto unit_off = [&](long long unit) { return (size_t)unit * N * d + (size_t)r * td; };
+    auto issue_qk = [&](long long unit) {
+        mbar_arrive_expect_tx(barQK, 2u * tile_bytes);
+        bulk_g2s(Qs, q + unit_off(unit), tile_bytes, barQK);
+        bulk_g2s(Ks, k + unit_off(unit), tile_bytes, barQK);
+    };
+    auto issue_v = [&](long long unit) {
+        mbar_arrive_expect_tx(barV, tile_bytes);
+        bulk_g2s(Vs, v + unit_off(unit), tile_bytes, barV);
+    };
+    auto tsync = [&]() { named_barrier(1 + team, NT * 32); };
+    uint32_t phase_qk = 0, phase_v = 0;
+    bool pend_qk = false, pend_v = false;  // copies issued and not yet waited for
+
+    // Output of unit kk (its core has run on buffer kk mod 2), staged in the
+    // V rows; returns once the bulk store has read the staging.
+    auto output_unit = [&](long long kk) {
+        const int b = (int)(kk & 1);
+        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barC + b, (uint32_t)((kk >> 1) & 1), kWaitNs));
+        if (!ok) {
+            if (lane == 0) {
+                atomicOr(fault, 1u);
+                *flag = 1u;
+            }
+            return;
+        }
+        unsigned char* bb = buf(b);
+        output_rows<T, M, NCOLC, 1, true>(reinterpret_cast<const uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W), Qs,
+                                          reinterpret_cast<const T*>(bb + Lay::B_KB),
+                                          reinterpret_cast<const T*>(bb + Lay::B_YT), Vs, d, g, t, lane, sl2);
+        fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
+        __syncwarp();
+        if (lane == 0) {
+            bulk_s2g(out + unit_off(u0 + kk * stride), Vs, tile_bytes);
+            bulk_commit();
+            bulk_wait_read_all();
+        }
+        __syncwarp();
+    };
+
+    if (u0 < n_units && lane == 0) {
+        issue_qk(u0);
+        issue_v(u0);
+    }
+    pend_qk = pend_v = u0 < n_units;
+    long long kk = 0;
+    for (;; ++kk) {
+        const long long u = u0 + kk * stride;
+        if (u >= n_units) break;
+        const int b = (int)(kk & 1);
+        unsigned char* bb = buf(b);
+        T* qbar = reinterpret_cast<T*>(bb + Lay::B_QB);
+        T* kbar = reinterpret_cast<T*>(bb + Lay::B_KB);
+        // ---------------- bounded wait for Q and K ----------------
+        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
+        if (!ok && lane == 0) {
+            atomicOr(fault, 1u);
+            *flag = 1u;
+        }
+        phase_qk ^= 1u;
+        pend_qk = !ok;
+        // ---------------- landmarks (Algorithm 1 step 1) ----------------
+        landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
+        landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
+        tsync();
+        if (*flag != 0u) break;
+        // ---------------- S_L, G_L^n fragments parked in buffer b ----------------
+        {
+            uint32_t* glf = reinterpret_cast<uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W);
+#pragma unroll
+            for (int tm = 0; tm < 4; ++tm) {
+                uint32_t f[KTL][4];
+                gl_tile<T, M, KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
+#pragma unroll
+                for (int kq = 0; kq < KTL; ++kq) {
+                    const int slot = (tm * KTL + kq) * 32 + lane;
+                    if constexpr (M >= 16)
+                        reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[kq][0], f[kq][1], f[kq][2], f[kq][3]);
+                    else
+                        reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[kq][0], f[kq][1]);
+                }
+            }
+        }
+        // ---------------- bounded wait for V ----------------
+        const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
+        if (!ok_v && lane == 0) {
+            atomicOr(fault, 1u);
+            *flag = 1u;
+        }
+        phase_v ^= 1u;
+        pend_v = !ok_v;
+        // ---------------- S_U, partial W_r and row maxima ----------------
+        float mU[1][2];
+        front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, NCOLC, mU);
+        if (t == 0) {
+            wpart[MP * NCOLC + g] = mU[0][0];
+            wpart[MP * NCOLC + g + 8] = mU[0][1];
+        }
+        tsync();
+        combine_partials<MP, NCOLC, WS, NT>(reinterpret_cast<const float*>(tb + Lay::WPART), Lay::STAGE / 4,
+                                             reinterpret_cast<float*>(bb + Lay::B_W),
+                                             reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
+        tsync();
+        if (*flag != 0u) break;
+        // ---------------- hand buffer b to the core warp ----------------
+        __syncwarp();
+        if (lane == 0) mbar_arrive(barF + b);
+        // Q, K and the partials are consumed: copy the next unit's Q and K rows.
+        const long long un = u + stride;
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (un < n_units && lane == 0) issue_qk(un);
+        pend_qk = pend_qk || un < n_units;
+        // ---------------- output of the previous unit ----------------
+        if (kk >= 1) output_unit(kk - 1);
+        // The V rows are free (consumed, and the staging has been read).
+        if (un < n_units && lane == 0) issue_v(un);
+        pend_v = pend_v || un < n_units;
+    }
+    if (kk >= 1 && *flag == 0u) output_unit(kk - 1);
+    if (lane == 0) bulk_wait_all();  // output stores complete before exit
+    // Fault path only: copies still in flight land before the CTA's memory is released.
+    if (pend_qk) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
+    if (pend_v) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
+}
+
+template <typename T, int M, int NCOL>
+cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                        int iters, cudaStream_t stream, unsigned int* fault) {
+    using Lay = TeamLayout<M, NCOL>;
+    auto kern = nystra_team_kernel<T, M, NCOL>;
+    const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
+    static int s_blocks = 0;  // persistent grid size, set on first use
+    if (s_blocks == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per_sm = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * 5 * 32, smem)) !=
+            cudaSuccess)
+            return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        s_blocks = sms * per_sm;
+    }
+    const long long want = (n_units + Lay::TEAMS - 1) / Lay::TEAMS;
+    const long long grid = want < s_blocks ? want : s_blocks;
+    const float sl2 = 1.4426950408889634f / sqrtf((float)d);
+    kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
+                                                                 n_units, d, iters, sl2, fault);
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace nystra
