@@ -51,7 +51,7 @@ int nystra_attention(const void* q, const void* k, const void* v, void* out, int
     if (units == 0) return NYSTRA_OK;
     const cudaStream_t s = (cudaStream_t)stream;
     const bool tc = (dtype == NYSTRA_BF16 || dtype == NYSTRA_F16) && d_h % 2 == 0 && d_h <= 32 &&
-                    (m == 8 || m == 16 || m == 32);
+                    (m == 8 || m == 16 || m == 32 || m == 64);
     cudaError_t e;
     if (tc && N == 64)
         e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, dtype, s);

@@ -61,9 +61,22 @@ namespace tc {
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
 constexpr size_t kSmemLimit = 232448;        // opt-in dynamic shared memory per CTA
 
-template <int M, int NCOL, int TPW, int WPU, bool GLS>
+// Shared scratch of the distributed core (m = 32, 64; see dist_core): two
+// matrices of fp16 pairs (hi plane, then lo plane; rows padded to m + 8
+// halves so ldmatrix is conflict-free) and an auxiliary float area.
+template <int M>
+struct DistScratch {
+    static constexpr int CW = M / 16, SS = M + 8;
+    static constexpr size_t PLANE = (size_t)M * SS * 2;
+    static constexpr size_t MAT = 2 * PLANE;
+    static constexpr size_t AUX = ((size_t)CW * M * 4 + 3 * CW * 4 + 15) / 16 * 16;  // column sums, maxima
+    static constexpr size_t BYTES = ((2 * MAT + AUX + 127) / 128) * 128;
+};
+
+template <int M, int NCOL, int TPW, int WPU, bool GLS, int CW = 1>
 struct Layout {
     static constexpr int N = TPW * WPU;
+    static constexpr int GW = WPU > CW ? WPU : CW;       // warps per group (token warps first)
     static constexpr int NCH = TPW / 64;                 // 64-token chunks per warp
     static constexpr int DS = (NCOL == 32) ? 30 : 32;    // staged row width bound (d_h <= DS)
     static constexpr int MT = (M + 15) / 16;             // landmark m-tiles
@@ -80,7 +93,8 @@ struct Layout {
     // A warp's partial W (fp32 MP x NCOL, then MP row maxima) lives in its
     // stage right after the Q rows, once K and V are consumed.
     static constexpr size_t WPART = (size_t)TPW * DS * 2;
-    static_assert((size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
+    static_assert(WPU == 1 || (size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2,
+                  "W partial must fit in K+V");
     // per-group shared memory
     // With one warp per unit and G_L^n parked, Y^T is written only after the
     // core has read Qbar/Kbar for the last time and is dead before the next
@@ -97,8 +111,19 @@ struct Layout {
                                               : QK_BYTES + YT_BYTES;  // m_U, log2 domain
     static constexpr size_t G_W = G_MU + MP * 4;
     static constexpr size_t G_BAR = G_W + MP * WS * 4;
-    static constexpr size_t G_FLAG = G_BAR + 16 * WPU;  // two mbarriers per warp
-    static constexpr size_t GROUP_BYTES = ((G_FLAG + 16 + 127) / 128) * 128;
+    static constexpr size_t G_FLAG = G_BAR + 16 * WPU;  // two mbarriers per token warp
+    // Distributed core (CW > 1): its scratch is group memory, or, with long
+    // stages (TPW >= 256), the first two token warps' K/V rows (consumed by
+    // the combine before the core starts; the next unit's K and V are copied
+    // after the core).
+    static constexpr bool SCR_IN_STAGE = (CW > 1) && (TPW >= 256);
+    static constexpr size_t SCR_BYTES = (CW > 1 && !SCR_IN_STAGE) ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0;
+    static_assert(!SCR_IN_STAGE || (WPU >= 2 && DistScratch<(M > 16 ? M : 32)>::MAT +
+                                                       DistScratch<(M > 16 ? M : 32)>::AUX <=
+                                                   2 * (size_t)TPW * DS * 2),
+                  "scratch must fit in two warps' K/V rows");
+    static constexpr size_t G_SCR = ((G_FLAG + 16 + 127) / 128) * 128;
+    static constexpr size_t GROUP_BYTES = ((G_SCR + SCR_BYTES + 127) / 128) * 128;
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
 };
 
@@ -702,6 +727,356 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
     }
         }
 
+// ---- distributed core for m = 32, 64: CW = m/16 warps, warp c owns rows 16c..16c+15 ----
+// The m x m operands no longer fit one warp's registers.  Each warp keeps the
+// A operands of its own rows (X and Z, fp16 pairs) and reads right-hand
+// factors from two shared-memory matrices (hi and lo planes, rows padded to
+// m + 8 halves so ldmatrix is conflict-free) that alternate roles: X in one,
+// -T2/4 in the other, T3/4 over X once every warp has used X, the next X over
+// -T2/4 once every warp has used it; three barriers per step.
+
+template <int M>
+__device__ __forceinline__ void dist_store(unsigned char* mat, int row, int col, const H2Pair& p) {
+    constexpr int SS = DistScratch<M>::SS;
+    *reinterpret_cast<uint32_t*>(mat + ((size_t)row * SS + col) * 2) = p.hi;
+    *reinterpret_cast<uint32_t*>(mat + DistScratch<M>::PLANE + ((size_t)row * SS + col) * 2) = p.lo;
+}
+
+// Own rows of s*acc into a scratch matrix.
+template <int M>
+__device__ __forceinline__ void dist_put(unsigned char* mat, const float (&acc)[M / 8][4], float s, int c, int g,
+                                         int t) {
+#pragma unroll
+    for (int n = 0; n < M / 8; ++n) {
+        dist_store<M>(mat, 16 * c + g, 8 * n + 2 * t, split_h2(s * acc[n][0], s * acc[n][1]));
+        dist_store<M>(mat, 16 * c + g + 8, 8 * n + 2 * t, split_h2(s * acc[n][2], s * acc[n][3]));
+    }
+}
+
+// The symmetric matrix defined by the lower triangle of s*acc: own blocks on
+// and below the diagonal (diagonal blocks mirrored) and their transposes.
+template <int M>
+__device__ __forceinline__ void dist_put_sym(unsigned char* mat, const float (&acc)[M / 8][4], float s, int c,
+                                             int g, int t, uint32_t sel) {
+#pragma unroll
+    for (int n = 0; n < M / 8; ++n)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int R = 2 * c + h;
+            if (R < n) continue;  // warp-uniform
+            H2Pair p = split_h2(s * acc[n][2 * h], s * acc[n][2 * h + 1]);
+            if (R == n) {
+                p.hi = prmt(p.hi, movmatrix_trans(p.hi), sel);
+                p.lo = prmt(p.lo, movmatrix_trans(p.lo), sel);
+                dist_store<M>(mat, 8 * R + g, 8 * n + 2 * t, p);
+            } else {
+                dist_store<M>(mat, 8 * R + g, 8 * n + 2 * t, p);
+                dist_store<M>(mat, 8 * n + g, 8 * R + 2 * t,
+                              H2Pair{movmatrix_trans(p.hi), movmatrix_trans(p.lo)});
+            }
+        }
+}
+
+// A operand of the own rows (tr: of the transpose's own rows) from a scratch matrix.
+template <int M, bool TR>
+__device__ __forceinline__ void dist_load_a(const unsigned char* mat, H2Pair (&a)[M / 16][4], int c, int lane) {
+    constexpr int SS = DistScratch<M>::SS;
+    const int blk = lane >> 3, rr = lane & 7;
+#pragma unroll
+    for (int kk = 0; kk < M / 16; ++kk) {
+        int row, col;
+        if (TR) {
+            row = 16 * kk + 8 * (blk >> 1) + rr;
+            col = 16 * c + 8 * (blk & 1);
+        } else {
+            row = 16 * c + 8 * (blk & 1) + rr;
+            col = 16 * kk + 8 * (blk >> 1);
+        }
+        uint32_t h[4], l[4];
+        const unsigned char* ph = mat + ((size_t)row * SS + col) * 2;
+        if (TR) {
+            ldsm_x4_t(h, ph);
+            ldsm_x4_t(l, ph + DistScratch<M>::PLANE);
+        } else {
+            ldsm_x4(h, ph);
+            ldsm_x4(l, ph + DistScratch<M>::PLANE);
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) a[kk][r] = H2Pair{h[r], l[r]};
+    }
+}
+
+// acc[a] = s I + A_a P^T over the own rows for NA left operands sharing the
+// right factor P (all m rows, from scratch); with CI also adds (-7I) P^T,
+// whose own-row block lies in k-step c (i7: its diagonal A register).
+template <int M, int NA, bool CI>
+__device__ __forceinline__ void dist_mm(const H2Pair (*const (&A)[NA])[4], const unsigned char* mat,
+                                        float (*const (&acc)[NA])[4], float s, uint32_t i7, int c, int g, int t,
+                                        int lane) {
+    using H = Mma16<__half>;
+    constexpr int SS = DistScratch<M>::SS, NT = M / 8;
+#pragma unroll
+    for (int a = 0; a < NA; ++a)
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                acc[a][n][e] = ((16 * c + 8 * (e >> 1) + g) == (8 * n + (e & 1) + 2 * t)) ? s : 0.f;
+    const int blk = lane >> 3, rr = lane & 7;
+#pragma unroll
+    for (int kk = 0; kk < M / 16; ++kk)
+#pragma unroll
+        for (int jp = 0; jp < NT / 2; ++jp) {
+            uint32_t bh[4], bl[4];
+            const unsigned char* ph = mat + ((size_t)(16 * jp + 8 * (blk >> 1) + rr) * SS + 16 * kk + 8 * (blk & 1)) * 2;
+            ldsm_x4(bh, ph);
+            ldsm_x4(bl, ph + DistScratch<M>::PLANE);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int n = 2 * jp + h;
+#pragma unroll
+                for (int a = 0; a < NA; ++a) {
+                    const H2Pair* Ak = A[a][kk];
+                    const uint32_t ahi[4] = {Ak[0].hi, Ak[1].hi, Ak[2].hi, Ak[3].hi};
+                    const uint32_t alo[4] = {Ak[0].lo, Ak[1].lo, Ak[2].lo, Ak[3].lo};
+                    H::k16(acc[a][n], alo, bh[2 * h], bh[2 * h + 1]);
+                    H::k16(acc[a][n], ahi, bl[2 * h], bl[2 * h + 1]);
+                    H::k16(acc[a][n], ahi, bh[2 * h], bh[2 * h + 1]);
+                }
+                if (CI && kk == c) {
+                    const uint32_t ci[4] = {i7, 0u, 0u, i7};
+                    H::k16(acc[0][n], ci, bl[2 * h], bl[2 * h + 1]);
+                    H::k16(acc[0][n], ci, bh[2 * h], bh[2 * h + 1]);
+                }
+            }
+        }
+}
+
+// Core on CW = M/16 warps (warp c of them calls with its index; bar_id is a
+// named barrier reserved for these warps; mat0, mat1, aux: DistScratch
+// areas): G_A^n from the landmarks and m_U (gmu, log2 domain), the iteration
+// of step 4, Y = Z W (W: fp32, row stride NCOL + 4 at mW) stored as Y^T at
+// yT.  Same arithmetic as core_warp.
+template <typename T, int M, int NCOL>
+__device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const float* gmu, const float* mW, T* yT,
+                                          unsigned char* mat0, unsigned char* mat1, float* aux, int iters, float sl2,
+                                          int c, int lane, int bar_id) {
+    using S = DistScratch<M>;
+    using Op = Mma16<T>;
+    constexpr int CW = S::CW, KT = M / 16, NT = M / 8, LS = 40, WS = NCOL + 4, NTO = NCOL / 8, YS = M + 8;
+    const int g = lane >> 2, t = lane & 3;
+    unsigned char* cur = mat0;
+    unsigned char* oth = mat1;
+    float* cols = aux;                // [CW][M] column-sum partials
+    float* slots = aux + CW * M;      // [3][CW] maxima
+    auto csync = [&]() { named_barrier(bar_id, CW * 32); };
+    const uint32_t sel = tril_selector(g, t);
+    uint32_t i7;
+    {
+        const __half2 h = __floats2half2_rn(g == 2 * t ? -7.f : 0.f, g == 2 * t + 1 ? -7.f : 0.f);
+        i7 = *reinterpret_cast<const uint32_t*>(&h);
+    }
+    H2Pair Xa[KT][4], Za[KT][4];
+    float acc[NT][4], zc[NT][4];
+    // ---- G_A^n, own rows ----
+    {
+        uint32_t aq[2][4];
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const T* r0 = qbar + (16 * c + g) * LS + 16 * kk + 2 * t;
+            aq[kk][0] = ld32(r0);
+            aq[kk][1] = ld32(r0 + 8 * LS);
+            aq[kk][2] = ld32(r0 + 8);
+            aq[kk][3] = ld32(r0 + 8 * LS + 8);
+        }
+        const float mu0 = gmu[16 * c + g], mu1 = gmu[16 * c + g + 8];
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            float sa[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int kk = 0; kk < 2; ++kk) {
+                const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
+                Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+            }
+            acc[n][0] = ex2(fmaf(sa[0], sl2, -mu0));
+            acc[n][1] = ex2(fmaf(sa[1], sl2, -mu0));
+            acc[n][2] = ex2(fmaf(sa[2], sl2, -mu1));
+            acc[n][3] = ex2(fmaf(sa[3], sl2, -mu1));
+        }
+    }
+    // ---- ||A||_inf, ||A||_1 (A > 0) and A into scratch ----
+    {
+        float r0 = 0.f, r1 = 0.f;
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+            r0 += acc[n][0] + acc[n][1];
+            r1 += acc[n][2] + acc[n][3];
+        }
+        r0 += __shfl_xor_sync(0xffffffffu, r0, 1);
+        r0 += __shfl_xor_sync(0xffffffffu, r0, 2);
+        r1 += __shfl_xor_sync(0xffffffffu, r1, 1);
+        r1 += __shfl_xor_sync(0xffffffffu, r1, 2);
+        const float rm = warp_max_nonneg(fmaxf(r0, r1));
+        if (lane == 0) slots[c] = rm;
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                float cs = acc[n][e] + acc[n][e + 2];
+                cs += __shfl_xor_sync(0xffffffffu, cs, 4);
+                cs += __shfl_xor_sync(0xffffffffu, cs, 8);
+                cs += __shfl_xor_sync(0xffffffffu, cs, 16);
+                if (g == 0) cols[c * M + 8 * n + 2 * t + e] = cs;
+            }
+    }
+    dist_put<M>(cur, acc, 1.f, c, g, t);  // A
+    csync();
+    float alpha;
+    {
+        float rmax = 0.f, cmax = 0.f;
+#pragma unroll
+        for (int w = 0; w < CW; ++w) rmax = fmaxf(rmax, slots[w]);
+        for (int col = lane; col < M; col += 32) {
+            float cs = 0.f;
+#pragma unroll
+            for (int w = 0; w < CW; ++w) cs += cols[w * M + col];
+            cmax = fmaxf(cmax, cs);
+        }
+        alpha = 1.f / (rmax * warp_max_nonneg(cmax));
+    }
+    {
+        H2Pair Aa[KT][4];
+#pragma unroll
+        for (int kk = 0; kk < KT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int n = 2 * kk + (r >> 1), e = 2 * (r & 1);
+                Aa[kk][r] = split_h2(acc[n][e], acc[n][e + 1]);
+            }
+        const H2Pair(*const As[1])[4] = {Aa};
+        float(*const Ds[1])[4] = {acc};
+        dist_mm<M, 1, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // A A^T
+    }
+    dist_load_a<M, true>(cur, Za, c, lane);  // Z_0 = A^T (a dropped)
+    dist_put_sym<M>(oth, acc, alpha, c, g, t, sel);  // X_0 = a A A^T
+    csync();
+    dist_load_a<M, false>(oth, Xa, c, lane);
+    {
+        unsigned char* tmp = cur;
+        cur = oth;
+        oth = tmp;
+    }
+    if (iters == 0) {
+#pragma unroll
+        for (int kk = 0; kk < KT; ++kk)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const uint32_t hb = Za[kk][r].hi, lb = Za[kk][r].lo;
+                const float2 h = __half22float2(*reinterpret_cast<const __half2*>(&hb));
+                const float2 l = __half22float2(*reinterpret_cast<const __half2*>(&lb));
+                const int n = 2 * kk + (r >> 1), e = 2 * (r & 1);
+                zc[n][e] = h.x + l.x;
+                zc[n][e + 1] = h.y + l.y;
+            }
+    }
+    // ---- iteration (step 4): X in cur ----
+#pragma unroll 1
+    for (int it = 0; it < iters; ++it) {
+        {
+            const H2Pair(*const As[1])[4] = {Xa};
+            float(*const Ds[1])[4] = {acc};
+            dist_mm<M, 1, true>(As, cur, Ds, 15.f, i7, c, g, t, lane);  // T2 = 15I - 7X + X X
+        }
+        dist_put<M>(oth, acc, -0.25f, c, g, t);  // -T2/4
+        csync();
+        {
+            const H2Pair(*const As[1])[4] = {Xa};
+            float(*const Ds[1])[4] = {acc};
+            dist_mm<M, 1, false>(As, oth, Ds, 3.25f, 0u, c, g, t, lane);  // T3/4
+        }
+        dist_put<M>(cur, acc, 1.f, c, g, t);  // every warp is done with X
+        csync();
+        if (it + 1 < iters) {
+            const H2Pair(*const As[2])[4] = {Za, Xa};
+            float(*const Ds[2])[4] = {zc, acc};
+            dist_mm<M, 2, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // Z T3/4, X T3/4
+            dist_put_sym<M>(oth, acc, 1.f, c, g, t, sel);            // every warp is done with -T2/4
+            float zm = 0.f;
+#pragma unroll
+            for (int n = 0; n < NT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) zm = fmaxf(zm, fabsf(zc[n][e]));
+            zm = warp_max_nonneg(zm);
+            if (lane == 0) slots[CW + c] = zm;
+            csync();
+            dist_load_a<M, false>(oth, Xa, c, lane);
+            unsigned char* tmp = cur;
+            cur = oth;
+            oth = tmp;
+            float zmax = 0.f;
+#pragma unroll
+            for (int w = 0; w < CW; ++w) zmax = fmaxf(zmax, slots[CW + w]);
+            const float sc = (zmax > 0.f && zmax < INFINITY) ? ldexpf(1.f, 10 - ilogbf(zmax)) : 1.f;
+#pragma unroll
+            for (int kk = 0; kk < KT; ++kk)
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    const int n = 2 * kk + (r >> 1), e = 2 * (r & 1);
+                    Za[kk][r] = split_h2(sc * zc[n][e], sc * zc[n][e + 1]);
+                }
+        } else {
+            const H2Pair(*const As[1])[4] = {Za};
+            float(*const Ds[1])[4] = {zc};
+            dist_mm<M, 1, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // Z T3/4
+        }
+    }
+    // ---- Y = Z W, own rows (split-tf32), stored as Y^T ----
+    {
+        float y[NTO][4];
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) y[j][0] = y[j][1] = y[j][2] = y[j][3] = 0.f;
+#pragma unroll
+        for (int kk = 0; kk < NT; ++kk) {
+            const uint32_t ah[4] = {__float_as_uint(zc[kk][0]), __float_as_uint(zc[kk][2]), __float_as_uint(zc[kk][1]),
+                                    __float_as_uint(zc[kk][3])};
+            const uint32_t al[4] = {tf32_lo(zc[kk][0]), tf32_lo(zc[kk][2]), tf32_lo(zc[kk][1]), tf32_lo(zc[kk][3])};
+#pragma unroll
+            for (int j = 0; j < NTO; ++j) {
+                const float y0 = mW[(8 * kk + 2 * t) * WS + 8 * j + g];
+                const float y1 = mW[(8 * kk + 2 * t + 1) * WS + 8 * j + g];
+                const uint32_t bh0 = __float_as_uint(y0), bh1 = __float_as_uint(y1);
+                const uint32_t bl0 = tf32_lo(y0), bl1 = tf32_lo(y1);
+                mma_tf32(y[j], al[0], al[1], al[2], al[3], bh0, bh1);
+                mma_tf32(y[j], ah[0], ah[1], ah[2], ah[3], bl0, bl1);
+                mma_tf32(y[j], ah[0], ah[1], ah[2], ah[3], bh0, bh1);
+            }
+        }
+        float scale = 1.f;
+        if (Op::kNarrowRange) {
+            float ym = 0.f;
+#pragma unroll
+            for (int j = 0; j < NTO; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) ym = fmaxf(ym, fabsf(y[j][e]));
+            ym = warp_max_nonneg(ym);
+            if (lane == 0) slots[2 * CW + c] = ym;
+            csync();
+            float ymax = 0.f;
+#pragma unroll
+            for (int w = 0; w < CW; ++w) ymax = fmaxf(ymax, slots[2 * CW + w]);
+            if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
+        }
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) {
+            const int rr = 16 * c + g, cc = 8 * j + 2 * t;
+            yT[cc * YS + rr] = from_f32<T>(y[j][0] * scale);
+            yT[(cc + 1) * YS + rr] = from_f32<T>(y[j][1] * scale);
+            yT[cc * YS + rr + 8] = from_f32<T>(y[j][2] * scale);
+            yT[(cc + 1) * YS + rr + 8] = from_f32<T>(y[j][3] * scale);
+        }
+    }
+}
+
 // Output for one warp's NCH chunks: O = (G_L^n Y_:d) / (G_L^n Y_d) (steps
 // 5-7); G_L^n fragments come from glf (parked) or are recomputed from Qs and
 // Kbar; rows are written row-major to obase (N_w x d).
@@ -775,25 +1150,28 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
         }
         }
 
-template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS>
-__global__ void __launch_bounds__(GROUPS * WPU * 32, 1)
+template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS, int CW>
+__global__ void __launch_bounds__(GROUPS * Layout<M, NCOL, TPW, WPU, GLS, CW>::GW * 32, 1)
 nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                  T* __restrict__ out, long long n_units, int d, int iters, float sl2,
                  unsigned int* fault, int active) {
-    using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
+    using Lay = Layout<M, NCOL, TPW, WPU, GLS, CW>;
     using Op = Mma16<T>;
     constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS,
-                  WS = Lay::WS, KTL = Lay::KTL;
+                  WS = Lay::WS, KTL = Lay::KTL, GW = Lay::GW;
     constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
     constexpr int LPW = TPW / L;  // landmarks owned by one warp
     static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
+    static_assert(CW == 1 || CW == M / 16, "the distributed core has one warp per 16 landmarks");
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int grp = warp / WPU, r = warp - grp * WPU;
+    const int grp = warp / GW, r = warp - grp * GW;
+    const bool tok = (GW == WPU) || r < WPU;  // token warp (owns TPW tokens); others only help the core
     const int g = lane >> 2, t = lane & 3;
     unsigned char* gb = smem_raw + (size_t)grp * Lay::GROUP_BYTES;
-    unsigned char* wb = smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES + (size_t)warp * Lay::WARP_BYTES;
+    unsigned char* wb = smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
+                        (size_t)(grp * WPU + (r < WPU ? r : WPU - 1)) * Lay::WARP_BYTES;
     const int td = TPW * d;  // elements per staged tensor
     T* Qs = reinterpret_cast<T*>(wb);
     T* Ks = Qs + td;
@@ -810,9 +1188,26 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
     volatile unsigned int* gflag = reinterpret_cast<volatile unsigned int*>(gb + Lay::G_FLAG);
 
     auto gsync = [&]() {
-        if constexpr (WPU == 1) __syncwarp();
-        else named_barrier(1 + grp, WPU * 32);
+        if constexpr (GW == 1) __syncwarp();
+        else named_barrier(1 + grp, GW * 32);
     };
+    // distributed-core scratch
+    unsigned char* mat0 = nullptr;
+    unsigned char* mat1 = nullptr;
+    float* aux = nullptr;
+    if constexpr (CW > 1) {
+        using DSc = DistScratch<(M > 16 ? M : 32)>;
+        if constexpr (Lay::SCR_IN_STAGE) {
+            unsigned char* w0 = smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES + (size_t)(grp * WPU) * Lay::WARP_BYTES;
+            mat0 = w0 + Lay::WPART;
+            aux = reinterpret_cast<float*>(mat0 + DSc::MAT);
+            mat1 = w0 + Lay::WARP_BYTES + Lay::WPART;
+        } else {
+            mat0 = gb + Lay::G_SCR;
+            mat1 = mat0 + DSc::MAT;
+            aux = reinterpret_cast<float*>(mat1 + DSc::MAT);
+        }
+    }
 
     // Only the first `active` groups of a CTA take units (see launch_cfg).
     const long long stride = (long long)gridDim.x * active;
@@ -828,14 +1223,14 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         bulk_g2s(Vs, v + unit_off(unit), tile_bytes, barV);
     };
 
-    if (lane == 0) {
+    if (tok && lane == 0) {
         mbar_init(barQK, 1);
         mbar_init(barV, 1);
         fence_mbar_init();
         if (r == 0) *gflag = 0u;
     }
     gsync();
-    if (u < n_units && lane == 0) {
+    if (tok && u < n_units && lane == 0) {
         arm_qk();
         issue_q(u);
         issue_k(u);
@@ -845,15 +1240,18 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
 
     for (; u < n_units; u += stride) {
         // ---------------- stage: bounded wait for Q and K ----------------
-        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
-        if (!ok && lane == 0) {
-            atomicOr(fault, 1u);
-            *gflag = 1u;  // the whole group stops after the next barrier
+        bool ok = true;
+        if (tok) {
+            ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
+            if (!ok && lane == 0) {
+                atomicOr(fault, 1u);
+                *gflag = 1u;  // the whole group stops after the next barrier
+            }
+            phase_qk ^= 1u;
         }
-        phase_qk ^= 1u;
 
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
-        {
+        if (tok) {
             landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
             landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
             if (M < MP && r == 0) {  // zero the padding landmark rows
@@ -865,10 +1263,10 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             }
         }
         gsync();
-        if (WPU == 1 ? !ok : (*gflag != 0u)) break;
+        if (GW == 1 ? !ok : (*gflag != 0u)) break;
 
         // ---------------- front [P1]: S_L, G_L^n fragments ----------------
-        if constexpr (GLS) {
+        if (GLS && tok) {
 #pragma unroll 1
             for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
@@ -887,71 +1285,92 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         }
 
         // ---------------- stage: bounded wait for V ----------------
-        const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
-        if (!ok_v && lane == 0) {
-            atomicOr(fault, 1u);
-            *gflag = 1u;
+        bool ok_v = true;
+        if (tok) {
+            ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
+            if (!ok_v && lane == 0) {
+                atomicOr(fault, 1u);
+                *gflag = 1u;
+            }
+            phase_v ^= 1u;
         }
-        phase_v ^= 1u;
-        if (WPU == 1 && !ok_v) break;
+        if (GW == 1 && !ok_v) break;
 
         // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
         float mU[MT][2];  // this warp's row maxima of S_U, log2 domain
-        front_su_w<T, M, NCOL, NCH>(qbar, Ks, Vs, d, g, t, sl2, WPU == 1 ? mW : wpart, WPU == 1 ? WS : NCOL, mU);
-        if (WPU > 1 && t == 0) {
+        if (tok) {
+            front_su_w<T, M, NCOL, NCH>(qbar, Ks, Vs, d, g, t, sl2, WPU == 1 ? mW : wpart, WPU == 1 ? WS : NCOL,
+                                        mU);
+            if ((WPU > 1 || CW > 1) && t == 0) {
+                float* mdst = WPU > 1 ? wpart + MP * NCOL : gmu;
 #pragma unroll
-            for (int mt = 0; mt < MT; ++mt) {
-                wpart[MP * NCOL + 16 * mt + g] = mU[mt][0];
-                wpart[MP * NCOL + 16 * mt + g + 8] = mU[mt][1];
+                for (int mt = 0; mt < MT; ++mt) {
+                    mdst[16 * mt + g] = mU[mt][0];
+                    mdst[16 * mt + g + 8] = mU[mt][1];
+                }
             }
         }
 
         // ---------------- combine (WPU > 1) ----------------
         if constexpr (WPU > 1) {
             gsync();
-            combine_partials<MP, NCOL, WS, WPU>(
-                reinterpret_cast<const float*>(smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
-                                               (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART),
-                Lay::WARP_BYTES / 4, mW, gmu, r, lane);
+            if (tok)
+                combine_partials<MP, NCOL, WS, WPU>(
+                    reinterpret_cast<const float*>(smem_raw + (size_t)GROUPS * Lay::GROUP_BYTES +
+                                                   (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART),
+                    Lay::WARP_BYTES / 4, mW, gmu, r, lane);
         }
         gsync();
-        if (WPU > 1 && *gflag != 0u) break;
+        if (GW > 1 && *gflag != 0u) break;
 
         // Q and K of this unit are consumed (in P2 Q stays for the output):
         // prefetch the next unit's rows.  V's region holds the output first.
+        // With the core's scratch in the K/V rows, K waits for the core.
         const long long un = u + stride;
-        fence_proxy_async_smem();  // this lane's reads of Q/K precede the async refill
-        __syncwarp();
-        if (un < n_units && lane == 0) {
-            arm_qk();
-            if constexpr (GLS) issue_q(un);
-            issue_k(un);
-        }
-
-        // ---------------- core (warp 0): G_A^n, Z_0, iteration, Y ----------------
-        if (r == 0) {
-            if constexpr (WPU > 1) {
-#pragma unroll
-                for (int mt = 0; mt < MT; ++mt) {
-                    mU[mt][0] = gmu[16 * mt + g];
-                    mU[mt][1] = gmu[16 * mt + g + 8];
-                }
+        auto prefetch_qk = [&]() {
+            fence_proxy_async_smem();  // this lane's reads of Q/K precede the async refill
+            __syncwarp();
+            if (tok && un < n_units && lane == 0) {
+                arm_qk();
+                if constexpr (GLS) issue_q(un);
+                issue_k(un);
             }
-            core_warp<T, M, NCOL>(qbar, kbar, mU, mW, yT, iters, sl2, g, t);
+        };
+        if constexpr (!Lay::SCR_IN_STAGE) prefetch_qk();
+
+        // ---------------- core: G_A^n, Z_0, iteration, Y ----------------
+        if constexpr (CW == 1) {
+            if (r == 0) {
+                if constexpr (WPU > 1) {
+#pragma unroll
+                    for (int mt = 0; mt < MT; ++mt) {
+                        mU[mt][0] = gmu[16 * mt + g];
+                        mU[mt][1] = gmu[16 * mt + g + 8];
+                    }
+                }
+                core_warp<T, M, NCOL>(qbar, kbar, mU, mW, yT, iters, sl2, g, t);
+            }
+        } else {
+            if (r < CW)
+                dist_core<T, (M > 16 ? M : 32), NCOL>(qbar, kbar, gmu, mW, yT, mat0, mat1, aux, iters, sl2, r, lane,
+                                                      1 + GROUPS + grp);
         }
         gsync();
+        if constexpr (Lay::SCR_IN_STAGE) prefetch_qk();
 
-        // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
-        output_rows<T, M, NCOL, NCH, GLS>(glf, Qs, kbar, yT, Vs, d, g, t, lane, sl2);
+        if (tok) {
+            // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
+            output_rows<T, M, NCOL, NCH, GLS>(glf, Qs, kbar, yT, Vs, d, g, t, lane, sl2);
 
-        // The output rows are staged in V's region: one bulk store, and once it
-        // has read shared memory, the next unit's V can land there.
-        fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
-        __syncwarp();
-        if (lane == 0) {
-            bulk_s2g(out + unit_off(u), Vs, tile_bytes);
-            bulk_commit();
-            bulk_wait_read_all();
+            // The output rows are staged in V's region: one bulk store, and once it
+            // has read shared memory, the next unit's V can land there.
+            fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
+            __syncwarp();
+            if (lane == 0) {
+                bulk_s2g(out + unit_off(u), Vs, tile_bytes);
+                bulk_commit();
+                bulk_wait_read_all();
+            }
         }
         // [P2] Q was needed until now: every warp of the group is done reading
         // the landmarks before anyone overwrites them.
@@ -959,34 +1378,38 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             fence_proxy_async_smem();  // reads of Q precede its refill
             gsync();
         }
-        if (un < n_units && lane == 0) {
+        if (tok && un < n_units && lane == 0) {
             if constexpr (!GLS) issue_q(un);
             issue_v(un);
         }
         __syncwarp();
     }
-    if (lane == 0) bulk_wait_all();  // outstanding output stores complete before exit
+    if (tok && lane == 0) bulk_wait_all();  // outstanding output stores complete before exit
 }
 
 // Largest number of groups per CTA that fits the shared-memory and register
 // budgets (M <= 16 needs about 160 registers per thread, M = 32 about 255).
-template <int M, int NCOL, int TPW, int WPU, bool GLS>
+template <int M, int NCOL, int TPW, int WPU, bool GLS, int CW>
 constexpr int groups_that_fit() {
-    using Lay = Layout<M, NCOL, TPW, WPU, GLS>;
+    using Lay = Layout<M, NCOL, TPW, WPU, GLS, CW>;
     const int by_smem = (int)(kSmemLimit / Lay::PER_GROUP);
-    const int by_regs = ((M <= 16) ? 12 : 8) / WPU;
+    const int by_regs = ((M <= 16) ? 12 : 8) / Lay::GW;
     const int n = by_smem < by_regs ? by_smem : by_regs;
-    return n > 15 ? 15 : n;
+    const int cap = (CW > 1) ? 7 : 15;  // named barriers: 1 + group barriers + core barriers <= 16
+    return n > cap ? cap : n;
 }
 
-template <typename T, int M, int NCOL, int TPW, int WPU>
+template <typename T, int M, int NCOL, int TPW, int WPU, int CW = 1>
 cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                        int iters, cudaStream_t stream, unsigned int* fault) {
-    constexpr bool kGls = groups_that_fit<M, NCOL, TPW, WPU, true>() >= 1;
-    constexpr int kGroups = groups_that_fit<M, NCOL, TPW, WPU, kGls>();
+    // G_L^n parked (P1) unless recomputing it (P2) fits more groups.
+    constexpr int kG1 = groups_that_fit<M, NCOL, TPW, WPU, true, CW>();
+    constexpr int kG2 = groups_that_fit<M, NCOL, TPW, WPU, false, CW>();
+    constexpr bool kGls = kG1 >= 1 && kG1 >= kG2;
+    constexpr int kGroups = kGls ? kG1 : kG2;
     static_assert(kGroups >= 1, "configuration does not fit on one SM");
-    using Lay = Layout<M, NCOL, TPW, WPU, kGls>;
-    auto kern = nystra_tc_kernel<T, M, NCOL, TPW, WPU, kGroups, kGls>;
+    using Lay = Layout<M, NCOL, TPW, WPU, kGls, CW>;
+    auto kern = nystra_tc_kernel<T, M, NCOL, TPW, WPU, kGroups, kGls, CW>;
     const size_t smem = (size_t)kGroups * Lay::PER_GROUP;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -995,7 +1418,7 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
         int dev = 0, sms = 0, per_sm = 0;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
         if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGroups * WPU * 32, smem)) !=
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGroups * Lay::GW * 32, smem)) !=
             cudaSuccess)
             return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
@@ -1011,8 +1434,8 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
     const long long want = (n_units + active - 1) / active;
     const long long grid = want < blocks ? want : blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
-    kern<<<(unsigned)grid, kGroups * WPU * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
-                                                              n_units, d, iters, sl2, fault, active);
+    kern<<<(unsigned)grid, kGroups * Lay::GW * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v,
+                                                                  (T*)out, n_units, d, iters, sl2, fault, active);
     return cudaGetLastError();
 }
 
@@ -1054,9 +1477,20 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
         case 16:
             return wide ? launch_cfg<T, 16, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_cfg<T, 16, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
-        default:
-            return wide ? launch_cfg<T, 32, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_cfg<T, 32, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
+        case 32: {
+            // several token warps: the core is split over two of them
+            constexpr int CW = WPU >= 2 ? 2 : 1;
+            return wide ? launch_cfg<T, 32, 40, TPW, WPU, CW>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 32, 32, TPW, WPU, CW>(q, k, v, out, n_units, d, iters, stream, fault);
+        }
+        default: {
+            // m = 64: the core on four warps; W partials of 64 rows need K/V
+            // rows of at least 128 tokens per token warp.
+            constexpr int TP = (TPW * WPU == 64) ? 64 : (TPW * WPU == 256) ? 128 : 256;
+            constexpr int WP = TPW * WPU / TP;
+            return wide ? launch_cfg<T, 64, 40, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 64, 32, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault);
+        }
     }
 }
 
