@@ -32,19 +32,20 @@ from paper_2506_08520_gb300 import binding, workloads  # noqa: E402
 METRIC = "Nystrom attention tokens*heads/s"
 
 # DRAM bytes (read + write) per launch from one ncu capture (profiles/), valid only
-# for the kernel sources they were taken with: reported as null once they change.
+# for the sources of the kernel they were taken with: reported as null once any
+# of those files changes.
 MEASURED_TRAFFIC = {
-    "swinir256-bf16": {"src_hash": "9ec59d17e4a3e9dd", "bytes": 74_096_640},
+    "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
+                       "src_hash": "4210bd8380471295", "bytes": 74_102_784},
 }
 
 
-def _kernel_src_hash() -> str:
-    import glob
+def _kernel_src_hash(files) -> str:
     import hashlib
     h = hashlib.sha256()
-    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2506_08520_gb300", "csrc", "*.cu*"))):
-        h.update(os.path.basename(f).encode())
-        with open(f, "rb") as fh:
+    for name in sorted(files):
+        h.update(name.encode())
+        with open(os.path.join(ROOT, "paper_2506_08520_gb300", "csrc", name), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 UNIT = "tokens*heads/s"
@@ -280,11 +281,11 @@ def run_cuda(args, wl):
     peak, peak_kind = _peaks()
     achieved = io_bytes / (kern_ms * 1e-3) / 1e9
     mt = MEASURED_TRAFFIC.get(wl.name)
-    traffic = mt["bytes"] if mt and mt["src_hash"] == _kernel_src_hash() else None
+    traffic = mt["bytes"] if mt and mt["src_hash"] == _kernel_src_hash(mt["files"]) else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
         "config": {"workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N,
                    "d_h": wl.d, "m": wl.m, "iters": wl.iters, "io_dtype": wl.dtype,
                    "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
