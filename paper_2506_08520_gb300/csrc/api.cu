@@ -50,8 +50,12 @@ int nystra_attention(const void* q, const void* k, const void* v, void* out, int
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
     const cudaStream_t s = (cudaStream_t)stream;
-    const bool tc = (dtype == NYSTRA_BF16 || dtype == NYSTRA_F16) && d_h % 2 == 0 && d_h <= 32 &&
-                    (m == 8 || m == 16 || m == 32 || m == 64);
+    // fp32 I/O on the tensor cores: 8x8 windows, m <= 16, at most the paper's 6
+    // iterations (beyond them the fp16-split iteration's round-off, amplified
+    // by ||G_A^n|| ||Z||, exceeds what fp32 I/O asks; the SIMT path iterates in fp32).
+    const bool tc16 = (dtype == NYSTRA_BF16 || dtype == NYSTRA_F16) && (m == 8 || m == 16 || m == 32 || m == 64);
+    const bool tc32 = dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
+    const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32;
     cudaError_t e;
     if (tc && N == 64)
         e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, dtype, s);

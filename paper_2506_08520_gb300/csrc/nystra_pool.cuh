@@ -1,13 +1,14 @@
 // Stage-pool PnP-Nystra kernel for 8x8 windows (N = 64 tokens), m <= 16,
-// even d_h <= 32, 16-bit I/O.  Included by the N = 64 translation unit after
-// nystra_tc.cuh, whose per-phase device functions it reuses.
+// even d_h <= 32, 16-bit or fp32 I/O (fp32: split bf16 operands, see Opnd).
+// Included by the N = 64 translation unit after nystra_tc.cuh, whose
+// per-phase device functions it reuses.
 //
 // One warp processes one (window, head) unit at a time, as the grouped
 // kernel does with one warp per unit, but a warp's Q, K and V rows are only
 // needed by its front phase (landmarks, S_L and G_L^n, S_U and W), while the
 // core (m x m iteration) and the output phase run on warp-private state.  A
-// CTA therefore keeps NW = 16 warps on NS = 8 shared staging buffers instead
-// of one buffer per warp: warp w always uses stage w mod NS, alternating with
+// CTA therefore keeps NW = 16 warps on NS = 8 shared staging buffers (8 on 4
+// for fp32 I/O) instead of one buffer per warp: warp w always uses stage w mod NS, alternating with
 // its partner warp (w + NS) mod NW.  When a warp's front phase has consumed
 // the stage it issues the bulk copies of the partner's next unit into it, so
 // the copy overlaps the warp's own core and output.  Each warp waits on its
@@ -27,24 +28,25 @@
 namespace nystra {
 namespace tc {
 
-template <int M, int NCOL>
+template <typename T, int M, int NCOL>
 struct PoolLayout {
-    static constexpr int NW = 16, NS = 8;              // warps, shared stages
+    static constexpr int ES = (int)sizeof(T);          // bytes per I/O element
+    static constexpr int NW = ES == 2 ? 16 : 8;        // warps
+    static constexpr int NS = NW / 2;                  // shared stages
     static constexpr int DS = (NCOL == 32) ? 30 : 32;  // staged row width bound (d_h <= DS)
     static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;  // k-steps of O = G_L^n Y
-    static constexpr int GLB = (M >= 16) ? 16 : 8;      // bytes per lane per G_L fragment
-    static constexpr size_t STAGE = 3 * 64 * DS * 2;    // Q, K, V rows of one unit
+    static constexpr size_t STAGE = 3 * 64 * DS * ES;   // Q, K, V rows of one unit
     // warp-private layout
     static constexpr size_t GLF = 0;
-    static constexpr size_t QB = GLF + 4 * KTL * 32 * GLB;
-    static constexpr size_t KB = QB + MP * LS * 2;
-    static constexpr size_t W = KB + MP * LS * 2;  // fp32 MP x NCOL, row stride WS
-    static constexpr size_t YT = QB;               // Y^T: written after the core's last landmark read
-    static constexpr size_t YT_BYTES = ((NCOL * YS * 2 + 15) / 16) * 16;
+    static constexpr size_t QB = GLF + 4 * KTL * 32 * GlPark<T, M>::BYTES;
+    static constexpr size_t KB = QB + MP * LS * ES;
+    static constexpr size_t W = KB + MP * LS * ES;  // fp32 MP x NCOL, row stride WS
+    static constexpr size_t YT = QB;                // Y^T: written after the core's last landmark read
+    static constexpr size_t YT_BYTES = ((NCOL * YS * ES + 15) / 16) * 16;
     static constexpr size_t OUT = YT + YT_BYTES;  // output tile: Kbar's tail and W are dead by then
     static constexpr size_t END_A = W + MP * WS * 4;
-    static constexpr size_t END_B = OUT + 64 * DS * 2;
+    static constexpr size_t END_B = OUT + 64 * DS * ES;
     static constexpr size_t BAR = (((END_A > END_B) ? END_A : END_B) + 15) / 16 * 16;
     static constexpr size_t CNT = BAR + 8;  // copies issued to this warp (fault path)
     static constexpr size_t PRIV = ((BAR + 16 + 127) / 128) * 128;
@@ -56,10 +58,10 @@ struct PoolLayout {
 };
 
 template <typename T, int M, int NCOL>
-__global__ void __launch_bounds__(PoolLayout<M, NCOL>::NW * 32, 1)
+__global__ void __launch_bounds__(PoolLayout<T, M, NCOL>::NW * 32, 1)
 nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, T* __restrict__ out,
                    long long n_units, int d, int iters, float sl2, unsigned int* fault) {
-    using P = PoolLayout<M, NCOL>;
+    using P = PoolLayout<T, M, NCOL>;
     constexpr int L = 64 / M;  // tokens per landmark segment
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -120,26 +122,20 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         landmarks_mma<T, 64, L>(Qs, qbar, 0, d, g, t);
         landmarks_mma<T, 64, L>(Ks, kbar, 0, d, g, t);
         if constexpr (M < P::MP) {  // zero the padding landmark rows
-            for (int idx = lane; idx < (P::MP - M) * 16; idx += 32) {
-                const int jr = M + (idx >> 4), p = idx & 15;
-                *reinterpret_cast<uint32_t*>(qbar + jr * P::LS + 2 * p) = 0u;
-                *reinterpret_cast<uint32_t*>(kbar + jr * P::LS + 2 * p) = 0u;
+            for (int idx = lane; idx < (P::MP - M) * 32; idx += 32) {
+                const int jr = M + (idx >> 5), e = idx & 31;
+                qbar[jr * P::LS + e] = from_f32<T>(0.f);
+                kbar[jr * P::LS + e] = from_f32<T>(0.f);
             }
         }
         __syncwarp();
         // ---------------- front: S_L, G_L^n fragments (parked) ----------------
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
-            uint32_t f[P::KTL][4];
+            typename Opnd<T>::Reg f[P::KTL][4];
             gl_tile<T, M, P::KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
-            for (int kk = 0; kk < P::KTL; ++kk) {
-                const int slot = (tm * P::KTL + kk) * 32 + lane;
-                if constexpr (M >= 16)
-                    reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[kk][0], f[kk][1], f[kk][2], f[kk][3]);
-                else
-                    reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[kk][0], f[kk][1]);
-            }
+            for (int kk = 0; kk < P::KTL; ++kk) GlPark<T, M>::put(glf, (tm * P::KTL + kk) * 32 + lane, f[kk]);
         }
         // ---------------- front: S_U, m_U, W = G_U^n [V | 1] ----------------
         float mU[1][2];
@@ -172,7 +168,7 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 template <typename T, int M, int NCOL>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault) {
-    using P = PoolLayout<M, NCOL>;
+    using P = PoolLayout<T, M, NCOL>;
     auto kern = nystra_pool_kernel<T, M, NCOL>;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {

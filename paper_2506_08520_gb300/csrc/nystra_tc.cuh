@@ -333,18 +333,19 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
 // fragments (A operand of O = G_L^n Y, k = landmarks).
 template <typename T, int M, int KTL>
 __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g, int t, float sl2,
-                                        uint32_t (&f)[KTL][4]) {
-    using Op = Mma16<T>;
+                                        typename Opnd<T>::Reg (&f)[KTL][4]) {
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int NTL = M / 8, LS = 40;
-    uint32_t a[2][4];
+    R a[2][4];
     const T* q1 = q0 + 8 * d;
 #pragma unroll
     for (int kk = 0; kk < 2; ++kk) {
         const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-        a[kk][0] = c0 < d ? ld32(q0 + c0) : 0u;
-        a[kk][1] = c0 < d ? ld32(q1 + c0) : 0u;
-        a[kk][2] = c1 < d ? ld32(q0 + c1) : 0u;
-        a[kk][3] = c1 < d ? ld32(q1 + c1) : 0u;
+        a[kk][0] = c0 < d ? O::ld(q0 + c0) : O::zero();
+        a[kk][1] = c0 < d ? O::ld(q1 + c0) : O::zero();
+        a[kk][2] = c1 < d ? O::ld(q0 + c1) : O::zero();
+        a[kk][3] = c1 < d ? O::ld(q1 + c1) : O::zero();
     }
     float sl[NTL][4];
 #pragma unroll
@@ -353,7 +354,7 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const T* kr = kbar + (8 * j + g) * LS + 16 * kk + 2 * t;
-            Op::k16(sl[j], a[kk], ld32(kr), ld32(kr + 8));
+            O::mma(sl[j], a[kk], O::ld(kr), O::ld(kr + 8));
         }
     }
     float mx0 = -INFINITY, mx1 = -INFINITY;
@@ -369,17 +370,61 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
     if constexpr (M >= 16) {
 #pragma unroll
         for (int kk = 0; kk < KTL; ++kk) {
-            f[kk][0] = Op::pack(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
-            f[kk][1] = Op::pack(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
-            f[kk][2] = Op::pack(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
-            f[kk][3] = Op::pack(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
+            f[kk][0] = O::pk(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
+            f[kk][1] = O::pk(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
+            f[kk][2] = O::pk(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
+            f[kk][3] = O::pk(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
         }
     } else {
-        f[0][0] = Op::pack(e0(sl[0][0]), e0(sl[0][1]));
-        f[0][1] = Op::pack(e1(sl[0][2]), e1(sl[0][3]));
-        f[0][2] = f[0][3] = 0u;
+        f[0][0] = O::pk(e0(sl[0][0]), e0(sl[0][1]));
+        f[0][1] = O::pk(e1(sl[0][2]), e1(sl[0][3]));
+        f[0][2] = f[0][3] = O::zero();
     }
 }
+
+// Parked G_L^n fragments: per lane and 16-token tile, KTL x 4 operand
+// registers (m >= 16) or 2 (m = 8), one or two 16-byte vectors.
+template <typename T, int M>
+struct GlPark {
+    using R = typename Opnd<T>::Reg;
+    static constexpr int REGS = (M >= 16) ? 4 : 2;                   // registers per k-step
+    static constexpr int BYTES = REGS * (int)sizeof(R);               // per lane per k-step
+    static __device__ __forceinline__ void put(uint32_t* glf, int slot, const R (&f)[4]) {
+        if constexpr (sizeof(R) == 4) {
+            if constexpr (M >= 16)
+                reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[0], f[1], f[2], f[3]);
+            else
+                reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[0], f[1]);
+        } else {
+            if constexpr (M >= 16) {
+                reinterpret_cast<uint4*>(glf)[2 * slot] = make_uint4(f[0].hi, f[1].hi, f[2].hi, f[3].hi);
+                reinterpret_cast<uint4*>(glf)[2 * slot + 1] = make_uint4(f[0].lo, f[1].lo, f[2].lo, f[3].lo);
+            } else {
+                reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[0].hi, f[1].hi, f[0].lo, f[1].lo);
+            }
+        }
+    }
+    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, R (&f)[4]) {
+        if constexpr (sizeof(R) == 4) {
+            if constexpr (M >= 16) {
+                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+                f[0] = x.x; f[1] = x.y; f[2] = x.z; f[3] = x.w;
+            } else {
+                const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
+                f[0] = x.x; f[1] = x.y; f[2] = f[3] = 0u;
+            }
+        } else {
+            if constexpr (M >= 16) {
+                const uint4 h = reinterpret_cast<const uint4*>(glf)[2 * slot];
+                const uint4 l = reinterpret_cast<const uint4*>(glf)[2 * slot + 1];
+                f[0] = {h.x, l.x}; f[1] = {h.y, l.y}; f[2] = {h.z, l.z}; f[3] = {h.w, l.w};
+            } else {
+                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+                f[0] = {x.x, x.z}; f[1] = {x.y, x.w}; f[2] = f[3] = Opnd<T>::zero();
+            }
+        }
+    }
+};
 
 // Landmark means of the segments one warp owns (Algorithm 1 step 1) on the
 // tensor cores: xbar = P X with the averaging matrix P (P[j][t] = 1/L when
@@ -390,12 +435,12 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
 // columns >= d come out as zeros.
 template <typename T, int TPW, int L>
 __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
-    using Op = Mma16<T>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int LPW = TPW / L;            // segments owned by the warp
     constexpr int MTL = (LPW + 15) / 16;    // m-tiles of landmark rows
     constexpr int LS = 40;
-    // 1/L in the I/O type, as the low / high half of a 32-bit register
-    const uint32_t inv = Op::pack(1.f / (float)L, 0.f) & 0xffffu;
+    constexpr float inv = 1.f / (float)L;
     float c[MTL][4][4];
 #pragma unroll
     for (int ml = 0; ml < MTL; ++ml)
@@ -405,16 +450,16 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
     for (int ks = 0; ks < TPW / 16; ++ks) {  // 16 tokens per k-step
         const int ml = (16 * ks / L) / 16;   // the one m-tile these tokens feed
         // A = P rows 16 ml + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
-        auto pv = [&](int row, int tok) -> uint32_t { return (tok / L == row) ? inv : 0u; };
+        auto pv = [&](int row, int tok) -> float { return (tok / L == row) ? inv : 0.f; };
         const int r0 = 16 * ml + g, r1 = r0 + 8, k0 = 16 * ks + 2 * t;
-        const uint32_t a[4] = {pv(r0, k0) | (pv(r0, k0 + 1) << 16), pv(r1, k0) | (pv(r1, k0 + 1) << 16),
-                               pv(r0, k0 + 8) | (pv(r0, k0 + 9) << 16), pv(r1, k0 + 8) | (pv(r1, k0 + 9) << 16)};
+        const R a[4] = {O::pk(pv(r0, k0), pv(r0, k0 + 1)), O::pk(pv(r1, k0), pv(r1, k0 + 1)),
+                        O::pk(pv(r0, k0 + 8), pv(r0, k0 + 9)), O::pk(pv(r1, k0 + 8), pv(r1, k0 + 9))};
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
             const int c0 = 8 * b + 2 * t;
-            const uint32_t x0 = c0 < d ? ld32(X + (16 * ks + g) * d + c0) : 0u;
-            const uint32_t x1 = c0 < d ? ld32(X + (16 * ks + 8 + g) * d + c0) : 0u;
-            Op::k16(c[ml][b], a, movmatrix_trans(x0), movmatrix_trans(x1));
+            const R x0 = c0 < d ? O::ld(X + (16 * ks + g) * d + c0) : O::zero();
+            const R x1 = c0 < d ? O::ld(X + (16 * ks + 8 + g) * d + c0) : O::zero();
+            O::mma(c[ml][b], a, O::tr(x0), O::tr(x1));
         }
     }
 #pragma unroll
@@ -422,10 +467,8 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 #pragma unroll
         for (int b = 0; b < 4; ++b) {
             const int row = 16 * ml + g, col = 8 * b + 2 * t;
-            if (row < LPW)
-                *reinterpret_cast<uint32_t*>(xbar + (j0 + row) * LS + col) = Op::pack(c[ml][b][0], c[ml][b][1]);
-            if (row + 8 < LPW)
-                *reinterpret_cast<uint32_t*>(xbar + (j0 + row + 8) * LS + col) = Op::pack(c[ml][b][2], c[ml][b][3]);
+            if (row < LPW) O::st2(xbar + (j0 + row) * LS + col, c[ml][b][0], c[ml][b][1]);
+            if (row + 8 < LPW) O::st2(xbar + (j0 + row + 8) * LS + col, c[ml][b][2], c[ml][b][3]);
         }
 }
 
@@ -439,19 +482,20 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 template <typename T, int M, int NCOL, int NCH>
 __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
                                            float* dst, int ws, float (&mU)[(M + 15) / 16][2]) {
-    using Op = Mma16<T>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int MT = (M + 15) / 16, LS = 40, NTO = NCOL / 8;
     float wall[MT][NTO][4];
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
-        uint32_t aq[2][4];
+        R aq[2][4];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-            aq[kk][0] = ld32(r0);
-            aq[kk][1] = ld32(r0 + 8 * LS);
-            aq[kk][2] = ld32(r0 + 8);
-            aq[kk][3] = ld32(r0 + 8 * LS + 8);
+            aq[kk][0] = O::ld(r0);
+            aq[kk][1] = O::ld(r0 + 8 * LS);
+            aq[kk][2] = O::ld(r0 + 8);
+            aq[kk][3] = O::ld(r0 + 8 * LS + 8);
         }
         const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
         float(&w)[NTO][4] = wall[mt];
@@ -470,9 +514,9 @@ __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* 
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) {
                     const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-                    const uint32_t b0 = c0 < d ? ld32(kr + c0) : 0u;
-                    const uint32_t b1 = c1 < d ? ld32(kr + c1) : 0u;
-                    Op::k16(s[nt], aq[kk], b0, b1);
+                    const R b0 = c0 < d ? O::ld(kr + c0) : O::zero();
+                    const R b1 = c1 < d ? O::ld(kr + c1) : O::zero();
+                    O::mma(s[nt], aq[kk], b0, b1);
                 }
             }
             float mx0 = run0, mx1 = run1;
@@ -497,17 +541,17 @@ __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* 
             // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
 #pragma unroll
             for (int kt = 0; kt < 4; ++kt) {
-                uint32_t a[4];
-                a[0] = v0 ? Op::pack(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : 0u;
-                a[1] = v1 ? Op::pack(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : 0u;
-                a[2] = v0 ? Op::pack(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : 0u;
-                a[3] = v1 ? Op::pack(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : 0u;
+                R a[4];
+                a[0] = v0 ? O::pk(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : O::zero();
+                a[1] = v1 ? O::pk(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : O::zero();
+                a[2] = v0 ? O::pk(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : O::zero();
+                a[3] = v1 ? O::pk(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : O::zero();
 #pragma unroll
                 for (int j = 0; j < NTO; ++j) {
                     const int c0 = 8 * j + 2 * t;
-                    const uint32_t x0 = c0 < d ? ld32(Vc + (16 * kt + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                    const uint32_t x1 = c0 < d ? ld32(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                    Op::k16(w[j], a, movmatrix_trans(x0), movmatrix_trans(x1));
+                    const R x0 = c0 < d ? O::ld(Vc + (16 * kt + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+                    const R x1 = c0 < d ? O::ld(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+                    O::mma(w[j], a, O::tr(x0), O::tr(x1));
                 }
             }
         }
@@ -562,7 +606,8 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
 template <typename T, int M, int NCOL>
 __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const float (&mU)[(M + 15) / 16][2],
                                           const float* mW, T* yT, int iters, float sl2, int g, int t) {
-    using Op = Mma16<T>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int MT = (M + 15) / 16, LS = 40, WS = NCOL + 4, NTO = NCOL / 8;
     constexpr int YS = (M < 16 ? 16 : M) + 8;
     const uint32_t sel = tril_selector(g, t);
@@ -577,14 +622,14 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
         Frag<MT> Ac;
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-            uint32_t aq[2][4];
+            R aq[2][4];
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
                 const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-                aq[kk][0] = ld32(r0);
-                aq[kk][1] = ld32(r0 + 8 * LS);
-                aq[kk][2] = ld32(r0 + 8);
-                aq[kk][3] = ld32(r0 + 8 * LS + 8);
+                aq[kk][0] = O::ld(r0);
+                aq[kk][1] = O::ld(r0 + 8 * LS);
+                aq[kk][2] = O::ld(r0 + 8);
+                aq[kk][3] = O::ld(r0 + 8 * LS + 8);
             }
 #pragma unroll
             for (int n = 0; n < 2 * MT; ++n) {
@@ -592,7 +637,7 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) {
                     const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
-                    Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                    O::mma(sa, aq[kk], O::ld(kr), O::ld(kr + 8));
                 }
                 const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
                 Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
@@ -702,7 +747,7 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
         // Numerator and denominator columns share the factor, so it cancels
         // in step 7.
         float scale = 1.f;
-        if (Op::kNarrowRange) {
+        if (O::kNarrowRange) {
             float ymax = 0.f;
 #pragma unroll
             for (int i = 0; i < MT; ++i)
@@ -862,7 +907,8 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
                                           unsigned char* mat0, unsigned char* mat1, float* aux, int iters, float sl2,
                                           int c, int lane, int bar_id) {
     using S = DistScratch<M>;
-    using Op = Mma16<T>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int CW = S::CW, KT = M / 16, NT = M / 8, LS = 40, WS = NCOL + 4, NTO = NCOL / 8, YS = M + 8;
     const int g = lane >> 2, t = lane & 3;
     unsigned char* cur = mat0;
@@ -880,14 +926,14 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
     float acc[NT][4], zc[NT][4];
     // ---- G_A^n, own rows ----
     {
-        uint32_t aq[2][4];
+        R aq[2][4];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const T* r0 = qbar + (16 * c + g) * LS + 16 * kk + 2 * t;
-            aq[kk][0] = ld32(r0);
-            aq[kk][1] = ld32(r0 + 8 * LS);
-            aq[kk][2] = ld32(r0 + 8);
-            aq[kk][3] = ld32(r0 + 8 * LS + 8);
+            aq[kk][0] = O::ld(r0);
+            aq[kk][1] = O::ld(r0 + 8 * LS);
+            aq[kk][2] = O::ld(r0 + 8);
+            aq[kk][3] = O::ld(r0 + 8 * LS + 8);
         }
         const float mu0 = gmu[16 * c + g], mu1 = gmu[16 * c + g + 8];
 #pragma unroll
@@ -896,7 +942,7 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
                 const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
-                Op::k16(sa, aq[kk], ld32(kr), ld32(kr + 8));
+                O::mma(sa, aq[kk], O::ld(kr), O::ld(kr + 8));
             }
             acc[n][0] = ex2(fmaf(sa[0], sl2, -mu0));
             acc[n][1] = ex2(fmaf(sa[1], sl2, -mu0));
@@ -1052,7 +1098,7 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
             }
         }
         float scale = 1.f;
-        if (Op::kNarrowRange) {
+        if (O::kNarrowRange) {
             float ym = 0.f;
 #pragma unroll
             for (int j = 0; j < NTO; ++j)
@@ -1083,16 +1129,17 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
 template <typename T, int M, int NCOL, int NCH, bool GLS>
 __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, const T* kbar, const T* yT,
                                             T* obase, int d, int g, int t, int lane, float sl2) {
-    using Op = Mma16<T>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int KTL = (M >= 16) ? M / 16 : 1, NTO = NCOL / 8, YS = (M < 16 ? 16 : M) + 8;
-    uint32_t by[KTL][NTO][2];
+    R by[KTL][NTO][2];
 #pragma unroll
     for (int kk = 0; kk < KTL; ++kk)
 #pragma unroll
         for (int j = 0; j < NTO; ++j) {
             const T* yr = yT + (8 * j + g) * YS + 16 * kk + 2 * t;
-            by[kk][j][0] = ld32(yr);
-            by[kk][j][1] = (M >= 16) ? ld32(yr + 8) : 0u;
+            by[kk][j][0] = O::ld(yr);
+            by[kk][j][1] = (M >= 16) ? O::ld(yr + 8) : O::zero();
         }
     const int jd = d >> 3, tdn = (d & 7) >> 1;
     const int src = (lane & ~3) | tdn;
@@ -1100,19 +1147,10 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
     for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
-            uint32_t f[KTL][4];
+            R f[KTL][4];
             if constexpr (GLS) {
 #pragma unroll
-                for (int kk = 0; kk < KTL; ++kk) {
-                    const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
-                    if constexpr (M >= 16) {
-                        const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
-                        f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = x.z; f[kk][3] = x.w;
-                    } else {
-                        const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
-                        f[kk][0] = x.x; f[kk][1] = x.y; f[kk][2] = f[kk][3] = 0u;
-                    }
-                }
+                for (int kk = 0; kk < KTL; ++kk) GlPark<T, M>::get(glf, ((ch * 4 + tm) * KTL + kk) * 32 + lane, f[kk]);
             } else {
                 gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
             }
@@ -1123,10 +1161,10 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
 #pragma unroll
                 for (int kk = 0; kk < KTL; ++kk)
 #pragma unroll
-                    for (int j = 0; j < NTO; ++j) Op::k16(o[j], f[kk], by[kk][j][0], by[kk][j][1]);
+                    for (int j = 0; j < NTO; ++j) O::mma(o[j], f[kk], by[kk][j][0], by[kk][j][1]);
             } else {
 #pragma unroll
-                for (int j = 0; j < NTO; ++j) Op::k8(o[j], f[0][0], f[0][1], by[0][j][0]);
+                for (int j = 0; j < NTO; ++j) O::mma8(o[j], f[0][0], f[0][1], by[0][j][0]);
             }
             float d0 = 0.f, d1 = 0.f;
 #pragma unroll
@@ -1143,12 +1181,12 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
             for (int j = 0; j < NTO; ++j) {
                 const int c = 8 * j + 2 * t;
                 if (c < d) {
-                    *reinterpret_cast<uint32_t*>(o0 + c) = Op::pack(o[j][0] * i0, o[j][1] * i0);
-                    *reinterpret_cast<uint32_t*>(o1 + c) = Op::pack(o[j][2] * i1, o[j][3] * i1);
+                    O::st2(o0 + c, o[j][0] * i0, o[j][1] * i0);
+                    O::st2(o1 + c, o[j][2] * i1, o[j][3] * i1);
                 }
             }
         }
-        }
+}
 
 template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS, int CW>
 __global__ void __launch_bounds__(GROUPS * Layout<M, NCOL, TPW, WPU, GLS, CW>::GW * 32, 1)
@@ -1156,7 +1194,6 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                  T* __restrict__ out, long long n_units, int d, int iters, float sl2,
                  unsigned int* fault, int active) {
     using Lay = Layout<M, NCOL, TPW, WPU, GLS, CW>;
-    using Op = Mma16<T>;
     constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS,
                   WS = Lay::WS, KTL = Lay::KTL, GW = Lay::GW;
     constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
@@ -1255,10 +1292,10 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
             landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
             if (M < MP && r == 0) {  // zero the padding landmark rows
-                for (int idx = lane; idx < (MP - M) * 16; idx += 32) {
-                    const int j = M + (idx >> 4), p = idx & 15;
-                    *reinterpret_cast<uint32_t*>(qbar + j * LS + 2 * p) = 0u;
-                    *reinterpret_cast<uint32_t*>(kbar + j * LS + 2 * p) = 0u;
+                for (int idx = lane; idx < (MP - M) * 32; idx += 32) {
+                    const int j = M + (idx >> 5), e = idx & 31;
+                    qbar[j * LS + e] = from_f32<T>(0.f);
+                    kbar[j * LS + e] = from_f32<T>(0.f);
                 }
             }
         }
@@ -1271,16 +1308,11 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
                 for (int tm = 0; tm < 4; ++tm) {
-                    uint32_t f[KTL][4];
+                    typename Opnd<T>::Reg f[KTL][4];
                     gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
-                    for (int kk = 0; kk < KTL; ++kk) {
-                        const int slot = ((ch * 4 + tm) * KTL + kk) * 32 + lane;
-                        if constexpr (M >= 16)
-                            reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[kk][0], f[kk][1], f[kk][2], f[kk][3]);
-                        else
-                            reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[kk][0], f[kk][1]);
-                    }
+                    for (int kk = 0; kk < KTL; ++kk)
+                        GlPark<T, M>::put(glf, ((ch * 4 + tm) * KTL + kk) * 32 + lane, f[kk]);
                 }
         }
 
@@ -1449,6 +1481,22 @@ template <typename T, int M, int NCOL>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault);
 
+// fp32 I/O: 8x8 windows with m <= 16 only (the stage-pool kernel).
+template <int TPW, int WPU>
+cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
+                       int iters, cudaStream_t stream, unsigned int* fault) {
+    if constexpr (TPW == 64 && WPU == 1) {
+        const bool wide = d > 30;
+        if (m == 8)
+            return wide ? launch_pool<float, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_pool<float, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (m == 16)
+            return wide ? launch_pool<float, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_pool<float, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    return cudaErrorInvalidValue;
+}
+
 // Dispatch on m and the output-column padding for one window size.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
@@ -1516,6 +1564,8 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
             if (e != cudaSuccess) return e;                                                                  \
         }                                                                                                    \
         unsigned int* fault = s_fault[dev];                                                                  \
+        if (dtype == 0)                                                                                      \
+            return nystra::tc::launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault);      \
         if (dtype == 1)                                                                                      \
             return nystra::tc::launch_n<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, \
                                                                  fault);                                     \

@@ -214,16 +214,10 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             uint32_t* glf = reinterpret_cast<uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W);
 #pragma unroll
             for (int tm = 0; tm < 4; ++tm) {
-                uint32_t f[KTL][4];
+                typename Opnd<T>::Reg f[KTL][4];
                 gl_tile<T, M, KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
-                for (int kq = 0; kq < KTL; ++kq) {
-                    const int slot = (tm * KTL + kq) * 32 + lane;
-                    if constexpr (M >= 16)
-                        reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[kq][0], f[kq][1], f[kq][2], f[kq][3]);
-                    else
-                        reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[kq][0], f[kq][1]);
-                }
+                for (int kq = 0; kq < KTL; ++kq) GlPark<T, M>::put(glf, (tm * KTL + kq) * 32 + lane, f[kq]);
             }
         }
         // ---------------- bounded wait for V ----------------

@@ -242,4 +242,64 @@ template <> struct Mma16<__half> {
     static constexpr bool kNarrowRange = true;  // values above 65504 overflow
 };
 
+// Operand policy for the products with token or d_h extents: how I/O-type
+// values become m16n8k16 operands.  16-bit I/O: one register holds two
+// elements.  fp32 I/O: each element is split into bf16 hi + lo (16
+// significant bits each, fp32's range) and a product takes three MMAs
+// (lo*hi + hi*lo + hi*hi), about 2^-16 relative error per product.
+struct RegPair {
+    uint32_t hi, lo;
+};
+template <typename T>
+struct Opnd {
+    using Op = Mma16<T>;
+    using Reg = uint32_t;
+    static constexpr bool kNarrowRange = Op::kNarrowRange;
+    static __device__ __forceinline__ Reg ld(const T* p) { return *reinterpret_cast<const uint32_t*>(p); }
+    static __device__ __forceinline__ Reg pk(float a, float b) { return Op::pack(a, b); }
+    static __device__ __forceinline__ Reg tr(Reg r) { return movmatrix_trans(r); }
+    static __device__ __forceinline__ Reg zero() { return 0u; }
+    static __device__ __forceinline__ Reg one() { return Op::kOne; }  // the pair (1, 0)
+    static __device__ __forceinline__ void mma(float (&c)[4], const Reg (&a)[4], Reg b0, Reg b1) {
+        Op::k16(c, a, b0, b1);
+    }
+    static __device__ __forceinline__ void mma8(float (&c)[4], Reg a0, Reg a1, Reg b0) { Op::k8(c, a0, a1, b0); }
+    static __device__ __forceinline__ void st2(T* p, float a, float b) {
+        *reinterpret_cast<uint32_t*>(p) = Op::pack(a, b);
+    }
+};
+template <>
+struct Opnd<float> {
+    using Op = Mma16<__nv_bfloat16>;
+    using Reg = RegPair;
+    static constexpr bool kNarrowRange = false;
+    static __device__ __forceinline__ Reg pk(float a, float b) {
+        const uint32_t h = Op::pack(a, b);
+        const float2 hf = Op::unpack(h);
+        return {h, Op::pack(a - hf.x, b - hf.y)};
+    }
+    static __device__ __forceinline__ Reg ld(const float* p) {
+        const float2 v = *reinterpret_cast<const float2*>(p);
+        return pk(v.x, v.y);
+    }
+    static __device__ __forceinline__ Reg tr(Reg r) { return {movmatrix_trans(r.hi), movmatrix_trans(r.lo)}; }
+    static __device__ __forceinline__ Reg zero() { return {0u, 0u}; }
+    static __device__ __forceinline__ Reg one() { return {Op::kOne, 0u}; }
+    static __device__ __forceinline__ void mma(float (&c)[4], const Reg (&a)[4], Reg b0, Reg b1) {
+        const uint32_t ah[4] = {a[0].hi, a[1].hi, a[2].hi, a[3].hi};
+        const uint32_t al[4] = {a[0].lo, a[1].lo, a[2].lo, a[3].lo};
+        Op::k16(c, al, b0.hi, b1.hi);
+        Op::k16(c, ah, b0.lo, b1.lo);
+        Op::k16(c, ah, b0.hi, b1.hi);
+    }
+    static __device__ __forceinline__ void mma8(float (&c)[4], Reg a0, Reg a1, Reg b0) {
+        Op::k8(c, a0.lo, a1.lo, b0.hi);
+        Op::k8(c, a0.hi, a1.hi, b0.lo);
+        Op::k8(c, a0.hi, a1.hi, b0.hi);
+    }
+    static __device__ __forceinline__ void st2(float* p, float a, float b) {
+        *reinterpret_cast<float2*>(p) = make_float2(a, b);
+    }
+};
+
 }  // namespace nystra
