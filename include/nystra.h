@@ -122,6 +122,23 @@ NYSTRA_API int nystra_last_cuda_error(void);
  */
 NYSTRA_API int nystra_status(void* stream);
 
+/*
+ * nystra_check -- the same as nystra_status (the name the method's
+ * integration notes use for the synchronising status helper).
+ */
+NYSTRA_API int nystra_check(void* stream);
+
+/*
+ * nystra_debug_wait_timeout -- test-only (the paper has no counterpart):
+ * launches one warp on `stream` that waits, through the same bounded
+ * mbarrier wait the kernels use, on an mbarrier nothing ever arrives on.
+ * After limit_ns nanoseconds of %globaltimer it gives up and records the
+ * timeout exactly as a kernel would, so the next nystra_status(stream)
+ * returns NYSTRA_ETIMEOUT and the context stays usable.  limit_ns must lie in
+ * [1000, 1000000000] (1 us to 1 s), else NYSTRA_EINVAL; nothing is allocated.
+ */
+NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

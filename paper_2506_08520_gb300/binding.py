@@ -51,6 +51,10 @@ def lib() -> ctypes.CDLL:
         L.nystra_last_cuda_error.restype = i
         L.nystra_status.argtypes = [vp]
         L.nystra_status.restype = i
+        L.nystra_check.argtypes = [vp]
+        L.nystra_check.restype = i
+        L.nystra_debug_wait_timeout.argtypes = [ctypes.c_ulonglong, vp]
+        L.nystra_debug_wait_timeout.restype = i
         _lib = L
     return _lib
 
@@ -76,6 +80,16 @@ def version() -> int:
 def status(stream=None) -> int:
     """Synchronise ``stream`` and return the device-side fault status."""
     return lib().nystra_status(_stream_ptr(stream))
+
+
+def check(stream=None) -> int:
+    """Same as ``status``."""
+    return lib().nystra_check(_stream_ptr(stream))
+
+
+def debug_wait_timeout(limit_ns: int, stream=None) -> int:
+    """Test-only: launch a wait that can only time out (see the header)."""
+    return lib().nystra_debug_wait_timeout(int(limit_ns), _stream_ptr(stream))
 
 
 # ------------------------------------------------------------ torch helpers

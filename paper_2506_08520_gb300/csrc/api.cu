@@ -104,6 +104,14 @@ int nystra_status(void* stream) {
     return (words & 1u) ? NYSTRA_ETIMEOUT : NYSTRA_OK;
 }
 
+int nystra_check(void* stream) { return nystra_status(stream); }
+
+int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream) {
+    if (limit_ns < 1000ull || limit_ns > 1000000000ull) return NYSTRA_EINVAL;
+    const cudaError_t e = nystra_host::launch_debug_wait(limit_ns, (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
 }  // extern "C"
 
 namespace nystra_host {
@@ -111,8 +119,9 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[4])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
-                                                   take_fault_word_tc_n1024, take_fault_word_exact_tc};
+    unsigned int (*const take[5])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
+                                                   take_fault_word_tc_n1024, take_fault_word_exact_tc,
+                                                   take_fault_word_debug};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

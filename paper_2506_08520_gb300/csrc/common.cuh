@@ -53,4 +53,6 @@ unsigned int take_fault_word_exact_tc(cudaError_t* err);
 // Device-side fault words (bit 0: a bounded wait gave up) of the translation
 // units whose kernels wait on barriers: OR-ed together, then cleared.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);
+cudaError_t launch_debug_wait(unsigned long long limit_ns, cudaStream_t stream);
+unsigned int take_fault_word_debug(cudaError_t* err);
 }  // namespace nystra_host

@@ -27,7 +27,8 @@ def declared_symbols():
 def test_header_declares_the_boundary():
     names = declared_symbols()
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
-                     "nystra_version", "nystra_status", "nystra_last_cuda_error"):
+                     "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
+                     "nystra_debug_wait_timeout"):
         assert required in names
 
 
@@ -94,3 +95,9 @@ def test_torch_wrappers_refuse_cpu_tensors(lib):
         nb.nystra(x, x, x)
     with pytest.raises(ValueError):
         nb.exact(x, x, x)
+
+
+@pytest.mark.parametrize("limit_ns", [0, 999, 1_000_000_001, 1 << 62])
+def test_debug_wait_limit_validation(lib, limit_ns):
+    # out-of-range limits are refused on the host, before any launch
+    assert nb.lib().nystra_debug_wait_timeout(limit_ns, None) == nb.NYSTRA_EINVAL
