@@ -427,49 +427,61 @@ struct GlPark {
 };
 
 // Landmark means of the segments one warp owns (Algorithm 1 step 1) on the
-// tensor cores: xbar = P X with the averaging matrix P (P[j][t] = 1/L when
-// token t lies in segment j; exact in 16 bits since L is a power of two) as A
-// operand and the staged tokens X (rows = tokens, k) as B operand, whose
-// fragments are 8x8 transposes of the row-major stage.  The fp32 means are
-// rounded to the I/O type and stored as rows j0.. of xbar (row stride LS);
-// columns >= d come out as zeros.
+// tensor cores, transposed: xbar^T = X^T P^T with the staged tokens X as
+// the A operand (features x tokens; fragments are 8x8 transposes of the
+// row-major stage) and the averaging matrix P^T (P[j][t] = 1/L when token t
+// lies in segment j; exact in 16 bits since L is a power of two) as B.  A
+// 16-token k-step only meets the n-tiles of its own segments, so a warp
+// issues 2 x TPW/16 products (x2 when L = 1).  The fp32 means are rounded
+// to the I/O type and stored as rows j0.. of xbar (row stride LS); columns
+// >= d come out as zeros.
 template <typename T, int TPW, int L>
 __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
     using O = Opnd<T>;
     using R = typename O::Reg;
-    constexpr int LPW = TPW / L;            // segments owned by the warp
-    constexpr int MTL = (LPW + 15) / 16;    // m-tiles of landmark rows
+    constexpr int LPW = TPW / L;          // segments owned by the warp
+    constexpr int NTJ = (LPW + 7) / 8;    // n-tiles of landmark columns
     constexpr int LS = 40;
     constexpr float inv = 1.f / (float)L;
-    float c[MTL][4][4];
+    float c[2][NTJ][4];
 #pragma unroll
-    for (int ml = 0; ml < MTL; ++ml)
+    for (int mf = 0; mf < 2; ++mf)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) c[ml][b][0] = c[ml][b][1] = c[ml][b][2] = c[ml][b][3] = 0.f;
+        for (int j = 0; j < NTJ; ++j) c[mf][j][0] = c[mf][j][1] = c[mf][j][2] = c[mf][j][3] = 0.f;
 #pragma unroll
     for (int ks = 0; ks < TPW / 16; ++ks) {  // 16 tokens per k-step
-        const int ml = (16 * ks / L) / 16;   // the one m-tile these tokens feed
-        // A = P rows 16 ml + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
-        auto pv = [&](int row, int tok) -> float { return (tok / L == row) ? inv : 0.f; };
-        const int r0 = 16 * ml + g, r1 = r0 + 8, k0 = 16 * ks + 2 * t;
-        const R a[4] = {O::pk(pv(r0, k0), pv(r0, k0 + 1)), O::pk(pv(r1, k0), pv(r1, k0 + 1)),
-                        O::pk(pv(r0, k0 + 8), pv(r0, k0 + 9)), O::pk(pv(r1, k0 + 8), pv(r1, k0 + 9))};
+        // A = X^T, features 16 mf + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
+        R a[2][4];
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int c0 = 8 * b + 2 * t;
-            const R x0 = c0 < d ? O::ld(X + (16 * ks + g) * d + c0) : O::zero();
-            const R x1 = c0 < d ? O::ld(X + (16 * ks + 8 + g) * d + c0) : O::zero();
-            O::mma(c[ml][b], a, O::tr(x0), O::tr(x1));
+        for (int mf = 0; mf < 2; ++mf)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+                const int f0 = 16 * mf + 8 * (r & 1) + 2 * t;
+                const R x = f0 < d ? O::ld(X + (16 * ks + 8 * (r >> 1) + g) * d + f0) : O::zero();
+                a[mf][r] = O::tr(x);
+            }
+        constexpr int kTok = 16;
+        const int jlo = (16 * ks / L) / 8, jhi = ((16 * ks + kTok - 1) / L) / 8;
+#pragma unroll
+        for (int j = 0; j < NTJ; ++j) {
+            if (j < jlo || j > jhi) continue;  // compile-time after unrolling
+            // B = P^T: tokens 16 ks + 2t (+1) (+8, +9), segment 8j + g
+            auto pv = [&](int tok) -> float { return (tok / L == 8 * j + g) ? inv : 0.f; };
+            const int k0 = 16 * ks + 2 * t;
+            const R b0 = O::pk(pv(k0), pv(k0 + 1)), b1 = O::pk(pv(k0 + 8), pv(k0 + 9));
+#pragma unroll
+            for (int mf = 0; mf < 2; ++mf) O::mma(c[mf][j], a[mf], b0, b1);
         }
     }
 #pragma unroll
-    for (int ml = 0; ml < MTL; ++ml)
+    for (int mf = 0; mf < 2; ++mf)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int row = 16 * ml + g, col = 8 * b + 2 * t;
-            if (row < LPW) O::st2(xbar + (j0 + row) * LS + col, c[ml][b][0], c[ml][b][1]);
-            if (row + 8 < LPW) O::st2(xbar + (j0 + row + 8) * LS + col, c[ml][b][2], c[ml][b][3]);
-        }
+        for (int j = 0; j < NTJ; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int lm = 8 * j + 2 * t + (e & 1), f = 16 * mf + g + 8 * (e >> 1);
+                if (lm < LPW) xbar[(j0 + lm) * LS + f] = from_f32<T>(c[mf][j][e]);
+            }
 }
 
 // Front, U side, for one warp's NCH chunks of 64 tokens: S_U = Qbar K^T with a
