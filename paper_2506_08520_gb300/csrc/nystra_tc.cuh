@@ -90,10 +90,10 @@ struct Layout {
     static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;
     static constexpr size_t GLF = STAGE;
     static constexpr size_t WARP_BYTES = ((GLF + (GLS ? (size_t)NCH * 4 * KTL * 32 * GLB : 0) + 127) / 128) * 128;
-    // A warp's partial W (fp32 MP x NCOL, then MP row maxima) lives in its
-    // stage right after the Q rows, once K and V are consumed.
+    // A warp's partial W (fp32 MP x NCOL, row stride WS, then MP row maxima)
+    // lives in its stage right after the Q rows, once K and V are consumed.
     static constexpr size_t WPART = (size_t)TPW * DS * 2;
-    static_assert(WPU == 1 || (size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2,
+    static_assert(WPU == 1 || (size_t)MP * WS * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2,
                   "W partial must fit in K+V");
     // per-group shared memory
     // With one warp per unit and G_L^n parked, Y^T is written only after the
@@ -592,12 +592,12 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
         const int i = e / NCOL, c = e - (e / NCOL) * NCOL;
         float mu = -INFINITY;
 #pragma unroll
-        for (int s2 = 0; s2 < WPU; ++s2) mu = fmaxf(mu, part0[(size_t)s2 * wstride + MP * NCOL + i]);
+        for (int s2 = 0; s2 < WPU; ++s2) mu = fmaxf(mu, part0[(size_t)s2 * wstride + MP * WS + i]);
         float acc = 0.f;
 #pragma unroll
         for (int s2 = 0; s2 < WPU; ++s2) {
             const float* ps = part0 + (size_t)s2 * wstride;
-            acc = fmaf(ex2(ps[MP * NCOL + i] - mu), ps[i * NCOL + c], acc);
+            acc = fmaf(ex2(ps[MP * WS + i] - mu), ps[i * WS + c], acc);
         }
         mW[i * WS + c] = acc;
         if (c == 0) gmu[i] = mu;
@@ -1343,10 +1343,9 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
         float mU[MT][2];  // this warp's row maxima of S_U, log2 domain
         if (tok) {
-            front_su_w<T, M, NCOL, NCH>(qbar, Ks, Vs, d, g, t, sl2, WPU == 1 ? mW : wpart, WPU == 1 ? WS : NCOL,
-                                        mU);
+            front_su_w<T, M, NCOL, NCH>(qbar, Ks, Vs, d, g, t, sl2, WPU == 1 ? mW : wpart, WS, mU);
             if ((WPU > 1 || CW > 1) && t == 0) {
-                float* mdst = WPU > 1 ? wpart + MP * NCOL : gmu;
+                float* mdst = WPU > 1 ? wpart + MP * WS : gmu;
 #pragma unroll
                 for (int mt = 0; mt < MT; ++mt) {
                     mdst[16 * mt + g] = mU[mt][0];

@@ -37,7 +37,7 @@ struct TeamLayout {
     static constexpr int GLB = (M >= 16) ? 16 : 8;
     static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;  // a token warp's Q, K, V rows
     static constexpr size_t WPART = (size_t)TPW * DS * 2;      // partial W_r after Q (K, V consumed)
-    static_assert((size_t)MP * NCOL * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
+    static_assert((size_t)MP * WS * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
     // one buffer of per-unit state
     static constexpr size_t GLF_W = 4 * KTL * 32 * GLB;  // one token warp's G_L^n fragments
     static constexpr size_t B_QB = 0;
@@ -230,10 +230,10 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         pend_v = !ok_v;
         // ---------------- S_U, partial W_r and row maxima ----------------
         float mU[1][2];
-        front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, NCOLC, mU);
+        front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU);
         if (t == 0) {
-            wpart[MP * NCOLC + g] = mU[0][0];
-            wpart[MP * NCOLC + g + 8] = mU[0][1];
+            wpart[MP * WS + g] = mU[0][0];
+            wpart[MP * WS + g + 8] = mU[0][1];
         }
         tsync();
         combine_partials<MP, NCOLC, WS, NT>(reinterpret_cast<const float*>(tb + Lay::WPART), Lay::STAGE / 4,
