@@ -1,0 +1,316 @@
+// Streaming team kernel for 32x32 windows (N = 1024 tokens), m <= 16, even
+// d_h <= 32, 16-bit I/O.  Included by the N = 1024 translation unit after
+// nystra_tc.cuh, whose per-phase device functions it reuses.
+//
+// A whole 32x32 unit (Q, K, V: 184 KB at d_h = 30) fills an SM, so staging
+// units whole leaves HBM idle while the front phase runs and serialises the
+// m x m core with everything else.  This kernel streams 64-token chunks
+// instead.  A team is four token warps (256 tokens each) plus a dedicated core
+// warp; per-unit state (landmarks, W, m_U, Y^T) is double-buffered, so the
+// core warp runs the iteration of unit k while the token warps work on unit
+// k + 1 and the output of unit k.  Each token warp walks a fixed sequence of
+// chunk tasks through a private ring of NSLOT chunk buffers, copying task
+// v + NSLOT into a buffer as soon as task v has released it:
+//
+//   Q(k)   Q chunk -> landmark sums of Qbar          (after the 4th: [sync])
+//   KV(k)  K and V chunks -> landmark sums of Kbar, S_U with running maxima,
+//          partial W_r = G_U^n [V | 1]               (after the 4th: [sync],
+//          combine into W and m_U, [sync], signal the core: mbarrier F_b)
+//   OUT(k-1) Q chunk of the previous unit, read again -> S_L, G_L^n (from the
+//          resident Kbar), O = (G_L^n Y_:d) / (G_L^n Y_d) once the core of
+//          that unit is done (mbarrier C_b), written in place over the Q rows
+//          and bulk-stored.
+//
+// Q is read twice (the second time usually from L2: it was read about one
+// unit earlier); K, V once; O written once.  [sync] is a named barrier over
+// the four token warps.  Every mbarrier wait is bounded; a warp whose wait
+// gives up keeps to the barrier sequence and the token warps leave together
+// after the next barrier, whose OR-reduction gives every warp the same verdict.
+#pragma once
+
+#include "nystra_tc.cuh"
+
+namespace nystra {
+namespace tc {
+
+template <int M, int NCOL>
+struct StreamLayout {
+    static constexpr int NT = 4, TPW = 256, N = NT * TPW, CH = 64, NCHK = TPW / CH;
+    static constexpr int DS = (NCOL == 32) ? 30 : 32;
+    static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int L = N / M, LPW = TPW / L;  // tokens per segment, segments per token warp
+    static constexpr size_t XB = (size_t)CH * DS * 2;  // one tensor's chunk
+    static constexpr size_t SLOT = 2 * XB;             // K and V (Q uses the first half)
+    static constexpr size_t WPB = (((size_t)MP * WS * 4 + MP * 4) + 127) / 128 * 128;  // W partial, row maxima
+    // per-unit state
+    static constexpr size_t B_QB = 0;
+    static constexpr size_t B_KB = B_QB + MP * LS * 2;
+    static constexpr size_t B_W = B_KB + MP * LS * 2;
+    static constexpr size_t B_MU = B_W + MP * WS * 4;
+    static constexpr size_t B_YT = B_MU + MP * 4;
+    static constexpr size_t BUF = ((B_YT + NCOL * YS * 2 + 127) / 128) * 128;
+    template <int S>
+    struct Team {
+        static constexpr size_t WARP = S * SLOT + WPB;  // ring, then the W partial
+        static constexpr size_t T_BUF = NT * WARP;
+        static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // slot bars [NT][S], F[2], C[2]
+        static constexpr size_t BYTES = ((T_BAR + (NT * S + 4) * 8 + 127) / 128) * 128;
+    };
+    static constexpr int TEAMS = 2;
+    static constexpr int NSLOT = (TEAMS * Team<3>::BYTES <= kSmemLimit) ? 3 : 2;
+    using TL = Team<NSLOT>;
+    static constexpr size_t TEAM = TL::BYTES;
+    static_assert(TEAMS * TEAM <= kSmemLimit, "two teams must fit");
+    static_assert(M <= 16 && L >= 16 && LPW <= 8, "segments per token warp fit one n-tile");
+    static_assert(XB % 16 == 0 && SLOT % 16 == 0 && TL::WARP % 16 == 0 && BUF % 16 == 0, "16-byte alignment");
+};
+
+// Chunk task v of a team that processes `count` units, in order: for each
+// unit k, Q(k) x 4, KV(k) x 4, then OUT(k - 1) x 4 (k >= 1); finally
+// OUT(count - 1) x 4.  12 * count tasks.
+struct StreamTask {
+    int k, type, c;  // unit (team-local), 0 = Q, 1 = KV, 2 = OUT, chunk
+};
+__device__ __forceinline__ StreamTask stream_task(int v, int count) {
+    int i;
+    if (v < 8) i = v;
+    else if (v < 12 * count - 4) i = v + 4;
+    else i = v + 12;
+    const int k = i / 12, r = i - 12 * k;
+    if (r < 8) return {k, r >> 2, r & 3};
+    return {k - 1, 2, r & 3};
+}
+
+template <typename T, int M, int NCOL>
+__global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
+nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
+                     T* __restrict__ out, long long n_units, int d, int iters, float sl2, unsigned int* fault) {
+    using Lay = StreamLayout<M, NCOL>;
+    using TL = typename Lay::TL;
+    using R = typename Opnd<T>::Reg;
+    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
+                  NSLOT = Lay::NSLOT, L = Lay::L, LPW = Lay::LPW, NTO = NCOL / 8;
+
+    extern __shared__ __align__(128) unsigned char smem_raw[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int team = warp / (NT + 1), r = warp - team * (NT + 1);  // r == NT: core warp
+    const int g = lane >> 2, t = lane & 3;
+    unsigned char* tb = smem_raw + (size_t)team * Lay::TEAM;
+    auto buf = [&](int b) { return tb + TL::T_BUF + (size_t)b * Lay::BUF; };
+    uint64_t* bars = reinterpret_cast<uint64_t*>(tb + TL::T_BAR);
+    uint64_t* barF = bars + NT * NSLOT;  // F[b]: the token warps' state for the core is ready
+    uint64_t* barC = barF + 2;           // C[b]: the core's Y^T is ready
+
+    const long long stride = (long long)gridDim.x * Lay::TEAMS;
+    const long long u0 = (long long)blockIdx.x * Lay::TEAMS + team;
+    const int count = u0 < n_units ? (int)((n_units - u0 + stride - 1) / stride) : 0;  // units of this team
+
+    if (threadIdx.x == 0) {
+        for (int tm = 0; tm < Lay::TEAMS; ++tm) {
+            uint64_t* bb = reinterpret_cast<uint64_t*>(smem_raw + (size_t)tm * Lay::TEAM + TL::T_BAR);
+            for (int i = 0; i < NT * NSLOT; ++i) mbar_init(bb + i, 1);
+            mbar_init(bb + NT * NSLOT, NT);
+            mbar_init(bb + NT * NSLOT + 1, NT);
+            mbar_init(bb + NT * NSLOT + 2, 1);
+            mbar_init(bb + NT * NSLOT + 3, 1);
+        }
+        fence_mbar_init();
+    }
+    // padding landmark rows (m < 16) stay zero: nothing else writes them
+    if constexpr (M < MP) {
+        for (int idx = threadIdx.x; idx < Lay::TEAMS * 2 * (MP - M) * 32; idx += blockDim.x) {
+            const int tm = idx / (2 * (MP - M) * 32), rem = idx - tm * 2 * (MP - M) * 32;
+            const int b = rem / ((MP - M) * 32), e = rem - b * (MP - M) * 32;
+            T* qb = reinterpret_cast<T*>(smem_raw + (size_t)tm * Lay::TEAM + TL::T_BUF + (size_t)b * Lay::BUF +
+                                         Lay::B_QB);
+            T* kb = reinterpret_cast<T*>(smem_raw + (size_t)tm * Lay::TEAM + TL::T_BUF + (size_t)b * Lay::BUF +
+                                         Lay::B_KB);
+            qb[(M + (e >> 5)) * LS + (e & 31)] = from_f32<T>(0.f);
+            kb[(M + (e >> 5)) * LS + (e & 31)] = from_f32<T>(0.f);
+        }
+    }
+    __syncthreads();
+
+    if (r == NT) {
+        // ======================= core warp =======================
+        for (int kk = 0; kk < count; ++kk) {
+            const int b = kk & 1;
+            const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, (uint32_t)((kk >> 1) & 1), kWaitNs));
+            if (!ok) {  // the token warps stopped (or stalled): stop too
+                if (lane == 0) atomicOr(fault, 1u);
+                break;
+            }
+            unsigned char* bb = buf(b);
+            const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
+            float mU[1][2] = {{gmu[g], gmu[g + 8]}};
+            core_warp<T, M, NCOL>(reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB),
+                                  mU, reinterpret_cast<const float*>(bb + Lay::B_W),
+                                  reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(barC + b);
+        }
+        return;
+    }
+
+    // ======================= token warp r =======================
+    unsigned char* wr = tb + (size_t)r * TL::WARP;
+    float* wpart = reinterpret_cast<float*>(wr + NSLOT * Lay::SLOT);
+    uint64_t* sbar = bars + r * NSLOT;
+    const uint32_t xbytes = (uint32_t)(Lay::CH * d * sizeof(T));
+    auto slot_x = [&](int s, int h) { return reinterpret_cast<T*>(wr + (size_t)s * Lay::SLOT + h * Lay::XB); };
+    auto chunk_off = [&](long long unit, int c) {
+        return ((size_t)unit * N + (size_t)r * TPW + (size_t)c * Lay::CH) * d;
+    };
+    const int total = 12 * count;
+    // L2 policies: the first read of Q is kept for its second read (OUT);
+    // every other read is its last.
+    const uint64_t keep = l2_evict_last(), drop = l2_evict_first();
+    // lane 0: copies of task vv into its slot
+    auto issue = [&](int vv) {
+        const StreamTask tk = stream_task(vv, count);
+        const int s = vv % NSLOT;
+        const size_t off = chunk_off(u0 + tk.k * stride, tk.c);
+        if (tk.type == 1) {
+            mbar_arrive_expect_tx(sbar + s, 2u * xbytes);
+            bulk_g2s_hint(slot_x(s, 0), k + off, xbytes, sbar + s, drop);
+            bulk_g2s_hint(slot_x(s, 1), v + off, xbytes, sbar + s, drop);
+        } else {
+            mbar_arrive_expect_tx(sbar + s, xbytes);
+            bulk_g2s_hint(slot_x(s, 0), q + off, xbytes, sbar + s, tk.type == 0 ? keep : drop);
+        }
+    };
+    auto tsync = [&]() { named_barrier(1 + team, NT * 32); };
+    // barrier that also tells every token warp whether any of them failed
+    auto tsync_or = [&](bool f) { return named_barrier_or(1 + team, NT * 32, f); };
+
+    int issued = 0, consumed = 0;
+    if (lane == 0)
+        for (; issued < NSLOT && issued < total; ++issued) issue(issued);
+    issued = __shfl_sync(0xffffffffu, issued, 0);
+
+    bool failed = false;  // a bounded wait of this warp gave up (warp-uniform)
+    float cq[2][1][4], ck[2][1][4], w[NTO][4];
+    float run0 = -INFINITY, run1 = -INFINITY;
+    R aq[2][4];
+    for (int vv = 0; vv < total; ++vv) {
+        const StreamTask tk = stream_task(vv, count);
+        const int s = vv % NSLOT;
+        const int b = tk.k & 1;
+        unsigned char* bb = buf(b);
+        // ---------------- bounded wait for this task's chunk ----------------
+        if (!failed) {
+            if (__all_sync(0xffffffffu, mbar_wait_bounded(sbar + s, (uint32_t)((vv / NSLOT) & 1), kWaitNs))) {
+                ++consumed;
+            } else {
+                failed = true;
+                if (lane == 0) atomicOr(fault, 1u);
+            }
+        }
+        T* X0 = slot_x(s, 0);
+        if (tk.type == 0) {
+            // ---------------- Q(k): landmark sums of Qbar ----------------
+            if (tk.c == 0)
+#pragma unroll
+                for (int mf = 0; mf < 2; ++mf) cq[mf][0][0] = cq[mf][0][1] = cq[mf][0][2] = cq[mf][0][3] = 0.f;
+            landmarks_acc<T, L, LPW>(X0, tk.c * Lay::CH, cq, d, g, t);
+            if (tk.c == Lay::NCHK - 1) {
+                landmarks_put<T, LPW>(cq, reinterpret_cast<T*>(bb + Lay::B_QB), r * LPW, g, t);
+                if (tsync_or(failed)) break;
+                qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), 0, g, t, aq);
+            }
+        } else if (tk.type == 1) {
+            // ---------------- KV(k): Kbar sums, S_U, partial W ----------------
+            if (tk.c == 0) {
+#pragma unroll
+                for (int mf = 0; mf < 2; ++mf) ck[mf][0][0] = ck[mf][0][1] = ck[mf][0][2] = ck[mf][0][3] = 0.f;
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
+                run0 = run1 = -INFINITY;
+            }
+            landmarks_acc<T, L, LPW>(X0, tk.c * Lay::CH, ck, d, g, t);
+            su_w_chunk<T, NCOL>(aq, X0, slot_x(s, 1), d, g, t, sl2, g < M, g + 8 < M, w, run0, run1, true);
+            if (tk.c == Lay::NCHK - 1) {
+                landmarks_put<T, LPW>(ck, reinterpret_cast<T*>(bb + Lay::B_KB), r * LPW, g, t);
+#pragma unroll
+                for (int j = 0; j < NTO; ++j) {
+                    const int c = 8 * j + 2 * t;
+                    *reinterpret_cast<float2*>(wpart + g * WS + c) = make_float2(w[j][0], w[j][1]);
+                    *reinterpret_cast<float2*>(wpart + (g + 8) * WS + c) = make_float2(w[j][2], w[j][3]);
+                }
+                if (t == 0) {
+                    wpart[MP * WS + g] = run0;
+                    wpart[MP * WS + g + 8] = run1;
+                }
+                tsync();
+                combine_partials<MP, NCOL, WS, NT>(reinterpret_cast<const float*>(tb + NSLOT * Lay::SLOT),
+                                                    TL::WARP / 4, reinterpret_cast<float*>(bb + Lay::B_W),
+                                                    reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
+                if (tsync_or(failed)) break;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(barF + b);
+            }
+        } else {
+            // ---------------- OUT(k): output rows of this chunk ----------------
+            if (tk.c == 0 && !failed) {
+                if (!__all_sync(0xffffffffu, mbar_wait_bounded(barC + b, (uint32_t)((tk.k >> 1) & 1), kWaitNs))) {
+                    failed = true;
+                    if (lane == 0) atomicOr(fault, 1u);
+                }
+            }
+            if (!failed) {
+                output_rows<T, M, NCOL, 1, false>(nullptr, X0, reinterpret_cast<const T*>(bb + Lay::B_KB),
+                                                  reinterpret_cast<const T*>(bb + Lay::B_YT), X0, d, g, t, lane,
+                                                  sl2);
+                fence_proxy_async_smem();  // this lane's writes precede the bulk store
+                __syncwarp();
+                if (lane == 0) {
+                    bulk_s2g(out + chunk_off(u0 + tk.k * stride, tk.c), X0, xbytes);
+                    bulk_commit();
+                    bulk_wait_read_all();
+                }
+            }
+        }
+        // The slot is released: copy the task NSLOT ahead into it.
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (issued < total && !failed) {
+            if (lane == 0) issue(issued);
+            ++issued;
+        }
+    }
+    if (lane == 0) bulk_wait_all();  // output stores complete before exit
+    // Fault path only: copies issued and not yet seen complete land before
+    // the CTA's shared memory is released.
+    for (int i = consumed; i < issued; ++i)
+        (void)__all_sync(0xffffffffu, mbar_wait_bounded(sbar + i % NSLOT, (uint32_t)((i / NSLOT) & 1), kWaitNs));
+}
+
+template <typename T, int M, int NCOL>
+cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                          int iters, cudaStream_t stream, unsigned int* fault) {
+    using Lay = StreamLayout<M, NCOL>;
+    auto kern = nystra_stream_kernel<T, M, NCOL>;
+    const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
+    static int s_blocks = 0;  // persistent grid size, set on first use
+    if (s_blocks == 0) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        int dev = 0, sms = 0, per_sm = 0;
+        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * 5 * 32, smem)) !=
+            cudaSuccess)
+            return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        s_blocks = sms * per_sm;
+    }
+    const long long want = (n_units + Lay::TEAMS - 1) / Lay::TEAMS;
+    const long long grid = want < s_blocks ? want : s_blocks;
+    const float sl2 = 1.4426950408889634f / sqrtf((float)d);
+    kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
+                                                                 n_units, d, iters, sl2, fault);
+    return cudaGetLastError();
+}
+
+}  // namespace tc
+}  // namespace nystra

@@ -111,7 +111,7 @@ struct Layout {
                                               : QK_BYTES + YT_BYTES;  // m_U, log2 domain
     static constexpr size_t G_W = G_MU + MP * 4;
     static constexpr size_t G_BAR = G_W + MP * WS * 4;
-    static constexpr size_t G_FLAG = G_BAR + 16 * WPU;  // two mbarriers per token warp
+    static constexpr size_t G_BAR_END = G_BAR + 16 * WPU;  // two mbarriers per token warp
     // Distributed core (CW > 1): its scratch is group memory, or, with long
     // stages (TPW >= 256), the first two token warps' K/V rows (consumed by
     // the combine before the core starts; the next unit's K and V are copied
@@ -122,7 +122,7 @@ struct Layout {
                                                        DistScratch<(M > 16 ? M : 32)>::AUX <=
                                                    2 * (size_t)TPW * DS * 2),
                   "scratch must fit in two warps' K/V rows");
-    static constexpr size_t G_SCR = ((G_FLAG + 16 + 127) / 128) * 128;
+    static constexpr size_t G_SCR = ((G_BAR_END + 16 + 127) / 128) * 128;
     static constexpr size_t GROUP_BYTES = ((G_SCR + SCR_BYTES + 127) / 128) * 128;
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
 };
@@ -404,24 +404,26 @@ struct GlPark {
             }
         }
     }
-    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, R (&f)[4]) {
-        if constexpr (sizeof(R) == 4) {
-            if constexpr (M >= 16) {
-                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
-                f[0] = x.x; f[1] = x.y; f[2] = x.z; f[3] = x.w;
-            } else {
-                const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
-                f[0] = x.x; f[1] = x.y; f[2] = f[3] = 0u;
-            }
+    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, uint32_t (&f)[4]) {
+        if constexpr (M >= 16) {
+            const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+            f[0] = x.x; f[1] = x.y; f[2] = x.z; f[3] = x.w;
         } else {
-            if constexpr (M >= 16) {
-                const uint4 h = reinterpret_cast<const uint4*>(glf)[2 * slot];
-                const uint4 l = reinterpret_cast<const uint4*>(glf)[2 * slot + 1];
-                f[0] = {h.x, l.x}; f[1] = {h.y, l.y}; f[2] = {h.z, l.z}; f[3] = {h.w, l.w};
-            } else {
-                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
-                f[0] = {x.x, x.z}; f[1] = {x.y, x.w}; f[2] = f[3] = Opnd<T>::zero();
-            }
+            const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
+            f[0] = x.x; f[1] = x.y; f[2] = f[3] = 0u;
+        }
+    }
+    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, RegPair (&f)[4]) {
+        const uint4* p = reinterpret_cast<const uint4*>(glf);
+        if constexpr (M >= 16) {
+            f[0] = {p[2 * slot].x, p[2 * slot + 1].x};
+            f[1] = {p[2 * slot].y, p[2 * slot + 1].y};
+            f[2] = {p[2 * slot].z, p[2 * slot + 1].z};
+            f[3] = {p[2 * slot].w, p[2 * slot + 1].w};
+        } else {
+            f[0] = {p[slot].x, p[slot].z};
+            f[1] = {p[slot].y, p[slot].w};
+            f[2] = f[3] = RegPair{0u, 0u};
         }
     }
 };
@@ -432,24 +434,21 @@ struct GlPark {
 // row-major stage) and the averaging matrix P^T (P[j][t] = 1/L when token t
 // lies in segment j; exact in 16 bits since L is a power of two) as B.  A
 // 16-token k-step only meets the n-tiles of its own segments, so a warp
-// issues 2 x TPW/16 products (x2 when L = 1).  The fp32 means are rounded
-// to the I/O type and stored as rows j0.. of xbar (row stride LS); columns
-// >= d come out as zeros.
-template <typename T, int TPW, int L>
-__device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
+// issues 2 x TPW/16 products (x2 when L = 1).
+//
+// landmarks_acc adds one 64-token chunk X (tokens tok0..tok0+63 of the warp's
+// range) to the accumulators c (features x the warp's LPW segments);
+// landmarks_put rounds the means to the I/O type and stores them as rows
+// j0.. of xbar (row stride LS); columns >= d come out as zeros.
+template <typename T, int L, int LPW>
+__device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2][(LPW + 7) / 8][4], int d, int g,
+                                              int t) {
     using O = Opnd<T>;
     using R = typename O::Reg;
-    constexpr int LPW = TPW / L;          // segments owned by the warp
-    constexpr int NTJ = (LPW + 7) / 8;    // n-tiles of landmark columns
-    constexpr int LS = 40;
+    constexpr int NTJ = (LPW + 7) / 8;
     constexpr float inv = 1.f / (float)L;
-    float c[2][NTJ][4];
 #pragma unroll
-    for (int mf = 0; mf < 2; ++mf)
-#pragma unroll
-        for (int j = 0; j < NTJ; ++j) c[mf][j][0] = c[mf][j][1] = c[mf][j][2] = c[mf][j][3] = 0.f;
-#pragma unroll
-    for (int ks = 0; ks < TPW / 16; ++ks) {  // 16 tokens per k-step
+    for (int ks = 0; ks < 4; ++ks) {  // 16 tokens per k-step
         // A = X^T, features 16 mf + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
         R a[2][4];
 #pragma unroll
@@ -460,19 +459,24 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
                 const R x = f0 < d ? O::ld(X + (16 * ks + 8 * (r >> 1) + g) * d + f0) : O::zero();
                 a[mf][r] = O::tr(x);
             }
-        constexpr int kTok = 16;
-        const int jlo = (16 * ks / L) / 8, jhi = ((16 * ks + kTok - 1) / L) / 8;
+        const int tk = tok0 + 16 * ks;
+        const int jlo = (tk / L) / 8, jhi = ((tk + 15) / L) / 8;
 #pragma unroll
         for (int j = 0; j < NTJ; ++j) {
-            if (j < jlo || j > jhi) continue;  // compile-time after unrolling
-            // B = P^T: tokens 16 ks + 2t (+1) (+8, +9), segment 8j + g
+            if (j < jlo || j > jhi) continue;  // warp-uniform
+            // B = P^T: tokens tk + 2t (+1) (+8, +9), segment 8j + g
             auto pv = [&](int tok) -> float { return (tok / L == 8 * j + g) ? inv : 0.f; };
-            const int k0 = 16 * ks + 2 * t;
+            const int k0 = tk + 2 * t;
             const R b0 = O::pk(pv(k0), pv(k0 + 1)), b1 = O::pk(pv(k0 + 8), pv(k0 + 9));
 #pragma unroll
             for (int mf = 0; mf < 2; ++mf) O::mma(c[mf][j], a[mf], b0, b1);
         }
     }
+}
+
+template <typename T, int LPW>
+__device__ __forceinline__ void landmarks_put(const float (&c)[2][(LPW + 7) / 8][4], T* xbar, int j0, int g, int t) {
+    constexpr int NTJ = (LPW + 7) / 8, LS = 40;
 #pragma unroll
     for (int mf = 0; mf < 2; ++mf)
 #pragma unroll
@@ -484,6 +488,20 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
             }
 }
 
+// All TPW tokens of the warp (a multiple of 64), then the store.
+template <typename T, int TPW, int L>
+__device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
+    constexpr int LPW = TPW / L, NTJ = (LPW + 7) / 8;
+    float c[2][NTJ][4];
+#pragma unroll
+    for (int mf = 0; mf < 2; ++mf)
+#pragma unroll
+        for (int j = 0; j < NTJ; ++j) c[mf][j][0] = c[mf][j][1] = c[mf][j][2] = c[mf][j][3] = 0.f;
+#pragma unroll
+    for (int ch = 0; ch < TPW / 64; ++ch) landmarks_acc<T, L, LPW>(X + ch * 64 * d, ch * 64, c, d, g, t);
+    landmarks_put<T, LPW>(c, xbar, j0, g, t);
+}
+
 // Front, U side, for one warp's NCH chunks of 64 tokens: S_U = Qbar K^T with a
 // running row max, G_U^n = exp(S_U - m_U) fed straight from registers as the
 // A operand of W_r = G_U^n [V | 1] (B fragments of [V | 1 | 0] by 8x8
@@ -491,82 +509,105 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 // the max grows.  W_r (MP x NCOL) is stored at dst with row stride ws after a
 // warp sync (so every lane is done reading K and V); the row maxima (log2
 // domain) are returned in mU.
+// One 64-token chunk of the U side for one 16-landmark m-tile (A operand aq
+// = Qbar rows; v0, v1: rows g, g + 8 are real landmarks): S_U = Qbar K^T,
+// the running row maxima run0/run1 (log2 domain), w rescaled when they grow,
+// G_U^n = exp(S_U - m) fed from registers as the A operand of
+// w += G_U^n [V | 1] (B fragments of [V | 1 | 0] by 8x8 transposes; the ones
+// column yields the denominator).
+template <typename T, int NCOL>
+__device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][4], const T* Kc, const T* Vc, int d,
+                                           int g, int t, float sl2, bool v0, bool v1, float (&w)[NCOL / 8][4],
+                                           float& run0, float& run1, bool rescale) {
+    using O = Opnd<T>;
+    using R = typename O::Reg;
+    constexpr int NTO = NCOL / 8;
+    float s[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+        s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+        const T* kr = Kc + (8 * nt + g) * d;
+#pragma unroll
+        for (int kk = 0; kk < 2; ++kk) {
+            const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
+            const R b0 = c0 < d ? O::ld(kr + c0) : O::zero();
+            const R b1 = c1 < d ? O::ld(kr + c1) : O::zero();
+            O::mma(s[nt], aq[kk], b0, b1);
+        }
+    }
+    float mx0 = run0, mx1 = run1;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
+        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
+    }
+    mx0 = quad_max(mx0);
+    mx1 = quad_max(mx1);
+    if (rescale) {  // online rescaling of the accumulated rows
+        const float f0 = ex2(run0 - mx0), f1 = ex2(run1 - mx1);
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) {
+            w[j][0] *= f0; w[j][1] *= f0; w[j][2] *= f1; w[j][3] *= f1;
+        }
+    }
+    run0 = mx0;
+    run1 = mx1;
+    auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
+    auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+#pragma unroll
+    for (int kt = 0; kt < 4; ++kt) {
+        R a[4];
+        a[0] = v0 ? O::pk(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : O::zero();
+        a[1] = v1 ? O::pk(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : O::zero();
+        a[2] = v0 ? O::pk(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : O::zero();
+        a[3] = v1 ? O::pk(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : O::zero();
+#pragma unroll
+        for (int j = 0; j < NTO; ++j) {
+            const int c0 = 8 * j + 2 * t;
+            const R x0 = c0 < d ? O::ld(Vc + (16 * kt + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+            const R x1 = c0 < d ? O::ld(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+            O::mma(w[j], a, O::tr(x0), O::tr(x1));
+        }
+    }
+}
+
+// A operand registers of Qbar's m-tile mt (row stride 40).
+template <typename T>
+__device__ __forceinline__ void qbar_afrag(const T* qbar, int mt, int g, int t, typename Opnd<T>::Reg (&aq)[2][4]) {
+    using O = Opnd<T>;
+    constexpr int LS = 40;
+#pragma unroll
+    for (int kk = 0; kk < 2; ++kk) {
+        const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
+        aq[kk][0] = O::ld(r0);
+        aq[kk][1] = O::ld(r0 + 8 * LS);
+        aq[kk][2] = O::ld(r0 + 8);
+        aq[kk][3] = O::ld(r0 + 8 * LS + 8);
+    }
+}
+
+// Front, U side, for one warp's NCH chunks of 64 tokens: su_w_chunk over the
+// chunks for every landmark m-tile.  W_r (MP x NCOL) is stored at dst with
+// row stride ws after a warp sync (so every lane is done reading K and V);
+// the row maxima (log2 domain) are returned in mU.
 template <typename T, int M, int NCOL, int NCH>
 __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
                                            float* dst, int ws, float (&mU)[(M + 15) / 16][2]) {
-    using O = Opnd<T>;
-    using R = typename O::Reg;
-    constexpr int MT = (M + 15) / 16, LS = 40, NTO = NCOL / 8;
+    using R = typename Opnd<T>::Reg;
+    constexpr int MT = (M + 15) / 16, NTO = NCOL / 8;
     float wall[MT][NTO][4];
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) {
         R aq[2][4];
-#pragma unroll
-        for (int kk = 0; kk < 2; ++kk) {
-            const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-            aq[kk][0] = O::ld(r0);
-            aq[kk][1] = O::ld(r0 + 8 * LS);
-            aq[kk][2] = O::ld(r0 + 8);
-            aq[kk][3] = O::ld(r0 + 8 * LS + 8);
-        }
+        qbar_afrag<T>(qbar, mt, g, t, aq);
         const bool v0 = (16 * mt + g) < M, v1 = (16 * mt + g + 8) < M;
         float(&w)[NTO][4] = wall[mt];
 #pragma unroll
         for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
         float run0 = -INFINITY, run1 = -INFINITY;
 #pragma unroll 1
-        for (int ch = 0; ch < NCH; ++ch) {
-            const T* Kc = Ks + ch * 64 * d;
-            const T* Vc = Vs + ch * 64 * d;
-            float s[8][4];
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-                const T* kr = Kc + (8 * nt + g) * d;
-#pragma unroll
-                for (int kk = 0; kk < 2; ++kk) {
-                    const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-                    const R b0 = c0 < d ? O::ld(kr + c0) : O::zero();
-                    const R b1 = c1 < d ? O::ld(kr + c1) : O::zero();
-                    O::mma(s[nt], aq[kk], b0, b1);
-                }
-            }
-            float mx0 = run0, mx1 = run1;
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
-                mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
-            }
-            mx0 = quad_max(mx0);
-            mx1 = quad_max(mx1);
-            if (NCH > 1) {  // online rescaling of the accumulated W rows
-                const float f0 = ex2(run0 - mx0), f1 = ex2(run1 - mx1);
-#pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    w[j][0] *= f0; w[j][1] *= f0; w[j][2] *= f1; w[j][3] *= f1;
-                }
-            }
-            run0 = mx0;
-            run1 = mx1;
-            auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
-            auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
-            // B fragments of [V | 1 | 0] (k = tokens, n = columns) by 8x8 transposes.
-#pragma unroll
-            for (int kt = 0; kt < 4; ++kt) {
-                R a[4];
-                a[0] = v0 ? O::pk(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : O::zero();
-                a[1] = v1 ? O::pk(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : O::zero();
-                a[2] = v0 ? O::pk(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : O::zero();
-                a[3] = v1 ? O::pk(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : O::zero();
-#pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    const int c0 = 8 * j + 2 * t;
-                    const R x0 = c0 < d ? O::ld(Vc + (16 * kt + g) * d + c0) : (c0 == d ? O::one() : O::zero());
-                    const R x1 = c0 < d ? O::ld(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? O::one() : O::zero());
-                    O::mma(w[j], a, O::tr(x0), O::tr(x1));
-                }
-            }
-        }
+        for (int ch = 0; ch < NCH; ++ch)
+            su_w_chunk<T, NCOL>(aq, Ks + ch * 64 * d, Vs + ch * 64 * d, d, g, t, sl2, v0, v1, w, run0, run1, NCH > 1);
         mU[mt][0] = run0;
         mU[mt][1] = run1;
     }
@@ -1234,11 +1275,19 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
     T* yT = reinterpret_cast<T*>(gb + Lay::G_YT);
     uint64_t* barQK = reinterpret_cast<uint64_t*>(gb + Lay::G_BAR) + 2 * r;  // Q and K rows
     uint64_t* barV = barQK + 1;                                                // V rows
-    volatile unsigned int* gflag = reinterpret_cast<volatile unsigned int*>(gb + Lay::G_FLAG);
 
     auto gsync = [&]() {
         if constexpr (GW == 1) __syncwarp();
         else named_barrier(1 + grp, GW * 32);
+    };
+    // group barrier that also tells every warp whether any warp's wait gave up
+    auto gsync_or = [&](bool f) -> bool {
+        if constexpr (GW == 1) {
+            __syncwarp();
+            return f;
+        } else {
+            return named_barrier_or(1 + grp, GW * 32, f);
+        }
     };
     // distributed-core scratch
     unsigned char* mat0 = nullptr;
@@ -1276,7 +1325,6 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         mbar_init(barQK, 1);
         mbar_init(barV, 1);
         fence_mbar_init();
-        if (r == 0) *gflag = 0u;
     }
     gsync();
     if (tok && u < n_units && lane == 0) {
@@ -1286,17 +1334,19 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         issue_v(u);
     }
     uint32_t phase_qk = 0, phase_v = 0;
+    bool pend_qk = tok && u < n_units, pend_v = pend_qk;  // copies issued and not yet seen complete
+    bool failed = false;  // a bounded wait of this warp gave up (warp-uniform)
 
     for (; u < n_units; u += stride) {
         // ---------------- stage: bounded wait for Q and K ----------------
-        bool ok = true;
-        if (tok) {
-            ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
-            if (!ok && lane == 0) {
-                atomicOr(fault, 1u);
-                *gflag = 1u;  // the whole group stops after the next barrier
+        if (tok && !failed) {
+            if (__all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs))) {
+                phase_qk ^= 1u;
+                pend_qk = false;
+            } else {
+                failed = true;  // the whole group stops at the next barrier
+                if (lane == 0) atomicOr(fault, 1u);
             }
-            phase_qk ^= 1u;
         }
 
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
@@ -1311,8 +1361,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                 }
             }
         }
-        gsync();
-        if (GW == 1 ? !ok : (*gflag != 0u)) break;
+        if (gsync_or(failed)) break;
 
         // ---------------- front [P1]: S_L, G_L^n fragments ----------------
         if (GLS && tok) {
@@ -1329,16 +1378,16 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         }
 
         // ---------------- stage: bounded wait for V ----------------
-        bool ok_v = true;
-        if (tok) {
-            ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
-            if (!ok_v && lane == 0) {
-                atomicOr(fault, 1u);
-                *gflag = 1u;
+        if (tok && !failed) {
+            if (__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs))) {
+                phase_v ^= 1u;
+                pend_v = false;
+            } else {
+                failed = true;
+                if (lane == 0) atomicOr(fault, 1u);
             }
-            phase_v ^= 1u;
         }
-        if (GW == 1 && !ok_v) break;
+        if (GW == 1 && failed) break;
 
         // ------- front: S_U, running m_U, G_U^n, W_r = G_U^n [V | 1] -------
         float mU[MT][2];  // this warp's row maxima of S_U, log2 domain
@@ -1363,8 +1412,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                                                    (size_t)(grp * WPU) * Lay::WARP_BYTES + Lay::WPART),
                     Lay::WARP_BYTES / 4, mW, gmu, r, lane);
         }
-        gsync();
-        if (GW > 1 && *gflag != 0u) break;
+        if (gsync_or(failed)) break;
 
         // Q and K of this unit are consumed (in P2 Q stays for the output):
         // prefetch the next unit's rows.  V's region holds the output first.
@@ -1373,10 +1421,13 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
         auto prefetch_qk = [&]() {
             fence_proxy_async_smem();  // this lane's reads of Q/K precede the async refill
             __syncwarp();
-            if (tok && un < n_units && lane == 0) {
-                arm_qk();
-                if constexpr (GLS) issue_q(un);
-                issue_k(un);
+            if (tok && un < n_units && !failed) {
+                if (lane == 0) {
+                    arm_qk();
+                    if constexpr (GLS) issue_q(un);
+                    issue_k(un);
+                }
+                pend_qk = true;
             }
         };
         if constexpr (!Lay::SCR_IN_STAGE) prefetch_qk();
@@ -1421,13 +1472,19 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             fence_proxy_async_smem();  // reads of Q precede its refill
             gsync();
         }
-        if (tok && un < n_units && lane == 0) {
-            if constexpr (!GLS) issue_q(un);
-            issue_v(un);
+        if (tok && un < n_units && !failed) {
+            if (lane == 0) {
+                if constexpr (!GLS) issue_q(un);
+                issue_v(un);
+            }
+            pend_v = true;
         }
         __syncwarp();
     }
     if (tok && lane == 0) bulk_wait_all();  // outstanding output stores complete before exit
+    // Fault path only: copies still in flight land before the CTA's memory is released.
+    if (tok && pend_qk) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
+    if (tok && pend_v) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
 }
 
 // Largest number of groups per CTA that fits the shared-memory and register
@@ -1508,6 +1565,11 @@ cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, l
     return cudaErrorInvalidValue;
 }
 
+// Streaming team kernel for 32x32 windows (nystra_stream.cuh, N = 1024 translation unit only).
+template <typename T, int M, int NCOL>
+cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                          int iters, cudaStream_t stream, unsigned int* fault);
+
 // Dispatch on m and the output-column padding for one window size.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
@@ -1528,6 +1590,14 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
         if (m == 16)
             return wide ? launch_team<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_team<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    if constexpr (TPW == 128 && WPU == 8) {
+        if (m == 8)
+            return wide ? launch_stream<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_stream<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (m == 16)
+            return wide ? launch_stream<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_stream<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
     switch (m) {
         case 8:

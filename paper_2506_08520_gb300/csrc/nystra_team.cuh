@@ -19,8 +19,9 @@
 // Core warp, unit k: wait F_b -> G_A^n, iteration, Y^T into buffer b ->
 //   signal C_b.
 // [sync] is a named barrier over the four token warps.  Every wait on an
-// mbarrier is bounded; a failed wait sets the team's flag, and the token
-// warps leave the loop together at the flag checks after a barrier.
+// mbarrier is bounded; a warp whose wait gives up keeps to the barrier
+// sequence, and the token warps leave the loop together after the next
+// barrier, whose OR-reduction gives every warp the same verdict.
 #pragma once
 
 #include "nystra_tc.cuh"
@@ -47,7 +48,7 @@ struct TeamLayout {
     static constexpr size_t B_YT = B_MU + MP * 4;
     static constexpr size_t B_GLF = B_YT + ((NCOL * YS * 2 + 15) / 16) * 16;
     static constexpr size_t BUF = B_GLF + NT * GLF_W;
-    // team memory: stages, two buffers, mbarriers, flag
+    // team memory: stages, two buffers, mbarriers
     static constexpr size_t T_BUF = NT * STAGE;
     static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // barQK[4], barV[4], F[2], C[2]
     static constexpr size_t T_FLAG = T_BAR + 12 * 8;
@@ -76,7 +77,6 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     uint64_t* bars = reinterpret_cast<uint64_t*>(tb + Lay::T_BAR);
     uint64_t* barF = bars + 8;  // F[b]: the token warps' state for the core is ready
     uint64_t* barC = bars + 10; // C[b]: the core's Y^T is ready
-    volatile unsigned int* flag = reinterpret_cast<volatile unsigned int*>(tb + Lay::T_FLAG);
 
     const long long stride = (long long)gridDim.x * Lay::TEAMS;
     const long long u0 = (long long)blockIdx.x * Lay::TEAMS + team;
@@ -89,7 +89,6 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             mbar_init(bb + 9, NT);
             mbar_init(bb + 10, 1);
             mbar_init(bb + 11, 1);
-            *reinterpret_cast<volatile unsigned int*>(smem_raw + (size_t)tm * Lay::TEAM + Lay::T_FLAG) = 0u;
         }
         fence_mbar_init();
     }
@@ -114,14 +113,10 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             const int b = (int)(kk & 1);
             const uint32_t par = (uint32_t)((kk >> 1) & 1);
             const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, par, kWaitNs));
-            if (!ok) {
-                if (lane == 0) {
-                    atomicOr(fault, 1u);
-                    *flag = 1u;
-                }
+            if (!ok) {  // the token warps stopped (or stalled): stop too
+                if (lane == 0) atomicOr(fault, 1u);
                 break;
             }
-            if (*flag != 0u) break;
             unsigned char* bb = buf(b);
             const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
             float mU[1][2] = {{gmu[g], gmu[g + 8]}};
@@ -154,19 +149,21 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         bulk_g2s(Vs, v + unit_off(unit), tile_bytes, barV);
     };
     auto tsync = [&]() { named_barrier(1 + team, NT * 32); };
+    // barrier that also tells every token warp whether any of them failed
+    auto tsync_or = [&](bool f) { return named_barrier_or(1 + team, NT * 32, f); };
     uint32_t phase_qk = 0, phase_v = 0;
-    bool pend_qk = false, pend_v = false;  // copies issued and not yet waited for
+    bool pend_qk = false, pend_v = false;  // copies issued and not yet seen complete
+    bool failed = false;                   // a bounded wait of this warp gave up (warp-uniform)
 
     // Output of unit kk (its core has run on buffer kk mod 2), staged in the
     // V rows; returns once the bulk store has read the staging.
     auto output_unit = [&](long long kk) {
         const int b = (int)(kk & 1);
+        if (failed) return;
         const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barC + b, (uint32_t)((kk >> 1) & 1), kWaitNs));
         if (!ok) {
-            if (lane == 0) {
-                atomicOr(fault, 1u);
-                *flag = 1u;
-            }
+            failed = true;
+            if (lane == 0) atomicOr(fault, 1u);
             return;
         }
         unsigned char* bb = buf(b);
@@ -197,18 +194,20 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         T* qbar = reinterpret_cast<T*>(bb + Lay::B_QB);
         T* kbar = reinterpret_cast<T*>(bb + Lay::B_KB);
         // ---------------- bounded wait for Q and K ----------------
-        const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
-        if (!ok && lane == 0) {
-            atomicOr(fault, 1u);
-            *flag = 1u;
+        if (!failed) {
+            const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
+            if (ok) {
+                phase_qk ^= 1u;
+                pend_qk = false;
+            } else {
+                failed = true;
+                if (lane == 0) atomicOr(fault, 1u);
+            }
         }
-        phase_qk ^= 1u;
-        pend_qk = !ok;
         // ---------------- landmarks (Algorithm 1 step 1) ----------------
         landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
         landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
-        tsync();
-        if (*flag != 0u) break;
+        if (tsync_or(failed)) break;
         // ---------------- S_L, G_L^n fragments parked in buffer b ----------------
         {
             uint32_t* glf = reinterpret_cast<uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W);
@@ -221,13 +220,16 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             }
         }
         // ---------------- bounded wait for V ----------------
-        const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
-        if (!ok_v && lane == 0) {
-            atomicOr(fault, 1u);
-            *flag = 1u;
+        if (!failed) {
+            const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
+            if (ok_v) {
+                phase_v ^= 1u;
+                pend_v = false;
+            } else {
+                failed = true;
+                if (lane == 0) atomicOr(fault, 1u);
+            }
         }
-        phase_v ^= 1u;
-        pend_v = !ok_v;
         // ---------------- S_U, partial W_r and row maxima ----------------
         float mU[1][2];
         front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU);
@@ -239,8 +241,7 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         combine_partials<MP, NCOLC, WS, NT>(reinterpret_cast<const float*>(tb + Lay::WPART), Lay::STAGE / 4,
                                              reinterpret_cast<float*>(bb + Lay::B_W),
                                              reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
-        tsync();
-        if (*flag != 0u) break;
+        if (tsync_or(failed)) break;
         // ---------------- hand buffer b to the core warp ----------------
         __syncwarp();
         if (lane == 0) mbar_arrive(barF + b);
@@ -248,15 +249,19 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         const long long un = u + stride;
         fence_proxy_async_smem();
         __syncwarp();
-        if (un < n_units && lane == 0) issue_qk(un);
-        pend_qk = pend_qk || un < n_units;
+        if (un < n_units && !failed) {
+            if (lane == 0) issue_qk(un);
+            pend_qk = true;
+        }
         // ---------------- output of the previous unit ----------------
         if (kk >= 1) output_unit(kk - 1);
         // The V rows are free (consumed, and the staging has been read).
-        if (un < n_units && lane == 0) issue_v(un);
-        pend_v = pend_v || un < n_units;
+        if (un < n_units && !failed) {
+            if (lane == 0) issue_v(un);
+            pend_v = true;
+        }
     }
-    if (kk >= 1 && *flag == 0u) output_unit(kk - 1);
+    if (kk >= 1) output_unit(kk - 1);
     if (lane == 0) bulk_wait_all();  // output stores complete before exit
     // Fault path only: copies still in flight land before the CTA's memory is released.
     if (pend_qk) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
