@@ -41,7 +41,8 @@ struct StreamLayout {
     static constexpr int L = N / M, LPW = TPW / L;  // tokens per segment, segments per token warp
     static constexpr size_t XB = (size_t)CH * DS * 2;  // one tensor's chunk
     static constexpr size_t SLOT = 2 * XB;             // K and V (Q uses the first half)
-    static constexpr size_t WPB = (((size_t)MP * WS * 4 + MP * 4) + 127) / 128 * 128;  // W partial, row maxima
+    static constexpr size_t WPB = (size_t)MP * WS * 4 + MP * 4;  // W partial, row maxima
+    static_assert(WPB <= XB, "the W partial lives in the V half of the last KV chunk's slot");
     // per-unit state
     static constexpr size_t B_QB = 0;
     static constexpr size_t B_KB = B_QB + MP * LS * 2;
@@ -51,16 +52,18 @@ struct StreamLayout {
     static constexpr size_t BUF = ((B_YT + NCOL * YS * 2 + 127) / 128) * 128;
     template <int S>
     struct Team {
-        static constexpr size_t WARP = S * SLOT + WPB;  // ring, then the W partial
+        static constexpr size_t WARP = S * SLOT;  // a token warp's ring of chunk buffers
         static constexpr size_t T_BUF = NT * WARP;
         static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // slot bars [NT][S], F[2], C[2]
         static constexpr size_t BYTES = ((T_BAR + (NT * S + 4) * 8 + 127) / 128) * 128;
     };
-    static constexpr int TEAMS = 2;
-    static constexpr int NSLOT = (TEAMS * Team<3>::BYTES <= kSmemLimit) ? 3 : 2;
+    // three teams with two-deep rings when they fit, else two with three-deep
+    static constexpr bool kThree = 3 * Team<2>::BYTES <= kSmemLimit;
+    static constexpr int TEAMS = kThree ? 3 : 2;
+    static constexpr int NSLOT = kThree ? 2 : 3;
     using TL = Team<NSLOT>;
     static constexpr size_t TEAM = TL::BYTES;
-    static_assert(TEAMS * TEAM <= kSmemLimit, "two teams must fit");
+    static_assert(TEAMS * TEAM <= kSmemLimit, "teams must fit");
     static_assert(M <= 16 && L >= 16 && LPW <= 8, "segments per token warp fit one n-tile");
     static_assert(XB % 16 == 0 && SLOT % 16 == 0 && TL::WARP % 16 == 0 && BUF % 16 == 0, "16-byte alignment");
 };
@@ -154,7 +157,6 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
 
     // ======================= token warp r =======================
     unsigned char* wr = tb + (size_t)r * TL::WARP;
-    float* wpart = reinterpret_cast<float*>(wr + NSLOT * Lay::SLOT);
     uint64_t* sbar = bars + r * NSLOT;
     const uint32_t xbytes = (uint32_t)(Lay::CH * d * sizeof(T));
     auto slot_x = [&](int s, int h) { return reinterpret_cast<T*>(wr + (size_t)s * Lay::SLOT + h * Lay::XB); };
@@ -231,6 +233,9 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             su_w_chunk<T, NCOL>(aq, X0, slot_x(s, 1), d, g, t, sl2, g < M, g + 8 < M, w, run0, run1, true);
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(ck, reinterpret_cast<T*>(bb + Lay::B_KB), r * LPW, g, t);
+                // the partial goes over this slot's V rows, consumed above
+                float* wpart = reinterpret_cast<float*>(slot_x(s, 1));
+                __syncwarp();
 #pragma unroll
                 for (int j = 0; j < NTO; ++j) {
                     const int c = 8 * j + 2 * t;
@@ -242,7 +247,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                     wpart[MP * WS + g + 8] = run1;
                 }
                 tsync();
-                combine_partials<MP, NCOL, WS, NT>(reinterpret_cast<const float*>(tb + NSLOT * Lay::SLOT),
+                combine_partials<MP, NCOL, WS, NT>(reinterpret_cast<const float*>(tb + (size_t)s * Lay::SLOT + Lay::XB),
                                                     TL::WARP / 4, reinterpret_cast<float*>(bb + Lay::B_W),
                                                     reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
                 if (tsync_or(failed)) break;
