@@ -285,13 +285,12 @@ __device__ __forceinline__ void transpose_hfrag(const HFrag<MT>& a, HFrag<MT>& b
 }
 
 // D = s I + A P^T (+ c I P^T when CI; i7 holds the A operand register of
-// c I's diagonal blocks) with fp16 two-term split operands: lo*hi + hi*lo
-// and hi*hi accumulate separately (shorter dependent chains).
+// c I's diagonal blocks) with fp16 two-term split operands, one fp32
+// accumulator per tile: the small terms lo*hi and hi*lo first, then hi*hi.
 template <int MT, bool CI>
 __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Frag<MT>& D, float s, uint32_t i7,
                                       int g, int t) {
     using H = Mma16<__half>;
-    float small[MT][2 * MT][4], big[MT][2 * MT][4];
 #pragma unroll
     for (int i = 0; i < MT; ++i)
 #pragma unroll
@@ -299,8 +298,7 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * j + (e & 1) + 2 * t);
-                big[i][j][e] = diag ? s : 0.f;
-                small[i][j][e] = 0.f;
+                D[i][j][e] = diag ? s : 0.f;
             }
 #pragma unroll
     for (int kk = 0; kk < MT; ++kk)
@@ -311,22 +309,19 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
             for (int i = 0; i < MT; ++i) {
                 const uint32_t ahi[4] = {A[i][kk][0].hi, A[i][kk][1].hi, A[i][kk][2].hi, A[i][kk][3].hi};
                 const uint32_t alo[4] = {A[i][kk][0].lo, A[i][kk][1].lo, A[i][kk][2].lo, A[i][kk][3].lo};
-                H::k16(small[i][j], alo, b0.hi, b1.hi);
-                H::k16(small[i][j], ahi, b0.lo, b1.lo);
-                H::k16(big[i][j], ahi, b0.hi, b1.hi);
                 if (CI && kk == i) {
                     const uint32_t ci[4] = {i7, 0u, 0u, i7};
-                    H::k16(big[i][j], ci, b0.hi, b1.hi);
-                    H::k16(small[i][j], ci, b0.lo, b1.lo);
+                    H::k16(D[i][j], ci, b0.lo, b1.lo);
                 }
+                H::k16(D[i][j], alo, b0.hi, b1.hi);
+                H::k16(D[i][j], ahi, b0.lo, b1.lo);
+                if (CI && kk == i) {
+                    const uint32_t ci[4] = {i7, 0u, 0u, i7};
+                    H::k16(D[i][j], ci, b0.hi, b1.hi);
+                }
+                H::k16(D[i][j], ahi, b0.hi, b1.hi);
             }
         }
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) D[i][j][e] = big[i][j][e] + small[i][j][e];
 }
 
 // S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
