@@ -29,6 +29,15 @@ SMALL = [
     (3, 256, 30, 64),
     (2, 1024, 32, 32),
     (2, 1024, 32, 64),
+    # few units (teams and pool warps left idle), ragged counts, narrow heads
+    (1, 64, 30, 8),
+    (13, 64, 30, 16),
+    (1, 256, 30, 16),
+    (5, 256, 32, 8),
+    (3, 256, 8, 16),
+    (1, 1024, 32, 8),
+    (3, 1024, 30, 16),
+    (2, 1024, 16, 16),
     (4, 48, 20, 12),     # odd sizes
     (3, 10, 3, 5),
     (6, 128, 64, 16),    # widest head
