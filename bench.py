@@ -35,8 +35,10 @@ METRIC = "Nystrom attention tokens*heads/s"
 # for the sources of the kernel they were taken with: reported as null once any
 # of those files changes.
 MEASURED_TRAFFIC = {
-    "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
-                       "src_hash": "4210bd8380471295", "bytes": 74_102_784},
+    "sr720p-w16-m16-bf16": {"files": ['common.cuh', 'nystra_team.cuh', 'nystra_tc.cuh', 'nystra_tc_n256.cu', 'ptx.cuh'],
+                            "src_hash": "9f800de2a1421374", "bytes": 1_296_393_984},
+    "sr720p-w32-m16-bf16": {"files": ['common.cuh', 'nystra_stream.cuh', 'nystra_tc.cuh', 'nystra_tc_n1024.cu', 'ptx.cuh'],
+                            "src_hash": "b759fc9b6a571ab1", "bytes": 1_481_127_680},
 }
 
 
