@@ -57,10 +57,11 @@ struct PoolLayout {
     static_assert(BYTES <= kSmemLimit, "pool does not fit in shared memory");
 };
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int DC>
 __global__ void __launch_bounds__(PoolLayout<T, M, NCOL>::NW * 32, 1)
 nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, T* __restrict__ out,
-                   long long n_units, int d, int iters, float sl2, unsigned int* fault) {
+                   long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+    const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using P = PoolLayout<T, M, NCOL>;
     constexpr int L = 64 / M;  // tokens per landmark segment
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -165,11 +166,11 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (*cnt > consumed) (void)__all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
 }
 
-template <typename T, int M, int NCOL>
-cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+template <typename T, int M, int NCOL, int DC>
+cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault) {
     using P = PoolLayout<T, M, NCOL>;
-    auto kern = nystra_pool_kernel<T, M, NCOL>;
+    auto kern = nystra_pool_kernel<T, M, NCOL, DC>;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
@@ -187,6 +188,19 @@ cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, 
     kern<<<(unsigned)grid, P::NW * 32, P::BYTES, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                              n_units, d, iters, sl2, fault);
     return cudaGetLastError();
+}
+
+// The common head widths get kernels with d_h as a compile-time constant
+// (constant strides and column bounds); others read it at run time.
+template <typename T, int M, int NCOL>
+cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                     int iters, cudaStream_t stream, unsigned int* fault) {
+    if constexpr (NCOL == 32) {
+        if (d == 30) return launch_pool_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+    } else {
+        if (d == 32) return launch_pool_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    return launch_pool_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc

@@ -84,10 +84,11 @@ __device__ __forceinline__ StreamTask stream_task(int v, int count) {
     return {k - 1, 2, r & 3};
 }
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int DC>
 __global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
 nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-                     T* __restrict__ out, long long n_units, int d, int iters, float sl2, unsigned int* fault) {
+                     T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+    const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using Lay = StreamLayout<M, NCOL>;
     using TL = typename Lay::TL;
     using R = typename Opnd<T>::Reg;
@@ -290,11 +291,11 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
         (void)__all_sync(0xffffffffu, mbar_wait_bounded(sbar + i % NSLOT, (uint32_t)((i / NSLOT) & 1), kWaitNs));
 }
 
-template <typename T, int M, int NCOL>
-cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+template <typename T, int M, int NCOL, int DC>
+cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                           int iters, cudaStream_t stream, unsigned int* fault) {
     using Lay = StreamLayout<M, NCOL>;
-    auto kern = nystra_stream_kernel<T, M, NCOL>;
+    auto kern = nystra_stream_kernel<T, M, NCOL, DC>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -315,6 +316,19 @@ cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out
     kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                                  n_units, d, iters, sl2, fault);
     return cudaGetLastError();
+}
+
+// The common head widths get kernels with d_h as a compile-time constant
+// (constant strides and column bounds); others read it at run time.
+template <typename T, int M, int NCOL>
+cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                     int iters, cudaStream_t stream, unsigned int* fault) {
+    if constexpr (NCOL == 32) {
+        if (d == 30) return launch_stream_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+    } else {
+        if (d == 32) return launch_stream_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    return launch_stream_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc

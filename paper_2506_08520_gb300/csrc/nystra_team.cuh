@@ -58,10 +58,11 @@ struct TeamLayout {
     static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
 };
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int DC>
 __global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
 nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-                   T* __restrict__ out, long long n_units, int d, int iters, float sl2, unsigned int* fault) {
+                   T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+    const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using Lay = TeamLayout<M, NCOL>;
     constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
                   KTL = Lay::KTL, NCOLC = NCOL;
@@ -268,11 +269,11 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (pend_v) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
 }
 
-template <typename T, int M, int NCOL>
-cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+template <typename T, int M, int NCOL, int DC>
+cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault) {
     using Lay = TeamLayout<M, NCOL>;
-    auto kern = nystra_team_kernel<T, M, NCOL>;
+    auto kern = nystra_team_kernel<T, M, NCOL, DC>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -293,6 +294,19 @@ cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, 
     kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                                  n_units, d, iters, sl2, fault);
     return cudaGetLastError();
+}
+
+// The common head widths get kernels with d_h as a compile-time constant
+// (constant strides and column bounds); others read it at run time.
+template <typename T, int M, int NCOL>
+cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                     int iters, cudaStream_t stream, unsigned int* fault) {
+    if constexpr (NCOL == 32) {
+        if (d == 30) return launch_team_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+    } else {
+        if (d == 32) return launch_team_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    return launch_team_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc
