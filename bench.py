@@ -35,10 +35,8 @@ METRIC = "Nystrom attention tokens*heads/s"
 # for the sources of the kernel they were taken with: reported as null once any
 # of those files changes.
 MEASURED_TRAFFIC = {
-    "sr720p-w16-m16-bf16": {"files": ['common.cuh', 'nystra_team.cuh', 'nystra_tc.cuh', 'nystra_tc_n256.cu', 'ptx.cuh'],
-                            "src_hash": "9f800de2a1421374", "bytes": 1_296_393_984},
-    "sr720p-w32-m16-bf16": {"files": ['common.cuh', 'nystra_stream.cuh', 'nystra_tc.cuh', 'nystra_tc_n1024.cu', 'ptx.cuh'],
-                            "src_hash": "b759fc9b6a571ab1", "bytes": 1_481_127_680},
+    "swinir256-bf16": {"files": ['common.cuh', 'nystra_pool.cuh', 'nystra_tc.cuh', 'nystra_tc_n64.cu', 'ptx.cuh'],
+                       "src_hash": "b5c70ca59f223184", "bytes": 73_732_096},
 }
 
 
