@@ -1585,6 +1585,9 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
         if (m == 16)
             return wide ? launch_team<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_team<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        // m = 32 with d_h <= 30 fits two teams per SM; d_h = 32 only one, so it
+        // stays on the grouped kernel
+        if (m == 32 && !wide) return launch_team<T, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
     if constexpr (TPW == 128 && WPU == 8) {
         if (m == 8)

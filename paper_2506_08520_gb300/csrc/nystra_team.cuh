@@ -1,5 +1,5 @@
-// Team PnP-Nystra kernel for 16x16 windows (N = 256 tokens), m <= 16, even
-// d_h <= 32, 16-bit I/O.  Included by the N = 256 translation unit after
+// Team PnP-Nystra kernel for 16x16 windows (N = 256 tokens), m <= 32, even
+// d_h <= 32, 16-bit I/O (m = 32: the core runs on two warps, dist_core).  Included by the N = 256 translation unit after
 // nystra_tc.cuh, whose per-phase device functions it reuses.
 //
 // In the grouped kernel the m x m core runs on one warp of a unit's group
@@ -32,8 +32,9 @@ namespace tc {
 template <int M, int NCOL>
 struct TeamLayout {
     static constexpr int NT = 4, TPW = 64, N = NT * TPW;  // token warps, tokens per token warp
+    static constexpr int CWN = M > 16 ? M / 16 : 1;        // core warps (m = 32: distributed core)
     static constexpr int DS = (NCOL == 32) ? 30 : 32;
-    static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int MP = M > 16 ? M : 16, LS = 40, WS = NCOL + 4, YS = MP + 8;
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;
     static constexpr int GLB = (M >= 16) ? 16 : 8;
     static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;  // a token warp's Q, K, V rows
@@ -51,15 +52,17 @@ struct TeamLayout {
     // team memory: stages, two buffers, mbarriers
     static constexpr size_t T_BUF = NT * STAGE;
     static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // barQK[4], barV[4], F[2], C[2]
-    static constexpr size_t T_FLAG = T_BAR + 12 * 8;
-    static constexpr size_t TEAM = ((T_FLAG + 16 + 127) / 128) * 128;
+    static constexpr size_t T_SCR = ((T_BAR + 12 * 8 + 127) / 128) * 128;  // distributed core's scratch
+    static constexpr size_t TEAM =
+        ((T_SCR + (CWN > 1 ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0) + 127) / 128) * 128;
     static constexpr int TEAMS = (int)(kSmemLimit / TEAM) < 3 ? (int)(kSmemLimit / TEAM) : 3;
+    static constexpr int WARPS = NT + CWN;  // per team
     static_assert(TEAMS >= 1, "team does not fit in shared memory");
     static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
 };
 
 template <typename T, int M, int NCOL, int DC>
-__global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
+__global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * TeamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                    T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
@@ -71,7 +74,7 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int team = warp / (NT + 1), r = warp - team * (NT + 1);  // r == NT: core warp
+    const int team = warp / Lay::WARPS, r = warp - team * Lay::WARPS;  // r >= NT: core warps
     const int g = lane >> 2, t = lane & 3;
     unsigned char* tb = smem_raw + (size_t)team * Lay::TEAM;
     auto buf = [&](int b) { return tb + Lay::T_BUF + (size_t)b * Lay::BUF; };
@@ -88,8 +91,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             for (int i = 0; i < 8; ++i) mbar_init(bb + i, 1);
             mbar_init(bb + 8, NT);
             mbar_init(bb + 9, NT);
-            mbar_init(bb + 10, 1);
-            mbar_init(bb + 11, 1);
+            mbar_init(bb + 10, Lay::CWN);
+            mbar_init(bb + 11, Lay::CWN);
         }
         fence_mbar_init();
     }
@@ -106,24 +109,38 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     }
     __syncthreads();
 
-    if (r == NT) {
-        // ======================= core warp =======================
+    if (r >= NT) {
+        // ======================= core warp(s) =======================
+        const int c = r - NT;
         for (long long kk = 0;; ++kk) {
             const long long u = u0 + kk * stride;
             if (u >= n_units) break;
             const int b = (int)(kk & 1);
             const uint32_t par = (uint32_t)((kk >> 1) & 1);
-            const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, par, kWaitNs));
+            bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, par, kWaitNs));
+            if constexpr (Lay::CWN > 1)  // the core warps decide together
+                ok = !named_barrier_or(1 + Lay::TEAMS + team, Lay::CWN * 32, !ok);
             if (!ok) {  // the token warps stopped (or stalled): stop too
                 if (lane == 0) atomicOr(fault, 1u);
                 break;
             }
             unsigned char* bb = buf(b);
             const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
-            float mU[1][2] = {{gmu[g], gmu[g + 8]}};
-            core_warp<T, M, NCOLC>(reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB),
-                                   mU, reinterpret_cast<const float*>(bb + Lay::B_W),
-                                   reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            if constexpr (Lay::CWN == 1) {
+                float mU[1][2] = {{gmu[g], gmu[g + 8]}};
+                core_warp<T, M, NCOLC>(reinterpret_cast<const T*>(bb + Lay::B_QB),
+                                       reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
+                                       reinterpret_cast<const float*>(bb + Lay::B_W),
+                                       reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            } else {
+                using DSc = DistScratch<(M > 16 ? M : 32)>;
+                unsigned char* scr = tb + Lay::T_SCR;
+                dist_core<T, (M > 16 ? M : 32), NCOLC>(
+                    reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB), gmu,
+                    reinterpret_cast<const float*>(bb + Lay::B_W), reinterpret_cast<T*>(bb + Lay::B_YT), scr,
+                    scr + DSc::MAT, reinterpret_cast<float*>(scr + 2 * DSc::MAT), iters, sl2, c, lane,
+                    1 + Lay::TEAMS + team);
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive(barC + b);
         }
@@ -232,11 +249,15 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             }
         }
         // ---------------- S_U, partial W_r and row maxima ----------------
-        float mU[1][2];
+        constexpr int MT = (M + 15) / 16;
+        float mU[MT][2];
         front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU);
         if (t == 0) {
-            wpart[MP * WS + g] = mU[0][0];
-            wpart[MP * WS + g + 8] = mU[0][1];
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+                wpart[MP * WS + 16 * mt + g] = mU[mt][0];
+                wpart[MP * WS + 16 * mt + g + 8] = mU[mt][1];
+            }
         }
         tsync();
         combine_partials<MP, NCOLC, WS, NT>(reinterpret_cast<const float*>(tb + Lay::WPART), Lay::STAGE / 4,
@@ -282,7 +303,7 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
         int dev = 0, sms = 0, per_sm = 0;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
         if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * 5 * 32, smem)) !=
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * Lay::WARPS * 32, smem)) !=
             cudaSuccess)
             return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
@@ -291,7 +312,7 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
     const long long want = (n_units + Lay::TEAMS - 1) / Lay::TEAMS;
     const long long grid = want < s_blocks ? want : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
-    kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
+    kern<<<(unsigned)grid, Lay::TEAMS * Lay::WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                                  n_units, d, iters, sl2, fault);
     return cudaGetLastError();
 }
