@@ -27,7 +27,7 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from paper_2506_08520_gb300 import binding, workloads  # noqa: E402
+from paper_2506_08520_gb300 import binding, shard, workloads  # noqa: E402
 
 METRIC = "Nystrom attention tokens*heads/s"
 
@@ -235,12 +235,9 @@ def run_cuda(args, wl):
         barrier()
     total_ms = starts[0].elapsed_time(ends[-1])
     kern_ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
-    t = torch.tensor([total_ms], device=dev)
-    if ws > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = shard.max_over_ranks(total_ms, dev)
     units_tokens = wl.n_windows * wl.heads * wl.N
-    value = ws * units_tokens * args.steps / (total_ms * 1e-3)
+    value = shard.aggregate_rate(units_tokens, args.steps, total_ms, ws)
 
     # exact window attention on the same inputs (the computation replaced)
     esteps = max(3, min(args.steps, 200))
@@ -272,11 +269,8 @@ def run_cuda(args, wl):
         ho.copy_(do, non_blocking=True)
     e1.record(stream)
     barrier()
-    e2e_ms = e0.elapsed_time(e1) / e2e_steps
-    t = torch.tensor([e2e_ms], device=dev)
-    if ws > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    e2e_value = ws * units_tokens / (float(t.item()) * 1e-3)
+    e2e_ms = shard.max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dev)
+    e2e_value = shard.aggregate_rate(units_tokens, 1, e2e_ms, ws)
 
     peak, peak_kind = _peaks()
     achieved = io_bytes / (kern_ms * 1e-3) / 1e9
