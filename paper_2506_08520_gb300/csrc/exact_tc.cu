@@ -1,5 +1,6 @@
 // Tensor-core exact window attention, Eq. 1: O = softmax(Q K^T / sqrt(d_h)) V,
-// 16-bit I/O, windows of N = 64, 256 or 1024 tokens, even d_h <= 32.
+// even d_h <= 32; 16-bit I/O for windows of N = 64, 256 or 1024 tokens, fp32
+// I/O (split bf16 operands, three MMAs per product) for N = 64 and 256.
 //
 // A group of WPU = N/64 warps processes one (window, head) unit; warp r
 // bulk-copies rows [64r, 64r+64) of Q, K and V into its private stage (one
@@ -24,15 +25,10 @@ namespace {
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr size_t kSmemLimit = 232448;
 
-template <typename T>
-__device__ __forceinline__ uint32_t ld32x(const T* p) {
-    return *reinterpret_cast<const uint32_t*>(p);
-}
-
-template <int NCOL, int WPU>
+template <typename T, int NCOL, int WPU>
 struct ExactLayout {
     static constexpr int DS = (NCOL == 32) ? 30 : 32;
-    static constexpr size_t STAGE = 3 * 64 * (size_t)DS * 2;
+    static constexpr size_t STAGE = 3 * 64 * (size_t)DS * sizeof(T);
     static constexpr size_t WARP_BYTES = ((STAGE + 127) / 128) * 128;
     static constexpr size_t GROUP_BYTES = ((8 * WPU + 16 + 127) / 128) * 128;  // mbarriers + flag
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
@@ -42,8 +38,9 @@ template <typename T, int NCOL, int WPU, int GROUPS>
 __global__ void __launch_bounds__(GROUPS * WPU * 32, 1)
 exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                 T* __restrict__ out, long long n_units, int d, float sl2, unsigned int* fault) {
-    using Lay = ExactLayout<NCOL, WPU>;
-    using Op = Mma16<T>;
+    using Lay = ExactLayout<T, NCOL, WPU>;
+    using O = Opnd<T>;
+    using R = typename O::Reg;
     constexpr int N = 64 * WPU, NTO = NCOL / 8;
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -94,16 +91,16 @@ exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __res
         T* obase = out + (size_t)u * N * d + (size_t)r * td;
 #pragma unroll 1
         for (int tm = 0; tm < 4; ++tm) {
-            uint32_t aq[2][4];
+            R aq[2][4];
             const T* q0 = Qs + (16 * tm + g) * d;
             const T* q1 = q0 + 8 * d;
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
                 const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-                aq[kk][0] = c0 < d ? ld32x(q0 + c0) : 0u;
-                aq[kk][1] = c0 < d ? ld32x(q1 + c0) : 0u;
-                aq[kk][2] = c1 < d ? ld32x(q0 + c1) : 0u;
-                aq[kk][3] = c1 < d ? ld32x(q1 + c1) : 0u;
+                aq[kk][0] = c0 < d ? O::ld(q0 + c0) : O::zero();
+                aq[kk][1] = c0 < d ? O::ld(q1 + c0) : O::zero();
+                aq[kk][2] = c1 < d ? O::ld(q0 + c1) : O::zero();
+                aq[kk][3] = c1 < d ? O::ld(q1 + c1) : O::zero();
             }
             float o[NTO][4];
 #pragma unroll
@@ -121,7 +118,8 @@ exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __res
 #pragma unroll
                     for (int kk = 0; kk < 2; ++kk) {
                         const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
-                        Op::k16(s[nt], aq[kk], c0 < d ? ld32x(kr + c0) : 0u, c1 < d ? ld32x(kr + c1) : 0u);
+                        O::mma(s[nt], aq[kk], c0 < d ? O::ld(kr + c0) : O::zero(),
+                               c1 < d ? O::ld(kr + c1) : O::zero());
                     }
                 }
                 float mx0 = run0, mx1 = run1;
@@ -141,18 +139,18 @@ exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __res
                 run1 = mx1;
 #pragma unroll
                 for (int kt = 0; kt < 4; ++kt) {
-                    uint32_t a[4];
-                    a[0] = Op::pack(ex2(fmaf(s[2 * kt][0], sl2, -mx0)), ex2(fmaf(s[2 * kt][1], sl2, -mx0)));
-                    a[1] = Op::pack(ex2(fmaf(s[2 * kt][2], sl2, -mx1)), ex2(fmaf(s[2 * kt][3], sl2, -mx1)));
-                    a[2] = Op::pack(ex2(fmaf(s[2 * kt + 1][0], sl2, -mx0)), ex2(fmaf(s[2 * kt + 1][1], sl2, -mx0)));
-                    a[3] = Op::pack(ex2(fmaf(s[2 * kt + 1][2], sl2, -mx1)), ex2(fmaf(s[2 * kt + 1][3], sl2, -mx1)));
+                    R a[4];
+                    a[0] = O::pk(ex2(fmaf(s[2 * kt][0], sl2, -mx0)), ex2(fmaf(s[2 * kt][1], sl2, -mx0)));
+                    a[1] = O::pk(ex2(fmaf(s[2 * kt][2], sl2, -mx1)), ex2(fmaf(s[2 * kt][3], sl2, -mx1)));
+                    a[2] = O::pk(ex2(fmaf(s[2 * kt + 1][0], sl2, -mx0)), ex2(fmaf(s[2 * kt + 1][1], sl2, -mx0)));
+                    a[3] = O::pk(ex2(fmaf(s[2 * kt + 1][2], sl2, -mx1)), ex2(fmaf(s[2 * kt + 1][3], sl2, -mx1)));
 #pragma unroll
                     for (int j = 0; j < NTO; ++j) {
                         const int c0 = 8 * j + 2 * t;
-                        const uint32_t x0 = c0 < d ? ld32x(Vc + (16 * kt + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                        const uint32_t x1 =
-                            c0 < d ? ld32x(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? Op::kOne : 0u);
-                        Op::k16(o[j], a, movmatrix_trans(x0), movmatrix_trans(x1));
+                        const R x0 = c0 < d ? O::ld(Vc + (16 * kt + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+                        const R x1 =
+                            c0 < d ? O::ld(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+                        O::mma(o[j], a, O::tr(x0), O::tr(x1));
                     }
                 }
             }
@@ -171,8 +169,8 @@ exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __res
             for (int j = 0; j < NTO; ++j) {
                 const int c = 8 * j + 2 * t;
                 if (c < d) {
-                    *reinterpret_cast<uint32_t*>(o0 + c) = Op::pack(o[j][0] * i0, o[j][1] * i0);
-                    *reinterpret_cast<uint32_t*>(o1 + c) = Op::pack(o[j][2] * i1, o[j][3] * i1);
+                    O::st2(o0 + c, o[j][0] * i0, o[j][1] * i0);
+                    O::st2(o1 + c, o[j][2] * i1, o[j][3] * i1);
                 }
             }
         }
@@ -188,9 +186,10 @@ exact_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __res
 template <typename T, int NCOL, int WPU>
 cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                        cudaStream_t stream, unsigned int* fault) {
-    using Lay = ExactLayout<NCOL, WPU>;
+    using Lay = ExactLayout<T, NCOL, WPU>;
     constexpr int by_smem = (int)(kSmemLimit / Lay::PER_GROUP);
-    constexpr int by_threads = 16 / WPU;  // at most 512 threads (registers stay <= 128)
+    // at most 512 threads (registers stay <= 128), 256 with split fp32 operands
+    constexpr int by_threads = (sizeof(T) == 4 ? 8 : 16) / WPU;
     constexpr int kGroups = by_smem < by_threads ? by_smem : by_threads;
     static_assert(kGroups >= 1, "does not fit");
     auto kern = exact_tc_kernel<T, NCOL, WPU, kGroups>;
@@ -228,8 +227,10 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
             return wide ? launch_cfg<T, 40, 4>(q, k, v, out, n_units, d, stream, fault)
                         : launch_cfg<T, 32, 4>(q, k, v, out, n_units, d, stream, fault);
         default:
-            return wide ? launch_cfg<T, 40, 16>(q, k, v, out, n_units, d, stream, fault)
-                        : launch_cfg<T, 32, 16>(q, k, v, out, n_units, d, stream, fault);
+            if constexpr (sizeof(T) == 4) return cudaErrorInvalidValue;  // not offered (see supports)
+            else
+                return wide ? launch_cfg<T, 40, 16>(q, k, v, out, n_units, d, stream, fault)
+                            : launch_cfg<T, 32, 16>(q, k, v, out, n_units, d, stream, fault);
     }
 }
 
@@ -238,7 +239,9 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
 
 namespace nystra_host {
 bool exact_tc_supports(int N, int d, int dtype) {
-    return (dtype == 1 || dtype == 2) && (N == 64 || N == 256 || N == 1024) && d >= 2 && d <= 32 && d % 2 == 0;
+    const bool shape = d >= 2 && d <= 32 && d % 2 == 0;
+    if (dtype == 0) return shape && (N == 64 || N == 256);
+    return (dtype == 1 || dtype == 2) && (N == 64 || N == 256 || N == 1024) && shape;
 }
 
 cudaError_t launch_exact_tc(const void* q, const void* k, const void* v, void* out, long long n_units, int N,
@@ -252,6 +255,7 @@ cudaError_t launch_exact_tc(const void* q, const void* k, const void* v, void* o
         e = cudaGetSymbolAddress((void**)&s_fault[dev], nystra::g_fault_exact_tc);
         if (e != cudaSuccess) return e;
     }
+    if (dtype == 0) return nystra::launch_t<float>(q, k, v, out, n_units, N, d, stream, s_fault[dev]);
     if (dtype == 1)
         return nystra::launch_t<__nv_bfloat16>(q, k, v, out, n_units, N, d, stream, s_fault[dev]);
     return nystra::launch_t<__half>(q, k, v, out, n_units, N, d, stream, s_fault[dev]);
