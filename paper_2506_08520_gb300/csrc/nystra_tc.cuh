@@ -1,39 +1,39 @@
-// Tensor-core PnP-Nystra kernel template, 16-bit I/O, windows of N = 64,
-// 256 or 1024 tokens (8x8, 16x16, 32x32 windows), m in {8, 16, 32}, even
-// d_h <= 32.  Included by one translation unit per N (nystra_tc_n*.cu).
+// Tensor-core PnP-Nystra: the per-phase device functions shared by every
+// tensor-core kernel, and the grouped kernel.  Windows of N = 64, 256 or 1024
+// tokens (8x8, 16x16, 32x32), m in {8, 16, 32, 64}, even d_h <= 32, 16-bit
+// I/O (fp32 I/O through the operand policy Opnd<float>, used by the 8x8 pool
+// kernel).  Included by one translation unit per N (nystra_tc_n*.cu), which
+// also includes the kernel for its common case: nystra_pool.cuh (8x8, m <=
+// 16), nystra_team.cuh (16x16, m <= 32), nystra_stream.cuh (32x32, m <= 16).
 //
-// Work decomposition.  A "group" of WPU warps processes one (window, head)
-// unit at a time; a CTA holds GROUPS groups and the grid is persistent
-// (groups stride over units).  Warp r of a group owns tokens
-// [r*TPW, (r+1)*TPW) of the unit and handles them in 64-token chunks.
-//
-// Per unit:
-//   stage    each warp bulk-copies its TPW rows of Q, K and V (contiguous in
-//            HBM) into its private stage; bounded waits.
+// Phases of one (window, head) unit:
+//   stage    bulk copies of Q, K, V rows (contiguous in HBM) into shared
+//            memory; bounded mbarrier waits.
 //   front    landmarks (Algorithm 1 step 1) of the segments a warp owns
-//            (segments never straddle warps: N/m <= TPW), to group memory;
-//            [P1] S_L = Q Kbar^T, G_L^n = exp(S_L - m_L) parked as MMA
-//            fragments;  S_U = Qbar K^T with a running row max across the
-//            warp's chunks, G_U^n fed straight from registers into
-//            W_r = G_U^n [V | 1], rescaled online when the max grows.
-//   combine  (WPU > 1) partial (W_r, m_r) of all warps are merged in a fixed
+//            (segments never straddle warps: N/m <= TPW); S_L = Q Kbar^T and
+//            G_L^n = exp(S_L - m_L) parked as MMA fragments [P1];
+//            S_U = Qbar K^T with a running row max across 64-token chunks,
+//            G_U^n fed straight from registers into W_r = G_U^n [V | 1],
+//            rescaled online when the max grows.
+//   combine  (several token warps) partial (W_r, m_r) merged in a fixed
 //            order: m_U = max_r m_r, W = sum_r exp(m_r - m_U) W_r, which is
 //            exactly G_U^n [V | 1] with the max over all N keys.
-//   core     warp 0: G_A^n = exp(Qbar Kbar^T - m_U), Z_0 = A^T/(||A||_1
-//            ||A||_inf), `iters` steps Z <- Z(13I - X(15I - X(7I - X)))/4 with
-//            X = A Z (step 4), Y = Z W, stored as a 16-bit B operand; all in
-//            registers.
-//   output   every warp: O = (G_L^n Y_:d) / (G_L^n Y_d) for its tokens
-//            (steps 5-7), staged row-major in its V region and written with
-//            one bulk store (whole sectors; scattered 4-byte stores of 60-byte
-//            rows touched ~11 sectors per 128 bytes).  [P2] S_L and G_L^n are
-//            computed here from the still-resident Q.
-//   copies   Q and K of the next unit are issued after the combine ([P2]: K
-//            only; Q after the output), V once the output store has read its
-//            staging, on two mbarriers, so V may land while the next unit's
-//            landmarks and S_L run.
-// P1 ("G_L parked") is used when the fragments fit in shared memory next to
-// the stage; otherwise P2.
+//   core     G_A^n = exp(Qbar Kbar^T - m_U), Z_0 = A^T/(||A||_1 ||A||_inf),
+//            `iters` steps Z <- Z(13I - X(15I - X(7I - X)))/4 with X = A Z
+//            (step 4), Y = Z W stored as a 16-bit B operand: core_warp (one
+//            warp, in registers, m <= 16) or dist_core (m/16 warps).
+//   output   O = (G_L^n Y_:d) / (G_L^n Y_d) (steps 5-7), staged row-major and
+//            written with one bulk store (rows of 60 bytes would otherwise be
+//            written as partial sectors); [P2] S_L and G_L^n recomputed from
+//            a still-resident Q.
+//
+// Grouped kernel (nystra_tc_kernel; every m = 32 or 64 the three kernels
+// above do not take).  A group of token warps owns one unit at a time, plus
+// helper warps when the distributed core needs more warps than there are
+// token warps; a CTA holds GROUPS groups and the grid is persistent.  The
+// next unit's Q and K are copied after the combine ([P2]: K only, Q after the
+// output), V once the output store has read its staging.  P1 ("G_L parked")
+// is used when it fits as many groups as P2.
 //
 // Arithmetic.  Products with token or d_h extents use mma.sync in the I/O
 // type with fp32 accumulation.  The m x m iteration needs close to fp32
@@ -41,15 +41,13 @@
 // iteration count): it uses fp16 two-term splits (x = hi + lo, three k16
 // products lo*hi + hi*lo + hi*hi, 22 significant bits), with Z rescaled by a
 // power of two every step to stay in fp16's range.  Y = Z W uses split-tf32
-// (W's range is not bounded).  The iteration runs in registers: it carries
-// the symmetric X = A Z_k next to Z (X_{k+1} = X_k T3/4, equal to A Z_{k+1}),
-// so every product has a symmetric or transposed right factor whose B
-// fragments are the lane's own A fragments, and X is made exactly symmetric
-// (lower triangle mirrored with 8x8 movmatrix transposes) after each update,
-// which keeps antisymmetric round-off from growing by up to 13/4 per step in
-// directions that have not converged.
-// Scores are kept in the log2 domain (scaled by log2(e)/sqrt(d_h)), so each
-// exponential is one FFMA and one ex2.
+// (W's range is not bounded).  The iteration carries the symmetric
+// X = A Z_k next to Z (X_{k+1} = X_k T3/4, equal to A Z_{k+1}), so every
+// product has a symmetric or transposed right factor, and X is made exactly
+// symmetric (lower triangle mirrored) after each update, which keeps
+// antisymmetric round-off from growing by up to 13/4 per step in directions
+// that have not converged.  Scores are kept in the log2 domain (scaled by
+// log2(e)/sqrt(d_h)), so each exponential is one FFMA and one ex2.
 #pragma once
 
 #include "common.cuh"
