@@ -1,5 +1,5 @@
-// Streaming team kernel for 32x32 windows (N = 1024 tokens), m <= 16, even
-// d_h <= 32, 16-bit I/O.  Included by the N = 1024 translation unit after
+// Streaming team kernel for 32x32 windows (N = 1024 tokens), m <= 32, even
+// d_h <= 32, 16-bit I/O (m = 32: the core runs on two warps, dist_core).  Included by the N = 1024 translation unit after
 // nystra_tc.cuh, whose per-phase device functions it reuses.
 //
 // A whole 32x32 unit (Q, K, V: 184 KB at d_h = 30) fills an SM, so staging
@@ -36,13 +36,15 @@ namespace tc {
 template <int M, int NCOL>
 struct StreamLayout {
     static constexpr int NT = 4, TPW = 256, N = NT * TPW, CH = 64, NCHK = TPW / CH;
+    static constexpr int CWN = M > 16 ? M / 16 : 1;  // core warps (m = 32: distributed core)
+    static constexpr int MT = (M + 15) / 16;         // landmark m-tiles
     static constexpr int DS = (NCOL == 32) ? 30 : 32;
-    static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int MP = MT * 16, LS = 40, WS = NCOL + 4, YS = MP + 8;
     static constexpr int L = N / M, LPW = TPW / L;  // tokens per segment, segments per token warp
     static constexpr size_t XB = (size_t)CH * DS * 2;  // one tensor's chunk
     static constexpr size_t SLOT = 2 * XB;             // K and V (Q uses the first half)
     static constexpr size_t WPB = (size_t)MP * WS * 4 + MP * 4;  // W partial, row maxima
-    static_assert(WPB <= XB, "the W partial lives in the V half of the last KV chunk's slot");
+    static_assert(WPB <= SLOT, "the W partial lives in the slot of the last K/V chunk");
     // per-unit state
     static constexpr size_t B_QB = 0;
     static constexpr size_t B_KB = B_QB + MP * LS * 2;
@@ -50,21 +52,26 @@ struct StreamLayout {
     static constexpr size_t B_MU = B_W + MP * WS * 4;
     static constexpr size_t B_YT = B_MU + MP * 4;
     static constexpr size_t BUF = ((B_YT + NCOL * YS * 2 + 127) / 128) * 128;
+    static constexpr size_t SCR = CWN > 1 ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0;
     template <int S>
     struct Team {
         static constexpr size_t WARP = S * SLOT;  // a token warp's ring of chunk buffers
         static constexpr size_t T_BUF = NT * WARP;
         static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // slot bars [NT][S], F[2], C[2]
-        static constexpr size_t BYTES = ((T_BAR + (NT * S + 4) * 8 + 127) / 128) * 128;
+        static constexpr size_t T_SCR = ((T_BAR + (NT * S + 4) * 8 + 127) / 128) * 128;
+        static constexpr size_t BYTES = ((T_SCR + SCR + 127) / 128) * 128;
     };
-    // three teams with two-deep rings when they fit, else two with three-deep
+    static constexpr int WARPS = NT + CWN;  // per team
+    // three teams with two-deep rings when they fit, else two with three-deep,
+    // else two with two-deep
     static constexpr bool kThree = 3 * Team<2>::BYTES <= kSmemLimit;
+    static constexpr bool kDeep = 2 * Team<3>::BYTES <= kSmemLimit;
     static constexpr int TEAMS = kThree ? 3 : 2;
-    static constexpr int NSLOT = kThree ? 2 : 3;
+    static constexpr int NSLOT = kThree ? 2 : (kDeep ? 3 : 2);
     using TL = Team<NSLOT>;
     static constexpr size_t TEAM = TL::BYTES;
     static_assert(TEAMS * TEAM <= kSmemLimit, "teams must fit");
-    static_assert(M <= 16 && L >= 16 && LPW <= 8, "segments per token warp fit one n-tile");
+    static_assert(M <= 32 && L >= 16 && LPW <= 8, "segments per token warp fit one n-tile");
     static_assert(XB % 16 == 0 && SLOT % 16 == 0 && TL::WARP % 16 == 0 && BUF % 16 == 0, "16-byte alignment");
 };
 
@@ -85,7 +92,7 @@ __device__ __forceinline__ StreamTask stream_task(int v, int count) {
 }
 
 template <typename T, int M, int NCOL, int DC>
-__global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * 5 * 32, 1)
+__global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * StreamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                      T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
@@ -93,11 +100,11 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     using TL = typename Lay::TL;
     using R = typename Opnd<T>::Reg;
     constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
-                  NSLOT = Lay::NSLOT, L = Lay::L, LPW = Lay::LPW, NTO = NCOL / 8;
+                  NSLOT = Lay::NSLOT, L = Lay::L, LPW = Lay::LPW, NTO = NCOL / 8, MT = Lay::MT;
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int team = warp / (NT + 1), r = warp - team * (NT + 1);  // r == NT: core warp
+    const int team = warp / Lay::WARPS, r = warp - team * Lay::WARPS;  // r >= NT: core warps
     const int g = lane >> 2, t = lane & 3;
     unsigned char* tb = smem_raw + (size_t)team * Lay::TEAM;
     auto buf = [&](int b) { return tb + TL::T_BUF + (size_t)b * Lay::BUF; };
@@ -115,8 +122,8 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             for (int i = 0; i < NT * NSLOT; ++i) mbar_init(bb + i, 1);
             mbar_init(bb + NT * NSLOT, NT);
             mbar_init(bb + NT * NSLOT + 1, NT);
-            mbar_init(bb + NT * NSLOT + 2, 1);
-            mbar_init(bb + NT * NSLOT + 3, 1);
+            mbar_init(bb + NT * NSLOT + 2, Lay::CWN);
+            mbar_init(bb + NT * NSLOT + 3, Lay::CWN);
         }
         fence_mbar_init();
     }
@@ -135,21 +142,35 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     }
     __syncthreads();
 
-    if (r == NT) {
-        // ======================= core warp =======================
+    if (r >= NT) {
+        // ======================= core warp(s) =======================
+        const int c = r - NT;
         for (int kk = 0; kk < count; ++kk) {
             const int b = kk & 1;
-            const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, (uint32_t)((kk >> 1) & 1), kWaitNs));
+            bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(barF + b, (uint32_t)((kk >> 1) & 1), kWaitNs));
+            if constexpr (Lay::CWN > 1)  // the core warps decide together
+                ok = !named_barrier_or(1 + Lay::TEAMS + team, Lay::CWN * 32, !ok);
             if (!ok) {  // the token warps stopped (or stalled): stop too
                 if (lane == 0) atomicOr(fault, 1u);
                 break;
             }
             unsigned char* bb = buf(b);
             const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
-            float mU[1][2] = {{gmu[g], gmu[g + 8]}};
-            core_warp<T, M, NCOL>(reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB),
-                                  mU, reinterpret_cast<const float*>(bb + Lay::B_W),
-                                  reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            if constexpr (Lay::CWN == 1) {
+                float mU[1][2] = {{gmu[g], gmu[g + 8]}};
+                core_warp<T, M, NCOL>(reinterpret_cast<const T*>(bb + Lay::B_QB),
+                                      reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
+                                      reinterpret_cast<const float*>(bb + Lay::B_W),
+                                      reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+            } else {
+                using DSc = DistScratch<(M > 16 ? M : 32)>;
+                unsigned char* scr = tb + TL::T_SCR;
+                dist_core<T, (M > 16 ? M : 32), NCOL>(
+                    reinterpret_cast<const T*>(bb + Lay::B_QB), reinterpret_cast<const T*>(bb + Lay::B_KB), gmu,
+                    reinterpret_cast<const float*>(bb + Lay::B_W), reinterpret_cast<T*>(bb + Lay::B_YT), scr,
+                    scr + DSc::MAT, reinterpret_cast<float*>(scr + 2 * DSc::MAT), iters, sl2, c, lane,
+                    1 + Lay::TEAMS + team);
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive(barC + b);
         }
@@ -192,9 +213,8 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     issued = __shfl_sync(0xffffffffu, issued, 0);
 
     bool failed = false;  // a bounded wait of this warp gave up (warp-uniform)
-    float cq[2][1][4], ck[2][1][4], w[NTO][4];
-    float run0 = -INFINITY, run1 = -INFINITY;
-    R aq[2][4];
+    float cq[2][1][4], ck[2][1][4], w[MT][NTO][4], run[MT][2];
+    R aq[MT][2][4];
     for (int vv = 0; vv < total; ++vv) {
         const StreamTask tk = stream_task(vv, count);
         const int s = vv % NSLOT;
@@ -219,7 +239,8 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(cq, reinterpret_cast<T*>(bb + Lay::B_QB), r * LPW, g, t);
                 if (tsync_or(failed)) break;
-                qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), 0, g, t, aq);
+#pragma unroll
+                for (int mt = 0; mt < MT; ++mt) qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), mt, g, t, aq[mt]);
             }
         } else if (tk.type == 1) {
             // ---------------- KV(k): Kbar sums, S_U, partial W ----------------
@@ -227,28 +248,39 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
 #pragma unroll
                 for (int mf = 0; mf < 2; ++mf) ck[mf][0][0] = ck[mf][0][1] = ck[mf][0][2] = ck[mf][0][3] = 0.f;
 #pragma unroll
-                for (int j = 0; j < NTO; ++j) w[j][0] = w[j][1] = w[j][2] = w[j][3] = 0.f;
-                run0 = run1 = -INFINITY;
+                for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) w[mt][j][0] = w[mt][j][1] = w[mt][j][2] = w[mt][j][3] = 0.f;
+                    run[mt][0] = run[mt][1] = -INFINITY;
+                }
             }
             landmarks_acc<T, L, LPW>(X0, tk.c * Lay::CH, ck, d, g, t);
-            su_w_chunk<T, NCOL>(aq, X0, slot_x(s, 1), d, g, t, sl2, g < M, g + 8 < M, w, run0, run1, true);
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt)
+                su_w_chunk<T, NCOL>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M, 16 * mt + g + 8 < M,
+                                    w[mt], run[mt][0], run[mt][1], true);
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(ck, reinterpret_cast<T*>(bb + Lay::B_KB), r * LPW, g, t);
-                // the partial goes over this slot's V rows, consumed above
-                float* wpart = reinterpret_cast<float*>(slot_x(s, 1));
+                // the partial goes over this slot's K and V rows, consumed above
+                float* wpart = reinterpret_cast<float*>(slot_x(s, 0));
                 __syncwarp();
 #pragma unroll
-                for (int j = 0; j < NTO; ++j) {
-                    const int c = 8 * j + 2 * t;
-                    *reinterpret_cast<float2*>(wpart + g * WS + c) = make_float2(w[j][0], w[j][1]);
-                    *reinterpret_cast<float2*>(wpart + (g + 8) * WS + c) = make_float2(w[j][2], w[j][3]);
-                }
+                for (int mt = 0; mt < MT; ++mt)
+#pragma unroll
+                    for (int j = 0; j < NTO; ++j) {
+                        const int c = 8 * j + 2 * t, rr = 16 * mt + g;
+                        *reinterpret_cast<float2*>(wpart + rr * WS + c) = make_float2(w[mt][j][0], w[mt][j][1]);
+                        *reinterpret_cast<float2*>(wpart + (rr + 8) * WS + c) = make_float2(w[mt][j][2], w[mt][j][3]);
+                    }
                 if (t == 0) {
-                    wpart[MP * WS + g] = run0;
-                    wpart[MP * WS + g + 8] = run1;
+#pragma unroll
+                    for (int mt = 0; mt < MT; ++mt) {
+                        wpart[MP * WS + 16 * mt + g] = run[mt][0];
+                        wpart[MP * WS + 16 * mt + g + 8] = run[mt][1];
+                    }
                 }
                 tsync();
-                combine_partials<MP, NCOL, WS, NT>(reinterpret_cast<const float*>(tb + (size_t)s * Lay::SLOT + Lay::XB),
+                combine_partials<MP, NCOL, WS, NT>(reinterpret_cast<const float*>(tb + (size_t)s * Lay::SLOT),
                                                     TL::WARP / 4, reinterpret_cast<float*>(bb + Lay::B_W),
                                                     reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
                 if (tsync_or(failed)) break;
@@ -304,7 +336,7 @@ cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* 
         int dev = 0, sms = 0, per_sm = 0;
         if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
         if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * 5 * 32, smem)) !=
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * Lay::WARPS * 32, smem)) !=
             cudaSuccess)
             return e;
         if (per_sm < 1) return cudaErrorInvalidConfiguration;
@@ -313,7 +345,7 @@ cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* 
     const long long want = (n_units + Lay::TEAMS - 1) / Lay::TEAMS;
     const long long grid = want < s_blocks ? want : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
-    kern<<<(unsigned)grid, Lay::TEAMS * 5 * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
+    kern<<<(unsigned)grid, Lay::TEAMS * Lay::WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                                  n_units, d, iters, sl2, fault);
     return cudaGetLastError();
 }

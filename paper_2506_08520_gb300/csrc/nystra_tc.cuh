@@ -1594,6 +1594,9 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
         if (m == 16)
             return wide ? launch_stream<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_stream<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (m == 32)
+            return wide ? launch_stream<T, 32, 40>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_stream<T, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
     switch (m) {
         case 8:

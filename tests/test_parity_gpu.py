@@ -38,6 +38,8 @@ SMALL = [
     (1, 1024, 32, 8),
     (3, 1024, 30, 16),
     (2, 1024, 16, 16),
+    (3, 1024, 30, 32),
+    (4, 256, 30, 32),
     (4, 48, 20, 12),     # odd sizes
     (3, 10, 3, 5),
     (6, 128, 64, 16),    # widest head
@@ -83,7 +85,7 @@ def test_nystra_edge_cases(N, d, m, iters, dtype):
 FULL = ["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4",
         "large-w16-m32", "large-w16-m64", "large-w32-m32", "large-w32-m64",
         "sr720p-w8-m16-bf16", "sr720p-w16-m16-f16", "sr720p-w32-m16-bf16", "sr720p-w8-m64-f16",
-        "sr720p-w32-m8-f16"]
+        "sr720p-w32-m8-f16", "sr720p-w16-m32-bf16", "sr720p-w32-m32-bf16"]
 
 
 @pytest.mark.parametrize("name", FULL)
