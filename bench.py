@@ -151,6 +151,24 @@ def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
     return passes * n * wl.N / dt, n, passes, dt, oracle.threads()
 
 
+def _l2_bytes() -> int:
+    if torch.cuda.is_available():
+        return int(torch.cuda.get_device_properties(0).L2_cache_size)
+    return 126 * 2**20  # GB300 (only when no GPU is visible)
+
+
+def _config(wl, ws: int):
+    """The `config` object both arms report: the workload and how the timed
+    launches avoid L2 residency (rotating input/output sets > 3x L2)."""
+    io_bytes = 4 * wl.units * wl.N * wl.d * {"f32": 4, "bf16": 2, "f16": 2}[wl.dtype]
+    nsets = max(2, -(-3 * _l2_bytes() // io_bytes))
+    return nsets, io_bytes, {
+        "workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N, "d_h": wl.d, "m": wl.m,
+        "iters": wl.iters, "io_dtype": wl.dtype,
+        "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
+        "parallelism": f"replica x{ws} (independent windows)"}
+
+
 def run_reference(args, wl):
     ws, rank, _ = _dist()
     if rank != 0:
@@ -178,8 +196,7 @@ def run_reference(args, wl):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic",
-        "config": {"workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N,
-                   "d_h": wl.d, "m": wl.m, "iters": wl.iters, "io_dtype": wl.dtype},
+        "config": _config(wl, ws)[2],
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
                          "sample": f"{n} of {qd.shape[0]} units per step (float64 C oracle, OpenMP)"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -198,10 +215,9 @@ def run_cuda(args, wl):
 
     q, k, v = workloads.make_qkv(wl)
     esize = q.element_size()
-    io_bytes = 4 * q.numel() * esize
-    l2 = torch.cuda.get_device_properties(dev).L2_cache_size
     # rotate input/output sets so that one step's data is never L2-resident
-    nsets = max(2, -(-3 * l2 // io_bytes))
+    nsets, io_bytes, config = _config(wl, ws)
+    assert io_bytes == 4 * q.numel() * esize
     sets = []
     for _ in range(nsets):
         sets.append(tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),))
@@ -286,10 +302,7 @@ def run_cuda(args, wl):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": {"workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N,
-                   "d_h": wl.d, "m": wl.m, "iters": wl.iters, "io_dtype": wl.dtype,
-                   "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
-                   "parallelism": f"replica x{ws} (independent windows)"},
+        "config": config,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
                      "bytes_per_launch": io_bytes, "kernel_ms": kern_ms},
