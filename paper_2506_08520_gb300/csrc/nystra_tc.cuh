@@ -1598,28 +1598,25 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
             return wide ? launch_stream<T, 32, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_stream<T, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
-    switch (m) {
-        case 8:
-            return wide ? launch_cfg<T, 8, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_cfg<T, 8, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
-        case 16:
-            return wide ? launch_cfg<T, 16, 40, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_cfg<T, 16, 32, TPW, WPU>(q, k, v, out, n_units, d, iters, stream, fault);
-        case 32: {
-            // several token warps: the core is split over two of them
-            constexpr int CW = WPU >= 2 ? 2 : 1;
-            return wide ? launch_cfg<T, 32, 40, TPW, WPU, CW>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_cfg<T, 32, 32, TPW, WPU, CW>(q, k, v, out, n_units, d, iters, stream, fault);
-        }
-        default: {
-            // m = 64: the core on four warps; W partials of 64 rows need K/V
-            // rows of at least 128 tokens per token warp.
-            constexpr int TP = (TPW * WPU == 64) ? 64 : (TPW * WPU == 256) ? 128 : 256;
-            constexpr int WP = TPW * WPU / TP;
-            return wide ? launch_cfg<T, 64, 40, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_cfg<T, 64, 32, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault);
-        }
+    // The grouped kernel: m = 32 at 8x8 windows (core in one warp's registers)
+    // and at 16x16 windows with d_h = 32 (core on two warps); every m = 64.
+    if (m == 32) {
+        if constexpr (TPW == 64 && WPU == 1)
+            return wide ? launch_cfg<T, 32, 40, 64, 1, 1>(q, k, v, out, n_units, d, iters, stream, fault)
+                        : launch_cfg<T, 32, 32, 64, 1, 1>(q, k, v, out, n_units, d, iters, stream, fault);
+        if constexpr (TPW == 64 && WPU == 4)
+            return launch_cfg<T, 32, 40, 64, 4, 2>(q, k, v, out, n_units, d, iters, stream, fault);
+        return cudaErrorInvalidValue;  // not reached: the stream kernel takes 32x32 windows
     }
+    if (m == 64) {
+        // the core on four warps; W partials of 64 rows need K/V rows of at
+        // least 128 tokens per token warp
+        constexpr int TP = (TPW * WPU == 64) ? 64 : (TPW * WPU == 256) ? 128 : 256;
+        constexpr int WP = TPW * WPU / TP;
+        return wide ? launch_cfg<T, 64, 40, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault)
+                    : launch_cfg<T, 64, 32, TP, WP, 4>(q, k, v, out, n_units, d, iters, stream, fault);
+    }
+    return cudaErrorInvalidValue;  // not reached: m is checked by the caller
 }
 
 }  // namespace tc
