@@ -55,7 +55,7 @@ def test_nystra_small(units, N, d, m, dtype):
     assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
 
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
 @pytest.mark.parametrize("N,d,m,iters", [
     (64, 30, 64, 6),     # m = N: every token is a landmark
     (64, 30, 1, 6),      # one landmark
@@ -64,7 +64,14 @@ def test_nystra_small(units, N, d, m, dtype):
     (64, 30, 16, 12),
     (1, 1, 1, 6),        # degenerate single token
     (64, 1, 16, 6),      # d_h = 1
+    (64, 2, 16, 6),      # narrowest head on the tensor cores
     (32, 64, 32, 6),
+    (256, 30, 16, 0),    # team kernel, Z_0 only
+    (256, 30, 8, 12),
+    (256, 2, 16, 6),
+    (1024, 30, 16, 1),   # streaming kernel
+    (1024, 30, 8, 12),
+    (1024, 32, 32, 0),
 ])
 def test_nystra_edge_cases(N, d, m, iters, dtype):
     q, k, v = workloads.random_qkv(3, N, d, dtype, seed=N + d + m + iters)
@@ -137,3 +144,16 @@ def test_status_clean_after_runs():
     q, k, v = (x.cuda() for x in workloads.random_qkv(4, 64, 30, "bf16", seed=7))
     binding.nystra(q, k, v, 16, 6)
     assert binding.status() == binding.NYSTRA_OK
+
+
+def test_fp16_large_values_keep_range():
+    # W = G_U^n [V | 1] reaches 64 x max|V| and Y = Z W is larger still: fp16
+    # I/O must scale Y into range (the factor cancels in the output ratio).
+    q, k, v = workloads.random_qkv(6, 64, 30, "f16", seed=5)
+    v = (v.float() * 400.0).half()
+    err, worst = check_nystra(q, k, v, 16, 6)
+    assert err <= TOL["f16"], f"max rel err {err:.3e} at unit {worst}"
+    q, k, v = workloads.random_qkv(2, 1024, 30, "f16", seed=6)
+    v = (v.float() * 400.0).half()
+    err, worst = check_nystra(q, k, v, 16, 6)
+    assert err <= TOL["f16"], f"max rel err {err:.3e} at unit {worst}"
