@@ -148,6 +148,38 @@ NYSTRA_API int nystra_check(void* stream);
  */
 NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream);
 
+/*
+ * nystra_debug_stages -- test-only (the paper has no counterpart): every
+ * intermediate of Algorithm 1 for ONE unit, as the tensor-core path for 8x8
+ * windows computes it.  One warp runs, for unit `unit` (window*heads + head)
+ * of the [n_windows, heads, N, d_h] tensors q, k, v, the same device functions
+ * the N = 64 kernel runs, and writes fp32 values, row-major, to `dump`
+ * (device memory, caller-owned, 16-byte aligned, nystra_debug_stages_size()
+ * floats), regions in this order:
+ *   Qbar  m x d_h      landmarks (step 1), as rounded to the I/O type
+ *   Kbar  m x d_h
+ *   G_L^n N x m        exp(S_L - m_L) (steps 2-3), as rounded to the I/O type
+ *   m_U   m            row maxima of S_U over all N keys (natural-log domain)
+ *   W     m x (d_h+1)  G_U^n [V | 1_N] (step 5); column d_h is G_U^n 1_N
+ *   G_A^n m x m        exp(S_A - m_U) (step 3)
+ *   Z     m x m        the pseudo-inverse after `iters` steps (step 4)
+ *   Y     m x (d_h+1)  Z W (the re-associated step 6)
+ *   O     N x d_h      the output (step 7), as rounded to the I/O type
+ * Supported: N = 64, m in {8, 16}, even d_h <= 32 (the shapes nystra_attention
+ * runs on this path), fp32 I/O only with iters <= 6; anything else returns
+ * NYSTRA_EINVAL, as do unit outside [0, n_windows*heads), null or misaligned
+ * pointers.  Asynchronous on `stream`; allocates nothing.  Returns NYSTRA_OK,
+ * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.
+ */
+NYSTRA_API int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windows, int heads,
+                                   int N, int d_h, int m, int iters, int dtype, long long unit, float* dump,
+                                   void* stream);
+
+/* Floats nystra_debug_stages writes for (N, d_h, m):
+ * 2 m d_h + N m + m + 2 m (d_h+1) + 2 m^2 + N d_h; NYSTRA_EINVAL (negative)
+ * for a shape it does not support.  Touches no device. */
+NYSTRA_API long long nystra_debug_stages_size(int N, int d_h, int m);
+
 #ifdef __cplusplus
 }
 #endif

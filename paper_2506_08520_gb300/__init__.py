@@ -5,8 +5,8 @@ library ``libnystra.so`` (see ``include/nystra.h``); ``workloads`` holds the
 seeded synthetic inputs.  The library is loaded on first use and every call
 fails loudly if it is missing: there is no CPU path.
 """
-from .binding import (NystraError, check, debug_wait_timeout, exact, exact_window_attention, nystra,
-                      nystra_attention, status, strerror, version)
+from .binding import (NystraError, check, debug_stages, debug_wait_timeout, exact, exact_window_attention,
+                      nystra, nystra_attention, status, strerror, version)
 
 __all__ = ["nystra", "exact", "nystra_attention", "exact_window_attention", "status", "check",
-           "debug_wait_timeout", "strerror", "version", "NystraError"]
+           "debug_wait_timeout", "debug_stages", "strerror", "version", "NystraError"]

@@ -55,6 +55,10 @@ def lib() -> ctypes.CDLL:
         L.nystra_check.restype = i
         L.nystra_debug_wait_timeout.argtypes = [ctypes.c_ulonglong, vp]
         L.nystra_debug_wait_timeout.restype = i
+        L.nystra_debug_stages.argtypes = [vp, vp, vp, i, i, i, i, i, i, i, ctypes.c_longlong, vp, vp]
+        L.nystra_debug_stages.restype = i
+        L.nystra_debug_stages_size.argtypes = [i, i, i]
+        L.nystra_debug_stages_size.restype = ctypes.c_longlong
         _lib = L
     return _lib
 
@@ -90,6 +94,21 @@ def check(stream=None) -> int:
 def debug_wait_timeout(limit_ns: int, stream=None) -> int:
     """Test-only: launch a wait that can only time out (see the header)."""
     return lib().nystra_debug_wait_timeout(int(limit_ns), _stream_ptr(stream))
+
+
+def nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, dtype, unit, dump, stream) -> int:
+    """Raw C-ABI call of the test-only stage dump (see the header)."""
+    return lib().nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, dtype, int(unit), dump, stream)
+
+
+def nystra_debug_stages_size(N: int, d_h: int, m: int) -> int:
+    return lib().nystra_debug_stages_size(N, d_h, m)
+
+
+# Regions of the stage dump, in the order and with the shapes the header gives.
+def _stage_shapes(N: int, d: int, m: int):
+    return [("qbar", (m, d)), ("kbar", (m, d)), ("GLn", (N, m)), ("mU", (m,)), ("W", (m, d + 1)),
+            ("GAn", (m, m)), ("Z", (m, m)), ("Y", (m, d + 1)), ("out", (N, d))]
 
 
 # ------------------------------------------------------------ torch helpers
@@ -148,4 +167,30 @@ def exact(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tensor |
                                     _DTYPE_CODE[q.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "exact_window_attention")
+    return out
+
+
+def debug_stages(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int, iters: int, unit: int,
+                 stream=None) -> dict:
+    """Test-only: every intermediate of one unit (fp32 CPU tensors by name)."""
+    _check(q, k, v, q)
+    nw, h, N, d = _geometry(q)
+    size = nystra_debug_stages_size(N, d, m)
+    if size < 0:
+        raise NystraError(int(size), "nystra_debug_stages_size")
+    dump = torch.empty(size, dtype=torch.float32, device=q.device)
+    with torch.cuda.device(q.device):
+        rc = nystra_debug_stages(q.data_ptr(), k.data_ptr(), v.data_ptr(), nw, h, N, d, m, iters,
+                                 _DTYPE_CODE[q.dtype], unit, dump.data_ptr(), _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_debug_stages")
+    torch.cuda.synchronize(q.device)
+    host = dump.cpu()
+    out, pos = {}, 0
+    for name, shape in _stage_shapes(N, d, m):
+        n = 1
+        for x in shape:
+            n *= x
+        out[name] = host[pos:pos + n].reshape(shape)
+        pos += n
     return out

@@ -106,6 +106,24 @@ int nystra_status(void* stream) {
 
 int nystra_check(void* stream) { return nystra_status(stream); }
 
+long long nystra_debug_stages_size(int N, int d_h, int m) {
+    if (N != 64 || (m != 8 && m != 16) || d_h < 2 || d_h > 32 || d_h % 2 != 0) return NYSTRA_EINVAL;
+    return nystra_host::debug_stages_size(N, d_h, m);
+}
+
+int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windows, int heads, int N, int d_h,
+                        int m, int iters, int dtype, long long unit, float* dump, void* stream) {
+    if (dtype != NYSTRA_F32 && dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;
+    if (nystra_debug_stages_size(N, d_h, m) < 0) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > NYSTRA_MAX_ITERS || (dtype == NYSTRA_F32 && iters > 6)) return NYSTRA_EINVAL;
+    if (n_windows < 0 || heads < 0 || unit < 0 || unit >= (long long)n_windows * heads) return NYSTRA_EINVAL;
+    if (!q || !k || !v || !dump) return NYSTRA_EINVAL;
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dump)) return NYSTRA_EINVAL;
+    const cudaError_t e = nystra_host::launch_debug_stages(q, k, v, unit, d_h, m, iters, dtype, dump,
+                                                           (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
 int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream) {
     if (limit_ns < 1000ull || limit_ns > 1000000000ull) return NYSTRA_EINVAL;
     const cudaError_t e = nystra_host::launch_debug_wait(limit_ns, (cudaStream_t)stream);

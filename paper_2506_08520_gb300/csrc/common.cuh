@@ -54,5 +54,9 @@ unsigned int take_fault_word_exact_tc(cudaError_t* err);
 // units whose kernels wait on barriers: OR-ed together, then cleared.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);
 cudaError_t launch_debug_wait(unsigned long long limit_ns, cudaStream_t stream);
+// Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
+long long debug_stages_size(int N, int d, int m);
+cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,
+                                int iters, int dtype, float* dump, cudaStream_t stream);
 unsigned int take_fault_word_debug(cudaError_t* err);
 }  // namespace nystra_host

@@ -647,11 +647,15 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
 // T2 = 15I - 7X + X X, T3 = 13I - X T2, Z <- Z T3/4 and X <- X T3/4 (equal to
 // A Z_{k+1}; its factors are polynomials in X and commute).  X is kept exactly
 // symmetric (lower triangle mirrored) after every update.  Scalar factors of
-// Z (a, 1/4 per step, the power-of-two range scaling) are dropped: O is a
-// ratio of two columns of G_L^n Z W, so they cancel.
-template <typename T, int M, int NCOL>
+// Z (a and the power-of-two range scaling) are dropped: O is a ratio of two
+// columns of G_L^n Z W, so they cancel.
+//
+// DUMP (test-only stage dump): dbg receives G_A^n (M x M), Z (M x M) and
+// Y = Z W (M x NCOL), row-major fp32, with the dropped factors restored.
+template <typename T, int M, int NCOL, bool DUMP = false>
 __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const float (&mU)[(M + 15) / 16][2],
-                                          const float* mW, T* yT, int iters, float sl2, int g, int t) {
+                                          const float* mW, T* yT, int iters, float sl2, int g, int t,
+                                          float* dbg = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int MT = (M + 15) / 16, LS = 40, WS = NCOL + 4, NTO = NCOL / 8;
@@ -664,6 +668,8 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
     }
     Frag<MT> Zc;
     HFrag<MT> Xh, Zh;
+    float zscale = 1.f;  // DUMP: Z = zscale 2^-esum Zc
+    int esum = 0;
     {
         Frag<MT> Ac;
 #pragma unroll
@@ -721,6 +727,18 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                 cmax = fmaxf(cmax, c);
             }
         const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
+        if constexpr (DUMP) {
+            zscale = alpha;
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                        if (r < M && c < M) dbg[r * M + c] = Ac[i][n][e];
+                    }
+        }
         HFrag<MT> Ah;
         to_hfrag<MT>(Ac, Ah);
         transpose_hfrag<MT>(Ah, Zh);  // Z_0 = A^T (a dropped)
@@ -756,9 +774,22 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
         if (it + 1 < iters) {
             mm_hT<MT, false>(Xh, Th, F, 0.f, 0u, g, t);  // X T3/4
             sym_hfrag<MT>(F, Xh, sel, 1.f);
-            frag_normalise<MT>(Zc);
+            const int ez = frag_normalise<MT>(Zc);
+            if constexpr (DUMP) esum += ez;
             to_hfrag<MT>(Zc, Zh);
         }
+    }
+    if constexpr (DUMP) {
+        const float zs = ldexpf(zscale, -esum);
+#pragma unroll
+        for (int i = 0; i < MT; ++i)
+#pragma unroll
+            for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
+                    if (r < M && c < M) dbg[M * M + r * M + c] = zs * Zc[i][n][e];
+                }
     }
 
     // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
@@ -788,6 +819,18 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                     mma_tf32(y[i][j], ah[i][0], ah[i][1], ah[i][2], ah[i][3], bh0, bh1);
                 }
             }
+        }
+        if constexpr (DUMP) {
+            const float zs = ldexpf(zscale, -esum);
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int j = 0; j < NTO; ++j)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int r = 16 * i + g + 8 * (e >> 1), c = 8 * j + 2 * t + (e & 1);
+                        if (r < M) dbg[2 * M * M + r * NCOL + c] = zs * y[i][j][e];
+                    }
         }
         // fp16 output has a narrow range: scale Y by a power of two.
         // Numerator and denominator columns share the factor, so it cancels

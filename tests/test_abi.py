@@ -28,7 +28,7 @@ def test_header_declares_the_boundary():
     names = declared_symbols()
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
                      "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
-                     "nystra_debug_wait_timeout"):
+                     "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size"):
         assert required in names
 
 
@@ -101,3 +101,35 @@ def test_torch_wrappers_refuse_cpu_tensors(lib):
 def test_debug_wait_limit_validation(lib, limit_ns):
     # out-of-range limits are refused on the host, before any launch
     assert nb.lib().nystra_debug_wait_timeout(limit_ns, None) == nb.NYSTRA_EINVAL
+
+
+@pytest.mark.parametrize("N,d,m", [(64, 30, 16), (64, 32, 8), (64, 2, 16)])
+def test_debug_stages_size(lib, N, d, m):
+    # Qbar, Kbar, G_L^n, m_U, W, G_A^n, Z, Y, O
+    want = 2 * m * d + N * m + m + 2 * m * (d + 1) + 2 * m * m + N * d
+    assert nb.nystra_debug_stages_size(N, d, m) == want
+
+
+@pytest.mark.parametrize("N,d,m", [(256, 30, 16), (64, 31, 16), (64, 34, 16), (64, 30, 32), (64, 30, 4)])
+def test_debug_stages_size_rejects_other_shapes(lib, N, d, m):
+    assert nb.nystra_debug_stages_size(N, d, m) == nb.NYSTRA_EINVAL
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(dtype=3), nb.NYSTRA_EDTYPE),
+    (dict(N=256), nb.NYSTRA_EINVAL),          # only the 8x8-window path
+    (dict(m=32), nb.NYSTRA_EINVAL),
+    (dict(d=31), nb.NYSTRA_EINVAL),
+    (dict(iters=-1), nb.NYSTRA_EINVAL),
+    (dict(dtype=0, iters=7), nb.NYSTRA_EINVAL),  # fp32 runs this path up to 6 steps
+    (dict(unit=8), nb.NYSTRA_EINVAL),         # units are 0..7
+    (dict(unit=-1), nb.NYSTRA_EINVAL),
+    (dict(dump=0), nb.NYSTRA_EINVAL),
+    (dict(dump=5 * P + 4), nb.NYSTRA_EINVAL),  # misaligned
+])
+def test_debug_stages_argument_validation(lib, args, code):
+    a = dict(N=64, d=30, m=16, iters=6, dtype=1, unit=0, dump=5 * P)
+    a.update(args)
+    rc = nb.nystra_debug_stages(P, 2 * P, 3 * P, 4, 2, a["N"], a["d"], a["m"], a["iters"], a["dtype"],
+                                a["unit"], a["dump"], None)
+    assert rc == code
