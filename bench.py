@@ -36,13 +36,13 @@ METRIC = "Nystrom attention tokens*heads/s"
 # of those files changes.
 MEASURED_TRAFFIC = {
     "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
-                       "src_hash": "b19d756531d7d231", "bytes": 74_126_848},
+                       "src_hash": "4d6cb7b635cf81f4", "bytes": 74_126_848},
     "sr720p-w16-m16-bf16": {"files": ["common.cuh", "nystra_team.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu",
                                       "ptx.cuh"],
-                            "src_hash": "ae66abaad8e6a0ee", "bytes": 1_296_214_016},
+                            "src_hash": "0cbb314f440ebe77", "bytes": 1_296_214_016},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-                            "src_hash": "33de39f2486d54db", "bytes": 1_490_684_928},
+                            "src_hash": "d05940aee4079126", "bytes": 1_490_684_928},
 }
 
 
