@@ -1,0 +1,128 @@
+"""Throughput sweep over the synthetic workloads: PnP-Nystra and the exact
+window attention it replaces, on the same device inputs.
+
+    python -m paper_2506_08520_gb300.sweep [--list] [name ...]
+
+One JSON line per workload: the median CUDA-event time of each kernel over
+rotating input/output sets (together more than 3x the L2 size, so every launch
+reads its inputs from HBM), the algorithmic bytes (Q, K, V read once, O written
+once), the achieved GB/s and its fraction of the measured HBM copy bandwidth,
+tokens*heads/s (for edge-padded maps also counting only the real tokens), and
+the speedup over exact attention.  A mix ("uformer-mix": Uformer stages 1 and
+4) launches its workloads back to back on one stream and is timed as one.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import sys
+
+import torch
+
+from . import binding, workloads
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+# Workloads launched back to back and timed as one step.
+MIXES = {"uformer-mix": ("uformer-s1", "uformer-s4")}
+
+DEFAULT = (["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4", "uformer-mix"]
+           + [f"large-w{w}-m{m}" for w in (16, 32) for m in (32, 64)]
+           + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")])
+
+
+def hbm_peak_gbs() -> tuple[float, str]:
+    """Measured HBM copy bandwidth of this GPU pool, else the fallback figure."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def _real_tokens(wl: workloads.Workload) -> int:
+    if wl.recipe == "map":
+        H, W, _ = wl.map_hw
+        return H * W * wl.heads
+    return wl.units * wl.N
+
+
+def _median_ms(launch, n_sets: int, reps: int) -> float:
+    stream = torch.cuda.current_stream()
+    for i in range(min(5, reps)):
+        launch(i % n_sets)
+    torch.cuda.synchronize()
+    evs = []
+    for i in range(reps):
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s.record(stream)
+        launch(i % n_sets)
+        e.record(stream)
+        evs.append((s, e))
+    torch.cuda.synchronize()
+    return statistics.median(s.elapsed_time(e) for s, e in evs)
+
+
+def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int = 10) -> dict:
+    parts = [workloads.WORKLOADS[n] for n in MIXES.get(name, (name,))]
+    io = sum(wl.io_bytes for wl in parts)
+    n_sets = max(2, -(-3 * l2_bytes // io))
+    dev = torch.device("cuda")
+    sets = []
+    for wl in parts:
+        q, k, v = workloads.make_qkv(wl)
+        sets.append([tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),)
+                     for _ in range(n_sets)])
+
+    def nystra(i):
+        for wl, ss in zip(parts, sets):
+            a, b, c, o = ss[i]
+            binding.nystra(a, b, c, wl.m, wl.iters, out=o)
+
+    def exact(i):
+        for ss in sets:
+            a, b, c, o = ss[i]
+            binding.exact(a, b, c, out=o)
+
+    t_n = _median_ms(nystra, n_sets, reps)
+    t_e = _median_ms(exact, n_sets, exact_reps)
+    tokens = sum(wl.units * wl.N for wl in parts)
+    gbs = io / (t_n * 1e-3) / 1e9
+    res = {"name": name, "units": sum(wl.units for wl in parts), "io_MB": io / 1e6, "nystra_ms": t_n,
+           "exact_ms": t_e, "GBps": gbs, "frac_of_hbm": gbs / peak,
+           "tokens_heads_per_s": tokens / (t_n * 1e-3), "speedup_vs_exact": t_e / t_n}
+    real = sum(_real_tokens(wl) for wl in parts)
+    if real != tokens:
+        res["real_tokens_heads_per_s"] = real / (t_n * 1e-3)
+    del sets
+    torch.cuda.empty_cache()
+    return res
+
+
+def main(argv=None) -> int:
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("names", nargs="*", help="workloads or mixes (default: all)")
+    ap.add_argument("--list", action="store_true", help="print the workload names and exit")
+    ap.add_argument("--reps", type=int, default=50)
+    args = ap.parse_args(argv)
+    names = args.names or DEFAULT
+    unknown = [n for n in names if n not in workloads.WORKLOADS and n not in MIXES]
+    if unknown:
+        ap.error(f"unknown workloads: {unknown}")
+    if args.list:
+        print("\n".join(names))
+        return 0
+    binding.lib()  # fail loudly without the library
+    l2 = int(torch.cuda.get_device_properties(0).L2_cache_size)
+    peak, kind = hbm_peak_gbs()
+    for n in names:
+        r = run(n, l2, peak, reps=args.reps)
+        r["peak_gbs"], r["peak_kind"] = peak, kind
+        print(json.dumps(r), flush=True)
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -29,3 +29,17 @@ def test_warmup_below_three_is_refused():
     r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--warmup", "1"],
                        capture_output=True, text=True, timeout=120, cwd=ROOT)
     assert r.returncode != 0
+
+
+def test_sweep_names_resolve():
+    from paper_2506_08520_gb300 import sweep, workloads
+    for name in sweep.DEFAULT:
+        assert name in workloads.WORKLOADS or name in sweep.MIXES, name
+    for parts in sweep.MIXES.values():
+        assert all(p in workloads.WORKLOADS for p in parts)
+
+
+def test_sweep_list_runs_without_a_gpu(capsys):
+    from paper_2506_08520_gb300 import sweep
+    assert sweep.main(["--list", "uformer-mix", "tiny"]) == 0
+    assert capsys.readouterr().out.split() == ["uformer-mix", "tiny"]
