@@ -75,20 +75,33 @@ struct StreamLayout {
     static_assert(XB % 16 == 0 && SLOT % 16 == 0 && TL::WARP % 16 == 0 && BUF % 16 == 0, "16-byte alignment");
 };
 
-// Chunk task v of a team that processes `count` units, in order: for each
-// unit k, Q(k) x 4, KV(k) x 4, then OUT(k - 1) x 4 (k >= 1); finally
-// OUT(count - 1) x 4.  12 * count tasks.
+// Chunk task v of a team that processes `count` units (12 * count tasks, in
+// blocks of four chunks).  SHORT (the one-warp core of m <= 16): Q(0), KV(0),
+// then for k >= 1 Q(k), OUT(k - 1), KV(k), finally OUT(count - 1): a unit's Q
+// rows are read again two blocks after their first read, while they are
+// still in L2, and the core of unit k runs during Q(k + 1).  Otherwise (the
+// slower distributed core of m = 32): Q(k), KV(k), OUT(k - 1) for each k,
+// finally OUT(count - 1), so the core has two blocks to finish.
 struct StreamTask {
     int k, type, c;  // unit (team-local), 0 = Q, 1 = KV, 2 = OUT, chunk
 };
+template <bool SHORT>
 __device__ __forceinline__ StreamTask stream_task(int v, int count) {
-    int i;
-    if (v < 8) i = v;
-    else if (v < 12 * count - 4) i = v + 4;
-    else i = v + 12;
-    const int k = i / 12, r = i - 12 * k;
-    if (r < 8) return {k, r >> 2, r & 3};
-    return {k - 1, 2, r & 3};
+    if constexpr (SHORT) {
+        const int blk = v >> 2, c = v & 3;
+        if (blk < 2) return {0, blk, c};
+        const int k = (blk - 2) / 3 + 1, r = blk - 2 - 3 * (k - 1);
+        if (k == count) return {count - 1, 2, c};
+        return r == 0 ? StreamTask{k, 0, c} : (r == 1 ? StreamTask{k - 1, 2, c} : StreamTask{k, 1, c});
+    } else {
+        int i;  // position in the sequence Q(k) KV(k) OUT(k - 1), k = 0 .. count (without OUT(-1), Q/KV(count))
+        if (v < 8) i = v;
+        else if (v < 12 * count - 4) i = v + 4;
+        else i = v + 12;
+        const int k = i / 12, r = i - 12 * k;
+        if (r < 8) return {k, r >> 2, r & 3};
+        return {k - 1, 2, r & 3};
+    }
 }
 
 template <typename T, int M, int NCOL, int DC>
@@ -191,7 +204,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     const uint64_t keep = l2_evict_last(), drop = l2_evict_first();
     // lane 0: copies of task vv into its slot
     auto issue = [&](int vv) {
-        const StreamTask tk = stream_task(vv, count);
+        const StreamTask tk = stream_task<(M <= 16)>(vv, count);
         const int s = vv % NSLOT;
         const size_t off = chunk_off(u0 + tk.k * stride, tk.c);
         if (tk.type == 1) {
@@ -216,7 +229,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     float cq[2][1][4], ck[2][1][4], w[MT][NTO][4], run[MT][2];
     R aq[MT][2][4];
     for (int vv = 0; vv < total; ++vv) {
-        const StreamTask tk = stream_task(vv, count);
+        const StreamTask tk = stream_task<(M <= 16)>(vv, count);
         const int s = vv % NSLOT;
         const int b = tk.k & 1;
         unsigned char* bb = buf(b);
@@ -239,12 +252,18 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(cq, reinterpret_cast<T*>(bb + Lay::B_QB), r * LPW, g, t);
                 if (tsync_or(failed)) break;
+                if constexpr (M > 16)  // KV(k) follows directly
 #pragma unroll
-                for (int mt = 0; mt < MT; ++mt) qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), mt, g, t, aq[mt]);
+                    for (int mt = 0; mt < MT; ++mt)
+                        qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), mt, g, t, aq[mt]);
             }
         } else if (tk.type == 1) {
             // ---------------- KV(k): Kbar sums, S_U, partial W ----------------
             if (tk.c == 0) {
+                if constexpr (M <= 16)  // OUT(k - 1) ran since Q(k): reload Qbar's operands
+#pragma unroll
+                    for (int mt = 0; mt < MT; ++mt)
+                        qbar_afrag<T>(reinterpret_cast<const T*>(bb + Lay::B_QB), mt, g, t, aq[mt]);
 #pragma unroll
                 for (int mf = 0; mf < 2; ++mf) ck[mf][0][0] = ck[mf][0][1] = ck[mf][0][2] = ck[mf][0][3] = 0.f;
 #pragma unroll
