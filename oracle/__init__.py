@@ -34,12 +34,17 @@ def _load():
         lib.oracle_nystra_attention.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int,
                                                 ctypes.c_int, ctypes.c_int, ctypes.c_int]
         lib.oracle_nystra_attention.restype = ctypes.c_int
+        lib.oracle_nystra_attention_pool.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int,
+                                                     ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int]
+        lib.oracle_nystra_attention_pool.restype = ctypes.c_int
         lib.oracle_landmarks.argtypes = [_D, ctypes.c_int, ctypes.c_int, ctypes.c_int, _D]
         lib.oracle_landmarks.restype = None
+        lib.oracle_landmarks_patches.argtypes = [_D, ctypes.c_int, ctypes.c_int, ctypes.c_int, _D]
+        lib.oracle_landmarks_patches.restype = None
         lib.oracle_pinv_iteration.argtypes = [_D, ctypes.c_int, ctypes.c_int, _D]
         lib.oracle_pinv_iteration.restype = None
         lib.oracle_nystra_stages.argtypes = [_D, _D, _D, _D, ctypes.c_int, ctypes.c_int,
-                                             ctypes.c_int, ctypes.c_int] + [_D] * 10
+                                             ctypes.c_int, ctypes.c_int, ctypes.c_int] + [_D] * 10
         lib.oracle_nystra_stages.restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -69,24 +74,37 @@ def exact_attention(q, k, v) -> np.ndarray:
     return out
 
 
-def nystra_attention(q, k, v, m: int, iters: int) -> np.ndarray:
-    """PnP-Nystra output (Algorithm 1, stabilised form), float64 ``[..., N, d]``."""
+POOLS = {"segments": 0, "patches": 1}
+
+
+def nystra_attention(q, k, v, m: int, iters: int, pool: str = "segments") -> np.ndarray:
+    """PnP-Nystra output (Algorithm 1, stabilised form), float64 ``[..., N, d]``.
+
+    ``pool``: "segments" (m contiguous token runs) or "patches" (a square
+    window pooled over a square grid of m square patches)."""
     q, k, v = _f64(q), _f64(k), _f64(v)
     N, d = q.shape[-2], q.shape[-1]
     out = np.empty_like(q)
-    rc = _load().oracle_nystra_attention(_p(q), _p(k), _p(v), _p(out), q.size // (N * d),
-                                         N, d, int(m), int(iters))
+    rc = _load().oracle_nystra_attention_pool(_p(q), _p(k), _p(v), _p(out), q.size // (N * d),
+                                              N, d, int(m), int(iters), POOLS[pool])
     if rc != 0:
-        raise ValueError(f"oracle: invalid m={m} for N={N} (m must divide N), iters={iters}")
+        raise ValueError(f"oracle: invalid m={m} for N={N} with {pool} pooling, iters={iters}")
     return out
 
 
-def landmarks(x, m: int) -> np.ndarray:
-    """Segment-mean landmarks of one unit ``[N, d]`` -> ``[m, d]`` (Alg. 1 step 1)."""
+def landmarks(x, m: int, pool: str = "segments") -> np.ndarray:
+    """Landmarks of one unit ``[N, d]`` -> ``[m, d]`` (Alg. 1 step 1): segment
+    means, or with ``pool="patches"`` square-patch means of a square window."""
     x = _f64(x)
     N, d = x.shape
     out = np.empty((m, d))
-    _load().oracle_landmarks(_p(x), N, d, int(m), _p(out))
+    if pool == "patches":
+        w, p = int(round(N ** 0.5)), int(round(m ** 0.5))
+        if w * w != N or p * p != m or w % p:
+            raise ValueError(f"oracle: {m} square patches do not tile a window of {N} tokens")
+        _load().oracle_landmarks_patches(_p(x), N, d, int(m), _p(out))
+    else:
+        _load().oracle_landmarks(_p(x), N, d, int(m), _p(out))
     return out
 
 
@@ -99,7 +117,7 @@ def pinv_iteration(A, iters: int) -> np.ndarray:
     return Z
 
 
-def nystra_stages(q, k, v, m: int, iters: int) -> dict:
+def nystra_stages(q, k, v, m: int, iters: int, pool: str = "segments") -> dict:
     """All intermediates of one unit (``q, k, v``: ``[N, d]``)."""
     q, k, v = _f64(q), _f64(k), _f64(v)
     N, d = q.shape
@@ -110,9 +128,9 @@ def nystra_stages(q, k, v, m: int, iters: int) -> dict:
     }
     out = np.empty((N, d))
     order = ["qbar", "kbar", "mL", "mU", "GLn", "GUn", "GAn", "Z", "num", "den"]
-    rc = _load().oracle_nystra_stages(_p(q), _p(k), _p(v), _p(out), N, d, int(m), int(iters),
+    rc = _load().oracle_nystra_stages(_p(q), _p(k), _p(v), _p(out), N, d, int(m), int(iters), POOLS[pool],
                                       *[_p(st[n]) for n in order])
     if rc != 0:
-        raise ValueError(f"oracle: invalid m={m} for N={N}")
+        raise ValueError(f"oracle: invalid m={m} for N={N} with {pool} pooling")
     st["out"] = out
     return st

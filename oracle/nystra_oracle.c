@@ -17,7 +17,10 @@
  * Readings where the paper is silent (each also listed in the design notes):
  *   - landmarks are means over m contiguous, non-overlapping segments of
  *     L = N/m tokens in the window's token order (Sec. 2.2 "average pooling
- *     over non-overlapping windows"); m must divide N;
+ *     over non-overlapping windows"); m must divide N.  The other reading,
+ *     pool = 1: a square window of w x w tokens (N = w^2, row-major) pooled
+ *     over a p x p grid of square b x b patches (m = p^2, b = w/p), landmark
+ *     j = (row j/p, column j%p) of that grid;
  *   - the scale is 1/sqrt(d) with d the per-head dimension (Eq. 1, Sec. 1);
  *   - the pseudo-inverse is the third-order iteration
  *       Z_{k+1} = 1/4 Z_k (13 I - A Z_k (15 I - A Z_k (7 I - A Z_k)))
@@ -115,6 +118,36 @@ void oracle_landmarks(const double* x, int N, int d, int m, double* xbar) {
         }
 }
 
+/* Integer square root of n, or -1 if n is not a perfect square. */
+static int exact_sqrt(int n) {
+    int r = 0;
+    while ((r + 1) * (r + 1) <= n) ++r;
+    return r * r == n ? r : -1;
+}
+
+/* pool = 1 needs N = w^2, m = p^2 and p dividing w. */
+static int pool_valid(int N, int m, int pool) {
+    if (pool == 0) return N % m == 0;
+    if (pool != 1) return 0;
+    const int w = exact_sqrt(N), p = exact_sqrt(m);
+    return w > 0 && p > 0 && w % p == 0;
+}
+
+/* Step 1 over square patches (pool = 1): token t = (t/w, t%w) of the w x w
+ * window; landmark j averages the b x b tokens of patch (j/p, j%p),
+ *   xbar[j][c] = (1/b^2) sum_{r = (j/p) b}^{(j/p) b + b-1}
+ *                        sum_{s = (j%p) b}^{(j%p) b + b-1} x[r w + s][c]. */
+void oracle_landmarks_patches(const double* x, int N, int d, int m, double* xbar) {
+    const int w = exact_sqrt(N), p = exact_sqrt(m), b = w / p;
+    for (int j = 0; j < m; ++j)
+        for (int c = 0; c < d; ++c) {
+            double acc = 0.0;
+            for (int r = (j / p) * b; r < (j / p) * b + b; ++r)
+                for (int s = (j % p) * b; s < (j % p) * b + b; ++s) acc += x[((size_t)r * w + s) * d + c];
+            xbar[(size_t)j * d + c] = acc / (double)(b * b);
+        }
+}
+
 /* ------------------------------------------------------------------ */
 /* Algorithm 1, step 4: approximate (pseudo-)inverse of the m x m      */
 /* matrix A by the third-order iteration of Razavi et al. (2014):      */
@@ -181,7 +214,7 @@ typedef struct {
 } stage_ptrs;
 
 static void nystra_unit(const double* q, const double* k, const double* v, double* o,
-                        int N, int d, int m, int iters, stage_ptrs st) {
+                        int N, int d, int m, int iters, int pool, stage_ptrs st) {
     const double s = 1.0 / sqrt((double)d);
     double* qbar = (double*)malloc(sizeof(double) * (size_t)m * d);
     double* kbar = (double*)malloc(sizeof(double) * (size_t)m * d);
@@ -198,8 +231,13 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
     double* den = (double*)malloc(sizeof(double) * (size_t)N);
 
     /* Step 1: landmark queries and keys. */
-    oracle_landmarks(q, N, d, m, qbar);
-    oracle_landmarks(k, N, d, m, kbar);
+    if (pool == 1) {
+        oracle_landmarks_patches(q, N, d, m, qbar);
+        oracle_landmarks_patches(k, N, d, m, kbar);
+    } else {
+        oracle_landmarks(q, N, d, m, qbar);
+        oracle_landmarks(k, N, d, m, kbar);
+    }
 
     /* Steps 2-3 with row-max stabilisation.  S_L, its row max m_L. */
     for (int i = 0; i < N; ++i) {
@@ -271,26 +309,33 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
     free(Z); free(P); free(GUV); free(GU1); free(num); free(den);
 }
 
-/* Batched PnP-Nystra output.  Returns 0, or -1 if m does not divide N. */
-int oracle_nystra_attention(const double* q, const double* k, const double* v, double* out,
-                            long n_units, int N, int d, int m, int iters) {
-    if (m < 1 || m > N || N % m != 0 || iters < 0) return -1;
+/* Batched PnP-Nystra output with landmark pooling `pool` (0 = segments,
+ * 1 = square patches).  Returns 0, or -1 for an m the pooling cannot form. */
+int oracle_nystra_attention_pool(const double* q, const double* k, const double* v, double* out,
+                                 long n_units, int N, int d, int m, int iters, int pool) {
+    if (m < 1 || m > N || !pool_valid(N, m, pool) || iters < 0) return -1;
     const size_t unit = (size_t)N * d;
     const stage_ptrs none = {0};
 #pragma omp parallel for schedule(dynamic, 4)
     for (long u = 0; u < n_units; ++u)
-        nystra_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d, m, iters, none);
+        nystra_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d, m, iters, pool, none);
     return 0;
+}
+
+/* Batched PnP-Nystra output, segment landmarks.  -1 if m does not divide N. */
+int oracle_nystra_attention(const double* q, const double* k, const double* v, double* out,
+                            long n_units, int N, int d, int m, int iters) {
+    return oracle_nystra_attention_pool(q, k, v, out, n_units, N, d, m, iters, 0);
 }
 
 /* Single-unit PnP-Nystra exposing every intermediate (NULL to skip). */
 int oracle_nystra_stages(const double* q, const double* k, const double* v, double* out,
-                         int N, int d, int m, int iters,
+                         int N, int d, int m, int iters, int pool,
                          double* qbar, double* kbar, double* mL, double* mU,
                          double* GLn, double* GUn, double* GAn, double* Z,
                          double* num, double* den) {
-    if (m < 1 || m > N || N % m != 0 || iters < 0) return -1;
+    if (m < 1 || m > N || !pool_valid(N, m, pool) || iters < 0) return -1;
     stage_ptrs st = {qbar, kbar, mL, mU, GLn, GUn, GAn, Z, num, den};
-    nystra_unit(q, k, v, out, N, d, m, iters, st);
+    nystra_unit(q, k, v, out, N, d, m, iters, pool, st);
     return 0;
 }

@@ -321,3 +321,90 @@ def test_table6_trend_more_landmarks_and_iterations():
     print("err vs m (8,16,32):", err_m, " err vs iters (1,3,6):", err_i)
     assert err_m[0] > err_m[2]
     assert err_i[0] > err_i[2]
+
+
+# --------------------------------------------------------------------------
+# Step 1, the other reading of "average pooling over non-overlapping windows":
+# square patches of a square window.
+# --------------------------------------------------------------------------
+def _patch_major(w, p):
+    """Token order that lists patch 0's tokens first, then patch 1's, ... (row-major patches)."""
+    b = w // p
+    return np.array([(pr * b + r) * w + pc * b + c
+                     for pr in range(p) for pc in range(p) for r in range(b) for c in range(b)])
+
+
+@pytest.mark.parametrize("w,p", [(8, 4), (8, 2), (16, 4), (16, 8), (32, 4), (8, 8), (8, 1)])
+def test_patch_landmarks_integer_exact(w, p):
+    """Integer tokens: patch means equal the mean over the b x b block of the w x w grid."""
+    rng = _rng(31 + w + p)
+    N, d, b = w * w, 3, w // p
+    x = rng.integers(-40, 40, size=(N, d)).astype(np.float64)
+    ref = x.reshape(p, b, p, b, d).mean(axis=(1, 3)).reshape(p * p, d)
+    assert np.array_equal(oracle.landmarks(x, p * p, "patches"), ref)
+
+
+@pytest.mark.parametrize("w,p", [(8, 4), (16, 4), (16, 8)])
+def test_patches_are_segments_of_the_patch_major_order(w, p):
+    """Patch pooling of a window equals segment pooling after reordering its tokens
+    patch by patch; attention is equivariant under the token reordering."""
+    rng = _rng(41 + w + p)
+    N, d, m = w * w, 6, p * p
+    q, k, v = (rng.standard_normal((2, N, d)) for _ in range(3))
+    pm = _patch_major(w, p)
+    assert sorted(pm) == list(range(N))
+    out = oracle.nystra_attention(q, k, v, m, 6, "patches")
+    seg = oracle.nystra_attention(q[:, pm], k[:, pm], v[:, pm], m, 6)
+    np.testing.assert_allclose(out[:, pm], seg, rtol=1e-11, atol=1e-12)
+    for u in range(2):
+        np.testing.assert_array_equal(oracle.landmarks(q[u], m, "patches"), oracle.landmarks(q[u, pm], m))
+
+
+def test_patch_permutations():
+    """Swapping tokens inside a patch permutes output rows; across patches it does not."""
+    rng = _rng(43)
+    w, p, d = 8, 2, 5
+    N, m = w * w, p * p
+    q, k, v = (rng.standard_normal((N, d)) for _ in range(3))
+    base = oracle.nystra_attention(q[None], k[None], v[None], m, 6, "patches")[0]
+    inside = np.arange(N)
+    inside[[0, 3 * w + 3]] = inside[[3 * w + 3, 0]]  # both in patch (0, 0) (b = 4)
+    out = oracle.nystra_attention(q[inside][None], k[inside][None], v[inside][None], m, 6, "patches")[0]
+    np.testing.assert_allclose(out, base[inside], rtol=1e-10, atol=1e-12)
+    across = np.arange(N)
+    across[[3, 4]] = across[[4, 3]]  # same segment of 16 tokens, different patches
+    out2 = oracle.nystra_attention(q[across][None], k[across][None], v[across][None], m, 6, "patches")[0]
+    assert np.abs(out2 - base[across]).max() > 1e-6
+
+
+def test_patch_special_cases():
+    """m = N (1 x 1 patches) and m = 1 (one patch) coincide with the segment reading."""
+    rng = _rng(44)
+    N, d = 16, 4
+    q, k, v = (0.5 * rng.standard_normal((2, N, d)) for _ in range(3))
+    for m in (1, N):
+        np.testing.assert_array_equal(oracle.nystra_attention(q, k, v, m, 6, "patches"),
+                                      oracle.nystra_attention(q, k, v, m, 6))
+
+
+def test_patch_corollary_exact_recovery():
+    """Tokens constant within each square patch: rank(G~) = m and G^ = G (Corollary 2.2)."""
+    rng = _rng(45)
+    w, p, d = 8, 4, 6
+    b, m = w // p, p * p
+    qs, ks = rng.standard_normal((p, p, d)), rng.standard_normal((p, p, d))
+    up = lambda x: np.repeat(np.repeat(x, b, axis=0), b, axis=1).reshape(w * w, d)
+    q, k = up(qs), up(ks)
+    v = rng.standard_normal((w * w, d))
+    ref = oracle.exact_attention(q[None], k[None], v[None])
+    out = oracle.nystra_attention(q[None], k[None], v[None], m, 80, "patches")
+    assert _rel(out, ref) < 1e-8
+    seg = oracle.nystra_attention(q[None], k[None], v[None], m, 80)
+    assert _rel(seg, ref) > 1e-3  # the segment reading does not see the patch structure
+
+
+@pytest.mark.parametrize("N,m", [(64, 8), (48, 16), (64, 9), (256, 36)])
+def test_patch_shapes_that_do_not_tile_are_rejected(N, m):
+    x = np.zeros((1, N, 4))
+    with pytest.raises(ValueError):
+        oracle.nystra_attention(x, x, x, m, 6, "patches")
