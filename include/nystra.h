@@ -53,6 +53,14 @@ extern "C" {
 /* Element type of q, k, v and out. */
 typedef enum { NYSTRA_F32 = 0, NYSTRA_BF16 = 1, NYSTRA_F16 = 2 } nystra_dtype;
 
+/* Landmark pooling (Algorithm 1 step 1; Sec. 2.2 pools landmarks by averaging
+ * over non-overlapping windows, which reads two ways):
+ *  SEGMENTS  m contiguous runs of N/m tokens in the window's token order;
+ *  PATCHES   the window as a w x w grid (N = w^2, tokens row-major) cut into
+ *            a p x p grid of square b x b patches (m = p^2, b = w/p), landmark
+ *            j = patch (j / p, j % p). */
+typedef enum { NYSTRA_LANDMARKS_SEGMENTS = 0, NYSTRA_LANDMARKS_PATCHES = 1 } nystra_landmarks;
+
 /* Status codes returned by every entry point (0 = success, negative = error). */
 enum {
     NYSTRA_OK = 0,
@@ -102,6 +110,19 @@ enum {
 NYSTRA_API int nystra_attention(const void* q, const void* k, const void* v, void* out,
                      int n_windows, int heads, int N, int d_h, int m, int iters,
                      int dtype, void* stream);
+
+/*
+ * nystra_attention_ex -- nystra_attention with a choice of landmark pooling.
+ * `landmarks` is a nystra_landmarks value; NYSTRA_LANDMARKS_PATCHES needs N
+ * and m perfect squares with sqrt(m) dividing sqrt(N) (else NYSTRA_EINVAL).
+ * nystra_attention(...) is nystra_attention_ex(..., NYSTRA_LANDMARKS_SEGMENTS,
+ * ...).  Square patches run on the tensor cores for 16-bit I/O with m = 16
+ * and N in {64, 256, 1024} (even d_h <= 32), on the fp32 SIMT path otherwise.
+ * Other arguments, layout and return codes as nystra_attention.
+ */
+NYSTRA_API int nystra_attention_ex(const void* q, const void* k, const void* v, void* out,
+                                   int n_windows, int heads, int N, int d_h, int m, int iters,
+                                   int landmarks, int dtype, void* stream);
 
 /*
  * exact_window_attention -- exact softmax attention per unit, Eq. (1):
@@ -165,6 +186,7 @@ NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stre
  *   Z     m x m        the pseudo-inverse after `iters` steps (step 4)
  *   Y     m x (d_h+1)  Z W (the re-associated step 6)
  *   O     N x d_h      the output (step 7), as rounded to the I/O type
+ * `landmarks` is a nystra_landmarks value (square patches: 16-bit I/O, m = 16).
  * Supported: N = 64, m in {8, 16}, even d_h <= 32 (the shapes nystra_attention
  * runs on this path), fp32 I/O only with iters <= 6; anything else returns
  * NYSTRA_EINVAL, as do unit outside [0, n_windows*heads), null or misaligned
@@ -172,8 +194,8 @@ NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stre
  * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.
  */
 NYSTRA_API int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windows, int heads,
-                                   int N, int d_h, int m, int iters, int dtype, long long unit, float* dump,
-                                   void* stream);
+                                   int N, int d_h, int m, int iters, int landmarks, int dtype, long long unit,
+                                   float* dump, void* stream);
 
 /* Floats nystra_debug_stages writes for (N, d_h, m):
  * 2 m d_h + N m + m + 2 m (d_h+1) + 2 m^2 + N d_h; NYSTRA_EINVAL (negative)

@@ -16,6 +16,8 @@ LIB_PATH = os.path.join(_HERE, "libnystra.so")
 
 NYSTRA_F32, NYSTRA_BF16, NYSTRA_F16 = 0, 1, 2
 NYSTRA_OK, NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH, NYSTRA_ETIMEOUT, NYSTRA_EDEVICE = 0, -1, -2, -3, -4, -5
+NYSTRA_LANDMARKS_SEGMENTS, NYSTRA_LANDMARKS_PATCHES = 0, 1
+LANDMARKS = {"segments": NYSTRA_LANDMARKS_SEGMENTS, "patches": NYSTRA_LANDMARKS_PATCHES}
 MAX_N, MAX_DH, MAX_M, MAX_ITERS = 1024, 64, 64, 100
 
 _DTYPE_CODE = {torch.float32: NYSTRA_F32, torch.bfloat16: NYSTRA_BF16, torch.float16: NYSTRA_F16}
@@ -55,7 +57,9 @@ def lib() -> ctypes.CDLL:
         L.nystra_check.restype = i
         L.nystra_debug_wait_timeout.argtypes = [ctypes.c_ulonglong, vp]
         L.nystra_debug_wait_timeout.restype = i
-        L.nystra_debug_stages.argtypes = [vp, vp, vp, i, i, i, i, i, i, i, ctypes.c_longlong, vp, vp]
+        L.nystra_debug_stages.argtypes = [vp, vp, vp, i, i, i, i, i, i, i, i, ctypes.c_longlong, vp, vp]
+        L.nystra_attention_ex.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, vp]
+        L.nystra_attention_ex.restype = i
         L.nystra_debug_stages.restype = i
         L.nystra_debug_stages_size.argtypes = [i, i, i]
         L.nystra_debug_stages_size.restype = ctypes.c_longlong
@@ -67,6 +71,11 @@ def lib() -> ctypes.CDLL:
 def nystra_attention(q, k, v, out, n_windows, heads, N, d_h, m, iters, dtype, stream) -> int:
     """Raw C-ABI call: pointers as ints, returns the status code."""
     return lib().nystra_attention(q, k, v, out, n_windows, heads, N, d_h, m, iters, dtype, stream)
+
+
+def nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream) -> int:
+    """Raw C-ABI call with a landmark pooling (NYSTRA_LANDMARKS_*)."""
+    return lib().nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream)
 
 
 def exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream) -> int:
@@ -96,9 +105,10 @@ def debug_wait_timeout(limit_ns: int, stream=None) -> int:
     return lib().nystra_debug_wait_timeout(int(limit_ns), _stream_ptr(stream))
 
 
-def nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, dtype, unit, dump, stream) -> int:
+def nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, landmarks, dtype, unit, dump, stream) -> int:
     """Raw C-ABI call of the test-only stage dump (see the header)."""
-    return lib().nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, dtype, int(unit), dump, stream)
+    return lib().nystra_debug_stages(q, k, v, n_windows, heads, N, d_h, m, iters, landmarks, dtype, int(unit), dump,
+                                     stream)
 
 
 def nystra_debug_stages_size(N: int, d_h: int, m: int) -> int:
@@ -143,14 +153,19 @@ def _check(q, k, v, out):
 
 
 def nystra(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int = 16, iters: int = 6,
-           out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
-    """PnP-Nystra attention of device tensors ``[n_windows, heads, N, d_h]``."""
+           out: torch.Tensor | None = None, stream=None, landmarks: str = "segments") -> torch.Tensor:
+    """PnP-Nystra attention of device tensors ``[n_windows, heads, N, d_h]``;
+    ``landmarks`` is "segments" (default) or "patches" (square patches)."""
     out = torch.empty_like(q) if out is None else out
     _check(q, k, v, out)
     nw, h, N, d = _geometry(q)
     with torch.cuda.device(q.device):
-        rc = nystra_attention(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
-                              m, iters, _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+        if landmarks == "segments":
+            rc = nystra_attention(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
+                                  m, iters, _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+        else:
+            rc = nystra_attention_ex(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
+                                     m, iters, LANDMARKS[landmarks], _DTYPE_CODE[q.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention")
     return out
@@ -171,7 +186,7 @@ def exact(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tensor |
 
 
 def debug_stages(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int, iters: int, unit: int,
-                 stream=None) -> dict:
+                 stream=None, landmarks: str = "segments") -> dict:
     """Test-only: every intermediate of one unit (fp32 CPU tensors by name)."""
     _check(q, k, v, q)
     nw, h, N, d = _geometry(q)
@@ -181,7 +196,8 @@ def debug_stages(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int, iter
     dump = torch.empty(size, dtype=torch.float32, device=q.device)
     with torch.cuda.device(q.device):
         rc = nystra_debug_stages(q.data_ptr(), k.data_ptr(), v.data_ptr(), nw, h, N, d, m, iters,
-                                 _DTYPE_CODE[q.dtype], unit, dump.data_ptr(), _stream_ptr(stream))
+                                 LANDMARKS[landmarks], _DTYPE_CODE[q.dtype], unit, dump.data_ptr(),
+                                 _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_debug_stages")
     torch.cuda.synchronize(q.device)

@@ -37,35 +37,57 @@ int check_common(const void* q, const void* k, const void* v, void* out, int n_w
     return NYSTRA_OK;
 }
 
+// Integer square root of n, or -1 if n is not a perfect square.
+int exact_sqrt(int n) {
+    int r = 0;
+    while ((r + 1) * (r + 1) <= n) ++r;
+    return r * r == n ? r : -1;
+}
+
 }  // namespace
 
 extern "C" {
 
-int nystra_attention(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
-                     int N, int d_h, int m, int iters, int dtype, void* stream) {
+int nystra_attention_ex(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                        int N, int d_h, int m, int iters, int landmarks, int dtype, void* stream) {
     int rc = check_common(q, k, v, out, n_windows, heads, N, d_h, dtype);
     if (rc != NYSTRA_OK) return rc;
     if (m < 1 || m > N || m > NYSTRA_MAX_M || N % m != 0) return NYSTRA_EINVAL;
     if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
+    const bool patches = landmarks == NYSTRA_LANDMARKS_PATCHES;
+    if (patches) {  // a square grid of square patches must tile the square window
+        const int w = exact_sqrt(N), p = exact_sqrt(m);
+        if (w < 0 || p < 0 || w % p != 0) return NYSTRA_EINVAL;
+    }
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
     const cudaStream_t s = (cudaStream_t)stream;
     // fp32 I/O on the tensor cores: 8x8 windows, m <= 16, at most the paper's 6
     // iterations (beyond them the fp16-split iteration's round-off, amplified
     // by ||G_A^n|| ||Z||, exceeds what fp32 I/O asks; the SIMT path iterates in fp32).
-    const bool tc16 = (dtype == NYSTRA_BF16 || dtype == NYSTRA_F16) && (m == 8 || m == 16 || m == 32 || m == 64);
-    const bool tc32 = dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
+    // Square patches on the tensor cores: 16-bit I/O with m = 16.
+    const bool io16 = dtype == NYSTRA_BF16 || dtype == NYSTRA_F16;
+    const bool tc16 = io16 && (patches ? m == 16 : (m == 8 || m == 16 || m == 32 || m == 64));
+    const bool tc32 = !patches && dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
     const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32;
+    const int pool = patches ? 1 : 0;
     cudaError_t e;
     if (tc && N == 64)
-        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, dtype, s);
+        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
     else if (tc && N == 256)
-        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, dtype, s);
+        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
     else if (tc && N == 1024)
-        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, dtype, s);
+        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
     else
-        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, dtype, s);
+        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, pool, dtype, s);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
+int nystra_attention(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                     int N, int d_h, int m, int iters, int dtype, void* stream) {
+    return nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, NYSTRA_LANDMARKS_SEGMENTS,
+                               dtype, stream);
 }
 
 int exact_window_attention(const void* q, const void* k, const void* v, void* out, int n_windows,
@@ -112,14 +134,17 @@ long long nystra_debug_stages_size(int N, int d_h, int m) {
 }
 
 int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windows, int heads, int N, int d_h,
-                        int m, int iters, int dtype, long long unit, float* dump, void* stream) {
+                        int m, int iters, int landmarks, int dtype, long long unit, float* dump, void* stream) {
     if (dtype != NYSTRA_F32 && dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;
     if (nystra_debug_stages_size(N, d_h, m) < 0) return NYSTRA_EINVAL;
     if (iters < 0 || iters > NYSTRA_MAX_ITERS || (dtype == NYSTRA_F32 && iters > 6)) return NYSTRA_EINVAL;
+    // square patches: the 16-bit I/O path with m = 16 (2x2 patches)
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
+    if (landmarks == NYSTRA_LANDMARKS_PATCHES && (m != 16 || dtype == NYSTRA_F32)) return NYSTRA_EINVAL;
     if (n_windows < 0 || heads < 0 || unit < 0 || unit >= (long long)n_windows * heads) return NYSTRA_EINVAL;
     if (!q || !k || !v || !dump) return NYSTRA_EINVAL;
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dump)) return NYSTRA_EINVAL;
-    const cudaError_t e = nystra_host::launch_debug_stages(q, k, v, unit, d_h, m, iters, dtype, dump,
+    const cudaError_t e = nystra_host::launch_debug_stages(q, k, v, unit, d_h, m, iters, landmarks, dtype, dump,
                                                            (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }

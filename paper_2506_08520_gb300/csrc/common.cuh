@@ -29,19 +29,21 @@ template <> __device__ __forceinline__ float ldg_f32<float>(const float* p) { re
 // Host-side launchers (one per kernel family), defined in their .cu files.
 // Each returns a cudaError_t of the launch.
 namespace nystra_host {
+// pool: landmark pooling, 0 = segments, 1 = square patches of a square window.
 cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, void* out,
-                                  long long n_units, int N, int d, int m, int iters, int dtype,
+                                  long long n_units, int N, int d, int m, int iters, int pool, int dtype,
                                   cudaStream_t stream);
 cudaError_t launch_exact_generic(const void* q, const void* k, const void* v, void* out,
                                  long long n_units, int N, int d, int dtype, cudaStream_t stream);
-// Tensor-core kernels, 16-bit I/O, windows of 64 / 256 / 1024 tokens
-// (nystra_tc_n*.cu); m in {8, 16, 32}, even d_h <= 32.
+// Tensor-core kernels, windows of 64 / 256 / 1024 tokens (nystra_tc_n*.cu):
+// 16-bit I/O with m in {8, 16, 32, 64}, fp32 I/O at N = 64 with m in {8, 16};
+// even d_h <= 32.  Square-patch landmarks (pool = 1): 16-bit I/O, m = 16.
 cudaError_t launch_nystra_tc_n64(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                 int d, int m, int iters, int dtype, cudaStream_t stream);
+                                 int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
 cudaError_t launch_nystra_tc_n256(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                  int d, int m, int iters, int dtype, cudaStream_t stream);
+                                  int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
 cudaError_t launch_nystra_tc_n1024(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                   int d, int m, int iters, int dtype, cudaStream_t stream);
+                                   int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
 unsigned int take_fault_word_tc_n64(cudaError_t* err);
 unsigned int take_fault_word_tc_n256(cudaError_t* err);
 unsigned int take_fault_word_tc_n1024(cudaError_t* err);
@@ -57,6 +59,6 @@ cudaError_t launch_debug_wait(unsigned long long limit_ns, cudaStream_t stream);
 // Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
 long long debug_stages_size(int N, int d, int m);
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,
-                                int iters, int dtype, float* dump, cudaStream_t stream);
+                                int iters, int pool, int dtype, float* dump, cudaStream_t stream);
 unsigned int take_fault_word_debug(cudaError_t* err);
 }  // namespace nystra_host

@@ -1,9 +1,10 @@
 // Test-only stage dump of the tensor-core path for 8x8 windows (N = 64,
-// m in {8, 16}, even d_h <= 32): one warp runs, for one unit, the same phase
-// functions the stage-pool kernel runs (landmarks_mma, gl_tile, front_su_w,
-// core_warp, output_rows) and writes every intermediate in fp32, so tests can
-// hold each step of Algorithm 1 against the float64 oracle on its own.  The
-// paper has no counterpart; nystra_attention never calls this.
+// m in {8, 16}, even d_h <= 32; square-patch landmarks with m = 16): one warp
+// runs, for one unit, the same phase functions the stage-pool kernel runs
+// (landmarks_mma, gl_tile, front_su_w, core_warp, output_rows) and writes
+// every intermediate in fp32, so tests can hold each step of Algorithm 1
+// against the float64 oracle on its own.  The paper has no counterpart;
+// nystra_attention never calls this.
 #include "common.cuh"
 #include "nystra_tc.cuh"
 
@@ -56,7 +57,7 @@ struct DumpOffsets {
     }
 };
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW>
 __global__ void __launch_bounds__(32, 1)
 nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, long long unit,
                     int d, int iters, float sl2, float* __restrict__ dump) {
@@ -85,8 +86,8 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
     __syncwarp();
 
     // step 1: landmarks
-    landmarks_mma<T, 64, L>(Qs, qbar, 0, d, g, t);
-    landmarks_mma<T, 64, L>(Ks, kbar, 0, d, g, t);
+    landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
+    landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
     if constexpr (M < P::MP) {
         for (int idx = lane; idx < (P::MP - M) * 32; idx += 32) {
             const int jr = M + (idx >> 5), e = idx & 31;
@@ -143,11 +144,11 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
     for (int i = lane; i < 64 * d; i += 32) dump[off.out + i] = to_f32(ob[i]);
 }
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_stage(const void* q, const void* k, const void* v, long long unit, int d, int iters,
                          float* dump, cudaStream_t stream) {
     using P = StageLayout<T, M, NCOL>;
-    auto kern = nystra_stage_kernel<T, M, NCOL>;
+    auto kern = nystra_stage_kernel<T, M, NCOL, PW>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
     if (e != cudaSuccess) return e;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
@@ -157,13 +158,19 @@ cudaError_t launch_stage(const void* q, const void* k, const void* v, long long 
 
 template <typename T>
 cudaError_t launch_stage_t(const void* q, const void* k, const void* v, long long unit, int d, int m, int iters,
-                           float* dump, cudaStream_t stream) {
+                           int pool, float* dump, cudaStream_t stream) {
     const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
+    if (pool != 0) {  // square patches: 16-bit I/O, m = 16, 2x2 patches of the 8x8 window
+        if constexpr (sizeof(T) == 2)
+            return wide ? launch_stage<T, 16, 40, 8>(q, k, v, unit, d, iters, dump, stream)
+                        : launch_stage<T, 16, 32, 8>(q, k, v, unit, d, iters, dump, stream);
+        return cudaErrorInvalidValue;  // not reached: checked by the caller
+    }
     if (m == 8)
-        return wide ? launch_stage<T, 8, 40>(q, k, v, unit, d, iters, dump, stream)
-                    : launch_stage<T, 8, 32>(q, k, v, unit, d, iters, dump, stream);
-    return wide ? launch_stage<T, 16, 40>(q, k, v, unit, d, iters, dump, stream)
-                : launch_stage<T, 16, 32>(q, k, v, unit, d, iters, dump, stream);
+        return wide ? launch_stage<T, 8, 40, 0>(q, k, v, unit, d, iters, dump, stream)
+                    : launch_stage<T, 8, 32, 0>(q, k, v, unit, d, iters, dump, stream);
+    return wide ? launch_stage<T, 16, 40, 0>(q, k, v, unit, d, iters, dump, stream)
+                : launch_stage<T, 16, 32, 0>(q, k, v, unit, d, iters, dump, stream);
 }
 
 }  // namespace
@@ -175,11 +182,11 @@ namespace nystra_host {
 long long debug_stages_size(int N, int d, int m) { return nystra::tc::DumpOffsets(N, d, m).total; }
 
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,
-                                int iters, int dtype, float* dump, cudaStream_t stream) {
+                                int iters, int pool, int dtype, float* dump, cudaStream_t stream) {
     using namespace nystra::tc;
-    if (dtype == 0) return launch_stage_t<float>(q, k, v, unit, d, m, iters, dump, stream);
-    if (dtype == 1) return launch_stage_t<__nv_bfloat16>(q, k, v, unit, d, m, iters, dump, stream);
-    return launch_stage_t<__half>(q, k, v, unit, d, m, iters, dump, stream);
+    if (dtype == 0) return launch_stage_t<float>(q, k, v, unit, d, m, iters, pool, dump, stream);
+    if (dtype == 1) return launch_stage_t<__nv_bfloat16>(q, k, v, unit, d, m, iters, pool, dump, stream);
+    return launch_stage_t<__half>(q, k, v, unit, d, m, iters, pool, dump, stream);
 }
 
 }  // namespace nystra_host

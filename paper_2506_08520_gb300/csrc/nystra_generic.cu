@@ -3,7 +3,7 @@
 // One CTA (256 threads) per (window, head) unit, all arithmetic in fp32 with
 // correctly rounded expf.  Q, K and V are streamed from global memory in
 // token chunks, so shared memory only holds the O(m^2 + m d) state:
-//   pass 1  landmarks Qbar, Kbar (segment means, Algorithm 1 step 1);
+//   pass 1  landmarks Qbar, Kbar (segment or square-patch means, Algorithm 1 step 1);
 //   pass 2  K and V chunks: S_U = s Qbar K^T with a running row max m_U and
 //           W = G_U^n [V | 1] accumulated with the usual online rescaling,
 //           so that at the end W = exp(S_U - m_U) [V | 1] for the final m_U;
@@ -48,9 +48,12 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads)
 nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                       T* __restrict__ out, long long n_units, int N, int d, int m, int iters,
-                      float scale) {
+                      int pw, float scale) {
     extern __shared__ float sm[];
     const int d1 = d + 1, L = N / m, tid = threadIdx.x;
+    int pp = 0;  // patches per patch row (square-patch landmarks)
+    if (pw > 0)
+        while ((pp + 1) * (pp + 1) <= m) ++pp;
     float* qbar = sm;              // m*d
     float* kbar = qbar + m * d;    // m*d
     float* W = kbar + m * d;       // m*d1   G_U^n [V | 1]
@@ -75,13 +78,23 @@ nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T*
         const T* vu = v + base;
         T* ou = out + base;
 
-        // ---- pass 1: landmarks (Algorithm 1 step 1) ----
+        // ---- pass 1: landmarks (Algorithm 1 step 1): segments of L tokens,
+        // or (pw > 0) pb x pb patches of the pw-wide window, pb^2 = L ----
         for (int idx = tid; idx < m * d; idx += blockDim.x) {
             const int j = idx / d, c = idx - (idx / d) * d;
             float a = 0.f, b = 0.f;
-            for (int t = j * L; t < (j + 1) * L; ++t) {
-                a += ldg_f32(qu + (size_t)t * d + c);
-                b += ldg_f32(ku + (size_t)t * d + c);
+            if (pw == 0) {
+                for (int t = j * L; t < (j + 1) * L; ++t) {
+                    a += ldg_f32(qu + (size_t)t * d + c);
+                    b += ldg_f32(ku + (size_t)t * d + c);
+                }
+            } else {
+                const int pb = pw / pp, r0 = (j / pp) * pb, s0 = (j % pp) * pb;
+                for (int r = r0; r < r0 + pb; ++r)
+                    for (int s = s0; s < s0 + pb; ++s) {
+                        a += ldg_f32(qu + (size_t)(r * pw + s) * d + c);
+                        b += ldg_f32(ku + (size_t)(r * pw + s) * d + c);
+                    }
             }
             qbar[idx] = a / (float)L;
             kbar[idx] = b / (float)L;
@@ -230,14 +243,17 @@ size_t generic_smem_bytes(int d, int m) {
 
 template <typename T>
 cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, long long n_units, int N,
-                     int d, int m, int iters, cudaStream_t stream) {
+                     int d, int m, int iters, int pool, cudaStream_t stream) {
+    int pw = 0;  // window width for square patches
+    if (pool != 0)
+        while ((pw + 1) * (pw + 1) <= N) ++pw;
     const size_t smem = generic_smem_bytes(d, m);
     cudaError_t e = cudaFuncSetAttribute(nystra_generic_kernel<T>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     const long long grid = n_units < (1LL << 30) ? n_units : (1LL << 30);
     nystra_generic_kernel<T><<<(unsigned)grid, kThreads, smem, stream>>>(
-        (const T*)q, (const T*)k, (const T*)v, (T*)out, n_units, N, d, m, iters, 1.0f / sqrtf((float)d));
+        (const T*)q, (const T*)k, (const T*)v, (T*)out, n_units, N, d, m, iters, pw, 1.0f / sqrtf((float)d));
     return cudaGetLastError();
 }
 
@@ -246,13 +262,13 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
 
 namespace nystra_host {
 cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, void* out,
-                                  long long n_units, int N, int d, int m, int iters, int dtype,
+                                  long long n_units, int N, int d, int m, int iters, int pool, int dtype,
                                   cudaStream_t stream) {
     using namespace nystra;
     switch (dtype) {
-        case 0: return launch_t<float>(q, k, v, out, n_units, N, d, m, iters, stream);
-        case 1: return launch_t<__nv_bfloat16>(q, k, v, out, n_units, N, d, m, iters, stream);
-        default: return launch_t<__half>(q, k, v, out, n_units, N, d, m, iters, stream);
+        case 0: return launch_t<float>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
+        case 1: return launch_t<__nv_bfloat16>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
+        default: return launch_t<__half>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
     }
 }
 }  // namespace nystra_host

@@ -57,7 +57,7 @@ struct PoolLayout {
     static_assert(BYTES <= kSmemLimit, "pool does not fit in shared memory");
 };
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 __global__ void __launch_bounds__(PoolLayout<T, M, NCOL>::NW * 32, 1)
 nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, T* __restrict__ out,
                    long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
@@ -120,8 +120,8 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         if (lane == 0) bulk_wait_read_all();
         __syncwarp();
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
-        landmarks_mma<T, 64, L>(Qs, qbar, 0, d, g, t);
-        landmarks_mma<T, 64, L>(Ks, kbar, 0, d, g, t);
+        landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
+        landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
         if constexpr (M < P::MP) {  // zero the padding landmark rows
             for (int idx = lane; idx < (P::MP - M) * 32; idx += 32) {
                 const int jr = M + (idx >> 5), e = idx & 31;
@@ -166,11 +166,11 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (*cnt > consumed) (void)__all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault) {
     using P = PoolLayout<T, M, NCOL>;
-    auto kern = nystra_pool_kernel<T, M, NCOL, DC>;
+    auto kern = nystra_pool_kernel<T, M, NCOL, DC, PW>;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
@@ -192,15 +192,15 @@ cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* ou
 
 // The common head widths get kernels with d_h as a compile-time constant
 // (constant strides and column bounds); others read it at run time.
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                      int iters, cudaStream_t stream, unsigned int* fault) {
     if constexpr (NCOL == 32) {
-        if (d == 30) return launch_pool_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 30) return launch_pool_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {
-        if (d == 32) return launch_pool_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 32) return launch_pool_dc<T, M, NCOL, 32, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     }
-    return launch_pool_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
+    return launch_pool_dc<T, M, NCOL, 0, PW>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc

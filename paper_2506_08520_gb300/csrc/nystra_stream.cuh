@@ -104,7 +104,7 @@ __device__ __forceinline__ StreamTask stream_task(int v, int count) {
     }
 }
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 __global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * StreamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                      T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
@@ -248,7 +248,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             if (tk.c == 0)
 #pragma unroll
                 for (int mf = 0; mf < 2; ++mf) cq[mf][0][0] = cq[mf][0][1] = cq[mf][0][2] = cq[mf][0][3] = 0.f;
-            landmarks_acc<T, L, LPW>(X0, tk.c * Lay::CH, cq, d, g, t);
+            landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, cq, d, g, t);
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(cq, reinterpret_cast<T*>(bb + Lay::B_QB), r * LPW, g, t);
                 if (tsync_or(failed)) break;
@@ -273,7 +273,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                     run[mt][0] = run[mt][1] = -INFINITY;
                 }
             }
-            landmarks_acc<T, L, LPW>(X0, tk.c * Lay::CH, ck, d, g, t);
+            landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, ck, d, g, t);
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt)
                 su_w_chunk<T, NCOL>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M, 16 * mt + g + 8 < M,
@@ -342,11 +342,11 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
         (void)__all_sync(0xffffffffu, mbar_wait_bounded(sbar + i % NSLOT, (uint32_t)((i / NSLOT) & 1), kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                           int iters, cudaStream_t stream, unsigned int* fault) {
     using Lay = StreamLayout<M, NCOL>;
-    auto kern = nystra_stream_kernel<T, M, NCOL, DC>;
+    auto kern = nystra_stream_kernel<T, M, NCOL, DC, PW>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -371,15 +371,15 @@ cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* 
 
 // The common head widths get kernels with d_h as a compile-time constant
 // (constant strides and column bounds); others read it at run time.
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                      int iters, cudaStream_t stream, unsigned int* fault) {
     if constexpr (NCOL == 32) {
-        if (d == 30) return launch_stream_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 30) return launch_stream_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {
-        if (d == 32) return launch_stream_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 32) return launch_stream_dc<T, M, NCOL, 32, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     }
-    return launch_stream_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
+    return launch_stream_dc<T, M, NCOL, 0, PW>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc

@@ -433,11 +433,38 @@ struct GlPark {
 // range) to the accumulators c (features x the warp's LPW segments);
 // landmarks_put rounds the means to the I/O type and stores them as rows
 // j0.. of xbar (row stride LS); columns >= d come out as zeros.
-template <typename T, int L, int LPW>
+//
+// PW > 0 pools square patches instead of segments: the window is PW tokens
+// wide, a landmark averages a B x B patch (B^2 = L) and the patches of a
+// patch row are numbered left to right.  A warp's token range starts on a
+// patch-row boundary, so its landmarks are again LPW consecutive rows.
+template <int L, int PW>
+struct Pooling {
+    static constexpr int B = (L == 1) ? 1 : (L == 4) ? 2 : (L == 16) ? 4 : (L == 64) ? 8 : (L == 256) ? 16 : 0;
+    static constexpr int P = PW > 0 ? PW / (B > 0 ? B : 1) : 0;  // patches per patch row
+    static_assert(PW == 0 || (B > 0 && B * B == L && PW % B == 0), "square patches must tile the window");
+    // warp-local landmark of warp-local token tok
+    static __device__ __forceinline__ int of(int tok) {
+        if constexpr (PW == 0) return tok / L;
+        else return ((tok / PW) / B) * P + (tok % PW) / B;
+    }
+    // n-tiles of landmarks (8 per tile) met by the 16 tokens tk .. tk+15
+    static __device__ __forceinline__ int tile_lo(int tk) {
+        if constexpr (PW == 0) return (tk / L) / 8;
+        else return (((tk / PW) / B) * P) / 8;
+    }
+    static __device__ __forceinline__ int tile_hi(int tk) {
+        if constexpr (PW == 0) return ((tk + 15) / L) / 8;
+        else return ((((tk + 15) / PW) / B) * P + P - 1) / 8;
+    }
+};
+
+template <typename T, int L, int LPW, int PW = 0>
 __device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2][(LPW + 7) / 8][4], int d, int g,
                                               int t) {
     using O = Opnd<T>;
     using R = typename O::Reg;
+    using Pool = Pooling<L, PW>;
     constexpr int NTJ = (LPW + 7) / 8;
     constexpr float inv = 1.f / (float)L;
 #pragma unroll
@@ -453,12 +480,12 @@ __device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2
                 a[mf][r] = O::tr(x);
             }
         const int tk = tok0 + 16 * ks;
-        const int jlo = (tk / L) / 8, jhi = ((tk + 15) / L) / 8;
+        const int jlo = Pool::tile_lo(tk), jhi = Pool::tile_hi(tk);
 #pragma unroll
         for (int j = 0; j < NTJ; ++j) {
             if (j < jlo || j > jhi) continue;  // warp-uniform
-            // B = P^T: tokens tk + 2t (+1) (+8, +9), segment 8j + g
-            auto pv = [&](int tok) -> float { return (tok / L == 8 * j + g) ? inv : 0.f; };
+            // B = P^T: tokens tk + 2t (+1) (+8, +9), landmark 8j + g
+            auto pv = [&](int tok) -> float { return (Pool::of(tok) == 8 * j + g) ? inv : 0.f; };
             const int k0 = tk + 2 * t;
             const R b0 = O::pk(pv(k0), pv(k0 + 1)), b1 = O::pk(pv(k0 + 8), pv(k0 + 9));
 #pragma unroll
@@ -482,7 +509,7 @@ __device__ __forceinline__ void landmarks_put(const float (&c)[2][(LPW + 7) / 8]
 }
 
 // All TPW tokens of the warp (a multiple of 64), then the store.
-template <typename T, int TPW, int L>
+template <typename T, int TPW, int L, int PW = 0>
 __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
     constexpr int LPW = TPW / L, NTJ = (LPW + 7) / 8;
     float c[2][NTJ][4];
@@ -491,7 +518,7 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 #pragma unroll
         for (int j = 0; j < NTJ; ++j) c[mf][j][0] = c[mf][j][1] = c[mf][j][2] = c[mf][j][3] = 0.f;
 #pragma unroll
-    for (int ch = 0; ch < TPW / 64; ++ch) landmarks_acc<T, L, LPW>(X + ch * 64 * d, ch * 64, c, d, g, t);
+    for (int ch = 0; ch < TPW / 64; ++ch) landmarks_acc<T, L, LPW, PW>(X + ch * 64 * d, ch * 64, c, d, g, t);
     landmarks_put<T, LPW>(c, xbar, j0, g, t);
 }
 
@@ -1575,13 +1602,14 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
     return cudaGetLastError();
 }
 
-// Stage-pool kernel for 8x8 windows (nystra_pool.cuh, N = 64 translation unit only).
-template <typename T, int M, int NCOL>
+// Stage-pool kernel for 8x8 windows (nystra_pool.cuh, N = 64 translation unit
+// only).  PW: 0 = segment landmarks, else square patches of a PW-wide window.
+template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault);
 
 // Team kernel for 16x16 windows (nystra_team.cuh, N = 256 translation unit only).
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault);
 
@@ -1602,7 +1630,7 @@ cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, l
 }
 
 // Streaming team kernel for 32x32 windows (nystra_stream.cuh, N = 1024 translation unit only).
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                           int iters, cudaStream_t stream, unsigned int* fault);
 
@@ -1662,6 +1690,25 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
     return cudaErrorInvalidValue;  // not reached: m is checked by the caller
 }
 
+// Square-patch landmarks on the tensor cores: 16-bit I/O, m = 16 (4 x 4
+// patches of 2x2, 4x4 or 8x8 tokens), one window size per translation unit.
+template <typename T, int TPW, int WPU>
+cudaError_t launch_patches(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
+                           int m, int iters, cudaStream_t stream, unsigned int* fault) {
+    const bool wide = d > 30;
+    if (m != 16) return cudaErrorInvalidValue;  // not reached: checked by the caller
+    if constexpr (TPW == 64 && WPU == 1)
+        return wide ? launch_pool<T, 16, 40, 8>(q, k, v, out, n_units, d, iters, stream, fault)
+                    : launch_pool<T, 16, 32, 8>(q, k, v, out, n_units, d, iters, stream, fault);
+    if constexpr (TPW == 64 && WPU == 4)
+        return wide ? launch_team<T, 16, 40, 16>(q, k, v, out, n_units, d, iters, stream, fault)
+                    : launch_team<T, 16, 32, 16>(q, k, v, out, n_units, d, iters, stream, fault);
+    if constexpr (TPW == 128 && WPU == 8)
+        return wide ? launch_stream<T, 16, 40, 32>(q, k, v, out, n_units, d, iters, stream, fault)
+                    : launch_stream<T, 16, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+    return cudaErrorInvalidValue;
+}
+
 }  // namespace tc
 }  // namespace nystra
 
@@ -1672,7 +1719,7 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
     }                                                                                                        \
     namespace nystra_host {                                                                                  \
     cudaError_t launch_nystra_tc_##NAME(const void* q, const void* k, const void* v, void* out,              \
-                                        long long n_units, int d, int m, int iters, int dtype,               \
+                                        long long n_units, int d, int m, int iters, int pool, int dtype,     \
                                         cudaStream_t stream) {                                               \
         static unsigned int* s_fault[64] = {};  /* device address of the fault word, per device */      \
         int dev = 0;                                                                                         \
@@ -1684,6 +1731,15 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
             if (e != cudaSuccess) return e;                                                                  \
         }                                                                                                    \
         unsigned int* fault = s_fault[dev];                                                                  \
+        if (pool != 0) {                                                                                     \
+            if (dtype == 1)                                                                                  \
+                return nystra::tc::launch_patches<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m,      \
+                                                                           iters, stream, fault);            \
+            if (dtype == 2)                                                                                  \
+                return nystra::tc::launch_patches<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters,      \
+                                                                    stream, fault);                          \
+            return cudaErrorInvalidValue; /* not reached: fp32 patches take the SIMT path */                 \
+        }                                                                                                    \
         if (dtype == 0)                                                                                      \
             return nystra::tc::launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault);      \
         if (dtype == 1)                                                                                      \

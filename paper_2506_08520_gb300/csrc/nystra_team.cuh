@@ -61,7 +61,7 @@ struct TeamLayout {
     static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
 };
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 __global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * TeamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                    T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
@@ -223,8 +223,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             }
         }
         // ---------------- landmarks (Algorithm 1 step 1) ----------------
-        landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
-        landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
+        landmarks_mma<T, TPW, L, PW>(Qs, qbar, r * LPW, d, g, t);
+        landmarks_mma<T, TPW, L, PW>(Ks, kbar, r * LPW, d, g, t);
         if (tsync_or(failed)) break;
         // ---------------- S_L, G_L^n fragments parked in buffer b ----------------
         {
@@ -290,11 +290,11 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (pend_v) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC>
+template <typename T, int M, int NCOL, int DC, int PW>
 cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault) {
     using Lay = TeamLayout<M, NCOL>;
-    auto kern = nystra_team_kernel<T, M, NCOL, DC>;
+    auto kern = nystra_team_kernel<T, M, NCOL, DC, PW>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -319,15 +319,15 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
 
 // The common head widths get kernels with d_h as a compile-time constant
 // (constant strides and column bounds); others read it at run time.
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                      int iters, cudaStream_t stream, unsigned int* fault) {
     if constexpr (NCOL == 32) {
-        if (d == 30) return launch_team_dc<T, M, NCOL, 30>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 30) return launch_team_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {
-        if (d == 32) return launch_team_dc<T, M, NCOL, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        if (d == 32) return launch_team_dc<T, M, NCOL, 32, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     }
-    return launch_team_dc<T, M, NCOL, 0>(q, k, v, out, n_units, d, iters, stream, fault);
+    return launch_team_dc<T, M, NCOL, 0, PW>(q, k, v, out, n_units, d, iters, stream, fault);
 }
 
 }  // namespace tc

@@ -30,7 +30,8 @@ MIXES = {"uformer-mix": ("uformer-s1", "uformer-s4")}
 
 DEFAULT = (["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4", "uformer-mix"]
            + [f"large-w{w}-m{m}" for w in (16, 32) for m in (32, 64)]
-           + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")])
+           + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")]
+           + ["swinir256-bf16-patches", "sr720p-w16-m16-bf16-patches", "sr720p-w32-m16-bf16-patches"])
 
 
 def hbm_peak_gbs() -> tuple[float, str]:
@@ -79,7 +80,7 @@ def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int =
     def nystra(i):
         for wl, ss in zip(parts, sets):
             a, b, c, o = ss[i]
-            binding.nystra(a, b, c, wl.m, wl.iters, out=o)
+            binding.nystra(a, b, c, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
 
     def exact(i):
         for ss in sets:

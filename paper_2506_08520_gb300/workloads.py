@@ -35,6 +35,7 @@ class Workload:
     seed: int
     recipe: str          # "iid" | "proj" | "lowrank" | "map"
     map_hw: tuple = ()   # (H, W, window) for recipe == "map"
+    landmarks: str = "segments"  # landmark pooling: "segments" | "patches"
 
     @property
     def units(self) -> int:
@@ -82,6 +83,9 @@ for _w in (8, 16, 32):
         for _dt in ("bf16", "f16"):
             _wl = _sr_map(_w, _m, _dt)
             WORKLOADS[_wl.name] = _wl
+# The same inputs with square-patch landmarks (4 x 4 patches).
+for _name in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16"):
+    WORKLOADS[_name + "-patches"] = WORKLOADS[_name].with_(name=_name + "-patches", landmarks="patches")
 
 
 def _cast(x: np.ndarray, dtype: str) -> torch.Tensor:

@@ -18,9 +18,9 @@ def per_unit_rel(out: np.ndarray, ref: np.ndarray) -> np.ndarray:
     return np.linalg.norm(o - r, axis=1) / np.linalg.norm(r, axis=1)
 
 
-def gpu_nystra(q, k, v, m, iters):
+def gpu_nystra(q, k, v, m, iters, landmarks="segments"):
     qd, kd, vd = (x.cuda() for x in (q, k, v))
-    out = binding.nystra(qd, kd, vd, m=m, iters=iters)
+    out = binding.nystra(qd, kd, vd, m=m, iters=iters, landmarks=landmarks)
     torch.cuda.synchronize()
     return out
 
@@ -46,12 +46,12 @@ def sample_units(n_units: int, k: int = 384, seed: int = 0) -> np.ndarray:
     return np.unique(idx)
 
 
-def check_nystra(q, k, v, m, iters, sample=None):
+def check_nystra(q, k, v, m, iters, sample=None, landmarks="segments"):
     """Run GPU on everything, the oracle on the sampled units; return (max err, worst unit)."""
-    out = units_view(gpu_nystra(q, k, v, m, iters).cpu())
+    out = units_view(gpu_nystra(q, k, v, m, iters, landmarks).cpu())
     qu, ku, vu = units_view(q), units_view(k), units_view(v)
     idx = np.arange(qu.shape[0]) if sample is None else sample
-    ref = oracle.nystra_attention(qu[idx], ku[idx], vu[idx], m, iters)
+    ref = oracle.nystra_attention(qu[idx], ku[idx], vu[idx], m, iters, landmarks)
     got = out[idx].double().numpy()
     assert np.isfinite(got).all(), "non-finite GPU output"
     err = per_unit_rel(got, ref)

@@ -28,7 +28,8 @@ def test_header_declares_the_boundary():
     names = declared_symbols()
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
                      "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
-                     "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size"):
+                     "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size",
+                     "nystra_attention_ex"):
         assert required in names
 
 
@@ -126,10 +127,27 @@ def test_debug_stages_size_rejects_other_shapes(lib, N, d, m):
     (dict(unit=-1), nb.NYSTRA_EINVAL),
     (dict(dump=0), nb.NYSTRA_EINVAL),
     (dict(dump=5 * P + 4), nb.NYSTRA_EINVAL),  # misaligned
+    (dict(lm=2), nb.NYSTRA_EINVAL),           # no such pooling
+    (dict(lm=1, m=8), nb.NYSTRA_EINVAL),      # 8 landmarks are no square grid
+    (dict(lm=1, dtype=0), nb.NYSTRA_EINVAL),  # patches: 16-bit I/O only here
 ])
 def test_debug_stages_argument_validation(lib, args, code):
     a = dict(N=64, d=30, m=16, iters=6, dtype=1, unit=0, dump=5 * P)
     a.update(args)
-    rc = nb.nystra_debug_stages(P, 2 * P, 3 * P, 4, 2, a["N"], a["d"], a["m"], a["iters"], a["dtype"],
-                                a["unit"], a["dump"], None)
+    rc = nb.nystra_debug_stages(P, 2 * P, 3 * P, 4, 2, a["N"], a["d"], a["m"], a["iters"], a.get("lm", 0),
+                                a["dtype"], a["unit"], a["dump"], None)
+    assert rc == code
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(N=64, m=16, lm=2), nb.NYSTRA_EINVAL),     # no such pooling
+    (dict(N=64, m=8, lm=1), nb.NYSTRA_EINVAL),      # m not a square
+    (dict(N=128, m=16, lm=1), nb.NYSTRA_EINVAL),    # N not a square
+    (dict(N=256, m=36, lm=1), nb.NYSTRA_EINVAL),    # 6 patches do not tile 16 columns (36 does not divide 256 either)
+    (dict(N=64, m=16, lm=1, nw=0), nb.NYSTRA_OK),   # empty: no-op
+    (dict(N=64, m=16, lm=0, nw=0), nb.NYSTRA_OK),
+])
+def test_nystra_ex_argument_validation(lib, args, code):
+    rc = nb.nystra_attention_ex(P, 2 * P, 3 * P, 64 * P, args.get("nw", 4), 2, args["N"], 30, args["m"], 6,
+                                args["lm"], 1, None)
     assert rc == code

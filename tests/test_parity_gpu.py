@@ -105,6 +105,50 @@ def test_nystra_workloads(name):
     assert err <= TOL[wl.dtype], f"{name}: max rel err {err:.3e} at unit {worst}"
 
 
+# Square-patch landmarks: the tensor-core kernels (16-bit I/O, m = 16) and the
+# SIMT path (every other square grid, fp32 I/O).
+PATCHES = [
+    # units, N, d, m
+    (7, 64, 30, 16),
+    (3, 64, 32, 16),
+    (5, 256, 30, 16),
+    (3, 256, 32, 16),
+    (2, 1024, 30, 16),
+    (2, 1024, 32, 16),
+    (3, 64, 30, 4),      # SIMT from here on
+    (3, 64, 30, 64),     # 1x1 patches
+    (3, 256, 30, 64),
+    (2, 1024, 30, 64),
+    (4, 16, 8, 4),
+    (3, 144, 12, 16),    # 12x12 window, 3x3 patches
+]
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
+@pytest.mark.parametrize("units,N,d,m", PATCHES)
+def test_nystra_patches_small(units, N, d, m, dtype):
+    q, k, v = workloads.random_qkv(units, N, d, dtype, seed=units * 77 + N + d + m)
+    err, worst = check_nystra(q, k, v, m, 6, landmarks="patches")
+    assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("name", ["swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-f16"])
+def test_nystra_patches_workloads(name):
+    wl = workloads.WORKLOADS[name]
+    q, k, v = workloads.make_qkv(wl)
+    err, worst = check_nystra(q, k, v, wl.m, wl.iters, sample_units(wl.units, 192), landmarks="patches")
+    print(f"{name} (patches): max rel err {err:.3e} (unit {worst})")
+    assert err <= TOL[wl.dtype], f"{name}: max rel err {err:.3e} at unit {worst}"
+
+
+def test_patches_differ_from_segments():
+    # the two readings give different landmarks, hence different outputs
+    q, k, v = (x.cuda() for x in workloads.random_qkv(4, 256, 30, "bf16", seed=3))
+    a = binding.nystra(q, k, v, 16, 6)
+    b = binding.nystra(q, k, v, 16, 6, landmarks="patches")
+    assert (a.float() - b.float()).abs().max().item() > 1e-2
+
+
 @pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
 @pytest.mark.parametrize("units,N,d", [(7, 64, 30), (3, 256, 32), (2, 1024, 32), (4, 48, 20), (3, 10, 64)])
 def test_exact_small(units, N, d, dtype):

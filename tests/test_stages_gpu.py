@@ -29,9 +29,9 @@ def _built():
     build.build()
 
 
-def _stages(q, k, v, m, iters, unit):
+def _stages(q, k, v, m, iters, unit, landmarks="segments"):
     qd, kd, vd = (x.cuda() for x in (q, k, v))
-    st = binding.debug_stages(qd, kd, vd, m, iters, unit)
+    st = binding.debug_stages(qd, kd, vd, m, iters, unit, landmarks=landmarks)
     return {n: x.double().numpy() for n, x in st.items()}
 
 
@@ -74,6 +74,38 @@ def test_landmarks_of_integer_tokens_equal_the_oracle_exactly(dtype):
             ref = oracle.landmarks(_unit(x, u), m)
             assert np.array_equal(st["qbar"], ref)
             assert np.array_equal(st["kbar"], ref)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f16"])
+@pytest.mark.parametrize("d", [30, 32, 8])
+def test_patch_indexing_is_bit_exact(dtype, d):
+    # Token (r, s) of the 8x8 window carries 8r + s + c in column c: the mean
+    # of 2x2 patch (pr, pc) is 8 (2 pr + 1/2) + 2 pc + 1/2 + c, exact in both
+    # 16-bit types (at most 89.5 = 179/2).
+    N = 64
+    x = (torch.arange(N, dtype=torch.float64)[:, None] + torch.arange(d, dtype=torch.float64)[None, :])
+    x = x.to(TORCH[dtype]).reshape(1, 1, N, d).contiguous()
+    st = _stages(x, x, x, 16, 6, 0, landmarks="patches")
+    j = np.arange(16)[:, None]
+    want = 8 * (2 * (j // 4) + 0.5) + 2 * (j % 4) + 0.5 + np.arange(d)[None, :]
+    assert np.array_equal(st["qbar"], want)
+    assert np.array_equal(st["kbar"], want)
+    g = torch.Generator().manual_seed(18)
+    xi = torch.randint(-8, 9, (2, 3, 64, d), generator=g).to(TORCH[dtype])
+    for u in (0, 4):
+        st = _stages(xi, xi, xi, 16, 6, u, landmarks="patches")
+        assert np.array_equal(st["qbar"], oracle.landmarks(_unit(xi, u), 16, "patches"))
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f16"])
+def test_patch_stage_dump_matches_the_product_kernel(dtype):
+    q, k, v = workloads.random_qkv(3, 64, 30, dtype, seed=21)
+    full = binding.nystra(q.cuda(), k.cuda(), v.cuda(), 16, 6, landmarks="patches").cpu()
+    for u in range(3):
+        st = _stages(q, k, v, 16, 6, u, landmarks="patches")
+        assert np.array_equal(_unit(full, u), st["out"])
+        ref = oracle.nystra_stages(_unit(q, u), _unit(k, u), _unit(v, u), 16, 6, "patches")
+        assert _relf(st["out"], ref["out"]) <= TOL[dtype]
 
 
 # ------------------------------------------------------------ steps 2-7
