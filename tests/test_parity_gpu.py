@@ -201,3 +201,23 @@ def test_fp16_large_values_keep_range():
     v = (v.float() * 400.0).half()
     err, worst = check_nystra(q, k, v, 16, 6)
     assert err <= TOL["f16"], f"max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("N,d,m", [(64, 30, 16), (256, 30, 16), (1024, 30, 16), (64, 30, 32), (256, 30, 32),
+                                   (1024, 32, 32), (256, 32, 64), (48, 20, 12)])
+def test_inputs_may_alias(N, d, m):
+    # the header allows q, k and v to be the same buffer (self-attention on one tensor)
+    q, _, _ = workloads.random_qkv(3, N, d, "bf16", seed=N + m)
+    x = q.cuda()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        a = binding.nystra(x, x, x, m, 6, stream=s)
+        b = binding.nystra(x.clone(), x.clone(), x.clone(), m, 6, stream=s)
+        if N <= 256:
+            ea = binding.exact(x, x, x, stream=s)
+            eb = binding.exact(x.clone(), x.clone(), x.clone(), stream=s)
+    s.synchronize()
+    assert torch.equal(a, b)
+    if N <= 256:
+        assert torch.equal(ea, eb)
