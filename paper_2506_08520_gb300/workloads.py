@@ -62,7 +62,7 @@ def _sr_map(window: int, m: int, dtype: str) -> Workload:
                     "map", (H, W, window))
 
 
-# Five workload families (sizes as in the paper's models).
+# Five workload families, sized like the paper's models (SwinIR, Uformer, Dehazeformer windows).
 WORKLOADS = {
     # SwinIR-like 64x64 feature map, 8x8 windows: 64 windows, 6 heads, d_h = 30.
     "tiny": Workload("tiny", 64, 6, 64, 30, 16, 6, "f32", 0, "iid"),
