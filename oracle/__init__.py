@@ -31,6 +31,13 @@ def _load():
         lib.oracle_threads.restype = ctypes.c_int
         lib.oracle_exact_attention.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int, ctypes.c_int]
         lib.oracle_exact_attention.restype = None
+        lib.oracle_exact_attention_bias.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int, ctypes.c_int, _D]
+        lib.oracle_exact_attention_bias.restype = None
+        lib.oracle_nystra_attention_bias.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int, ctypes.c_int,
+                                                     ctypes.c_int, ctypes.c_int, ctypes.c_int, _D]
+        lib.oracle_nystra_attention_bias.restype = ctypes.c_int
+        lib.oracle_pool_bias.argtypes = [_D, ctypes.c_int, ctypes.c_int, ctypes.c_int, _D, _D, _D]
+        lib.oracle_pool_bias.restype = None
         lib.oracle_nystra_attention.argtypes = [_D, _D, _D, _D, ctypes.c_long, ctypes.c_int,
                                                 ctypes.c_int, ctypes.c_int, ctypes.c_int]
         lib.oracle_nystra_attention.restype = ctypes.c_int
@@ -65,28 +72,44 @@ def threads() -> int:
     return int(_load().oracle_threads())
 
 
-def exact_attention(q, k, v) -> np.ndarray:
-    """Exact softmax attention, Eq. (1), per unit; float64 ``[..., N, d]``."""
+def _bias(bias, q):
+    """An additive score bias ``[..., N, N]`` broadcast over the units of q."""
+    N = q.shape[-2]
+    b = np.broadcast_to(_f64(bias), q.shape[:-2] + (N, N))
+    return np.ascontiguousarray(b)
+
+
+def exact_attention(q, k, v, bias=None) -> np.ndarray:
+    """Exact softmax attention, Eq. (1), per unit; float64 ``[..., N, d]``.
+    ``bias``: optional additive score bias ``[..., N, N]`` (before the softmax)."""
     q, k, v = _f64(q), _f64(k), _f64(v)
     N, d = q.shape[-2], q.shape[-1]
     out = np.empty_like(q)
-    _load().oracle_exact_attention(_p(q), _p(k), _p(v), _p(out), q.size // (N * d), N, d)
+    if bias is None:
+        _load().oracle_exact_attention(_p(q), _p(k), _p(v), _p(out), q.size // (N * d), N, d)
+    else:
+        b = _bias(bias, q)
+        _load().oracle_exact_attention_bias(_p(q), _p(k), _p(v), _p(out), q.size // (N * d), N, d, _p(b))
     return out
 
 
 POOLS = {"segments": 0, "patches": 1}
 
 
-def nystra_attention(q, k, v, m: int, iters: int, pool: str = "segments") -> np.ndarray:
+def nystra_attention(q, k, v, m: int, iters: int, pool: str = "segments", bias=None) -> np.ndarray:
     """PnP-Nystra output (Algorithm 1, stabilised form), float64 ``[..., N, d]``.
 
     ``pool``: "segments" (m contiguous token runs) or "patches" (a square
-    window pooled over a square grid of m square patches)."""
+    window pooled over a square grid of m square patches).  ``bias``: optional
+    additive score bias ``[..., N, N]``, seen by the landmark blocks as the mean
+    over each landmark's tokens."""
     q, k, v = _f64(q), _f64(k), _f64(v)
     N, d = q.shape[-2], q.shape[-1]
     out = np.empty_like(q)
-    rc = _load().oracle_nystra_attention_pool(_p(q), _p(k), _p(v), _p(out), q.size // (N * d),
-                                              N, d, int(m), int(iters), POOLS[pool])
+    b = None if bias is None else _bias(bias, q)
+    rc = _load().oracle_nystra_attention_bias(_p(q), _p(k), _p(v), _p(out), q.size // (N * d),
+                                              N, d, int(m), int(iters), POOLS[pool],
+                                              None if b is None else _p(b))
     if rc != 0:
         raise ValueError(f"oracle: invalid m={m} for N={N} with {pool} pooling, iters={iters}")
     return out
@@ -106,6 +129,16 @@ def landmarks(x, m: int, pool: str = "segments") -> np.ndarray:
     else:
         _load().oracle_landmarks(_p(x), N, d, int(m), _p(out))
     return out
+
+
+def pool_bias(B, m: int, pool: str = "segments"):
+    """One unit's score bias ``[N, N]`` through the landmarks: (B_L ``[N, m]``,
+    B_U ``[m, N]``, B_A ``[m, m]``), each entry the mean over the landmarks' tokens."""
+    B = _f64(B)
+    N = B.shape[0]
+    BL, BU, BA = np.empty((N, m)), np.empty((m, N)), np.empty((m, m))
+    _load().oracle_pool_bias(_p(B), N, int(m), POOLS[pool], _p(BL), _p(BU), _p(BA))
+    return BL, BU, BA
 
 
 def pinv_iteration(A, iters: int) -> np.ndarray:

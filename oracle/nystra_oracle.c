@@ -26,7 +26,12 @@
  *       Z_{k+1} = 1/4 Z_k (13 I - A Z_k (15 I - A Z_k (7 I - A Z_k)))
  *     started from Z_0 = A^T / (||A||_1 ||A||_inf) and run for `iters`
  *     steps, applied to the normalised core block A = G_A^n (Sec. 2.2);
- *   - no guard on the denominator (Alg. 1 step 7 divides as written).
+ *   - no guard on the denominator (Alg. 1 step 7 divides as written);
+ *   - an additive score bias B (N x N, the relative-position bias and masks
+ *     of window attention; Eq. 1 has none) enters every block the way the
+ *     landmarks enter it: a landmark stands for the mean of its tokens, so
+ *     S_L[i][j] += mean_{t in j} B[i][t], S_U[j][t] += mean_{s in j} B[s][t]
+ *     and S_A[i][j] += mean_{s in i, t in j} B[s][t].
  *
  * Parallelism: units are spread over OpenMP threads; each unit is computed
  * sequentially, so the result does not depend on the thread count.
@@ -67,14 +72,14 @@ static void matmul(const double* A, const double* B, double* C, int r, int n, in
 /* the shift cancels in the row normalisation (Eq. 2).                 */
 /* ------------------------------------------------------------------ */
 static void exact_unit(const double* q, const double* k, const double* v, double* o,
-                       int N, int d, double* row) {
+                       int N, int d, const double* B, double* row) {
     const double s = 1.0 / sqrt((double)d);
     for (int i = 0; i < N; ++i) {
         double mx = -INFINITY;
         for (int j = 0; j < N; ++j) {
             double a = 0.0;
             for (int c = 0; c < d; ++c) a += q[(size_t)i * d + c] * k[(size_t)j * d + c];
-            row[j] = s * a;
+            row[j] = s * a + (B ? B[(size_t)i * N + j] : 0.0);
             if (row[j] > mx) mx = row[j];
         }
         double den = 0.0;
@@ -90,17 +95,25 @@ static void exact_unit(const double* q, const double* k, const double* v, double
     }
 }
 
-void oracle_exact_attention(const double* q, const double* k, const double* v, double* out,
-                            long n_units, int N, int d) {
+/* Exact attention of every unit; bias (NULL or N x N per unit) is added to
+ * the scaled scores before the softmax. */
+void oracle_exact_attention_bias(const double* q, const double* k, const double* v, double* out,
+                                 long n_units, int N, int d, const double* bias) {
     const size_t unit = (size_t)N * d;
 #pragma omp parallel
     {
         double* row = (double*)malloc(sizeof(double) * (size_t)N);
 #pragma omp for schedule(dynamic, 4)
         for (long u = 0; u < n_units; ++u)
-            exact_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d, row);
+            exact_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d,
+                       bias ? bias + (size_t)u * N * N : 0, row);
         free(row);
     }
+}
+
+void oracle_exact_attention(const double* q, const double* k, const double* v, double* out,
+                            long n_units, int N, int d) {
+    oracle_exact_attention_bias(q, k, v, out, n_units, N, d, 0);
 }
 
 /* ------------------------------------------------------------------ */
@@ -145,6 +158,33 @@ void oracle_landmarks_patches(const double* x, int N, int d, int m, double* xbar
             for (int r = (j / p) * b; r < (j / p) * b + b; ++r)
                 for (int s = (j % p) * b; s < (j % p) * b + b; ++s) acc += x[((size_t)r * w + s) * d + c];
             xbar[(size_t)j * d + c] = acc / (double)(b * b);
+        }
+}
+
+/* Landmark of token t: its segment (pool = 0) or its square patch (pool = 1). */
+static int landmark_of(int t, int N, int m, int pool) {
+    if (pool == 0) return t / (N / m);
+    const int w = exact_sqrt(N), p = exact_sqrt(m), b = w / p;
+    return ((t / w) / b) * p + (t % w) / b;
+}
+
+/* The additive score bias B (N x N) of one unit seen through the landmarks:
+ *   BL[i][j] = mean over tokens t of landmark j of B[i][t]          (N x m)
+ *   BU[j][t] = mean over tokens s of landmark j of B[s][t]          (m x N)
+ *   BA[i][j] = mean over s of landmark i, t of landmark j of B[s][t] (m x m)
+ * Every landmark averages L = N/m tokens under either pooling. */
+void oracle_pool_bias(const double* B, int N, int m, int pool, double* BL, double* BU, double* BA) {
+    const double L = (double)(N / m);
+    memset(BL, 0, sizeof(double) * (size_t)N * m);
+    memset(BU, 0, sizeof(double) * (size_t)m * N);
+    memset(BA, 0, sizeof(double) * (size_t)m * m);
+    for (int s = 0; s < N; ++s)
+        for (int t = 0; t < N; ++t) {
+            const double b = B[(size_t)s * N + t];
+            const int js = landmark_of(s, N, m, pool), jt = landmark_of(t, N, m, pool);
+            BL[(size_t)s * m + jt] += b / L;
+            BU[(size_t)js * N + t] += b / L;
+            BA[(size_t)js * m + jt] += b / (L * L);
         }
 }
 
@@ -214,7 +254,7 @@ typedef struct {
 } stage_ptrs;
 
 static void nystra_unit(const double* q, const double* k, const double* v, double* o,
-                        int N, int d, int m, int iters, int pool, stage_ptrs st) {
+                        int N, int d, int m, int iters, int pool, const double* B, stage_ptrs st) {
     const double s = 1.0 / sqrt((double)d);
     double* qbar = (double*)malloc(sizeof(double) * (size_t)m * d);
     double* kbar = (double*)malloc(sizeof(double) * (size_t)m * d);
@@ -239,14 +279,21 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
         oracle_landmarks(k, N, d, m, kbar);
     }
 
+    /* The score bias through the landmarks (zero without a bias). */
+    double* BL = (double*)calloc((size_t)N * m, sizeof(double));
+    double* BU = (double*)calloc((size_t)m * N, sizeof(double));
+    double* BA = (double*)calloc((size_t)m * m, sizeof(double));
+    if (B) oracle_pool_bias(B, N, m, pool, BL, BU, BA);
+
     /* Steps 2-3 with row-max stabilisation.  S_L, its row max m_L. */
     for (int i = 0; i < N; ++i) {
         double mx = -INFINITY;
         for (int j = 0; j < m; ++j) {
             double a = 0.0;
             for (int c = 0; c < d; ++c) a += q[(size_t)i * d + c] * kbar[(size_t)j * d + c];
-            GL[(size_t)i * m + j] = s * a;
-            if (s * a > mx) mx = s * a;
+            const double sl = s * a + BL[(size_t)i * m + j];
+            GL[(size_t)i * m + j] = sl;
+            if (sl > mx) mx = sl;
         }
         mL[i] = mx;
     }
@@ -256,8 +303,9 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
         for (int j = 0; j < N; ++j) {
             double a = 0.0;
             for (int c = 0; c < d; ++c) a += qbar[(size_t)i * d + c] * k[(size_t)j * d + c];
-            GU[(size_t)i * N + j] = s * a;
-            if (s * a > mx) mx = s * a;
+            const double su = s * a + BU[(size_t)i * N + j];
+            GU[(size_t)i * N + j] = su;
+            if (su > mx) mx = su;
         }
         mU[i] = mx;
     }
@@ -271,7 +319,7 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
         for (int j = 0; j < m; ++j) {
             double a = 0.0;
             for (int c = 0; c < d; ++c) a += qbar[(size_t)i * d + c] * kbar[(size_t)j * d + c];
-            GA[(size_t)i * m + j] = exp(s * a - mU[i]);
+            GA[(size_t)i * m + j] = exp(s * a + BA[(size_t)i * m + j] - mU[i]);
         }
 
     /* Step 4: pseudo-inverse of G_A^n. */
@@ -305,21 +353,30 @@ static void nystra_unit(const double* q, const double* k, const double* v, doubl
     if (st.num) memcpy(st.num, num, sizeof(double) * (size_t)N * d);
     if (st.den) memcpy(st.den, den, sizeof(double) * (size_t)N);
 
+    free(BL); free(BU); free(BA);
     free(qbar); free(kbar); free(mL); free(mU); free(GL); free(GU); free(GA);
     free(Z); free(P); free(GUV); free(GU1); free(num); free(den);
 }
 
 /* Batched PnP-Nystra output with landmark pooling `pool` (0 = segments,
- * 1 = square patches).  Returns 0, or -1 for an m the pooling cannot form. */
-int oracle_nystra_attention_pool(const double* q, const double* k, const double* v, double* out,
-                                 long n_units, int N, int d, int m, int iters, int pool) {
+ * 1 = square patches) and an additive score bias (NULL, or N x N per unit).
+ * Returns 0, or -1 for an m the pooling cannot form. */
+int oracle_nystra_attention_bias(const double* q, const double* k, const double* v, double* out,
+                                 long n_units, int N, int d, int m, int iters, int pool, const double* bias) {
     if (m < 1 || m > N || !pool_valid(N, m, pool) || iters < 0) return -1;
     const size_t unit = (size_t)N * d;
     const stage_ptrs none = {0};
 #pragma omp parallel for schedule(dynamic, 4)
     for (long u = 0; u < n_units; ++u)
-        nystra_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d, m, iters, pool, none);
+        nystra_unit(q + u * unit, k + u * unit, v + u * unit, out + u * unit, N, d, m, iters, pool,
+                    bias ? bias + (size_t)u * N * N : 0, none);
     return 0;
+}
+
+/* Without a bias. */
+int oracle_nystra_attention_pool(const double* q, const double* k, const double* v, double* out,
+                                 long n_units, int N, int d, int m, int iters, int pool) {
+    return oracle_nystra_attention_bias(q, k, v, out, n_units, N, d, m, iters, pool, 0);
 }
 
 /* Batched PnP-Nystra output, segment landmarks.  -1 if m does not divide N. */
@@ -336,6 +393,6 @@ int oracle_nystra_stages(const double* q, const double* k, const double* v, doub
                          double* num, double* den) {
     if (m < 1 || m > N || !pool_valid(N, m, pool) || iters < 0) return -1;
     stage_ptrs st = {qbar, kbar, mL, mU, GLn, GUn, GAn, Z, num, den};
-    nystra_unit(q, k, v, out, N, d, m, iters, pool, st);
+    nystra_unit(q, k, v, out, N, d, m, iters, pool, 0, st);
     return 0;
 }

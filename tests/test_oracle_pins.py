@@ -408,3 +408,90 @@ def test_patch_shapes_that_do_not_tile_are_rejected(N, m):
     x = np.zeros((1, N, 4))
     with pytest.raises(ValueError):
         oracle.nystra_attention(x, x, x, m, 6, "patches")
+
+
+# --------------------------------------------------------------------------
+# An additive score bias (window attention's relative-position bias and
+# masks): each landmark block sees the mean bias over its landmarks' tokens.
+# --------------------------------------------------------------------------
+def test_exact_attention_with_bias_bruteforce():
+    rng = _rng(51)
+    N, d = 6, 3
+    q, k, v = (rng.standard_normal((N, d)) for _ in range(3))
+    B = rng.standard_normal((N, N))
+    ref = np.empty((N, d))
+    for i in range(N):
+        w = [math.exp(sum(q[i, c] * k[j, c] for c in range(d)) / math.sqrt(d) + B[i, j]) for j in range(N)]
+        for c in range(d):
+            ref[i, c] = sum(w[j] * v[j, c] for j in range(N)) / sum(w)
+    np.testing.assert_allclose(oracle.exact_attention(q[None], k[None], v[None], B)[0], ref, rtol=1e-12)
+
+
+def _landmark_ids(N, m, pool):
+    if pool == "segments":
+        return np.arange(N) // (N // m)
+    w, p = int(round(N ** 0.5)), int(round(m ** 0.5))
+    b = w // p
+    r, c = np.divmod(np.arange(N), w)
+    return (r // b) * p + c // b
+
+
+@pytest.mark.parametrize("pool,N,m", [("segments", 64, 16), ("segments", 32, 4), ("patches", 64, 16),
+                                      ("patches", 256, 16), ("patches", 64, 4)])
+def test_pool_bias_is_the_mean_over_landmark_tokens(pool, N, m):
+    rng = _rng(52 + N + m)
+    B = rng.standard_normal((N, N))
+    BL, BU, BA = oracle.pool_bias(B, m, pool)
+    ids = _landmark_ids(N, m, pool)
+    for j in range(m):
+        np.testing.assert_allclose(BL[:, j], B[:, ids == j].mean(axis=1), rtol=1e-12, atol=1e-14)
+        np.testing.assert_allclose(BU[j], B[ids == j].mean(axis=0), rtol=1e-12, atol=1e-14)
+        for i in range(m):
+            np.testing.assert_allclose(BA[i, j], B[np.ix_(ids == i, ids == j)].mean(), rtol=1e-12, atol=1e-14)
+
+
+def test_zero_bias_changes_nothing():
+    rng = _rng(53)
+    q, k, v = (rng.standard_normal((2, 64, 8)) for _ in range(3))
+    for pool in ("segments", "patches"):
+        np.testing.assert_array_equal(oracle.nystra_attention(q, k, v, 16, 6, pool, np.zeros((64, 64))),
+                                      oracle.nystra_attention(q, k, v, 16, 6, pool))
+
+
+def test_row_constant_bias_cancels():
+    """B[i][t] = c_i shifts whole rows of S_L, S_U and S_A with their maxima: G^n is unchanged."""
+    rng = _rng(54)
+    N, d = 64, 8
+    q, k, v = (rng.standard_normal((2, N, d)) for _ in range(3))
+    B = np.repeat(3.0 * rng.standard_normal((N, 1)), N, axis=1)
+    for pool in ("segments", "patches"):
+        np.testing.assert_allclose(oracle.nystra_attention(q, k, v, 16, 6, pool, B),
+                                   oracle.nystra_attention(q, k, v, 16, 6, pool), rtol=1e-10, atol=1e-12)
+    np.testing.assert_allclose(oracle.exact_attention(q, k, v, B), oracle.exact_attention(q, k, v),
+                               rtol=1e-10, atol=1e-12)
+
+
+def test_bias_with_every_token_a_landmark_is_exact_biased_attention():
+    rng = _rng(55)
+    U, N, d = 2, 16, 6
+    q, k, v = (0.5 * rng.standard_normal((U, N, d)) for _ in range(3))
+    B = 0.5 * rng.standard_normal((U, N, N))
+    ref = oracle.exact_attention(q, k, v, B)
+    assert _rel(oracle.nystra_attention(q, k, v, N, 80, "segments", B), ref) < 1e-8
+    assert _rel(oracle.nystra_attention(q, k, v, N, 80, "patches", B), ref) < 1e-8
+
+
+def test_block_constant_bias_exact_recovery():
+    """Tokens constant per segment and a bias constant per pair of segments keep
+    rank(G~) = m, so a converged inverse recovers exact biased attention."""
+    rng = _rng(56)
+    N, d, m = 64, 8, 8
+    L = N // m
+    q = np.repeat(rng.standard_normal((m, d)), L, axis=0)
+    k = np.repeat(rng.standard_normal((m, d)), L, axis=0)
+    v = rng.standard_normal((N, d))
+    B = np.kron(rng.standard_normal((m, m)), np.ones((L, L)))
+    ref = oracle.exact_attention(q[None], k[None], v[None], B)
+    assert _rel(oracle.nystra_attention(q[None], k[None], v[None], m, 80, "segments", B), ref) < 1e-8
+    # the bias matters: dropping it moves the output
+    assert _rel(oracle.nystra_attention(q[None], k[None], v[None], m, 80), ref) > 1e-3
