@@ -125,6 +125,43 @@ NYSTRA_API int nystra_attention_ex(const void* q, const void* k, const void* v, 
                                    int landmarks, int dtype, void* stream);
 
 /*
+ * Additive score bias (window attention's relative-position bias and masks).
+ * Eq. (1) has none; a window-attention layer adds B (N x N per head, or per
+ * window and head) to Q K^T / sqrt(d_h) before the softmax.  Here a landmark
+ * stands for the mean of its tokens, so it also carries the mean of their
+ * biases: the blocks of Sec. 2.2 become
+ *   S_L[i][j] += mean_{t in j} B[i][t],   S_U[j][t] += mean_{s in j} B[s][t],
+ *   S_A[i][j] += mean_{s in i, t in j} B[s][t]
+ * (with m = N and a converged inverse this is exact biased attention).  Use
+ * finite mask values (e.g. -100): an infinite one poisons every landmark whose
+ * tokens it touches.
+ *
+ * nystra_pool_bias -- the three landmark blocks of n_bias biases:
+ *   bias    [n_bias, N, N] fp32 (device, caller-owned);
+ *   bias_L  [n_bias, N, m], bias_U [n_bias, m, N], bias_A [n_bias, m, m] fp32
+ *           outputs (device, caller-owned, no overlap with each other or bias).
+ * `landmarks` as for nystra_attention_ex.  All pointers 16-byte aligned.  Meant
+ * to run once per model constant.  Returns NYSTRA_OK, NYSTRA_EINVAL (shape,
+ * pointer, alignment or overlap) or NYSTRA_ELAUNCH.
+ */
+NYSTRA_API int nystra_pool_bias(const float* bias, int n_bias, int N, int m, int landmarks, float* bias_L,
+                                float* bias_U, float* bias_A, void* stream);
+
+/*
+ * nystra_attention_bias -- nystra_attention_ex with a pooled score bias.
+ * bias_L/U/A as written by nystra_pool_bias for bias_windows * heads slices:
+ * bias_windows = 1 (one bias per head, shared by every window: the
+ * relative-position bias) or n_windows (per window and head: masks of
+ * shifted windows).  Unit (w, h) uses slice h, or w * heads + h.  The blocks
+ * must not overlap out.  Runs on the fp32 SIMT path.  Other arguments and
+ * return codes as nystra_attention_ex.
+ */
+NYSTRA_API int nystra_attention_bias(const void* q, const void* k, const void* v, void* out, int n_windows,
+                                     int heads, int N, int d_h, int m, int iters, int landmarks,
+                                     const float* bias_L, const float* bias_U, const float* bias_A,
+                                     int bias_windows, int dtype, void* stream);
+
+/*
  * exact_window_attention -- exact softmax attention per unit, Eq. (1):
  * O = softmax(Q K^T / sqrt(d_h)) V with row-max-shifted exponentials
  * (Eq. 2).  This is the computation PnP-Nystra replaces; it serves as the

@@ -60,6 +60,10 @@ def lib() -> ctypes.CDLL:
         L.nystra_debug_stages.argtypes = [vp, vp, vp, i, i, i, i, i, i, i, i, ctypes.c_longlong, vp, vp]
         L.nystra_attention_ex.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, i, vp]
         L.nystra_attention_ex.restype = i
+        L.nystra_pool_bias.argtypes = [vp, i, i, i, i, vp, vp, vp, vp]
+        L.nystra_pool_bias.restype = i
+        L.nystra_attention_bias.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i, vp]
+        L.nystra_attention_bias.restype = i
         L.nystra_debug_stages.restype = i
         L.nystra_debug_stages_size.argtypes = [i, i, i]
         L.nystra_debug_stages_size.restype = ctypes.c_longlong
@@ -76,6 +80,16 @@ def nystra_attention(q, k, v, out, n_windows, heads, N, d_h, m, iters, dtype, st
 def nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream) -> int:
     """Raw C-ABI call with a landmark pooling (NYSTRA_LANDMARKS_*)."""
     return lib().nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream)
+
+
+def nystra_pool_bias(bias, n_bias, N, m, landmarks, bias_L, bias_U, bias_A, stream) -> int:
+    return lib().nystra_pool_bias(bias, n_bias, N, m, landmarks, bias_L, bias_U, bias_A, stream)
+
+
+def nystra_attention_bias(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L, bias_U, bias_A,
+                          bias_windows, dtype, stream) -> int:
+    return lib().nystra_attention_bias(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L, bias_U,
+                                       bias_A, bias_windows, dtype, stream)
 
 
 def exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream) -> int:
@@ -209,4 +223,40 @@ def debug_stages(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int, iter
             n *= x
         out[name] = host[pos:pos + n].reshape(shape)
         pos += n
+    return out
+
+
+def pool_bias(bias: torch.Tensor, m: int, landmarks: str = "segments", stream=None):
+    """Landmark blocks (B_L, B_U, B_A) of an fp32 device bias ``[..., N, N]``."""
+    if not bias.is_cuda or bias.dtype != torch.float32 or not bias.is_contiguous():
+        raise ValueError("bias must be a contiguous fp32 CUDA tensor")
+    N = bias.shape[-1]
+    lead = bias.shape[:-2]
+    n = bias.numel() // (N * N)
+    bL = torch.empty(lead + (N, m), dtype=torch.float32, device=bias.device)
+    bU = torch.empty(lead + (m, N), dtype=torch.float32, device=bias.device)
+    bA = torch.empty(lead + (m, m), dtype=torch.float32, device=bias.device)
+    with torch.cuda.device(bias.device):
+        rc = nystra_pool_bias(bias.data_ptr(), n, N, m, LANDMARKS[landmarks], bL.data_ptr(), bU.data_ptr(),
+                              bA.data_ptr(), _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_pool_bias")
+    return bL, bU, bA
+
+
+def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: int = 16, iters: int = 6,
+                  out: torch.Tensor | None = None, stream=None, landmarks: str = "segments") -> torch.Tensor:
+    """PnP-Nystra with a score bias already pooled by ``pool_bias``: blocks of
+    shape ``[heads, ...]`` (shared by all windows) or ``[n_windows, heads, ...]``."""
+    out = torch.empty_like(q) if out is None else out
+    _check(q, k, v, out)
+    nw, h, N, d = _geometry(q)
+    bL, bU, bA = pooled
+    bw = bL.numel() // (h * N * m)
+    with torch.cuda.device(q.device):
+        rc = nystra_attention_bias(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d, m, iters,
+                                   LANDMARKS[landmarks], bL.data_ptr(), bU.data_ptr(), bA.data_ptr(), bw,
+                                   _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_attention_bias")
     return out

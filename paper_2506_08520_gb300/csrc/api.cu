@@ -21,6 +21,12 @@ bool overlaps(const void* a, const void* b, size_t bytes) {
     return x < y + bytes && y < x + bytes;
 }
 
+// [a, a + na) and [b, b + nb) intersect.
+bool overlaps2(const void* a, size_t na, const void* b, size_t nb) {
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return x < y + nb && y < x + na;
+}
+
 size_t elem_size(int dtype) { return dtype == NYSTRA_F32 ? 4 : 2; }
 
 // Shared checks of both entry points.  Returns NYSTRA_OK or an error code.
@@ -48,8 +54,13 @@ int exact_sqrt(int n) {
 
 extern "C" {
 
-int nystra_attention_ex(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
-                        int N, int d_h, int m, int iters, int landmarks, int dtype, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// The body of every PnP-Nystra entry point; bias.L == nullptr: no bias.
+int nystra_call(const void* q, const void* k, const void* v, void* out, int n_windows, int heads, int N,
+                int d_h, int m, int iters, int landmarks, int dtype, void* stream, const nystra::NystraBias& bias) {
     int rc = check_common(q, k, v, out, n_windows, heads, N, d_h, dtype);
     if (rc != NYSTRA_OK) return rc;
     if (m < 1 || m > N || m > NYSTRA_MAX_M || N % m != 0) return NYSTRA_EINVAL;
@@ -70,7 +81,7 @@ int nystra_attention_ex(const void* q, const void* k, const void* v, void* out, 
     const bool io16 = dtype == NYSTRA_BF16 || dtype == NYSTRA_F16;
     const bool tc16 = io16 && (patches ? m == 16 : (m == 8 || m == 16 || m == 32 || m == 64));
     const bool tc32 = !patches && dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
-    const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32;
+    const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32 && bias.L == nullptr;
     const int pool = patches ? 1 : 0;
     cudaError_t e;
     if (tc && N == 64)
@@ -80,8 +91,62 @@ int nystra_attention_ex(const void* q, const void* k, const void* v, void* out, 
     else if (tc && N == 1024)
         e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
     else
-        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, pool, dtype, s);
+        e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, pool, dtype, s, bias);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
+}  // namespace
+
+extern "C" {
+
+int nystra_attention_ex(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                        int N, int d_h, int m, int iters, int landmarks, int dtype, void* stream) {
+    return nystra_call(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream, {});
+}
+
+int nystra_pool_bias(const float* bias, int n_bias, int N, int m, int landmarks, float* bias_L, float* bias_U,
+                     float* bias_A, void* stream) {
+    if (n_bias < 0 || N < 1 || N > NYSTRA_MAX_N || m < 1 || m > N || m > NYSTRA_MAX_M || N % m != 0)
+        return NYSTRA_EINVAL;
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
+    if (landmarks == NYSTRA_LANDMARKS_PATCHES) {
+        const int w = exact_sqrt(N), p = exact_sqrt(m);
+        if (w < 0 || p < 0 || w % p != 0) return NYSTRA_EINVAL;
+    }
+    if (n_bias == 0) return NYSTRA_OK;
+    if (!bias || !bias_L || !bias_U || !bias_A) return NYSTRA_EINVAL;
+    if (!aligned16(bias) || !aligned16(bias_L) || !aligned16(bias_U) || !aligned16(bias_A)) return NYSTRA_EINVAL;
+    const size_t in = (size_t)n_bias * N * N * 4, nm = (size_t)n_bias * N * m * 4, mm = (size_t)n_bias * m * m * 4;
+    if (overlaps2(bias, in, bias_L, nm) || overlaps2(bias, in, bias_U, nm) || overlaps2(bias, in, bias_A, mm) ||
+        overlaps2(bias_L, nm, bias_U, nm) || overlaps2(bias_L, nm, bias_A, mm) || overlaps2(bias_U, nm, bias_A, mm))
+        return NYSTRA_EINVAL;
+    const cudaError_t e = nystra_host::launch_pool_bias(bias, n_bias, N, m, landmarks, bias_L, bias_U, bias_A,
+                                                        (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
+int nystra_attention_bias(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,
+                          int N, int d_h, int m, int iters, int landmarks, const float* bias_L, const float* bias_U,
+                          const float* bias_A, int bias_windows, int dtype, void* stream) {
+    if (n_windows > 0 && heads > 0) {
+        if (bias_windows != 1 && bias_windows != n_windows) return NYSTRA_EINVAL;
+        if (!bias_L || !bias_U || !bias_A) return NYSTRA_EINVAL;
+        if (!aligned16(bias_L) || !aligned16(bias_U) || !aligned16(bias_A)) return NYSTRA_EINVAL;
+        if (N >= 1 && m >= 1) {
+            const size_t es = dtype == NYSTRA_F32 ? 4 : 2;
+            const size_t ob = (size_t)n_windows * heads * N * d_h * es;
+            const size_t nm = (size_t)bias_windows * heads * N * m * 4, mm = (size_t)bias_windows * heads * m * m * 4;
+            if (overlaps2(out, ob, bias_L, nm) || overlaps2(out, ob, bias_U, nm) || overlaps2(out, ob, bias_A, mm))
+                return NYSTRA_EINVAL;
+        }
+    }
+    nystra::NystraBias b;
+    b.L = bias_L;
+    b.U = bias_U;
+    b.A = bias_A;
+    b.heads = heads > 0 ? heads : 1;
+    b.per_window = bias_windows != 1 ? 1 : 0;
+    return nystra_call(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, dtype, stream, b);
 }
 
 int nystra_attention(const void* q, const void* k, const void* v, void* out, int n_windows, int heads,

@@ -24,6 +24,17 @@ template <> __device__ __forceinline__ __half from_f32<__half>(float x) { return
 template <typename T> __device__ __forceinline__ float ldg_f32(const T* p) { return to_f32(p[0]); }
 template <> __device__ __forceinline__ float ldg_f32<float>(const float* p) { return __ldg(p); }
 
+// An additive score bias seen through the landmarks (null pointers: none):
+// per slice, L is N x m, U is m x N and A is m x m (fp32, row-major).  Unit
+// u = window * heads + head uses slice u (per_window) or u % heads.
+struct NystraBias {
+    const float* L = nullptr;
+    const float* U = nullptr;
+    const float* A = nullptr;
+    int heads = 1;
+    int per_window = 0;
+};
+
 }  // namespace nystra
 
 // Host-side launchers (one per kernel family), defined in their .cu files.
@@ -32,7 +43,10 @@ namespace nystra_host {
 // pool: landmark pooling, 0 = segments, 1 = square patches of a square window.
 cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, void* out,
                                   long long n_units, int N, int d, int m, int iters, int pool, int dtype,
-                                  cudaStream_t stream);
+                                  cudaStream_t stream, const nystra::NystraBias& bias = {});
+// Pools bias [n_bias, N, N] into its landmark blocks (bias.cu).
+cudaError_t launch_pool_bias(const float* bias, long long n_bias, int N, int m, int pool, float* bias_L,
+                             float* bias_U, float* bias_A, cudaStream_t stream);
 cudaError_t launch_exact_generic(const void* q, const void* k, const void* v, void* out,
                                  long long n_units, int N, int d, int dtype, cudaStream_t stream);
 // Tensor-core kernels, windows of 64 / 256 / 1024 tokens (nystra_tc_n*.cu):

@@ -48,7 +48,7 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads)
 nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                       T* __restrict__ out, long long n_units, int N, int d, int m, int iters,
-                      int pw, float scale) {
+                      int pw, float scale, NystraBias bias) {
     extern __shared__ float sm[];
     const int d1 = d + 1, L = N / m, tid = threadIdx.x;
     int pp = 0;  // patches per patch row (square-patch landmarks)
@@ -77,6 +77,11 @@ nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T*
         const T* ku = k + base;
         const T* vu = v + base;
         T* ou = out + base;
+        // score bias through the landmarks (null without one): slice of this unit
+        const long long bs = bias.per_window ? u : u % bias.heads;
+        const float* bLu = bias.L ? bias.L + (size_t)bs * N * m : nullptr;
+        const float* bUu = bias.U ? bias.U + (size_t)bs * m * N : nullptr;
+        const float* bAu = bias.A ? bias.A + (size_t)bs * m * m : nullptr;
 
         // ---- pass 1: landmarks (Algorithm 1 step 1): segments of L tokens,
         // or (pw > 0) pb x pb patches of the pw-wide window, pb^2 = L ----
@@ -115,7 +120,7 @@ nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T*
                 const int i = idx / nt, t = idx - (idx / nt) * nt;
                 float a = 0.f;
                 for (int c = 0; c < d; ++c) a = fmaf(qbar[i * d + c], cb[t * d + c], a);
-                S[i * kChunk + t] = scale * a;
+                S[i * kChunk + t] = scale * a + (bUu ? __ldg(bUu + (size_t)i * N + t0 + t) : 0.f);
             }
             __syncthreads();
             for (int i = tid; i < m; i += blockDim.x) {
@@ -148,7 +153,7 @@ nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T*
             const int i = idx / m, j = idx - (idx / m) * m;
             float a = 0.f;
             for (int c = 0; c < d; ++c) a = fmaf(qbar[i * d + c], kbar[j * d + c], a);
-            A[idx] = expf(scale * a - mU[i]);
+            A[idx] = expf(scale * a + (bAu ? __ldg(bAu + idx) : 0.f) - mU[i]);
         }
         __syncthreads();
         if (tid < 32) {
@@ -203,7 +208,7 @@ nystra_generic_kernel(const T* __restrict__ q, const T* __restrict__ k, const T*
                 const int t = idx / m, j = idx - (idx / m) * m;
                 float a = 0.f;
                 for (int c = 0; c < d; ++c) a = fmaf(cb[t * d + c], kbar[j * d + c], a);
-                S[t * m + j] = scale * a;
+                S[t * m + j] = scale * a + (bLu ? __ldg(bLu + (size_t)(t0 + t) * m + j) : 0.f);
             }
             __syncthreads();
             for (int t = tid; t < nt; t += blockDim.x) {
@@ -243,7 +248,7 @@ size_t generic_smem_bytes(int d, int m) {
 
 template <typename T>
 cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, long long n_units, int N,
-                     int d, int m, int iters, int pool, cudaStream_t stream) {
+                     int d, int m, int iters, int pool, const NystraBias& bias, cudaStream_t stream) {
     int pw = 0;  // window width for square patches
     if (pool != 0)
         while ((pw + 1) * (pw + 1) <= N) ++pw;
@@ -253,7 +258,8 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
     if (e != cudaSuccess) return e;
     const long long grid = n_units < (1LL << 30) ? n_units : (1LL << 30);
     nystra_generic_kernel<T><<<(unsigned)grid, kThreads, smem, stream>>>(
-        (const T*)q, (const T*)k, (const T*)v, (T*)out, n_units, N, d, m, iters, pw, 1.0f / sqrtf((float)d));
+        (const T*)q, (const T*)k, (const T*)v, (T*)out, n_units, N, d, m, iters, pw, 1.0f / sqrtf((float)d),
+        bias);
     return cudaGetLastError();
 }
 
@@ -263,12 +269,12 @@ cudaError_t launch_t(const void* q, const void* k, const void* v, void* out, lon
 namespace nystra_host {
 cudaError_t launch_nystra_generic(const void* q, const void* k, const void* v, void* out,
                                   long long n_units, int N, int d, int m, int iters, int pool, int dtype,
-                                  cudaStream_t stream) {
+                                  cudaStream_t stream, const nystra::NystraBias& bias) {
     using namespace nystra;
     switch (dtype) {
-        case 0: return launch_t<float>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
-        case 1: return launch_t<__nv_bfloat16>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
-        default: return launch_t<__half>(q, k, v, out, n_units, N, d, m, iters, pool, stream);
+        case 0: return launch_t<float>(q, k, v, out, n_units, N, d, m, iters, pool, bias, stream);
+        case 1: return launch_t<__nv_bfloat16>(q, k, v, out, n_units, N, d, m, iters, pool, bias, stream);
+        default: return launch_t<__half>(q, k, v, out, n_units, N, d, m, iters, pool, bias, stream);
     }
 }
 }  // namespace nystra_host

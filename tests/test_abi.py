@@ -29,7 +29,7 @@ def test_header_declares_the_boundary():
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
                      "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
                      "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size",
-                     "nystra_attention_ex"):
+                     "nystra_attention_ex", "nystra_pool_bias", "nystra_attention_bias"):
         assert required in names
 
 
@@ -150,4 +150,37 @@ def test_debug_stages_argument_validation(lib, args, code):
 def test_nystra_ex_argument_validation(lib, args, code):
     rc = nb.nystra_attention_ex(P, 2 * P, 3 * P, 64 * P, args.get("nw", 4), 2, args["N"], 30, args["m"], 6,
                                 args["lm"], 1, None)
+    assert rc == code
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(N=64, m=15), nb.NYSTRA_EINVAL),          # m does not divide N
+    (dict(N=64, m=8, lm=1), nb.NYSTRA_EINVAL),     # no square grid
+    (dict(N=64, m=16, lm=2), nb.NYSTRA_EINVAL),
+    (dict(nb=-1), nb.NYSTRA_EINVAL),
+    (dict(nb=0), nb.NYSTRA_OK),                    # nothing to pool
+    (dict(bias=0), nb.NYSTRA_EINVAL),
+    (dict(bL=5 * P + 4), nb.NYSTRA_EINVAL),        # misaligned
+    (dict(bU=P), nb.NYSTRA_EINVAL),                # output overlaps the bias
+])
+def test_pool_bias_argument_validation(lib, args, code):
+    a = dict(N=64, m=16, lm=0, nb=6, bias=P, bL=8 * P, bU=9 * P, bA=10 * P)
+    a.update(args)
+    rc = nb.nystra_pool_bias(a["bias"], a["nb"], a["N"], a["m"], a["lm"], a["bL"], a["bU"], a["bA"], None)
+    assert rc == code
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(bw=3), nb.NYSTRA_EINVAL),               # neither 1 nor n_windows
+    (dict(bL=0), nb.NYSTRA_EINVAL),
+    (dict(bA=10 * P + 8), nb.NYSTRA_EINVAL),      # misaligned
+    (dict(bL=64 * P), nb.NYSTRA_EINVAL),          # overlaps out
+    (dict(m=15), nb.NYSTRA_EINVAL),
+    (dict(nw=0), nb.NYSTRA_OK),                   # empty: no-op
+])
+def test_attention_bias_argument_validation(lib, args, code):
+    a = dict(nw=4, m=16, bL=8 * P, bU=9 * P, bA=10 * P, bw=1)
+    a.update(args)
+    rc = nb.nystra_attention_bias(P, 2 * P, 3 * P, 64 * P, a["nw"], 2, 64, 30, a["m"], 6, 0, a["bL"], a["bU"],
+                                  a["bA"], a["bw"], 1, None)
     assert rc == code
