@@ -127,6 +127,14 @@ class ClockSampler:
                 "reasons": reasons, "samples": len(rows)}
 
 
+def _oracle_bias(wl, lo: int, hi: int):
+    """The score bias of units lo .. hi - 1 for the oracle (unit u uses head u % heads), or None."""
+    bias = workloads.make_bias(wl)
+    if bias is None:
+        return None
+    return bias.double().numpy()[np.arange(lo, hi) % wl.heads]
+
+
 def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
     """Time the float64 oracle on a bounded sample of the workload's units."""
     import oracle  # CPU baseline only
@@ -135,7 +143,7 @@ def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
     # calibrate on a few units, then size the sample to the budget
     n0 = min(64, qd.shape[0])
     t0 = time.perf_counter()
-    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters, wl.landmarks)
+    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters, wl.landmarks, _oracle_bias(wl, 0, n0))
     per_unit = max((time.perf_counter() - t0) / n0, 1e-9)
     n = int(min(qd.shape[0], max(1, budget_s / per_unit)))
     if max_units:
@@ -143,7 +151,7 @@ def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
     # repeat passes over the sample until the budget is used (at least one pass)
     passes, t0 = 0, time.perf_counter()
     while True:
-        oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters, wl.landmarks)
+        oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters, wl.landmarks, _oracle_bias(wl, 0, n))
         passes += 1
         dt = time.perf_counter() - t0
         if dt >= budget_s:
@@ -164,7 +172,7 @@ def _config(wl, ws: int):
     nsets = max(2, -(-3 * _l2_bytes() // io_bytes))
     return nsets, io_bytes, {
         "workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N, "d_h": wl.d, "m": wl.m,
-        "iters": wl.iters, "io_dtype": wl.dtype, "landmarks": wl.landmarks,
+        "iters": wl.iters, "io_dtype": wl.dtype, "landmarks": wl.landmarks, "bias": wl.bias or "none",
         "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
         "parallelism": f"replica x{ws} (independent windows)"}
 
@@ -180,16 +188,16 @@ def run_reference(args, wl):
     qd, kd, vd = (x.reshape(-1, wl.N, wl.d).double().numpy() for x in (q, k, v))
     n0 = min(32, qd.shape[0])
     t0 = time.perf_counter()
-    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters, wl.landmarks)
+    oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters, wl.landmarks, _oracle_bias(wl, 0, n0))
     per_unit = max((time.perf_counter() - t0) / n0, 1e-9)
     n = int(min(qd.shape[0], max(1, per_step_budget / per_unit)))
     for _ in range(args.warmup):
-        oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters, wl.landmarks)
+        oracle.nystra_attention(qd[:n], kd[:n], vd[:n], wl.m, wl.iters, wl.landmarks, _oracle_bias(wl, 0, n))
     t0 = time.perf_counter()
     for s in range(args.steps):
         off = (s * n) % max(1, qd.shape[0] - n + 1)
         oracle.nystra_attention(qd[off:off + n], kd[off:off + n], vd[off:off + n], wl.m, wl.iters,
-                                wl.landmarks)
+                                wl.landmarks, _oracle_bias(wl, off, off + n))
     dt = time.perf_counter() - t0
     value = args.steps * n * wl.N / dt
     line = {
@@ -224,6 +232,8 @@ def run_cuda(args, wl):
         sets.append(tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),))
     stream = torch.cuda.current_stream(dev)
     sptr = stream.cuda_stream
+    bias = workloads.make_bias(wl)  # a model constant: pooled once, outside the timed region
+    pooled = None if bias is None else binding.pool_bias(bias.to(dev), wl.m, wl.landmarks)
     shape = (wl.n_windows, wl.heads, wl.N, wl.d)
     dcode = {"f32": 0, "bf16": 1, "f16": 2}[wl.dtype]
 
@@ -232,6 +242,10 @@ def run_cuda(args, wl):
         if exact:
             rc = binding.exact_window_attention(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(),
                                                 *shape, dcode, sptr)
+        elif pooled is not None:
+            rc = binding.nystra_attention_bias(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
+                                               wl.m, wl.iters, binding.LANDMARKS[wl.landmarks],
+                                               *(x.data_ptr() for x in pooled), 1, dcode, sptr)
         elif wl.landmarks == "patches":
             rc = binding.nystra_attention_ex(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
                                              wl.m, wl.iters, binding.NYSTRA_LANDMARKS_PATCHES, dcode, sptr)
@@ -290,7 +304,10 @@ def run_cuda(args, wl):
         dq, dk, dv, do = sets[i % 2]
         with torch.cuda.stream(streams[i % 2]):
             dq.copy_(hq, non_blocking=True); dk.copy_(hk, non_blocking=True); dv.copy_(hv, non_blocking=True)
-            binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do, landmarks=wl.landmarks)
+            if pooled is None:
+                binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do, landmarks=wl.landmarks)
+            else:
+                binding.nystra_biased(dq, dk, dv, pooled, wl.m, wl.iters, out=do, landmarks=wl.landmarks)
             hos[i % 2].copy_(do, non_blocking=True)
 
     e2e_steps = max(4, min(args.steps, 50))

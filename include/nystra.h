@@ -153,8 +153,10 @@ NYSTRA_API int nystra_pool_bias(const float* bias, int n_bias, int N, int m, int
  * bias_windows = 1 (one bias per head, shared by every window: the
  * relative-position bias) or n_windows (per window and head: masks of
  * shifted windows).  Unit (w, h) uses slice h, or w * heads + h.  The blocks
- * must not overlap out.  Runs on the fp32 SIMT path.  Other arguments and
- * return codes as nystra_attention_ex.
+ * must not overlap out.  m in {8, 16} runs on the tensor-core kernels of
+ * nystra_attention (with the bias added to the scaled scores before each row
+ * maximum), other shapes on the fp32 SIMT path.  Other arguments and return
+ * codes as nystra_attention_ex.
  */
 NYSTRA_API int nystra_attention_bias(const void* q, const void* k, const void* v, void* out, int n_windows,
                                      int heads, int N, int d_h, int m, int iters, int landmarks,

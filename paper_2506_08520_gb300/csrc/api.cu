@@ -81,15 +81,18 @@ int nystra_call(const void* q, const void* k, const void* v, void* out, int n_wi
     const bool io16 = dtype == NYSTRA_BF16 || dtype == NYSTRA_F16;
     const bool tc16 = io16 && (patches ? m == 16 : (m == 8 || m == 16 || m == 32 || m == 64));
     const bool tc32 = !patches && dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
-    const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32 && bias.L == nullptr;
+    // A score bias on the tensor cores: the one-warp core, m <= 16.
+    const bool biased = bias.L != nullptr;
+    const bool tc = (tc16 || tc32) && d_h % 2 == 0 && d_h <= 32 && (!biased || m <= 16);
+    const nystra::NystraBias* bp = biased ? &bias : nullptr;
     const int pool = patches ? 1 : 0;
     cudaError_t e;
     if (tc && N == 64)
-        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
+        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else if (tc && N == 256)
-        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
+        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else if (tc && N == 1024)
-        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s);
+        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else
         e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, pool, dtype, s, bias);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);

@@ -51,13 +51,17 @@ cudaError_t launch_exact_generic(const void* q, const void* k, const void* v, vo
                                  long long n_units, int N, int d, int dtype, cudaStream_t stream);
 // Tensor-core kernels, windows of 64 / 256 / 1024 tokens (nystra_tc_n*.cu):
 // 16-bit I/O with m in {8, 16, 32, 64}, fp32 I/O at N = 64 with m in {8, 16};
-// even d_h <= 32.  Square-patch landmarks (pool = 1): 16-bit I/O, m = 16.
+// even d_h <= 32.  Square-patch landmarks (pool = 1): 16-bit I/O, m = 16.  A
+// score bias (bias != nullptr): m in {8, 16}.
 cudaError_t launch_nystra_tc_n64(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                 int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
+                                 int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                 const nystra::NystraBias* bias = nullptr);
 cudaError_t launch_nystra_tc_n256(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                  int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
+                                  int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                 const nystra::NystraBias* bias = nullptr);
 cudaError_t launch_nystra_tc_n1024(const void* q, const void* k, const void* v, void* out, long long n_units,
-                                   int d, int m, int iters, int pool, int dtype, cudaStream_t stream);
+                                   int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                 const nystra::NystraBias* bias = nullptr);
 unsigned int take_fault_word_tc_n64(cudaError_t* err);
 unsigned int take_fault_word_tc_n256(cudaError_t* err);
 unsigned int take_fault_word_tc_n1024(cudaError_t* err);

@@ -57,10 +57,10 @@ struct PoolLayout {
     static_assert(BYTES <= kSmemLimit, "pool does not fit in shared memory");
 };
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS>
 __global__ void __launch_bounds__(PoolLayout<T, M, NCOL>::NW * 32, 1)
 nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, T* __restrict__ out,
-                   long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+                   long long n_units, int d_in, int iters, float sl2, unsigned int* fault, NystraBias bias) {
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using P = PoolLayout<T, M, NCOL>;
     constexpr int L = 64 / M;  // tokens per landmark segment
@@ -108,6 +108,11 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     for (long long j = w;; j += P::NW) {
         const long long u = unit_of(j);
         if (u >= n_units) break;
+        // BIAS: this unit's blocks of the score bias (N = 64)
+        const long long bs = BIAS ? (bias.per_window ? u : u % bias.heads) : 0;
+        const float* bLu = BIAS ? bias.L + (size_t)bs * 64 * M : nullptr;
+        const float* bUu = BIAS ? bias.U + (size_t)bs * M * 64 : nullptr;
+        const float* bAu = BIAS ? bias.A + (size_t)bs * M * M : nullptr;
         const bool ok = __all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
         if (!ok) {
             if (lane == 0) atomicOr(fault, 1u);
@@ -134,13 +139,14 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
             typename Opnd<T>::Reg f[P::KTL][4];
-            gl_tile<T, M, P::KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
+            gl_tile<T, M, P::KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
+                                        BIAS ? bLu + (16 * tm + g) * M : nullptr);
 #pragma unroll
             for (int kk = 0; kk < P::KTL; ++kk) GlPark<T, M>::put(glf, (tm * P::KTL + kk) * 32 + lane, f[kk]);
         }
         // ---------------- front: S_U, m_U, W = G_U^n [V | 1] ----------------
         float mU[1][2];
-        front_su_w<T, M, NCOL, 1>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU);
+        front_su_w<T, M, NCOL, 1, BIAS>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU, bUu, 64);
         // The stage is consumed: hand it to the partner's next unit.
         fence_proxy_async_smem();
         __syncwarp();
@@ -148,7 +154,7 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         if (lane == 0 && un < n_units)
             issue(un, reinterpret_cast<uint64_t*>(pp + P::BAR), reinterpret_cast<uint32_t*>(pp + P::CNT));
         // ---------------- core: G_A^n, Z_0, iteration, Y ----------------
-        core_warp<T, M, NCOL>(qbar, kbar, mU, mW, yT, iters, sl2, g, t);
+        core_warp<T, M, NCOL, false, BIAS>(qbar, kbar, mU, mW, yT, iters, sl2, g, t, nullptr, bAu);
         __syncwarp();
         // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
         output_rows<T, M, NCOL, 1, true>(glf, Qs, kbar, yT, ob, d, g, t, lane, sl2);
@@ -166,11 +172,11 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (*cnt > consumed) (void)__all_sync(0xffffffffu, mbar_wait_bounded(bar, phase, kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS = false>
 cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                        int iters, cudaStream_t stream, unsigned int* fault) {
+                        int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
     using P = PoolLayout<T, M, NCOL>;
-    auto kern = nystra_pool_kernel<T, M, NCOL, DC, PW>;
+    auto kern = nystra_pool_kernel<T, M, NCOL, DC, PW, BIAS>;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
@@ -186,7 +192,7 @@ cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* ou
     const long long grid = n_units < s_blocks ? n_units : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, P::NW * 32, P::BYTES, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
-                                                             n_units, d, iters, sl2, fault);
+                                                             n_units, d, iters, sl2, fault, bias);
     return cudaGetLastError();
 }
 
@@ -194,7 +200,9 @@ cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* ou
 // (constant strides and column bounds); others read it at run time.
 template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                     int iters, cudaStream_t stream, unsigned int* fault) {
+                     int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
+    if (bias)  // a score bias: d_h read at run time (one kernel per shape, not per width)
+        return launch_pool_dc<T, M, NCOL, 0, PW, true>(q, k, v, out, n_units, d, iters, stream, fault, *bias);
     if constexpr (NCOL == 32) {
         if (d == 30) return launch_pool_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {

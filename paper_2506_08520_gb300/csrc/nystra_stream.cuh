@@ -104,10 +104,12 @@ __device__ __forceinline__ StreamTask stream_task(int v, int count) {
     }
 }
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS>
 __global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * StreamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-                     T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+                     T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault,
+                     NystraBias bias) {
+    static_assert(!BIAS || M <= 16, "a score bias runs with the one-warp core");
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using Lay = StreamLayout<M, NCOL>;
     using TL = typename Lay::TL;
@@ -171,10 +173,14 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
             if constexpr (Lay::CWN == 1) {
                 float mU[1][2] = {{gmu[g], gmu[g + 8]}};
-                core_warp<T, M, NCOL>(reinterpret_cast<const T*>(bb + Lay::B_QB),
-                                      reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
-                                      reinterpret_cast<const float*>(bb + Lay::B_W),
-                                      reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+                const long long uk = u0 + kk * stride;
+                const float* bAu =
+                    BIAS ? bias.A + (size_t)(bias.per_window ? uk : uk % bias.heads) * M * M : nullptr;
+                core_warp<T, M, NCOL, false, BIAS>(reinterpret_cast<const T*>(bb + Lay::B_QB),
+                                                   reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
+                                                   reinterpret_cast<const float*>(bb + Lay::B_W),
+                                                   reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t, nullptr,
+                                                   bAu);
             } else {
                 using DSc = DistScratch<(M > 16 ? M : 32)>;
                 unsigned char* scr = tb + TL::T_SCR;
@@ -233,6 +239,8 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
         const int s = vv % NSLOT;
         const int b = tk.k & 1;
         unsigned char* bb = buf(b);
+        // BIAS: the unit's score-bias slice (N = 1024 tokens, M landmarks)
+        const long long bsl = BIAS ? (bias.per_window ? u0 + tk.k * stride : (u0 + tk.k * stride) % bias.heads) : 0;
         // ---------------- bounded wait for this task's chunk ----------------
         if (!failed) {
             if (__all_sync(0xffffffffu, mbar_wait_bounded(sbar + s, (uint32_t)((vv / NSLOT) & 1), kWaitNs))) {
@@ -276,8 +284,12 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, ck, d, g, t);
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt)
-                su_w_chunk<T, NCOL>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M, 16 * mt + g + 8 < M,
-                                    w[mt], run[mt][0], run[mt][1], true);
+                su_w_chunk<T, NCOL, BIAS>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M,
+                                          16 * mt + g + 8 < M, w[mt], run[mt][0], run[mt][1], true,
+                                          BIAS ? bias.U + (size_t)bsl * M * N + (size_t)(16 * mt + g) * N +
+                                                     r * TPW + tk.c * Lay::CH
+                                               : nullptr,
+                                          N);
             if (tk.c == Lay::NCHK - 1) {
                 landmarks_put<T, LPW>(ck, reinterpret_cast<T*>(bb + Lay::B_KB), r * LPW, g, t);
                 // the partial goes over this slot's K and V rows, consumed above
@@ -315,9 +327,10 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                 }
             }
             if (!failed) {
-                output_rows<T, M, NCOL, 1, false>(nullptr, X0, reinterpret_cast<const T*>(bb + Lay::B_KB),
-                                                  reinterpret_cast<const T*>(bb + Lay::B_YT), X0, d, g, t, lane,
-                                                  sl2);
+                output_rows<T, M, NCOL, 1, false, BIAS>(
+                    nullptr, X0, reinterpret_cast<const T*>(bb + Lay::B_KB), reinterpret_cast<const T*>(bb + Lay::B_YT),
+                    X0, d, g, t, lane, sl2,
+                    BIAS ? bias.L + (size_t)bsl * N * M + (size_t)(r * TPW + tk.c * Lay::CH) * M : nullptr);
                 fence_proxy_async_smem();  // this lane's writes precede the bulk store
                 __syncwarp();
                 if (lane == 0) {
@@ -342,11 +355,11 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
         (void)__all_sync(0xffffffffu, mbar_wait_bounded(sbar + i % NSLOT, (uint32_t)((i / NSLOT) & 1), kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS = false>
 cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                          int iters, cudaStream_t stream, unsigned int* fault) {
+                          int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
     using Lay = StreamLayout<M, NCOL>;
-    auto kern = nystra_stream_kernel<T, M, NCOL, DC, PW>;
+    auto kern = nystra_stream_kernel<T, M, NCOL, DC, PW, BIAS>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -365,7 +378,7 @@ cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* 
     const long long grid = want < s_blocks ? want : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, Lay::TEAMS * Lay::WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
-                                                                 n_units, d, iters, sl2, fault);
+                                                                 n_units, d, iters, sl2, fault, bias);
     return cudaGetLastError();
 }
 
@@ -373,7 +386,10 @@ cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* 
 // (constant strides and column bounds); others read it at run time.
 template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                     int iters, cudaStream_t stream, unsigned int* fault) {
+                     int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
+    if constexpr (M <= 16)
+        if (bias)  // a score bias: d_h read at run time
+            return launch_stream_dc<T, M, NCOL, 0, PW, true>(q, k, v, out, n_units, d, iters, stream, fault, *bias);
     if constexpr (NCOL == 32) {
         if (d == 30) return launch_stream_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {

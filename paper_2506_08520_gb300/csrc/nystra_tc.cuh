@@ -57,6 +57,7 @@ namespace nystra {
 namespace tc {
 
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
+constexpr float kLog2e = 1.4426950408889634f;  // score bias into the log2 domain of ex2
 constexpr size_t kSmemLimit = 232448;        // opt-in dynamic shared memory per CTA
 
 // Shared scratch of the distributed core (m = 32, 64; see dist_core): two
@@ -324,9 +325,11 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
 
 // S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
 // fragments (A operand of O = G_L^n Y, k = landmarks).
-template <typename T, int M, int KTL>
+// BIAS: bl points at row g of the tile in the N x M block B_L of the score
+// bias (row stride M); log2(e) B_L enters the exponent beside the scaled score.
+template <typename T, int M, int KTL, bool BIAS = false>
 __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g, int t, float sl2,
-                                        typename Opnd<T>::Reg (&f)[KTL][4]) {
+                                        typename Opnd<T>::Reg (&f)[KTL][4], const float* bl = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int NTL = M / 8, LS = 40;
@@ -350,16 +353,28 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
             O::mma(sl[j], a[kk], O::ld(kr), O::ld(kr + 8));
         }
     }
+    if constexpr (BIAS) {  // scores in the log2 domain, bias included: e0/e1 below take them as they are
+#pragma unroll
+        for (int j = 0; j < NTL; ++j) {
+            const float2 b0 = __ldg(reinterpret_cast<const float2*>(bl + 8 * j + 2 * t));
+            const float2 b1 = __ldg(reinterpret_cast<const float2*>(bl + 8 * M + 8 * j + 2 * t));
+            sl[j][0] = fmaf(sl[j][0], sl2, kLog2e * b0.x);
+            sl[j][1] = fmaf(sl[j][1], sl2, kLog2e * b0.y);
+            sl[j][2] = fmaf(sl[j][2], sl2, kLog2e * b1.x);
+            sl[j][3] = fmaf(sl[j][3], sl2, kLog2e * b1.y);
+        }
+    }
     float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
     for (int j = 0; j < NTL; ++j) {
         mx0 = fmaxf(mx0, fmaxf(sl[j][0], sl[j][1]));
         mx1 = fmaxf(mx1, fmaxf(sl[j][2], sl[j][3]));
     }
-    mx0 = quad_max(mx0) * sl2;
-    mx1 = quad_max(mx1) * sl2;
-    auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
-    auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+    const float ssl = BIAS ? 1.f : sl2;
+    mx0 = quad_max(mx0) * ssl;
+    mx1 = quad_max(mx1) * ssl;
+    auto e0 = [&](float x) { return ex2(fmaf(x, ssl, -mx0)); };
+    auto e1 = [&](float x) { return ex2(fmaf(x, ssl, -mx1)); };
     if constexpr (M >= 16) {
 #pragma unroll
         for (int kk = 0; kk < KTL; ++kk) {
@@ -535,10 +550,13 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 // G_U^n = exp(S_U - m) fed from registers as the A operand of
 // w += G_U^n [V | 1] (B fragments of [V | 1 | 0] by 8x8 transposes; the ones
 // column yields the denominator).
-template <typename T, int NCOL>
+// BIAS: bu points at the chunk's first key in row g of the m-tile in the
+// M x N block B_U of the score bias (row stride bn).
+template <typename T, int NCOL, bool BIAS = false>
 __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][4], const T* Kc, const T* Vc, int d,
                                            int g, int t, float sl2, bool v0, bool v1, float (&w)[NCOL / 8][4],
-                                           float& run0, float& run1, bool rescale) {
+                                           float& run0, float& run1, bool rescale, const float* bu = nullptr,
+                                           int bn = 0) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int NTO = NCOL / 8;
@@ -555,11 +573,24 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][
             O::mma(s[nt], aq[kk], b0, b1);
         }
     }
+    if constexpr (BIAS) {  // scores in the log2 domain, bias included (rows beyond m stay unbiased)
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt) {
+            const float2 b0 = v0 ? __ldg(reinterpret_cast<const float2*>(bu + 8 * nt + 2 * t)) : make_float2(0.f, 0.f);
+            const float2 b1 = v1 ? __ldg(reinterpret_cast<const float2*>(bu + 8 * bn + 8 * nt + 2 * t))
+                                 : make_float2(0.f, 0.f);
+            s[nt][0] = fmaf(s[nt][0], sl2, kLog2e * b0.x);
+            s[nt][1] = fmaf(s[nt][1], sl2, kLog2e * b0.y);
+            s[nt][2] = fmaf(s[nt][2], sl2, kLog2e * b1.x);
+            s[nt][3] = fmaf(s[nt][3], sl2, kLog2e * b1.y);
+        }
+    }
+    const float ssl = BIAS ? 1.f : sl2;
     float mx0 = run0, mx1 = run1;
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
-        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * sl2);
-        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * sl2);
+        mx0 = fmaxf(mx0, fmaxf(s[nt][0], s[nt][1]) * ssl);
+        mx1 = fmaxf(mx1, fmaxf(s[nt][2], s[nt][3]) * ssl);
     }
     mx0 = quad_max(mx0);
     mx1 = quad_max(mx1);
@@ -572,8 +603,8 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][
     }
     run0 = mx0;
     run1 = mx1;
-    auto e0 = [&](float x) { return ex2(fmaf(x, sl2, -mx0)); };
-    auto e1 = [&](float x) { return ex2(fmaf(x, sl2, -mx1)); };
+    auto e0 = [&](float x) { return ex2(fmaf(x, ssl, -mx0)); };
+    auto e1 = [&](float x) { return ex2(fmaf(x, ssl, -mx1)); };
 #pragma unroll
     for (int kt = 0; kt < 4; ++kt) {
         R a[4];
@@ -610,9 +641,12 @@ __device__ __forceinline__ void qbar_afrag(const T* qbar, int mt, int g, int t, 
 // chunks for every landmark m-tile.  W_r (MP x NCOL) is stored at dst with
 // row stride ws after a warp sync (so every lane is done reading K and V);
 // the row maxima (log2 domain) are returned in mU.
-template <typename T, int M, int NCOL, int NCH>
+// BIAS: bu is the unit's M x N block B_U of the score bias, offset to the
+// first key of Ks (row stride bn).
+template <typename T, int M, int NCOL, int NCH, bool BIAS = false>
 __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
-                                           float* dst, int ws, float (&mU)[(M + 15) / 16][2]) {
+                                           float* dst, int ws, float (&mU)[(M + 15) / 16][2],
+                                           const float* bu = nullptr, int bn = 0) {
     using R = typename Opnd<T>::Reg;
     constexpr int MT = (M + 15) / 16, NTO = NCOL / 8;
     float wall[MT][NTO][4];
@@ -627,7 +661,8 @@ __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* 
         float run0 = -INFINITY, run1 = -INFINITY;
 #pragma unroll 1
         for (int ch = 0; ch < NCH; ++ch)
-            su_w_chunk<T, NCOL>(aq, Ks + ch * 64 * d, Vs + ch * 64 * d, d, g, t, sl2, v0, v1, w, run0, run1, NCH > 1);
+            su_w_chunk<T, NCOL, BIAS>(aq, Ks + ch * 64 * d, Vs + ch * 64 * d, d, g, t, sl2, v0, v1, w, run0, run1,
+                                      NCH > 1, BIAS ? bu + (size_t)(16 * mt + g) * bn + ch * 64 : nullptr, bn);
         mU[mt][0] = run0;
         mU[mt][1] = run1;
     }
@@ -679,10 +714,11 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
 //
 // DUMP (test-only stage dump): dbg receives G_A^n (M x M), Z (M x M) and
 // Y = Z W (M x NCOL), row-major fp32, with the dropped factors restored.
-template <typename T, int M, int NCOL, bool DUMP = false>
+// BIAS: ba is the unit's M x M block B_A of the score bias.
+template <typename T, int M, int NCOL, bool DUMP = false, bool BIAS = false>
 __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const float (&mU)[(M + 15) / 16][2],
                                           const float* mW, T* yT, int iters, float sl2, int g, int t,
-                                          float* dbg = nullptr) {
+                                          float* dbg = nullptr, const float* ba = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int MT = (M + 15) / 16, LS = 40, WS = NCOL + 4, NTO = NCOL / 8;
@@ -719,10 +755,21 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                     O::mma(sa, aq[kk], O::ld(kr), O::ld(kr + 8));
                 }
                 const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
-                Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
-                Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
-                Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
-                Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+                if constexpr (BIAS) {  // log2(e) B_A joins the shift (c and c + 1 < M together: M is even)
+                    const float2 b0 = (r0 < M && c < M) ? __ldg(reinterpret_cast<const float2*>(ba + r0 * M + c))
+                                                        : make_float2(0.f, 0.f);
+                    const float2 b1 = (r1 < M && c < M) ? __ldg(reinterpret_cast<const float2*>(ba + r1 * M + c))
+                                                        : make_float2(0.f, 0.f);
+                    Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, fmaf(kLog2e, b0.x, -mU[mt][0]))) : 0.f;
+                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, fmaf(kLog2e, b0.y, -mU[mt][0]))) : 0.f;
+                    Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, fmaf(kLog2e, b1.x, -mU[mt][1]))) : 0.f;
+                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, fmaf(kLog2e, b1.y, -mU[mt][1]))) : 0.f;
+                } else {
+                    Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
+                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
+                    Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
+                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+                }
             }
         }
         // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
@@ -1242,9 +1289,12 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
 // Output for one warp's NCH chunks: O = (G_L^n Y_:d) / (G_L^n Y_d) (steps
 // 5-7); G_L^n fragments come from glf (parked) or are recomputed from Qs and
 // Kbar; rows are written row-major to obase (N_w x d).
-template <typename T, int M, int NCOL, int NCH, bool GLS>
+// BIAS (recomputed G_L^n only): bl is B_L of the score bias at the warp's
+// first token (row stride M).
+template <typename T, int M, int NCOL, int NCH, bool GLS, bool BIAS = false>
 __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, const T* kbar, const T* yT,
-                                            T* obase, int d, int g, int t, int lane, float sl2) {
+                                            T* obase, int d, int g, int t, int lane, float sl2,
+                                            const float* bl = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int KTL = (M >= 16) ? M / 16 : 1, NTO = NCOL / 8, YS = (M < 16 ? 16 : M) + 8;
@@ -1268,7 +1318,8 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
 #pragma unroll
                 for (int kk = 0; kk < KTL; ++kk) GlPark<T, M>::get(glf, ((ch * 4 + tm) * KTL + kk) * 32 + lane, f[kk]);
             } else {
-                gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
+                gl_tile<T, M, KTL, BIAS>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f,
+                                         BIAS ? bl + (size_t)(ch * 64 + 16 * tm + g) * M : nullptr);
             }
             float o[NTO][4];
 #pragma unroll
@@ -1606,25 +1657,25 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
 // only).  PW: 0 = segment landmarks, else square patches of a PW-wide window.
 template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_pool(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                        int iters, cudaStream_t stream, unsigned int* fault);
+                        int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias = nullptr);
 
 // Team kernel for 16x16 windows (nystra_team.cuh, N = 256 translation unit only).
 template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                        int iters, cudaStream_t stream, unsigned int* fault);
+                        int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias = nullptr);
 
 // fp32 I/O: 8x8 windows with m <= 16 only (the stage-pool kernel).
 template <int TPW, int WPU>
 cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
-                       int iters, cudaStream_t stream, unsigned int* fault) {
+                       int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias = nullptr) {
     if constexpr (TPW == 64 && WPU == 1) {
         const bool wide = d > 30;
         if (m == 8)
-            return wide ? launch_pool<float, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_pool<float, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_pool<float, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_pool<float, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         if (m == 16)
-            return wide ? launch_pool<float, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_pool<float, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_pool<float, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_pool<float, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     }
     return cudaErrorInvalidValue;
 }
@@ -1632,39 +1683,41 @@ cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, l
 // Streaming team kernel for 32x32 windows (nystra_stream.cuh, N = 1024 translation unit only).
 template <typename T, int M, int NCOL, int PW = 0>
 cudaError_t launch_stream(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                          int iters, cudaStream_t stream, unsigned int* fault);
+                          int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias = nullptr);
 
 // Dispatch on m and the output-column padding for one window size.
+// bias (m <= 16 only: the one-warp core) selects the kernels with a score bias.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
-                     int iters, cudaStream_t stream, unsigned int* fault) {
+                     int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias = nullptr) {
     const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
+    if (bias && m > 16) return cudaErrorInvalidValue;  // not reached: the caller sends these to the SIMT path
     if constexpr (TPW == 64 && WPU == 1) {
         if (m == 8)
-            return wide ? launch_pool<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_pool<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_pool<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_pool<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         if (m == 16)
-            return wide ? launch_pool<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_pool<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_pool<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_pool<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     }
     if constexpr (TPW == 64 && WPU == 4) {
         if (m == 8)
-            return wide ? launch_team<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_team<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_team<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_team<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         if (m == 16)
-            return wide ? launch_team<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_team<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_team<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_team<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         // m = 32 with d_h <= 30 fits two teams per SM; d_h = 32 only one, so it
         // stays on the grouped kernel
         if (m == 32 && !wide) return launch_team<T, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
     }
     if constexpr (TPW == 128 && WPU == 8) {
         if (m == 8)
-            return wide ? launch_stream<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_stream<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_stream<T, 8, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_stream<T, 8, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         if (m == 16)
-            return wide ? launch_stream<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault)
-                        : launch_stream<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+            return wide ? launch_stream<T, 16, 40>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                        : launch_stream<T, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
         if (m == 32)
             return wide ? launch_stream<T, 32, 40>(q, k, v, out, n_units, d, iters, stream, fault)
                         : launch_stream<T, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
@@ -1694,18 +1747,19 @@ cudaError_t launch_n(const void* q, const void* k, const void* v, void* out, lon
 // patches of 2x2, 4x4 or 8x8 tokens), one window size per translation unit.
 template <typename T, int TPW, int WPU>
 cudaError_t launch_patches(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                           int m, int iters, cudaStream_t stream, unsigned int* fault) {
+                           int m, int iters, cudaStream_t stream, unsigned int* fault,
+                           const NystraBias* bias = nullptr) {
     const bool wide = d > 30;
     if (m != 16) return cudaErrorInvalidValue;  // not reached: checked by the caller
     if constexpr (TPW == 64 && WPU == 1)
-        return wide ? launch_pool<T, 16, 40, 8>(q, k, v, out, n_units, d, iters, stream, fault)
-                    : launch_pool<T, 16, 32, 8>(q, k, v, out, n_units, d, iters, stream, fault);
+        return wide ? launch_pool<T, 16, 40, 8>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                    : launch_pool<T, 16, 32, 8>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     if constexpr (TPW == 64 && WPU == 4)
-        return wide ? launch_team<T, 16, 40, 16>(q, k, v, out, n_units, d, iters, stream, fault)
-                    : launch_team<T, 16, 32, 16>(q, k, v, out, n_units, d, iters, stream, fault);
+        return wide ? launch_team<T, 16, 40, 16>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                    : launch_team<T, 16, 32, 16>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     if constexpr (TPW == 128 && WPU == 8)
-        return wide ? launch_stream<T, 16, 40, 32>(q, k, v, out, n_units, d, iters, stream, fault)
-                    : launch_stream<T, 16, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault);
+        return wide ? launch_stream<T, 16, 40, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias)
+                    : launch_stream<T, 16, 32, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     return cudaErrorInvalidValue;
 }
 
@@ -1720,7 +1774,7 @@ cudaError_t launch_patches(const void* q, const void* k, const void* v, void* ou
     namespace nystra_host {                                                                                  \
     cudaError_t launch_nystra_tc_##NAME(const void* q, const void* k, const void* v, void* out,              \
                                         long long n_units, int d, int m, int iters, int pool, int dtype,     \
-                                        cudaStream_t stream) {                                               \
+                                        cudaStream_t stream, const nystra::NystraBias* bias) {               \
         static unsigned int* s_fault[64] = {};  /* device address of the fault word, per device */      \
         int dev = 0;                                                                                         \
         cudaError_t e = cudaGetDevice(&dev);                                                                 \
@@ -1734,18 +1788,18 @@ cudaError_t launch_patches(const void* q, const void* k, const void* v, void* ou
         if (pool != 0) {                                                                                     \
             if (dtype == 1)                                                                                  \
                 return nystra::tc::launch_patches<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m,      \
-                                                                           iters, stream, fault);            \
+                                                                           iters, stream, fault, bias);      \
             if (dtype == 2)                                                                                  \
                 return nystra::tc::launch_patches<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters,      \
-                                                                    stream, fault);                          \
+                                                                    stream, fault, bias);                    \
             return cudaErrorInvalidValue; /* not reached: fp32 patches take the SIMT path */                 \
         }                                                                                                    \
         if (dtype == 0)                                                                                      \
-            return nystra::tc::launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault);      \
+            return nystra::tc::launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias);\
         if (dtype == 1)                                                                                      \
             return nystra::tc::launch_n<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, \
-                                                                 fault);                                     \
-        return nystra::tc::launch_n<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault);    \
+                                                                 fault, bias);                               \
+        return nystra::tc::launch_n<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias); \
     }                                                                                                        \
     unsigned int take_fault_word_tc_##NAME(cudaError_t* err) {                                               \
         unsigned int w = 0, zero = 0;                                                                        \

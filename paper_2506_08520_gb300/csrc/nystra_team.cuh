@@ -61,10 +61,12 @@ struct TeamLayout {
     static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
 };
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS>
 __global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * TeamLayout<M, NCOL>::WARPS * 32, 1)
 nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
-                   T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault) {
+                   T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault,
+                   NystraBias bias) {
+    static_assert(!BIAS || M <= 16, "a score bias runs with the one-warp core");
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using Lay = TeamLayout<M, NCOL>;
     constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
@@ -128,10 +130,13 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             const float* gmu = reinterpret_cast<const float*>(bb + Lay::B_MU);
             if constexpr (Lay::CWN == 1) {
                 float mU[1][2] = {{gmu[g], gmu[g + 8]}};
-                core_warp<T, M, NCOLC>(reinterpret_cast<const T*>(bb + Lay::B_QB),
-                                       reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
-                                       reinterpret_cast<const float*>(bb + Lay::B_W),
-                                       reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t);
+                const float* bAu =
+                    BIAS ? bias.A + (size_t)(bias.per_window ? u : u % bias.heads) * M * M : nullptr;
+                core_warp<T, M, NCOLC, false, BIAS>(reinterpret_cast<const T*>(bb + Lay::B_QB),
+                                                    reinterpret_cast<const T*>(bb + Lay::B_KB), mU,
+                                                    reinterpret_cast<const float*>(bb + Lay::B_W),
+                                                    reinterpret_cast<T*>(bb + Lay::B_YT), iters, sl2, g, t,
+                                                    nullptr, bAu);
             } else {
                 using DSc = DistScratch<(M > 16 ? M : 32)>;
                 unsigned char* scr = tb + Lay::T_SCR;
@@ -207,6 +212,9 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     for (;; ++kk) {
         const long long u = u0 + kk * stride;
         if (u >= n_units) break;
+        const long long bs = BIAS ? (bias.per_window ? u : u % bias.heads) : 0;
+        const float* bLu = BIAS ? bias.L + (size_t)bs * N * M : nullptr;
+        const float* bUu = BIAS ? bias.U + (size_t)bs * M * N : nullptr;
         const int b = (int)(kk & 1);
         unsigned char* bb = buf(b);
         T* qbar = reinterpret_cast<T*>(bb + Lay::B_QB);
@@ -232,7 +240,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 #pragma unroll
             for (int tm = 0; tm < 4; ++tm) {
                 typename Opnd<T>::Reg f[KTL][4];
-                gl_tile<T, M, KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
+                gl_tile<T, M, KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
+                                         BIAS ? bLu + (size_t)(r * TPW + 16 * tm + g) * M : nullptr);
 #pragma unroll
                 for (int kq = 0; kq < KTL; ++kq) GlPark<T, M>::put(glf, (tm * KTL + kq) * 32 + lane, f[kq]);
             }
@@ -251,7 +260,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         // ---------------- S_U, partial W_r and row maxima ----------------
         constexpr int MT = (M + 15) / 16;
         float mU[MT][2];
-        front_su_w<T, M, NCOLC, 1>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU);
+        front_su_w<T, M, NCOLC, 1, BIAS>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU,
+                                         BIAS ? bUu + r * TPW : nullptr, N);
         if (t == 0) {
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
@@ -290,11 +300,11 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     if (pend_v) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
 }
 
-template <typename T, int M, int NCOL, int DC, int PW>
+template <typename T, int M, int NCOL, int DC, int PW, bool BIAS = false>
 cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                        int iters, cudaStream_t stream, unsigned int* fault) {
+                        int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
     using Lay = TeamLayout<M, NCOL>;
-    auto kern = nystra_team_kernel<T, M, NCOL, DC, PW>;
+    auto kern = nystra_team_kernel<T, M, NCOL, DC, PW, BIAS>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static int s_blocks = 0;  // persistent grid size, set on first use
     if (s_blocks == 0) {
@@ -313,7 +323,7 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
     const long long grid = want < s_blocks ? want : s_blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, Lay::TEAMS * Lay::WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
-                                                                 n_units, d, iters, sl2, fault);
+                                                                 n_units, d, iters, sl2, fault, bias);
     return cudaGetLastError();
 }
 
@@ -321,7 +331,10 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
 // (constant strides and column bounds); others read it at run time.
 template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
-                     int iters, cudaStream_t stream, unsigned int* fault) {
+                     int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
+    if constexpr (M <= 16)
+        if (bias)  // a score bias: d_h read at run time
+            return launch_team_dc<T, M, NCOL, 0, PW, true>(q, k, v, out, n_units, d, iters, stream, fault, *bias);
     if constexpr (NCOL == 32) {
         if (d == 30) return launch_team_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {

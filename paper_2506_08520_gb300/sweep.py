@@ -8,8 +8,10 @@ rotating input/output sets (together more than 3x the L2 size, so every launch
 reads its inputs from HBM), the algorithmic bytes (Q, K, V read once, O written
 once), the achieved GB/s and its fraction of the measured HBM copy bandwidth,
 tokens*heads/s (for edge-padded maps also counting only the real tokens), and
-the speedup over exact attention.  A mix ("uformer-mix": Uformer stages 1 and
-4) launches its workloads back to back on one stream and is timed as one.
+the speedup over exact attention (which runs without the bias).  A mix
+("uformer-mix": Uformer stages 1 and 4) launches its workloads back to back on
+one stream and is timed as one.  A workload with a relative-position bias
+pools it once (a model constant) and times the biased call.
 """
 from __future__ import annotations
 
@@ -31,7 +33,8 @@ MIXES = {"uformer-mix": ("uformer-s1", "uformer-s4")}
 DEFAULT = (["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4", "uformer-mix"]
            + [f"large-w{w}-m{m}" for w in (16, 32) for m in (32, 64)]
            + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")]
-           + ["swinir256-bf16-patches", "sr720p-w16-m16-bf16-patches", "sr720p-w32-m16-bf16-patches"])
+           + [f"{n}-{x}" for x in ("patches", "relpos")
+              for n in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16")])
 
 
 def hbm_peak_gbs() -> tuple[float, str]:
@@ -71,16 +74,21 @@ def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int =
     io = sum(wl.io_bytes for wl in parts)
     n_sets = max(2, -(-3 * l2_bytes // io))
     dev = torch.device("cuda")
-    sets = []
+    sets, pooled = [], []
     for wl in parts:
         q, k, v = workloads.make_qkv(wl)
         sets.append([tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),)
                      for _ in range(n_sets)])
+        bias = workloads.make_bias(wl)  # pooled once: a model constant
+        pooled.append(None if bias is None else binding.pool_bias(bias.to(dev), wl.m, wl.landmarks))
 
     def nystra(i):
-        for wl, ss in zip(parts, sets):
+        for wl, ss, pb in zip(parts, sets, pooled):
             a, b, c, o = ss[i]
-            binding.nystra(a, b, c, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+            if pb is None:
+                binding.nystra(a, b, c, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+            else:
+                binding.nystra_biased(a, b, c, pb, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
 
     def exact(i):
         for ss in sets:
@@ -97,7 +105,7 @@ def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int =
     real = sum(_real_tokens(wl) for wl in parts)
     if real != tokens:
         res["real_tokens_heads_per_s"] = real / (t_n * 1e-3)
-    del sets
+    del sets, pooled
     torch.cuda.empty_cache()
     return res
 

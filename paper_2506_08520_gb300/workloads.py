@@ -36,6 +36,7 @@ class Workload:
     recipe: str          # "iid" | "proj" | "lowrank" | "map"
     map_hw: tuple = ()   # (H, W, window) for recipe == "map"
     landmarks: str = "segments"  # landmark pooling: "segments" | "patches"
+    bias: str = ""               # score bias: "" (none) | "relpos" (per-head relative-position bias)
 
     @property
     def units(self) -> int:
@@ -83,9 +84,11 @@ for _w in (8, 16, 32):
         for _dt in ("bf16", "f16"):
             _wl = _sr_map(_w, _m, _dt)
             WORKLOADS[_wl.name] = _wl
-# The same inputs with square-patch landmarks (4 x 4 patches).
+# The same inputs with square-patch landmarks (4 x 4 patches), and with a
+# relative-position score bias.
 for _name in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16"):
     WORKLOADS[_name + "-patches"] = WORKLOADS[_name].with_(name=_name + "-patches", landmarks="patches")
+    WORKLOADS[_name + "-relpos"] = WORKLOADS[_name].with_(name=_name + "-relpos", bias="relpos")
 
 
 def _cast(x: np.ndarray, dtype: str) -> torch.Tensor:
@@ -160,3 +163,23 @@ def random_qkv(n_units: int, N: int, d: int, dtype: str = "f32", seed: int = 0, 
     """i.i.d. N(0, scale^2) inputs ``[n_units, N, d]`` for small parity and edge cases."""
     rng = np.random.default_rng(seed)
     return tuple(_cast(scale * rng.standard_normal((n_units, N, d)), dtype) for _ in range(3))
+
+
+def relpos_bias(window: int, heads: int, seed: int, scale: float = 0.5) -> np.ndarray:
+    """A relative-position score bias of a window x window window, as Swin-style
+    layers add it: a seeded table of (2 window - 1)^2 offsets per head, indexed
+    by the row and column offset of each token pair.  fp32 ``[heads, N, N]``."""
+    rng = np.random.default_rng(seed)
+    table = scale * rng.standard_normal(((2 * window - 1) ** 2, heads))
+    r, c = np.divmod(np.arange(window * window), window)
+    idx = (r[:, None] - r[None, :] + window - 1) * (2 * window - 1) + (c[:, None] - c[None, :] + window - 1)
+    return np.ascontiguousarray(table[idx].transpose(2, 0, 1)).astype(np.float32)
+
+
+def make_bias(wl: Workload | str):
+    """The workload's score bias ``[heads, N, N]`` (fp32 host tensor), or None."""
+    if isinstance(wl, str):
+        wl = WORKLOADS[wl]
+    if not wl.bias:
+        return None
+    return torch.from_numpy(relpos_bias(int(round(wl.N ** 0.5)), wl.heads, wl.seed + 100))

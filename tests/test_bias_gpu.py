@@ -96,3 +96,21 @@ def test_zero_bias_equals_the_unbiased_call():
     torch.cuda.synchronize()
     err = per_unit_rel(a.double().cpu().numpy(), b.double().cpu().numpy())
     assert err.max() <= TOL["bf16"]
+
+
+@pytest.mark.parametrize("name", ["swinir256-bf16-relpos", "sr720p-w16-m16-bf16-relpos",
+                                  "sr720p-w32-m16-bf16-relpos"])
+def test_relpos_workloads(name):
+    from tests.parity import sample_units
+    wl = workloads.WORKLOADS[name]
+    q, k, v = workloads.make_qkv(wl)
+    bias = workloads.make_bias(wl)
+    pooled = binding.pool_bias(bias.cuda(), wl.m, wl.landmarks)
+    out = binding.nystra_biased(q.cuda(), k.cuda(), v.cuda(), pooled, wl.m, wl.iters).cpu()
+    idx = sample_units(wl.units, 192)
+    qu, ku, vu, ou = (x.reshape(-1, wl.N, wl.d) for x in (q, k, v, out))
+    b = bias.double().numpy()[idx % wl.heads]  # unit u is head u % heads
+    ref = oracle.nystra_attention(qu[idx], ku[idx], vu[idx], wl.m, wl.iters, wl.landmarks, b)
+    err = per_unit_rel(ou[idx].double().numpy(), ref)
+    print(f"{name}: max rel err {err.max():.3e}")
+    assert err.max() <= TOL[wl.dtype]
