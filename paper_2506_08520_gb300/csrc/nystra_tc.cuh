@@ -126,11 +126,6 @@ struct Layout {
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
 };
 
-template <typename T>
-__device__ __forceinline__ uint32_t ld32(const T* p) {
-    return *reinterpret_cast<const uint32_t*>(p);
-}
-
 // C-layout fragments of an MP x MP fp32 matrix: f[i][n][e] is row
 // 16i + g + 8(e >> 1), column 8n + 2t + (e & 1).
 template <int MT>

@@ -130,11 +130,6 @@ __device__ __forceinline__ float ex2(float x) {
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
 }
-__device__ __forceinline__ uint32_t to_tf32(float x) {
-    uint32_t r;
-    asm("cvt.rna.tf32.f32 %0, %1;" : "=r"(r) : "f"(x));
-    return r;
-}
 // Transpose of an 8x8 matrix of 16-bit elements held one row pair per lane
 // (lane 4r + c holds row r, columns 2c and 2c+1).
 __device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x) {
@@ -164,16 +159,6 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
                  : "r"(smem_addr(p))
                  : "memory");
 }
-__device__ __forceinline__ float warp_sum(float x) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    return x;
-}
-__device__ __forceinline__ float warp_max(float x) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
-    return x;
-}
 // Max over the warp of non-negative floats: their bit patterns order like
 // unsigned integers, so one redux.sync does it.
 __device__ __forceinline__ float warp_max_nonneg(float x) {
@@ -189,13 +174,9 @@ __device__ __forceinline__ float quad_max(float x) {
 // itself is passed as hi) and lo = x - hi, exact in fp32 and again truncated
 // to tf32 by the hardware.  hi + lo equals x to within 2^-20 |x|; the three
 // products lo*hi, hi*lo and hi*hi give a product accurate to about 2^-19.
-struct Tf32Pair {
-    uint32_t hi, lo;
-};
 __device__ __forceinline__ uint32_t tf32_lo(float x) {
     return __float_as_uint(x - __uint_as_float(__float_as_uint(x) & 0xffffe000u));
 }
-__device__ __forceinline__ Tf32Pair split_tf32(float x) { return {__float_as_uint(x), tf32_lo(x)}; }
 
 // m16n8k8 tf32 MMA, fp32 accumulate: c += a (16x8, row) * b (8x8, col).
 __device__ __forceinline__ void mma_tf32(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
@@ -204,13 +185,6 @@ __device__ __forceinline__ void mma_tf32(float (&c)[4], uint32_t a0, uint32_t a1
         "{%0,%1,%2,%3};"
         : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
         : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-// c += a * b in split-tf32 (a: 4 A-fragment registers, b: 2 B-fragment registers).
-__device__ __forceinline__ void mma_tf32x3(float (&c)[4], const Tf32Pair (&a)[4], const Tf32Pair (&b)[2]) {
-    mma_tf32(c, a[0].lo, a[1].lo, a[2].lo, a[3].lo, b[0].hi, b[1].hi);
-    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].lo, b[1].lo);
-    mma_tf32(c, a[0].hi, a[1].hi, a[2].hi, a[3].hi, b[0].hi, b[1].hi);
 }
 
 // fp16 two-term split of a pair of fp32 values: hi = rn(x), lo = rn(x - hi)
