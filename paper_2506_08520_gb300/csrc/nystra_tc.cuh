@@ -4,7 +4,9 @@
 // I/O (fp32 I/O through the operand policy Opnd<float>, used by the 8x8 pool
 // kernel).  Included by one translation unit per N (nystra_tc_n*.cu), which
 // also includes the kernel for its common case: nystra_pool.cuh (8x8, m <=
-// 16), nystra_team.cuh (16x16, m <= 32), nystra_stream.cuh (32x32, m <= 16).
+// 16), nystra_team.cuh (16x16, m <= 32), nystra_stream.cuh (32x32, m <= 32).
+// Compile-time options of those kernels: square-patch landmarks (Pooling,
+// PW > 0) and an additive score bias (BIAS, m <= 16).
 //
 // Phases of one (window, head) unit:
 //   stage    bulk copies of Q, K, V rows (contiguous in HBM) into shared
