@@ -36,13 +36,13 @@ METRIC = "Nystrom attention tokens*heads/s"
 # of those files changes.
 MEASURED_TRAFFIC = {
     "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
-                       "src_hash": "45318e4c874e1563", "bytes": 74_007_296},
+                       "src_hash": "18461915ec80da1f", "bytes": 73_978_880},
     "sr720p-w16-m16-bf16": {"files": ["common.cuh", "nystra_team.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu",
                                       "ptx.cuh"],
-                            "src_hash": "2f07d283f0f2609e", "bytes": 1_296_338_176},
+                            "src_hash": "db325f6b5b3db04f", "bytes": 1_296_579_840},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-                            "src_hash": "819a6737ed00b785", "bytes": 1_349_984_256},
+                            "src_hash": "c2f79d75bf44c177", "bytes": 1_351_302_656},
 }
 
 
