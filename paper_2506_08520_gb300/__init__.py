@@ -1,9 +1,18 @@
 """GB300-native (sm_103a) PnP-Nystra window attention.
 
-``nystra(q, k, v, m, iters)`` and ``exact(q, k, v)`` call the C-ABI CUDA
-library ``libnystra.so`` (see ``include/nystra.h``); ``workloads`` holds the
-seeded synthetic inputs.  The library is loaded on first use and every call
-fails loudly if it is missing: there is no CPU path.
+Device tensors ``[n_windows, heads, N, d_h]`` (fp32, bf16 or fp16)::
+
+    import paper_2506_08520_gb300 as pn
+    o = pn.nystra(q, k, v, m=16, iters=6)                      # segment landmarks
+    o = pn.nystra(q, k, v, m=16, iters=6, landmarks="patches") # square patches
+    pooled = pn.pool_bias(bias, m=16)                          # bias [heads, N, N] fp32, once
+    o = pn.nystra_biased(q, k, v, pooled, m=16, iters=6)       # with a score bias
+    e = pn.exact(q, k, v)                                      # exact window attention
+
+Every call goes through the C ABI of ``libnystra.so`` (``include/nystra.h``),
+loaded on first use; it fails loudly if the library is missing: there is no
+CPU path.  ``workloads`` holds the seeded synthetic inputs; ``sweep`` times
+them (``python -m paper_2506_08520_gb300.sweep``).
 """
 from .binding import (NystraError, check, debug_stages, debug_wait_timeout, exact, exact_window_attention,
                       nystra, nystra_attention, nystra_attention_bias, nystra_attention_ex, nystra_biased,
