@@ -26,7 +26,8 @@
  *           splits every operand into bf16 hi + lo (three products each).
  *           Shapes outside the tensor-core paths (odd d_h or d_h > 32, N not
  *           64/256/1024, m not 8/16/32/64, fp32 I/O with N != 64 or more than
- *           6 iterations) run in fp32 SIMT arithmetic.  The output is rounded
+ *           6 iterations, 16-bit I/O with more than 12) run in fp32 SIMT
+ *           arithmetic.  The output is rounded
  *           to nearest-even.  Against a float64 evaluation the max relative
  *           Frobenius error per unit is <= 1e-4 (fp32 I/O) and <= 2e-2 (16-bit
  *           I/O) at the paper's iteration counts.
@@ -227,7 +228,7 @@ NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stre
  *   O     N x d_h      the output (step 7), as rounded to the I/O type
  * `landmarks` is a nystra_landmarks value (square patches: 16-bit I/O, m = 16).
  * Supported: N = 64, m in {8, 16}, even d_h <= 32 (the shapes nystra_attention
- * runs on this path), fp32 I/O only with iters <= 6; anything else returns
+ * runs on this path: iters <= 12, and <= 6 for fp32 I/O); anything else returns
  * NYSTRA_EINVAL, as do unit outside [0, n_windows*heads), null or misaligned
  * pointers.  Asynchronous on `stream`; allocates nothing.  Returns NYSTRA_OK,
  * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.

@@ -78,8 +78,12 @@ int nystra_call(const void* q, const void* k, const void* v, void* out, int n_wi
     // iterations (beyond them the fp16-split iteration's round-off, amplified
     // by ||G_A^n|| ||Z||, exceeds what fp32 I/O asks; the SIMT path iterates in fp32).
     // Square patches on the tensor cores: 16-bit I/O with m = 16.
+    // 16-bit I/O on the tensor cores up to 12 iterations: their iteration
+    // carries X = A Z beside Z (one product per step fewer), and over many
+    // steps X drifts from A Z until the polynomial leaves its basin; the SIMT
+    // path forms X = A Z afresh every step.
     const bool io16 = dtype == NYSTRA_BF16 || dtype == NYSTRA_F16;
-    const bool tc16 = io16 && (patches ? m == 16 : (m == 8 || m == 16 || m == 32 || m == 64));
+    const bool tc16 = io16 && iters <= 12 && (patches ? m == 16 : (m == 8 || m == 16 || m == 32 || m == 64));
     const bool tc32 = !patches && dtype == NYSTRA_F32 && N == 64 && (m == 8 || m == 16) && iters <= 6;
     // A score bias on the tensor cores: the one-warp core, m <= 16.
     const bool biased = bias.L != nullptr;
@@ -205,7 +209,7 @@ int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windo
                         int m, int iters, int landmarks, int dtype, long long unit, float* dump, void* stream) {
     if (dtype != NYSTRA_F32 && dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;
     if (nystra_debug_stages_size(N, d_h, m) < 0) return NYSTRA_EINVAL;
-    if (iters < 0 || iters > NYSTRA_MAX_ITERS || (dtype == NYSTRA_F32 && iters > 6)) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > 12 || (dtype == NYSTRA_F32 && iters > 6)) return NYSTRA_EINVAL;
     // square patches: the 16-bit I/O path with m = 16 (2x2 patches)
     if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
     if (landmarks == NYSTRA_LANDMARKS_PATCHES && (m != 16 || dtype == NYSTRA_F32)) return NYSTRA_EINVAL;

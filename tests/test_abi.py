@@ -123,6 +123,7 @@ def test_debug_stages_size_rejects_other_shapes(lib, N, d, m):
     (dict(d=31), nb.NYSTRA_EINVAL),
     (dict(iters=-1), nb.NYSTRA_EINVAL),
     (dict(dtype=0, iters=7), nb.NYSTRA_EINVAL),  # fp32 runs this path up to 6 steps
+    (dict(iters=13), nb.NYSTRA_EINVAL),          # 16-bit up to 12
     (dict(unit=8), nb.NYSTRA_EINVAL),         # units are 0..7
     (dict(unit=-1), nb.NYSTRA_EINVAL),
     (dict(dump=0), nb.NYSTRA_EINVAL),

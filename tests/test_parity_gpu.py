@@ -232,3 +232,17 @@ def test_inputs_may_alias(N, d, m):
     assert torch.equal(a, b)
     if N <= 256:
         assert torch.equal(ea, eb)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16", "f16"])
+@pytest.mark.parametrize("N,d,m", [(64, 30, 16), (256, 30, 16), (1024, 30, 16), (256, 30, 32), (1024, 32, 32),
+                                   (64, 30, 64), (48, 20, 12)])
+def test_maximum_iteration_count_stays_finite(N, d, m, dtype):
+    # 100 steps (the limit): far past convergence, Z keeps inverting ever
+    # smaller singular values; the power-of-two rescaling of Z and Y must keep
+    # every path finite in every I/O type
+    q, k, v = (x.cuda() for x in workloads.random_qkv(3, N, d, dtype, seed=N + m))
+    out = binding.nystra(q, k, v, m, 100)
+    torch.cuda.synchronize()
+    assert binding.status() == binding.NYSTRA_OK
+    assert bool(torch.isfinite(out.float()).all())
