@@ -246,3 +246,16 @@ def test_maximum_iteration_count_stays_finite(N, d, m, dtype):
     torch.cuda.synchronize()
     assert binding.status() == binding.NYSTRA_OK
     assert bool(torch.isfinite(out.float()).all())
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f16"])
+@pytest.mark.parametrize("N,d,m", [(64, 30, 16), (256, 30, 16), (1024, 30, 16), (256, 30, 32)])
+def test_parity_holds_for_sharper_logits(N, d, m, dtype):
+    # Q, K scaled by 1.25: logit standard deviation 1.56 instead of 1.  The
+    # bar holds here; for much sharper attention G_A^n becomes so
+    # ill-conditioned that six iterations amplify any rounding of the landmarks
+    # and blocks (see the design notes' precision envelope).
+    q, k, v = workloads.random_qkv(8, N, d, "f32", seed=N + m + 5)
+    q, k, v = ((x * (1.25 if i < 2 else 1.0)).to(workloads.DTYPES[dtype]) for i, x in enumerate((q, k, v)))
+    err, worst = check_nystra(q, k, v, m, 6)
+    assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
