@@ -168,7 +168,9 @@ def test_exact_small(units, N, d, dtype):
     assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
 
 
-@pytest.mark.parametrize("name", ["swinir256-bf16", "large-w32-m32", "sr720p-w16-m16-bf16"])
+@pytest.mark.parametrize("name", ["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4",
+                                  "large-w16-m32", "large-w32-m32", "sr720p-w8-m16-bf16", "sr720p-w16-m16-bf16",
+                                  "sr720p-w32-m16-f16"])
 def test_exact_workloads(name):
     wl = workloads.WORKLOADS[name]
     q, k, v = workloads.make_qkv(wl)
@@ -259,3 +261,14 @@ def test_parity_holds_for_sharper_logits(N, d, m, dtype):
     q, k, v = ((x * (1.25 if i < 2 else 1.0)).to(workloads.DTYPES[dtype]) for i, x in enumerate((q, k, v)))
     err, worst = check_nystra(q, k, v, m, 6)
     assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+
+
+@pytest.mark.parametrize("N,d,m", [(64, 30, 16), (256, 30, 16), (1024, 30, 16), (256, 32, 64), (48, 20, 12)])
+def test_units_are_independent(N, d, m):
+    # every unit is computed on its own: permuting units permutes outputs, bit for bit
+    q, k, v = (x.cuda() for x in workloads.random_qkv(37, N, d, "bf16", seed=N + d))
+    perm = torch.randperm(37, generator=torch.Generator().manual_seed(1)).cuda()
+    a = binding.nystra(q, k, v, m, 6)
+    b = binding.nystra(q[perm].contiguous(), k[perm].contiguous(), v[perm].contiguous(), m, 6)
+    torch.cuda.synchronize()
+    assert torch.equal(a[perm], b)
