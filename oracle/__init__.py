@@ -167,3 +167,31 @@ def nystra_stages(q, k, v, m: int, iters: int, pool: str = "segments") -> dict:
         raise ValueError(f"oracle: invalid m={m} for N={N} with {pool} pooling")
     st["out"] = out
     return st
+
+
+def project_qkv(x, w_qkv, b_qkv, heads: int):
+    """The projections of Eq. (1), Q = X W_Q, K = X W_K, V = X W_V, for every
+    window, split into heads.  ``x``: ``[n_windows, N, C]`` tokens, C = heads*d.
+    ``w_qkv``: ``[3C, C]``, the transposes of W_Q, W_K, W_V stacked (row o holds
+    output feature o: the layout of a linear layer's weight), so Q[:, f] is
+    x @ w_qkv[f] and K, V take rows C + f and 2C + f.  ``b_qkv``: optional
+    ``[3C]`` bias of the restoration models' projection layers (Eq. (1) has
+    none).  Head h owns features h*d .. h*d + d - 1 of each.  Returns float64
+    q, k, v ``[n_windows, heads, N, d]``."""
+    x, w = _f64(x), _f64(w_qkv)
+    nw, N, C = x.shape
+    if C % heads or w.shape != (3 * C, C):
+        raise ValueError(f"oracle: w_qkv {w.shape} does not project C={C} for {heads} heads")
+    y = x @ w.T  # [nw, N, 3C]
+    if b_qkv is not None:
+        y = y + _f64(b_qkv)
+    y = y.reshape(nw, N, 3, heads, C // heads).transpose(2, 0, 3, 1, 4)
+    return tuple(np.ascontiguousarray(y[i]) for i in range(3))
+
+
+def nystra_attention_qkv(x, w_qkv, b_qkv, heads: int, m: int, iters: int, pool: str = "segments",
+                         bias=None) -> np.ndarray:
+    """PnP-Nystra of the projected tokens: project_qkv, then nystra_attention.
+    float64 ``[n_windows, heads, N, d]``."""
+    q, k, v = project_qkv(x, w_qkv, b_qkv, heads)
+    return nystra_attention(q, k, v, m, iters, pool, bias)

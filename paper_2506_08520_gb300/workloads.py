@@ -10,7 +10,8 @@ available, so each workload below is a synthetic stand-in with the same
 window geometry (8x8 / 16x16 / 32x32 windows), head count and head width.
 
 All tensors use the layout ``[n_windows, heads, N, d_h]`` (row-major,
-contiguous), tokens of a window in row-major spatial order.
+contiguous), tokens of a window in row-major spatial order; the tokens of the
+fused-projection workloads are ``[n_windows, N, heads*d_h]``.
 """
 from __future__ import annotations
 
@@ -37,6 +38,7 @@ class Workload:
     map_hw: tuple = ()   # (H, W, window) for recipe == "map"
     landmarks: str = "segments"  # landmark pooling: "segments" | "patches"
     bias: str = ""               # score bias: "" (none) | "relpos" (per-head relative-position bias)
+    front: str = ""              # "" (inputs are Q, K, V) | "qkv" (inputs are the tokens X and W_QKV)
 
     @property
     def units(self) -> int:
@@ -47,9 +49,18 @@ class Workload:
         return (self.n_windows, self.heads, self.N, self.d)
 
     @property
+    def C(self) -> int:
+        """Token width heads * d_h (the projections' input width)."""
+        return self.heads * self.d
+
+    @property
     def io_bytes(self) -> int:
-        """Q, K, V read once and O written once."""
-        return 4 * self.units * self.N * self.d * torch.tensor([], dtype=DTYPES[self.dtype]).element_size()
+        """Q, K, V read once and O written once; with the fused projection, X
+        and the weights read once and O written once."""
+        es = torch.tensor([], dtype=DTYPES[self.dtype]).element_size()
+        if self.front == "qkv":
+            return (2 * self.units * self.N * self.d + 3 * self.C * self.C) * es
+        return 4 * self.units * self.N * self.d * es
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
@@ -89,6 +100,10 @@ for _w in (8, 16, 32):
 for _name in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16"):
     WORKLOADS[_name + "-patches"] = WORKLOADS[_name].with_(name=_name + "-patches", landmarks="patches")
     WORKLOADS[_name + "-relpos"] = WORKLOADS[_name].with_(name=_name + "-relpos", bias="relpos")
+# The same windows given as tokens X and projection weights (fused Q/K/V projection).
+for _name in ("swinir256-bf16", "uformer-s1", "uformer-s4", "sr720p-w8-m16-bf16", "sr720p-w8-m16-f16",
+              "swinir256-bf16-relpos"):
+    WORKLOADS[_name + "-qkv"] = WORKLOADS[_name].with_(name=_name + "-qkv", front="qkv")
 
 
 def _cast(x: np.ndarray, dtype: str) -> torch.Tensor:
@@ -157,6 +172,42 @@ def make_qkv(wl: Workload | str):
     if isinstance(wl, str):
         wl = WORKLOADS[wl]
     return tuple(_cast(x, wl.dtype) for x in _RECIPES[wl.recipe](wl))
+
+
+def _tokens_and_weights(wl: Workload):
+    """Float64 tokens X ``[n_windows, N, C]`` and weights ``[3C, C]`` (row o is
+    output feature o: the Q, K, V weights transposed and stacked).  The "proj"
+    recipe returns the very draws ``_proj`` multiplies; the others draw X (an
+    edge-padded feature map for "map") and W ~ N(0, 1/C)."""
+    C = wl.C
+    rng = np.random.default_rng(wl.seed)
+    if wl.recipe == "map":
+        H, W, window = wl.map_hw
+        X = _partition(rng.standard_normal((1, H, W, C), dtype=np.float32), window)[:, 0]
+    else:
+        X = rng.standard_normal((wl.n_windows * wl.N, C)).reshape(wl.n_windows, wl.N, C)
+    Ws = [rng.standard_normal((C, C)) / np.sqrt(C) for _ in range(3)]
+    return X, np.concatenate([Wt.T for Wt in Ws], axis=0)
+
+
+def make_x_wqkv(wl: Workload | str):
+    """Seeded host tensors (x ``[n_windows, N, C]``, w_qkv ``[3C, C]``) in the
+    workload's I/O dtype, for the fused projection."""
+    if isinstance(wl, str):
+        wl = WORKLOADS[wl]
+    return tuple(_cast(a, wl.dtype) for a in _tokens_and_weights(wl))
+
+
+def random_x_wqkv(n_windows: int, N: int, heads: int, d: int, dtype: str = "bf16", seed: int = 0,
+                  with_bias: bool = True):
+    """i.i.d. tokens N(0, 1), weights N(0, 1/C) and (optionally) an fp32 bias
+    N(0, 0.1^2) for small parity and edge cases of the fused projection."""
+    rng = np.random.default_rng(seed)
+    C = heads * d
+    x = _cast(rng.standard_normal((n_windows, N, C)), dtype)
+    w = _cast(rng.standard_normal((3 * C, C)) / np.sqrt(C), dtype)
+    b = torch.from_numpy(0.1 * rng.standard_normal(3 * C)).float() if with_bias else None
+    return x, w, b
 
 
 def random_qkv(n_units: int, N: int, d: int, dtype: str = "f32", seed: int = 0, scale: float = 1.0):

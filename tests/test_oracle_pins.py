@@ -495,3 +495,74 @@ def test_block_constant_bias_exact_recovery():
     assert _rel(oracle.nystra_attention(q[None], k[None], v[None], m, 80, "segments", B), ref) < 1e-8
     # the bias matters: dropping it moves the output
     assert _rel(oracle.nystra_attention(q[None], k[None], v[None], m, 80), ref) > 1e-3
+
+
+# --------------------------------------------------------------------------
+# The projections of Eq. (1) (the fused Q/K/V front end).
+# --------------------------------------------------------------------------
+def _perm_weights(rng, C):
+    perms = [rng.permutation(C) for _ in range(3)]
+    w = np.zeros((3 * C, C))
+    for i, p in enumerate(perms):
+        w[i * C + np.arange(C), p] = 1.0
+    return w, perms
+
+
+def test_projection_with_permutation_weights_gathers_columns():
+    """Row o of w_qkv holding a single 1 at column p[o] makes output feature o
+    the token feature p[o], exactly: this fixes which of w or its transpose
+    multiplies, the Q/K/V order of the stacked rows and the head split."""
+    rng = _rng(60)
+    nw, N, heads, d = 3, 16, 3, 4
+    C = heads * d
+    x = rng.standard_normal((nw, N, C))
+    w, perms = _perm_weights(rng, C)
+    for got, p in zip(oracle.project_qkv(x, w, None, heads), perms):
+        for h in range(heads):
+            np.testing.assert_array_equal(got[:, h], x[:, :, p[h * d:(h + 1) * d]])
+
+
+def test_projection_bias_only_gives_the_value_bias():
+    """W = 0: every token of a window projects to the bias, all scores are
+    equal, and attention of identical values returns that value; the Nystrom
+    blocks are all-ones, whose pseudo-inverse J/m^2 the iteration starts at and
+    keeps.  So O = b_V's head slice exactly, for any m, pooling and iteration count."""
+    rng = _rng(61)
+    nw, N, heads, d = 2, 64, 2, 6
+    C = heads * d
+    x = rng.standard_normal((nw, N, C))
+    b = rng.standard_normal(3 * C)
+    want = np.broadcast_to(b[2 * C:].reshape(heads, 1, d), (nw, heads, N, d))
+    for m, pool, iters in ((16, "segments", 6), (4, "patches", 3), (64, "segments", 0)):
+        out = oracle.nystra_attention_qkv(x, np.zeros((3 * C, C)), b, heads, m, iters, pool)
+        np.testing.assert_allclose(out, want, rtol=1e-12, atol=1e-12)
+
+
+def test_projection_scaled_identities_reduce_to_split_heads():
+    """w_qkv = [I; 2I; -I] makes Q, 2Q, -Q the heads of x itself (a reshape,
+    no arithmetic), so the fused result is PnP-Nystra of those slices."""
+    rng = _rng(62)
+    nw, N, heads, d = 2, 64, 3, 8
+    C = heads * d
+    x = rng.standard_normal((nw, N, C))
+    I = np.eye(C)
+    xs = x.reshape(nw, N, heads, d).transpose(0, 2, 1, 3)
+    got = oracle.nystra_attention_qkv(x, np.vstack([I, 2 * I, -I]), None, heads, 16, 6)
+    np.testing.assert_allclose(got, oracle.nystra_attention(xs, 2 * xs, -xs, 16, 6), rtol=0, atol=1e-13)
+
+
+def test_projection_reproduces_the_projected_workload_recipe():
+    """The fused-projection workload hands the oracle the very draws the
+    SwinIR-like recipe multiplies (Q, K, V = X W with W [in, out]), so its
+    projections equal that recipe's Q, K, V."""
+    wl = workloads.WORKLOADS["swinir256-bf16"].with_(n_windows=3)
+    X, W = workloads._tokens_and_weights(wl)
+    for got, ref in zip(oracle.project_qkv(X, W, None, wl.heads), workloads._proj(wl)):
+        np.testing.assert_allclose(got, ref, rtol=0, atol=1e-12)
+
+
+def test_projection_shapes_are_checked():
+    with pytest.raises(ValueError):
+        oracle.project_qkv(np.zeros((1, 4, 6)), np.zeros((18, 4)), None, 3)
+    with pytest.raises(ValueError):
+        oracle.project_qkv(np.zeros((1, 4, 6)), np.zeros((18, 6)), None, 4)
