@@ -3,7 +3,9 @@
 One step = one ``nystra_attention`` call over the whole batch of the workload
 (default: SwinIR-like denoising at 256x256 -- 1024 windows of 8x8 tokens,
 6 heads, d_h = 30, m = 16 landmarks, 6 pseudo-inverse iterations, bf16 I/O).
-Prints ONE JSON line (rank 0).  Metric: tokens*heads per second.
+Prints ONE JSON line (rank 0).  Metric: tokens*heads per second.  A "-qkv"
+workload times the fused Q/K/V projection front end instead (one
+``nystra_attention_qkv`` call; tensor roofline, unfused path as comparator).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the float64 CPU oracle, host cores
@@ -135,11 +137,23 @@ def _oracle_bias(wl, lo: int, hi: int):
     return bias.double().numpy()[np.arange(lo, hi) % wl.heads]
 
 
-def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
-    """Time the float64 oracle on a bounded sample of the workload's units."""
+def _oracle_inputs(wl):
+    """Host float64 (q, k, v) ``[units, N, d]`` the oracle times; for a fused
+    front end the oracle's own projections of the workload's tokens."""
     import oracle  # CPU baseline only
-    qu, ku, vu = (x.reshape(-1, wl.N, wl.d) for x in (q, k, v))
-    qd, kd, vd = (x.double().numpy() for x in (qu, ku, vu))
+    if wl.front == "qkv":
+        x, w = workloads.make_x_wqkv(wl)
+        q, k, v = oracle.project_qkv(x, w, None, wl.heads)
+        return tuple(a.reshape(-1, wl.N, wl.d) for a in (q, k, v))
+    return tuple(x.reshape(-1, wl.N, wl.d).double().numpy() for x in workloads.make_qkv(wl))
+
+
+def _time_oracle(wl, q, k, v, budget_s: float, max_units: int | None = None):
+    """Time the float64 oracle on a bounded sample of the workload's units
+    (q, k, v: float64 ``[units, N, d]``; a fused front end's projections are
+    made outside the timed region)."""
+    import oracle  # CPU baseline only
+    qd, kd, vd = q, k, v
     # calibrate on a few units, then size the sample to the budget
     n0 = min(64, qd.shape[0])
     t0 = time.perf_counter()
@@ -168,24 +182,47 @@ def _l2_bytes() -> int:
 def _config(wl, ws: int):
     """The `config` object both arms report: the workload and how the timed
     launches avoid L2 residency (rotating input/output sets > 3x L2)."""
-    io_bytes = 4 * wl.units * wl.N * wl.d * {"f32": 4, "bf16": 2, "f16": 2}[wl.dtype]
+    io_bytes = wl.io_bytes
     nsets = max(2, -(-3 * _l2_bytes() // io_bytes))
-    return nsets, io_bytes, {
+    cfg = {
         "workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N, "d_h": wl.d, "m": wl.m,
         "iters": wl.iters, "io_dtype": wl.dtype, "landmarks": wl.landmarks, "bias": wl.bias or "none",
         "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
         "parallelism": f"replica x{ws} (independent windows)"}
+    if wl.front == "qkv":
+        cfg["front"] = "fused Q/K/V projection (tokens and W_QKV in)"
+    return nsets, io_bytes, cfg
+
+
+def unit_flops(wl) -> int:
+    """Algorithmic flops of one (window, head) unit: the products of the
+    method (S_L, S_U, S_A, W = G_U^n [V | 1], the iteration's four m x m
+    products per step, Y = Z W, O = G_L^n Y), the landmark sums and, for a
+    fused front end, the unit's share of the projection (2 N C 3 d_h)."""
+    N, d, m = wl.N, wl.d, wl.m
+    f = (2 * N * m * d + 2 * m * N * d + 2 * m * m * d + 2 * m * N * (d + 1) + 8 * wl.iters * m ** 3
+         + 2 * m * m * (d + 1) + 2 * N * m * (d + 1) + 2 * N * d)
+    if wl.front == "qkv":
+        f += 2 * N * wl.C * 3 * d
+    return f
+
+
+def _tensor_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
 
 
 def run_reference(args, wl):
     ws, rank, _ = _dist()
     if rank != 0:
         return
-    q, k, v = workloads.make_qkv(wl)
     import oracle
     # per-step sample sized so that warmup+steps fit in about a minute
     per_step_budget = max(0.002, 60.0 / max(1, args.steps + args.warmup))
-    qd, kd, vd = (x.reshape(-1, wl.N, wl.d).double().numpy() for x in (q, k, v))
+    qd, kd, vd = _oracle_inputs(wl)
     n0 = min(32, qd.shape[0])
     t0 = time.perf_counter()
     oracle.nystra_attention(qd[:n0], kd[:n0], vd[:n0], wl.m, wl.iters, wl.landmarks, _oracle_bias(wl, 0, n0))
@@ -207,7 +244,8 @@ def run_reference(args, wl):
         "data": "synthetic",
         "config": _config(wl, ws)[2],
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.threads(), "kind": "oracle",
-                         "sample": f"{n} of {qd.shape[0]} units per step (float64 C oracle, OpenMP)"},
+                         "sample": f"{n} of {qd.shape[0]} units per step (float64 C oracle, OpenMP"
+                                   + ("; projections made beforehand)" if wl.front == "qkv" else ")")},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -346,10 +384,150 @@ def run_cuda(args, wl):
         "clocks": clk.summary(),
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
-        val, n, passes, dt, cores = _time_oracle(wl, q, k, v, budget_s=args.cpu_budget)
+        val, n, passes, dt, cores = _time_oracle(wl, *_oracle_inputs(wl), budget_s=args.cpu_budget)
         line["cpu_baseline"] = {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle",
                                 "sample": f"{n} of {wl.units} units x {passes} passes, {dt:.1f} s "
                                           "(float64 C oracle, OpenMP)"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+
+
+def run_cuda_qkv(args, wl):
+    """One step = one nystra_attention_qkv call: the window tokens and W_QKV in,
+    the projections of Eq. (1) and PnP-Nystra fused.  Its comparator is the
+    unfused path it replaces (cuBLAS projection, head split, nystra_attention)."""
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    binding.lib()  # fail loudly if the library is missing
+
+    x, w = workloads.make_x_wqkv(wl)
+    esize = x.element_size()
+    nsets, io_bytes, config = _config(wl, ws)
+    assert io_bytes == (2 * x.numel() + w.numel()) * esize
+    wd = w.to(dev)  # a model constant: resident
+    sets = [(x.to(dev), torch.empty(wl.shape, dtype=x.dtype, device=dev)) for _ in range(nsets)]
+    stream = torch.cuda.current_stream(dev)
+    sptr = stream.cuda_stream
+    bias = workloads.make_bias(wl)
+    pooled = None if bias is None else binding.pool_bias(bias.to(dev), wl.m, wl.landmarks)
+    bp = (0, 0, 0) if pooled is None else tuple(t.data_ptr() for t in pooled)
+    dcode = {"bf16": 1, "f16": 2}[wl.dtype]
+
+    def step(i):
+        xd, od = sets[i % nsets]
+        rc = binding.nystra_attention_qkv(xd.data_ptr(), wd.data_ptr(), 0, od.data_ptr(), wl.n_windows, wl.heads,
+                                          wl.N, wl.d, wl.m, wl.iters, binding.LANDMARKS[wl.landmarks], *bp,
+                                          1 if pooled is not None else 0, dcode, sptr)
+        if rc != 0:
+            raise binding.NystraError(rc, "bench step")
+
+    def unfused_step(i):
+        xd, od = sets[i % nsets]
+        y = xd.reshape(-1, wl.C) @ wd.T
+        q, k, v = (y.view(wl.n_windows, wl.N, 3, wl.heads, wl.d)[:, :, j].transpose(1, 2).contiguous()
+                   for j in range(3))
+        if pooled is None:
+            binding.nystra(q, k, v, wl.m, wl.iters, out=od, landmarks=wl.landmarks)
+        else:
+            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=od, landmarks=wl.landmarks)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
+
+    for i in range(args.warmup):
+        step(i)
+    barrier()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        barrier()
+        for i in range(args.steps):
+            starts[i].record(stream)
+            step(i)
+            ends[i].record(stream)
+        barrier()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    kern_ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
+    total_ms = shard.max_over_ranks(total_ms, dev)
+    units_tokens = wl.units * wl.N
+    value = shard.aggregate_rate(units_tokens, args.steps, total_ms, ws)
+
+    usteps = max(3, min(args.steps, 100))
+    for i in range(3):
+        unfused_step(i)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for i in range(usteps):
+        unfused_step(i)
+    e1.record(stream)
+    barrier()
+    unfused_ms = e0.elapsed_time(e1) / usteps
+
+    # End to end: every step copies its tokens from pinned host memory and
+    # reads the output back (the weights are a resident model constant).
+    hx = x.pin_memory()
+    hos = [torch.empty(wl.shape, dtype=x.dtype).pin_memory() for _ in range(2)]
+    streams = [torch.cuda.Stream(dev) for _ in range(2)]
+
+    def e2e_step(i):
+        xd, od = sets[i % 2]
+        with torch.cuda.stream(streams[i % 2]):
+            xd.copy_(hx, non_blocking=True)
+            binding.nystra_qkv(xd, wd, wl.heads, wl.m, wl.iters, pooled=pooled, out=od, landmarks=wl.landmarks)
+            hos[i % 2].copy_(od, non_blocking=True)
+
+    e2e_steps = max(4, min(args.steps, 50))
+    for i in range(2):
+        e2e_step(i)
+    barrier()
+    e0.record(streams[0])
+    streams[1].wait_event(e0)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    done1 = torch.cuda.Event()
+    done1.record(streams[1])
+    streams[0].wait_event(done1)
+    e1.record(streams[0])
+    barrier()
+    e2e_ms = shard.max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dev)
+    e2e_value = shard.aggregate_rate(units_tokens, 1, e2e_ms, ws)
+
+    peak, peak_kind = _tensor_peak()
+    flops = unit_flops(wl) * wl.units
+    achieved = flops / (kern_ms * 1e-3) / 1e12
+    mt = MEASURED_TRAFFIC.get(wl.name)
+    traffic = mt["bytes"] if mt and mt["src_hash"] == _kernel_src_hash(mt["files"]) else None
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": config,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "flops_per_launch": flops, "bytes_per_launch": io_bytes, "kernel_ms": kern_ms,
+                     "hbm_GBps": io_bytes / (kern_ms * 1e-3) / 1e9},
+        "comparator": {"kernel": "cuBLAS projection + head split + nystra_attention", "ms_per_step": unfused_ms,
+                       "value": units_tokens / (unfused_ms * 1e-3), "speedup": unfused_ms / (total_ms / args.steps)},
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": x.numel() * esize,
+                "d2h_bytes_per_step": x.numel() * esize, "streams": 2},
+        "gpu_launches": args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        val, n, passes, dt, cores = _time_oracle(wl, *_oracle_inputs(wl), budget_s=args.cpu_budget)
+        line["cpu_baseline"] = {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle",
+                                "sample": f"{n} of {wl.units} units x {passes} passes, {dt:.1f} s "
+                                          "(float64 C oracle, OpenMP; projections made beforehand)"}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if ws > 1:
@@ -371,6 +549,8 @@ def main():
     wl = workloads.WORKLOADS[args.workload]
     if args.impl == "reference":
         run_reference(args, wl)
+    elif wl.front == "qkv":
+        run_cuda_qkv(args, wl)
     else:
         run_cuda(args, wl)
 

@@ -168,6 +168,40 @@ NYSTRA_API int nystra_attention_bias(const void* q, const void* k, const void* v
                                      int bias_windows, int dtype, void* stream);
 
 /*
+ * nystra_attention_qkv -- the projections of Eq. (1) fused with PnP-Nystra:
+ * per window, Q = X W_Q, K = X W_K, V = X W_V (+ an optional projection
+ * bias, which the restoration models' layers add and Eq. (1) omits), split
+ * into heads of d_h features, then nystra_attention_ex on every (window,
+ * head) unit.  Q, K and V stay on chip: the call reads the tokens and the
+ * weights instead of Q, K and V.
+ *
+ * Arguments
+ *  x       [n_windows, N, C] tokens, C = heads * d_h, each window's tokens in
+ *          the order nystra_attention_ex pools them (device, caller-owned).
+ *  w_qkv   [3C, C]: row o holds the weights of output feature o, rows 0..C-1
+ *          for Q, C..2C-1 for K, 2C..3C-1 for V (the transposes of W_Q, W_K,
+ *          W_V stacked: the layout of a linear layer's weight); head h owns
+ *          features h*d_h .. h*d_h + d_h - 1 of each.  Same dtype as x.
+ *  b_qkv   [3C] fp32 projection bias, or NULL for none.
+ *  out     [n_windows, heads, N, d_h] output, as nystra_attention writes it.
+ *  bias_L, bias_U, bias_A, bias_windows   an optional pooled score bias as for
+ *          nystra_attention_bias; bias_L == NULL for none.
+ *  Other arguments as nystra_attention_ex.
+ * The projected Q, K, V are rounded to the I/O type before the attention, as
+ * an unfused projection would store them.  Supported: 16-bit I/O (fp32 returns
+ * NYSTRA_EDTYPE), N = 64, m in {8, 16} (square patches: m = 16), even
+ * d_h <= 32, C <= NYSTRA_QKV_MAX_C, iters <= 12; anything else returns
+ * NYSTRA_EINVAL, as do null (other than b_qkv and the bias) or not 16-byte
+ * aligned pointers and an out that overlaps an input.  Returns NYSTRA_OK,
+ * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.
+ */
+#define NYSTRA_QKV_MAX_C 352
+NYSTRA_API int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, void* out,
+                                    int n_windows, int heads, int N, int d_h, int m, int iters, int landmarks,
+                                    const float* bias_L, const float* bias_U, const float* bias_A,
+                                    int bias_windows, int dtype, void* stream);
+
+/*
  * exact_window_attention -- exact softmax attention per unit, Eq. (1):
  * O = softmax(Q K^T / sqrt(d_h)) V with row-max-shifted exponentials
  * (Eq. 2).  This is the computation PnP-Nystra replaces; it serves as the

@@ -19,6 +19,7 @@ NYSTRA_OK, NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH, NYSTRA_ETIMEOUT, NYSTRA
 NYSTRA_LANDMARKS_SEGMENTS, NYSTRA_LANDMARKS_PATCHES = 0, 1
 LANDMARKS = {"segments": NYSTRA_LANDMARKS_SEGMENTS, "patches": NYSTRA_LANDMARKS_PATCHES}
 MAX_N, MAX_DH, MAX_M, MAX_ITERS = 1024, 64, 64, 100
+QKV_MAX_C = 352
 
 _DTYPE_CODE = {torch.float32: NYSTRA_F32, torch.bfloat16: NYSTRA_BF16, torch.float16: NYSTRA_F16}
 
@@ -64,6 +65,8 @@ def lib() -> ctypes.CDLL:
         L.nystra_pool_bias.restype = i
         L.nystra_attention_bias.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i, vp]
         L.nystra_attention_bias.restype = i
+        L.nystra_attention_qkv.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i, vp]
+        L.nystra_attention_qkv.restype = i
         L.nystra_debug_stages.restype = i
         L.nystra_debug_stages_size.argtypes = [i, i, i]
         L.nystra_debug_stages_size.restype = ctypes.c_longlong
@@ -90,6 +93,12 @@ def nystra_attention_bias(q, k, v, out, n_windows, heads, N, d_h, m, iters, land
                           bias_windows, dtype, stream) -> int:
     return lib().nystra_attention_bias(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L, bias_U,
                                        bias_A, bias_windows, dtype, stream)
+
+
+def nystra_attention_qkv(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L, bias_U,
+                         bias_A, bias_windows, dtype, stream) -> int:
+    return lib().nystra_attention_qkv(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L,
+                                      bias_U, bias_A, bias_windows, dtype, stream)
 
 
 def exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream) -> int:
@@ -259,4 +268,45 @@ def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: 
                                    _DTYPE_CODE[q.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention_bias")
+    return out
+
+
+def nystra_qkv(x: torch.Tensor, w_qkv: torch.Tensor, heads: int, m: int = 16, iters: int = 6,
+               b_qkv: torch.Tensor | None = None, pooled=None, out: torch.Tensor | None = None, stream=None,
+               landmarks: str = "segments") -> torch.Tensor:
+    """Fused projection + PnP-Nystra: tokens ``x`` ``[n_windows, N, C]``, weights
+    ``w_qkv`` ``[3C, C]`` (a linear layer's weight: Q rows, then K, then V),
+    optional fp32 bias ``b_qkv`` ``[3C]`` and pooled score bias (as for
+    ``nystra_biased``).  Returns ``[n_windows, heads, N, C / heads]``."""
+    if x.dim() != 3 or w_qkv.dim() != 2:
+        raise ValueError("expected x [n_windows, N, C] and w_qkv [3C, C]")
+    nw, N, C = x.shape
+    if heads < 1 or C % heads:
+        raise ValueError(f"C={C} does not split into {heads} heads")
+    d = C // heads
+    if tuple(w_qkv.shape) != (3 * C, C):
+        raise ValueError(f"w_qkv must be [{3 * C}, {C}]")
+    out = torch.empty((nw, heads, N, d), dtype=x.dtype, device=x.device) if out is None else out
+    for t in (x, w_qkv, out):
+        if not t.is_cuda or not t.is_contiguous() or t.dtype != x.dtype:
+            raise ValueError("x, w_qkv and out must be contiguous CUDA tensors of one dtype (no CPU path)")
+    if x.dtype not in _DTYPE_CODE:
+        raise ValueError(f"unsupported dtype {x.dtype}")
+    if tuple(out.shape) != (nw, heads, N, d):
+        raise ValueError(f"out must be [{nw}, {heads}, {N}, {d}]")
+    bp = 0
+    if b_qkv is not None:
+        if not b_qkv.is_cuda or b_qkv.dtype != torch.float32 or not b_qkv.is_contiguous() or b_qkv.numel() != 3 * C:
+            raise ValueError(f"b_qkv must be a contiguous fp32 CUDA tensor of {3 * C} values")
+        bp = b_qkv.data_ptr()
+    bL = bU = bA = 0
+    bw = 0
+    if pooled is not None:
+        bL, bU, bA = (t.data_ptr() for t in pooled)
+        bw = pooled[0].numel() // (heads * N * m)
+    with torch.cuda.device(x.device):
+        rc = nystra_attention_qkv(x.data_ptr(), w_qkv.data_ptr(), bp, out.data_ptr(), nw, heads, N, d, m, iters,
+                                  LANDMARKS[landmarks], bL, bU, bA, bw, _DTYPE_CODE[x.dtype], _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_attention_qkv")
     return out

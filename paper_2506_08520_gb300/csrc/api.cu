@@ -52,10 +52,6 @@ int exact_sqrt(int n) {
 
 }  // namespace
 
-extern "C" {
-
-}  // extern "C"
-
 namespace {
 
 // The body of every PnP-Nystra entry point; bias.L == nullptr: no bias.
@@ -160,6 +156,48 @@ int nystra_attention(const void* q, const void* k, const void* v, void* out, int
                      int N, int d_h, int m, int iters, int dtype, void* stream) {
     return nystra_attention_ex(q, k, v, out, n_windows, heads, N, d_h, m, iters, NYSTRA_LANDMARKS_SEGMENTS,
                                dtype, stream);
+}
+
+int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, void* out, int n_windows, int heads,
+                         int N, int d_h, int m, int iters, int landmarks, const float* bias_L, const float* bias_U,
+                         const float* bias_A, int bias_windows, int dtype, void* stream) {
+    if (dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;  // 16-bit I/O only
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (N != 64 || d_h < 2 || d_h > 32 || d_h % 2 != 0 || (m != 8 && m != 16)) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > 12) return NYSTRA_EINVAL;
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
+    if (landmarks == NYSTRA_LANDMARKS_PATCHES && m != 16) return NYSTRA_EINVAL;
+    if ((long long)heads * d_h > NYSTRA_QKV_MAX_C) return NYSTRA_EINVAL;
+    if ((long long)n_windows * heads == 0) return NYSTRA_OK;
+    const size_t C = (size_t)heads * d_h;
+    const size_t xb = (size_t)n_windows * N * C * 2, wb = 3 * C * C * 2, ob = xb;
+    if (!x || !w_qkv || !out) return NYSTRA_EINVAL;
+    if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(out) || (b_qkv && !aligned16(b_qkv))) return NYSTRA_EINVAL;
+    if (overlaps2(out, ob, x, xb) || overlaps2(out, ob, w_qkv, wb) || (b_qkv && overlaps2(out, ob, b_qkv, 3 * C * 4)))
+        return NYSTRA_EINVAL;
+    nystra::NystraBias b;
+    if (bias_L) {
+        if (bias_windows != 1 && bias_windows != n_windows) return NYSTRA_EINVAL;
+        if (!bias_U || !bias_A) return NYSTRA_EINVAL;
+        if (!aligned16(bias_L) || !aligned16(bias_U) || !aligned16(bias_A)) return NYSTRA_EINVAL;
+        const size_t nm = (size_t)bias_windows * heads * N * m * 4, mm = (size_t)bias_windows * heads * m * m * 4;
+        if (overlaps2(out, ob, bias_L, nm) || overlaps2(out, ob, bias_U, nm) || overlaps2(out, ob, bias_A, mm))
+            return NYSTRA_EINVAL;
+        b.L = bias_L;
+        b.U = bias_U;
+        b.A = bias_A;
+        b.heads = heads;
+        b.per_window = bias_windows != 1 ? 1 : 0;
+    }
+    const nystra::NystraBias* bp = bias_L ? &b : nullptr;
+    const int pool = landmarks == NYSTRA_LANDMARKS_PATCHES ? 1 : 0;
+    const cudaError_t e =
+        dtype == NYSTRA_BF16
+            ? nystra_host::launch_nystra_qkv_bf16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
+                                                  (cudaStream_t)stream, bp)
+            : nystra_host::launch_nystra_qkv_f16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
+                                                 (cudaStream_t)stream, bp);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
 int exact_window_attention(const void* q, const void* k, const void* v, void* out, int n_windows,

@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace nystra {
 
 // Element I/O: 16-bit inputs are widened exactly; outputs are rounded to
@@ -34,6 +36,32 @@ struct NystraBias {
     int heads = 1;
     int per_window = 0;
 };
+
+// Persistent grid size of `kern` on the current device: SMs x CTAs resident
+// at `smem` bytes of dynamic shared memory, after opting the kernel in to that
+// much.  Both are per device, so both are cached per device ordinal in
+// `cache` (a zero-initialised static of the launcher).
+constexpr int kMaxDevices = 64;
+template <typename K>
+cudaError_t persistent_grid(K kern, int threads, size_t smem, std::atomic<int> (&cache)[kMaxDevices], int* blocks) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+    int b = cache[dev].load(std::memory_order_relaxed);
+    if (b == 0) {
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+            return e;
+        int sms = 0, per_sm = 0;
+        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem)) != cudaSuccess) return e;
+        if (per_sm < 1) return cudaErrorInvalidConfiguration;
+        b = sms * per_sm;
+        cache[dev].store(b, std::memory_order_relaxed);
+    }
+    *blocks = b;
+    return cudaSuccess;
+}
 
 }  // namespace nystra
 
@@ -74,6 +102,14 @@ unsigned int take_fault_word_exact_tc(cudaError_t* err);
 // units whose kernels wait on barriers: OR-ed together, then cleared.
 unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err);
 cudaError_t launch_debug_wait(unsigned long long limit_ns, cudaStream_t stream);
+// Fused Q/K/V projection + PnP-Nystra, 8x8 windows, m in {8, 16} (square
+// patches: m = 16), even d_h <= 32, heads * d_h <= 352 (nystra_qkv_*.cu).
+cudaError_t launch_nystra_qkv_bf16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                   long long n_windows, int heads, int d, int m, int iters, int pool,
+                                   cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkv_f16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                  long long n_windows, int heads, int d, int m, int iters, int pool,
+                                  cudaStream_t stream, const nystra::NystraBias* bias);
 // Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
 long long debug_stages_size(int N, int d, int m);
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,

@@ -194,21 +194,12 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
     static_assert(kGroups >= 1, "does not fit");
     auto kern = exact_tc_kernel<T, NCOL, WPU, kGroups>;
     const size_t smem = (size_t)kGroups * Lay::PER_GROUP;
-    static int s_blocks = 0;
-    if (s_blocks == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        int dev = 0, sms = 0, per_sm = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGroups * WPU * 32, smem)) !=
-            cudaSuccess)
-            return e;
-        if (per_sm < 1) return cudaErrorInvalidConfiguration;
-        s_blocks = sms * per_sm;
-    }
+    static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device
+    int blocks = 0;
+    if (cudaError_t e = persistent_grid(kern, kGroups * WPU * 32, smem, s_blocks, &blocks); e != cudaSuccess)
+        return e;
     const long long want = (n_units + kGroups - 1) / kGroups;
-    const long long grid = want < s_blocks ? want : s_blocks;
+    const long long grid = want < blocks ? want : blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, kGroups * WPU * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                               n_units, d, sl2, fault);

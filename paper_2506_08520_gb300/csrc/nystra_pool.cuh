@@ -177,19 +177,11 @@ cudaError_t launch_pool_dc(const void* q, const void* k, const void* v, void* ou
                         int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
     using P = PoolLayout<T, M, NCOL>;
     auto kern = nystra_pool_kernel<T, M, NCOL, DC, PW, BIAS>;
-    static int s_blocks = 0;  // persistent grid size, set on first use
-    if (s_blocks == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
-        if (e != cudaSuccess) return e;
-        int dev = 0, sms = 0, per_sm = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, P::NW * 32, P::BYTES)) != cudaSuccess)
-            return e;
-        if (per_sm < 1) return cudaErrorInvalidConfiguration;
-        s_blocks = sms * per_sm;
-    }
-    const long long grid = n_units < s_blocks ? n_units : s_blocks;
+    static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device
+    int blocks = 0;
+    if (cudaError_t e = persistent_grid(kern, P::NW * 32, P::BYTES, s_blocks, &blocks); e != cudaSuccess)
+        return e;
+    const long long grid = n_units < blocks ? n_units : blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, P::NW * 32, P::BYTES, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                              n_units, d, iters, sl2, fault, bias);

@@ -1622,23 +1622,13 @@ cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, l
     using Lay = Layout<M, NCOL, TPW, WPU, kGls, CW>;
     auto kern = nystra_tc_kernel<T, M, NCOL, TPW, WPU, kGroups, kGls, CW>;
     const size_t smem = (size_t)kGroups * Lay::PER_GROUP;
-    static int s_blocks = 0;  // persistent grid size, set on first use
-    if (s_blocks == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        int dev = 0, sms = 0, per_sm = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kGroups * Lay::GW * 32, smem)) !=
-            cudaSuccess)
-            return e;
-        if (per_sm < 1) return cudaErrorInvalidConfiguration;
-        s_blocks = sms * per_sm;
-    }
+    static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device
+    int blocks = 0;
+    if (cudaError_t e = persistent_grid(kern, kGroups * Lay::GW * 32, smem, s_blocks, &blocks); e != cudaSuccess)
+        return e;
     // Wave quantisation: every group processes ceil(units / groups) units, so
     // use the fewest groups per CTA that still reach the minimal number of
     // rounds (fewer co-resident groups contend less for the SM).
-    const long long blocks = s_blocks;
     const long long rounds = (n_units + blocks * kGroups - 1) / (blocks * kGroups);
     int active = (int)((n_units + blocks * rounds - 1) / (blocks * rounds));
     active = active < 1 ? 1 : (active > kGroups ? kGroups : active);

@@ -306,21 +306,12 @@ cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* ou
     using Lay = TeamLayout<M, NCOL>;
     auto kern = nystra_team_kernel<T, M, NCOL, DC, PW, BIAS>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
-    static int s_blocks = 0;  // persistent grid size, set on first use
-    if (s_blocks == 0) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        int dev = 0, sms = 0, per_sm = 0;
-        if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
-        if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, Lay::TEAMS * Lay::WARPS * 32, smem)) !=
-            cudaSuccess)
-            return e;
-        if (per_sm < 1) return cudaErrorInvalidConfiguration;
-        s_blocks = sms * per_sm;
-    }
+    static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device
+    int blocks = 0;
+    if (cudaError_t e = persistent_grid(kern, Lay::TEAMS * Lay::WARPS * 32, smem, s_blocks, &blocks); e != cudaSuccess)
+        return e;
     const long long want = (n_units + Lay::TEAMS - 1) / Lay::TEAMS;
-    const long long grid = want < s_blocks ? want : s_blocks;
+    const long long grid = want < blocks ? want : blocks;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, Lay::TEAMS * Lay::WARPS * 32, smem, stream>>>((const T*)q, (const T*)k, (const T*)v, (T*)out,
                                                                  n_units, d, iters, sl2, fault, bias);

@@ -11,7 +11,10 @@ tokens*heads/s (for edge-padded maps also counting only the real tokens), and
 the speedup over exact attention (which runs without the bias).  A mix
 ("uformer-mix": Uformer stages 1 and 4) launches its workloads back to back on
 one stream and is timed as one.  A workload with a relative-position bias
-pools it once (a model constant) and times the biased call.
+pools it once (a model constant) and times the biased call.  A fused-projection
+workload ("-qkv": tokens X and W_QKV in, algorithmic bytes X + W + O) is timed
+against the unfused path it replaces: one cuBLAS projection X W_QKV^T (torch),
+the copy that splits heads, and nystra_attention.
 """
 from __future__ import annotations
 
@@ -34,7 +37,8 @@ DEFAULT = (["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4
            + [f"large-w{w}-m{m}" for w in (16, 32) for m in (32, 64)]
            + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")]
            + [f"{n}-{x}" for x in ("patches", "relpos")
-              for n in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16")])
+              for n in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16")]
+           + [n for n in workloads.WORKLOADS if n.endswith("-qkv")])
 
 
 def hbm_peak_gbs() -> tuple[float, str]:
@@ -69,7 +73,49 @@ def _median_ms(launch, n_sets: int, reps: int) -> float:
     return statistics.median(s.elapsed_time(e) for s, e in evs)
 
 
+def run_qkv(wl: workloads.Workload, l2_bytes: int, peak: float, reps: int = 50) -> dict:
+    """The fused projection against projecting first (cuBLAS + head split + nystra_attention)."""
+    io = wl.io_bytes
+    n_sets = max(2, -(-3 * l2_bytes // io))
+    dev = torch.device("cuda")
+    x, w = workloads.make_x_wqkv(wl)
+    w = w.to(dev)
+    bias = workloads.make_bias(wl)
+    pooled = None if bias is None else binding.pool_bias(bias.to(dev), wl.m, wl.landmarks)
+    sets = [(x.to(dev), torch.empty(wl.shape, dtype=x.dtype, device=dev)) for _ in range(n_sets)]
+
+    def fused(i):
+        xs, o = sets[i]
+        binding.nystra_qkv(xs, w, wl.heads, wl.m, wl.iters, pooled=pooled, out=o, landmarks=wl.landmarks)
+
+    def unfused(i):
+        xs, o = sets[i]
+        y = xs.reshape(-1, wl.C) @ w.T
+        q, k, v = (y.view(wl.n_windows, wl.N, 3, wl.heads, wl.d)[:, :, j].transpose(1, 2).contiguous()
+                   for j in range(3))
+        if pooled is None:
+            binding.nystra(q, k, v, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+        else:
+            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+
+    t_f = _median_ms(fused, n_sets, reps)
+    t_u = _median_ms(unfused, n_sets, max(10, reps // 5))
+    tokens = wl.units * wl.N
+    gbs = io / (t_f * 1e-3) / 1e9
+    res = {"name": wl.name, "units": wl.units, "io_MB": io / 1e6, "nystra_ms": t_f, "unfused_ms": t_u,
+           "GBps": gbs, "frac_of_hbm": gbs / peak, "tokens_heads_per_s": tokens / (t_f * 1e-3),
+           "speedup_vs_unfused": t_u / t_f}
+    real = _real_tokens(wl)
+    if real != tokens:
+        res["real_tokens_heads_per_s"] = real / (t_f * 1e-3)
+    del sets
+    torch.cuda.empty_cache()
+    return res
+
+
 def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int = 10) -> dict:
+    if name in workloads.WORKLOADS and workloads.WORKLOADS[name].front == "qkv":
+        return run_qkv(workloads.WORKLOADS[name], l2_bytes, peak, reps)
     parts = [workloads.WORKLOADS[n] for n in MIXES.get(name, (name,))]
     io = sum(wl.io_bytes for wl in parts)
     n_sets = max(2, -(-3 * l2_bytes // io))

@@ -29,7 +29,7 @@ def test_header_declares_the_boundary():
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
                      "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
                      "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size",
-                     "nystra_attention_ex", "nystra_pool_bias", "nystra_attention_bias"):
+                     "nystra_attention_ex", "nystra_pool_bias", "nystra_attention_bias", "nystra_attention_qkv"):
         assert required in names
 
 
@@ -185,3 +185,39 @@ def test_attention_bias_argument_validation(lib, args, code):
     rc = nb.nystra_attention_bias(P, 2 * P, 3 * P, 64 * P, a["nw"], 2, 64, 30, a["m"], 6, 0, a["bL"], a["bU"],
                                   a["bA"], a["bw"], 1, None)
     assert rc == code
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(dtype=0), nb.NYSTRA_EDTYPE),            # fp32: 16-bit I/O only
+    (dict(dtype=7), nb.NYSTRA_EDTYPE),
+    (dict(N=256), nb.NYSTRA_EINVAL),              # 8x8 windows only
+    (dict(m=32), nb.NYSTRA_EINVAL),
+    (dict(d=31), nb.NYSTRA_EINVAL),               # odd d_h
+    (dict(d=34), nb.NYSTRA_EINVAL),               # d_h > 32
+    (dict(heads=12, d=32), nb.NYSTRA_EINVAL),     # C = 384 > NYSTRA_QKV_MAX_C
+    (dict(iters=13), nb.NYSTRA_EINVAL),
+    (dict(lm=1, m=8), nb.NYSTRA_EINVAL),          # square patches need m = 16
+    (dict(lm=2), nb.NYSTRA_EINVAL),
+    (dict(x=0), nb.NYSTRA_EINVAL),
+    (dict(w=2 * P + 4), nb.NYSTRA_EINVAL),        # misaligned
+    (dict(b=3 * P + 8), nb.NYSTRA_EINVAL),
+    (dict(out=P + 64), nb.NYSTRA_EINVAL),         # overlaps x
+    (dict(out=3 * P), nb.NYSTRA_EINVAL),          # overlaps the projection bias
+    (dict(bL=8 * P, bw=3), nb.NYSTRA_EINVAL),     # bias windows neither 1 nor n_windows
+    (dict(bL=8 * P, bA=0), nb.NYSTRA_EINVAL),
+    (dict(bL=64 * P), nb.NYSTRA_EINVAL),          # score bias overlaps out
+    (dict(nw=0), nb.NYSTRA_OK),                   # empty: no-op
+    (dict(heads=0), nb.NYSTRA_OK),
+])
+def test_attention_qkv_argument_validation(lib, args, code):
+    a = dict(x=P, w=2 * P, b=3 * P, out=64 * P, nw=4, heads=6, N=64, d=30, m=16, iters=6, lm=0,
+             bL=0, bU=9 * P, bA=10 * P, bw=1, dtype=1)
+    a.update(args)
+    rc = nb.nystra_attention_qkv(a["x"], a["w"], a["b"], a["out"], a["nw"], a["heads"], a["N"], a["d"], a["m"],
+                                 a["iters"], a["lm"], a["bL"], a["bU"], a["bA"], a["bw"], a["dtype"], None)
+    assert rc == code
+
+
+def test_qkv_max_width_matches_the_header():
+    text = open(HEADER).read()
+    assert f"#define NYSTRA_QKV_MAX_C {nb.QKV_MAX_C}" in text
