@@ -272,9 +272,10 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[5])(cudaError_t*) = {take_fault_word_tc_n64, take_fault_word_tc_n256,
-                                                   take_fault_word_tc_n1024, take_fault_word_exact_tc,
-                                                   take_fault_word_debug};
+    unsigned int (*const take[7])(cudaError_t*) = {take_fault_word_tc_n64,    take_fault_word_tc_n256,
+                                                   take_fault_word_tc_n1024,  take_fault_word_exact_tc,
+                                                   take_fault_word_debug,     take_fault_word_qkv_bf16,
+                                                   take_fault_word_qkv_f16};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

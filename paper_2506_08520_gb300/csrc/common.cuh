@@ -110,6 +110,8 @@ cudaError_t launch_nystra_qkv_bf16(const void* x, const void* wqkv, const float*
 cudaError_t launch_nystra_qkv_f16(const void* x, const void* wqkv, const float* bqkv, void* out,
                                   long long n_windows, int heads, int d, int m, int iters, int pool,
                                   cudaStream_t stream, const nystra::NystraBias* bias);
+unsigned int take_fault_word_qkv_bf16(cudaError_t* err);
+unsigned int take_fault_word_qkv_f16(cudaError_t* err);
 // Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
 long long debug_stages_size(int N, int d, int m);
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,

@@ -18,12 +18,24 @@
 // Warps.  Each of the NW warps takes one unit at a time (window i = w,
 // w + NW, ... of its CTA).  It projects in two halves of 32 tokens: A
 // fragments (token rows, C contiguous 16-bit values) straight from global
-// memory, loaded three k-steps ahead of their MMAs, against the three weight
+// memory, loaded three k-steps ahead of their MMAs (two with shared stages,
+// whose 12 warps leave fewer registers), against the three weight
 // blocks at once (96 fp32 accumulators); the results plus bias, rounded to
-// the I/O type as an unfused projection would store them, go to the warp's
-// private Q, K, V stage.  Then the pool kernel's phases run on that stage and
-// the output tile leaves with one bulk store.  Nothing is handed between
-// warps, so the kernel has no waits.
+// the I/O type as an unfused projection would store them, go to a Q, K, V
+// stage.  The core and the output run on warp-private state; the output tile
+// leaves with one bulk store.
+//
+// Stages.  A stage is dead once the front phase has read it (G_L^n is
+// parked, so the output does not read Q again).  With a short projection
+// (C <= 64) two warps share each stage (PAIR: 12 warps on 6 stages, as the
+// pool kernel shares its stages): warp w and warp w + NS take turns in the
+// order of their windows (stage w mod NS serves windows i = w mod NS, + NS,
+// + 2 NS, ...), the k-th user waiting, on the stage's mbarrier (bounded), for
+// the (k-1)-th to arrive after its front phase; the extra warps hide the
+// core's latency.  A longer projection keeps the stage busy for most of a
+// unit, so sharing would serialise the two warps' projections: 8 warps with a
+// stage each, and no waits (measured: 12 shared-stage warps are 16% faster at
+// C = 32, 2-12% slower at C = 180).
 #pragma once
 
 #include "nystra_pool.cuh"
@@ -31,16 +43,19 @@
 namespace nystra {
 namespace tc {
 
-template <typename T, int M, int NCOL>
+template <typename T, int M, int NCOL, bool PAIR>
 struct QkvLayout {
     using PL = PoolLayout<T, M, NCOL>;
-    static constexpr int NW = 8;                           // warps per CTA
-    static constexpr size_t WARP = PL::STAGE + PL::PRIV;   // private Q/K/V stage + the pool kernel's state
-    static constexpr size_t FRAG = 3 * 4 * 32 * 8;         // weight fragments per k-step: 3 blocks x 4 n-tiles x 32 lanes x 8 B
-    // k-steps ks = ceil(C / 16): the weights first, then the warps
-    static constexpr size_t warps_at(int ks) { return (size_t)ks * FRAG; }
-    static constexpr size_t bytes(int ks) { return warps_at(ks) + NW * WARP; }
-    static_assert(WARP % 128 == 0 && FRAG % 128 == 0, "regions stay 128-byte aligned");
+    static constexpr int NW = PAIR ? 12 : 8;         // warps per CTA
+    static constexpr int NS = PAIR ? NW / 2 : NW;    // Q/K/V stages
+    static constexpr size_t HDR = 128;               // the stages' mbarriers
+    static constexpr size_t FRAG = 3 * 4 * 32 * 8;   // weight fragments per k-step: 3 blocks x 4 n-tiles x 32 lanes x 8 B
+    // k-steps ks = ceil(C / 16): header, weights, stages, warp-private state
+    static constexpr size_t stages_at(int ks) { return HDR + (size_t)ks * FRAG; }
+    static constexpr size_t priv_at(int ks) { return stages_at(ks) + NS * PL::STAGE; }
+    static constexpr size_t bytes(int ks) { return priv_at(ks) + NW * PL::PRIV; }
+    static_assert(NS * 8 <= HDR, "one mbarrier per stage");
+    static_assert(PL::STAGE % 128 == 0 && PL::PRIV % 128 == 0 && FRAG % 128 == 0, "regions stay 128-byte aligned");
 };
 
 __device__ __forceinline__ uint32_t ldg_u32(const void* p) { return __ldg(reinterpret_cast<const unsigned int*>(p)); }
@@ -67,8 +82,9 @@ __device__ __forceinline__ void stage_weights(const T* __restrict__ wqkv, int C,
 }
 
 // Q, K, V of one unit ([64, d] each, row-major, consecutive in `qkv`) from the
-// window's tokens xw ([64, C] in global memory) and the staged fragments.
-template <typename T>
+// window's tokens xw ([64, C] in global memory) and the staged fragments; the
+// A fragments are loaded DEPTH k-steps ahead of their MMAs.
+template <typename T, int DEPTH>
 __device__ __forceinline__ void project_unit(const T* __restrict__ xw, const uint2* wf,
                                              const float* __restrict__ bqkv, int C, int h, int d, int ks, T* qkv,
                                              int g, int t, int lane) {
@@ -109,18 +125,32 @@ __device__ __forceinline__ void project_unit(const T* __restrict__ xw, const uin
                     Op::k16(acc[mat][nt][1], a[1], b.x, b.y);
                 }
         };
-        uint32_t a0[2][4], a1[2][4], a2[2][4];
-        lda(0, a0);
-        lda(1, a1);
-        lda(2, a2);
+        // k-steps at or beyond ks load nothing (v0 = v1 = false)
+        if constexpr (DEPTH == 3) {
+            uint32_t a0[2][4], a1[2][4], a2[2][4];
+            lda(0, a0);
+            lda(1, a1);
+            lda(2, a2);
 #pragma unroll 1
-        for (int kk = 0; kk < ks; kk += 3) {  // k-steps at or beyond ks load nothing (v0 = v1 = false)
-            mma_step(kk, a0);
-            lda(kk + 3, a0);
-            if (kk + 1 < ks) mma_step(kk + 1, a1);
-            lda(kk + 4, a1);
-            if (kk + 2 < ks) mma_step(kk + 2, a2);
-            lda(kk + 5, a2);
+            for (int kk = 0; kk < ks; kk += 3) {
+                mma_step(kk, a0);
+                lda(kk + 3, a0);
+                if (kk + 1 < ks) mma_step(kk + 1, a1);
+                lda(kk + 4, a1);
+                if (kk + 2 < ks) mma_step(kk + 2, a2);
+                lda(kk + 5, a2);
+            }
+        } else {
+            uint32_t a0[2][4], a1[2][4];
+            lda(0, a0);
+            lda(1, a1);
+#pragma unroll 1
+            for (int kk = 0; kk < ks; kk += 2) {
+                mma_step(kk, a0);
+                lda(kk + 2, a0);
+                if (kk + 1 < ks) mma_step(kk + 1, a1);
+                lda(kk + 3, a1);
+            }
         }
         // + bias, rounded to the I/O type, into the stage
 #pragma unroll
@@ -145,12 +175,12 @@ __device__ __forceinline__ void project_unit(const T* __restrict__ xw, const uin
     }
 }
 
-template <typename T, int M, int NCOL, int PW, bool BIAS>
-__global__ void __launch_bounds__(QkvLayout<T, M, NCOL>::NW * 32, 1)
+template <typename T, int M, int NCOL, int PW, bool BIAS, bool PAIR>
+__global__ void __launch_bounds__(QkvLayout<T, M, NCOL, PAIR>::NW * 32, 1)
 nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const float* __restrict__ bqkv,
                   T* __restrict__ out, long long n_windows, int heads, int d, int ks, int iters, float sl2,
-                  NystraBias bias) {
-    using P = QkvLayout<T, M, NCOL>;
+                  unsigned int* fault, NystraBias bias) {
+    using P = QkvLayout<T, M, NCOL, PAIR>;
     using PL = typename P::PL;
     constexpr int L = 64 / M;  // tokens per landmark segment
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -160,12 +190,13 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
     const int h = (int)(blockIdx.x % heads);
     const long long Gh = gridDim.x / heads, w0 = blockIdx.x / heads;
 
-    uint2* wf = reinterpret_cast<uint2*>(smem_raw);
-    unsigned char* pw = smem_raw + P::warps_at(ks) + (size_t)w * P::WARP;
-    T* Qs = reinterpret_cast<T*>(pw);
+    const int st = w % P::NS;  // this warp's stage (PAIR: shared with warp (w + NS) mod NW)
+    uint64_t* sbar = reinterpret_cast<uint64_t*>(smem_raw) + st;
+    uint2* wf = reinterpret_cast<uint2*>(smem_raw + P::HDR);
+    T* Qs = reinterpret_cast<T*>(smem_raw + P::stages_at(ks) + (size_t)st * PL::STAGE);
     T* Ks = Qs + 64 * d;
     T* Vs = Qs + 128 * d;
-    unsigned char* pv = pw + PL::STAGE;
+    unsigned char* pv = smem_raw + P::priv_at(ks) + (size_t)w * PL::PRIV;
     uint32_t* glf = reinterpret_cast<uint32_t*>(pv + PL::GLF);
     T* qbar = reinterpret_cast<T*>(pv + PL::QB);
     T* kbar = reinterpret_cast<T*>(pv + PL::KB);
@@ -174,6 +205,10 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
     T* ob = reinterpret_cast<T*>(pv + PL::OUT);
     const uint32_t tile_bytes = (uint32_t)(64 * d * sizeof(T));
 
+    if (threadIdx.x == 0) {
+        for (int j = 0; j < P::NS; ++j) mbar_init(reinterpret_cast<uint64_t*>(smem_raw) + j, 1);
+        fence_mbar_init();
+    }
     stage_weights<T>(wqkv, C, h, d, ks, wf);
     __syncthreads();
 
@@ -181,12 +216,19 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
         const long long win = w0 + i * Gh;
         if (win >= n_windows) break;
         const long long u = win * heads + h;
+        // the stage's k-th use (windows st, st + NS, ... alternate between the
+        // two warps): wait until use k - 1 has finished its front phase
+        const long long k = (i - st) / P::NS;
+        if (PAIR && k > 0 && !__all_sync(0xffffffffu, mbar_wait_bounded(sbar, (uint32_t)((k - 1) & 1), kWaitNs))) {
+            if (lane == 0) atomicOr(fault, 1u);
+            break;
+        }
         const long long bs = BIAS ? (bias.per_window ? u : h) : 0;
         const float* bLu = BIAS ? bias.L + (size_t)bs * 64 * M : nullptr;
         const float* bUu = BIAS ? bias.U + (size_t)bs * M * 64 : nullptr;
         const float* bAu = BIAS ? bias.A + (size_t)bs * M * M : nullptr;
         // ---------------- projection (Eq. 1) into the stage ----------------
-        project_unit<T>(x + (size_t)win * 64 * C, wf, bqkv, C, h, d, ks, Qs, g, t, lane);
+        project_unit<T, PAIR ? 2 : 3>(x + (size_t)win * 64 * C, wf, bqkv, C, h, d, ks, Qs, g, t, lane);
         // the previous unit's output store has read its staging (which
         // overlaps the landmarks and W written below)
         if (lane == 0) bulk_wait_read_all();
@@ -214,6 +256,11 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
         // ---------------- front: S_U, m_U, W = G_U^n [V | 1] ----------------
         float mU[1][2];
         front_su_w<T, M, NCOL, 1, BIAS>(qbar, Ks, Vs, d, g, t, sl2, mW, PL::WS, mU, bUu, 64);
+        // the stage has been read: hand it to the other warp's next window
+        if constexpr (PAIR) {
+            __syncwarp();
+            if (lane == 0) mbar_arrive(sbar);
+        }
         // ---------------- core: G_A^n, Z_0, iteration, Y ----------------
         core_warp<T, M, NCOL, false, BIAS>(qbar, kbar, mU, mW, yT, iters, sl2, g, t, nullptr, bAu);
         __syncwarp();
@@ -229,11 +276,12 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
     if (lane == 0) bulk_wait_all();  // output stores complete before exit
 }
 
-template <typename T, int M, int NCOL, int PW, bool BIAS>
+template <typename T, int M, int NCOL, int PW, bool BIAS, bool PAIR>
 cudaError_t launch_qkv_cfg(const void* x, const void* wqkv, const float* bqkv, void* out, long long n_windows,
-                           int heads, int d, int iters, cudaStream_t stream, const NystraBias& bias) {
-    using P = QkvLayout<T, M, NCOL>;
-    auto kern = nystra_qkv_kernel<T, M, NCOL, PW, BIAS>;
+                           int heads, int d, int iters, cudaStream_t stream, unsigned int* fault,
+                           const NystraBias& bias) {
+    using P = QkvLayout<T, M, NCOL, PAIR>;
+    auto kern = nystra_qkv_kernel<T, M, NCOL, PW, BIAS, PAIR>;
     const int C = heads * d, ks = (C + 15) / 16;
     const size_t smem = P::bytes(ks);
     if (smem > kSmemLimit) return cudaErrorInvalidValue;  // not reached: the caller bounds C
@@ -248,28 +296,44 @@ cudaError_t launch_qkv_cfg(const void* x, const void* wqkv, const float* bqkv, v
     const long long grid = per_head * heads;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);
     kern<<<(unsigned)grid, P::NW * 32, smem, stream>>>((const T*)x, (const T*)wqkv, bqkv, (T*)out, n_windows,
-                                                        heads, d, ks, iters, sl2, bias);
+                                                        heads, d, ks, iters, sl2, fault, bias);
     return cudaGetLastError();
 }
 
-// m in {8, 16} (square patches: m = 16); d_h read at run time.
+// m in {8, 16} (square patches: m = 16); d_h read at run time; shared
+// stages for C <= 64.
+template <typename T, int M, int NCOL, int PW>
+cudaError_t launch_qkv_m(const void* x, const void* wqkv, const float* bqkv, void* out, long long n_windows,
+                         int heads, int d, int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
+    const NystraBias b = bias ? *bias : NystraBias{};
+    const bool pair = heads * d <= 64;
+    if (bias)
+        return pair ? launch_qkv_cfg<T, M, NCOL, PW, true, true>(x, wqkv, bqkv, out, n_windows, heads, d, iters,
+                                                                  stream, fault, b)
+                    : launch_qkv_cfg<T, M, NCOL, PW, true, false>(x, wqkv, bqkv, out, n_windows, heads, d, iters,
+                                                                   stream, fault, b);
+    return pair ? launch_qkv_cfg<T, M, NCOL, PW, false, true>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream,
+                                                               fault, b)
+                : launch_qkv_cfg<T, M, NCOL, PW, false, false>(x, wqkv, bqkv, out, n_windows, heads, d, iters,
+                                                                stream, fault, b);
+}
+
 template <typename T>
 cudaError_t launch_qkv(const void* x, const void* wqkv, const float* bqkv, void* out, long long n_windows,
-                       int heads, int d, int m, int iters, int pool, cudaStream_t stream, const NystraBias* bias) {
+                       int heads, int d, int m, int iters, int pool, cudaStream_t stream, unsigned int* fault,
+                       const NystraBias* bias) {
     const bool wide = d > 30;  // the ones column needs a fifth n-tile when d_h = 32
-    const NystraBias b = bias ? *bias : NystraBias{};
-#define NYSTRA_QKV_GO(MM, PW)                                                                                  \
-    return bias ? (wide ? launch_qkv_cfg<T, MM, 40, PW, true>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, b) \
-                        : launch_qkv_cfg<T, MM, 32, PW, true>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, b)) \
-                : (wide ? launch_qkv_cfg<T, MM, 40, PW, false>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, b) \
-                        : launch_qkv_cfg<T, MM, 32, PW, false>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, b))
     if (pool != 0) {
         if (m != 16) return cudaErrorInvalidValue;  // not reached: checked by the caller
-        NYSTRA_QKV_GO(16, 8);
+        return wide ? launch_qkv_m<T, 16, 40, 8>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias)
+                    : launch_qkv_m<T, 16, 32, 8>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias);
     }
-    if (m == 8) NYSTRA_QKV_GO(8, 0);
-    if (m == 16) NYSTRA_QKV_GO(16, 0);
-#undef NYSTRA_QKV_GO
+    if (m == 8)
+        return wide ? launch_qkv_m<T, 8, 40, 0>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias)
+                    : launch_qkv_m<T, 8, 32, 0>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias);
+    if (m == 16)
+        return wide ? launch_qkv_m<T, 16, 40, 0>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias)
+                    : launch_qkv_m<T, 16, 32, 0>(x, wqkv, bqkv, out, n_windows, heads, d, iters, stream, fault, bias);
     return cudaErrorInvalidValue;
 }
 
@@ -277,13 +341,46 @@ cudaError_t launch_qkv(const void* x, const void* wqkv, const float* bqkv, void*
 }  // namespace nystra
 
 // Largest token width C = heads * d_h the fused kernel takes (nystra.h):
-// its weight fragments fit beside the warps' state in both layouts.
+// its weight fragments fit beside the stages and the warps' state (shared
+// stages only up to C = 64).
 namespace nystra {
 namespace tc {
 constexpr int kQkvMaxC = 352;
-static_assert(QkvLayout<__half, 16, 40>::bytes(kQkvMaxC / 16) <= kSmemLimit &&
-                  QkvLayout<__half, 16, 32>::bytes(kQkvMaxC / 16) <= kSmemLimit &&
-                  QkvLayout<__half, 8, 40>::bytes(kQkvMaxC / 16) <= kSmemLimit,
+static_assert(QkvLayout<__half, 16, 40, false>::bytes(kQkvMaxC / 16) <= kSmemLimit &&
+                  QkvLayout<__half, 16, 32, false>::bytes(kQkvMaxC / 16) <= kSmemLimit &&
+                  QkvLayout<__half, 8, 40, false>::bytes(kQkvMaxC / 16) <= kSmemLimit &&
+                  QkvLayout<__half, 16, 40, true>::bytes(64 / 16) <= kSmemLimit &&
+                  QkvLayout<__half, 8, 40, true>::bytes(64 / 16) <= kSmemLimit,
               "the widest projection must fit in shared memory");
 }  // namespace tc
 }  // namespace nystra
+
+// One translation unit per I/O type defines its fault word and entry point.
+#define NYSTRA_QKV_DEFINE(NAME, T)                                                                          \
+    namespace nystra {                                                                                      \
+    __device__ unsigned int g_fault_qkv_##NAME;                                                             \
+    }                                                                                                       \
+    namespace nystra_host {                                                                                 \
+    cudaError_t launch_nystra_qkv_##NAME(const void* x, const void* wqkv, const float* bqkv, void* out,     \
+                                         long long n_windows, int heads, int d, int m, int iters, int pool, \
+                                         cudaStream_t stream, const nystra::NystraBias* bias) {             \
+        static unsigned int* s_fault[nystra::kMaxDevices] = {}; /* fault word's address, per device */     \
+        int dev = 0;                                                                                        \
+        cudaError_t e = cudaGetDevice(&dev);                                                                \
+        if (e != cudaSuccess) return e;                                                                     \
+        if (dev < 0 || dev >= nystra::kMaxDevices) return cudaErrorInvalidDevice;                          \
+        if (!s_fault[dev]) {                                                                                \
+            e = cudaGetSymbolAddress((void**)&s_fault[dev], nystra::g_fault_qkv_##NAME);                    \
+            if (e != cudaSuccess) return e;                                                                 \
+        }                                                                                                   \
+        return nystra::tc::launch_qkv<T>(x, wqkv, bqkv, out, n_windows, heads, d, m, iters, pool, stream,   \
+                                         s_fault[dev], bias);                                               \
+    }                                                                                                       \
+    unsigned int take_fault_word_qkv_##NAME(cudaError_t* err) {                                             \
+        unsigned int w = 0, zero = 0;                                                                       \
+        *err = cudaMemcpyFromSymbol(&w, nystra::g_fault_qkv_##NAME, sizeof(w));                             \
+        if (*err == cudaSuccess && w != 0)                                                                  \
+            *err = cudaMemcpyToSymbol(nystra::g_fault_qkv_##NAME, &zero, sizeof(zero));                     \
+        return w;                                                                                           \
+    }                                                                                                       \
+    }

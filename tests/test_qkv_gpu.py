@@ -36,6 +36,8 @@ CASES = [  # n_windows, heads, d_h, m, pooling, dtype, projection bias
     (4, 6, 30, 16, "patches", "bf16", True),      # square-patch landmarks
     (3, 2, 16, 16, "segments", "bf16", True),     # d_h = 16: two empty n-tiles
     (3, 11, 32, 16, "segments", "bf16", True),    # C = 352, the widest
+    (2, 2, 32, 8, "segments", "f16", True),       # C = 64: the widest with shared stages
+    (3, 2, 30, 16, "patches", "bf16", True),      # shared stages, square patches
     (2, 5, 6, 8, "segments", "f16", True),        # C = 30: C % 4 != 0
     (2, 176, 2, 8, "segments", "bf16", True),     # more heads than SMs: CTAs beyond one wave
     (1, 6, 30, 16, "segments", "bf16", False),    # one window
