@@ -48,7 +48,7 @@ struct QkvLayout {
     using PL = PoolLayout<T, M, NCOL>;
     static constexpr int NW = PAIR ? 12 : 8;         // warps per CTA
     static constexpr int NS = PAIR ? NW / 2 : NW;    // Q/K/V stages
-    static constexpr size_t HDR = 128;               // the stages' mbarriers
+    static constexpr size_t HDR = 128;               // the shared stages' mbarriers
     static constexpr size_t FRAG = 3 * 4 * 32 * 8;   // weight fragments per k-step: 3 blocks x 4 n-tiles x 32 lanes x 8 B
     // k-steps ks = ceil(C / 16): header, weights, stages, warp-private state
     static constexpr size_t stages_at(int ks) { return HDR + (size_t)ks * FRAG; }
