@@ -38,13 +38,16 @@ METRIC = "Nystrom attention tokens*heads/s"
 # of those files changes.
 MEASURED_TRAFFIC = {
     "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
-                       "src_hash": "18461915ec80da1f", "bytes": 73_978_880},
+                       "src_hash": "0d6b9b4b0c940865", "bytes": 73_427_968},
     "sr720p-w16-m16-bf16": {"files": ["common.cuh", "nystra_team.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu",
                                       "ptx.cuh"],
-                            "src_hash": "db325f6b5b3db04f", "bytes": 1_296_579_840},
+                            "src_hash": "e91802655794bad2", "bytes": 1_296_480_256},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-                            "src_hash": "c2f79d75bf44c177", "bytes": 1_351_302_656},
+                            "src_hash": "93de88be9dc1f252", "bytes": 1_349_584_944},
+    "swinir256-bf16-qkv": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_qkv.cuh", "nystra_qkv_bf16.cu",
+                                     "nystra_tc.cuh", "ptx.cuh"],
+                           "src_hash": "3f65ce1aaad8de7b", "bytes": 23_849_216},
 }
 
 
