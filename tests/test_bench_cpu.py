@@ -43,3 +43,24 @@ def test_sweep_list_runs_without_a_gpu(capsys):
     from paper_2506_08520_gb300 import sweep
     assert sweep.main(["--list", "uformer-mix", "tiny"]) == 0
     assert capsys.readouterr().out.split() == ["uformer-mix", "tiny"]
+
+
+def test_reference_arm_of_the_fused_projection_workload():
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "3",
+                        "--warmup", "3", "--workload", "uformer-s4-qkv"], capture_output=True, text=True,
+                       timeout=600, cwd=ROOT)
+    assert r.returncode == 0, r.stderr
+    j = json.loads([l for l in r.stdout.splitlines() if l.startswith("{")][-1])
+    assert j["impl"] == "reference" and j["value"] > 0
+    assert j["config"]["workload"] == "uformer-s4-qkv" and "front" in j["config"]
+    assert "projections made beforehand" in j["cpu_baseline"]["sample"]
+
+
+def test_unit_flops_counts_the_projection():
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2506_08520_gb300 import workloads
+    wl = workloads.WORKLOADS["swinir256-bf16"]
+    fused = workloads.WORKLOADS["swinir256-bf16-qkv"]
+    assert bench.unit_flops(fused) - bench.unit_flops(wl) == 2 * 64 * 180 * 90
+    assert fused.io_bytes == (2 * 1024 * 64 * 180 + 3 * 180 * 180) * 2
