@@ -142,3 +142,33 @@ def test_fused_workloads(name):
     err = per_unit_rel(got, ref)
     print(f"{name}: max rel err {err.max():.3e}")
     assert err.max() <= TOL[wl.dtype]
+
+
+def _window_masks(n_windows, w=8, seed=0):
+    """Shifted-window-like masks: tokens of different regions do not attend to
+    each other (-100, finite); every other window is unmasked."""
+    rng = np.random.default_rng(seed)
+    N = w * w
+    masks = np.zeros((n_windows, N, N))
+    for i in range(0, n_windows, 2):
+        region = (np.arange(N) % w >= w // 2).astype(int) + 2 * (np.arange(N) // w >= rng.integers(1, w))
+        masks[i] = np.where(region[:, None] == region[None, :], 0.0, -100.0)
+    return masks
+
+
+@pytest.mark.parametrize("heads,d,dtype,per_window", [(2, 30, "bf16", False),   # shared stages (C = 60)
+                                                      (2, 30, "f16", True),     # shared stages, per-window masks
+                                                      (6, 30, "bf16", True)])   # private stages, per-window masks
+def test_fused_projection_score_bias_variants(heads, d, dtype, per_window):
+    nw, m = 4, 16
+    x, w, b = workloads.random_x_wqkv(nw, 64, heads, d, dtype, seed=heads * 10 + d)
+    B = workloads.relpos_bias(8, heads, seed=15)[None].astype(np.float64)       # [1, heads, N, N]
+    if per_window:
+        B = B + _window_masks(nw)[:, None]                                       # [nw, heads, N, N]
+    B32 = np.ascontiguousarray(B.astype(np.float32))
+    pooled = binding.pool_bias(torch.from_numpy(B32).cuda(), m)
+    out = _run(x, w, b, heads, m, pooled=pooled)
+    ref = oracle.nystra_attention_qkv(x, w, b, heads, m, 6, "segments",
+                                      np.broadcast_to(B32.astype(np.float64), (nw, heads, 64, 64)))
+    err = per_unit_rel(out.double().numpy(), ref)
+    assert err.max() <= TOL[dtype], f"max rel err {err.max():.3e} at unit {int(err.argmax())}"
