@@ -14,6 +14,8 @@
  *  Layout   q, k, v and out are contiguous row-major tensors of shape
  *           [n_windows, heads, N, d_h]; one "unit" = one (window, head) pair,
  *           whose N x d_h block starts at element (w*heads + h) * N * d_h.
+ *           (nystra_attention_qkv takes the tokens x [n_windows, N, heads*d_h]
+ *           and the projection weights instead of q, k, v; see there.)
  *  Memory   every pointer is DEVICE memory owned by the caller, 16-byte
  *           aligned, and stays valid until the work on `stream` completes.
  *           q, k and v may alias one another; out must not overlap any input.
