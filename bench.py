@@ -1,8 +1,10 @@
 """Benchmark of the PnP-Nystra window-attention hot path on GB300.
 
 One step = one ``nystra_attention`` call over the whole batch of the workload
-(default: SwinIR-like denoising at 256x256 -- 1024 windows of 8x8 tokens,
-6 heads, d_h = 30, m = 16 landmarks, 6 pseudo-inverse iterations, bf16 I/O).
+(default: the 1280x720 super-resolution map -- 6 heads, d_h = 30, 32x32
+windows edge-padded to 736 rows (920 windows), m = 16 landmarks, 6
+pseudo-inverse iterations, bf16 I/O; the 16x16-window map and SwinIR-like
+denoising at 256x256 are timed beside it under "extra_workloads").
 Prints ONE JSON line (rank 0).  Metric: tokens*heads per second.  A "-qkv"
 workload times the fused Q/K/V projection front end instead (one
 ``nystra_attention_qkv`` call; tensor roofline, unfused path as comparator).
@@ -60,7 +62,14 @@ def _kernel_src_hash(files) -> str:
             h.update(fh.read())
     return h.hexdigest()[:16]
 UNIT = "tokens*heads/s"
-DEFAULT_WORKLOAD = "swinir256-bf16"
+# The largest memory-bound configuration: the 1280x720 map with 32x32 windows
+# and m = 16 landmarks (1357 MB of Q, K, V, O per call).
+DEFAULT_WORKLOAD = "sr720p-w32-m16-bf16"
+# Reported beside a headline workload, each with its own roofline and comparator.
+EXTRA_WORKLOADS = {
+    "sr720p-w32-m16-bf16": ["sr720p-w16-m16-bf16", "swinir256-bf16"],
+    "sr720p-w16-m16-bf16": ["sr720p-w32-m16-bf16", "swinir256-bf16"],
+}
 
 
 def _peaks():
@@ -260,23 +269,17 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
-def run_cuda(args, wl):
-    ws, rank, local = _dist()
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=dev)
-    binding.lib()  # fail loudly if the library is missing
-
+def _time_kernel(wl, dev, steps: int, warmup: int, ws: int, sampler=None):
+    """Device-resident timing of one workload: `steps` launches of
+    ``nystra_attention`` (bracketed by barriers, CUDA events on the launching
+    stream, rotating input/output sets > 3x L2), then the exact window
+    attention kernel on the same inputs.  Returns the timing record, the
+    host inputs (for the end-to-end loop) and the device sets."""
     q, k, v = workloads.make_qkv(wl)
     esize = q.element_size()
-    # rotate input/output sets so that one step's data is never L2-resident
     nsets, io_bytes, config = _config(wl, ws)
     assert io_bytes == 4 * q.numel() * esize
-    sets = []
-    for _ in range(nsets):
-        sets.append(tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),))
+    sets = [tuple(x.to(dev) for x in (q, k, v)) + (torch.empty_like(q, device=dev),) for _ in range(nsets)]
     stream = torch.cuda.current_stream(dev)
     sptr = stream.cuda_stream
     bias = workloads.make_bias(wl)  # a model constant: pooled once, outside the timed region
@@ -284,7 +287,7 @@ def run_cuda(args, wl):
     shape = (wl.n_windows, wl.heads, wl.N, wl.d)
     dcode = {"f32": 0, "bf16": 1, "f16": 2}[wl.dtype]
 
-    def step(i, fn=binding.nystra_attention, exact=False):
+    def step(i, exact=False):
         qd, kd, vd, od = sets[i % nsets]
         if exact:
             rc = binding.exact_window_attention(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(),
@@ -297,8 +300,8 @@ def run_cuda(args, wl):
             rc = binding.nystra_attention_ex(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
                                              wl.m, wl.iters, binding.NYSTRA_LANDMARKS_PATCHES, dcode, sptr)
         else:
-            rc = fn(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape, wl.m, wl.iters,
-                    dcode, sptr)
+            rc = binding.nystra_attention(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
+                                          wl.m, wl.iters, dcode, sptr)
         if rc != 0:
             raise binding.NystraError(rc, "bench step")
 
@@ -308,26 +311,37 @@ def run_cuda(args, wl):
             torch.distributed.barrier()
         torch.cuda.synchronize(dev)
 
-    for i in range(args.warmup):
+    w0 = time.perf_counter()
+    for i in range(warmup):
         step(i)
     barrier()
-    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    with ClockSampler(local) as clk:
+    per_launch = (time.perf_counter() - w0) / max(1, warmup)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    if sampler is not None:
+        sampler.__enter__()
+    try:
+        # Untimed launches of the same kernel while the clock sampler runs, so
+        # that its samples see the GPU under this load even when the timed
+        # region itself is shorter than the sampling interval.
+        if sampler is not None:
+            for i in range(min(20000, int(0.6 / max(per_launch, 1e-6)))):
+                step(i)
         barrier()
-        for i in range(args.steps):
+        for i in range(steps):
             starts[i].record(stream)
             step(i)
             ends[i].record(stream)
         barrier()
+    finally:
+        if sampler is not None:
+            sampler.__exit__()
     total_ms = starts[0].elapsed_time(ends[-1])
     kern_ms = statistics.mean(s.elapsed_time(e) for s, e in zip(starts, ends))
     total_ms = shard.max_over_ranks(total_ms, dev)
-    units_tokens = wl.n_windows * wl.heads * wl.N
-    value = shard.aggregate_rate(units_tokens, args.steps, total_ms, ws)
 
     # exact window attention on the same inputs (the computation replaced)
-    esteps = max(3, min(args.steps, 200))
+    esteps = max(3, min(steps, 200))
     for i in range(3):
         step(i, exact=True)
     barrier()
@@ -338,6 +352,44 @@ def run_cuda(args, wl):
     e1.record(stream)
     barrier()
     exact_ms = e0.elapsed_time(e1) / esteps
+
+    peak, peak_kind = _peaks()
+    achieved = io_bytes / (kern_ms * 1e-3) / 1e9
+    mt = MEASURED_TRAFFIC.get(wl.name)
+    traffic = mt["bytes"] if mt and mt["src_hash"] == _kernel_src_hash(mt["files"]) else None
+    units_tokens = wl.n_windows * wl.heads * wl.N
+    rec = {
+        "total_ms": total_ms, "kern_ms": kern_ms, "config": config, "pooled": pooled,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
+                     "bytes_per_launch": io_bytes, "kernel_ms": kern_ms},
+        "comparator": {"kernel": "exact_window_attention", "ms_per_step": exact_ms,
+                       "value": units_tokens / (exact_ms * 1e-3), "speedup": exact_ms / (total_ms / steps)},
+    }
+    return rec, (q, k, v), sets
+
+
+def run_cuda(args, wl):
+    ws, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    binding.lib()  # fail loudly if the library is missing
+
+    clk = ClockSampler(local)
+    rec, (q, k, v), sets = _time_kernel(wl, dev, args.steps, args.warmup, ws, sampler=clk)
+    total_ms, pooled = rec["total_ms"], rec["pooled"]
+    esize = q.element_size()
+    units_tokens = wl.n_windows * wl.heads * wl.N
+    value = shard.aggregate_rate(units_tokens, args.steps, total_ms, ws)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if ws > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize(dev)
 
     # End to end through the public API: every step copies its inputs from
     # pinned host memory, makes the call and reads the output back.  Two
@@ -361,6 +413,7 @@ def run_cuda(args, wl):
     for i in range(2):
         e2e_step(i)
     barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(streams[0])
     streams[1].wait_event(e0)
     for i in range(e2e_steps):
@@ -372,26 +425,31 @@ def run_cuda(args, wl):
     barrier()
     e2e_ms = shard.max_over_ranks(e0.elapsed_time(e1) / e2e_steps, dev)
     e2e_value = shard.aggregate_rate(units_tokens, 1, e2e_ms, ws)
+    del sets, hq, hk, hv, hos
 
-    peak, peak_kind = _peaks()
-    achieved = io_bytes / (kern_ms * 1e-3) / 1e9
-    mt = MEASURED_TRAFFIC.get(wl.name)
-    traffic = mt["bytes"] if mt and mt["src_hash"] == _kernel_src_hash(mt["files"]) else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": config,
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": traffic, "peak_kind": peak_kind,
-                     "bytes_per_launch": io_bytes, "kernel_ms": kern_ms},
-        "comparator": {"kernel": "exact_window_attention", "ms_per_step": exact_ms,
-                       "value": units_tokens / (exact_ms * 1e-3), "speedup": exact_ms / (total_ms / args.steps)},
+        "config": rec["config"], "roofline": rec["roofline"], "comparator": rec["comparator"],
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 3 * q.numel() * esize,
                 "d2h_bytes_per_step": q.numel() * esize, "streams": 2},
         "gpu_launches": args.steps,
         "clocks": clk.summary(),
     }
+    # The other workloads the headline sits beside, each with its own roofline
+    # and comparator (same timing rules; not part of `value`).
+    extra = []
+    for name in ([] if args.no_extra else EXTRA_WORKLOADS.get(wl.name, [])):
+        xwl = workloads.WORKLOADS[name]
+        xrec, _, xsets = _time_kernel(xwl, dev, max(args.steps, 20), args.warmup, ws)
+        del xsets
+        extra.append({"workload": name, "value": shard.aggregate_rate(xwl.units * xwl.N, max(args.steps, 20),
+                                                                      xrec["total_ms"], ws),
+                      "ms_per_step": xrec["total_ms"] / max(args.steps, 20), "config": xrec["config"],
+                      "roofline": xrec["roofline"], "comparator": xrec["comparator"]})
+    if extra:
+        line["extra_workloads"] = extra
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         val, n, passes, dt, cores = _time_oracle(wl, *_oracle_inputs(wl), budget_s=args.cpu_budget)
         line["cpu_baseline"] = {"value": val, "unit": UNIT, "cores": cores, "kind": "oracle",
@@ -552,6 +610,7 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
     ap.add_argument("--cpu-budget", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true", help="time the headline workload only")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
