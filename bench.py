@@ -67,8 +67,8 @@ UNIT = "tokens*heads/s"
 DEFAULT_WORKLOAD = "sr720p-w32-m16-bf16"
 # Reported beside a headline workload, each with its own roofline and comparator.
 EXTRA_WORKLOADS = {
-    "sr720p-w32-m16-bf16": ["sr720p-w16-m16-bf16", "swinir256-bf16"],
-    "sr720p-w16-m16-bf16": ["sr720p-w32-m16-bf16", "swinir256-bf16"],
+    "sr720p-w32-m16-bf16": ["sr720p-w32-m16-bf16-f16", "sr720p-w16-m16-bf16", "swinir256-bf16"],
+    "sr720p-w16-m16-bf16": ["sr720p-w16-m16-bf16-f16", "sr720p-w32-m16-bf16", "swinir256-bf16"],
 }
 
 
@@ -205,6 +205,7 @@ def _config(wl, ws: int):
     cfg = {
         "workload": wl.name, "n_windows": wl.n_windows, "heads": wl.heads, "N": wl.N, "d_h": wl.d, "m": wl.m,
         "iters": wl.iters, "io_dtype": wl.dtype, "landmarks": wl.landmarks, "bias": wl.bias or "none",
+        "factors": "hi+lo 16-bit pairs" if wl.factors == "pairs" else "16-bit (NYSTRA_FACTORS_16)",
         "l2": f"rotating {nsets} input/output sets ({nsets * io_bytes / 1e6:.0f} MB > 3x L2)",
         "parallelism": f"replica x{ws} (independent windows)"}
     if wl.front == "qkv":
@@ -294,11 +295,11 @@ def _time_kernel(wl, dev, steps: int, warmup: int, ws: int, sampler=None):
                                                 *shape, dcode, sptr)
         elif pooled is not None:
             rc = binding.nystra_attention_bias(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
-                                               wl.m, wl.iters, binding.LANDMARKS[wl.landmarks],
+                                               wl.m, wl.iters, binding._lm(wl.landmarks, wl.factors),
                                                *(x.data_ptr() for x in pooled), 1, dcode, sptr)
-        elif wl.landmarks == "patches":
+        elif wl.landmarks == "patches" or wl.factors != "pairs":
             rc = binding.nystra_attention_ex(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
-                                             wl.m, wl.iters, binding.NYSTRA_LANDMARKS_PATCHES, dcode, sptr)
+                                             wl.m, wl.iters, binding._lm(wl.landmarks, wl.factors), dcode, sptr)
         else:
             rc = binding.nystra_attention(qd.data_ptr(), kd.data_ptr(), vd.data_ptr(), od.data_ptr(), *shape,
                                           wl.m, wl.iters, dcode, sptr)
@@ -404,9 +405,10 @@ def run_cuda(args, wl):
         with torch.cuda.stream(streams[i % 2]):
             dq.copy_(hq, non_blocking=True); dk.copy_(hk, non_blocking=True); dv.copy_(hv, non_blocking=True)
             if pooled is None:
-                binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do, landmarks=wl.landmarks)
+                binding.nystra(dq, dk, dv, wl.m, wl.iters, out=do, landmarks=wl.landmarks, factors=wl.factors)
             else:
-                binding.nystra_biased(dq, dk, dv, pooled, wl.m, wl.iters, out=do, landmarks=wl.landmarks)
+                binding.nystra_biased(dq, dk, dv, pooled, wl.m, wl.iters, out=do, landmarks=wl.landmarks,
+                                      factors=wl.factors)
             hos[i % 2].copy_(do, non_blocking=True)
 
     e2e_steps = max(4, min(args.steps, 50))
@@ -489,7 +491,7 @@ def run_cuda_qkv(args, wl):
     def step(i):
         xd, od = sets[i % nsets]
         rc = binding.nystra_attention_qkv(xd.data_ptr(), wd.data_ptr(), 0, od.data_ptr(), wl.n_windows, wl.heads,
-                                          wl.N, wl.d, wl.m, wl.iters, binding.LANDMARKS[wl.landmarks], *bp,
+                                          wl.N, wl.d, wl.m, wl.iters, binding._lm(wl.landmarks, wl.factors), *bp,
                                           1 if pooled is not None else 0, dcode, sptr)
         if rc != 0:
             raise binding.NystraError(rc, "bench step")
@@ -550,7 +552,8 @@ def run_cuda_qkv(args, wl):
         xd, od = sets[i % 2]
         with torch.cuda.stream(streams[i % 2]):
             xd.copy_(hx, non_blocking=True)
-            binding.nystra_qkv(xd, wd, wl.heads, wl.m, wl.iters, pooled=pooled, out=od, landmarks=wl.landmarks)
+            binding.nystra_qkv(xd, wd, wl.heads, wl.m, wl.iters, pooled=pooled, out=od, landmarks=wl.landmarks,
+                               factors=wl.factors)
             hos[i % 2].copy_(od, non_blocking=True)
 
     e2e_steps = max(4, min(args.steps, 50))

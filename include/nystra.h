@@ -67,6 +67,21 @@ typedef enum { NYSTRA_F32 = 0, NYSTRA_BF16 = 1, NYSTRA_F16 = 2 } nystra_dtype;
  *            j = patch (j / p, j % p). */
 typedef enum { NYSTRA_LANDMARKS_SEGMENTS = 0, NYSTRA_LANDMARKS_PATCHES = 1 } nystra_landmarks;
 
+/* Option flag, OR-ed into the `landmarks` argument of nystra_attention_ex,
+ * nystra_attention_bias and nystra_attention_qkv (not nystra_pool_bias or
+ * nystra_debug_stages, which reject it with NYSTRA_EINVAL):
+ *  FACTORS_16  16-bit I/O on the tensor cores rounds the derived factors
+ *              (landmarks, G_L^n, G_U^n, Y) to the I/O type instead of
+ *              carrying each as a hi + lo pair of that type.  One MMA per
+ *              product instead of two or three: faster (about 1.2x on 32x32
+ *              windows), and within the 2e-2 bar only while attention stays
+ *              soft (logits q.k/sqrt(d_h) of standard deviation up to about
+ *              1.5); sharper attention makes G_A^n ill-conditioned and the
+ *              method amplifies that rounding.  No effect on fp32 I/O or the
+ *              SIMT path.  Not a step of the paper: a speed/accuracy choice of
+ *              this implementation. */
+#define NYSTRA_FACTORS_16 16
+
 /* Status codes returned by every entry point (0 = success, negative = error). */
 enum {
     NYSTRA_OK = 0,

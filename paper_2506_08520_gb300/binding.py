@@ -18,6 +18,14 @@ NYSTRA_F32, NYSTRA_BF16, NYSTRA_F16 = 0, 1, 2
 NYSTRA_OK, NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH, NYSTRA_ETIMEOUT, NYSTRA_EDEVICE = 0, -1, -2, -3, -4, -5
 NYSTRA_LANDMARKS_SEGMENTS, NYSTRA_LANDMARKS_PATCHES = 0, 1
 LANDMARKS = {"segments": NYSTRA_LANDMARKS_SEGMENTS, "patches": NYSTRA_LANDMARKS_PATCHES}
+# Option flag OR-ed into the landmarks argument: derived factors rounded to
+# the 16-bit I/O type (faster, accurate only for soft attention; nystra.h).
+NYSTRA_FACTORS_16 = 16
+FACTORS = {"pairs": 0, "16": NYSTRA_FACTORS_16}
+
+
+def _lm(landmarks: str, factors: str = "pairs") -> int:
+    return LANDMARKS[landmarks] | FACTORS[factors]
 MAX_N, MAX_DH, MAX_M, MAX_ITERS = 1024, 64, 64, 100
 QKV_MAX_C = 352
 
@@ -176,19 +184,22 @@ def _check(q, k, v, out):
 
 
 def nystra(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int = 16, iters: int = 6,
-           out: torch.Tensor | None = None, stream=None, landmarks: str = "segments") -> torch.Tensor:
+           out: torch.Tensor | None = None, stream=None, landmarks: str = "segments",
+           factors: str = "pairs") -> torch.Tensor:
     """PnP-Nystra attention of device tensors ``[n_windows, heads, N, d_h]``;
-    ``landmarks`` is "segments" (default) or "patches" (square patches)."""
+    ``landmarks`` is "segments" (default) or "patches" (square patches);
+    ``factors`` "pairs" (default: derived factors as 16-bit hi + lo pairs) or
+    "16" (rounded to the 16-bit I/O type, NYSTRA_FACTORS_16)."""
     out = torch.empty_like(q) if out is None else out
     _check(q, k, v, out)
     nw, h, N, d = _geometry(q)
     with torch.cuda.device(q.device):
-        if landmarks == "segments":
+        if landmarks == "segments" and factors == "pairs":
             rc = nystra_attention(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
                                   m, iters, _DTYPE_CODE[q.dtype], _stream_ptr(stream))
         else:
             rc = nystra_attention_ex(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d,
-                                     m, iters, LANDMARKS[landmarks], _DTYPE_CODE[q.dtype], _stream_ptr(stream))
+                                     m, iters, _lm(landmarks, factors), _DTYPE_CODE[q.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention")
     return out
@@ -254,7 +265,8 @@ def pool_bias(bias: torch.Tensor, m: int, landmarks: str = "segments", stream=No
 
 
 def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: int = 16, iters: int = 6,
-                  out: torch.Tensor | None = None, stream=None, landmarks: str = "segments") -> torch.Tensor:
+                  out: torch.Tensor | None = None, stream=None, landmarks: str = "segments",
+                  factors: str = "pairs") -> torch.Tensor:
     """PnP-Nystra with a score bias already pooled by ``pool_bias``: blocks of
     shape ``[heads, ...]`` (shared by all windows) or ``[n_windows, heads, ...]``."""
     out = torch.empty_like(q) if out is None else out
@@ -264,7 +276,7 @@ def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: 
     bw = bL.numel() // (h * N * m)
     with torch.cuda.device(q.device):
         rc = nystra_attention_bias(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d, m, iters,
-                                   LANDMARKS[landmarks], bL.data_ptr(), bU.data_ptr(), bA.data_ptr(), bw,
+                                   _lm(landmarks, factors), bL.data_ptr(), bU.data_ptr(), bA.data_ptr(), bw,
                                    _DTYPE_CODE[q.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention_bias")
@@ -273,7 +285,7 @@ def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: 
 
 def nystra_qkv(x: torch.Tensor, w_qkv: torch.Tensor, heads: int, m: int = 16, iters: int = 6,
                b_qkv: torch.Tensor | None = None, pooled=None, out: torch.Tensor | None = None, stream=None,
-               landmarks: str = "segments") -> torch.Tensor:
+               landmarks: str = "segments", factors: str = "pairs") -> torch.Tensor:
     """Fused projection + PnP-Nystra: tokens ``x`` ``[n_windows, N, C]``, weights
     ``w_qkv`` ``[3C, C]`` (a linear layer's weight: Q rows, then K, then V),
     optional fp32 bias ``b_qkv`` ``[3C]`` and pooled score bias (as for
@@ -306,7 +318,7 @@ def nystra_qkv(x: torch.Tensor, w_qkv: torch.Tensor, heads: int, m: int = 16, it
         bw = pooled[0].numel() // (heads * N * m)
     with torch.cuda.device(x.device):
         rc = nystra_attention_qkv(x.data_ptr(), w_qkv.data_ptr(), bp, out.data_ptr(), nw, heads, N, d, m, iters,
-                                  LANDMARKS[landmarks], bL, bU, bA, bw, _DTYPE_CODE[x.dtype], _stream_ptr(stream))
+                                  _lm(landmarks, factors), bL, bU, bA, bw, _DTYPE_CODE[x.dtype], _stream_ptr(stream))
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention_qkv")
     return out

@@ -2,6 +2,8 @@
 // Declarations and the full contract are in include/nystra.h.
 #include <stdint.h>
 
+#include <atomic>
+
 #include "common.cuh"
 #include "nystra.h"
 
@@ -43,6 +45,36 @@ int check_common(const void* q, const void* k, const void* v, void* out, int n_w
     return NYSTRA_OK;
 }
 
+// Whether the current device is an sm_103 GPU (the kernels' only target);
+// false when there is no usable device.  Cached per device ordinal.
+bool device_ok() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= nystra::kMaxDevices) {
+        (void)cudaGetLastError();
+        return false;
+    }
+    static std::atomic<int> cache[nystra::kMaxDevices];  // 0 unknown, 1 sm_103, 2 other
+    int c = cache[dev].load(std::memory_order_relaxed);
+    if (c == 0) {
+        int major = 0, minor = 0;
+        const bool ok = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) == cudaSuccess &&
+                        cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) == cudaSuccess &&
+                        major == 10 && minor == 3;
+        if (!ok) (void)cudaGetLastError();
+        c = ok ? 1 : 2;
+        cache[dev].store(c, std::memory_order_relaxed);
+    }
+    return c == 1;
+}
+
+// Landmark pooling and option flags of the `landmarks` argument.
+constexpr int kPoolMask = 15;
+bool flags_ok(int landmarks) {
+    const int pool = landmarks & kPoolMask, rest = landmarks & ~kPoolMask;
+    return (pool == NYSTRA_LANDMARKS_SEGMENTS || pool == NYSTRA_LANDMARKS_PATCHES) &&
+           (rest == 0 || rest == NYSTRA_FACTORS_16);
+}
+
 // Integer square root of n, or -1 if n is not a perfect square.
 int exact_sqrt(int n) {
     int r = 0;
@@ -61,14 +93,16 @@ int nystra_call(const void* q, const void* k, const void* v, void* out, int n_wi
     if (rc != NYSTRA_OK) return rc;
     if (m < 1 || m > N || m > NYSTRA_MAX_M || N % m != 0) return NYSTRA_EINVAL;
     if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
-    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
-    const bool patches = landmarks == NYSTRA_LANDMARKS_PATCHES;
+    if (!flags_ok(landmarks)) return NYSTRA_EINVAL;
+    const bool patches = (landmarks & kPoolMask) == NYSTRA_LANDMARKS_PATCHES;
+    const bool f16 = (landmarks & NYSTRA_FACTORS_16) != 0;  // derived factors rounded to 16 bits
     if (patches) {  // a square grid of square patches must tile the square window
         const int w = exact_sqrt(N), p = exact_sqrt(m);
         if (w < 0 || p < 0 || w % p != 0) return NYSTRA_EINVAL;
     }
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
+    if (!device_ok()) return NYSTRA_EDEVICE;
     const cudaStream_t s = (cudaStream_t)stream;
     // fp32 I/O on the tensor cores: 8x8 windows, m <= 16, at most the paper's 6
     // iterations (beyond them the fp16-split iteration's round-off, amplified
@@ -87,12 +121,18 @@ int nystra_call(const void* q, const void* k, const void* v, void* out, int n_wi
     const nystra::NystraBias* bp = biased ? &bias : nullptr;
     const int pool = patches ? 1 : 0;
     cudaError_t e;
+    // NYSTRA_FACTORS_16 selects the kernels whose derived factors are 16-bit
+    // (16-bit I/O on the tensor cores; the SIMT path is fp32 throughout).
+    const bool s16 = f16 && io16;
     if (tc && N == 64)
-        e = nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
+        e = s16 ? nystra_host::launch_nystra_tc_n64_s16(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp)
+                : nystra_host::launch_nystra_tc_n64(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else if (tc && N == 256)
-        e = nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
+        e = s16 ? nystra_host::launch_nystra_tc_n256_s16(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp)
+                : nystra_host::launch_nystra_tc_n256(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else if (tc && N == 1024)
-        e = nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
+        e = s16 ? nystra_host::launch_nystra_tc_n1024_s16(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp)
+                : nystra_host::launch_nystra_tc_n1024(q, k, v, out, units, d_h, m, iters, pool, dtype, s, bp);
     else
         e = nystra_host::launch_nystra_generic(q, k, v, out, units, N, d_h, m, iters, pool, dtype, s, bias);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
@@ -123,6 +163,7 @@ int nystra_pool_bias(const float* bias, int n_bias, int N, int m, int landmarks,
     if (overlaps2(bias, in, bias_L, nm) || overlaps2(bias, in, bias_U, nm) || overlaps2(bias, in, bias_A, mm) ||
         overlaps2(bias_L, nm, bias_U, nm) || overlaps2(bias_L, nm, bias_A, mm) || overlaps2(bias_U, nm, bias_A, mm))
         return NYSTRA_EINVAL;
+    if (!device_ok()) return NYSTRA_EDEVICE;
     const cudaError_t e = nystra_host::launch_pool_bias(bias, n_bias, N, m, landmarks, bias_L, bias_U, bias_A,
                                                         (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
@@ -165,8 +206,10 @@ int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, v
     if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
     if (N != 64 || d_h < 2 || d_h > 32 || d_h % 2 != 0 || (m != 8 && m != 16)) return NYSTRA_EINVAL;
     if (iters < 0 || iters > 12) return NYSTRA_EINVAL;
-    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
-    if (landmarks == NYSTRA_LANDMARKS_PATCHES && m != 16) return NYSTRA_EINVAL;
+    if (!flags_ok(landmarks)) return NYSTRA_EINVAL;
+    const bool patches = (landmarks & kPoolMask) == NYSTRA_LANDMARKS_PATCHES;
+    const bool s16 = (landmarks & NYSTRA_FACTORS_16) != 0;
+    if (patches && m != 16) return NYSTRA_EINVAL;
     if ((long long)heads * d_h > NYSTRA_QKV_MAX_C) return NYSTRA_EINVAL;
     if ((long long)n_windows * heads == 0) return NYSTRA_OK;
     const size_t C = (size_t)heads * d_h;
@@ -190,13 +233,20 @@ int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, v
         b.per_window = bias_windows != 1 ? 1 : 0;
     }
     const nystra::NystraBias* bp = bias_L ? &b : nullptr;
-    const int pool = landmarks == NYSTRA_LANDMARKS_PATCHES ? 1 : 0;
-    const cudaError_t e =
-        dtype == NYSTRA_BF16
-            ? nystra_host::launch_nystra_qkv_bf16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
-                                                  (cudaStream_t)stream, bp)
-            : nystra_host::launch_nystra_qkv_f16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
-                                                 (cudaStream_t)stream, bp);
+    const int pool = patches ? 1 : 0;
+    if (!device_ok()) return NYSTRA_EDEVICE;
+    const cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e;
+    if (dtype == NYSTRA_BF16)
+        e = s16 ? nystra_host::launch_nystra_qkv_bf16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                          pool, st, bp)
+                : nystra_host::launch_nystra_qkv_bf16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
+                                                      st, bp);
+    else
+        e = s16 ? nystra_host::launch_nystra_qkv_f16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                         pool, st, bp)
+                : nystra_host::launch_nystra_qkv_f16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
+                                                     st, bp);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
@@ -206,6 +256,7 @@ int exact_window_attention(const void* q, const void* k, const void* v, void* ou
     if (rc != NYSTRA_OK) return rc;
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
+    if (!device_ok()) return NYSTRA_EDEVICE;
     cudaError_t e = nystra_host::exact_tc_supports(N, d_h, dtype)
                         ? nystra_host::launch_exact_tc(q, k, v, out, units, N, d_h, dtype, (cudaStream_t)stream)
                         : nystra_host::launch_exact_generic(q, k, v, out, units, N, d_h, dtype,
@@ -254,6 +305,7 @@ int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windo
     if (n_windows < 0 || heads < 0 || unit < 0 || unit >= (long long)n_windows * heads) return NYSTRA_EINVAL;
     if (!q || !k || !v || !dump) return NYSTRA_EINVAL;
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(dump)) return NYSTRA_EINVAL;
+    if (!device_ok()) return NYSTRA_EDEVICE;
     const cudaError_t e = nystra_host::launch_debug_stages(q, k, v, unit, d_h, m, iters, landmarks, dtype, dump,
                                                            (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
@@ -261,6 +313,7 @@ int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windo
 
 int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream) {
     if (limit_ns < 1000ull || limit_ns > 1000000000ull) return NYSTRA_EINVAL;
+    if (!device_ok()) return NYSTRA_EDEVICE;
     const cudaError_t e = nystra_host::launch_debug_wait(limit_ns, (cudaStream_t)stream);
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
@@ -272,10 +325,11 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[7])(cudaError_t*) = {take_fault_word_tc_n64,    take_fault_word_tc_n256,
-                                                   take_fault_word_tc_n1024,  take_fault_word_exact_tc,
-                                                   take_fault_word_debug,     take_fault_word_qkv_bf16,
-                                                   take_fault_word_qkv_f16};
+    unsigned int (*const take[12])(cudaError_t*) = {
+        take_fault_word_tc_n64,      take_fault_word_tc_n256,      take_fault_word_tc_n1024,
+        take_fault_word_tc_n64_s16,  take_fault_word_tc_n256_s16,  take_fault_word_tc_n1024_s16,
+        take_fault_word_exact_tc,    take_fault_word_debug,        take_fault_word_qkv_bf16,
+        take_fault_word_qkv_f16,     take_fault_word_qkv_bf16_s16, take_fault_word_qkv_f16_s16};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

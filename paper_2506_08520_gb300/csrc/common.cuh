@@ -23,6 +23,23 @@ template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(flo
 }
 template <> __device__ __forceinline__ __half from_f32<__half>(float x) { return __float2half_rn(x); }
 
+// 16-bit I/O whose derived factors (landmarks, G_L^n, G_U^n, Y) are rounded
+// to that 16-bit type instead of being carried as hi + lo pairs: the faster,
+// less accurate arithmetic a caller selects with NYSTRA_FACTORS_16.  Same
+// size and bits as T; only the kernels' operand policies differ (Opnd).
+template <typename T>
+struct Single16 {
+    T v;
+};
+__device__ __forceinline__ float to_f32(Single16<__nv_bfloat16> x) { return __bfloat162float(x.v); }
+__device__ __forceinline__ float to_f32(Single16<__half> x) { return __half2float(x.v); }
+template <> __device__ __forceinline__ Single16<__nv_bfloat16> from_f32<Single16<__nv_bfloat16>>(float x) {
+    return {__float2bfloat16_rn(x)};
+}
+template <> __device__ __forceinline__ Single16<__half> from_f32<Single16<__half>>(float x) {
+    return {__float2half_rn(x)};
+}
+
 template <typename T> __device__ __forceinline__ float ldg_f32(const T* p) { return to_f32(p[0]); }
 template <> __device__ __forceinline__ float ldg_f32<float>(const float* p) { return __ldg(p); }
 
@@ -90,9 +107,23 @@ cudaError_t launch_nystra_tc_n256(const void* q, const void* k, const void* v, v
 cudaError_t launch_nystra_tc_n1024(const void* q, const void* k, const void* v, void* out, long long n_units,
                                    int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
                                  const nystra::NystraBias* bias = nullptr);
+// The same with the derived factors rounded to 16 bits (Single16; 16-bit I/O
+// only, nystra_tc_n*_s16.cu).
+cudaError_t launch_nystra_tc_n64_s16(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                     int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                     const nystra::NystraBias* bias = nullptr);
+cudaError_t launch_nystra_tc_n256_s16(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                      int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                      const nystra::NystraBias* bias = nullptr);
+cudaError_t launch_nystra_tc_n1024_s16(const void* q, const void* k, const void* v, void* out, long long n_units,
+                                       int d, int m, int iters, int pool, int dtype, cudaStream_t stream,
+                                       const nystra::NystraBias* bias = nullptr);
 unsigned int take_fault_word_tc_n64(cudaError_t* err);
 unsigned int take_fault_word_tc_n256(cudaError_t* err);
 unsigned int take_fault_word_tc_n1024(cudaError_t* err);
+unsigned int take_fault_word_tc_n64_s16(cudaError_t* err);
+unsigned int take_fault_word_tc_n256_s16(cudaError_t* err);
+unsigned int take_fault_word_tc_n1024_s16(cudaError_t* err);
 // Tensor-core exact attention, 16-bit I/O, N in {64, 256, 1024}, even d_h <= 32 (exact_tc.cu).
 bool exact_tc_supports(int N, int d, int dtype);
 cudaError_t launch_exact_tc(const void* q, const void* k, const void* v, void* out, long long n_units, int N,
@@ -110,8 +141,16 @@ cudaError_t launch_nystra_qkv_bf16(const void* x, const void* wqkv, const float*
 cudaError_t launch_nystra_qkv_f16(const void* x, const void* wqkv, const float* bqkv, void* out,
                                   long long n_windows, int heads, int d, int m, int iters, int pool,
                                   cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkv_bf16_s16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                       long long n_windows, int heads, int d, int m, int iters, int pool,
+                                       cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkv_f16_s16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                      long long n_windows, int heads, int d, int m, int iters, int pool,
+                                      cudaStream_t stream, const nystra::NystraBias* bias);
 unsigned int take_fault_word_qkv_bf16(cudaError_t* err);
 unsigned int take_fault_word_qkv_f16(cudaError_t* err);
+unsigned int take_fault_word_qkv_bf16_s16(cudaError_t* err);
+unsigned int take_fault_word_qkv_f16_s16(cudaError_t* err);
 // Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
 long long debug_stages_size(int N, int d, int m);
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,

@@ -12,29 +12,33 @@ namespace nystra {
 namespace tc {
 namespace {
 
-// Two elements of an operand register, widened to fp32.
-template <typename T>
-__device__ __forceinline__ float2 reg_f2(uint32_t r) {
-    return Mma16<T>::unpack(r);
-}
+// Two elements of a derived operand register (hi + lo pair in the MMA type
+// of T: bf16 for fp32 I/O), widened to fp32.
 template <typename T>
 __device__ __forceinline__ float2 reg_f2(RegPair r) {
-    const float2 h = Mma16<__nv_bfloat16>::unpack(r.hi), l = Mma16<__nv_bfloat16>::unpack(r.lo);
+    using Op = typename Opnd<T>::Op;
+    const float2 h = Op::unpack(r.hi), l = Op::unpack(r.lo);
     return make_float2(h.x + l.x, h.y + l.y);
+}
+// A stored derived value (landmark) widened to fp32.
+template <typename T>
+__device__ __forceinline__ float lm_f32(const T* p) {
+    if constexpr (sizeof(T) == 2) return to_f32(p[0]) + to_f32(p[LmS<T>::LO]);
+    else return p[0];
 }
 
 template <typename T, int M, int NCOL>
 struct StageLayout {
     static constexpr int ES = (int)sizeof(T);
-    static constexpr int DS = 32, MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int DS = 32, MP = 16, LS = LmS<T>::LS, WS = NCOL + 4;
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;
     static constexpr size_t QKV = 0;                                   // Q, K, V rows (64 x d each)
     static constexpr size_t QB = QKV + 3 * 64 * DS * ES;               // Qbar, MP x LS
-    static constexpr size_t KB = QB + MP * LS * ES;                    // Kbar, MP x LS
-    static constexpr size_t GLF = (KB + MP * LS * ES + 15) / 16 * 16;  // parked G_L^n fragments
+    static constexpr size_t KB = QB + LmS<T>::bytes(MP);               // Kbar, MP x LS
+    static constexpr size_t GLF = (KB + LmS<T>::bytes(MP) + 15) / 16 * 16;  // parked G_L^n fragments
     static constexpr size_t W = GLF + 4 * KTL * 32 * GlPark<T, M>::BYTES;  // fp32 MP x WS
-    static constexpr size_t YT = W + MP * WS * 4;                      // Y^T, NCOL x YS
-    static constexpr size_t OUT = (YT + NCOL * YS * ES + 15) / 16 * 16;  // output rows, 64 x d
+    static constexpr size_t YT = W + MP * WS * 4;                      // Y^T (YtS layout)
+    static constexpr size_t OUT = (YT + YtS<T, M>::bytes(NCOL) + 15) / 16 * 16;  // output rows, 64 x d
     static constexpr size_t DBG = OUT + 64 * DS * ES;                  // core dump: 2 M^2 + M NCOL floats
     static constexpr size_t BYTES = DBG + (2 * M * M + M * NCOL) * 4;
 };
@@ -89,22 +93,19 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
     landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
     landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
     if constexpr (M < P::MP) {
-        for (int idx = lane; idx < (P::MP - M) * 32; idx += 32) {
-            const int jr = M + (idx >> 5), e = idx & 31;
-            qbar[jr * P::LS + e] = from_f32<T>(0.f);
-            kbar[jr * P::LS + e] = from_f32<T>(0.f);
-        }
+        landmarks_zero<T>(qbar, M, P::MP, lane, 32);
+        landmarks_zero<T>(kbar, M, P::MP, lane, 32);
     }
     __syncwarp();
     for (int i = lane; i < M * d; i += 32) {
-        dump[off.qbar + i] = to_f32(qbar[(i / d) * P::LS + i % d]);
-        dump[off.kbar + i] = to_f32(kbar[(i / d) * P::LS + i % d]);
+        dump[off.qbar + i] = lm_f32<T>(qbar + (i / d) * P::LS + i % d);
+        dump[off.kbar + i] = lm_f32<T>(kbar + (i / d) * P::LS + i % d);
     }
 
     // steps 2-3: S_L, m_L, G_L^n (the operand registers of O = G_L^n Y)
 #pragma unroll
     for (int tm = 0; tm < 4; ++tm) {
-        typename Opnd<T>::Reg f[P::KTL][4];
+        typename Opnd<T>::DReg f[P::KTL][4];
         gl_tile<T, M, P::KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
         for (int kk = 0; kk < P::KTL; ++kk) {

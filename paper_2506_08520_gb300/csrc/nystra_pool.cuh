@@ -7,8 +7,8 @@
 // kernel does with one warp per unit, but a warp's Q, K and V rows are only
 // needed by its front phase (landmarks, S_L and G_L^n, S_U and W), while the
 // core (m x m iteration) and the output phase run on warp-private state.  A
-// CTA therefore keeps NW = 16 warps on NS = 8 shared staging buffers (8 on 4
-// for fp32 I/O) instead of one buffer per warp: warp w always uses stage w mod NS, alternating with
+// CTA therefore keeps NW warps on NS = NW / 2 shared staging buffers (as many
+// as fit: 12 on 6) instead of one buffer per warp: warp w always uses stage w mod NS, alternating with
 // its partner warp (w + NS) mod NW.  When a warp's front phase has consumed
 // the stage it issues the bulk copies of the partner's next unit into it, so
 // the copy overlaps the warp's own core and output.  Each warp waits on its
@@ -31,25 +31,31 @@ namespace tc {
 template <typename T, int M, int NCOL>
 struct PoolLayout {
     static constexpr int ES = (int)sizeof(T);          // bytes per I/O element
-    static constexpr int NW = ES == 2 ? 16 : 8;        // warps
-    static constexpr int NS = NW / 2;                  // shared stages
     static constexpr int DS = (NCOL == 32) ? 30 : 32;  // staged row width bound (d_h <= DS)
-    static constexpr int MP = 16, LS = 40, WS = NCOL + 4, YS = 24;
+    static constexpr int MP = 16, LS = LmS<T>::LS, WS = NCOL + 4, YS = YtS<T, M>::YS;
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;  // k-steps of O = G_L^n Y
     static constexpr size_t STAGE = 3 * 64 * DS * ES;   // Q, K, V rows of one unit
     // warp-private layout
     static constexpr size_t GLF = 0;
     static constexpr size_t QB = GLF + 4 * KTL * 32 * GlPark<T, M>::BYTES;
-    static constexpr size_t KB = QB + MP * LS * ES;
-    static constexpr size_t W = KB + MP * LS * ES;  // fp32 MP x NCOL, row stride WS
-    static constexpr size_t YT = QB;                // Y^T: written after the core's last landmark read
-    static constexpr size_t YT_BYTES = ((NCOL * YS * ES + 15) / 16) * 16;
+    static constexpr size_t KB = QB + LmS<T>::bytes(MP);
+    static constexpr size_t W = KB + LmS<T>::bytes(MP);  // fp32 MP x NCOL, row stride WS
+    static constexpr size_t YT = QB;                     // Y^T: written after the core's last landmark read
+    static constexpr size_t YT_BYTES = YtS<T, M>::bytes(NCOL);
     static constexpr size_t OUT = YT + YT_BYTES;  // output tile: Kbar's tail and W are dead by then
     static constexpr size_t END_A = W + MP * WS * 4;
     static constexpr size_t END_B = OUT + 64 * DS * ES;
     static constexpr size_t BAR = (((END_A > END_B) ? END_A : END_B) + 15) / 16 * 16;
     static constexpr size_t CNT = BAR + 8;  // copies issued to this warp (fault path)
     static constexpr size_t PRIV = ((BAR + 16 + 127) / 128) * 128;
+    // warps: the most (up to 16 for 16-bit I/O, 8 for fp32), in pairs sharing a stage, that fit
+    static constexpr int fit_warps() {
+        int n = ES == 2 ? 16 : 8;
+        while (n > 2 && (size_t)(n / 2) * STAGE + (size_t)n * PRIV > kSmemLimit) n -= 2;
+        return n;
+    }
+    static constexpr int NW = fit_warps();
+    static constexpr int NS = NW / 2;  // shared stages
     static constexpr size_t BYTES = NS * STAGE + NW * PRIV;
     static_assert(NW == 2 * NS, "each stage alternates between two warps");
     static_assert(YT + YT_BYTES <= W, "Y^T must not overlap W (read while Y^T is produced)");
@@ -128,17 +134,14 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
         landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
         if constexpr (M < P::MP) {  // zero the padding landmark rows
-            for (int idx = lane; idx < (P::MP - M) * 32; idx += 32) {
-                const int jr = M + (idx >> 5), e = idx & 31;
-                qbar[jr * P::LS + e] = from_f32<T>(0.f);
-                kbar[jr * P::LS + e] = from_f32<T>(0.f);
-            }
+            landmarks_zero<T>(qbar, M, P::MP, lane, 32);
+            landmarks_zero<T>(kbar, M, P::MP, lane, 32);
         }
         __syncwarp();
         // ---------------- front: S_L, G_L^n fragments (parked) ----------------
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
-            typename Opnd<T>::Reg f[P::KTL][4];
+            typename Opnd<T>::DReg f[P::KTL][4];
             gl_tile<T, M, P::KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
                                         BIAS ? bLu + (16 * tm + g) * M : nullptr);
 #pragma unroll

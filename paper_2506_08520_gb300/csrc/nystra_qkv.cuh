@@ -46,10 +46,12 @@ namespace tc {
 template <typename T, int M, int NCOL, bool PAIR>
 struct QkvLayout {
     using PL = PoolLayout<T, M, NCOL>;
-    static constexpr int NW = PAIR ? 12 : 8;         // warps per CTA
-    static constexpr int NS = PAIR ? NW / 2 : NW;    // Q/K/V stages
     static constexpr size_t HDR = 128;               // the shared stages' mbarriers
     static constexpr size_t FRAG = 3 * 4 * 32 * 8;   // weight fragments per k-step: 3 blocks x 4 n-tiles x 32 lanes x 8 B
+    // warps per CTA: 12 on 6 shared stages (C <= 64), else as many with a
+    // stage each as fit beside the widest projection's weights (C = 352)
+    static constexpr int NW = PAIR ? 12 : (int)((kSmemLimit - HDR - 22 * FRAG) / (PL::STAGE + PL::PRIV));
+    static constexpr int NS = PAIR ? NW / 2 : NW;    // Q/K/V stages
     // k-steps ks = ceil(C / 16): header, weights, stages, warp-private state
     static constexpr size_t stages_at(int ks) { return HDR + (size_t)ks * FRAG; }
     static constexpr size_t priv_at(int ks) { return stages_at(ks) + NS * PL::STAGE; }
@@ -237,17 +239,14 @@ nystra_qkv_kernel(const T* __restrict__ x, const T* __restrict__ wqkv, const flo
         landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
         landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
         if constexpr (M < PL::MP) {  // zero the padding landmark rows
-            for (int idx = lane; idx < (PL::MP - M) * 32; idx += 32) {
-                const int jr = M + (idx >> 5), e = idx & 31;
-                qbar[jr * PL::LS + e] = from_f32<T>(0.f);
-                kbar[jr * PL::LS + e] = from_f32<T>(0.f);
-            }
+            landmarks_zero<T>(qbar, M, PL::MP, lane, 32);
+            landmarks_zero<T>(kbar, M, PL::MP, lane, 32);
         }
         __syncwarp();
         // ---------------- front: S_L, G_L^n fragments (parked) ----------------
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
-            typename Opnd<T>::Reg f[PL::KTL][4];
+            typename Opnd<T>::DReg f[PL::KTL][4];
             gl_tile<T, M, PL::KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
                                          BIAS ? bLu + (16 * tm + g) * M : nullptr);
 #pragma unroll

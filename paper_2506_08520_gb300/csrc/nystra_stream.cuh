@@ -33,25 +33,29 @@
 namespace nystra {
 namespace tc {
 
-template <int M, int NCOL>
+template <typename T, int M, int NCOL>
 struct StreamLayout {
     static constexpr int NT = 4, TPW = 256, N = NT * TPW, CH = 64, NCHK = TPW / CH;
     static constexpr int CWN = M > 16 ? M / 16 : 1;  // core warps (m = 32: distributed core)
     static constexpr int MT = (M + 15) / 16;         // landmark m-tiles
     static constexpr int DS = (NCOL == 32) ? 30 : 32;
-    static constexpr int MP = MT * 16, LS = 40, WS = NCOL + 4, YS = MP + 8;
+    static constexpr int MP = MT * 16, LS = LmS<T>::LS, WS = NCOL + 4;
     static constexpr int L = N / M, LPW = TPW / L;  // tokens per segment, segments per token warp
     static constexpr size_t XB = (size_t)CH * DS * 2;  // one tensor's chunk
     static constexpr size_t SLOT = 2 * XB;             // K and V (Q uses the first half)
     static constexpr size_t WPB = (size_t)MP * WS * 4 + MP * 4;  // W partial, row maxima
     static_assert(WPB <= SLOT, "the W partial lives in the slot of the last K/V chunk");
-    // per-unit state
+    // per-unit state.  Y^T is written by the core once it has read Qbar, W
+    // and m_U for the last time, so it overlays them; a unit's Qbar is next
+    // written two units later, after a token-warp barrier that follows every
+    // warp's output pass of the unit (see the task order).
     static constexpr size_t B_QB = 0;
-    static constexpr size_t B_KB = B_QB + MP * LS * 2;
-    static constexpr size_t B_W = B_KB + MP * LS * 2;
+    static constexpr size_t B_W = B_QB + LmS<T>::bytes(MP);
     static constexpr size_t B_MU = B_W + MP * WS * 4;
-    static constexpr size_t B_YT = B_MU + MP * 4;
-    static constexpr size_t BUF = ((B_YT + NCOL * YS * 2 + 127) / 128) * 128;
+    static constexpr size_t B_KB = ((B_MU + MP * 4 + 15) / 16) * 16;
+    static constexpr size_t B_YT = B_QB;
+    static constexpr size_t BUF = ((B_KB + LmS<T>::bytes(MP) + 127) / 128) * 128;
+    static_assert(YtS<T, M>::bytes(NCOL) <= B_KB, "Y^T must fit over Qbar, W and m_U");
     static constexpr size_t SCR = CWN > 1 ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0;
     template <int S>
     struct Team {
@@ -66,7 +70,7 @@ struct StreamLayout {
     // else two with two-deep
     static constexpr bool kThree = 3 * Team<2>::BYTES <= kSmemLimit;
     static constexpr bool kDeep = 2 * Team<3>::BYTES <= kSmemLimit;
-    static constexpr int TEAMS = kThree ? 3 : 2;
+    static constexpr int TEAMS = kThree ? 3 : (2 * Team<2>::BYTES <= kSmemLimit ? 2 : 1);
     static constexpr int NSLOT = kThree ? 2 : (kDeep ? 3 : 2);
     using TL = Team<NSLOT>;
     static constexpr size_t TEAM = TL::BYTES;
@@ -105,16 +109,16 @@ __device__ __forceinline__ StreamTask stream_task(int v, int count) {
 }
 
 template <typename T, int M, int NCOL, int DC, int PW, bool BIAS>
-__global__ void __launch_bounds__(StreamLayout<M, NCOL>::TEAMS * StreamLayout<M, NCOL>::WARPS * 32, 1)
+__global__ void __launch_bounds__(StreamLayout<T, M, NCOL>::TEAMS * StreamLayout<T, M, NCOL>::WARPS * 32, 1)
 nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                      T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault,
                      NystraBias bias) {
     static_assert(!BIAS || M <= 16, "a score bias runs with the one-warp core");
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
-    using Lay = StreamLayout<M, NCOL>;
+    using Lay = StreamLayout<T, M, NCOL>;
     using TL = typename Lay::TL;
-    using R = typename Opnd<T>::Reg;
-    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
+    using R = typename Opnd<T>::DReg;
+    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, WS = Lay::WS,
                   NSLOT = Lay::NSLOT, L = Lay::L, LPW = Lay::LPW, NTO = NCOL / 8, MT = Lay::MT;
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -151,8 +155,8 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                                          Lay::B_QB);
             T* kb = reinterpret_cast<T*>(smem_raw + (size_t)tm * Lay::TEAM + TL::T_BUF + (size_t)b * Lay::BUF +
                                          Lay::B_KB);
-            qb[(M + (e >> 5)) * LS + (e & 31)] = from_f32<T>(0.f);
-            kb[(M + (e >> 5)) * LS + (e & 31)] = from_f32<T>(0.f);
+            landmarks_zero<T>(qb, M + (e >> 5), M + (e >> 5) + 1, e & 31, 32);
+            landmarks_zero<T>(kb, M + (e >> 5), M + (e >> 5) + 1, e & 31, 32);
         }
     }
     __syncthreads();
@@ -258,6 +262,11 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                 for (int mf = 0; mf < 2; ++mf) cq[mf][0][0] = cq[mf][0][1] = cq[mf][0][2] = cq[mf][0][3] = 0.f;
             landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, cq, d, g, t);
             if (tk.c == Lay::NCHK - 1) {
+                // Qbar overlays the Y^T of unit k - 2: with the long core's
+                // task order (m = 32) a warp's OUT(k - 2) precedes this task
+                // without a barrier in between, so wait for every warp's.
+                if constexpr (M > 16)
+                    if (tsync_or(failed)) break;
                 landmarks_put<T, LPW>(cq, reinterpret_cast<T*>(bb + Lay::B_QB), r * LPW, g, t);
                 if (tsync_or(failed)) break;
                 if constexpr (M > 16)  // KV(k) follows directly
@@ -358,7 +367,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
 template <typename T, int M, int NCOL, int DC, int PW, bool BIAS = false>
 cudaError_t launch_stream_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                           int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
-    using Lay = StreamLayout<M, NCOL>;
+    using Lay = StreamLayout<T, M, NCOL>;
     auto kern = nystra_stream_kernel<T, M, NCOL, DC, PW, BIAS>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device

@@ -62,6 +62,12 @@ constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s bound on any single wait
 constexpr float kLog2e = 1.4426950408889634f;  // score bias into the log2 domain of ex2
 constexpr size_t kSmemLimit = 232448;        // opt-in dynamic shared memory per CTA
 
+// 2^e as an fp32 bit pattern (e clamped to the normal range [-126, 127]).
+__device__ __forceinline__ float pow2i(int e) {
+    e = e < -126 ? -126 : (e > 127 ? 127 : e);
+    return __int_as_float((e + 127) << 23);
+}
+
 // Shared scratch of the distributed core (m = 32, 64; see dist_core): two
 // matrices of fp16 pairs (hi plane, then lo plane; rows padded to m + 8
 // halves so ldmatrix is conflict-free) and an auxiliary float area.
@@ -70,11 +76,14 @@ struct DistScratch {
     static constexpr int CW = M / 16, SS = M + 8;
     static constexpr size_t PLANE = (size_t)M * SS * 2;
     static constexpr size_t MAT = 2 * PLANE;
-    static constexpr size_t AUX = ((size_t)CW * M * 4 + 3 * CW * 4 + 15) / 16 * 16;  // column sums, maxima
+    static constexpr size_t AUX = ((size_t)CW * M * 4 + 4 * CW * 4 + 15) / 16 * 16;  // column sums, maxima
     static constexpr size_t BYTES = ((2 * MAT + AUX + 127) / 128) * 128;
 };
 
-template <int M, int NCOL, int TPW, int WPU, bool GLS, int CW = 1>
+template <typename T, int M>
+struct GlPark;  // parked G_L^n fragments (defined with the front phase)
+
+template <typename T, int M, int NCOL, int TPW, int WPU, bool GLS, int CW = 1>
 struct Layout {
     static constexpr int N = TPW * WPU;
     static constexpr int GW = WPU > CW ? WPU : CW;       // warps per group (token warps first)
@@ -82,11 +91,11 @@ struct Layout {
     static constexpr int DS = (NCOL == 32) ? 30 : 32;    // staged row width bound (d_h <= DS)
     static constexpr int MT = (M + 15) / 16;             // landmark m-tiles
     static constexpr int MP = MT * 16;                   // padded landmark count
-    static constexpr int LS = 40;                        // Qbar/Kbar row stride (16-bit elements)
+    static constexpr int LS = LmS<T>::LS;                // Qbar/Kbar row stride
     static constexpr int WS = NCOL + 4;                  // fp32 W row stride
-    static constexpr int YS = (M < 16 ? 16 : M) + 8;     // Y^T row stride (16-bit elements)
+    static constexpr int YS = YtS<T, M>::YS;             // Y^T row stride
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;   // k-steps of O = G_L^n Y
-    static constexpr int GLB = (M >= 16) ? 16 : 8;       // bytes per lane per G_L fragment
+    static constexpr int GLB = GlPark<T, M>::BYTES;      // bytes per lane per G_L fragment
     // per-warp private memory: stage (Q, K, V rows of the warp), G_L fragments
     static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;
     static constexpr size_t GLF = STAGE;
@@ -96,22 +105,22 @@ struct Layout {
     static constexpr size_t WPART = (size_t)TPW * DS * 2;
     static_assert(WPU == 1 || (size_t)MP * WS * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2,
                   "W partial must fit in K+V");
-    // per-group shared memory
-    // With one warp per unit and G_L^n parked, Y^T is written only after the
-    // core has read Qbar/Kbar for the last time and is dead before the next
-    // unit's landmarks, so it overlays them.  (With several warps a fast warp
-    // could write the next landmarks while another still reads Y^T; without
-    // parking, the output phase still reads Kbar.)
-    static constexpr bool YT_OVERLAY = (WPU == 1) && GLS;
-    static constexpr size_t QK_BYTES = 2 * MP * LS * 2;
-    static constexpr size_t YT_BYTES = ((NCOL * YS * 2 + 15) / 16) * 16;
+    // per-group shared memory: Qbar | W | m_U | Kbar (| Y^T).  Y^T is written
+    // by the core once it has read Qbar, W and m_U for the last time, so it
+    // overlays them when no warp can write the next unit's landmarks while
+    // another still reads Y^T: with one warp per unit, or when G_L^n is
+    // recomputed (the output is followed by a group barrier before the next
+    // unit's Q lands).
+    static constexpr bool YT_OVERLAY = (WPU == 1) || !GLS;
+    static constexpr size_t QB_BYTES = LmS<T>::bytes(MP);
+    static constexpr size_t YT_BYTES = YtS<T, M>::bytes(NCOL);
     static constexpr size_t G_QBAR = 0;
-    static constexpr size_t G_KBAR = G_QBAR + MP * LS * 2;
-    static constexpr size_t G_YT = YT_OVERLAY ? G_QBAR : QK_BYTES;
-    static constexpr size_t G_MU = YT_OVERLAY ? (QK_BYTES > YT_BYTES ? QK_BYTES : YT_BYTES)
-                                              : QK_BYTES + YT_BYTES;  // m_U, log2 domain
-    static constexpr size_t G_W = G_MU + MP * 4;
-    static constexpr size_t G_BAR = G_W + MP * WS * 4;
+    static constexpr size_t G_W = G_QBAR + QB_BYTES;  // fp32 MP x WS
+    static constexpr size_t G_MU = G_W + MP * WS * 4;  // m_U, log2 domain
+    static constexpr size_t G_KBAR = ((G_MU + MP * 4 + 15) / 16) * 16;
+    static constexpr size_t G_YT = YT_OVERLAY ? G_QBAR : G_KBAR + QB_BYTES;
+    static_assert(!YT_OVERLAY || YT_BYTES <= G_KBAR, "Y^T must fit over Qbar, W and m_U");
+    static constexpr size_t G_BAR = ((YT_OVERLAY ? G_KBAR + QB_BYTES : G_YT + YT_BYTES) + 15) / 16 * 16;
     static constexpr size_t G_BAR_END = G_BAR + 16 * WPU;  // two mbarriers per token warp
     // Distributed core (CW > 1): its scratch is group memory, or, with long
     // stages (TPW >= 256), the first two token warps' K/V rows (consumed by
@@ -191,7 +200,7 @@ __device__ __forceinline__ int frag_normalise(Frag<MT>& f) {
     mx = warp_max_nonneg(mx);
     if (!(mx > 0.f) || !(mx < INFINITY)) return 0;
     const int e = 10 - ilogbf(mx);
-    const float s = ldexpf(1.f, e);
+    const float s = pow2i(e);
 #pragma unroll
     for (int i = 0; i < MT; ++i)
 #pragma unroll
@@ -280,22 +289,11 @@ __device__ __forceinline__ void transpose_hfrag(const HFrag<MT>& a, HFrag<MT>& b
             }
 }
 
-// D = s I + A P^T (+ c I P^T when CI; i7 holds the A operand register of
-// c I's diagonal blocks) with fp16 two-term split operands, one fp32
-// accumulator per tile: the small terms lo*hi and hi*lo first, then hi*hi.
-template <int MT, bool CI>
-__device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Frag<MT>& D, float s, uint32_t i7,
-                                      int g, int t) {
+// D += A P^T with fp16 two-term split operands, the small terms lo*hi and
+// hi*lo first, then hi*hi.
+template <int MT>
+__device__ __forceinline__ void mm_hT_acc(const HFrag<MT>& A, const HFrag<MT>& P, Frag<MT>& D) {
     using H = Mma16<__half>;
-#pragma unroll
-    for (int i = 0; i < MT; ++i)
-#pragma unroll
-        for (int j = 0; j < 2 * MT; ++j)
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const bool diag = (16 * i + 8 * (e >> 1) + g) == (8 * j + (e & 1) + 2 * t);
-                D[i][j][e] = diag ? s : 0.f;
-            }
 #pragma unroll
     for (int kk = 0; kk < MT; ++kk)
 #pragma unroll
@@ -305,20 +303,68 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
             for (int i = 0; i < MT; ++i) {
                 const uint32_t ahi[4] = {A[i][kk][0].hi, A[i][kk][1].hi, A[i][kk][2].hi, A[i][kk][3].hi};
                 const uint32_t alo[4] = {A[i][kk][0].lo, A[i][kk][1].lo, A[i][kk][2].lo, A[i][kk][3].lo};
-                if (CI && kk == i) {
-                    const uint32_t ci[4] = {i7, 0u, 0u, i7};
-                    H::k16(D[i][j], ci, b0.lo, b1.lo);
-                }
                 H::k16(D[i][j], alo, b0.hi, b1.hi);
                 H::k16(D[i][j], ahi, b0.lo, b1.lo);
-                if (CI && kk == i) {
-                    const uint32_t ci[4] = {i7, 0u, 0u, i7};
-                    H::k16(D[i][j], ci, b0.hi, b1.hi);
-                }
                 H::k16(D[i][j], ahi, b0.hi, b1.hi);
             }
         }
 }
+
+// D = s I.
+template <int MT>
+__device__ __forceinline__ void frag_diag(Frag<MT>& D, float s, int g, int t) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int j = 0; j < 2 * MT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                D[i][j][e] = ((16 * i + 8 * (e >> 1) + g) == (8 * j + (e & 1) + 2 * t)) ? s : 0.f;
+}
+
+// D += s (hi + lo) of the split A operand P, element by element (fp32): C-layout
+// element (i, n, e) is half (e & 1) of register (e >> 1) | ((n & 1) << 1) of
+// P's m-tile i, k-step n / 2.
+template <int MT>
+__device__ __forceinline__ void frag_add_h(Frag<MT>& D, const HFrag<MT>& P, float s) {
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const H2Pair x = P[i][n >> 1][h | ((n & 1) << 1)];
+                const float2 a = __half22float2(*reinterpret_cast<const __half2*>(&x.hi));
+                const float2 b = __half22float2(*reinterpret_cast<const __half2*>(&x.lo));
+                D[i][n][2 * h] = fmaf(s, a.x + b.x, D[i][n][2 * h]);
+                D[i][n][2 * h + 1] = fmaf(s, a.y + b.y, D[i][n][2 * h + 1]);
+            }
+}
+
+// Largest |D| over the warp.
+template <int MT>
+__device__ __forceinline__ float frag_absmax(const Frag<MT>& D) {
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < MT; ++i)
+#pragma unroll
+        for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) mx = fmaxf(mx, fabsf(D[i][n][e]));
+    return warp_max_nonneg(mx);
+}
+
+// Largest value over the warp (any sign).
+__device__ __forceinline__ float warp_max_f(float x) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
+    return x;
+}
+
+// Exponent e with 2^e x in [2^10, 2^11) (0 when x is 0 or not finite): an
+// fp16 pair of a matrix scaled so keeps 22 significant bits for every entry
+// down to 2^-13 of its largest one.
+__device__ __forceinline__ int h2_exponent(float x) { return (x > 0.f && x < INFINITY) ? 10 - ilogbf(x) : 0; }
 
 // S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
 // fragments (A operand of O = G_L^n Y, k = landmarks).
@@ -326,10 +372,10 @@ __device__ __forceinline__ void mm_hT(const HFrag<MT>& A, const HFrag<MT>& P, Fr
 // bias (row stride M); log2(e) B_L enters the exponent beside the scaled score.
 template <typename T, int M, int KTL, bool BIAS = false>
 __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g, int t, float sl2,
-                                        typename Opnd<T>::Reg (&f)[KTL][4], const float* bl = nullptr) {
+                                        typename Opnd<T>::DReg (&f)[KTL][4], const float* bl = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
-    constexpr int NTL = M / 8, LS = 40;
+    constexpr int NTL = M / 8, LS = LmS<T>::LS, LO = LmS<T>::LO;
     R a[2][4];
     const T* q1 = q0 + 8 * d;
 #pragma unroll
@@ -347,7 +393,7 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const T* kr = kbar + (8 * j + g) * LS + 16 * kk + 2 * t;
-            O::mma(sl[j], a[kk], O::ld(kr), O::ld(kr + 8));
+            O::mma(sl[j], a[kk], DSt<T>::ld(kr, LO), DSt<T>::ld(kr + 8, LO));
         }
     }
     if constexpr (BIAS) {  // scores in the log2 domain, bias included: e0/e1 below take them as they are
@@ -375,60 +421,63 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
     if constexpr (M >= 16) {
 #pragma unroll
         for (int kk = 0; kk < KTL; ++kk) {
-            f[kk][0] = O::pk(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
-            f[kk][1] = O::pk(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
-            f[kk][2] = O::pk(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
-            f[kk][3] = O::pk(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
+            f[kk][0] = O::dpk(e0(sl[2 * kk][0]), e0(sl[2 * kk][1]));
+            f[kk][1] = O::dpk(e1(sl[2 * kk][2]), e1(sl[2 * kk][3]));
+            f[kk][2] = O::dpk(e0(sl[2 * kk + 1][0]), e0(sl[2 * kk + 1][1]));
+            f[kk][3] = O::dpk(e1(sl[2 * kk + 1][2]), e1(sl[2 * kk + 1][3]));
         }
     } else {
-        f[0][0] = O::pk(e0(sl[0][0]), e0(sl[0][1]));
-        f[0][1] = O::pk(e1(sl[0][2]), e1(sl[0][3]));
-        f[0][2] = f[0][3] = O::zero();
+        f[0][0] = O::dpk(e0(sl[0][0]), e0(sl[0][1]));
+        f[0][1] = O::dpk(e1(sl[0][2]), e1(sl[0][3]));
+        f[0][2] = f[0][3] = O::dzero();
     }
 }
 
 // Parked G_L^n fragments: per lane and 16-token tile, KTL x 4 operand
-// registers (m >= 16) or 2 (m = 8), one or two 16-byte vectors.
+// registers (m >= 16) or 2 (m = 8): single 16-bit registers (Single16 I/O:
+// one or a half 16-byte vector per k-step) or hi + lo pairs (two or one).
 template <typename T, int M>
 struct GlPark {
-    using R = typename Opnd<T>::Reg;
-    static constexpr int REGS = (M >= 16) ? 4 : 2;                   // registers per k-step
-    static constexpr int BYTES = REGS * (int)sizeof(R);               // per lane per k-step
+    using R = typename Opnd<T>::DReg;
+    static constexpr bool kPair = sizeof(R) == 8;
+    static constexpr int REGS = (M >= 16) ? 4 : 2;              // registers per k-step
+    static constexpr int BYTES = REGS * (int)sizeof(R);          // per lane per k-step
     static __device__ __forceinline__ void put(uint32_t* glf, int slot, const R (&f)[4]) {
-        if constexpr (sizeof(R) == 4) {
+        if constexpr (!kPair) {
             if constexpr (M >= 16)
                 reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[0], f[1], f[2], f[3]);
             else
                 reinterpret_cast<uint2*>(glf)[slot] = make_uint2(f[0], f[1]);
+        } else if constexpr (M >= 16) {
+            reinterpret_cast<uint4*>(glf)[2 * slot] = make_uint4(f[0].hi, f[1].hi, f[2].hi, f[3].hi);
+            reinterpret_cast<uint4*>(glf)[2 * slot + 1] = make_uint4(f[0].lo, f[1].lo, f[2].lo, f[3].lo);
         } else {
+            reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[0].hi, f[1].hi, f[0].lo, f[1].lo);
+        }
+    }
+    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, R (&f)[4]) {
+        if constexpr (!kPair) {
             if constexpr (M >= 16) {
-                reinterpret_cast<uint4*>(glf)[2 * slot] = make_uint4(f[0].hi, f[1].hi, f[2].hi, f[3].hi);
-                reinterpret_cast<uint4*>(glf)[2 * slot + 1] = make_uint4(f[0].lo, f[1].lo, f[2].lo, f[3].lo);
+                const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
+                f[0] = x.x; f[1] = x.y; f[2] = x.z; f[3] = x.w;
             } else {
-                reinterpret_cast<uint4*>(glf)[slot] = make_uint4(f[0].hi, f[1].hi, f[0].lo, f[1].lo);
+                const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
+                f[0] = x.x; f[1] = x.y; f[2] = f[3] = 0u;
             }
-        }
-    }
-    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, uint32_t (&f)[4]) {
-        if constexpr (M >= 16) {
-            const uint4 x = reinterpret_cast<const uint4*>(glf)[slot];
-            f[0] = x.x; f[1] = x.y; f[2] = x.z; f[3] = x.w;
         } else {
-            const uint2 x = reinterpret_cast<const uint2*>(glf)[slot];
-            f[0] = x.x; f[1] = x.y; f[2] = f[3] = 0u;
-        }
-    }
-    static __device__ __forceinline__ void get(const uint32_t* glf, int slot, RegPair (&f)[4]) {
-        const uint4* p = reinterpret_cast<const uint4*>(glf);
-        if constexpr (M >= 16) {
-            f[0] = {p[2 * slot].x, p[2 * slot + 1].x};
-            f[1] = {p[2 * slot].y, p[2 * slot + 1].y};
-            f[2] = {p[2 * slot].z, p[2 * slot + 1].z};
-            f[3] = {p[2 * slot].w, p[2 * slot + 1].w};
-        } else {
-            f[0] = {p[slot].x, p[slot].z};
-            f[1] = {p[slot].y, p[slot].w};
-            f[2] = f[3] = RegPair{0u, 0u};
+            const uint4* p = reinterpret_cast<const uint4*>(glf);
+            if constexpr (M >= 16) {
+                const uint4 h = p[2 * slot], l = p[2 * slot + 1];
+                f[0] = {h.x, l.x};
+                f[1] = {h.y, l.y};
+                f[2] = {h.z, l.z};
+                f[3] = {h.w, l.w};
+            } else {
+                const uint4 x = p[slot];
+                f[0] = {x.x, x.z};
+                f[1] = {x.y, x.w};
+                f[2] = f[3] = R{0u, 0u};
+            }
         }
     }
 };
@@ -443,8 +492,8 @@ struct GlPark {
 //
 // landmarks_acc adds one 64-token chunk X (tokens tok0..tok0+63 of the warp's
 // range) to the accumulators c (features x the warp's LPW segments);
-// landmarks_put rounds the means to the I/O type and stores them as rows
-// j0.. of xbar (row stride LS); columns >= d come out as zeros.
+// landmarks_put stores the means as rows j0.. of xbar (LmS layout: hi + lo
+// 16-bit pairs, or fp32 for fp32 I/O); columns >= d come out as zeros.
 //
 // PW > 0 pools square patches instead of segments: the window is PW tokens
 // wide, a landmark averages a B x B patch (B^2 = L) and the patches of a
@@ -508,7 +557,7 @@ __device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2
 
 template <typename T, int LPW>
 __device__ __forceinline__ void landmarks_put(const float (&c)[2][(LPW + 7) / 8][4], T* xbar, int j0, int g, int t) {
-    constexpr int NTJ = (LPW + 7) / 8, LS = 40;
+    constexpr int NTJ = (LPW + 7) / 8, LS = LmS<T>::LS, LO = LmS<T>::LO;
 #pragma unroll
     for (int mf = 0; mf < 2; ++mf)
 #pragma unroll
@@ -516,8 +565,16 @@ __device__ __forceinline__ void landmarks_put(const float (&c)[2][(LPW + 7) / 8]
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const int lm = 8 * j + 2 * t + (e & 1), f = 16 * mf + g + 8 * (e >> 1);
-                if (lm < LPW) xbar[(j0 + lm) * LS + f] = from_f32<T>(c[mf][j][e]);
+                if (lm < LPW) DSt<T>::put(xbar + (j0 + lm) * LS + f, LO, c[mf][j][e]);
             }
+}
+
+// Zero landmark rows lo .. hi - 1 of xbar (padding rows when m < 16), all 32
+// feature columns of both parts; `idx0`, `step`: this thread's share.
+template <typename T>
+__device__ __forceinline__ void landmarks_zero(T* xbar, int lo, int hi, int idx0, int step) {
+    constexpr int LS = LmS<T>::LS, LO = LmS<T>::LO;
+    for (int idx = idx0; idx < (hi - lo) * 32; idx += step) DSt<T>::zero(xbar + (lo + (idx >> 5)) * LS + (idx & 31), LO);
 }
 
 // All TPW tokens of the warp (a multiple of 64), then the store.
@@ -550,7 +607,7 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 // BIAS: bu points at the chunk's first key in row g of the m-tile in the
 // M x N block B_U of the score bias (row stride bn).
 template <typename T, int NCOL, bool BIAS = false>
-__device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][4], const T* Kc, const T* Vc, int d,
+__device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::DReg (&aq)[2][4], const T* Kc, const T* Vc, int d,
                                            int g, int t, float sl2, bool v0, bool v1, float (&w)[NCOL / 8][4],
                                            float& run0, float& run1, bool rescale, const float* bu = nullptr,
                                            int bn = 0) {
@@ -604,11 +661,11 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][
     auto e1 = [&](float x) { return ex2(fmaf(x, ssl, -mx1)); };
 #pragma unroll
     for (int kt = 0; kt < 4; ++kt) {
-        R a[4];
-        a[0] = v0 ? O::pk(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : O::zero();
-        a[1] = v1 ? O::pk(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : O::zero();
-        a[2] = v0 ? O::pk(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : O::zero();
-        a[3] = v1 ? O::pk(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : O::zero();
+        typename O::DReg a[4];
+        a[0] = v0 ? O::dpk(e0(s[2 * kt][0]), e0(s[2 * kt][1])) : O::dzero();
+        a[1] = v1 ? O::dpk(e1(s[2 * kt][2]), e1(s[2 * kt][3])) : O::dzero();
+        a[2] = v0 ? O::dpk(e0(s[2 * kt + 1][0]), e0(s[2 * kt + 1][1])) : O::dzero();
+        a[3] = v1 ? O::dpk(e1(s[2 * kt + 1][2]), e1(s[2 * kt + 1][3])) : O::dzero();
 #pragma unroll
         for (int j = 0; j < NTO; ++j) {
             const int c0 = 8 * j + 2 * t;
@@ -619,18 +676,17 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::Reg (&aq)[2][
     }
 }
 
-// A operand registers of Qbar's m-tile mt (row stride 40).
+// A operand registers (hi + lo pairs) of Qbar's m-tile mt.
 template <typename T>
-__device__ __forceinline__ void qbar_afrag(const T* qbar, int mt, int g, int t, typename Opnd<T>::Reg (&aq)[2][4]) {
-    using O = Opnd<T>;
-    constexpr int LS = 40;
+__device__ __forceinline__ void qbar_afrag(const T* qbar, int mt, int g, int t, typename Opnd<T>::DReg (&aq)[2][4]) {
+    constexpr int LS = LmS<T>::LS, LO = LmS<T>::LO;
 #pragma unroll
     for (int kk = 0; kk < 2; ++kk) {
         const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-        aq[kk][0] = O::ld(r0);
-        aq[kk][1] = O::ld(r0 + 8 * LS);
-        aq[kk][2] = O::ld(r0 + 8);
-        aq[kk][3] = O::ld(r0 + 8 * LS + 8);
+        aq[kk][0] = DSt<T>::ld(r0, LO);
+        aq[kk][1] = DSt<T>::ld(r0 + 8 * LS, LO);
+        aq[kk][2] = DSt<T>::ld(r0 + 8, LO);
+        aq[kk][3] = DSt<T>::ld(r0 + 8 * LS + 8, LO);
     }
 }
 
@@ -644,7 +700,7 @@ template <typename T, int M, int NCOL, int NCH, bool BIAS = false>
 __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
                                            float* dst, int ws, float (&mU)[(M + 15) / 16][2],
                                            const float* bu = nullptr, int bn = 0) {
-    using R = typename Opnd<T>::Reg;
+    using R = typename Opnd<T>::DReg;
     constexpr int MT = (M + 15) / 16, NTO = NCOL / 8;
     float wall[MT][NTO][4];
 #pragma unroll
@@ -700,14 +756,18 @@ __device__ __forceinline__ void combine_partials(const float* part0, size_t wstr
 // Core, one warp: G_A^n = exp(Qbar Kbar^T - m_U) (mU: row maxima of this
 // warp's rows of S_U in the log2 domain), the iterative pseudo-inverse
 // (step 4) and Y = Z W (W = G_U^n [V | 1], fp32 row-major with stride WS at
-// mW), stored as Y^T (16-bit B operand) at yT.
+// mW), stored as Y^T (hi + lo B operand pairs, YtS layout) at yT.
 //
 // The iteration is run in registers on the symmetric X = A Z_k (Z_0 = a A^T):
 // T2 = 15I - 7X + X X, T3 = 13I - X T2, Z <- Z T3/4 and X <- X T3/4 (equal to
 // A Z_{k+1}; its factors are polynomials in X and commute).  X is kept exactly
 // symmetric (lower triangle mirrored) after every update.  Scalar factors of
 // Z (a and the power-of-two range scaling) are dropped: O is a ratio of two
-// columns of G_L^n Z W, so they cancel.
+// columns of G_L^n Z W, so they cancel.  Every matrix is split into fp16
+// pairs at a power-of-two scale that puts its largest entry in [2^10, 2^11)
+// (A once, X, -T2/4, T3/4 and Z every step), and the products are rescaled
+// in fp32, so no operand underflows fp16 however small G_A^n's entries are
+// (sharp attention: rows of G_A^n far below 1).
 //
 // DUMP (test-only stage dump): dbg receives G_A^n (M x M), Z (M x M) and
 // Y = Z W (M x NCOL), row-major fp32, with the dropped factors restored.
@@ -717,31 +777,27 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                                           const float* mW, T* yT, int iters, float sl2, int g, int t,
                                           float* dbg = nullptr, const float* ba = nullptr) {
     using O = Opnd<T>;
-    using R = typename O::Reg;
-    constexpr int MT = (M + 15) / 16, LS = 40, WS = NCOL + 4, NTO = NCOL / 8;
-    constexpr int YS = (M < 16 ? 16 : M) + 8;
+    using D = typename O::DReg;
+    constexpr int MT = (M + 15) / 16, LS = LmS<T>::LS, LO = LmS<T>::LO, WS = NCOL + 4, NTO = NCOL / 8;
+    constexpr int YS = YtS<T, M>::YS, YLO = YtS<T, M>::LO;
     const uint32_t sel = tril_selector(g, t);
-    uint32_t i7;  // A operand register of -7I's diagonal blocks
-    {
-        const __half2 h = __floats2half2_rn(g == 2 * t ? -7.f : 0.f, g == 2 * t + 1 ? -7.f : 0.f);
-        i7 = *reinterpret_cast<const uint32_t*>(&h);
-    }
     Frag<MT> Zc;
     HFrag<MT> Xh, Zh;
+    int ex = 0;          // Xh holds 2^ex X
     float zscale = 1.f;  // DUMP: Z = zscale 2^-esum Zc
     int esum = 0;
     {
         Frag<MT> Ac;
 #pragma unroll
         for (int mt = 0; mt < MT; ++mt) {
-            R aq[2][4];
+            D aq[2][4];
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
                 const T* r0 = qbar + (16 * mt + g) * LS + 16 * kk + 2 * t;
-                aq[kk][0] = O::ld(r0);
-                aq[kk][1] = O::ld(r0 + 8 * LS);
-                aq[kk][2] = O::ld(r0 + 8);
-                aq[kk][3] = O::ld(r0 + 8 * LS + 8);
+                aq[kk][0] = DSt<T>::ld(r0, LO);
+                aq[kk][1] = DSt<T>::ld(r0 + 8 * LS, LO);
+                aq[kk][2] = DSt<T>::ld(r0 + 8, LO);
+                aq[kk][3] = DSt<T>::ld(r0 + 8 * LS + 8, LO);
             }
 #pragma unroll
             for (int n = 0; n < 2 * MT; ++n) {
@@ -749,27 +805,50 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
 #pragma unroll
                 for (int kk = 0; kk < 2; ++kk) {
                     const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
-                    O::mma(sa, aq[kk], O::ld(kr), O::ld(kr + 8));
+                    O::mma(sa, aq[kk], DSt<T>::ld(kr, LO), DSt<T>::ld(kr + 8, LO));
                 }
+                // log2 of G_A^n (-inf outside the m x m block)
                 const int r0 = 16 * mt + g, r1 = r0 + 8, c = 8 * n + 2 * t;
                 if constexpr (BIAS) {  // log2(e) B_A joins the shift (c and c + 1 < M together: M is even)
                     const float2 b0 = (r0 < M && c < M) ? __ldg(reinterpret_cast<const float2*>(ba + r0 * M + c))
                                                         : make_float2(0.f, 0.f);
                     const float2 b1 = (r1 < M && c < M) ? __ldg(reinterpret_cast<const float2*>(ba + r1 * M + c))
                                                         : make_float2(0.f, 0.f);
-                    Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, fmaf(kLog2e, b0.x, -mU[mt][0]))) : 0.f;
-                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, fmaf(kLog2e, b0.y, -mU[mt][0]))) : 0.f;
-                    Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, fmaf(kLog2e, b1.x, -mU[mt][1]))) : 0.f;
-                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, fmaf(kLog2e, b1.y, -mU[mt][1]))) : 0.f;
+                    Ac[mt][n][0] = (r0 < M && c < M) ? fmaf(sa[0], sl2, fmaf(kLog2e, b0.x, -mU[mt][0])) : -INFINITY;
+                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? fmaf(sa[1], sl2, fmaf(kLog2e, b0.y, -mU[mt][0])) : -INFINITY;
+                    Ac[mt][n][2] = (r1 < M && c < M) ? fmaf(sa[2], sl2, fmaf(kLog2e, b1.x, -mU[mt][1])) : -INFINITY;
+                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? fmaf(sa[3], sl2, fmaf(kLog2e, b1.y, -mU[mt][1])) : -INFINITY;
                 } else {
-                    Ac[mt][n][0] = (r0 < M && c < M) ? ex2(fmaf(sa[0], sl2, -mU[mt][0])) : 0.f;
-                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? ex2(fmaf(sa[1], sl2, -mU[mt][0])) : 0.f;
-                    Ac[mt][n][2] = (r1 < M && c < M) ? ex2(fmaf(sa[2], sl2, -mU[mt][1])) : 0.f;
-                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? ex2(fmaf(sa[3], sl2, -mU[mt][1])) : 0.f;
+                    Ac[mt][n][0] = (r0 < M && c < M) ? fmaf(sa[0], sl2, -mU[mt][0]) : -INFINITY;
+                    Ac[mt][n][1] = (r0 < M && c + 1 < M) ? fmaf(sa[1], sl2, -mU[mt][0]) : -INFINITY;
+                    Ac[mt][n][2] = (r1 < M && c < M) ? fmaf(sa[2], sl2, -mU[mt][1]) : -INFINITY;
+                    Ac[mt][n][3] = (r1 < M && c + 1 < M) ? fmaf(sa[3], sl2, -mU[mt][1]) : -INFINITY;
                 }
             }
         }
-        // ||A||_inf (max row sum) and ||A||_1 (max column sum); A > 0.
+        // 2^ea G_A^n with its largest entry in [2^10, 2^11): the shift enters
+        // the exponent, so no entry underflows for being small in absolute
+        // terms (sharp attention can put a whole row of G_A^n far below 1).
+        int ea;
+        {
+            float lmax = -INFINITY;
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) lmax = fmaxf(lmax, Ac[i][n][e]);
+            lmax = warp_max_f(lmax);
+            ea = (lmax > -INFINITY && lmax < INFINITY) ? 10 - (int)floorf(lmax) : 0;
+            const float fa = (float)ea;
+#pragma unroll
+            for (int i = 0; i < MT; ++i)
+#pragma unroll
+                for (int n = 0; n < 2 * MT; ++n)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) Ac[i][n][e] = ex2(Ac[i][n][e] + fa);
+        }
+        // ||A||_inf (max row sum) and ||A||_1 (max column sum) of 2^ea A; A > 0.
         float rmax = 0.f, cmax = 0.f;
 #pragma unroll
         for (int i = 0; i < MT; ++i) {
@@ -797,9 +876,10 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                 c += __shfl_xor_sync(0xffffffffu, c, 16);
                 cmax = fmaxf(cmax, c);
             }
-        const float alpha = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
+        // a A A^T = (2^ea A)(2^ea A)^T / (||2^ea A||_1 ||2^ea A||_inf)
+        const float x0 = 1.f / (warp_max_nonneg(rmax) * warp_max_nonneg(cmax));
         if constexpr (DUMP) {
-            zscale = alpha;
+            zscale = ldexpf(x0, ea);  // Z_0 = a A^T = x0 2^ea (2^ea A)^T
 #pragma unroll
             for (int i = 0; i < MT; ++i)
 #pragma unroll
@@ -807,14 +887,16 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
                         const int r = 16 * i + g + 8 * (e >> 1), c = 8 * n + 2 * t + (e & 1);
-                        if (r < M && c < M) dbg[r * M + c] = Ac[i][n][e];
+                        if (r < M && c < M) dbg[r * M + c] = ldexpf(Ac[i][n][e], -ea);
                     }
         }
         HFrag<MT> Ah;
         to_hfrag<MT>(Ac, Ah);
-        transpose_hfrag<MT>(Ah, Zh);  // Z_0 = A^T (a dropped)
-        mm_hT<MT, false>(Ah, Ah, Ac, 0.f, 0u, g, t);
-        sym_hfrag<MT>(Ac, Xh, sel, alpha);  // X_0 = a A A^T
+        transpose_hfrag<MT>(Ah, Zh);  // Z_0 = (2^ea A)^T (a and 2^ea dropped)
+        frag_diag<MT>(Ac, 0.f, g, t);
+        mm_hT_acc<MT>(Ah, Ah, Ac);  // X_0 = x0 Ac
+        ex = h2_exponent(x0 * frag_absmax<MT>(Ac));
+        sym_hfrag<MT>(Ac, Xh, sel, x0 * pow2i(ex));
         if (iters == 0) {
 #pragma unroll
             for (int i = 0; i < MT; ++i)
@@ -832,19 +914,34 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
         }
     }
 
-    // pseudo-inverse iteration (step 4)
+    // pseudo-inverse iteration (step 4).  X is split at a scale 2^ex chosen
+    // from its largest entry; -T2/4 and T3/4 at the fixed 2^10 (X's
+    // eigenvalues lie in [0, 1], so their entries stay within a few units).
+    constexpr int kT = 10;
 #pragma unroll 1
     for (int it = 0; it < iters; ++it) {
         Frag<MT> F;
         HFrag<MT> Th;
-        mm_hT<MT, true>(Xh, Xh, F, 15.f, i7, g, t);  // T2 = 15I - 7X + X X
-        to_hfrag_scaled<MT>(F, Th, -0.25f);           // -T2/4
-        mm_hT<MT, false>(Xh, Th, F, 3.25f, 0u, g, t);  // T3/4 = 13/4 I - X T2/4
-        to_hfrag<MT>(F, Th);
-        mm_hT<MT, false>(Zh, Th, Zc, 0.f, 0u, g, t);   // Z T3/4
+        // 2^(2 ex) T2 = 2^(2 ex) (15 I - 7 X) + (2^ex X)(2^ex X)
+        const float sx = pow2i(ex);
+        frag_diag<MT>(F, 15.f * sx * sx, g, t);
+        frag_add_h<MT>(F, Xh, -7.f * sx);
+        mm_hT_acc<MT>(Xh, Xh, F);
+        to_hfrag_scaled<MT>(F, Th, -0.25f * pow2i(kT - 2 * ex));  // 2^kT (-T2/4)
+        // 2^(ex + kT) T3/4 = 2^(ex + kT) 13/4 I + (2^ex X)(2^kT (-T2/4))
+        frag_diag<MT>(F, 3.25f * pow2i(ex + kT), g, t);
+        mm_hT_acc<MT>(Xh, Th, F);
+        to_hfrag_scaled<MT>(F, Th, pow2i(-ex));  // 2^kT T3/4
+        frag_diag<MT>(Zc, 0.f, g, t);
+        mm_hT_acc<MT>(Zh, Th, Zc);  // Z 2^kT T3/4
+        if constexpr (DUMP) esum += kT;
         if (it + 1 < iters) {
-            mm_hT<MT, false>(Xh, Th, F, 0.f, 0u, g, t);  // X T3/4
-            sym_hfrag<MT>(F, Xh, sel, 1.f);
+            frag_diag<MT>(F, 0.f, g, t);
+            mm_hT_acc<MT>(Xh, Th, F);  // 2^(ex + kT) X T3/4
+            const float f = pow2i(-(ex + kT));
+            const int en = h2_exponent(f * frag_absmax<MT>(F));
+            sym_hfrag<MT>(F, Xh, sel, f * pow2i(en));
+            ex = en;
             const int ez = frag_normalise<MT>(Zc);
             if constexpr (DUMP) esum += ez;
             to_hfrag<MT>(Zc, Zh);
@@ -863,7 +960,7 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                 }
     }
 
-    // Y = Z W (split-tf32), stored as Y^T, a 16-bit B operand
+    // Y = Z W (split-tf32), stored as Y^T (hi + lo B operand pairs)
     {
         float y[MT][NTO][4];
 #pragma unroll
@@ -903,9 +1000,8 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
                         if (r < M) dbg[2 * M * M + r * NCOL + c] = zs * y[i][j][e];
                     }
         }
-        // fp16 output has a narrow range: scale Y by a power of two.
-        // Numerator and denominator columns share the factor, so it cancels
-        // in step 7.
+        // fp16 has a narrow range: Y is scaled by a power of two.  Numerator
+        // and denominator columns share the factor, so it cancels in step 7.
         float scale = 1.f;
         if (O::kNarrowRange) {
             float ymax = 0.f;
@@ -916,21 +1012,21 @@ __device__ __forceinline__ void core_warp(const T* qbar, const T* kbar, const fl
 #pragma unroll
                     for (int e = 0; e < 4; ++e) ymax = fmaxf(ymax, fabsf(y[i][j][e]));
             ymax = warp_max_nonneg(ymax);
-            if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
+            if (ymax > 0.f && ymax < INFINITY) scale = pow2i(14 - ilogbf(ymax));
         }
-        __syncwarp();  // Y^T may overlay the landmarks: every lane has read them
+        __syncwarp();  // Y^T may overlay the landmarks and W: every lane has read them
 #pragma unroll
         for (int i = 0; i < MT; ++i)
 #pragma unroll
             for (int j = 0; j < NTO; ++j) {
                 const int rr = 16 * i + g, c = 8 * j + 2 * t;
-                yT[c * YS + rr] = from_f32<T>(y[i][j][0] * scale);
-                yT[(c + 1) * YS + rr] = from_f32<T>(y[i][j][1] * scale);
-                yT[c * YS + rr + 8] = from_f32<T>(y[i][j][2] * scale);
-                yT[(c + 1) * YS + rr + 8] = from_f32<T>(y[i][j][3] * scale);
+                DSt<T>::put(yT + c * YS + rr, YLO, y[i][j][0] * scale);
+                DSt<T>::put(yT + (c + 1) * YS + rr, YLO, y[i][j][1] * scale);
+                DSt<T>::put(yT + c * YS + rr + 8, YLO, y[i][j][2] * scale);
+                DSt<T>::put(yT + (c + 1) * YS + rr + 8, YLO, y[i][j][3] * scale);
             }
     }
-        }
+}
 
 // ---- distributed core for m = 32, 64: CW = m/16 warps, warp c owns rows 16c..16c+15 ----
 // The m x m operands no longer fit one warp's registers.  Each warp keeps the
@@ -1061,39 +1157,44 @@ __device__ __forceinline__ void dist_mm(const H2Pair (*const (&A)[NA])[4], const
 // named barrier reserved for these warps; mat0, mat1, aux: DistScratch
 // areas): G_A^n from the landmarks and m_U (gmu, log2 domain), the iteration
 // of step 4, Y = Z W (W: fp32, row stride NCOL + 4 at mW) stored as Y^T at
-// yT.  Same arithmetic as core_warp.
+// yT.  Same arithmetic as core_warp, except that X, -T2/4 and T3/4 are split
+// at the fixed scale 2^10 (their entries stay within a few units, since X's
+// eigenvalues lie in [0, 1]), which saves a barrier per scale; A is split at
+// 2^ea with its largest entry in [2^10, 2^11), Z renormalised every step.
 template <typename T, int M, int NCOL>
 __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const float* gmu, const float* mW, T* yT,
                                           unsigned char* mat0, unsigned char* mat1, float* aux, int iters, float sl2,
                                           int c, int lane, int bar_id) {
     using S = DistScratch<M>;
     using O = Opnd<T>;
-    using R = typename O::Reg;
-    constexpr int CW = S::CW, KT = M / 16, NT = M / 8, LS = 40, WS = NCOL + 4, NTO = NCOL / 8, YS = M + 8;
+    using D = typename O::DReg;
+    constexpr int CW = S::CW, KT = M / 16, NT = M / 8, LS = LmS<T>::LS, LO = LmS<T>::LO, WS = NCOL + 4,
+                  NTO = NCOL / 8, YS = YtS<T, M>::YS, YLO = YtS<T, M>::LO;
     const int g = lane >> 2, t = lane & 3;
     unsigned char* cur = mat0;
     unsigned char* oth = mat1;
     float* cols = aux;                // [CW][M] column-sum partials
-    float* slots = aux + CW * M;      // [3][CW] maxima
+    float* slots = aux + CW * M;      // [4][CW] maxima
     auto csync = [&]() { named_barrier(bar_id, CW * 32); };
     const uint32_t sel = tril_selector(g, t);
-    uint32_t i7;
+    constexpr float kS = 1024.f, kS2 = 1048576.f;  // fixed scale 2^10 of X, -T2/4, T3/4 (and its square)
+    uint32_t i7;  // A operand register of -7 kS I's diagonal blocks
     {
-        const __half2 h = __floats2half2_rn(g == 2 * t ? -7.f : 0.f, g == 2 * t + 1 ? -7.f : 0.f);
+        const __half2 h = __floats2half2_rn(g == 2 * t ? -7.f * kS : 0.f, g == 2 * t + 1 ? -7.f * kS : 0.f);
         i7 = *reinterpret_cast<const uint32_t*>(&h);
     }
     H2Pair Xa[KT][4], Za[KT][4];
     float acc[NT][4], zc[NT][4];
     // ---- G_A^n, own rows ----
     {
-        R aq[2][4];
+        D aq[2][4];
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const T* r0 = qbar + (16 * c + g) * LS + 16 * kk + 2 * t;
-            aq[kk][0] = O::ld(r0);
-            aq[kk][1] = O::ld(r0 + 8 * LS);
-            aq[kk][2] = O::ld(r0 + 8);
-            aq[kk][3] = O::ld(r0 + 8 * LS + 8);
+            aq[kk][0] = DSt<T>::ld(r0, LO);
+            aq[kk][1] = DSt<T>::ld(r0 + 8 * LS, LO);
+            aq[kk][2] = DSt<T>::ld(r0 + 8, LO);
+            aq[kk][3] = DSt<T>::ld(r0 + 8 * LS + 8, LO);
         }
         const float mu0 = gmu[16 * c + g], mu1 = gmu[16 * c + g + 8];
 #pragma unroll
@@ -1102,13 +1203,33 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
 #pragma unroll
             for (int kk = 0; kk < 2; ++kk) {
                 const T* kr = kbar + (8 * n + g) * LS + 16 * kk + 2 * t;
-                O::mma(sa, aq[kk], O::ld(kr), O::ld(kr + 8));
+                O::mma(sa, aq[kk], DSt<T>::ld(kr, LO), DSt<T>::ld(kr + 8, LO));
             }
-            acc[n][0] = ex2(fmaf(sa[0], sl2, -mu0));
-            acc[n][1] = ex2(fmaf(sa[1], sl2, -mu0));
-            acc[n][2] = ex2(fmaf(sa[2], sl2, -mu1));
-            acc[n][3] = ex2(fmaf(sa[3], sl2, -mu1));
+            acc[n][0] = fmaf(sa[0], sl2, -mu0);  // log2 of G_A^n
+            acc[n][1] = fmaf(sa[1], sl2, -mu0);
+            acc[n][2] = fmaf(sa[2], sl2, -mu1);
+            acc[n][3] = fmaf(sa[3], sl2, -mu1);
         }
+    }
+    // 2^ea G_A^n with its largest entry in [2^10, 2^11) (the shift enters the
+    // exponent, as in core_warp)
+    {
+        float lm = -INFINITY;
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) lm = fmaxf(lm, acc[n][e]);
+        lm = warp_max_f(lm);
+        if (lane == 0) slots[3 * CW + c] = lm;
+        csync();
+        float lmax = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < CW; ++w) lmax = fmaxf(lmax, slots[3 * CW + w]);
+        const float fa = (lmax > -INFINITY && lmax < INFINITY) ? (float)(10 - (int)floorf(lmax)) : 0.f;
+#pragma unroll
+        for (int n = 0; n < NT; ++n)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) acc[n][e] = ex2(acc[n][e] + fa);
     }
     // ---- ||A||_inf, ||A||_1 (A > 0) and A into scratch ----
     {
@@ -1135,9 +1256,9 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
                 if (g == 0) cols[c * M + 8 * n + 2 * t + e] = cs;
             }
     }
-    dist_put<M>(cur, acc, 1.f, c, g, t);  // A
+    dist_put<M>(cur, acc, 1.f, c, g, t);  // 2^ea A
     csync();
-    float alpha;
+    float alpha;  // a A A^T = alpha (2^ea A)(2^ea A)^T
     {
         float rmax = 0.f, cmax = 0.f;
 #pragma unroll
@@ -1161,10 +1282,10 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
             }
         const H2Pair(*const As[1])[4] = {Aa};
         float(*const Ds[1])[4] = {acc};
-        dist_mm<M, 1, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // A A^T
+        dist_mm<M, 1, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // (2^ea A)(2^ea A)^T
     }
-    dist_load_a<M, true>(cur, Za, c, lane);  // Z_0 = A^T (a dropped)
-    dist_put_sym<M>(oth, acc, alpha, c, g, t, sel);  // X_0 = a A A^T
+    dist_load_a<M, true>(cur, Za, c, lane);  // Z_0 = (2^ea A)^T (a and 2^ea dropped)
+    dist_put_sym<M>(oth, acc, kS * alpha, c, g, t, sel);  // kS X_0
     csync();
     dist_load_a<M, false>(oth, Xa, c, lane);
     {
@@ -1191,22 +1312,22 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
         {
             const H2Pair(*const As[1])[4] = {Xa};
             float(*const Ds[1])[4] = {acc};
-            dist_mm<M, 1, true>(As, cur, Ds, 15.f, i7, c, g, t, lane);  // T2 = 15I - 7X + X X
+            dist_mm<M, 1, true>(As, cur, Ds, 15.f * kS2, i7, c, g, t, lane);  // kS^2 T2 = kS^2 (15I - 7X + X X)
         }
-        dist_put<M>(oth, acc, -0.25f, c, g, t);  // -T2/4
+        dist_put<M>(oth, acc, -0.25f / kS, c, g, t);  // kS (-T2/4)
         csync();
         {
             const H2Pair(*const As[1])[4] = {Xa};
             float(*const Ds[1])[4] = {acc};
-            dist_mm<M, 1, false>(As, oth, Ds, 3.25f, 0u, c, g, t, lane);  // T3/4
+            dist_mm<M, 1, false>(As, oth, Ds, 3.25f * kS2, 0u, c, g, t, lane);  // kS^2 T3/4
         }
-        dist_put<M>(cur, acc, 1.f, c, g, t);  // every warp is done with X
+        dist_put<M>(cur, acc, 1.f / kS, c, g, t);  // kS T3/4 (every warp is done with X)
         csync();
         if (it + 1 < iters) {
             const H2Pair(*const As[2])[4] = {Za, Xa};
             float(*const Ds[2])[4] = {zc, acc};
-            dist_mm<M, 2, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // Z T3/4, X T3/4
-            dist_put_sym<M>(oth, acc, 1.f, c, g, t, sel);            // every warp is done with -T2/4
+            dist_mm<M, 2, false>(As, cur, Ds, 0.f, 0u, c, g, t, lane);  // Z kS T3/4, kS^2 X T3/4
+            dist_put_sym<M>(oth, acc, 1.f / kS, c, g, t, sel);       // every warp is done with -T2/4
             float zm = 0.f;
 #pragma unroll
             for (int n = 0; n < NT; ++n)
@@ -1222,7 +1343,7 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
             float zmax = 0.f;
 #pragma unroll
             for (int w = 0; w < CW; ++w) zmax = fmaxf(zmax, slots[CW + w]);
-            const float sc = (zmax > 0.f && zmax < INFINITY) ? ldexpf(1.f, 10 - ilogbf(zmax)) : 1.f;
+            const float sc = (zmax > 0.f && zmax < INFINITY) ? pow2i(10 - ilogbf(zmax)) : 1.f;
 #pragma unroll
             for (int kk = 0; kk < KT; ++kk)
 #pragma unroll
@@ -1270,15 +1391,16 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
             float ymax = 0.f;
 #pragma unroll
             for (int w = 0; w < CW; ++w) ymax = fmaxf(ymax, slots[2 * CW + w]);
-            if (ymax > 0.f) scale = ldexpf(1.f, 14 - ilogbf(ymax));
+            if (ymax > 0.f && ymax < INFINITY) scale = pow2i(14 - ilogbf(ymax));
         }
+        csync();  // Y^T may overlay W, which every core warp reads in full
 #pragma unroll
         for (int j = 0; j < NTO; ++j) {
             const int rr = 16 * c + g, cc = 8 * j + 2 * t;
-            yT[cc * YS + rr] = from_f32<T>(y[j][0] * scale);
-            yT[(cc + 1) * YS + rr] = from_f32<T>(y[j][1] * scale);
-            yT[cc * YS + rr + 8] = from_f32<T>(y[j][2] * scale);
-            yT[(cc + 1) * YS + rr + 8] = from_f32<T>(y[j][3] * scale);
+            DSt<T>::put(yT + cc * YS + rr, YLO, y[j][0] * scale);
+            DSt<T>::put(yT + (cc + 1) * YS + rr, YLO, y[j][1] * scale);
+            DSt<T>::put(yT + cc * YS + rr + 8, YLO, y[j][2] * scale);
+            DSt<T>::put(yT + (cc + 1) * YS + rr + 8, YLO, y[j][3] * scale);
         }
     }
 }
@@ -1293,16 +1415,16 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
                                             T* obase, int d, int g, int t, int lane, float sl2,
                                             const float* bl = nullptr) {
     using O = Opnd<T>;
-    using R = typename O::Reg;
-    constexpr int KTL = (M >= 16) ? M / 16 : 1, NTO = NCOL / 8, YS = (M < 16 ? 16 : M) + 8;
+    using R = typename O::DReg;
+    constexpr int KTL = (M >= 16) ? M / 16 : 1, NTO = NCOL / 8, YS = YtS<T, M>::YS, YLO = YtS<T, M>::LO;
     R by[KTL][NTO][2];
 #pragma unroll
     for (int kk = 0; kk < KTL; ++kk)
 #pragma unroll
         for (int j = 0; j < NTO; ++j) {
             const T* yr = yT + (8 * j + g) * YS + 16 * kk + 2 * t;
-            by[kk][j][0] = O::ld(yr);
-            by[kk][j][1] = (M >= 16) ? O::ld(yr + 8) : O::zero();
+            by[kk][j][0] = DSt<T>::ld(yr, YLO);
+            by[kk][j][1] = (M >= 16) ? DSt<T>::ld(yr + 8, YLO) : O::dzero();
         }
     const int jd = d >> 3, tdn = (d & 7) >> 1;
     const int src = (lane & ~3) | tdn;
@@ -1353,15 +1475,16 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
 }
 
 template <typename T, int M, int NCOL, int TPW, int WPU, int GROUPS, bool GLS, int CW>
-__global__ void __launch_bounds__(GROUPS * Layout<M, NCOL, TPW, WPU, GLS, CW>::GW * 32, 1)
+__global__ void __launch_bounds__(GROUPS * Layout<T, M, NCOL, TPW, WPU, GLS, CW>::GW * 32, 1)
 nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                  T* __restrict__ out, long long n_units, int d, int iters, float sl2,
                  unsigned int* fault, int active) {
-    using Lay = Layout<M, NCOL, TPW, WPU, GLS, CW>;
+    using Lay = Layout<T, M, NCOL, TPW, WPU, GLS, CW>;
     constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS,
                   WS = Lay::WS, KTL = Lay::KTL, GW = Lay::GW;
     constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
     constexpr int LPW = TPW / L;  // landmarks owned by one warp
+    static_assert(sizeof(T) == 2, "the grouped kernel takes 16-bit I/O (its layout assumes it)");
     static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
     static_assert(CW == 1 || CW == M / 16, "the distributed core has one warp per 16 landmarks");
 
@@ -1465,11 +1588,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             landmarks_mma<T, TPW, L>(Qs, qbar, r * LPW, d, g, t);
             landmarks_mma<T, TPW, L>(Ks, kbar, r * LPW, d, g, t);
             if (M < MP && r == 0) {  // zero the padding landmark rows
-                for (int idx = lane; idx < (MP - M) * 32; idx += 32) {
-                    const int j = M + (idx >> 5), e = idx & 31;
-                    qbar[j * LS + e] = from_f32<T>(0.f);
-                    kbar[j * LS + e] = from_f32<T>(0.f);
-                }
+                landmarks_zero<T>(qbar, M, MP, lane, 32);
+                landmarks_zero<T>(kbar, M, MP, lane, 32);
             }
         }
         if (gsync_or(failed)) break;
@@ -1480,7 +1600,7 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
             for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
                 for (int tm = 0; tm < 4; ++tm) {
-                    typename Opnd<T>::Reg f[KTL][4];
+                    typename Opnd<T>::DReg f[KTL][4];
                     gl_tile<T, M, KTL>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
                     for (int kk = 0; kk < KTL; ++kk)
@@ -1600,9 +1720,9 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
 
 // Largest number of groups per CTA that fits the shared-memory and register
 // budgets (M <= 16 needs about 160 registers per thread, M = 32 about 255).
-template <int M, int NCOL, int TPW, int WPU, bool GLS, int CW>
+template <typename T, int M, int NCOL, int TPW, int WPU, bool GLS, int CW>
 constexpr int groups_that_fit() {
-    using Lay = Layout<M, NCOL, TPW, WPU, GLS, CW>;
+    using Lay = Layout<T, M, NCOL, TPW, WPU, GLS, CW>;
     const int by_smem = (int)(kSmemLimit / Lay::PER_GROUP);
     const int by_regs = ((M <= 16) ? 12 : 8) / Lay::GW;
     const int n = by_smem < by_regs ? by_smem : by_regs;
@@ -1614,12 +1734,12 @@ template <typename T, int M, int NCOL, int TPW, int WPU, int CW = 1>
 cudaError_t launch_cfg(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                        int iters, cudaStream_t stream, unsigned int* fault) {
     // G_L^n parked (P1) unless recomputing it (P2) fits more groups.
-    constexpr int kG1 = groups_that_fit<M, NCOL, TPW, WPU, true, CW>();
-    constexpr int kG2 = groups_that_fit<M, NCOL, TPW, WPU, false, CW>();
+    constexpr int kG1 = groups_that_fit<T, M, NCOL, TPW, WPU, true, CW>();
+    constexpr int kG2 = groups_that_fit<T, M, NCOL, TPW, WPU, false, CW>();
     constexpr bool kGls = kG1 >= 1 && kG1 >= kG2;
     constexpr int kGroups = kGls ? kG1 : kG2;
     static_assert(kGroups >= 1, "configuration does not fit on one SM");
-    using Lay = Layout<M, NCOL, TPW, WPU, kGls, CW>;
+    using Lay = Layout<T, M, NCOL, TPW, WPU, kGls, CW>;
     auto kern = nystra_tc_kernel<T, M, NCOL, TPW, WPU, kGroups, kGls, CW>;
     const size_t smem = (size_t)kGroups * Lay::PER_GROUP;
     static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device
@@ -1665,6 +1785,16 @@ cudaError_t launch_f32(const void* q, const void* k, const void* v, void* out, l
                         : launch_pool<float, 16, 32>(q, k, v, out, n_units, d, iters, stream, fault, bias);
     }
     return cudaErrorInvalidValue;
+}
+
+// fp32 I/O only in the translation units that take it (F32).
+template <bool F32, int TPW, int WPU>
+cudaError_t launch_f32_if(const void* q, const void* k, const void* v, void* out, long long n_units, int d, int m,
+                          int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
+    if constexpr (F32)
+        return launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias);
+    else
+        return cudaErrorInvalidValue;  // not reached: the caller routes fp32 I/O elsewhere
 }
 
 // Streaming team kernel for 32x32 windows (nystra_stream.cuh, N = 1024 translation unit only).
@@ -1753,8 +1883,12 @@ cudaError_t launch_patches(const void* q, const void* k, const void* v, void* ou
 }  // namespace tc
 }  // namespace nystra
 
-// One translation unit per window size defines its fault word and entry points.
-#define NYSTRA_TC_DEFINE(NAME, TPW, WPU)                                                                     \
+// One translation unit per window size and factor precision defines its fault
+// word and entry points: BF and HF are the kernels' element types for bf16 and
+// fp16 I/O (the plain types carry the derived factors as hi + lo pairs,
+// Single16<...> rounds them to 16 bits); F32 says whether this unit also
+// takes fp32 I/O (the 8x8 stage-pool kernel).
+#define NYSTRA_TC_DEFINE(NAME, TPW, WPU, BF, HF, F32)                                                        \
     namespace nystra {                                                                                       \
     __device__ unsigned int g_fault_tc_##NAME;                                                               \
     }                                                                                                        \
@@ -1774,19 +1908,19 @@ cudaError_t launch_patches(const void* q, const void* k, const void* v, void* ou
         unsigned int* fault = s_fault[dev];                                                                  \
         if (pool != 0) {                                                                                     \
             if (dtype == 1)                                                                                  \
-                return nystra::tc::launch_patches<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m,      \
-                                                                           iters, stream, fault, bias);      \
+                return nystra::tc::launch_patches<BF, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream,  \
+                                                                fault, bias);                                \
             if (dtype == 2)                                                                                  \
-                return nystra::tc::launch_patches<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters,      \
-                                                                    stream, fault, bias);                    \
+                return nystra::tc::launch_patches<HF, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream,  \
+                                                                fault, bias);                                \
             return cudaErrorInvalidValue; /* not reached: fp32 patches take the SIMT path */                 \
         }                                                                                                    \
         if (dtype == 0)                                                                                      \
-            return nystra::tc::launch_f32<TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias);\
+            return nystra::tc::launch_f32_if<F32, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, \
+                                                            bias);                                           \
         if (dtype == 1)                                                                                      \
-            return nystra::tc::launch_n<__nv_bfloat16, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, \
-                                                                 fault, bias);                               \
-        return nystra::tc::launch_n<__half, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias); \
+            return nystra::tc::launch_n<BF, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias); \
+        return nystra::tc::launch_n<HF, TPW, WPU>(q, k, v, out, n_units, d, m, iters, stream, fault, bias);  \
     }                                                                                                        \
     unsigned int take_fault_word_tc_##NAME(cudaError_t* err) {                                               \
         unsigned int w = 0, zero = 0;                                                                        \

@@ -4,4 +4,4 @@
 #include "nystra_tc.cuh"
 #include "nystra_stream.cuh"
 
-NYSTRA_TC_DEFINE(n1024, 128, 8)
+NYSTRA_TC_DEFINE(n1024, 128, 8, __nv_bfloat16, __half, false)

@@ -4,4 +4,4 @@
 #include "nystra_tc.cuh"
 #include "nystra_team.cuh"
 
-NYSTRA_TC_DEFINE(n256, 64, 4)
+NYSTRA_TC_DEFINE(n256, 64, 4, __nv_bfloat16, __half, false)

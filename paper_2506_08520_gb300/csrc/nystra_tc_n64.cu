@@ -4,4 +4,4 @@
 #include "nystra_tc.cuh"
 #include "nystra_pool.cuh"
 
-NYSTRA_TC_DEFINE(n64, 64, 1)
+NYSTRA_TC_DEFINE(n64, 64, 1, __nv_bfloat16, __half, true)

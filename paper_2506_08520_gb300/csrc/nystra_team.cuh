@@ -11,13 +11,19 @@
 // unit k + 1 and then the output of unit k.
 //
 // Token warp r, unit k (buffer b = k mod 2):
-//   wait Q, K rows -> landmarks -> [sync] -> S_L, G_L^n parked -> wait V ->
-//   S_U, partial W_r -> [sync] -> combine into W, m_U -> [sync] -> signal the
-//   core (mbarrier F_b) -> copy Q, K of unit k + 1 -> wait for the core of
-//   unit k - 1 (mbarrier C_{1-b}) -> output of unit k - 1 staged in the V
-//   rows and bulk-stored -> copy V of unit k + 1.
+//   wait Q, K rows -> landmarks -> [sync] -> wait V -> S_U, partial W_r ->
+//   copy the Q rows of unit k - 1 again (into the V rows, now consumed) ->
+//   [sync] -> combine into W, m_U -> [sync] -> signal the core (mbarrier
+//   F_b) -> copy Q, K of unit k + 1 -> wait for the core of unit k - 1
+//   (mbarrier C_{1-b}) and for its Q rows -> output of unit k - 1 (S_L and
+//   G_L^n from those rows and Kbar, then O) written in place over them and
+//   bulk-stored -> copy V of unit k + 1.
 // Core warp, unit k: wait F_b -> G_A^n, iteration, Y^T into buffer b ->
 //   signal C_b.
+// G_L^n is recomputed in the output pass rather than parked: its hi + lo
+// pairs would take 16 KB per unit, which costs a team per SM, while reading a
+// unit's Q rows a second time (3.75 KB per token warp, usually from L2: they
+// were read about one unit earlier) costs no shared memory.
 // [sync] is a named barrier over the four token warps.  Every wait on an
 // mbarrier is bounded; a warp whose wait gives up keeps to the barrier
 // sequence, and the token warps leave the loop together after the next
@@ -29,26 +35,23 @@
 namespace nystra {
 namespace tc {
 
-template <int M, int NCOL>
+template <typename T, int M, int NCOL>
 struct TeamLayout {
     static constexpr int NT = 4, TPW = 64, N = NT * TPW;  // token warps, tokens per token warp
     static constexpr int CWN = M > 16 ? M / 16 : 1;        // core warps (m = 32: distributed core)
     static constexpr int DS = (NCOL == 32) ? 30 : 32;
-    static constexpr int MP = M > 16 ? M : 16, LS = 40, WS = NCOL + 4, YS = MP + 8;
+    static constexpr int MP = M > 16 ? M : 16, LS = LmS<T>::LS, WS = NCOL + 4;
     static constexpr int KTL = (M >= 16) ? M / 16 : 1;
-    static constexpr int GLB = (M >= 16) ? 16 : 8;
     static constexpr size_t STAGE = 3 * (size_t)TPW * DS * 2;  // a token warp's Q, K, V rows
     static constexpr size_t WPART = (size_t)TPW * DS * 2;      // partial W_r after Q (K, V consumed)
     static_assert((size_t)MP * WS * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2, "W partial must fit in K+V");
     // one buffer of per-unit state
-    static constexpr size_t GLF_W = 4 * KTL * 32 * GLB;  // one token warp's G_L^n fragments
     static constexpr size_t B_QB = 0;
-    static constexpr size_t B_KB = B_QB + MP * LS * 2;
-    static constexpr size_t B_W = B_KB + MP * LS * 2;
+    static constexpr size_t B_KB = B_QB + LmS<T>::bytes(MP);
+    static constexpr size_t B_W = B_KB + LmS<T>::bytes(MP);
     static constexpr size_t B_MU = B_W + MP * WS * 4;
-    static constexpr size_t B_YT = B_MU + MP * 4;
-    static constexpr size_t B_GLF = B_YT + ((NCOL * YS * 2 + 15) / 16) * 16;
-    static constexpr size_t BUF = B_GLF + NT * GLF_W;
+    static constexpr size_t B_YT = ((B_MU + MP * 4 + 15) / 16) * 16;
+    static constexpr size_t BUF = ((B_YT + YtS<T, M>::bytes(NCOL) + 127) / 128) * 128;
     // team memory: stages, two buffers, mbarriers
     static constexpr size_t T_BUF = NT * STAGE;
     static constexpr size_t T_BAR = T_BUF + 2 * BUF;  // barQK[4], barV[4], F[2], C[2]
@@ -58,17 +61,17 @@ struct TeamLayout {
     static constexpr int TEAMS = (int)(kSmemLimit / TEAM) < 3 ? (int)(kSmemLimit / TEAM) : 3;
     static constexpr int WARPS = NT + CWN;  // per team
     static_assert(TEAMS >= 1, "team does not fit in shared memory");
-    static_assert(STAGE % 16 == 0 && BUF % 16 == 0 && B_GLF % 16 == 0, "16-byte alignment");
+    static_assert(STAGE % 16 == 0 && BUF % 16 == 0, "16-byte alignment");
 };
 
 template <typename T, int M, int NCOL, int DC, int PW, bool BIAS>
-__global__ void __launch_bounds__(TeamLayout<M, NCOL>::TEAMS * TeamLayout<M, NCOL>::WARPS * 32, 1)
+__global__ void __launch_bounds__(TeamLayout<T, M, NCOL>::TEAMS * TeamLayout<T, M, NCOL>::WARPS * 32, 1)
 nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v,
                    T* __restrict__ out, long long n_units, int d_in, int iters, float sl2, unsigned int* fault,
                    NystraBias bias) {
     static_assert(!BIAS || M <= 16, "a score bias runs with the one-warp core");
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
-    using Lay = TeamLayout<M, NCOL>;
+    using Lay = TeamLayout<T, M, NCOL>;
     constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
                   KTL = Lay::KTL, NCOLC = NCOL;
     constexpr int L = N / M, LPW = TPW / L;
@@ -105,8 +108,10 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             const int b = rem / ((MP - M) * 16), e = rem - b * (MP - M) * 16;
             unsigned char* bb = smem_raw + (size_t)tm * Lay::TEAM + Lay::T_BUF + (size_t)b * Lay::BUF;
             const int jr = M + (e >> 4), p = e & 15;
-            *reinterpret_cast<uint32_t*>(bb + Lay::B_QB + (jr * LS + 2 * p) * 2) = 0u;
-            *reinterpret_cast<uint32_t*>(bb + Lay::B_KB + (jr * LS + 2 * p) * 2) = 0u;
+            landmarks_zero<T>(reinterpret_cast<T*>(bb + Lay::B_QB), jr, jr + 1, 2 * p, 64);
+            landmarks_zero<T>(reinterpret_cast<T*>(bb + Lay::B_QB), jr, jr + 1, 2 * p + 1, 64);
+            landmarks_zero<T>(reinterpret_cast<T*>(bb + Lay::B_KB), jr, jr + 1, 2 * p, 64);
+            landmarks_zero<T>(reinterpret_cast<T*>(bb + Lay::B_KB), jr, jr + 1, 2 * p + 1, 64);
         }
     }
     __syncthreads();
@@ -159,17 +164,24 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     T* Vs = Qs + 2 * td;
     float* wpart = reinterpret_cast<float*>(tb + (size_t)r * Lay::STAGE + Lay::WPART);
     uint64_t* barQK = bars + r;
-    uint64_t* barV = bars + 4 + r;
+    uint64_t* barV = bars + 4 + r;  // V rows, and the Q rows read again for the output (alternately)
     const uint32_t tile_bytes = (uint32_t)(td * sizeof(T));
     auto unit_off = [&](long long unit) { return (size_t)unit * N * d + (size_t)r * td; };
+    // L2 policies: the first read of Q is kept for its second read (the
+    // output pass, about one unit later); every other read is its last.
+    const uint64_t keep = l2_evict_last(), drop = l2_evict_first();
     auto issue_qk = [&](long long unit) {
         mbar_arrive_expect_tx(barQK, 2u * tile_bytes);
-        bulk_g2s(Qs, q + unit_off(unit), tile_bytes, barQK);
-        bulk_g2s(Ks, k + unit_off(unit), tile_bytes, barQK);
+        bulk_g2s_hint(Qs, q + unit_off(unit), tile_bytes, barQK, keep);
+        bulk_g2s_hint(Ks, k + unit_off(unit), tile_bytes, barQK, drop);
     };
     auto issue_v = [&](long long unit) {
         mbar_arrive_expect_tx(barV, tile_bytes);
-        bulk_g2s(Vs, v + unit_off(unit), tile_bytes, barV);
+        bulk_g2s_hint(Vs, v + unit_off(unit), tile_bytes, barV, drop);
+    };
+    auto issue_q_again = [&](long long unit) {  // the output pass's Q rows, into the V rows
+        mbar_arrive_expect_tx(barV, tile_bytes);
+        bulk_g2s_hint(Vs, q + unit_off(unit), tile_bytes, barV, drop);
     };
     auto tsync = [&]() { named_barrier(1 + team, NT * 32); };
     // barrier that also tells every token warp whether any of them failed
@@ -177,9 +189,21 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     uint32_t phase_qk = 0, phase_v = 0;
     bool pend_qk = false, pend_v = false;  // copies issued and not yet seen complete
     bool failed = false;                   // a bounded wait of this warp gave up (warp-uniform)
+    auto wait_v = [&]() {  // bounded wait for the copy on barV (V rows or Q rows again)
+        if (failed) return;
+        if (__all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs))) {
+            phase_v ^= 1u;
+            pend_v = false;
+        } else {
+            failed = true;
+            if (lane == 0) atomicOr(fault, 1u);
+        }
+    };
 
-    // Output of unit kk (its core has run on buffer kk mod 2), staged in the
-    // V rows; returns once the bulk store has read the staging.
+    // Output of unit kk (its core has run on buffer kk mod 2, its Q rows have
+    // been copied again into the V rows): S_L, G_L^n and O tile by tile,
+    // written in place over those Q rows; returns once the bulk store has
+    // read them.
     auto output_unit = [&](long long kk) {
         const int b = (int)(kk & 1);
         if (failed) return;
@@ -189,14 +213,19 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             if (lane == 0) atomicOr(fault, 1u);
             return;
         }
+        wait_v();
+        if (failed) return;
         unsigned char* bb = buf(b);
-        output_rows<T, M, NCOLC, 1, true>(reinterpret_cast<const uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W), Qs,
-                                          reinterpret_cast<const T*>(bb + Lay::B_KB),
-                                          reinterpret_cast<const T*>(bb + Lay::B_YT), Vs, d, g, t, lane, sl2);
-        fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
+        const long long uk = u0 + kk * stride;
+        const float* bLu =
+            BIAS ? bias.L + (size_t)(bias.per_window ? uk : uk % bias.heads) * N * M + (size_t)r * TPW * M : nullptr;
+        output_rows<T, M, NCOLC, 1, false, BIAS>(nullptr, Vs, reinterpret_cast<const T*>(bb + Lay::B_KB),
+                                                 reinterpret_cast<const T*>(bb + Lay::B_YT), Vs, d, g, t, lane, sl2,
+                                                 bLu);
+        fence_proxy_async_smem();  // this lane's writes precede the bulk store
         __syncwarp();
         if (lane == 0) {
-            bulk_s2g(out + unit_off(u0 + kk * stride), Vs, tile_bytes);
+            bulk_s2g(out + unit_off(uk), Vs, tile_bytes);
             bulk_commit();
             bulk_wait_read_all();
         }
@@ -209,11 +238,11 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     }
     pend_qk = pend_v = u0 < n_units;
     long long kk = 0;
+    bool broke = false;  // the token warps left the loop together after a failed wait
     for (;; ++kk) {
         const long long u = u0 + kk * stride;
         if (u >= n_units) break;
         const long long bs = BIAS ? (bias.per_window ? u : u % bias.heads) : 0;
-        const float* bLu = BIAS ? bias.L + (size_t)bs * N * M : nullptr;
         const float* bUu = BIAS ? bias.U + (size_t)bs * M * N : nullptr;
         const int b = (int)(kk & 1);
         unsigned char* bb = buf(b);
@@ -233,30 +262,12 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         // ---------------- landmarks (Algorithm 1 step 1) ----------------
         landmarks_mma<T, TPW, L, PW>(Qs, qbar, r * LPW, d, g, t);
         landmarks_mma<T, TPW, L, PW>(Ks, kbar, r * LPW, d, g, t);
-        if (tsync_or(failed)) break;
-        // ---------------- S_L, G_L^n fragments parked in buffer b ----------------
-        {
-            uint32_t* glf = reinterpret_cast<uint32_t*>(bb + Lay::B_GLF + r * Lay::GLF_W);
-#pragma unroll
-            for (int tm = 0; tm < 4; ++tm) {
-                typename Opnd<T>::Reg f[KTL][4];
-                gl_tile<T, M, KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
-                                         BIAS ? bLu + (size_t)(r * TPW + 16 * tm + g) * M : nullptr);
-#pragma unroll
-                for (int kq = 0; kq < KTL; ++kq) GlPark<T, M>::put(glf, (tm * KTL + kq) * 32 + lane, f[kq]);
-            }
+        if (tsync_or(failed)) {
+            broke = true;
+            break;
         }
         // ---------------- bounded wait for V ----------------
-        if (!failed) {
-            const bool ok_v = __all_sync(0xffffffffu, mbar_wait_bounded(barV, phase_v, kWaitNs));
-            if (ok_v) {
-                phase_v ^= 1u;
-                pend_v = false;
-            } else {
-                failed = true;
-                if (lane == 0) atomicOr(fault, 1u);
-            }
-        }
+        wait_v();
         // ---------------- S_U, partial W_r and row maxima ----------------
         constexpr int MT = (M + 15) / 16;
         float mU[MT][2];
@@ -273,11 +284,15 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         combine_partials<MP, NCOLC, WS, NT>(reinterpret_cast<const float*>(tb + Lay::WPART), Lay::STAGE / 4,
                                              reinterpret_cast<float*>(bb + Lay::B_W),
                                              reinterpret_cast<float*>(bb + Lay::B_MU), r, lane);
-        if (tsync_or(failed)) break;
+        if (tsync_or(failed)) {
+            broke = true;
+            break;
+        }
         // ---------------- hand buffer b to the core warp ----------------
         __syncwarp();
         if (lane == 0) mbar_arrive(barF + b);
-        // Q, K and the partials are consumed: copy the next unit's Q and K rows.
+        // Q, K, V and the partials are consumed: copy the next unit's Q and K
+        // rows, and the previous unit's Q rows again (into the V rows) for its output.
         const long long un = u + stride;
         fence_proxy_async_smem();
         __syncwarp();
@@ -285,15 +300,25 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             if (lane == 0) issue_qk(un);
             pend_qk = true;
         }
+        if (kk >= 1 && !failed) {
+            if (lane == 0) issue_q_again(u - stride);
+            pend_v = true;
+        }
         // ---------------- output of the previous unit ----------------
         if (kk >= 1) output_unit(kk - 1);
-        // The V rows are free (consumed, and the staging has been read).
+        // The V rows are free (the output's staging has been read).
         if (un < n_units && !failed) {
             if (lane == 0) issue_v(un);
             pend_v = true;
         }
     }
-    if (kk >= 1) output_unit(kk - 1);
+    if (kk >= 1 && !broke && !failed) {  // the last unit's output: its Q rows again, then the output
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) issue_q_again(u0 + (kk - 1) * stride);
+        pend_v = true;
+        output_unit(kk - 1);
+    }
     if (lane == 0) bulk_wait_all();  // output stores complete before exit
     // Fault path only: copies still in flight land before the CTA's memory is released.
     if (pend_qk) (void)__all_sync(0xffffffffu, mbar_wait_bounded(barQK, phase_qk, kWaitNs));
@@ -303,7 +328,7 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 template <typename T, int M, int NCOL, int DC, int PW, bool BIAS = false>
 cudaError_t launch_team_dc(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                         int iters, cudaStream_t stream, unsigned int* fault, NystraBias bias = {}) {
-    using Lay = TeamLayout<M, NCOL>;
+    using Lay = TeamLayout<T, M, NCOL>;
     auto kern = nystra_team_kernel<T, M, NCOL, DC, PW, BIAS>;
     const size_t smem = (size_t)Lay::TEAMS * Lay::TEAM;
     static std::atomic<int> s_blocks[kMaxDevices];  // persistent grid size per device

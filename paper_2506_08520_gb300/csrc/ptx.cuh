@@ -6,6 +6,8 @@
 #include <cuda_fp16.h>
 #include <stdint.h>
 
+#include "common.cuh"
+
 namespace nystra {
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -254,6 +256,14 @@ template <> struct Mma16<__half> {
 // elements.  fp32 I/O: each element is split into bf16 hi + lo (16
 // significant bits each, fp32's range) and a product takes three MMAs
 // (lo*hi + hi*lo + hi*hi), about 2^-16 relative error per product.
+//
+// Derived operands (DReg: the landmarks, G_L^n, G_U^n and Y, which the
+// kernels compute in fp32) are always such hi + lo pairs in the MMA type, so
+// that they keep 16 (bf16) or 22 (fp16) significant bits: rounding them to a
+// single 16-bit value perturbs the Nystrom output by the method's own
+// amplification of the landmark-block conditioning, which grows quickly as
+// attention sharpens.  A product of a raw I/O operand with a derived one
+// takes two MMAs (lo first), of two derived operands three.
 struct RegPair {
     uint32_t hi, lo;
 };
@@ -261,6 +271,7 @@ template <typename T>
 struct Opnd {
     using Op = Mma16<T>;
     using Reg = uint32_t;
+    using DReg = RegPair;
     static constexpr bool kNarrowRange = Op::kNarrowRange;
     static __device__ __forceinline__ Reg ld(const T* p) { return *reinterpret_cast<const uint32_t*>(p); }
     static __device__ __forceinline__ Reg pk(float a, float b) { return Op::pack(a, b); }
@@ -274,11 +285,45 @@ struct Opnd {
     static __device__ __forceinline__ void st2(T* p, float a, float b) {
         *reinterpret_cast<uint32_t*>(p) = Op::pack(a, b);
     }
+    // ---- derived operands ----
+    static __device__ __forceinline__ DReg dpk(float a, float b) {
+        const uint32_t h = Op::pack(a, b);
+        const float2 hf = Op::unpack(h);
+        return {h, Op::pack(a - hf.x, b - hf.y)};
+    }
+    static __device__ __forceinline__ DReg dzero() { return {0u, 0u}; }
+    static __device__ __forceinline__ DReg dtr(DReg r) { return {movmatrix_trans(r.hi), movmatrix_trans(r.lo)}; }
+    // raw x derived
+    static __device__ __forceinline__ void mma(float (&c)[4], const Reg (&a)[4], DReg b0, DReg b1) {
+        Op::k16(c, a, b0.lo, b1.lo);
+        Op::k16(c, a, b0.hi, b1.hi);
+    }
+    // derived x raw
+    static __device__ __forceinline__ void mma(float (&c)[4], const DReg (&a)[4], Reg b0, Reg b1) {
+        const uint32_t ah[4] = {a[0].hi, a[1].hi, a[2].hi, a[3].hi};
+        const uint32_t al[4] = {a[0].lo, a[1].lo, a[2].lo, a[3].lo};
+        Op::k16(c, al, b0, b1);
+        Op::k16(c, ah, b0, b1);
+    }
+    // derived x derived (the lo*lo term is below the pair's precision)
+    static __device__ __forceinline__ void mma(float (&c)[4], const DReg (&a)[4], DReg b0, DReg b1) {
+        const uint32_t ah[4] = {a[0].hi, a[1].hi, a[2].hi, a[3].hi};
+        const uint32_t al[4] = {a[0].lo, a[1].lo, a[2].lo, a[3].lo};
+        Op::k16(c, al, b0.hi, b1.hi);
+        Op::k16(c, ah, b0.lo, b1.lo);
+        Op::k16(c, ah, b0.hi, b1.hi);
+    }
+    static __device__ __forceinline__ void mma8(float (&c)[4], DReg a0, DReg a1, DReg b0) {
+        Op::k8(c, a0.lo, a1.lo, b0.hi);
+        Op::k8(c, a0.hi, a1.hi, b0.lo);
+        Op::k8(c, a0.hi, a1.hi, b0.hi);
+    }
 };
 template <>
 struct Opnd<float> {
     using Op = Mma16<__nv_bfloat16>;
     using Reg = RegPair;
+    using DReg = RegPair;
     static constexpr bool kNarrowRange = false;
     static __device__ __forceinline__ Reg pk(float a, float b) {
         const uint32_t h = Op::pack(a, b);
@@ -307,6 +352,102 @@ struct Opnd<float> {
     static __device__ __forceinline__ void st2(float* p, float a, float b) {
         *reinterpret_cast<float2*>(p) = make_float2(a, b);
     }
+    static __device__ __forceinline__ DReg dpk(float a, float b) { return pk(a, b); }
+    static __device__ __forceinline__ DReg dzero() { return zero(); }
+    static __device__ __forceinline__ DReg dtr(DReg r) { return tr(r); }
+};
+
+// Single16<T>: derived operands rounded to the 16-bit I/O type (one register,
+// one MMA per product), as a caller selecting NYSTRA_FACTORS_16 asks for.
+template <typename T>
+struct Mma16<Single16<T>> : Mma16<T> {};
+template <typename T>
+struct Opnd<Single16<T>> {
+    using Op = Mma16<T>;
+    using Reg = uint32_t;
+    using DReg = uint32_t;
+    static constexpr bool kNarrowRange = Op::kNarrowRange;
+    static __device__ __forceinline__ Reg ld(const Single16<T>* p) { return *reinterpret_cast<const uint32_t*>(p); }
+    static __device__ __forceinline__ Reg pk(float a, float b) { return Op::pack(a, b); }
+    static __device__ __forceinline__ Reg tr(Reg r) { return movmatrix_trans(r); }
+    static __device__ __forceinline__ Reg zero() { return 0u; }
+    static __device__ __forceinline__ Reg one() { return Op::kOne; }
+    static __device__ __forceinline__ void mma(float (&c)[4], const Reg (&a)[4], Reg b0, Reg b1) {
+        Op::k16(c, a, b0, b1);
+    }
+    static __device__ __forceinline__ void mma8(float (&c)[4], Reg a0, Reg a1, Reg b0) { Op::k8(c, a0, a1, b0); }
+    static __device__ __forceinline__ void st2(Single16<T>* p, float a, float b) {
+        *reinterpret_cast<uint32_t*>(p) = Op::pack(a, b);
+    }
+    static __device__ __forceinline__ DReg dpk(float a, float b) { return pk(a, b); }
+    static __device__ __forceinline__ DReg dzero() { return 0u; }
+    static __device__ __forceinline__ DReg dtr(DReg r) { return tr(r); }
+};
+
+// Storage of derived operands in shared memory.  16-bit I/O: the hi and lo
+// parts of a row live in one row of the T-typed array, lo at element offset
+// `lo` (LmS: landmark rows of 32 features, hi in columns 0..31 and lo in
+// 32..63, row stride 72 = 36 words, so the 8 rows of a fragment load fall in
+// distinct banks); fp32 I/O: one fp32 value, split when loaded.
+template <typename T>
+struct DSt {
+    static __device__ __forceinline__ void put(T* p, int lo, float x) {
+        const T h = from_f32<T>(x);
+        p[0] = h;
+        p[lo] = from_f32<T>(x - to_f32(h));
+    }
+    static __device__ __forceinline__ void zero(T* p, int lo) {
+        p[0] = from_f32<T>(0.f);
+        p[lo] = from_f32<T>(0.f);
+    }
+    // the pair register of elements p[0], p[1]
+    static __device__ __forceinline__ RegPair ld(const T* p, int lo) {
+        return {*reinterpret_cast<const uint32_t*>(p), *reinterpret_cast<const uint32_t*>(p + lo)};
+    }
+};
+template <>
+struct DSt<float> {
+    static __device__ __forceinline__ void put(float* p, int, float x) { p[0] = x; }
+    static __device__ __forceinline__ void zero(float* p, int) { p[0] = 0.f; }
+    static __device__ __forceinline__ RegPair ld(const float* p, int) { return Opnd<float>::ld(p); }
+};
+template <typename T>
+struct DSt<Single16<T>> {
+    static __device__ __forceinline__ void put(Single16<T>* p, int, float x) { p[0] = from_f32<Single16<T>>(x); }
+    static __device__ __forceinline__ void zero(Single16<T>* p, int) { p[0] = from_f32<Single16<T>>(0.f); }
+    static __device__ __forceinline__ uint32_t ld(const Single16<T>* p, int) {
+        return *reinterpret_cast<const uint32_t*>(p);
+    }
+};
+// Landmark rows (Qbar, Kbar): row stride and lo offset in elements of T.
+template <typename T>
+struct LmS {
+    static constexpr int LS = sizeof(T) == 2 ? 72 : 40;
+    static constexpr int LO = sizeof(T) == 2 ? 32 : 0;
+    static constexpr size_t bytes(int rows) { return (size_t)rows * LS * sizeof(T); }
+};
+template <typename T>
+struct LmS<Single16<T>> {  // one 16-bit value per element, row stride 40 (20 words: conflict-free)
+    static constexpr int LS = 40;
+    static constexpr int LO = 0;
+    static constexpr size_t bytes(int rows) { return (size_t)rows * LS * 2; }
+};
+// Y^T rows (features and the ones column) over MY = max(16, m) landmarks:
+// 16-bit I/O hi in columns 0..MY-1, lo in MY..2MY-1, row stride 2 MY + 8
+// (fragment loads conflict-free); fp32 I/O stride MY + 8.
+template <typename T, int M>
+struct YtS {
+    static constexpr int MY = M < 16 ? 16 : M;
+    static constexpr int YS = sizeof(T) == 2 ? 2 * MY + 8 : MY + 8;
+    static constexpr int LO = sizeof(T) == 2 ? MY : 0;
+    static constexpr size_t bytes(int ncol) { return (((size_t)ncol * YS * sizeof(T)) + 15) / 16 * 16; }
+};
+template <typename T, int M>
+struct YtS<Single16<T>, M> {
+    static constexpr int MY = M < 16 ? 16 : M;
+    static constexpr int YS = MY + 8;
+    static constexpr int LO = 0;
+    static constexpr size_t bytes(int ncol) { return (((size_t)ncol * YS * 2) + 15) / 16 * 16; }
 };
 
 }  // namespace nystra

@@ -86,7 +86,8 @@ def run_qkv(wl: workloads.Workload, l2_bytes: int, peak: float, reps: int = 50) 
 
     def fused(i):
         xs, o = sets[i]
-        binding.nystra_qkv(xs, w, wl.heads, wl.m, wl.iters, pooled=pooled, out=o, landmarks=wl.landmarks)
+        binding.nystra_qkv(xs, w, wl.heads, wl.m, wl.iters, pooled=pooled, out=o, landmarks=wl.landmarks,
+                           factors=wl.factors)
 
     def unfused(i):
         xs, o = sets[i]
@@ -94,9 +95,10 @@ def run_qkv(wl: workloads.Workload, l2_bytes: int, peak: float, reps: int = 50) 
         q, k, v = (y.view(wl.n_windows, wl.N, 3, wl.heads, wl.d)[:, :, j].transpose(1, 2).contiguous()
                    for j in range(3))
         if pooled is None:
-            binding.nystra(q, k, v, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+            binding.nystra(q, k, v, wl.m, wl.iters, out=o, landmarks=wl.landmarks, factors=wl.factors)
         else:
-            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=o, landmarks=wl.landmarks,
+                                  factors=wl.factors)
 
     t_f = _median_ms(fused, n_sets, reps)
     t_u = _median_ms(unfused, n_sets, max(10, reps // 5))
@@ -132,9 +134,10 @@ def run(name: str, l2_bytes: int, peak: float, reps: int = 50, exact_reps: int =
         for wl, ss, pb in zip(parts, sets, pooled):
             a, b, c, o = ss[i]
             if pb is None:
-                binding.nystra(a, b, c, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+                binding.nystra(a, b, c, wl.m, wl.iters, out=o, landmarks=wl.landmarks, factors=wl.factors)
             else:
-                binding.nystra_biased(a, b, c, pb, wl.m, wl.iters, out=o, landmarks=wl.landmarks)
+                binding.nystra_biased(a, b, c, pb, wl.m, wl.iters, out=o, landmarks=wl.landmarks,
+                                      factors=wl.factors)
 
     def exact(i):
         for ss in sets:

@@ -39,6 +39,7 @@ class Workload:
     landmarks: str = "segments"  # landmark pooling: "segments" | "patches"
     bias: str = ""               # score bias: "" (none) | "relpos" (per-head relative-position bias)
     front: str = ""              # "" (inputs are Q, K, V) | "qkv" (inputs are the tokens X and W_QKV)
+    factors: str = "pairs"       # derived factors: "pairs" (hi + lo, default) | "16" (NYSTRA_FACTORS_16)
 
     @property
     def units(self) -> int:
@@ -100,6 +101,10 @@ for _w in (8, 16, 32):
 for _name in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16"):
     WORKLOADS[_name + "-patches"] = WORKLOADS[_name].with_(name=_name + "-patches", landmarks="patches")
     WORKLOADS[_name + "-relpos"] = WORKLOADS[_name].with_(name=_name + "-relpos", bias="relpos")
+# The same inputs with the derived factors rounded to 16 bits (NYSTRA_FACTORS_16).
+for _name in ("swinir256-bf16", "sr720p-w8-m16-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16",
+              "sr720p-w32-m32-bf16", "large-w16-m64", "large-w32-m32", "uformer-s1"):
+    WORKLOADS[_name + "-f16"] = WORKLOADS[_name].with_(name=_name + "-f16", factors="16")
 # The same windows given as tokens X and projection weights (fused Q/K/V projection).
 for _name in ("swinir256-bf16", "uformer-s1", "uformer-s4", "sr720p-w8-m16-bf16", "sr720p-w8-m16-f16",
               "swinir256-bf16-relpos"):
