@@ -14,7 +14,7 @@
  * (window, head) pair with Q, K, V in R^{N x d}, stored row-major and
  * contiguous; unit u starts at offset u*N*d.  All arithmetic is float64.
  *
- * Readings where the paper is silent (each also listed in the design notes):
+ * Readings where the paper is silent:
  *   - landmarks are means over m contiguous, non-overlapping segments of
  *     L = N/m tokens in the window's token order (Sec. 2.2 "average pooling
  *     over non-overlapping windows"); m must divide N.  The other reading,

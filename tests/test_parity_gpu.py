@@ -8,7 +8,8 @@ import torch
 import oracle
 
 from paper_2506_08520_gb300 import binding, workloads
-from tests.parity import TOL, check_exact, check_nystra, sample_units
+from tests.parity import (TOL, check_exact, check_nystra, gpu_nystra, io_ulp_sensitivity, nystra_float32,
+                          per_unit_rel, sample_units, units_view)
 
 pytestmark = pytest.mark.gpu
 
@@ -75,17 +76,27 @@ def test_nystra_small(units, N, d, m, dtype):
 ])
 def test_nystra_edge_cases(N, d, m, iters, dtype):
     q, k, v = workloads.random_qkv(3, N, d, dtype, seed=N + d + m + iters)
-    err, worst = check_nystra(q, k, v, m, iters)
-    tol = TOL[dtype]
-    if iters > 6:
-        # Beyond the paper's 4-6 iterations the computed inverse inverts smaller
-        # singular values, and round-off in G_A^n is amplified by about
-        # ||G_A^n||_2 ||Z||_2 (about 17-20 at 6 iterations on these inputs, where
-        # the 1e-4 fp32 bar applies); scale the bar by that growth.
-        kappa = max(np.linalg.norm(st["GAn"], 2) * np.linalg.norm(st["Z"], 2)
-                    for st in (oracle.nystra_stages(q[u], k[u], v[u], m, iters) for u in range(3)))
-        tol = tol * max(1.0, kappa / 20.0)
-    assert err <= tol, f"max rel err {err:.3e} at unit {worst} (tol {tol:.2e})"
+    if iters <= 6:  # the paper's iteration counts (Sec. 3.1: 4-6; Table 6: 1, 3, 6): the fixed bar
+        err, worst = check_nystra(q, k, v, m, iters)
+        assert err <= TOL[dtype], f"max rel err {err:.3e} at unit {worst}"
+        return
+    # Beyond them the iteration inverts ever smaller singular values of G_A^n
+    # and the method itself amplifies rounding of its inputs.  A unit's bar is
+    # the larger of the fixed one and the float64 oracle's own response:
+    # 16-bit I/O, to one ulp of the I/O type on every element of Q, K and V;
+    # fp32 I/O (the SIMT path, fp32 throughout), to evaluating the same
+    # algorithm in float32 (4x: the kernel's products accumulate in another
+    # order).
+    out = units_view(gpu_nystra(q, k, v, m, iters).cpu()).double().numpy()
+    ref = oracle.nystra_attention(units_view(q), units_view(k), units_view(v), m, iters)
+    assert np.isfinite(out).all()
+    err = per_unit_rel(out, ref)
+    if dtype == "f32":
+        bar = np.maximum(TOL[dtype], 4.0 * per_unit_rel(nystra_float32(q, k, v, m, iters), ref))
+    else:
+        bar = np.maximum(TOL[dtype], io_ulp_sensitivity(q, k, v, m, iters))
+    w = int(np.argmax(err / bar))
+    assert (err <= bar).all(), f"unit {w}: err {err[w]:.3e} > bar {bar[w]:.3e}"
 
 
 # Full-size workloads: the GPU computes every unit, the oracle a sample.  All
@@ -253,10 +264,10 @@ def test_maximum_iteration_count_stays_finite(N, d, m, dtype):
 @pytest.mark.parametrize("dtype", ["bf16", "f16"])
 @pytest.mark.parametrize("N,d,m", [(64, 30, 16), (256, 30, 16), (1024, 30, 16), (256, 30, 32)])
 def test_parity_holds_for_sharper_logits(N, d, m, dtype):
-    # Q, K scaled by 1.25: logit standard deviation 1.56 instead of 1.  The
-    # bar holds here; for much sharper attention G_A^n becomes so
-    # ill-conditioned that six iterations amplify any rounding of the landmarks
-    # and blocks (see the design notes' precision envelope).
+    # Q, K scaled by 1.25: logit standard deviation 1.56 instead of 1; the
+    # fixed bar holds for every unit.  Sharper attention makes G_A^n
+    # ill-conditioned enough that some units' bars come from the oracle's own
+    # sensitivity (test_sharp_gpu.py).
     q, k, v = workloads.random_qkv(8, N, d, "f32", seed=N + m + 5)
     q, k, v = ((x * (1.25 if i < 2 else 1.0)).to(workloads.DTYPES[dtype]) for i, x in enumerate((q, k, v)))
     err, worst = check_nystra(q, k, v, m, 6)

@@ -172,3 +172,62 @@ def test_fused_projection_score_bias_variants(heads, d, dtype, per_window):
                                       np.broadcast_to(B32.astype(np.float64), (nw, heads, 64, 64)))
     err = per_unit_rel(out.double().numpy(), ref)
     assert err.max() <= TOL[dtype], f"max rel err {err.max():.3e} at unit {int(err.argmax())}"
+
+
+@pytest.mark.parametrize("m,pool,bias", [(16, "segments", "window"), (8, "segments", None), (16, "patches", None),
+                                         (8, "segments", "head")])
+def test_shared_stage_handoff_over_many_windows(m, pool, bias):
+    """C = 60 <= 64: two warps share each Q/K/V stage and hand it over through
+    the stage's bounded mbarrier.  4096 windows give every CTA dozens of
+    windows, so every warp waits on the hand-off many times: with a per-window
+    score bias, with m = 8 and with square patches.  Sampled units against
+    the oracle."""
+    nw, heads, d = 4096, 2, 30
+    x, w, b = workloads.random_x_wqkv(nw, 64, heads, d, "bf16", seed=m + len(pool) + (0 if bias is None else 7))
+    pooled, B = None, None
+    if bias is not None:
+        B = workloads.relpos_bias(8, heads, seed=3)[None].astype(np.float32)      # [1, heads, N, N]
+        if bias == "window":
+            B = np.ascontiguousarray(B + _window_masks(nw, seed=4)[:, None].astype(np.float32))
+        pooled = binding.pool_bias(torch.from_numpy(B).cuda(), m, pool)
+    out = _run(x, w, b, heads, m, pool=pool, pooled=pooled)
+    idx = sample_units(nw * heads, 160)
+    win, head = idx // heads, idx % heads
+    uw = np.unique(win)
+    q, k, v = oracle.project_qkv(x[torch.from_numpy(uw)], w, b, heads)
+    pos = np.searchsorted(uw, win)
+    bsl = None
+    if B is not None:
+        bsl = B.astype(np.float64)[win if B.shape[0] > 1 else np.zeros_like(win), head]
+    ref = oracle.nystra_attention(q[pos, head], k[pos, head], v[pos, head], m, 6, pool, bsl)
+    got = out.reshape(nw * heads, 64, d)[torch.from_numpy(idx)].double().numpy()
+    err = per_unit_rel(got, ref)
+    assert err.max() <= TOL["bf16"], f"max rel err {err.max():.3e} at sampled unit {int(idx[err.argmax()])}"
+
+
+def test_fused_projection_with_16bit_factors():
+    """NYSTRA_FACTORS_16 on the fused path: the same bar on soft inputs, and
+    a different (single-rounding) kernel from the default."""
+    x, w, b = workloads.random_x_wqkv(6, 64, 6, 30, "bf16", seed=21)
+    ref = oracle.nystra_attention_qkv(x, w, b, 6, 16, 6)
+    outs = []
+    for factors in ("pairs", "16"):
+        o = binding.nystra_qkv(x.cuda(), w.cuda(), 6, 16, 6, b_qkv=b.cuda(), factors=factors)
+        torch.cuda.synchronize()
+        assert binding.status() == binding.NYSTRA_OK
+        outs.append(o.cpu())
+        assert per_unit_rel(o.cpu().double().numpy(), ref).max() <= TOL["bf16"]
+    assert not torch.equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("s", [2.0, 4.0])
+def test_fused_projection_sharp_attention_is_finite(s):
+    """W_Q, W_K scaled by s (logit std s^2): finite wherever the oracle is."""
+    x, w, b = workloads.random_x_wqkv(8, 64, 6, 30, "bf16", seed=int(s) + 30)
+    C = 180
+    w = w.clone()
+    w[:2 * C] = (w[:2 * C].float() * s).bfloat16()
+    out = _run(x, w, b, 6, 16)
+    ref = oracle.nystra_attention_qkv(x, w, b, 6, 16, 6)
+    fin = np.isfinite(ref).all(axis=(-2, -1))
+    assert np.isfinite(out.double().numpy()[fin]).all()
