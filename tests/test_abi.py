@@ -221,3 +221,42 @@ def test_attention_qkv_argument_validation(lib, args, code):
 def test_qkv_max_width_matches_the_header():
     text = open(HEADER).read()
     assert f"#define NYSTRA_QKV_MAX_C {nb.QKV_MAX_C}" in text
+
+
+@pytest.mark.parametrize("lm,m,nw,code", [
+    (nb.NYSTRA_FACTORS_16, 16, 0, nb.NYSTRA_OK),                               # segments, 16-bit factors: valid
+    (nb.NYSTRA_FACTORS_16 | nb.NYSTRA_LANDMARKS_PATCHES, 16, 0, nb.NYSTRA_OK),  # square patches too
+    (nb.NYSTRA_FACTORS_16 | nb.NYSTRA_LANDMARKS_PATCHES, 8, 4, nb.NYSTRA_EINVAL),  # 8 is no square
+    (32, 16, 4, nb.NYSTRA_EINVAL),                                            # no such flag
+    (nb.NYSTRA_FACTORS_16 | 2, 16, 4, nb.NYSTRA_EINVAL),                      # no such pooling
+])
+def test_factor_flag_validation(lib, lm, m, nw, code):
+    assert nb.nystra_attention_ex(P, 2 * P, 3 * P, 64 * P, nw, 2, 64, 30, m, 6, lm, 1, None) == code
+
+
+def test_factor_flag_is_refused_where_it_has_no_meaning(lib):
+    # pooling a bias and the stage dump take a pooling only
+    assert nb.nystra_pool_bias(P, 1, 64, 16, nb.NYSTRA_FACTORS_16, 2 * P, 3 * P, 4 * P, None) == nb.NYSTRA_EINVAL
+    assert nb.nystra_debug_stages(P, 2 * P, 3 * P, 1, 1, 64, 30, 16, 6, nb.NYSTRA_FACTORS_16, 1, 0, 4 * P,
+                                  None) == nb.NYSTRA_EINVAL
+
+
+def _has_gpu():
+    import torch
+    return torch.cuda.is_available()
+
+
+@pytest.mark.skipif(_has_gpu(), reason="checks the answer of a host without a usable sm_103 device")
+def test_valid_calls_without_an_sm103_device_return_edevice(lib):
+    # every argument is valid, so the calls reach the device check, which
+    # finds no sm_103 GPU and refuses before any launch
+    assert nb.nystra_attention(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 16, 6, 1, None) == nb.NYSTRA_EDEVICE
+    assert nb.nystra_attention_ex(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 16, 6, nb.NYSTRA_FACTORS_16, 1,
+                                  None) == nb.NYSTRA_EDEVICE
+    assert nb.exact_window_attention(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 1, None) == nb.NYSTRA_EDEVICE
+    assert nb.nystra_pool_bias(P, 1, 64, 16, 0, 2 * P, 3 * P, 4 * P, None) == nb.NYSTRA_EDEVICE
+    assert nb.nystra_attention_qkv(P, 2 * P, 0, 64 * P, 4, 2, 64, 30, 16, 6, 0, 0, 0, 0, 0, 1,
+                                   None) == nb.NYSTRA_EDEVICE
+    assert nb.nystra_debug_stages(P, 2 * P, 3 * P, 4, 2, 64, 30, 16, 6, 0, 1, 0, 4 * P, None) == nb.NYSTRA_EDEVICE
+    assert nb.lib().nystra_debug_wait_timeout(10_000, None) == nb.NYSTRA_EDEVICE
+    assert nb.strerror(nb.NYSTRA_EDEVICE) == "unsupported device (sm_103 required)"
