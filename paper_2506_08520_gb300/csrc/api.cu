@@ -204,13 +204,16 @@ int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, v
                          const float* bias_A, int bias_windows, int dtype, void* stream) {
     if (dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;  // 16-bit I/O only
     if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
-    if (N != 64 || d_h < 2 || d_h > 32 || d_h % 2 != 0 || (m != 8 && m != 16)) return NYSTRA_EINVAL;
+    if (N != 64 && N != 256 && N != 1024) return NYSTRA_EINVAL;
+    if (d_h < 2 || d_h > 32 || d_h % 2 != 0) return NYSTRA_EINVAL;
+    if (m != 8 && m != 16 && !(N == 1024 && m == 32)) return NYSTRA_EINVAL;
     if (iters < 0 || iters > 12) return NYSTRA_EINVAL;
     if (!flags_ok(landmarks)) return NYSTRA_EINVAL;
     const bool patches = (landmarks & kPoolMask) == NYSTRA_LANDMARKS_PATCHES;
     const bool s16 = (landmarks & NYSTRA_FACTORS_16) != 0;
     if (patches && m != 16) return NYSTRA_EINVAL;
     if ((long long)heads * d_h > NYSTRA_QKV_MAX_C) return NYSTRA_EINVAL;
+    if (bias_L && m > 16) return NYSTRA_EINVAL;  // a score bias runs with the one-warp core
     if ((long long)n_windows * heads == 0) return NYSTRA_OK;
     const size_t C = (size_t)heads * d_h;
     const size_t xb = (size_t)n_windows * N * C * 2, wb = 3 * C * C * 2, ob = xb;
@@ -237,16 +240,29 @@ int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, v
     if (!device_ok()) return NYSTRA_EDEVICE;
     const cudaStream_t st = (cudaStream_t)stream;
     cudaError_t e;
-    if (dtype == NYSTRA_BF16)
-        e = s16 ? nystra_host::launch_nystra_qkv_bf16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
-                                                          pool, st, bp)
-                : nystra_host::launch_nystra_qkv_bf16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
-                                                      st, bp);
-    else
-        e = s16 ? nystra_host::launch_nystra_qkv_f16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
-                                                         pool, st, bp)
-                : nystra_host::launch_nystra_qkv_f16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters, pool,
-                                                     st, bp);
+    if (N == 64) {
+        if (dtype == NYSTRA_BF16)
+            e = s16 ? nystra_host::launch_nystra_qkv_bf16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                              pool, st, bp)
+                    : nystra_host::launch_nystra_qkv_bf16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                          pool, st, bp);
+        else
+            e = s16 ? nystra_host::launch_nystra_qkv_f16_s16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                             pool, st, bp)
+                    : nystra_host::launch_nystra_qkv_f16(x, w_qkv, b_qkv, out, n_windows, heads, d_h, m, iters,
+                                                         pool, st, bp);
+    } else {  // 16x16 and 32x32 windows: the streaming kernel's structure
+        if (dtype == NYSTRA_BF16)
+            e = s16 ? nystra_host::launch_nystra_qkvs_bf16_s16(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m,
+                                                               iters, pool, st, bp)
+                    : nystra_host::launch_nystra_qkvs_bf16(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iters,
+                                                           pool, st, bp);
+        else
+            e = s16 ? nystra_host::launch_nystra_qkvs_f16_s16(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m,
+                                                              iters, pool, st, bp)
+                    : nystra_host::launch_nystra_qkvs_f16(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iters,
+                                                          pool, st, bp);
+    }
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
@@ -325,11 +341,13 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[12])(cudaError_t*) = {
-        take_fault_word_tc_n64,      take_fault_word_tc_n256,      take_fault_word_tc_n1024,
-        take_fault_word_tc_n64_s16,  take_fault_word_tc_n256_s16,  take_fault_word_tc_n1024_s16,
-        take_fault_word_exact_tc,    take_fault_word_debug,        take_fault_word_qkv_bf16,
-        take_fault_word_qkv_f16,     take_fault_word_qkv_bf16_s16, take_fault_word_qkv_f16_s16};
+    unsigned int (*const take[16])(cudaError_t*) = {
+        take_fault_word_tc_n64,       take_fault_word_tc_n256,       take_fault_word_tc_n1024,
+        take_fault_word_tc_n64_s16,   take_fault_word_tc_n256_s16,   take_fault_word_tc_n1024_s16,
+        take_fault_word_exact_tc,     take_fault_word_debug,         take_fault_word_qkv_bf16,
+        take_fault_word_qkv_f16,      take_fault_word_qkv_bf16_s16,  take_fault_word_qkv_f16_s16,
+        take_fault_word_qkvs_bf16,    take_fault_word_qkvs_f16,      take_fault_word_qkvs_bf16_s16,
+        take_fault_word_qkvs_f16_s16};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

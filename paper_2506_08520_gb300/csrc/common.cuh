@@ -147,6 +147,23 @@ cudaError_t launch_nystra_qkv_bf16_s16(const void* x, const void* wqkv, const fl
 cudaError_t launch_nystra_qkv_f16_s16(const void* x, const void* wqkv, const float* bqkv, void* out,
                                       long long n_windows, int heads, int d, int m, int iters, int pool,
                                       cudaStream_t stream, const nystra::NystraBias* bias);
+// Fused Q/K/V projection + PnP-Nystra for N = 256 or 1024 (nystra_qkvs_*.cu).
+cudaError_t launch_nystra_qkvs_bf16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                    long long n_windows, int heads, int N, int d, int m, int iters, int pool,
+                                    cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkvs_f16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                   long long n_windows, int heads, int N, int d, int m, int iters, int pool,
+                                   cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkvs_bf16_s16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                        long long n_windows, int heads, int N, int d, int m, int iters, int pool,
+                                        cudaStream_t stream, const nystra::NystraBias* bias);
+cudaError_t launch_nystra_qkvs_f16_s16(const void* x, const void* wqkv, const float* bqkv, void* out,
+                                       long long n_windows, int heads, int N, int d, int m, int iters, int pool,
+                                       cudaStream_t stream, const nystra::NystraBias* bias);
+unsigned int take_fault_word_qkvs_bf16(cudaError_t* err);
+unsigned int take_fault_word_qkvs_f16(cudaError_t* err);
+unsigned int take_fault_word_qkvs_bf16_s16(cudaError_t* err);
+unsigned int take_fault_word_qkvs_f16_s16(cudaError_t* err);
 unsigned int take_fault_word_qkv_bf16(cudaError_t* err);
 unsigned int take_fault_word_qkv_f16(cudaError_t* err);
 unsigned int take_fault_word_qkv_bf16_s16(cudaError_t* err);

@@ -107,7 +107,8 @@ for _name in ("swinir256-bf16", "sr720p-w8-m16-bf16", "sr720p-w16-m16-bf16", "sr
     WORKLOADS[_name + "-f16"] = WORKLOADS[_name].with_(name=_name + "-f16", factors="16")
 # The same windows given as tokens X and projection weights (fused Q/K/V projection).
 for _name in ("swinir256-bf16", "uformer-s1", "uformer-s4", "sr720p-w8-m16-bf16", "sr720p-w8-m16-f16",
-              "swinir256-bf16-relpos"):
+              "swinir256-bf16-relpos", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16", "sr720p-w32-m32-bf16",
+              "sr720p-w16-m16-bf16-relpos"):
     WORKLOADS[_name + "-qkv"] = WORKLOADS[_name].with_(name=_name + "-qkv", front="qkv")
 
 

@@ -190,8 +190,11 @@ def test_attention_bias_argument_validation(lib, args, code):
 @pytest.mark.parametrize("args,code", [
     (dict(dtype=0), nb.NYSTRA_EDTYPE),            # fp32: 16-bit I/O only
     (dict(dtype=7), nb.NYSTRA_EDTYPE),
-    (dict(N=256), nb.NYSTRA_EINVAL),              # 8x8 windows only
-    (dict(m=32), nb.NYSTRA_EINVAL),
+    (dict(N=128), nb.NYSTRA_EINVAL),              # windows of 64, 256 or 1024 tokens
+    (dict(m=32), nb.NYSTRA_EINVAL),               # m = 32 only with 32x32 windows
+    (dict(N=256, m=32), nb.NYSTRA_EINVAL),
+    (dict(N=1024, m=32, bL=8 * P), nb.NYSTRA_EINVAL),  # a score bias needs m <= 16
+    (dict(N=256, m=64), nb.NYSTRA_EINVAL),
     (dict(d=31), nb.NYSTRA_EINVAL),               # odd d_h
     (dict(d=34), nb.NYSTRA_EINVAL),               # d_h > 32
     (dict(heads=12, d=32), nb.NYSTRA_EINVAL),     # C = 384 > NYSTRA_QKV_MAX_C

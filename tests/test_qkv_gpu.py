@@ -120,7 +120,8 @@ def test_fused_projection_with_a_score_bias():
 
 
 @pytest.mark.parametrize("name", ["swinir256-bf16-qkv", "uformer-s1-qkv", "uformer-s4-qkv", "sr720p-w8-m16-f16-qkv",
-                                  "swinir256-bf16-relpos-qkv"])
+                                  "swinir256-bf16-relpos-qkv", "sr720p-w16-m16-bf16-qkv", "sr720p-w32-m16-bf16-qkv",
+                                  "sr720p-w32-m32-bf16-qkv", "sr720p-w16-m16-bf16-relpos-qkv"])
 def test_fused_workloads(name):
     """Full-size workloads in the launch configuration the benchmark times,
     checked on sampled units (first, last, strided and random)."""
@@ -231,3 +232,75 @@ def test_fused_projection_sharp_attention_is_finite(s):
     ref = oracle.nystra_attention_qkv(x, w, b, 6, 16, 6)
     fin = np.isfinite(ref).all(axis=(-2, -1))
     assert np.isfinite(out.double().numpy()[fin]).all()
+
+
+# 16x16 and 32x32 windows (the streaming structure, chunks projected in place)
+LARGE = [  # n_windows, N, heads, d_h, m, pooling, dtype, projection bias
+    (3, 256, 6, 30, 16, "segments", "bf16", True),    # SwinIR heads, C = 180
+    (5, 256, 1, 32, 8, "segments", "f16", False),     # one head, C = 32
+    (2, 256, 3, 30, 16, "patches", "bf16", True),     # square patches (4x4 of 4x4 tokens)
+    (2, 1024, 6, 30, 16, "segments", "bf16", True),
+    (2, 1024, 4, 32, 32, "segments", "bf16", True),   # m = 32: the two-warp core
+    (2, 1024, 2, 16, 16, "patches", "f16", True),     # square patches (4x4 of 8x8 tokens)
+    (1, 1024, 11, 32, 16, "segments", "bf16", True),  # C = 352, the widest
+    (3, 256, 8, 32, 16, "segments", "f16", True),     # C = 256
+    (2, 1024, 5, 6, 8, "segments", "bf16", True),     # C = 30: a partial k-step
+]
+
+
+@pytest.mark.parametrize("nw,N,heads,d,m,pool,dtype,with_b", LARGE)
+def test_fused_projection_large_windows(nw, N, heads, d, m, pool, dtype, with_b):
+    x, w, b = workloads.random_x_wqkv(nw, N, heads, d, dtype, seed=nw * 5 + N + heads + d + m, with_bias=with_b)
+    out = _run(x, w, b, heads, m, pool=pool)
+    ref = oracle.nystra_attention_qkv(x, w, b, heads, m, 6, pool)
+    err = per_unit_rel(out.double().numpy(), ref)
+    assert err.max() <= TOL[dtype], f"max rel err {err.max():.3e} at unit {int(err.argmax())}"
+
+
+@pytest.mark.parametrize("N", [256, 1024])
+def test_fused_large_windows_equal_projecting_first(N):
+    """The fused call and the unfused path (projected in fp32, rounded to bf16,
+    then nystra_attention) agree to the rounding of Q, K, V."""
+    nw, heads, d = 3, 6, 30
+    x, w, b = workloads.random_x_wqkv(nw, N, heads, d, "bf16", seed=N)
+    fused = _run(x, w, b, heads, 16).double()
+    y = (x.cuda().float() @ w.cuda().float().T + b.cuda()).bfloat16()
+    q, k, v = (y.reshape(nw, N, 3, heads, d)[:, :, i].transpose(1, 2).contiguous() for i in range(3))
+    unfused = binding.nystra(q, k, v, 16, 6).cpu().double()
+    assert per_unit_rel(fused.numpy(), unfused.numpy()).max() <= 1e-2
+
+
+@pytest.mark.parametrize("N,per_window", [(256, False), (1024, True)])
+def test_fused_large_windows_with_a_score_bias(N, per_window):
+    nw, heads, d, m = 3, 2, 30, 16
+    w_ = int(round(N ** 0.5))
+    x, w, b = workloads.random_x_wqkv(nw, N, heads, d, "bf16", seed=N + 3)
+    B = workloads.relpos_bias(w_, heads, seed=5)[None].astype(np.float32)       # [1, heads, N, N]
+    if per_window:
+        B = np.ascontiguousarray(B + np.random.default_rng(1).normal(0, 0.5, (nw, 1, N, N)).astype(np.float32))
+    pooled = binding.pool_bias(torch.from_numpy(B).cuda(), m)
+    out = _run(x, w, b, heads, m, pooled=pooled)
+    ref = oracle.nystra_attention_qkv(x, w, b, heads, m, 6, "segments",
+                                      np.broadcast_to(B.astype(np.float64), (nw, heads, N, N)))
+    err = per_unit_rel(out.double().numpy(), ref)
+    assert err.max() <= TOL["bf16"], f"max rel err {err.max():.3e}"
+
+
+def test_fused_large_windows_many_windows_and_16bit_factors():
+    """Enough windows that every team of every CTA processes several units
+    (both buffers of the double-buffered state, both task orders' steady
+    state); both factor precisions on soft inputs.  Sampled units."""
+    nw, N, heads, d, m = 600, 256, 2, 30, 16
+    x, w, b = workloads.random_x_wqkv(nw, N, heads, d, "bf16", seed=77)
+    idx = sample_units(nw * heads, 96)
+    win, head = idx // heads, idx % heads
+    uw = np.unique(win)
+    q, k, v = oracle.project_qkv(x[torch.from_numpy(uw)], w, b, heads)
+    pos = np.searchsorted(uw, win)
+    ref = oracle.nystra_attention(q[pos, head], k[pos, head], v[pos, head], m, 6)
+    for factors in ("pairs", "16"):
+        out = binding.nystra_qkv(x.cuda(), w.cuda(), heads, m, 6, b_qkv=b.cuda(), factors=factors)
+        torch.cuda.synchronize()
+        assert binding.status() == binding.NYSTRA_OK
+        got = out.reshape(nw * heads, N, d)[torch.from_numpy(idx)].cpu().double().numpy()
+        assert per_unit_rel(got, ref).max() <= TOL["bf16"], factors
