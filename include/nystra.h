@@ -22,20 +22,26 @@
  *           The library allocates no device memory per call.
  *  dtype    element type of q, k, v and out (nystra_dtype).
  *  Precision products run on the tensor cores with fp32 accumulation: 16-bit
- *           inputs enter them as they are, intermediate factors (landmarks,
- *           G_L^n, G_U^n, Y) are rounded to the I/O type, the pseudo-inverse
- *           iteration uses fp16 two-term splits (about 22 bits), and fp32 I/O
- *           splits every operand into bf16 hi + lo (three products each).
- *           Shapes outside the tensor-core paths (odd d_h or d_h > 32, N not
+ *           inputs enter them as they are; the factors computed from them
+ *           (landmarks, G_L^n, G_U^n, Y) are carried as hi + lo pairs of the
+ *           I/O type (16 significant bits in bf16; NYSTRA_FACTORS_16 rounds
+ *           them to a single 16-bit value instead); the pseudo-inverse
+ *           iteration uses fp16 two-term splits (about 22 bits) of matrices
+ *           scaled by powers of two so that none underflows; fp32 I/O splits
+ *           every operand into bf16 hi + lo (three products each).  Shapes
+ *           outside the tensor-core paths (odd d_h or d_h > 32, N not
  *           64/256/1024, m not 8/16/32/64, fp32 I/O with N != 64 or more than
  *           6 iterations, 16-bit I/O with more than 12) run in fp32 SIMT
- *           arithmetic.  The output is rounded
- *           to nearest-even.  Against a float64 evaluation the max relative
- *           Frobenius error per unit is <= 1e-4 (fp32 I/O) and <= 2e-2 (16-bit
- *           I/O) at the paper's iteration counts for logits q.k/sqrt(d_h) of
- *           standard deviation up to about 1.5.  Sharper attention makes G_A^n
- *           ill-conditioned and the method amplifies any rounding (the 16-bit
- *           tensor-core path first: it rounds landmarks to the I/O type).
+ *           arithmetic.  The output is rounded to nearest-even.  Against a
+ *           float64 evaluation the max relative Frobenius error per unit is
+ *           <= 1e-4 (fp32 I/O) and <= 2e-2 (16-bit I/O) at the paper's
+ *           iteration counts for logits q.k/sqrt(d_h) of standard deviation
+ *           up to about 1.5.  Sharper attention makes G_A^n ill-conditioned
+ *           and the method amplifies any rounding: a unit whose float64
+ *           output moves by more than the bar when its landmarks are rounded
+ *           once to 16 significant bits cannot be held to the bar by any
+ *           evaluation at that precision.  Results stay finite wherever the
+ *           float64 evaluation is.
  *  Stream   `stream` is a cudaStream_t (NULL = legacy default stream).  Calls
  *           are asynchronous: a return of NYSTRA_OK means the kernels were
  *           enqueued; results are ready when the stream is synchronised.
@@ -134,8 +140,9 @@ NYSTRA_API int nystra_attention(const void* q, const void* k, const void* v, voi
 
 /*
  * nystra_attention_ex -- nystra_attention with a choice of landmark pooling.
- * `landmarks` is a nystra_landmarks value; NYSTRA_LANDMARKS_PATCHES needs N
- * and m perfect squares with sqrt(m) dividing sqrt(N) (else NYSTRA_EINVAL).
+ * `landmarks` is a nystra_landmarks value, optionally OR-ed with
+ * NYSTRA_FACTORS_16; NYSTRA_LANDMARKS_PATCHES needs N and m perfect squares
+ * with sqrt(m) dividing sqrt(N) (else NYSTRA_EINVAL).
  * nystra_attention(...) is nystra_attention_ex(..., NYSTRA_LANDMARKS_SEGMENTS,
  * ...).  Square patches run on the tensor cores for 16-bit I/O with m = 16
  * and N in {64, 256, 1024} (even d_h <= 32), on the fp32 SIMT path otherwise.
@@ -163,7 +170,8 @@ NYSTRA_API int nystra_attention_ex(const void* q, const void* k, const void* v, 
  *           outputs (device, caller-owned, no overlap with each other or bias).
  * `landmarks` as for nystra_attention_ex.  All pointers 16-byte aligned.  Meant
  * to run once per model constant.  Returns NYSTRA_OK, NYSTRA_EINVAL (shape,
- * pointer, alignment or overlap) or NYSTRA_ELAUNCH.
+ * pointer, alignment, overlap, or a `landmarks` value with option flags),
+ * NYSTRA_ELAUNCH or NYSTRA_EDEVICE.
  */
 NYSTRA_API int nystra_pool_bias(const float* bias, int n_bias, int N, int m, int landmarks, float* bias_L,
                                 float* bias_U, float* bias_A, void* stream);
@@ -206,11 +214,13 @@ NYSTRA_API int nystra_attention_bias(const void* q, const void* k, const void* v
  *  Other arguments as nystra_attention_ex.
  * The projected Q, K, V are rounded to the I/O type before the attention, as
  * an unfused projection would store them.  Supported: 16-bit I/O (fp32 returns
- * NYSTRA_EDTYPE), N = 64, m in {8, 16} (square patches: m = 16), even
- * d_h <= 32, C <= NYSTRA_QKV_MAX_C, iters <= 12; anything else returns
- * NYSTRA_EINVAL, as do null (other than b_qkv and the bias) or not 16-byte
- * aligned pointers and an out that overlaps an input.  Returns NYSTRA_OK,
- * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.
+ * NYSTRA_EDTYPE), N in {64, 256, 1024} (8x8, 16x16, 32x32 windows), m in
+ * {8, 16} (also 32 with N = 1024, without a score bias; square patches:
+ * m = 16), even d_h <= 32, C <= NYSTRA_QKV_MAX_C, iters <= 12; anything else
+ * returns NYSTRA_EINVAL, as do null (other than b_qkv and the bias) or not
+ * 16-byte aligned pointers and an out that overlaps an input.  `landmarks`
+ * may carry NYSTRA_FACTORS_16.  Returns NYSTRA_OK, NYSTRA_EINVAL,
+ * NYSTRA_EDTYPE, NYSTRA_ELAUNCH or NYSTRA_EDEVICE.
  */
 #define NYSTRA_QKV_MAX_C 352
 NYSTRA_API int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, void* out,
@@ -243,6 +253,9 @@ NYSTRA_API int nystra_last_cuda_error(void);
  * recorded by kernels on the current device since the previous call:
  * NYSTRA_ETIMEOUT if a bounded wait gave up, else NYSTRA_OK (or
  * NYSTRA_ELAUNCH if the synchronisation itself failed).  Clears the record.
+ * The record is per device, not per stream: a timeout in a kernel still
+ * running on another stream is reported by whichever call reads the record
+ * after it is set (synchronise those streams first to attribute it).
  */
 NYSTRA_API int nystra_status(void* stream);
 
@@ -259,7 +272,8 @@ NYSTRA_API int nystra_check(void* stream);
  * After limit_ns nanoseconds of %globaltimer it gives up and records the
  * timeout exactly as a kernel would, so the next nystra_status(stream)
  * returns NYSTRA_ETIMEOUT and the context stays usable.  limit_ns must lie in
- * [1000, 1000000000] (1 us to 1 s), else NYSTRA_EINVAL; nothing is allocated.
+ * [1000, 1000000000] (1 us to 1 s), else NYSTRA_EINVAL; NYSTRA_EDEVICE without
+ * an sm_103 device; nothing is allocated.
  */
 NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stream);
 
@@ -271,9 +285,9 @@ NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stre
  * the N = 64 kernel runs, and writes fp32 values, row-major, to `dump`
  * (device memory, caller-owned, 16-byte aligned, nystra_debug_stages_size()
  * floats), regions in this order:
- *   Qbar  m x d_h      landmarks (step 1), as rounded to the I/O type
+ *   Qbar  m x d_h      landmarks (step 1), as the kernel carries them (hi + lo)
  *   Kbar  m x d_h
- *   G_L^n N x m        exp(S_L - m_L) (steps 2-3), as rounded to the I/O type
+ *   G_L^n N x m        exp(S_L - m_L) (steps 2-3), as carried (hi + lo)
  *   m_U   m            row maxima of S_U over all N keys (natural-log domain)
  *   W     m x (d_h+1)  G_U^n [V | 1_N] (step 5); column d_h is G_U^n 1_N
  *   G_A^n m x m        exp(S_A - m_U) (step 3)
@@ -284,8 +298,9 @@ NYSTRA_API int nystra_debug_wait_timeout(unsigned long long limit_ns, void* stre
  * Supported: N = 64, m in {8, 16}, even d_h <= 32 (the shapes nystra_attention
  * runs on this path: iters <= 12, and <= 6 for fp32 I/O); anything else returns
  * NYSTRA_EINVAL, as do unit outside [0, n_windows*heads), null or misaligned
- * pointers.  Asynchronous on `stream`; allocates nothing.  Returns NYSTRA_OK,
- * NYSTRA_EINVAL, NYSTRA_EDTYPE or NYSTRA_ELAUNCH.
+ * pointers (and a `landmarks` value with option flags).  Asynchronous on
+ * `stream`; allocates nothing.  Returns NYSTRA_OK, NYSTRA_EINVAL,
+ * NYSTRA_EDTYPE, NYSTRA_ELAUNCH or NYSTRA_EDEVICE.
  */
 NYSTRA_API int nystra_debug_stages(const void* q, const void* k, const void* v, int n_windows, int heads,
                                    int N, int d_h, int m, int iters, int landmarks, int dtype, long long unit,
