@@ -105,35 +105,43 @@ struct Layout {
     static constexpr size_t WPART = (size_t)TPW * DS * 2;
     static_assert(WPU == 1 || (size_t)MP * WS * 4 + MP * 4 <= 2 * (size_t)TPW * DS * 2,
                   "W partial must fit in K+V");
-    // per-group shared memory: Qbar | W | m_U | Kbar (| Y^T).  Y^T is written
-    // by the core once it has read Qbar, W and m_U for the last time, so it
-    // overlays them when no warp can write the next unit's landmarks while
-    // another still reads Y^T: with one warp per unit, or when G_L^n is
-    // recomputed (the output is followed by a group barrier before the next
-    // unit's Q lands).
-    static constexpr bool YT_OVERLAY = (WPU == 1) || !GLS;
-    static constexpr size_t QB_BYTES = LmS<T>::bytes(MP);
-    static constexpr size_t YT_BYTES = YtS<T, M>::bytes(NCOL);
-    static constexpr size_t G_QBAR = 0;
-    static constexpr size_t G_W = G_QBAR + QB_BYTES;  // fp32 MP x WS
-    static constexpr size_t G_MU = G_W + MP * WS * 4;  // m_U, log2 domain
-    static constexpr size_t G_KBAR = ((G_MU + MP * 4 + 15) / 16) * 16;
-    static constexpr size_t G_YT = YT_OVERLAY ? G_QBAR : G_KBAR + QB_BYTES;
-    static_assert(!YT_OVERLAY || YT_BYTES <= G_KBAR, "Y^T must fit over Qbar, W and m_U");
-    static constexpr size_t G_BAR = ((YT_OVERLAY ? G_KBAR + QB_BYTES : G_YT + YT_BYTES) + 15) / 16 * 16;
-    static constexpr size_t G_BAR_END = G_BAR + 16 * WPU;  // two mbarriers per token warp
     // Distributed core (CW > 1): its scratch is group memory, or, with long
     // stages (TPW >= 256), the first two token warps' K/V rows (consumed by
     // the combine before the core starts; the next unit's K and V are copied
     // after the core).
     static constexpr bool SCR_IN_STAGE = (CW > 1) && (TPW >= 256);
-    static constexpr size_t SCR_BYTES = (CW > 1 && !SCR_IN_STAGE) ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0;
+    static constexpr bool SCR_IN_GROUP = (CW > 1) && !SCR_IN_STAGE;
+    static constexpr size_t SCR_BYTES = SCR_IN_GROUP ? DistScratch<(M > 16 ? M : 32)>::BYTES : 0;
     static_assert(!SCR_IN_STAGE || (WPU >= 2 && DistScratch<(M > 16 ? M : 32)>::MAT +
                                                        DistScratch<(M > 16 ? M : 32)>::AUX <=
                                                    2 * (size_t)TPW * DS * 2),
                   "scratch must fit in two warps' K/V rows");
-    static constexpr size_t G_SCR = ((G_BAR_END + 16 + 127) / 128) * 128;
-    static constexpr size_t GROUP_BYTES = ((G_SCR + SCR_BYTES + 127) / 128) * 128;
+    static constexpr size_t QB_BYTES = LmS<T>::bytes(MP);
+    static constexpr size_t YT_BYTES = YtS<T, M>::bytes(NCOL);
+    // Per-group shared memory.  Y^T is written by the core once it has read
+    // Qbar, W and m_U for the last time, so it overlays them when no warp can
+    // write the next unit's landmarks or W while another still reads Y^T:
+    // with one warp per unit, or when G_L^n is recomputed (the output is
+    // followed by a group barrier before the next unit's Q lands); with the
+    // distributed core, whose scratch starts after every core warp has read
+    // its Qbar rows, the scratch overlays Qbar and Y^T overlays W and m_U.
+    //   one-warp core:     Qbar | W | m_U | Kbar (| Y^T) | bars
+    //   distributed core:  W | m_U | Kbar | bars | Qbar (inside the scratch)
+    static constexpr bool YT_OVERLAY = SCR_IN_GROUP || (WPU == 1) || !GLS;
+    static constexpr size_t G_W = SCR_IN_GROUP ? 0 : QB_BYTES;  // fp32 MP x WS
+    static constexpr size_t G_MU = G_W + MP * WS * 4;           // m_U, log2 domain
+    static constexpr size_t G_KBAR = ((G_MU + MP * 4 + 15) / 16) * 16;
+    static constexpr size_t G_BAR = SCR_IN_GROUP ? ((G_KBAR + QB_BYTES + 15) / 16) * 16
+                                                 : (((YT_OVERLAY ? G_KBAR + QB_BYTES : G_KBAR + QB_BYTES + YT_BYTES) +
+                                                     15) / 16) * 16;
+    static constexpr size_t G_BAR_END = G_BAR + 16 * WPU;  // two mbarriers per token warp
+    static constexpr size_t G_QBAR = SCR_IN_GROUP ? ((G_BAR_END + 16 + 127) / 128) * 128 : 0;
+    static constexpr size_t G_YT = SCR_IN_GROUP ? G_W : (YT_OVERLAY ? G_QBAR : G_KBAR + QB_BYTES);
+    static_assert(!YT_OVERLAY || YT_BYTES <= (SCR_IN_GROUP ? G_KBAR : G_KBAR - G_QBAR),
+                  "Y^T must fit over the regions it overlays");
+    static constexpr size_t G_SCR = SCR_IN_GROUP ? G_QBAR : ((G_BAR_END + 16 + 127) / 128) * 128;
+    static constexpr size_t GROUP_BYTES =
+        ((SCR_IN_GROUP ? G_QBAR + (SCR_BYTES > QB_BYTES ? SCR_BYTES : QB_BYTES) : G_SCR) + 127) / 128 * 128;
     static constexpr size_t PER_GROUP = GROUP_BYTES + WPU * WARP_BYTES;
 };
 
