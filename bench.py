@@ -67,8 +67,8 @@ UNIT = "tokens*heads/s"
 DEFAULT_WORKLOAD = "sr720p-w32-m16-bf16"
 # Reported beside a headline workload, each with its own roofline and comparator.
 EXTRA_WORKLOADS = {
-    "sr720p-w32-m16-bf16": ["sr720p-w32-m16-bf16-f16", "sr720p-w16-m16-bf16", "swinir256-bf16"],
-    "sr720p-w16-m16-bf16": ["sr720p-w16-m16-bf16-f16", "sr720p-w32-m16-bf16", "swinir256-bf16"],
+    "sr720p-w32-m16-bf16": ["sr720p-w32-m16-bf16-s16", "sr720p-w16-m16-bf16", "swinir256-bf16"],
+    "sr720p-w16-m16-bf16": ["sr720p-w16-m16-bf16-s16", "sr720p-w32-m16-bf16", "swinir256-bf16"],
 }
 
 

@@ -38,7 +38,8 @@ DEFAULT = (["tiny", "swinir256-f32", "swinir256-bf16", "uformer-s1", "uformer-s4
            + [f"sr720p-w{w}-m{m}-{dt}" for w in (8, 16, 32) for m in (8, 16, 32, 64) for dt in ("bf16", "f16")]
            + [f"{n}-{x}" for x in ("patches", "relpos")
               for n in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16")]
-           + [n for n in workloads.WORKLOADS if n.endswith("-qkv")])
+           + [n for n in workloads.WORKLOADS if n.endswith("-qkv")]
+           + [n for n in workloads.WORKLOADS if n.endswith("-s16")])
 
 
 def hbm_peak_gbs() -> tuple[float, str]:

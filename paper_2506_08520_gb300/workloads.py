@@ -104,7 +104,7 @@ for _name in ("swinir256-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16"):
 # The same inputs with the derived factors rounded to 16 bits (NYSTRA_FACTORS_16).
 for _name in ("swinir256-bf16", "sr720p-w8-m16-bf16", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16",
               "sr720p-w32-m32-bf16", "large-w16-m64", "large-w32-m32", "uformer-s1"):
-    WORKLOADS[_name + "-f16"] = WORKLOADS[_name].with_(name=_name + "-f16", factors="16")
+    WORKLOADS[_name + "-s16"] = WORKLOADS[_name].with_(name=_name + "-s16", factors="16")
 # The same windows given as tokens X and projection weights (fused Q/K/V projection).
 for _name in ("swinir256-bf16", "uformer-s1", "uformer-s4", "sr720p-w8-m16-bf16", "sr720p-w8-m16-f16",
               "swinir256-bf16-relpos", "sr720p-w16-m16-bf16", "sr720p-w32-m16-bf16", "sr720p-w32-m32-bf16",
