@@ -39,17 +39,17 @@ METRIC = "Nystrom attention tokens*heads/s"
 # for the sources of the kernel they were taken with: reported as null once any
 # of those files changes.
 MEASURED_TRAFFIC = {
-    "swinir256-bf16": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_tc.cuh", "nystra_tc_n64.cu", "ptx.cuh"],
-                       "src_hash": "0d6b9b4b0c940865", "bytes": 73_427_968},
     "sr720p-w16-m16-bf16": {"files": ["common.cuh", "nystra_team.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu",
                                       "ptx.cuh"],
-                            "src_hash": "e91802655794bad2", "bytes": 1_296_480_256},
+        "src_hash": "8e80904b0aac3611", "bytes": 1_273_993_216},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-                            "src_hash": "93de88be9dc1f252", "bytes": 1_349_584_944},
-    "swinir256-bf16-qkv": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_qkv.cuh", "nystra_qkv_bf16.cu",
-                                     "nystra_tc.cuh", "ptx.cuh"],
-                           "src_hash": "3f65ce1aaad8de7b", "bytes": 23_849_216},
+        "src_hash": "4f0cc7aee22308d1", "bytes": 1_341_827_704},
+    "large-w16-m64": {"files": ["common.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu", "nystra_team.cuh", "ptx.cuh"],
+        "src_hash": "8e80904b0aac3611", "bytes": 245_142_272},
+    "sr720p-w32-m16-bf16-qkv": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_qkv.cuh", "nystra_qkv_stream.cuh",
+                                          "nystra_qkvs_bf16.cu", "nystra_tc.cuh", "ptx.cuh"],
+        "src_hash": "0ecb2b5c71d59518", "bytes": 640_227_072},
 }
 
 
