@@ -61,7 +61,10 @@ struct DumpOffsets {
     }
 };
 
-template <typename T, int M, int NCOL, int PW>
+// RS: token order of the staged rows, as the product kernel takes it for
+// this d_h (row_step of its compile-time width), so that the dumped output
+// is the product kernel's bit for bit.
+template <typename T, int M, int NCOL, int PW, int RS>
 __global__ void __launch_bounds__(32, 1)
 nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __restrict__ v, long long unit,
                     int d, int iters, float sl2, float* __restrict__ dump) {
@@ -90,8 +93,8 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
     __syncwarp();
 
     // step 1: landmarks
-    landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
-    landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
+    landmarks_mma<T, 64, L, PW, RS>(Qs, qbar, 0, d, g, t);
+    landmarks_mma<T, 64, L, PW, RS>(Ks, kbar, 0, d, g, t);
     if constexpr (M < P::MP) {
         landmarks_zero<T>(qbar, M, P::MP, lane, 32);
         landmarks_zero<T>(kbar, M, P::MP, lane, 32);
@@ -106,14 +109,14 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
 #pragma unroll
     for (int tm = 0; tm < 4; ++tm) {
         typename Opnd<T>::DReg f[P::KTL][4];
-        gl_tile<T, M, P::KTL>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f);
+        gl_tile<T, M, P::KTL, false, RS>(Qs + mtok<RS>(tm, g) * d, kbar, d, g, t, sl2, f);
 #pragma unroll
         for (int kk = 0; kk < P::KTL; ++kk) {
             GlPark<T, M>::put(glf, (tm * P::KTL + kk) * 32 + lane, f[kk]);
 #pragma unroll
             for (int r = 0; r < (M >= 16 ? 4 : 2); ++r) {
                 const float2 x = reg_f2<T>(f[kk][r]);
-                const int row = 16 * tm + g + 8 * (r & 1), col = 16 * kk + 8 * (r >> 1) + 2 * t;
+                const int row = mtok<RS>(tm, g) + (r & 1) * mrow<RS>(), col = 16 * kk + 8 * (r >> 1) + 2 * t;
                 dump[off.gl + row * M + col] = x.x;
                 dump[off.gl + row * M + col + 1] = x.y;
             }
@@ -122,7 +125,7 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
 
     // steps 2-3, 5: S_U, m_U, W = G_U^n [V | 1]
     float mU[1][2];
-    front_su_w<T, M, NCOL, 1>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU);
+    front_su_w<T, M, NCOL, 1, false, RS>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU);
     __syncwarp();
     if (t == 0) {  // m_U is kept in the log2 domain
         if (g < M) dump[off.mu + g] = mU[0][0] * 0.69314718055994531f;
@@ -140,7 +143,7 @@ nystra_stage_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* _
     for (int i = lane; i < M * (d + 1); i += 32) dump[off.y + i] = dbg[2 * M * M + (i / (d + 1)) * NCOL + i % (d + 1)];
 
     // step 7: O = (G_L^n Y_:d) / (G_L^n Y_d)
-    output_rows<T, M, NCOL, 1, true>(glf, Qs, kbar, yT, ob, d, g, t, lane, sl2);
+    output_rows<T, M, NCOL, 1, true, false, RS>(glf, Qs, kbar, yT, ob, d, g, t, lane, sl2);
     __syncwarp();
     for (int i = lane; i < 64 * d; i += 32) dump[off.out + i] = to_f32(ob[i]);
 }
@@ -149,7 +152,8 @@ template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_stage(const void* q, const void* k, const void* v, long long unit, int d, int iters,
                          float* dump, cudaStream_t stream) {
     using P = StageLayout<T, M, NCOL>;
-    auto kern = nystra_stage_kernel<T, M, NCOL, PW>;
+    // the product kernel compiles d_h = 30 in (row_step(30)); other widths keep token order
+    auto kern = d == 30 ? nystra_stage_kernel<T, M, NCOL, PW, row_step(30)> : nystra_stage_kernel<T, M, NCOL, PW, 1>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)P::BYTES);
     if (e != cudaSuccess) return e;
     const float sl2 = 1.4426950408889634f / sqrtf((float)d);

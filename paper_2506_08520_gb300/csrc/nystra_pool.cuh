@@ -70,6 +70,7 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using P = PoolLayout<T, M, NCOL>;
     constexpr int L = 64 / M;  // tokens per landmark segment
+    constexpr int RS = row_step(DC);  // token order of the staged rows (bank-conflict-free fragment loads)
     extern __shared__ __align__(128) unsigned char smem_raw[];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int g = lane >> 2, t = lane & 3;
@@ -131,8 +132,8 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         if (lane == 0) bulk_wait_read_all();
         __syncwarp();
         // ---------------- front: landmarks (Algorithm 1 step 1) ----------------
-        landmarks_mma<T, 64, L, PW>(Qs, qbar, 0, d, g, t);
-        landmarks_mma<T, 64, L, PW>(Ks, kbar, 0, d, g, t);
+        landmarks_mma<T, 64, L, PW, RS>(Qs, qbar, 0, d, g, t);
+        landmarks_mma<T, 64, L, PW, RS>(Ks, kbar, 0, d, g, t);
         if constexpr (M < P::MP) {  // zero the padding landmark rows
             landmarks_zero<T>(qbar, M, P::MP, lane, 32);
             landmarks_zero<T>(kbar, M, P::MP, lane, 32);
@@ -142,14 +143,14 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
 #pragma unroll
         for (int tm = 0; tm < 4; ++tm) {
             typename Opnd<T>::DReg f[P::KTL][4];
-            gl_tile<T, M, P::KTL, BIAS>(Qs + (16 * tm + g) * d, kbar, d, g, t, sl2, f,
-                                        BIAS ? bLu + (16 * tm + g) * M : nullptr);
+            gl_tile<T, M, P::KTL, BIAS, RS>(Qs + mtok<RS>(tm, g) * d, kbar, d, g, t, sl2, f,
+                                            BIAS ? bLu + mtok<RS>(tm, g) * M : nullptr);
 #pragma unroll
             for (int kk = 0; kk < P::KTL; ++kk) GlPark<T, M>::put(glf, (tm * P::KTL + kk) * 32 + lane, f[kk]);
         }
         // ---------------- front: S_U, m_U, W = G_U^n [V | 1] ----------------
         float mU[1][2];
-        front_su_w<T, M, NCOL, 1, BIAS>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU, bUu, 64);
+        front_su_w<T, M, NCOL, 1, BIAS, RS>(qbar, Ks, Vs, d, g, t, sl2, mW, P::WS, mU, bUu, 64);
         // The stage is consumed: hand it to the partner's next unit.
         fence_proxy_async_smem();
         __syncwarp();
@@ -160,7 +161,7 @@ nystra_pool_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         core_warp<T, M, NCOL, false, BIAS>(qbar, kbar, mU, mW, yT, iters, sl2, g, t, nullptr, bAu);
         __syncwarp();
         // ---------------- output: O = (G_L^n Y_:d) / (G_L^n Y_d) ----------------
-        output_rows<T, M, NCOL, 1, true>(glf, Qs, kbar, yT, ob, d, g, t, lane, sl2);
+        output_rows<T, M, NCOL, 1, true, false, RS>(glf, Qs, kbar, yT, ob, d, g, t, lane, sl2);
         fence_proxy_async_smem();  // this lane's staging writes precede the bulk store
         __syncwarp();
         if (lane == 0) {

@@ -118,6 +118,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     using Lay = StreamLayout<T, M, NCOL>;
     using TL = typename Lay::TL;
     using R = typename Opnd<T>::DReg;
+    constexpr int RS = row_step(DC);  // token order of the chunk rows (bank-conflict-free fragment loads)
     constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, WS = Lay::WS,
                   NSLOT = Lay::NSLOT, L = Lay::L, LPW = Lay::LPW, NTO = NCOL / 8, MT = Lay::MT;
 
@@ -260,7 +261,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
             if (tk.c == 0)
 #pragma unroll
                 for (int mf = 0; mf < 2; ++mf) cq[mf][0][0] = cq[mf][0][1] = cq[mf][0][2] = cq[mf][0][3] = 0.f;
-            landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, cq, d, g, t);
+            landmarks_acc<T, L, LPW, PW, RS>(X0, tk.c * Lay::CH, cq, d, g, t);
             if (tk.c == Lay::NCHK - 1) {
                 // Qbar overlays the Y^T of unit k - 2: with the long core's
                 // task order (m = 32) a warp's OUT(k - 2) precedes this task
@@ -290,10 +291,10 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                     run[mt][0] = run[mt][1] = -INFINITY;
                 }
             }
-            landmarks_acc<T, L, LPW, PW>(X0, tk.c * Lay::CH, ck, d, g, t);
+            landmarks_acc<T, L, LPW, PW, RS>(X0, tk.c * Lay::CH, ck, d, g, t);
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt)
-                su_w_chunk<T, NCOL, BIAS>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M,
+                su_w_chunk<T, NCOL, BIAS, RS>(aq[mt], X0, slot_x(s, 1), d, g, t, sl2, 16 * mt + g < M,
                                           16 * mt + g + 8 < M, w[mt], run[mt][0], run[mt][1], true,
                                           BIAS ? bias.U + (size_t)bsl * M * N + (size_t)(16 * mt + g) * N +
                                                      r * TPW + tk.c * Lay::CH
@@ -336,7 +337,7 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                 }
             }
             if (!failed) {
-                output_rows<T, M, NCOL, 1, false, BIAS>(
+                output_rows<T, M, NCOL, 1, false, BIAS, RS>(
                     nullptr, X0, reinterpret_cast<const T*>(bb + Lay::B_KB), reinterpret_cast<const T*>(bb + Lay::B_YT),
                     X0, d, g, t, lane, sl2,
                     BIAS ? bias.L + (size_t)bsl * N * M + (size_t)(r * TPW + tk.c * Lay::CH) * M : nullptr);

@@ -68,6 +68,33 @@ __device__ __forceinline__ float pow2i(int e) {
     return __int_as_float((e + 127) << 23);
 }
 
+// Token order of staged rows within a 64-token chunk (rows of d_h 16-bit
+// values, contiguous).  A fragment load has lane (g, t) read word t (+ a
+// constant) of row g of an 8-row tile; row i of tile j is token ctok<RS>(j, i)
+// of the chunk: every RS-th token, tiles interleaved within groups of 8 RS
+// tokens.  With w = d_h / 2 words per row the 8 rows of a tile start 4 words
+// apart modulo 32, so the 32 lanes read 32 distinct banks, when RS = 4 for odd
+// w (d_h = 30: 15-word rows, which collide two by two in token order) and
+// RS = 2 for w = 2 mod 4; otherwise token order itself is conflict-free or no
+// order is (w = 0 mod 8).  A contraction over tokens only needs its two
+// operands in the same order, and each output row goes back to its own token,
+// so the kernels pick the order freely.  Rows g and g + 8 of a 16-row tile tm
+// are tiles 2 tm and 2 tm + 1: tokens mtok<RS>(tm, g) and that + mrow<RS>().
+constexpr int row_step(int d) { return d <= 0 ? 1 : ((d / 2) % 2 == 1 ? 4 : ((d / 2) % 4 == 2 ? 2 : 1)); }
+template <int RS>
+__device__ __forceinline__ int ctok(int j, int i) {
+    return 8 * RS * (j / RS) + (j % RS) + RS * i;
+}
+template <int RS>
+__device__ __forceinline__ int mtok(int tm, int g) {
+    return ctok<RS>(2 * tm, g);
+}
+template <int RS>
+__host__ __device__ constexpr int mrow() {
+    return RS == 1 ? 8 : 1;
+}
+static_assert(row_step(30) == 4 && row_step(28) == 2 && row_step(32) == 1 && row_step(0) == 1, "row steps");
+
 // Shared scratch of the distributed core (m = 32, 64; see dist_core): two
 // matrices of fp16 pairs (hi plane, then lo plane; rows padded to m + 8
 // halves so ldmatrix is conflict-free) and an auxiliary float area.
@@ -374,18 +401,19 @@ __device__ __forceinline__ float warp_max_f(float x) {
 // down to 2^-13 of its largest one.
 __device__ __forceinline__ int h2_exponent(float x) { return (x > 0.f && x < INFINITY) ? 10 - ilogbf(x) : 0; }
 
-// S_L for one 16-token tile of the stage (rows q0..q0+15) and its G_L^n
-// fragments (A operand of O = G_L^n Y, k = landmarks).
+// S_L for one 16-token tile of the stage and its G_L^n fragments (A operand
+// of O = G_L^n Y, k = landmarks).  q0: row g of the tile (token mtok<RS>(tm,
+// g) of its chunk); row g + 8 lies mrow<RS>() rows further on.
 // BIAS: bl points at row g of the tile in the N x M block B_L of the score
 // bias (row stride M); log2(e) B_L enters the exponent beside the scaled score.
-template <typename T, int M, int KTL, bool BIAS = false>
+template <typename T, int M, int KTL, bool BIAS = false, int RS = 1>
 __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g, int t, float sl2,
                                         typename Opnd<T>::DReg (&f)[KTL][4], const float* bl = nullptr) {
     using O = Opnd<T>;
     using R = typename O::Reg;
     constexpr int NTL = M / 8, LS = LmS<T>::LS, LO = LmS<T>::LO;
     R a[2][4];
-    const T* q1 = q0 + 8 * d;
+    const T* q1 = q0 + mrow<RS>() * d;
 #pragma unroll
     for (int kk = 0; kk < 2; ++kk) {
         const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
@@ -408,7 +436,7 @@ __device__ __forceinline__ void gl_tile(const T* q0, const T* kbar, int d, int g
 #pragma unroll
         for (int j = 0; j < NTL; ++j) {
             const float2 b0 = __ldg(reinterpret_cast<const float2*>(bl + 8 * j + 2 * t));
-            const float2 b1 = __ldg(reinterpret_cast<const float2*>(bl + 8 * M + 8 * j + 2 * t));
+            const float2 b1 = __ldg(reinterpret_cast<const float2*>(bl + mrow<RS>() * M + 8 * j + 2 * t));
             sl[j][0] = fmaf(sl[j][0], sl2, kLog2e * b0.x);
             sl[j][1] = fmaf(sl[j][1], sl2, kLog2e * b0.y);
             sl[j][2] = fmaf(sl[j][2], sl2, kLog2e * b1.x);
@@ -511,7 +539,7 @@ template <int L, int PW>
 struct Pooling {
     static constexpr int B = (L == 1) ? 1 : (L == 4) ? 2 : (L == 16) ? 4 : (L == 64) ? 8 : (L == 256) ? 16 : 0;
     static constexpr int P = PW > 0 ? PW / (B > 0 ? B : 1) : 0;  // patches per patch row
-    static_assert(PW == 0 || (B > 0 && B * B == L && PW % B == 0), "square patches must tile the window");
+    static_assert(PW == 0 || (B > 0 && B * B == L && PW % (B > 0 ? B : 1) == 0), "square patches must tile the window");
     // warp-local landmark of warp-local token tok
     static __device__ __forceinline__ int of(int tok) {
         if constexpr (PW == 0) return tok / L;
@@ -528,7 +556,7 @@ struct Pooling {
     }
 };
 
-template <typename T, int L, int LPW, int PW = 0>
+template <typename T, int L, int LPW, int PW = 0, int RS = 1>
 __device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2][(LPW + 7) / 8][4], int d, int g,
                                               int t) {
     using O = Opnd<T>;
@@ -537,26 +565,27 @@ __device__ __forceinline__ void landmarks_acc(const T* X, int tok0, float (&c)[2
     constexpr int NTJ = (LPW + 7) / 8;
     constexpr float inv = 1.f / (float)L;
 #pragma unroll
-    for (int ks = 0; ks < 4; ++ks) {  // 16 tokens per k-step
-        // A = X^T, features 16 mf + g (+8), tokens 16 ks + 2t (+1) (+8, +9)
+    for (int ks = 0; ks < 4; ++ks) {  // 16 tokens per k-step: 8-row tiles 2 ks and 2 ks + 1
+        // A = X^T, features 16 mf + g (+8); k = 8 b + 2t (+1): token ctok(2 ks + b, 2t (+1))
         R a[2][4];
 #pragma unroll
         for (int mf = 0; mf < 2; ++mf)
 #pragma unroll
             for (int r = 0; r < 4; ++r) {
                 const int f0 = 16 * mf + 8 * (r & 1) + 2 * t;
-                const R x = f0 < d ? O::ld(X + (16 * ks + 8 * (r >> 1) + g) * d + f0) : O::zero();
+                const R x = f0 < d ? O::ld(X + ctok<RS>(2 * ks + (r >> 1), g) * d + f0) : O::zero();
                 a[mf][r] = O::tr(x);
             }
-        const int tk = tok0 + 16 * ks;
-        const int jlo = Pool::tile_lo(tk), jhi = Pool::tile_hi(tk);
+        // the k-step's tokens lie in [lo, hi] of the chunk
+        const int lo = 8 * RS * ((2 * ks) / RS), hi = 8 * RS * ((2 * ks + 1) / RS) + 8 * RS - 1;
+        const int jlo = Pool::tile_lo(tok0 + lo), jhi = Pool::tile_hi(tok0 + hi - 15);
 #pragma unroll
         for (int j = 0; j < NTJ; ++j) {
             if (j < jlo || j > jhi) continue;  // warp-uniform
-            // B = P^T: tokens tk + 2t (+1) (+8, +9), landmark 8j + g
-            auto pv = [&](int tok) -> float { return (Pool::of(tok) == 8 * j + g) ? inv : 0.f; };
-            const int k0 = tk + 2 * t;
-            const R b0 = O::pk(pv(k0), pv(k0 + 1)), b1 = O::pk(pv(k0 + 8), pv(k0 + 9));
+            // B = P^T: the tokens of k = 2t (+1) (+8, +9), landmark 8j + g
+            auto pv = [&](int tok) -> float { return (Pool::of(tok0 + tok) == 8 * j + g) ? inv : 0.f; };
+            const R b0 = O::pk(pv(ctok<RS>(2 * ks, 2 * t)), pv(ctok<RS>(2 * ks, 2 * t + 1)));
+            const R b1 = O::pk(pv(ctok<RS>(2 * ks + 1, 2 * t)), pv(ctok<RS>(2 * ks + 1, 2 * t + 1)));
 #pragma unroll
             for (int mf = 0; mf < 2; ++mf) O::mma(c[mf][j], a[mf], b0, b1);
         }
@@ -586,7 +615,7 @@ __device__ __forceinline__ void landmarks_zero(T* xbar, int lo, int hi, int idx0
 }
 
 // All TPW tokens of the warp (a multiple of 64), then the store.
-template <typename T, int TPW, int L, int PW = 0>
+template <typename T, int TPW, int L, int PW = 0, int RS = 1>
 __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d, int g, int t) {
     constexpr int LPW = TPW / L, NTJ = (LPW + 7) / 8;
     float c[2][NTJ][4];
@@ -595,7 +624,7 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 #pragma unroll
         for (int j = 0; j < NTJ; ++j) c[mf][j][0] = c[mf][j][1] = c[mf][j][2] = c[mf][j][3] = 0.f;
 #pragma unroll
-    for (int ch = 0; ch < TPW / 64; ++ch) landmarks_acc<T, L, LPW, PW>(X + ch * 64 * d, ch * 64, c, d, g, t);
+    for (int ch = 0; ch < TPW / 64; ++ch) landmarks_acc<T, L, LPW, PW, RS>(X + ch * 64 * d, ch * 64, c, d, g, t);
     landmarks_put<T, LPW>(c, xbar, j0, g, t);
 }
 
@@ -614,7 +643,8 @@ __device__ __forceinline__ void landmarks_mma(const T* X, T* xbar, int j0, int d
 // column yields the denominator).
 // BIAS: bu points at the chunk's first key in row g of the m-tile in the
 // M x N block B_U of the score bias (row stride bn).
-template <typename T, int NCOL, bool BIAS = false>
+// RS: token order of the chunk's rows (n-tile nt, row i = token ctok<RS>(nt, i)).
+template <typename T, int NCOL, bool BIAS = false, int RS = 1>
 __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::DReg (&aq)[2][4], const T* Kc, const T* Vc, int d,
                                            int g, int t, float sl2, bool v0, bool v1, float (&w)[NCOL / 8][4],
                                            float& run0, float& run1, bool rescale, const float* bu = nullptr,
@@ -626,7 +656,7 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::DReg (&aq)[2]
 #pragma unroll
     for (int nt = 0; nt < 8; ++nt) {
         s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
-        const T* kr = Kc + (8 * nt + g) * d;
+        const T* kr = Kc + ctok<RS>(nt, g) * d;
 #pragma unroll
         for (int kk = 0; kk < 2; ++kk) {
             const int c0 = 16 * kk + 2 * t, c1 = c0 + 8;
@@ -638,9 +668,13 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::DReg (&aq)[2]
     if constexpr (BIAS) {  // scores in the log2 domain, bias included (rows beyond m stay unbiased)
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt) {
-            const float2 b0 = v0 ? __ldg(reinterpret_cast<const float2*>(bu + 8 * nt + 2 * t)) : make_float2(0.f, 0.f);
-            const float2 b1 = v1 ? __ldg(reinterpret_cast<const float2*>(bu + 8 * bn + 8 * nt + 2 * t))
-                                 : make_float2(0.f, 0.f);
+            // keys of columns 2t, 2t + 1 of n-tile nt
+            auto ld2 = [&](const float* p) -> float2 {
+                if constexpr (RS == 1) return __ldg(reinterpret_cast<const float2*>(p + 8 * nt + 2 * t));
+                else return make_float2(__ldg(p + ctok<RS>(nt, 2 * t)), __ldg(p + ctok<RS>(nt, 2 * t + 1)));
+            };
+            const float2 b0 = v0 ? ld2(bu) : make_float2(0.f, 0.f);
+            const float2 b1 = v1 ? ld2(bu + 8 * bn) : make_float2(0.f, 0.f);
             s[nt][0] = fmaf(s[nt][0], sl2, kLog2e * b0.x);
             s[nt][1] = fmaf(s[nt][1], sl2, kLog2e * b0.y);
             s[nt][2] = fmaf(s[nt][2], sl2, kLog2e * b1.x);
@@ -677,8 +711,8 @@ __device__ __forceinline__ void su_w_chunk(const typename Opnd<T>::DReg (&aq)[2]
 #pragma unroll
         for (int j = 0; j < NTO; ++j) {
             const int c0 = 8 * j + 2 * t;
-            const R x0 = c0 < d ? O::ld(Vc + (16 * kt + g) * d + c0) : (c0 == d ? O::one() : O::zero());
-            const R x1 = c0 < d ? O::ld(Vc + (16 * kt + 8 + g) * d + c0) : (c0 == d ? O::one() : O::zero());
+            const R x0 = c0 < d ? O::ld(Vc + ctok<RS>(2 * kt, g) * d + c0) : (c0 == d ? O::one() : O::zero());
+            const R x1 = c0 < d ? O::ld(Vc + ctok<RS>(2 * kt + 1, g) * d + c0) : (c0 == d ? O::one() : O::zero());
             O::mma(w[j], a, O::tr(x0), O::tr(x1));
         }
     }
@@ -704,7 +738,7 @@ __device__ __forceinline__ void qbar_afrag(const T* qbar, int mt, int g, int t, 
 // the row maxima (log2 domain) are returned in mU.
 // BIAS: bu is the unit's M x N block B_U of the score bias, offset to the
 // first key of Ks (row stride bn).
-template <typename T, int M, int NCOL, int NCH, bool BIAS = false>
+template <typename T, int M, int NCOL, int NCH, bool BIAS = false, int RS = 1>
 __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* Vs, int d, int g, int t, float sl2,
                                            float* dst, int ws, float (&mU)[(M + 15) / 16][2],
                                            const float* bu = nullptr, int bn = 0) {
@@ -722,7 +756,7 @@ __device__ __forceinline__ void front_su_w(const T* qbar, const T* Ks, const T* 
         float run0 = -INFINITY, run1 = -INFINITY;
 #pragma unroll 1
         for (int ch = 0; ch < NCH; ++ch)
-            su_w_chunk<T, NCOL, BIAS>(aq, Ks + ch * 64 * d, Vs + ch * 64 * d, d, g, t, sl2, v0, v1, w, run0, run1,
+            su_w_chunk<T, NCOL, BIAS, RS>(aq, Ks + ch * 64 * d, Vs + ch * 64 * d, d, g, t, sl2, v0, v1, w, run0, run1,
                                       NCH > 1, BIAS ? bu + (size_t)(16 * mt + g) * bn + ch * 64 : nullptr, bn);
         mU[mt][0] = run0;
         mU[mt][1] = run1;
@@ -1415,10 +1449,11 @@ __device__ __forceinline__ void dist_core(const T* qbar, const T* kbar, const fl
 
 // Output for one warp's NCH chunks: O = (G_L^n Y_:d) / (G_L^n Y_d) (steps
 // 5-7); G_L^n fragments come from glf (parked) or are recomputed from Qs and
-// Kbar; rows are written row-major to obase (N_w x d).
+// Kbar; rows are written row-major to obase (N_w x d), each to its own token
+// (tiles in the RS token order of the chunks).
 // BIAS (recomputed G_L^n only): bl is B_L of the score bias at the warp's
 // first token (row stride M).
-template <typename T, int M, int NCOL, int NCH, bool GLS, bool BIAS = false>
+template <typename T, int M, int NCOL, int NCH, bool GLS, bool BIAS = false, int RS = 1>
 __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, const T* kbar, const T* yT,
                                             T* obase, int d, int g, int t, int lane, float sl2,
                                             const float* bl = nullptr) {
@@ -1445,8 +1480,8 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
 #pragma unroll
                 for (int kk = 0; kk < KTL; ++kk) GlPark<T, M>::get(glf, ((ch * 4 + tm) * KTL + kk) * 32 + lane, f[kk]);
             } else {
-                gl_tile<T, M, KTL, BIAS>(Qs + (ch * 64 + 16 * tm + g) * d, kbar, d, g, t, sl2, f,
-                                         BIAS ? bl + (size_t)(ch * 64 + 16 * tm + g) * M : nullptr);
+                gl_tile<T, M, KTL, BIAS, RS>(Qs + (ch * 64 + mtok<RS>(tm, g)) * d, kbar, d, g, t, sl2, f,
+                                             BIAS ? bl + (size_t)(ch * 64 + mtok<RS>(tm, g)) * M : nullptr);
             }
             float o[NTO][4];
 #pragma unroll
@@ -1469,8 +1504,8 @@ __device__ __forceinline__ void output_rows(const uint32_t* glf, const T* Qs, co
                 }
             const float i0 = __fdividef(1.f, __shfl_sync(0xffffffffu, d0, src));
             const float i1 = __fdividef(1.f, __shfl_sync(0xffffffffu, d1, src));
-            T* o0 = obase + (ch * 64 + 16 * tm + g) * d;
-            T* o1 = o0 + 8 * d;
+            T* o0 = obase + (ch * 64 + mtok<RS>(tm, g)) * d;
+            T* o1 = o0 + mrow<RS>() * d;
 #pragma unroll
             for (int j = 0; j < NTO; ++j) {
                 const int c = 8 * j + 2 * t;
@@ -1488,8 +1523,8 @@ nystra_tc_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __re
                  T* __restrict__ out, long long n_units, int d, int iters, float sl2,
                  unsigned int* fault, int active) {
     using Lay = Layout<T, M, NCOL, TPW, WPU, GLS, CW>;
-    constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, LS = Lay::LS,
-                  WS = Lay::WS, KTL = Lay::KTL, GW = Lay::GW;
+    constexpr int N = Lay::N, NCH = Lay::NCH, MT = Lay::MT, MP = Lay::MP, WS = Lay::WS, KTL = Lay::KTL,
+                  GW = Lay::GW;
     constexpr int L = N / M;      // tokens per landmark segment (<= TPW)
     constexpr int LPW = TPW / L;  // landmarks owned by one warp
     static_assert(sizeof(T) == 2, "the grouped kernel takes 16-bit I/O (its layout assumes it)");

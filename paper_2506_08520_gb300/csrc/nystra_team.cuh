@@ -72,9 +72,9 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
     static_assert(!BIAS || M <= 16, "a score bias runs with the one-warp core");
     const int d = DC ? DC : d_in;  // d_h, a compile-time constant for the common head widths
     using Lay = TeamLayout<T, M, NCOL>;
-    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, LS = Lay::LS, WS = Lay::WS,
-                  KTL = Lay::KTL, NCOLC = NCOL;
+    constexpr int NT = Lay::NT, TPW = Lay::TPW, N = Lay::N, MP = Lay::MP, WS = Lay::WS, NCOLC = NCOL;
     constexpr int L = N / M, LPW = TPW / L;
+    constexpr int RS = row_step(DC);  // token order of the staged rows (bank-conflict-free fragment loads)
     static_assert(L <= TPW && TPW % L == 0, "segments must not straddle warps");
 
     extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -219,7 +219,7 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         const long long uk = u0 + kk * stride;
         const float* bLu =
             BIAS ? bias.L + (size_t)(bias.per_window ? uk : uk % bias.heads) * N * M + (size_t)r * TPW * M : nullptr;
-        output_rows<T, M, NCOLC, 1, false, BIAS>(nullptr, Vs, reinterpret_cast<const T*>(bb + Lay::B_KB),
+        output_rows<T, M, NCOLC, 1, false, BIAS, RS>(nullptr, Vs, reinterpret_cast<const T*>(bb + Lay::B_KB),
                                                  reinterpret_cast<const T*>(bb + Lay::B_YT), Vs, d, g, t, lane, sl2,
                                                  bLu);
         fence_proxy_async_smem();  // this lane's writes precede the bulk store
@@ -260,8 +260,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             }
         }
         // ---------------- landmarks (Algorithm 1 step 1) ----------------
-        landmarks_mma<T, TPW, L, PW>(Qs, qbar, r * LPW, d, g, t);
-        landmarks_mma<T, TPW, L, PW>(Ks, kbar, r * LPW, d, g, t);
+        landmarks_mma<T, TPW, L, PW, RS>(Qs, qbar, r * LPW, d, g, t);
+        landmarks_mma<T, TPW, L, PW, RS>(Ks, kbar, r * LPW, d, g, t);
         if (tsync_or(failed)) {
             broke = true;
             break;
@@ -271,7 +271,7 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         // ---------------- S_U, partial W_r and row maxima ----------------
         constexpr int MT = (M + 15) / 16;
         float mU[MT][2];
-        front_su_w<T, M, NCOLC, 1, BIAS>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU,
+        front_su_w<T, M, NCOLC, 1, BIAS, RS>(qbar, Ks, Vs, d, g, t, sl2, wpart, WS, mU,
                                          BIAS ? bUu + r * TPW : nullptr, N);
         if (t == 0) {
 #pragma unroll
