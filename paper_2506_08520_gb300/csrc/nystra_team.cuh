@@ -260,8 +260,25 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
             }
         }
         // ---------------- landmarks (Algorithm 1 step 1) ----------------
-        landmarks_mma<T, TPW, L, PW, RS>(Qs, qbar, r * LPW, d, g, t);
-        landmarks_mma<T, TPW, L, PW, RS>(Ks, kbar, r * LPW, d, g, t);
+        // Buffer b's Kbar was last read by the output of unit kk - 2, which
+        // every token warp ran in the previous iteration after that
+        // iteration's last barrier: the sums go to registers first, and a
+        // barrier separates those outputs from the stores.
+        {
+            constexpr int NTJ = (LPW + 7) / 8;
+            float cq[2][NTJ][4], ck[2][NTJ][4];
+#pragma unroll
+            for (int mf = 0; mf < 2; ++mf)
+#pragma unroll
+                for (int j = 0; j < NTJ; ++j)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) cq[mf][j][e] = ck[mf][j][e] = 0.f;
+            landmarks_acc<T, L, LPW, PW, RS>(Qs, 0, cq, d, g, t);
+            landmarks_acc<T, L, LPW, PW, RS>(Ks, 0, ck, d, g, t);
+            tsync();
+            landmarks_put<T, LPW>(cq, qbar, r * LPW, g, t);
+            landmarks_put<T, LPW>(ck, kbar, r * LPW, g, t);
+        }
         if (tsync_or(failed)) {
             broke = true;
             break;
