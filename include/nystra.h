@@ -229,6 +229,35 @@ NYSTRA_API int nystra_attention_qkv(const void* x, const void* w_qkv, const floa
                                     int bias_windows, int dtype, void* stream);
 
 /*
+ * nystra_project_qkv -- the projections of Eq. (1) on their own: per window,
+ * Q = X W_Q, K = X W_K, V = X W_V (+ an optional projection bias), split into
+ * heads of d_h features and written in the [n_windows, heads, N, d_h] layout
+ * nystra_attention and exact_window_attention read.  One GEMM of the
+ * n_windows * N token rows against the stacked weights on the fifth-
+ * generation tensor cores (tcgen05: operands in shared memory, fp32
+ * accumulators in tensor memory), the head split done as the accumulators
+ * are stored.  Followed by nystra_attention_ex it computes what
+ * nystra_attention_qkv computes, with Q, K and V passing through HBM.
+ *
+ * Arguments
+ *  x, w_qkv, b_qkv   as nystra_attention_qkv (tokens [n_windows, N, C],
+ *          C = heads * d_h; weights [3C, C]; fp32 bias [3C] or NULL).
+ *  q, k, v [n_windows, heads, N, d_h] outputs (device, caller-owned), each
+ *          element the fp32-accumulated dot product plus bias, rounded to
+ *          the I/O type (nearest-even).
+ * Supported: 16-bit I/O (fp32 returns NYSTRA_EDTYPE), N a multiple of 32 in
+ * [32, NYSTRA_PROJ_MAX_N], even d_h <= 32, C <= NYSTRA_PROJ_MAX_C; anything
+ * else returns NYSTRA_EINVAL, as do null (other than b_qkv) or not 16-byte
+ * aligned pointers, and outputs that overlap an input or one another.  The
+ * library allocates nothing; asynchronous on `stream`.  Returns NYSTRA_OK,
+ * NYSTRA_EINVAL, NYSTRA_EDTYPE, NYSTRA_ELAUNCH or NYSTRA_EDEVICE.
+ */
+#define NYSTRA_PROJ_MAX_C 384
+#define NYSTRA_PROJ_MAX_N 65536
+NYSTRA_API int nystra_project_qkv(const void* x, const void* w_qkv, const float* b_qkv, void* q, void* k, void* v,
+                                  int n_windows, int heads, int N, int d_h, int dtype, void* stream);
+
+/*
  * exact_window_attention -- exact softmax attention per unit, Eq. (1):
  * O = softmax(Q K^T / sqrt(d_h)) V with row-max-shifted exponentials
  * (Eq. 2).  This is the computation PnP-Nystra replaces; it serves as the

@@ -28,6 +28,7 @@ def _lm(landmarks: str, factors: str = "pairs") -> int:
     return LANDMARKS[landmarks] | FACTORS[factors]
 MAX_N, MAX_DH, MAX_M, MAX_ITERS = 1024, 64, 64, 100
 QKV_MAX_C = 352
+PROJ_MAX_C, PROJ_MAX_N = 384, 65536
 
 _DTYPE_CODE = {torch.float32: NYSTRA_F32, torch.bfloat16: NYSTRA_BF16, torch.float16: NYSTRA_F16}
 
@@ -75,6 +76,8 @@ def lib() -> ctypes.CDLL:
         L.nystra_attention_bias.restype = i
         L.nystra_attention_qkv.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i, vp]
         L.nystra_attention_qkv.restype = i
+        L.nystra_project_qkv.argtypes = [vp, vp, vp, vp, vp, vp, i, i, i, i, i, vp]
+        L.nystra_project_qkv.restype = i
         L.nystra_debug_stages.restype = i
         L.nystra_debug_stages_size.argtypes = [i, i, i]
         L.nystra_debug_stages_size.restype = ctypes.c_longlong
@@ -107,6 +110,10 @@ def nystra_attention_qkv(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iter
                          bias_A, bias_windows, dtype, stream) -> int:
     return lib().nystra_attention_qkv(x, w_qkv, b_qkv, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L,
                                       bias_U, bias_A, bias_windows, dtype, stream)
+
+
+def nystra_project_qkv(x, w_qkv, b_qkv, q, k, v, n_windows, heads, N, d_h, dtype, stream) -> int:
+    return lib().nystra_project_qkv(x, w_qkv, b_qkv, q, k, v, n_windows, heads, N, d_h, dtype, stream)
 
 
 def exact_window_attention(q, k, v, out, n_windows, heads, N, d_h, dtype, stream) -> int:
@@ -322,3 +329,41 @@ def nystra_qkv(x: torch.Tensor, w_qkv: torch.Tensor, heads: int, m: int = 16, it
     if rc != NYSTRA_OK:
         raise NystraError(rc, "nystra_attention_qkv")
     return out
+
+
+def project_qkv(x: torch.Tensor, w_qkv: torch.Tensor, heads: int, b_qkv: torch.Tensor | None = None,
+                out=None, stream=None):
+    """Q, K, V projections of tokens ``x`` ``[n_windows, N, C]`` by ``w_qkv``
+    ``[3C, C]`` (+ optional fp32 ``b_qkv`` ``[3C]``), split into heads: returns
+    ``(q, k, v)``, each ``[n_windows, heads, N, C / heads]`` in x's dtype,
+    ready for ``nystra``/``exact``.  ``out`` may give the three tensors."""
+    if x.dim() != 3 or w_qkv.dim() != 2:
+        raise ValueError("expected x [n_windows, N, C] and w_qkv [3C, C]")
+    nw, N, C = x.shape
+    if heads < 1 or C % heads:
+        raise ValueError(f"C={C} does not split into {heads} heads")
+    d = C // heads
+    if tuple(w_qkv.shape) != (3 * C, C):
+        raise ValueError(f"w_qkv must be [{3 * C}, {C}]")
+    if out is None:
+        out = tuple(torch.empty((nw, heads, N, d), dtype=x.dtype, device=x.device) for _ in range(3))
+    for t in (x, w_qkv, *out):
+        if not t.is_cuda or not t.is_contiguous() or t.dtype != x.dtype:
+            raise ValueError("x, w_qkv and the outputs must be contiguous CUDA tensors of one dtype (no CPU path)")
+    if x.dtype not in _DTYPE_CODE:
+        raise ValueError(f"unsupported dtype {x.dtype}")
+    for t in out:
+        if tuple(t.shape) != (nw, heads, N, d):
+            raise ValueError(f"outputs must be [{nw}, {heads}, {N}, {d}]")
+    bp = 0
+    if b_qkv is not None:
+        if not b_qkv.is_cuda or b_qkv.dtype != torch.float32 or not b_qkv.is_contiguous() or b_qkv.numel() != 3 * C:
+            raise ValueError(f"b_qkv must be a contiguous fp32 CUDA tensor of {3 * C} values")
+        bp = b_qkv.data_ptr()
+    q, k, v = out
+    with torch.cuda.device(x.device):
+        rc = nystra_project_qkv(x.data_ptr(), w_qkv.data_ptr(), bp, q.data_ptr(), k.data_ptr(), v.data_ptr(), nw,
+                                heads, N, d, _DTYPE_CODE[x.dtype], _stream_ptr(stream))
+    if rc != NYSTRA_OK:
+        raise NystraError(rc, "nystra_project_qkv")
+    return q, k, v

@@ -266,6 +266,34 @@ int nystra_attention_qkv(const void* x, const void* w_qkv, const float* b_qkv, v
     return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
 }
 
+int nystra_project_qkv(const void* x, const void* w_qkv, const float* b_qkv, void* q, void* k, void* v,
+                       int n_windows, int heads, int N, int d_h, int dtype, void* stream) {
+    if (dtype != NYSTRA_BF16 && dtype != NYSTRA_F16) return NYSTRA_EDTYPE;  // 16-bit I/O only
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (N < 32 || N > NYSTRA_PROJ_MAX_N || N % 32 != 0) return NYSTRA_EINVAL;
+    if (d_h < 2 || d_h > 32 || d_h % 2 != 0) return NYSTRA_EINVAL;
+    if ((long long)heads * d_h > NYSTRA_PROJ_MAX_C) return NYSTRA_EINVAL;
+    if ((long long)n_windows * heads == 0) return NYSTRA_OK;
+    if (!x || !w_qkv || !q || !k || !v) return NYSTRA_EINVAL;
+    if (!aligned16(x) || !aligned16(w_qkv) || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+        (b_qkv && !aligned16(b_qkv)))
+        return NYSTRA_EINVAL;
+    const size_t C = (size_t)heads * d_h;
+    const size_t xb = (size_t)n_windows * N * C * 2, wb = 3 * C * C * 2, bb = 3 * C * 4, ob = xb;
+    const void* outs[3] = {q, k, v};
+    for (int i = 0; i < 3; ++i) {
+        if (overlaps2(outs[i], ob, x, xb) || overlaps2(outs[i], ob, w_qkv, wb) ||
+            (b_qkv && overlaps2(outs[i], ob, b_qkv, bb)))
+            return NYSTRA_EINVAL;
+        for (int j = i + 1; j < 3; ++j)
+            if (overlaps2(outs[i], ob, outs[j], ob)) return NYSTRA_EINVAL;
+    }
+    if (!device_ok()) return NYSTRA_EDEVICE;
+    const cudaError_t e = nystra_host::launch_project_qkv(x, w_qkv, b_qkv, q, k, v, n_windows, heads, N, d_h, dtype,
+                                                          (cudaStream_t)stream);
+    return e == cudaSuccess ? NYSTRA_OK : fail_cuda(e);
+}
+
 int exact_window_attention(const void* q, const void* k, const void* v, void* out, int n_windows,
                            int heads, int N, int d_h, int dtype, void* stream) {
     int rc = check_common(q, k, v, out, n_windows, heads, N, d_h, dtype);
@@ -341,13 +369,13 @@ unsigned int take_fault_words(cudaStream_t stream, cudaError_t* err) {
     *err = cudaStreamSynchronize(stream);
     if (*err != cudaSuccess) return 0u;
     unsigned int w = 0;
-    unsigned int (*const take[16])(cudaError_t*) = {
+    unsigned int (*const take[17])(cudaError_t*) = {
         take_fault_word_tc_n64,       take_fault_word_tc_n256,       take_fault_word_tc_n1024,
         take_fault_word_tc_n64_s16,   take_fault_word_tc_n256_s16,   take_fault_word_tc_n1024_s16,
         take_fault_word_exact_tc,     take_fault_word_debug,         take_fault_word_qkv_bf16,
         take_fault_word_qkv_f16,      take_fault_word_qkv_bf16_s16,  take_fault_word_qkv_f16_s16,
         take_fault_word_qkvs_bf16,    take_fault_word_qkvs_f16,      take_fault_word_qkvs_bf16_s16,
-        take_fault_word_qkvs_f16_s16};
+        take_fault_word_qkvs_f16_s16, take_fault_word_proj};
     for (auto f : take) {
         w |= f(err);
         if (*err != cudaSuccess) return w;

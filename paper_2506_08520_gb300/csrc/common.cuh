@@ -168,6 +168,11 @@ unsigned int take_fault_word_qkv_bf16(cudaError_t* err);
 unsigned int take_fault_word_qkv_f16(cudaError_t* err);
 unsigned int take_fault_word_qkv_bf16_s16(cudaError_t* err);
 unsigned int take_fault_word_qkv_f16_s16(cudaError_t* err);
+// Q/K/V projection with the head split on the fifth-generation tensor cores
+// (project_qkv.cu): x [n_windows * N, heads * d] -> q, k, v [n_windows, heads, N, d].
+cudaError_t launch_project_qkv(const void* x, const void* w, const float* b, void* q, void* k, void* v,
+                               long long n_windows, int heads, int N, int d, int dtype, cudaStream_t stream);
+unsigned int take_fault_word_proj(cudaError_t* err);
 // Test-only stage dump of the 8x8-window tensor-core path (debug_stages.cu).
 long long debug_stages_size(int N, int d, int m);
 cudaError_t launch_debug_stages(const void* q, const void* k, const void* v, long long unit, int d, int m,

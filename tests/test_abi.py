@@ -29,7 +29,8 @@ def test_header_declares_the_boundary():
     for required in ("nystra_attention", "exact_window_attention", "nystra_strerror",
                      "nystra_version", "nystra_status", "nystra_check", "nystra_last_cuda_error",
                      "nystra_debug_wait_timeout", "nystra_debug_stages", "nystra_debug_stages_size",
-                     "nystra_attention_ex", "nystra_pool_bias", "nystra_attention_bias", "nystra_attention_qkv"):
+                     "nystra_attention_ex", "nystra_pool_bias", "nystra_attention_bias", "nystra_attention_qkv",
+                     "nystra_project_qkv"):
         assert required in names
 
 
@@ -224,6 +225,38 @@ def test_attention_qkv_argument_validation(lib, args, code):
 def test_qkv_max_width_matches_the_header():
     text = open(HEADER).read()
     assert f"#define NYSTRA_QKV_MAX_C {nb.QKV_MAX_C}" in text
+    assert f"#define NYSTRA_PROJ_MAX_C {nb.PROJ_MAX_C}" in text
+    assert f"#define NYSTRA_PROJ_MAX_N {nb.PROJ_MAX_N}" in text
+
+
+@pytest.mark.parametrize("args,code", [
+    (dict(dtype=0), nb.NYSTRA_EDTYPE),            # fp32: 16-bit I/O only
+    (dict(dtype=7), nb.NYSTRA_EDTYPE),
+    (dict(N=48), nb.NYSTRA_EINVAL),               # not a multiple of 32
+    (dict(N=0), nb.NYSTRA_EINVAL),
+    (dict(N=65536 + 32), nb.NYSTRA_EINVAL),
+    (dict(d=31), nb.NYSTRA_EINVAL),               # odd d_h
+    (dict(d=34), nb.NYSTRA_EINVAL),               # d_h > 32
+    (dict(heads=13, d=30), nb.NYSTRA_EINVAL),     # C = 390 > NYSTRA_PROJ_MAX_C
+    (dict(nw=-1), nb.NYSTRA_EINVAL),
+    (dict(x=0), nb.NYSTRA_EINVAL),
+    (dict(vv=0), nb.NYSTRA_EINVAL),
+    (dict(w=2 * P + 4), nb.NYSTRA_EINVAL),        # misaligned
+    (dict(b=3 * P + 8), nb.NYSTRA_EINVAL),
+    (dict(q=P + 64), nb.NYSTRA_EINVAL),           # q overlaps x
+    (dict(k=64 * P + 4096), nb.NYSTRA_EINVAL),    # k overlaps q
+    (dict(v=3 * P), nb.NYSTRA_EINVAL),            # v overlaps the bias
+    (dict(nw=0), nb.NYSTRA_OK),                   # empty: no-op
+    (dict(heads=0), nb.NYSTRA_OK),
+])
+def test_project_qkv_argument_validation(lib, args, code):
+    a = dict(x=P, w=2 * P, b=3 * P, q=64 * P, k=96 * P, vv=128 * P, nw=4, heads=6, N=64, d=30, dtype=1)
+    if "v" in args:
+        args = dict(args, vv=args.pop("v"))
+    a.update(args)
+    rc = nb.nystra_project_qkv(a["x"], a["w"], a["b"], a["q"], a["k"], a["vv"], a["nw"], a["heads"], a["N"], a["d"],
+                               a["dtype"], None)
+    assert rc == code
 
 
 @pytest.mark.parametrize("lm,m,nw,code", [
@@ -260,6 +293,7 @@ def test_valid_calls_without_an_sm103_device_return_edevice(lib):
     assert nb.nystra_pool_bias(P, 1, 64, 16, 0, 2 * P, 3 * P, 4 * P, None) == nb.NYSTRA_EDEVICE
     assert nb.nystra_attention_qkv(P, 2 * P, 0, 64 * P, 4, 2, 64, 30, 16, 6, 0, 0, 0, 0, 0, 1,
                                    None) == nb.NYSTRA_EDEVICE
+    assert nb.nystra_project_qkv(P, 2 * P, 0, 64 * P, 96 * P, 128 * P, 4, 2, 64, 30, 1, None) == nb.NYSTRA_EDEVICE
     assert nb.nystra_debug_stages(P, 2 * P, 3 * P, 4, 2, 64, 30, 16, 6, 0, 1, 0, 4 * P, None) == nb.NYSTRA_EDEVICE
     assert nb.lib().nystra_debug_wait_timeout(10_000, None) == nb.NYSTRA_EDEVICE
     assert nb.strerror(nb.NYSTRA_EDEVICE) == "unsupported device (sm_103 required)"
