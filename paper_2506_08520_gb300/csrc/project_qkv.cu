@@ -11,27 +11,29 @@
 // of the accumulator.
 //
 // CTA (one per SM, head-group stationary): the head group's weights B
-// [96 HB, K] are staged once in shared memory (K-major core matrices); tiles
-// of 128 token rows stream through a ring of NS k-blocks of 64 columns.
-//   warps 0-3  epilogue: warp e reads TMEM lanes 32e..32e+31 (token rows),
-//              adds the bias, rounds to the I/O type and bulk-stores each
-//              (head, part) block of 32 rows x d_h (one contiguous run of the
-//              head-split output) from a two-slot staging area;
+// [96 HB, K] are staged once in shared memory (K-major core matrices).  A
+// tile of 128 token rows is 128 C contiguous 16-bit values in HBM, so one
+// 1-D bulk copy brings it into a row-major staging buffer (two buffers where
+// they fit); the rows are C values long (360 bytes at C = 180, not 16-byte
+// aligned, so neither a tensor-map copy nor the MMA can take them as they
+// are), and the loader warps rewrite each k-block of 64 columns into a ring
+// stage in the core-matrix layout the MMA reads.
+//   warps 0-3  epilogue: warp e reads TMEM lanes 32e..32e+31 (token rows)
+//              one (head, part) block of 32 columns at a time, adds the bias,
+//              rounds to the I/O type into a private slot (32 rows x d_h, the
+//              contiguous run of the head-split output those rows form) and
+//              copies the slot out with coalesced 16-byte stores;
 //   warp 4     allocates TMEM (two accumulators of 96 HB fp32 columns); lane 0
 //              issues tcgen05.mma (M = 128, N = 96 HB, K = 16) and commits
 //              each k-block to the ring's "empty" barrier and each tile to an
 //              accumulator's "full" barrier;
-//   warps 5-8  loaders: X rows are C 16-bit values (360 bytes at C = 180, not
-//              16-byte aligned, so no tensor-map copy can move them); each
-//              k-block goes in as 8-byte (or 4-byte) cp.async granules placed
-//              in the core-matrix layout, completed by cp.async.wait_group,
-//              made visible to the tensor cores by a proxy fence, then
-//              signalled on the stage's "full" barrier.
-// Ring stage s always holds k-block s mod KB (NS is a multiple of KB), so the
-// zero padding beyond C is written once.  Every mbarrier wait is bounded
-// (2 s); on expiry a warp records the fault and leaves its loop, the others
-// follow at their next bounded wait, and the MMA thread drains its MMAs
-// before TMEM is freed.
+//   warps 5-8  loaders: thread 0 issues the tile's bulk copy; all rewrite the
+//              staged rows k-block by k-block (8-byte pieces when C % 4 == 0,
+//              else 4-byte; zeros beyond C), fence them for the tensor cores
+//              and signal the stage's "full" barrier.
+// Every mbarrier wait is bounded (2 s); on expiry a warp records the fault
+// and leaves its loop, the others follow at their next bounded wait, and the
+// MMA thread drains its MMAs before TMEM is freed.
 #include <atomic>
 
 #include "common.cuh"
@@ -47,19 +49,20 @@ namespace proj {
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr int BM = 128, KBLK = 64, STAGE = BM * KBLK * 2, HEAD_COLS = 96;
 constexpr int EPI = 4, MMAW = 4, LOAD0 = 5, WARPS = 9, THREADS = WARPS * 32, LOADERS = 4 * 32;
-constexpr int SLOT = 2048;  // one (head, part) block of 32 rows x d_h <= 32 16-bit values
-constexpr int LAG = 3;      // k-blocks a loader keeps in flight before signalling the oldest
+constexpr int ESLOT = 32 * 32 * 2;  // an epilogue warp's block of 32 rows x d_h <= 32 16-bit values
+constexpr int kSmemMax = 232448 - 1024;
+constexpr int kBarLoad = 1;  // named barrier of the loader warps
 
 struct Geo {
-    int C, heads, d, N, HB, NHG, KB, NS, KSTEPS, NTILE, KP;
+    int C, heads, d, N, HB, NHG, KB, NS, SD, KSTEPS, NTILE, KP, XT;
     long long T, n_tiles;
     // shared-memory offsets (bytes from the 1024-aligned base)
-    int oB, oA, oStage, oBias, oBar, oTmem, bytes;
+    int oB, oX, oA, oE, oBias, oBar, oTmem, bytes;
 };
 
 __host__ __device__ inline int align_up(int x, int a) { return (x + a - 1) / a * a; }
 
-__host__ inline Geo geometry(int C, int heads, int d, int N, long long T, int HB) {
+__host__ inline Geo geometry(int C, int heads, int d, int N, long long T, int HB, int SD, int NS) {
     Geo g{};
     g.C = C;
     g.heads = heads;
@@ -67,20 +70,38 @@ __host__ inline Geo geometry(int C, int heads, int d, int N, long long T, int HB
     g.N = N;
     g.T = T;
     g.HB = HB;
+    g.SD = SD;
+    g.NS = NS;
     g.NHG = (heads + HB - 1) / HB;
     g.KB = (C + KBLK - 1) / KBLK;
-    g.NS = g.KB * (6 / g.KB);
     g.KSTEPS = (C + 15) / 16;
     g.NTILE = HEAD_COLS * HB;
     g.KP = g.KB * KBLK;
+    g.XT = align_up(BM * C * 2, 128);  // one staged tile of token rows
     g.n_tiles = (T + BM - 1) / BM;
     g.oB = 0;
-    g.oA = align_up(g.NTILE * g.KP * 2, 1024);
-    g.oStage = g.oA + g.NS * STAGE;
-    g.oBias = g.oStage + EPI * 2 * SLOT;
+    g.oX = align_up(g.NTILE * g.KP * 2, 1024);
+    g.oA = g.oX + SD * g.XT;
+    g.oE = g.oA + NS * STAGE;
+    g.oBias = g.oE + EPI * ESLOT;
     g.oBar = align_up(g.oBias + g.NTILE * 4, 16);
-    g.oTmem = g.oBar + (2 * g.NS + 5) * 8;
+    g.oTmem = g.oBar + (2 * NS + SD + 5) * 8;
     g.bytes = align_up(g.oTmem + 16, 128);
+    return g;
+}
+
+// The largest configuration that fits: two staging buffers, two heads per
+// CTA and a four-deep ring where possible, in that order of preference.
+__host__ inline Geo fit(int C, int heads, int d, int N, long long T) {
+    const int cand[9][3] = {{2, 2, 4}, {2, 2, 3}, {2, 2, 2}, {2, 1, 4}, {2, 1, 2},
+                            {1, 2, 4}, {1, 2, 2}, {1, 1, 4}, {1, 1, 2}};  // SD, HB, NS
+    Geo g{};
+    for (const auto& c : cand) {
+        if (c[1] == 2 && heads < 2) continue;
+        g = geometry(C, heads, d, N, T, c[1], c[0], c[2]);
+        if (g.bytes <= kSmemMax) return g;
+    }
+    g.bytes = -1;
     return g;
 }
 
@@ -121,13 +142,16 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
     unsigned char* sm = smem_raw;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int C = geo.C, d = geo.d, N = geo.N, heads = geo.heads, HB = geo.HB, KB = geo.KB, NS = geo.NS;
-    const int NTILE = geo.NTILE, KCB = geo.KP / 8;
+    const int SD = geo.SD, NTILE = geo.NTILE, KCB = geo.KP / 8;
     unsigned char* sB = sm + geo.oB;
+    unsigned char* sX = sm + geo.oX;
     unsigned char* sA = sm + geo.oA;
+    unsigned char* sE = sm + geo.oE;
     float* sBias = reinterpret_cast<float*>(sm + geo.oBias);
     uint64_t* full = reinterpret_cast<uint64_t*>(sm + geo.oBar);
     uint64_t* empty = full + NS;
-    uint64_t* accf = empty + NS;
+    uint64_t* xfull = empty + NS;  // staged tile landed, per staging buffer
+    uint64_t* accf = xfull + SD;
     uint64_t* acce = accf + 2;
     uint64_t* drain = acce + 2;
     uint32_t* tslot = reinterpret_cast<uint32_t*>(sm + geo.oTmem);
@@ -141,6 +165,7 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             mbar_init(full + s, LOADERS);
             mbar_init(empty + s, 1);
         }
+        for (int b = 0; b < SD; ++b) mbar_init(xfull + b, 1);
         for (int b = 0; b < 2; ++b) {
             mbar_init(accf + b, 1);
             mbar_init(acce + b, EPI);
@@ -152,10 +177,8 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
         t5::tmem_alloc(tslot, ncols);
         t5::tmem_relinquish();
     }
-    // Zero the ring (its padding beyond C is never written again), stage the
-    // head group's weights in the core-matrix layout (zero rows for padding
-    // features and absent heads, zero columns beyond C) and its bias.
-    for (int i = tid; i < NS * STAGE / 16; i += THREADS) reinterpret_cast<uint4*>(sA)[i] = make_uint4(0, 0, 0, 0);
+    // Stage the head group's weights in the core-matrix layout (zero rows for
+    // padding features and absent heads, zero columns beyond C) and its bias.
     for (int i = tid; i < NTILE * (geo.KP / 2); i += THREADS) {
         const int n = i / (geo.KP / 2), kk = 2 * (i - n * (geo.KP / 2));
         const int hl = n / HEAD_COLS, p = (n % HEAD_COLS) / 32, f = n % 32, h = hg * HB + hl;
@@ -168,7 +191,7 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
         const int hl = n / HEAD_COLS, p = (n % HEAD_COLS) / 32, f = n % 32, h = hg * HB + hl;
         sBias[n] = (bqkv && f < d && h < heads) ? __ldg(bqkv + (size_t)p * C + (size_t)h * d + f) : 0.f;
     }
-    fence_proxy_async_smem();  // generic writes of the ring and B before the tensor cores read them
+    fence_proxy_async_smem();  // generic writes of B before the tensor cores read them
     t5::fence_before_sync();
     __syncthreads();
     t5::fence_after_sync();
@@ -177,47 +200,71 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
     if (warp >= LOAD0) {
         // ======================= loaders =======================
         const int lt = tid - LOAD0 * 32;
-        constexpr int GB = G8 ? 8 : 4, GPC = 128 / GB, RPC = 16 / GB;  // granule bytes, per core matrix, per row
-        uint32_t it = 0, done = 0;
-        bool failed = false;
-        for (long long j = slot; j < geo.n_tiles && !failed; j += P) {
+        auto issue_tile = [&](long long j, int b) {  // thread lt == 0: bulk copy of tile j into buffer b
             const long long m0 = j * BM;
+            const long long rows = geo.T - m0 < BM ? geo.T - m0 : BM;  // a multiple of 32
+            const uint32_t bytes = (uint32_t)(rows * C * 2);
+            mbar_arrive_expect_tx(xfull + b, bytes);
+            bulk_g2s(sX + b * geo.XT, x + (size_t)m0 * C, bytes, xfull + b);
+        };
+        long long j = slot;
+        uint32_t issued[2] = {0u, 0u}, landed[2] = {0u, 0u};  // copies per staging buffer (thread lt == 0)
+        if (lt == 0)
+            for (int b = 0; b < SD && j + (long long)b * P < geo.n_tiles; ++b) {
+                issue_tile(j + (long long)b * P, b);
+                ++issued[b];
+            }
+        uint32_t it = 0, a = 0;
+        bool failed = false;  // a bounded wait of this warp gave up (warp-uniform)
+        for (; j < geo.n_tiles; j += P, ++a) {
+            const int xb = (int)(a % SD);
+            if (!wait_all(xfull + xb, (a / SD) & 1u)) failed = true;
+            else if (lt == 0) ++landed[xb];
+            const unsigned char* xs = sX + xb * geo.XT;
             for (int kb = 0; kb < KB; ++kb, ++it) {
                 const int s = (int)(it % NS);
-                if (it >= (uint32_t)NS && !wait_all(empty + s, ((it / NS) - 1) & 1u)) {
-                    failed = true;
-                    if (lane == 0) atomicOr(fault, 1u);
-                    break;
-                }
+                if (!failed && it >= (uint32_t)NS && !wait_all(empty + s, ((it / NS) - 1) & 1u)) failed = true;
+                if (failed) continue;
                 unsigned char* st = sA + s * STAGE;
-                for (int g = lt; g < 16 * 8 * GPC; g += LOADERS) {
-                    const int cm = g / GPC, wg = g - cm * GPC;
-                    const int rg = cm >> 3, kc = cm & 7, row = rg * 8 + wg / RPC, piece = wg % RPC;
-                    const int kk = kb * KBLK + kc * 8 + piece * (GB / 2);
-                    if (kk < C && m0 + row < geo.T) {
-                        if constexpr (G8)
-                            t5::cp_async8(st + ((rg * 8 + kc) << 7) + ((wg / RPC) << 4) + piece * GB,
-                                          x + (size_t)(m0 + row) * C + kk);
-                        else
-                            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(smem_addr(
-                                             st + ((rg * 8 + kc) << 7) + ((wg / RPC) << 4) + piece * GB)),
-                                         "l"(x + (size_t)(m0 + row) * C + kk)
-                                         : "memory");
+                if constexpr (G8) {  // 8-byte pieces: 16 per core matrix, lanes 0-15 / 16-31 fill two
+#pragma unroll 4
+                    for (int i = 0; i < 16; ++i) {
+                        const int g = lt + LOADERS * i, cm = g >> 4, w16 = g & 15;
+                        const int row = ((cm >> 3) << 3) + (w16 >> 1), kk = kb * KBLK + ((cm & 7) << 3) + ((w16 & 1) << 2);
+                        uint2 val = make_uint2(0u, 0u);
+                        if (kk < C) val = *reinterpret_cast<const uint2*>(xs + ((size_t)row * C + kk) * 2);
+                        *reinterpret_cast<uint2*>(st + (cm << 7) + ((w16 >> 1) << 4) + ((w16 & 1) << 3)) = val;
+                    }
+                } else {  // 4-byte pieces: 32 per core matrix
+#pragma unroll 4
+                    for (int i = 0; i < 32; ++i) {
+                        const int g = lt + LOADERS * i, cm = g >> 5, w32 = g & 31;
+                        const int row = ((cm >> 3) << 3) + (w32 >> 2), kk = kb * KBLK + ((cm & 7) << 3) + ((w32 & 3) << 1);
+                        uint32_t val = 0u;
+                        if (kk < C) val = *reinterpret_cast<const uint32_t*>(xs + ((size_t)row * C + kk) * 2);
+                        *reinterpret_cast<uint32_t*>(st + (cm << 7) + ((w32 >> 2) << 4) + ((w32 & 3) << 2)) = val;
                     }
                 }
-                t5::cp_async_commit();
-                if (it >= (uint32_t)LAG) {  // k-block it - LAG has landed: hand it to the tensor cores
-                    t5::cp_async_wait<LAG>();
-                    fence_proxy_async_smem();
-                    mbar_arrive(full + (done % NS));
-                    ++done;
-                }
+                fence_proxy_async_smem();  // the rewritten stage before the tensor cores read it
+                mbar_arrive(full + s);
+            }
+            // Every loader has read staging buffer xb (the loaders leave
+            // together if any of them gave up): refill it with the tile SD ahead.
+            fence_proxy_async_smem();
+            if (named_barrier_or(kBarLoad, LOADERS, failed)) {
+                if (lt == 0) atomicOr(fault, 1u);
+                break;
+            }
+            const long long jn = j + (long long)SD * P;
+            if (lt == 0 && jn < geo.n_tiles) {
+                issue_tile(jn, xb);
+                ++issued[xb];
             }
         }
-        t5::cp_async_wait<0>();
-        fence_proxy_async_smem();
-        if (!failed)
-            for (; done < it; ++done) mbar_arrive(full + (done % NS));
+        // Fault path: copies in flight land before the CTA's memory is released.
+        if (lt == 0)
+            for (int b = 0; b < SD; ++b)
+                if (landed[b] < issued[b]) (void)mbar_wait_bounded(xfull + b, landed[b] & 1u, kWaitNs);
     } else if (warp == MMAW) {
         // ======================= MMA issue =======================
         if (lane == 0) {
@@ -262,9 +309,10 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
     } else {
         // ======================= epilogue (warp e: TMEM lanes 32e..) =======================
         const int e = warp;
-        unsigned char* stg = sm + geo.oStage + e * 2 * SLOT;
-        T* const dst_base[3] = {q, k, v};
-        uint32_t a = 0, nst = 0;
+        unsigned char* slot_e = sE + e * ESLOT;  // this warp's 32 rows x d_h of one (head, part) block
+        const int words = d / 2;                 // 32-bit words per row
+        const int chunks = 4 * d;                // 16-byte pieces of the block (32 rows x 2 d bytes)
+        uint32_t a = 0;
         for (long long j = slot; j < geo.n_tiles; j += P, ++a) {
             const int buf = (int)(a & 1);
             if (!wait_all(accf + buf, (a >> 1) & 1u)) {
@@ -278,40 +326,42 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             const int t0 = (int)(T0 - wi * N);
             for (int hl = 0; hl < HB; ++hl) {
                 const int h = hg * HB + hl;
+#pragma unroll 1
                 for (int p = 0; p < 3; ++p) {
                     uint32_t r[32];
                     const int col = buf * NTILE + hl * HEAD_COLS + p * 32;
                     t5::ld_32x32b_x32(tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)col, r);
                     t5::wait_ld();
-                    if (!valid || h >= heads) continue;  // warp-uniform
-                    unsigned char* sl = stg + (nst & 1) * SLOT;
-                    if (nst >= 2) {
-                        if (lane == 0) t5::bulk_wait_read_1();  // the slot's previous store has read it
+                    if (hl == HB - 1 && p == 2) {  // the tile's last TMEM read: release the accumulator
+                        t5::fence_before_sync();
                         __syncwarp();
+                        if (lane == 0) mbar_arrive(acce + buf);
                     }
-                    uint32_t* row = reinterpret_cast<uint32_t*>(sl) + lane * (d / 2);
+                    if (!valid || h >= heads) continue;  // warp-uniform
+                    // row `lane` of the block, rounded, into the slot (odd word
+                    // counts: conflict-free 4-byte stores)
+                    uint32_t* row = reinterpret_cast<uint32_t*>(slot_e) + lane * words;
                     const float* bs = sBias + hl * HEAD_COLS + p * 32;
 #pragma unroll
                     for (int f = 0; f < 16; ++f)
                         if (2 * f < d)
                             row[f] = Pack<T>::pk(__uint_as_float(r[2 * f]) + bs[2 * f],
                                                  __uint_as_float(r[2 * f + 1]) + bs[2 * f + 1]);
-                    fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0) {
-                        T* dst = dst_base[p] + (((size_t)wi * heads + h) * N + t0) * d;
-                        bulk_s2g(dst, sl, (uint32_t)(64 * d));
-                        bulk_commit();
+                    // the block is one contiguous run of the head-split output:
+                    // coalesced 16-byte copies out
+                    T* dstp = (p == 0 ? q : (p == 1 ? k : v)) + (((size_t)wi * heads + h) * N + t0) * d;
+                    const uint4* src4 = reinterpret_cast<const uint4*>(slot_e);
+                    uint4* dst4 = reinterpret_cast<uint4*>(dstp);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int c = lane + 32 * i;
+                        if (c < chunks) dst4[c] = src4[c];
                     }
-                    ++nst;
+                    __syncwarp();  // the slot is read before the next block overwrites it
                 }
             }
-            t5::fence_before_sync();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(acce + buf);
         }
-        if (lane == 0) bulk_wait_all();
-        __syncwarp();
     }
     t5::fence_before_sync();
     __syncthreads();
@@ -353,11 +403,6 @@ cudaError_t launch_proj_t(const void* x, const void* w, const float* b, void* q,
 }
 }  // namespace
 
-// Shared memory (bytes) the projection needs for C inputs and HB heads per CTA.
-int project_qkv_smem(int C, int heads, int HB) {
-    return nystra::proj::geometry(C, heads, 2, 64, 64, HB).bytes + 1024;
-}
-
 cudaError_t launch_project_qkv(const void* x, const void* w, const float* b, void* q, void* k, void* v,
                                long long n_windows, int heads, int N, int d, int dtype, cudaStream_t stream) {
     int dev = 0;
@@ -373,9 +418,8 @@ cudaError_t launch_project_qkv(const void* x, const void* w, const float* b, voi
         if ((e = cudaGetSymbolAddress((void**)&s_fault[dev], nystra::g_fault_proj)) != cudaSuccess) return e;
     }
     const int C = heads * d;
-    // two heads per CTA where both fit (fewer passes over X), else one
-    const int HB = (heads >= 2 && project_qkv_smem(C, heads, 2) <= 232448) ? 2 : 1;
-    const nystra::proj::Geo g = nystra::proj::geometry(C, heads, d, N, n_windows * N, HB);
+    const nystra::proj::Geo g = nystra::proj::fit(C, heads, d, N, n_windows * N);
+    if (g.bytes < 0) return cudaErrorInvalidValue;
     const bool g8 = C % 4 == 0;
     if (dtype == 1)
         return g8 ? launch_proj_t<__nv_bfloat16, true>(x, w, b, q, k, v, g, stream, s_fault[dev], sms)

@@ -14,7 +14,9 @@ one stream and is timed as one.  A workload with a relative-position bias
 pools it once (a model constant) and times the biased call.  A fused-projection
 workload ("-qkv": tokens X and W_QKV in, algorithmic bytes X + W + O) is timed
 against the unfused path it replaces: one cuBLAS projection X W_QKV^T (torch),
-the copy that splits heads, and nystra_attention.
+the copy that splits heads, and nystra_attention; and against the library's
+own two-pass path: nystra_project_qkv (the projection with the head split on
+the tcgen05 tensor cores, timed alone too) followed by nystra_attention.
 """
 from __future__ import annotations
 
@@ -101,13 +103,33 @@ def run_qkv(wl: workloads.Workload, l2_bytes: int, peak: float, reps: int = 50) 
             binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=o, landmarks=wl.landmarks,
                                   factors=wl.factors)
 
+    qkv = tuple(torch.empty(wl.shape, dtype=x.dtype, device=dev) for _ in range(3))
+
+    def project(i):
+        binding.project_qkv(sets[i][0], w, wl.heads, out=qkv)
+
+    def two_pass(i):
+        xs, o = sets[i]
+        q, k, v = binding.project_qkv(xs, w, wl.heads, out=qkv)
+        if pooled is None:
+            binding.nystra(q, k, v, wl.m, wl.iters, out=o, landmarks=wl.landmarks, factors=wl.factors)
+        else:
+            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=o, landmarks=wl.landmarks,
+                                  factors=wl.factors)
+
     t_f = _median_ms(fused, n_sets, reps)
     t_u = _median_ms(unfused, n_sets, max(10, reps // 5))
+    t_p = _median_ms(project, n_sets, reps)
+    t_2 = _median_ms(two_pass, n_sets, reps)
     tokens = wl.units * wl.N
     gbs = io / (t_f * 1e-3) / 1e9
+    proj_bytes = x.numel() * x.element_size() * 4 + w.numel() * w.element_size()  # X in, Q K V out, W
     res = {"name": wl.name, "units": wl.units, "io_MB": io / 1e6, "nystra_ms": t_f, "unfused_ms": t_u,
            "GBps": gbs, "frac_of_hbm": gbs / peak, "tokens_heads_per_s": tokens / (t_f * 1e-3),
-           "speedup_vs_unfused": t_u / t_f}
+           "speedup_vs_unfused": t_u / t_f, "project_ms": t_p,
+           "project_frac_of_hbm": proj_bytes / (t_p * 1e-3) / 1e9 / peak,
+           "project_TFLOPs": 2.0 * x.numel() * 3 * wl.C / (t_p * 1e-3) / 1e12,
+           "two_pass_ms": t_2, "speedup_vs_two_pass": t_2 / t_f}
     real = _real_tokens(wl)
     if real != tokens:
         res["real_tokens_heads_per_s"] = real / (t_f * 1e-3)
