@@ -326,18 +326,21 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             const int t0 = (int)(T0 - wi * N);
             for (int hl = 0; hl < HB; ++hl) {
                 const int h = hg * HB + hl;
-#pragma unroll 1
+                // the head's three blocks in one go: their TMEM loads overlap
+                uint32_t r[3][32];
+                const uint32_t ta = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)(buf * NTILE + hl * HEAD_COLS);
+                t5::ld_32x32b_x32(ta, r[0]);
+                t5::ld_32x32b_x32(ta + 32, r[1]);
+                t5::ld_32x32b_x32(ta + 64, r[2]);
+                t5::wait_ld();
+                if (hl == HB - 1) {  // the tile's last TMEM reads: release the accumulator
+                    t5::fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(acce + buf);
+                }
+                if (!valid || h >= heads) continue;  // warp-uniform
+#pragma unroll
                 for (int p = 0; p < 3; ++p) {
-                    uint32_t r[32];
-                    const int col = buf * NTILE + hl * HEAD_COLS + p * 32;
-                    t5::ld_32x32b_x32(tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)col, r);
-                    t5::wait_ld();
-                    if (hl == HB - 1 && p == 2) {  // the tile's last TMEM read: release the accumulator
-                        t5::fence_before_sync();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(acce + buf);
-                    }
-                    if (!valid || h >= heads) continue;  // warp-uniform
                     // row `lane` of the block, rounded, into the slot (odd word
                     // counts: conflict-free 4-byte stores)
                     uint32_t* row = reinterpret_cast<uint32_t*>(slot_e) + lane * words;
@@ -345,8 +348,8 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
 #pragma unroll
                     for (int f = 0; f < 16; ++f)
                         if (2 * f < d)
-                            row[f] = Pack<T>::pk(__uint_as_float(r[2 * f]) + bs[2 * f],
-                                                 __uint_as_float(r[2 * f + 1]) + bs[2 * f + 1]);
+                            row[f] = Pack<T>::pk(__uint_as_float(r[p][2 * f]) + bs[2 * f],
+                                                 __uint_as_float(r[p][2 * f + 1]) + bs[2 * f + 1]);
                     __syncwarp();
                     // the block is one contiguous run of the head-split output:
                     // coalesced 16-byte copies out
