@@ -18,16 +18,16 @@
 // aligned, so neither a tensor-map copy nor the MMA can take them as they
 // are), and the loader warps rewrite each k-block of 64 columns into a ring
 // stage in the core-matrix layout the MMA reads.
-//   warps 0-3  epilogue: warp e reads TMEM lanes 32e..32e+31 (token rows)
-//              one (head, part) block of 32 columns at a time, adds the bias,
+//   warps 0-7  epilogue: warp w reads TMEM lanes 32 (w mod 4) .. + 31 (token
+//              rows) of head w / 4's three blocks of 32 columns, adds the bias,
 //              rounds to the I/O type into a private slot (32 rows x d_h, the
 //              contiguous run of the head-split output those rows form) and
 //              copies the slot out with coalesced 16-byte stores;
-//   warp 4     allocates TMEM (two accumulators of 96 HB fp32 columns); lane 0
+//   warp 8     allocates TMEM (two accumulators of 96 HB fp32 columns); lane 0
 //              issues tcgen05.mma (M = 128, N = 96 HB, K = 16) and commits
 //              each k-block to the ring's "empty" barrier and each tile to an
 //              accumulator's "full" barrier;
-//   warps 5-8  loaders: thread 0 issues the tile's bulk copy; all rewrite the
+//   warps 9-12 loaders: thread 0 issues the tile's bulk copy; all rewrite the
 //              staged rows k-block by k-block (8-byte pieces when C % 4 == 0,
 //              else 4-byte; zeros beyond C), fence them for the tensor cores
 //              and signal the stage's "full" barrier.
@@ -48,7 +48,7 @@ namespace proj {
 
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr int BM = 128, KBLK = 64, STAGE = BM * KBLK * 2, HEAD_COLS = 96;
-constexpr int EPI = 4, MMAW = 4, LOAD0 = 5, WARPS = 9, THREADS = WARPS * 32, LOADERS = 4 * 32;
+constexpr int EPI = 8, MMAW = 8, LOAD0 = 9, WARPS = 13, THREADS = WARPS * 32, LOADERS = 4 * 32;
 constexpr int ESLOT = 32 * 32 * 2;  // an epilogue warp's block of 32 rows x d_h <= 32 16-bit values
 constexpr int kSmemMax = 232448 - 1024;
 constexpr int kBarLoad = 1;  // named barrier of the loader warps
@@ -111,22 +111,26 @@ __device__ __forceinline__ int cm_off(int r, int k, int kc_row) {
     return (((r >> 3) * kc_row + (k >> 3)) << 7) + ((r & 7) << 4) + ((k & 7) << 1);
 }
 
+// Two fp32 values rounded (nearest-even) to the I/O type and packed, the
+// first in the low half (the lower address).
 template <typename T>
 struct Pack;
 template <>
 struct Pack<__nv_bfloat16> {
     static constexpr bool kBF16 = true;
     static __device__ __forceinline__ uint32_t pk(float a, float b) {
-        __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-        return *reinterpret_cast<uint32_t*>(&h);
+        uint32_t r;
+        asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
+        return r;
     }
 };
 template <>
 struct Pack<__half> {
     static constexpr bool kBF16 = false;
     static __device__ __forceinline__ uint32_t pk(float a, float b) {
-        __half2 h = __floats2half2_rn(a, b);
-        return *reinterpret_cast<uint32_t*>(&h);
+        uint32_t r;
+        asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
+        return r;
     }
 };
 
@@ -208,18 +212,18 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             bulk_g2s(sX + b * geo.XT, x + (size_t)m0 * C, bytes, xfull + b);
         };
         long long j = slot;
-        uint32_t issued[2] = {0u, 0u}, landed[2] = {0u, 0u};  // copies per staging buffer (thread lt == 0)
+        uint32_t issued = 0, landed = 0;  // copies into the staging buffers, in tile order (thread lt == 0)
         if (lt == 0)
             for (int b = 0; b < SD && j + (long long)b * P < geo.n_tiles; ++b) {
                 issue_tile(j + (long long)b * P, b);
-                ++issued[b];
+                ++issued;
             }
         uint32_t it = 0, a = 0;
         bool failed = false;  // a bounded wait of this warp gave up (warp-uniform)
         for (; j < geo.n_tiles; j += P, ++a) {
             const int xb = (int)(a % SD);
             if (!wait_all(xfull + xb, (a / SD) & 1u)) failed = true;
-            else if (lt == 0) ++landed[xb];
+            else ++landed;
             const unsigned char* xs = sX + xb * geo.XT;
             for (int kb = 0; kb < KB; ++kb, ++it) {
                 const int s = (int)(it % NS);
@@ -256,15 +260,17 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
                 break;
             }
             const long long jn = j + (long long)SD * P;
-            if (lt == 0 && jn < geo.n_tiles) {
-                issue_tile(jn, xb);
-                ++issued[xb];
+            if (jn < geo.n_tiles) {
+                if (lt == 0) issue_tile(jn, xb);
+                ++issued;
             }
         }
-        // Fault path: copies in flight land before the CTA's memory is released.
+        // Fault path: copies in flight land before the CTA's memory is released
+        // (tile a' goes to buffer a' mod SD; its landing is that buffer's
+        // (a' / SD)-th phase).
         if (lt == 0)
-            for (int b = 0; b < SD; ++b)
-                if (landed[b] < issued[b]) (void)mbar_wait_bounded(xfull + b, landed[b] & 1u, kWaitNs);
+            for (uint32_t t2 = landed; t2 < issued; ++t2)
+                (void)mbar_wait_bounded(xfull + (t2 % SD), (t2 / SD) & 1u, kWaitNs);
     } else if (warp == MMAW) {
         // ======================= MMA issue =======================
         if (lane == 0) {
@@ -307,9 +313,9 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
         }
         __syncwarp();
     } else {
-        // ======================= epilogue (warp e: TMEM lanes 32e..) =======================
-        const int e = warp;
-        unsigned char* slot_e = sE + e * ESLOT;  // this warp's 32 rows x d_h of one (head, part) block
+        // ================ epilogue (warp w: TMEM lanes 32 (w mod 4).., head w / 4) ================
+        const int e = warp & 3, hl = warp >> 2;
+        unsigned char* slot_e = sE + warp * ESLOT;  // this warp's 32 rows x d_h of one (head, part) block
         const int words = d / 2;                 // 32-bit words per row
         const int chunks = 4 * d;                // 16-byte pieces of the block (32 rows x 2 d bytes)
         uint32_t a = 0;
@@ -324,7 +330,12 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             const bool valid = T0 < geo.T;
             const long long wi = T0 / N;
             const int t0 = (int)(T0 - wi * N);
-            for (int hl = 0; hl < HB; ++hl) {
+            if (hl >= HB) {  // a head group of one head: the second set of warps has no block
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acce + buf);
+                continue;
+            }
+            {
                 const int h = hg * HB + hl;
                 // the head's three blocks in one go: their TMEM loads overlap
                 uint32_t r[3][32];
@@ -333,11 +344,9 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
                 t5::ld_32x32b_x32(ta + 32, r[1]);
                 t5::ld_32x32b_x32(ta + 64, r[2]);
                 t5::wait_ld();
-                if (hl == HB - 1) {  // the tile's last TMEM reads: release the accumulator
-                    t5::fence_before_sync();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(acce + buf);
-                }
+                t5::fence_before_sync();  // this warp's TMEM reads of the tile precede the release
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acce + buf);
                 if (!valid || h >= heads) continue;  // warp-uniform
 #pragma unroll
                 for (int p = 0; p < 3; ++p) {
