@@ -28,9 +28,10 @@
 //              each k-block to the ring's "empty" barrier and each tile to an
 //              accumulator's "full" barrier;
 //   warps 9-12 loaders: thread 0 issues the tile's bulk copy; all rewrite the
-//              staged rows k-block by k-block (8-byte pieces when C % 4 == 0,
-//              else 4-byte; zeros beyond C), fence them for the tensor cores
-//              and signal the stage's "full" barrier.
+//              staged rows k-block by k-block (a 16-byte core-matrix row from
+//              two 8-byte loads when C % 4 == 0, else 4-byte pieces; zeros
+//              beyond C), fence them for the tensor cores and signal the
+//              stage's "full" barrier.
 // Every mbarrier wait is bounded (2 s); on expiry a warp records the fault
 // and leaves its loop, the others follow at their next bounded wait, and the
 // MMA thread drains its MMAs before TMEM is freed.
@@ -230,14 +231,24 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
                 if (!failed && it >= (uint32_t)NS && !wait_all(empty + s, ((it / NS) - 1) & 1u)) failed = true;
                 if (failed) continue;
                 unsigned char* st = sA + s * STAGE;
-                if constexpr (G8) {  // 8-byte pieces: 16 per core matrix, lanes 0-15 / 16-31 fill two
+                if constexpr (G8) {
+                    // one core-matrix row (8 columns, 16 bytes) per lane and step:
+                    // a quarter-warp fills one core matrix (128 contiguous
+                    // bytes), the two quarters of a half-warp take row groups
+                    // 8 rows apart, whose 360-byte-pitch rows fall in disjoint
+                    // banks (C = 180); two 8-byte loads (odd rows are only
+                    // 8-byte aligned), one 16-byte store
+                    const int wq = lt >> 3, i8 = lt & 7;  // quarter of the loader warps (0..15), row in the group
 #pragma unroll 4
-                    for (int i = 0; i < 16; ++i) {
-                        const int g = lt + LOADERS * i, cm = g >> 4, w16 = g & 15;
-                        const int row = ((cm >> 3) << 3) + (w16 >> 1), kk = kb * KBLK + ((cm & 7) << 3) + ((w16 & 1) << 2);
-                        uint2 val = make_uint2(0u, 0u);
-                        if (kk < C) val = *reinterpret_cast<const uint2*>(xs + ((size_t)row * C + kk) * 2);
-                        *reinterpret_cast<uint2*>(st + (cm << 7) + ((w16 >> 1) << 4) + ((w16 & 1) << 3)) = val;
+                    for (int i = 0; i < 8; ++i) {
+                        const int cm = i * 16 + wq, rg = cm & 15, kc = cm >> 4;
+                        const int row = (rg << 3) + i8, kk = kb * KBLK + (kc << 3);
+                        const unsigned char* src = xs + ((size_t)row * C + kk) * 2;
+                        uint2 lo = make_uint2(0u, 0u), hi = make_uint2(0u, 0u);
+                        if (kk < C) lo = *reinterpret_cast<const uint2*>(src);
+                        if (kk + 4 < C) hi = *reinterpret_cast<const uint2*>(src + 8);
+                        *reinterpret_cast<uint4*>(st + (((rg << 3) + kc) << 7) + (i8 << 4)) =
+                            make_uint4(lo.x, lo.y, hi.x, hi.y);
                     }
                 } else {  // 4-byte pieces: 32 per core matrix
 #pragma unroll 4
