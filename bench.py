@@ -41,10 +41,10 @@ METRIC = "Nystrom attention tokens*heads/s"
 MEASURED_TRAFFIC = {
     "sr720p-w16-m16-bf16": {"files": ["common.cuh", "nystra_team.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu",
                                       "ptx.cuh"],
-        "src_hash": "8e80904b0aac3611", "bytes": 1_273_993_216},
+        "src_hash": "7af52e1124a8ee7a", "bytes": 995_420_928 + 277_827_584},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-        "src_hash": "4f0cc7aee22308d1", "bytes": 1_341_827_704},
+        "src_hash": "16d68e7fa606f183", "bytes": 1_063_135_744 + 280_318_208},
     "large-w16-m64": {"files": ["common.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu", "nystra_team.cuh", "ptx.cuh"],
         "src_hash": "8e80904b0aac3611", "bytes": 245_142_272},
     "sr720p-w32-m16-bf16-qkv": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_qkv.cuh", "nystra_qkv_stream.cuh",
@@ -530,17 +530,41 @@ def run_cuda_qkv(args, wl):
     units_tokens = wl.units * wl.N
     value = shard.aggregate_rate(units_tokens, args.steps, total_ms, ws)
 
+    # the library's two-pass path: nystra_project_qkv (the projection with the
+    # head split on the tcgen05 tensor cores) into resident Q, K, V, then
+    # nystra_attention; and the projection alone
+    qkv = tuple(torch.empty(wl.shape, dtype=x.dtype, device=dev) for _ in range(3))
+
+    def project_step(i):
+        binding.project_qkv(sets[i % nsets][0], wd, wl.heads, out=qkv, stream=stream)
+
+    def two_pass_step(i):
+        xd, od = sets[i % nsets]
+        q, k, v = binding.project_qkv(xd, wd, wl.heads, out=qkv, stream=stream)
+        if pooled is None:
+            binding.nystra(q, k, v, wl.m, wl.iters, out=od, landmarks=wl.landmarks, factors=wl.factors)
+        else:
+            binding.nystra_biased(q, k, v, pooled, wl.m, wl.iters, out=od, landmarks=wl.landmarks,
+                                  factors=wl.factors)
+
     usteps = max(3, min(args.steps, 100))
-    for i in range(3):
-        unfused_step(i)
-    barrier()
+
+    def time_steps(fn):
+        for i in range(3):
+            fn(i)
+        barrier()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for i in range(usteps):
+            fn(i)
+        a1.record(stream)
+        barrier()
+        return a0.elapsed_time(a1) / usteps
+
+    unfused_ms = time_steps(unfused_step)
+    project_ms = time_steps(project_step)
+    two_pass_ms = time_steps(two_pass_step)
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for i in range(usteps):
-        unfused_step(i)
-    e1.record(stream)
-    barrier()
-    unfused_ms = e0.elapsed_time(e1) / usteps
 
     # End to end: every step copies its tokens from pinned host memory and
     # reads the output back (the weights are a resident model constant).
@@ -588,6 +612,12 @@ def run_cuda_qkv(args, wl):
                      "hbm_GBps": io_bytes / (kern_ms * 1e-3) / 1e9},
         "comparator": {"kernel": "cuBLAS projection + head split + nystra_attention", "ms_per_step": unfused_ms,
                        "value": units_tokens / (unfused_ms * 1e-3), "speedup": unfused_ms / (total_ms / args.steps)},
+        "two_pass": {"kernels": "nystra_project_qkv (tcgen05) + nystra_attention", "ms_per_step": two_pass_ms,
+                     "value": units_tokens / (two_pass_ms * 1e-3),
+                     "speedup_vs_fused": (total_ms / args.steps) / two_pass_ms,
+                     "project_ms": project_ms,
+                     "project_hbm_GBps": (4 * x.numel() * esize + w.numel() * esize) / (project_ms * 1e-3) / 1e9,
+                     "project_TFLOPs": 2.0 * x.numel() * 3 * wl.C / (project_ms * 1e-3) / 1e12},
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": x.numel() * esize,
                 "d2h_bytes_per_step": x.numel() * esize, "streams": 2},
         "gpu_launches": args.steps,
