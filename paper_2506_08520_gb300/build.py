@@ -1,8 +1,11 @@
-"""Build ``libnystra.so`` (the C-ABI CUDA library) in-tree for sm_103a.
+"""Build ``libnystra.so`` (the C-ABI CUDA library) in-tree for sm_103a, and
+``libnystra_host.so`` (the multi-core CPU path, ``host/nystra_host.c``).
 
 Each ``csrc/*.cu`` translation unit is compiled in parallel with nvcc, then
 linked into ``paper_2506_08520_gb300/libnystra.so``.  Objects go to
 ``paper_2506_08520_gb300/_build/`` (git-ignored).  Rebuilds only what changed.
+The CPU library is plain C for the host's compiler defaults (no
+machine-specific flags: the same source builds for x86-64 and Arm).
 """
 from __future__ import annotations
 
@@ -19,6 +22,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libnystra.so")
+HOST_SRC = os.path.join(PKG, "host", "nystra_host.c")
+HOST_LIB = os.path.join(PKG, "libnystra_host.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "--expt-relaxed-constexpr", "-Xcompiler", "-fPIC",
@@ -68,6 +73,23 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
     return LIB
 
 
+def build_host(verbose: bool = False) -> str:
+    """Compile the multi-core CPU path into ``libnystra_host.so``."""
+    deps = [HOST_SRC, os.path.join(INCLUDE, "nystra_host.h"), os.path.join(INCLUDE, "nystra.h")]
+    if os.path.exists(HOST_LIB) and os.path.getmtime(HOST_LIB) >= max(os.path.getmtime(f) for f in deps):
+        return HOST_LIB
+    tmp = HOST_LIB + f".tmp{os.getpid()}"
+    cmd = [os.environ.get("CC", "gcc"), "-O3", "-std=c11", "-fopenmp", "-fno-math-errno", "-fPIC", "-shared",
+           "-fvisibility=hidden", "-I", INCLUDE, "-o", tmp, HOST_SRC, "-lm"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(f"host library build failed:\n{r.stderr}")
+    os.replace(tmp, HOST_LIB)
+    if verbose:
+        print("built", HOST_LIB)
+    return HOST_LIB
+
+
 def ptxas_report(src: str) -> str:
     """Registers / spills / shared memory per kernel (``-Xptxas -v``) for one source file."""
     cmd = [_nvcc(), *ARCH, *NVCC_FLAGS, "-Xptxas", "-v", "-c", src, "-o", os.devnull]
@@ -80,3 +102,4 @@ if __name__ == "__main__":
             print(ptxas_report(s))
     else:
         build(verbose=True)
+        build_host(verbose=True)

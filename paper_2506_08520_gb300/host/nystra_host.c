@@ -1,0 +1,382 @@
+/*
+ * Multi-core CPU path of PnP-Nystra window attention (fp32), declared in
+ * include/nystra_host.h.
+ *
+ * Per (window, head) unit, Algorithm 1 in the stabilised form of Sec. 2.2,
+ * evaluated as G_L^n (Z (G_U^n [V | 1])):
+ *   1. landmarks Qbar, Kbar: means of the m segments of N/m tokens (or of
+ *      the square patches of the window);
+ *   2. S_U = s Qbar K^T (kept transposed, N x m) with the row maxima m_U over
+ *      all N keys; G_U^n = exp(S_U - m_U); W = G_U^n [V | 1] (m x (d+1));
+ *   3. A = G_A^n = exp(s Qbar Kbar^T - m_U);
+ *   4. Z_0 = A^T / (||A||_1 ||A||_inf), then `iters` steps
+ *      Z <- Z (13 I - X (15 I - X (7 I - X))) / 4 with X = A Z;
+ *   5. Y = Z W;
+ *   6. per token i: S_L = s q_i Kbar^T, G_L^n = exp(S_L - max), and
+ *      o_i = (G_L^n Y_:d) / (G_L^n Y_d).
+ * s = 1/sqrt(d).  Every inner loop runs over a contiguous landmark or feature
+ * index with no reduction carried along it (dot products accumulate one
+ * input dimension per pass over a vector of outputs), so -O3 vectorises it
+ * for the host's SIMD unit without reassociating any sum.  Units are spread
+ * over OpenMP threads; each unit runs on one thread in a fixed order.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#include "nystra_host.h"
+
+enum { MAXN = NYSTRA_MAX_N, MAXD = NYSTRA_MAX_DH, MAXM = NYSTRA_MAX_M, NBLK = 64, MAXDP = 80 };
+
+static int isqrt_exact(int n) {
+    int r = 0;
+    while ((r + 1) * (r + 1) <= n) ++r;
+    return r * r == n ? r : -1;
+}
+
+static int overlaps(const void* a, const void* b, size_t bytes) {
+    const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+    return x < y + bytes && y < x + bytes;
+}
+
+/* Per-thread scratch of one unit. */
+typedef struct {
+    float qbar[MAXM * MAXD], kbar[MAXM * MAXD];
+    float qbarT[MAXD * MAXM], kbarT[MAXD * MAXM];
+    float st[MAXN * MAXM];            /* S_U^T, then G_U^n transposed (N x m) */
+    float vp[MAXN * MAXDP];           /* [V | 1 | 0]: d + 1 columns padded to DP, a multiple of 16 */
+    float w[MAXM * MAXDP];            /* W = G_U^n [V | 1] (padded columns: zero) */
+    float a[MAXM * MAXM], z[MAXM * MAXM], x[MAXM * MAXM], t1[MAXM * MAXM], t2[MAXM * MAXM];
+    float y[MAXM * MAXDP];            /* Y = Z W */
+    float mu[MAXM];
+    float num[NBLK * MAXDP];          /* G_L^n Y for a block of tokens */
+    int seg[MAXN];                    /* landmark of each token */
+} Scratch;
+
+/* C[r x c] = A[r x n] B[n x c] (row-major), inner loop over c. */
+static void mm(const float* A, const float* B, float* C, int r, int n, int c) {
+    for (int i = 0; i < r; ++i) {
+        float* ci = C + (size_t)i * c;
+        for (int j = 0; j < c; ++j) ci[j] = 0.f;
+        for (int l = 0; l < n; ++l) {
+            const float av = A[(size_t)i * n + l];
+            const float* bl = B + (size_t)l * c;
+            for (int j = 0; j < c; ++j) ci[j] += av * bl[j];
+        }
+    }
+}
+
+/* C[r x c] (+)= A[r x n] B[n x c], all row-major with leading dimensions
+ * lda, ldb, ldc: blocks of 4 rows x 16 columns of C accumulate in registers
+ * over n (the 16 columns are one vector loop), remainders element by element. */
+static void gemm_nn(const float* A, int lda, const float* B, int ldb, float* C, int ldc, int r, int n, int c,
+                    int accumulate) {
+    int i = 0;
+    for (; i + 4 <= r; i += 4) {
+        int j = 0;
+        for (; j + 16 <= c; j += 16) {
+            float acc[4][16];
+            for (int a = 0; a < 4; ++a)
+                for (int b = 0; b < 16; ++b) acc[a][b] = accumulate ? C[(size_t)(i + a) * ldc + j + b] : 0.f;
+            for (int l = 0; l < n; ++l) {
+                const float* bl = B + (size_t)l * ldb + j;
+                const float a0 = A[(size_t)i * lda + l], a1 = A[(size_t)(i + 1) * lda + l];
+                const float a2 = A[(size_t)(i + 2) * lda + l], a3 = A[(size_t)(i + 3) * lda + l];
+                for (int b = 0; b < 16; ++b) {
+                    acc[0][b] += a0 * bl[b];
+                    acc[1][b] += a1 * bl[b];
+                    acc[2][b] += a2 * bl[b];
+                    acc[3][b] += a3 * bl[b];
+                }
+            }
+            for (int a = 0; a < 4; ++a)
+                for (int b = 0; b < 16; ++b) C[(size_t)(i + a) * ldc + j + b] = acc[a][b];
+        }
+        for (; j < c; ++j)
+            for (int a = 0; a < 4; ++a) {
+                float acc = accumulate ? C[(size_t)(i + a) * ldc + j] : 0.f;
+                for (int l = 0; l < n; ++l) acc += A[(size_t)(i + a) * lda + l] * B[(size_t)l * ldb + j];
+                C[(size_t)(i + a) * ldc + j] = acc;
+            }
+    }
+    for (; i < r; ++i)
+        for (int j = 0; j < c; ++j) {
+            float acc = accumulate ? C[(size_t)i * ldc + j] : 0.f;
+            for (int l = 0; l < n; ++l) acc += A[(size_t)i * lda + l] * B[(size_t)l * ldb + j];
+            C[(size_t)i * ldc + j] = acc;
+        }
+}
+
+/* C[r x c] = A^T B with A [n x r] and B [n x c] row-major (leading
+ * dimensions lda, ldb; C dense): 4 x 16 register blocks accumulated over n. */
+static void gemm_tn(const float* A, int lda, const float* B, int ldb, float* C, int r, int n, int c) {
+    int i = 0;
+    for (; i + 4 <= r; i += 4) {
+        int j = 0;
+        for (; j + 16 <= c; j += 16) {
+            float acc[4][16];
+            for (int a = 0; a < 4; ++a)
+                for (int b = 0; b < 16; ++b) acc[a][b] = 0.f;
+            for (int l = 0; l < n; ++l) {
+                const float* al = A + (size_t)l * lda + i;
+                const float* bl = B + (size_t)l * ldb + j;
+                for (int b = 0; b < 16; ++b) {
+                    acc[0][b] += al[0] * bl[b];
+                    acc[1][b] += al[1] * bl[b];
+                    acc[2][b] += al[2] * bl[b];
+                    acc[3][b] += al[3] * bl[b];
+                }
+            }
+            for (int a = 0; a < 4; ++a)
+                for (int b = 0; b < 16; ++b) C[(size_t)(i + a) * c + j + b] = acc[a][b];
+        }
+        for (; j < c; ++j)
+            for (int a = 0; a < 4; ++a) {
+                float acc = 0.f;
+                for (int l = 0; l < n; ++l) acc += A[(size_t)l * lda + i + a] * B[(size_t)l * ldb + j];
+                C[(size_t)(i + a) * c + j] = acc;
+            }
+    }
+    for (; i < r; ++i)
+        for (int j = 0; j < c; ++j) {
+            float acc = 0.f;
+            for (int l = 0; l < n; ++l) acc += A[(size_t)l * lda + i] * B[(size_t)l * ldb + j];
+            C[(size_t)i * c + j] = acc;
+        }
+}
+
+static void one_unit(const float* Q, const float* K, const float* V, float* O, int N, int d, int m, int iters,
+                     Scratch* S) {
+    const float s = 1.0f / sqrtf((float)d);
+    const int dp = (d + 1 + 15) / 16 * 16;  /* columns of [V | 1] padded for full register blocks */
+    /* 1. landmarks: sums over each landmark's tokens, then the mean */
+    memset(S->qbar, 0, sizeof(float) * (size_t)m * d);
+    memset(S->kbar, 0, sizeof(float) * (size_t)m * d);
+    int cnt[MAXM];
+    for (int j = 0; j < m; ++j) cnt[j] = 0;
+    for (int t = 0; t < N; ++t) {
+        const int j = S->seg[t];
+        ++cnt[j];
+        float* qb = S->qbar + (size_t)j * d;
+        float* kb = S->kbar + (size_t)j * d;
+        const float* qt = Q + (size_t)t * d;
+        const float* kt = K + (size_t)t * d;
+        for (int c = 0; c < d; ++c) {
+            qb[c] += qt[c];
+            kb[c] += kt[c];
+        }
+    }
+    for (int j = 0; j < m; ++j) {
+        const float inv = 1.0f / (float)cnt[j];
+        for (int c = 0; c < d; ++c) {
+            S->qbar[(size_t)j * d + c] *= inv;
+            S->kbar[(size_t)j * d + c] *= inv;
+            S->qbarT[(size_t)c * m + j] = S->qbar[(size_t)j * d + c];
+            S->kbarT[(size_t)c * m + j] = S->kbar[(size_t)j * d + c];
+        }
+    }
+    /* 2. S_U^T = K Qbar^T (N x m, scaled by s), the maxima over all N keys,
+     *    G_U^n, and W = G_U^n [V | 1] (the ones column: the row sums) */
+    gemm_nn(K, d, S->qbarT, m, S->st, m, N, d, m, 0);
+    for (int i = 0; i < m; ++i) S->mu[i] = -INFINITY;
+    for (int t = 0; t < N; ++t) {
+        float* row = S->st + (size_t)t * m;
+        for (int i = 0; i < m; ++i) {
+            row[i] *= s;
+            S->mu[i] = row[i] > S->mu[i] ? row[i] : S->mu[i];
+        }
+    }
+    for (int t = 0; t < N; ++t) {
+        float* row = S->st + (size_t)t * m;
+        for (int i = 0; i < m; ++i) row[i] = expf(row[i] - S->mu[i]);
+        float* vr = S->vp + (size_t)t * dp;
+        const float* vt = V + (size_t)t * d;
+        for (int c = 0; c < d; ++c) vr[c] = vt[c];
+        vr[d] = 1.f;
+        for (int c = d + 1; c < dp; ++c) vr[c] = 0.f;
+    }
+    gemm_tn(S->st, m, S->vp, dp, S->w, m, N, dp);
+    /* 3. A = exp(s Qbar Kbar^T - m_U), row-wise */
+    mm(S->qbar, S->kbarT, S->a, m, d, m);
+    for (int i = 0; i < m; ++i)
+        for (int j = 0; j < m; ++j) S->a[(size_t)i * m + j] = expf(s * S->a[(size_t)i * m + j] - S->mu[i]);
+    /* 4. Z_0 = A^T / (||A||_1 ||A||_inf), then the iteration */
+    float n1 = 0.f, ninf = 0.f;
+    for (int j = 0; j < m; ++j) {
+        float col = 0.f;
+        for (int i = 0; i < m; ++i) col += fabsf(S->a[(size_t)i * m + j]);
+        n1 = col > n1 ? col : n1;
+    }
+    for (int i = 0; i < m; ++i) {
+        float rw = 0.f;
+        for (int j = 0; j < m; ++j) rw += fabsf(S->a[(size_t)i * m + j]);
+        ninf = rw > ninf ? rw : ninf;
+    }
+    const float a0 = 1.0f / (n1 * ninf);
+    for (int i = 0; i < m; ++i)
+        for (int j = 0; j < m; ++j) S->z[(size_t)i * m + j] = a0 * S->a[(size_t)j * m + i];
+    for (int k = 0; k < iters; ++k) {
+        mm(S->a, S->z, S->x, m, m, m);                        /* X = A Z */
+        for (int e = 0; e < m * m; ++e) S->t1[e] = -S->x[e];  /* 7I - X */
+        for (int i = 0; i < m; ++i) S->t1[(size_t)i * m + i] += 7.f;
+        mm(S->x, S->t1, S->t2, m, m, m);                      /* X (7I - X) */
+        for (int e = 0; e < m * m; ++e) S->t2[e] = -S->t2[e]; /* 15I - X (7I - X) */
+        for (int i = 0; i < m; ++i) S->t2[(size_t)i * m + i] += 15.f;
+        mm(S->x, S->t2, S->t1, m, m, m);                      /* X (15I - ...) */
+        for (int e = 0; e < m * m; ++e) S->t1[e] = -S->t1[e]; /* 13I - X (...) */
+        for (int i = 0; i < m; ++i) S->t1[(size_t)i * m + i] += 13.f;
+        mm(S->z, S->t1, S->t2, m, m, m);                      /* Z (13I - ...) */
+        for (int e = 0; e < m * m; ++e) S->z[e] = 0.25f * S->t2[e];
+    }
+    /* 5. Y = Z W */
+    mm(S->z, S->w, S->y, m, m, dp);
+    /* 6. outputs: S_L = Q Kbar^T (N x m, into st), G_L^n row by row, then
+     *    (G_L^n Y) into st's room after it, divided by its last column */
+    gemm_nn(Q, d, S->kbarT, m, S->st, m, N, d, m, 0);
+    for (int t = 0; t < N; ++t) {
+        float* row = S->st + (size_t)t * m;
+        float mx = -INFINITY;
+        for (int j = 0; j < m; ++j) {
+            row[j] *= s;
+            mx = row[j] > mx ? row[j] : mx;
+        }
+        for (int j = 0; j < m; ++j) row[j] = expf(row[j] - mx);
+    }
+    float* num = S->num;
+    for (int t0 = 0; t0 < N; t0 += NBLK) {
+        const int nb = N - t0 < NBLK ? N - t0 : NBLK;
+        gemm_nn(S->st + (size_t)t0 * m, m, S->y, dp, num, dp, nb, m, dp, 0);
+        for (int t = 0; t < nb; ++t) {
+            const float inv = 1.0f / num[(size_t)t * dp + d];
+            float* ot = O + (size_t)(t0 + t) * d;
+            for (int c = 0; c < d; ++c) ot[c] = num[(size_t)t * dp + c] * inv;
+        }
+    }
+}
+
+static int threads_or_default(int threads) {
+#ifdef _OPENMP
+    return threads > 0 ? threads : omp_get_max_threads();
+#else
+    (void)threads;
+    return 1;
+#endif
+}
+
+int nystra_host_threads(void) { return threads_or_default(0); }
+
+int nystra_attention_host(const float* q, const float* k, const float* v, float* out, int n_windows, int heads,
+                          int N, int d_h, int m, int iters, int landmarks, int threads) {
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (N < 1 || N > MAXN || d_h < 1 || d_h > MAXD) return NYSTRA_EINVAL;
+    if (m < 1 || m > N || m > MAXM || N % m != 0) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
+    int wdt = 0, pgrid = 0;
+    if (landmarks == NYSTRA_LANDMARKS_PATCHES) {
+        wdt = isqrt_exact(N);
+        pgrid = isqrt_exact(m);
+        if (wdt < 0 || pgrid < 0 || wdt % pgrid != 0) return NYSTRA_EINVAL;
+    }
+    const long long units = (long long)n_windows * heads;
+    if (units == 0) return NYSTRA_OK;
+    if (!q || !k || !v || !out) return NYSTRA_EINVAL;
+    const size_t bytes = (size_t)units * N * d_h * sizeof(float);
+    if (overlaps(out, q, bytes) || overlaps(out, k, bytes) || overlaps(out, v, bytes)) return NYSTRA_EINVAL;
+    const int nt = threads_or_default(threads);
+    int status = NYSTRA_OK;
+#pragma omp parallel num_threads(nt)
+    {
+        Scratch* S = (Scratch*)malloc(sizeof(Scratch));
+        if (!S) {
+#pragma omp atomic write
+            status = NYSTRA_EINVAL;
+        } else {
+            /* landmark of each token: segments of N/m, or b x b patches of the w x w window */
+            for (int t = 0; t < N; ++t) {
+                if (landmarks == NYSTRA_LANDMARKS_SEGMENTS) {
+                    S->seg[t] = t / (N / m);
+                } else {
+                    const int b = wdt / pgrid, row = t / wdt, col = t % wdt;
+                    S->seg[t] = (row / b) * pgrid + col / b;
+                }
+            }
+#pragma omp for schedule(static)
+            for (long long u = 0; u < units; ++u) {
+                const size_t off = (size_t)u * N * d_h;
+                one_unit(q + off, k + off, v + off, out + off, N, d_h, m, iters, S);
+            }
+            free(S);
+        }
+    }
+    return status;
+}
+
+int exact_window_attention_host(const float* q, const float* k, const float* v, float* out, int n_windows,
+                                int heads, int N, int d_h, int threads) {
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (N < 1 || N > MAXN || d_h < 1 || d_h > MAXD) return NYSTRA_EINVAL;
+    const long long units = (long long)n_windows * heads;
+    if (units == 0) return NYSTRA_OK;
+    if (!q || !k || !v || !out) return NYSTRA_EINVAL;
+    const size_t bytes = (size_t)units * N * d_h * sizeof(float);
+    if (overlaps(out, q, bytes) || overlaps(out, k, bytes) || overlaps(out, v, bytes)) return NYSTRA_EINVAL;
+    const int nt = threads_or_default(threads);
+    int status = NYSTRA_OK;
+    const float s = 1.0f / sqrtf((float)d_h);
+    const int dp = (d_h + 1 + 15) / 16 * 16;  /* [V | 1] padded for full register blocks */
+#pragma omp parallel num_threads(nt)
+    {
+        /* per thread: K^T (d x N), [V | 1 | 0] (N x dp), scores and numerators of a block of queries */
+        float* kT = (float*)malloc(sizeof(float) * (size_t)MAXD * MAXN);
+        float* vp = (float*)malloc(sizeof(float) * (size_t)MAXN * MAXDP);
+        float* p = (float*)malloc(sizeof(float) * (size_t)NBLK * MAXN);
+        float* num = (float*)malloc(sizeof(float) * (size_t)NBLK * MAXDP);
+        if (!kT || !vp || !p || !num) {
+#pragma omp atomic write
+            status = NYSTRA_EINVAL;
+        } else {
+#pragma omp for schedule(static)
+            for (long long u = 0; u < units; ++u) {
+                const size_t off = (size_t)u * N * d_h;
+                const float *Q = q + off, *K = k + off, *V = v + off;
+                float* O = out + off;
+                for (int t = 0; t < N; ++t) {
+                    for (int c = 0; c < d_h; ++c) {
+                        kT[(size_t)c * N + t] = K[(size_t)t * d_h + c];
+                        vp[(size_t)t * dp + c] = V[(size_t)t * d_h + c];
+                    }
+                    vp[(size_t)t * dp + d_h] = 1.f;  /* the ones column: the softmax denominators */
+                    for (int c = d_h + 1; c < dp; ++c) vp[(size_t)t * dp + c] = 0.f;
+                }
+                for (int i0 = 0; i0 < N; i0 += NBLK) {
+                    const int nb = N - i0 < NBLK ? N - i0 : NBLK;
+                    gemm_nn(Q + (size_t)i0 * d_h, d_h, kT, N, p, N, nb, d_h, N, 0);  /* scores Q K^T */
+                    for (int i = 0; i < nb; ++i) {
+                        float* pr = p + (size_t)i * N;
+                        float mx = -INFINITY;
+                        for (int t = 0; t < N; ++t) {
+                            pr[t] *= s;
+                            mx = pr[t] > mx ? pr[t] : mx;
+                        }
+                        for (int t = 0; t < N; ++t) pr[t] = expf(pr[t] - mx);
+                    }
+                    gemm_nn(p, N, vp, dp, num, dp, nb, N, dp, 0);  /* exp(scores) [V | 1] */
+                    for (int i = 0; i < nb; ++i) {
+                        const float inv = 1.0f / num[(size_t)i * dp + d_h];
+                        for (int c = 0; c < d_h; ++c) O[(size_t)(i0 + i) * d_h + c] = num[(size_t)i * dp + c] * inv;
+                    }
+                }
+            }
+        }
+        free(kT);
+        free(vp);
+        free(p);
+        free(num);
+    }
+    return status;
+}
