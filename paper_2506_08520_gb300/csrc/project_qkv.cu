@@ -18,16 +18,16 @@
 // aligned, so neither a tensor-map copy nor the MMA can take them as they
 // are), and the loader warps rewrite each k-block of 64 columns into a ring
 // stage in the core-matrix layout the MMA reads.
-//   warps 0-7  epilogue: warp w reads TMEM lanes 32 (w mod 4) .. + 31 (token
-//              rows) of head w / 4's three blocks of 32 columns, adds the bias,
+//   warps 0-11 epilogue: warp w reads TMEM lanes 32 (w mod 4) .. + 31 (token
+//              rows) of part w / 4 (Q, K or V) of each head, adds the bias,
 //              rounds to the I/O type into a private slot (32 rows x d_h, the
 //              contiguous run of the head-split output those rows form) and
 //              copies the slot out with coalesced 16-byte stores;
-//   warp 8     allocates TMEM (two accumulators of 96 HB fp32 columns); lane 0
+//   warp 12    allocates TMEM (two accumulators of 96 HB fp32 columns); lane 0
 //              issues tcgen05.mma (M = 128, N = 96 HB, K = 16) and commits
 //              each k-block to the ring's "empty" barrier and each tile to an
 //              accumulator's "full" barrier;
-//   warps 9-12 loaders: thread 0 issues the tile's bulk copy; all rewrite the
+//   warps 13-20 loaders: thread 0 issues the tile's bulk copy; all rewrite the
 //              staged rows k-block by k-block (a 16-byte core-matrix row from
 //              two 8-byte loads when C % 4 == 0, else 4-byte pieces; zeros
 //              beyond C), fence them for the tensor cores and signal the
@@ -49,7 +49,7 @@ namespace proj {
 
 constexpr uint64_t kWaitNs = 2000000000ull;
 constexpr int BM = 128, KBLK = 64, STAGE = BM * KBLK * 2, HEAD_COLS = 96;
-constexpr int EPI = 8, MMAW = 8, LOAD0 = 9, WARPS = 13, THREADS = WARPS * 32, LOADERS = 4 * 32;
+constexpr int EPI = 12, MMAW = 12, LOAD0 = 13, WARPS = 21, THREADS = WARPS * 32, LOADERS = 8 * 32;
 constexpr int ESLOT = 32 * 32 * 2;  // an epilogue warp's block of 32 rows x d_h <= 32 16-bit values
 constexpr int kSmemMax = 232448 - 1024;
 constexpr int kBarLoad = 1;  // named barrier of the loader warps
@@ -238,10 +238,11 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
                     // 8 rows apart, whose 360-byte-pitch rows fall in disjoint
                     // banks (C = 180); two 8-byte loads (odd rows are only
                     // 8-byte aligned), one 16-byte store
-                    const int wq = lt >> 3, i8 = lt & 7;  // quarter of the loader warps (0..15), row in the group
-#pragma unroll 4
-                    for (int i = 0; i < 8; ++i) {
-                        const int cm = i * 16 + wq, rg = cm & 15, kc = cm >> 4;
+                    const int wq = lt >> 3, i8 = lt & 7;  // quarter-warp of the loaders, row in the group
+                    constexpr int QW = LOADERS / 8;       // quarter-warps of the loaders
+#pragma unroll
+                    for (int i = 0; i < 128 / QW; ++i) {
+                        const int cm = i * QW + wq, rg = cm & 15, kc = cm >> 4;
                         const int row = (rg << 3) + i8, kk = kb * KBLK + (kc << 3);
                         const unsigned char* src = xs + ((size_t)row * C + kk) * 2;
                         uint2 lo = make_uint2(0u, 0u), hi = make_uint2(0u, 0u);
@@ -252,7 +253,7 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
                     }
                 } else {  // 4-byte pieces: 32 per core matrix
 #pragma unroll 4
-                    for (int i = 0; i < 32; ++i) {
+                    for (int i = 0; i < 16 * 8 * 32 / LOADERS; ++i) {
                         const int g = lt + LOADERS * i, cm = g >> 5, w32 = g & 31;
                         const int row = ((cm >> 3) << 3) + (w32 >> 2), kk = kb * KBLK + ((cm & 7) << 3) + ((w32 & 3) << 1);
                         uint32_t val = 0u;
@@ -324,11 +325,13 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
         }
         __syncwarp();
     } else {
-        // ================ epilogue (warp w: TMEM lanes 32 (w mod 4).., head w / 4) ================
-        const int e = warp & 3, hl = warp >> 2;
+        // ============ epilogue (warp w: TMEM lanes 32 (w mod 4).., part w / 4 of each head) ============
+        const int e = warp & 3, p = warp >> 2;
         unsigned char* slot_e = sE + warp * ESLOT;  // this warp's 32 rows x d_h of one (head, part) block
-        const int words = d / 2;                 // 32-bit words per row
-        const int chunks = 4 * d;                // 16-byte pieces of the block (32 rows x 2 d bytes)
+        const int words = d / 2;                    // 32-bit words per row
+        const int chunks = 4 * d;                   // 16-byte pieces of the block (32 rows x 2 d bytes)
+        T* const dst = p == 0 ? q : (p == 1 ? k : v);
+        const bool biased = bqkv != nullptr;
         uint32_t a = 0;
         for (long long j = slot; j < geo.n_tiles; j += P, ++a) {
             const int buf = (int)(a & 1);
@@ -341,48 +344,45 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             const bool valid = T0 < geo.T;
             const long long wi = T0 / N;
             const int t0 = (int)(T0 - wi * N);
-            if (hl >= HB) {  // a head group of one head: the second set of warps has no block
-                __syncwarp();
-                if (lane == 0) mbar_arrive(acce + buf);
-                continue;
-            }
-            {
+            // part p of every head of the group in one go: the TMEM loads overlap
+            uint32_t r[2][32];
+            const uint32_t ta = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)(buf * NTILE + p * 32);
+            t5::ld_32x32b_x32(ta, r[0]);
+            if (HB == 2) t5::ld_32x32b_x32(ta + HEAD_COLS, r[1]);
+            t5::wait_ld();
+            t5::fence_before_sync();  // this warp's TMEM reads of the tile precede the release
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acce + buf);
+            if (!valid) continue;  // warp-uniform
+#pragma unroll
+            for (int hl = 0; hl < 2; ++hl) {
                 const int h = hg * HB + hl;
-                // the head's three blocks in one go: their TMEM loads overlap
-                uint32_t r[3][32];
-                const uint32_t ta = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)(buf * NTILE + hl * HEAD_COLS);
-                t5::ld_32x32b_x32(ta, r[0]);
-                t5::ld_32x32b_x32(ta + 32, r[1]);
-                t5::ld_32x32b_x32(ta + 64, r[2]);
-                t5::wait_ld();
-                t5::fence_before_sync();  // this warp's TMEM reads of the tile precede the release
-                __syncwarp();
-                if (lane == 0) mbar_arrive(acce + buf);
-                if (!valid || h >= heads) continue;  // warp-uniform
+                if (hl >= HB || h >= heads) break;  // warp-uniform
+                // row `lane` of the block, rounded, into the slot (odd word
+                // counts: conflict-free 4-byte stores)
+                uint32_t* row = reinterpret_cast<uint32_t*>(slot_e) + lane * words;
+                const float* bs = sBias + hl * HEAD_COLS + p * 32;
 #pragma unroll
-                for (int p = 0; p < 3; ++p) {
-                    // row `lane` of the block, rounded, into the slot (odd word
-                    // counts: conflict-free 4-byte stores)
-                    uint32_t* row = reinterpret_cast<uint32_t*>(slot_e) + lane * words;
-                    const float* bs = sBias + hl * HEAD_COLS + p * 32;
-#pragma unroll
-                    for (int f = 0; f < 16; ++f)
-                        if (2 * f < d)
-                            row[f] = Pack<T>::pk(__uint_as_float(r[p][2 * f]) + bs[2 * f],
-                                                 __uint_as_float(r[p][2 * f + 1]) + bs[2 * f + 1]);
-                    __syncwarp();
-                    // the block is one contiguous run of the head-split output:
-                    // coalesced 16-byte copies out
-                    T* dstp = (p == 0 ? q : (p == 1 ? k : v)) + (((size_t)wi * heads + h) * N + t0) * d;
-                    const uint4* src4 = reinterpret_cast<const uint4*>(slot_e);
-                    uint4* dst4 = reinterpret_cast<uint4*>(dstp);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int c = lane + 32 * i;
-                        if (c < chunks) dst4[c] = src4[c];
+                for (int f = 0; f < 16; ++f)
+                    if (2 * f < d) {
+                        float x0 = __uint_as_float(r[hl][2 * f]), x1 = __uint_as_float(r[hl][2 * f + 1]);
+                        if (biased) {
+                            x0 += bs[2 * f];
+                            x1 += bs[2 * f + 1];
+                        }
+                        row[f] = Pack<T>::pk(x0, x1);
                     }
-                    __syncwarp();  // the slot is read before the next block overwrites it
+                __syncwarp();
+                // the block is one contiguous run of the head-split output:
+                // coalesced 16-byte copies out
+                const uint4* src4 = reinterpret_cast<const uint4*>(slot_e);
+                uint4* dst4 = reinterpret_cast<uint4*>(dst + (((size_t)wi * heads + h) * N + t0) * d);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int c = lane + 32 * i;
+                    if (c < chunks) dst4[c] = src4[c];
                 }
+                __syncwarp();  // the slot is read before the next block overwrites it
             }
         }
     }
