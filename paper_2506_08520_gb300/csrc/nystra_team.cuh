@@ -366,8 +366,20 @@ template <typename T, int M, int NCOL, int PW>
 cudaError_t launch_team(const void* q, const void* k, const void* v, void* out, long long n_units, int d,
                      int iters, cudaStream_t stream, unsigned int* fault, const NystraBias* bias) {
     if constexpr (M <= 16)
-        if (bias)  // a score bias: d_h read at run time
+        if (bias) {  // a score bias: the common head widths compiled in for m = 16 with segment
+                     // landmarks (the common case), d_h read at run time otherwise
+            if constexpr (M != 16 || PW != 0) {
+            } else if constexpr (NCOL == 32) {
+                if (d == 30)
+                    return launch_team_dc<T, M, NCOL, 30, PW, true>(q, k, v, out, n_units, d, iters, stream, fault,
+                                                                      *bias);
+            } else {
+                if (d == 32)
+                    return launch_team_dc<T, M, NCOL, 32, PW, true>(q, k, v, out, n_units, d, iters, stream, fault,
+                                                                      *bias);
+            }
             return launch_team_dc<T, M, NCOL, 0, PW, true>(q, k, v, out, n_units, d, iters, stream, fault, *bias);
+        }
     if constexpr (NCOL == 32) {
         if (d == 30) return launch_team_dc<T, M, NCOL, 30, PW>(q, k, v, out, n_units, d, iters, stream, fault);
     } else {
