@@ -344,20 +344,25 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
             const bool valid = T0 < geo.T;
             const long long wi = T0 / N;
             const int t0 = (int)(T0 - wi * N);
-            // part p of every head of the group in one go: the TMEM loads overlap
-            uint32_t r[2][32];
-            const uint32_t ta = tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)(buf * NTILE + p * 32);
-            t5::ld_32x32b_x32(ta, r[0]);
-            if (HB == 2) t5::ld_32x32b_x32(ta + HEAD_COLS, r[1]);
-            t5::wait_ld();
-            t5::fence_before_sync();  // this warp's TMEM reads of the tile precede the release
-            __syncwarp();
-            if (lane == 0) mbar_arrive(acce + buf);
-            if (!valid) continue;  // warp-uniform
-#pragma unroll
-            for (int hl = 0; hl < 2; ++hl) {
+            if (!valid) {  // rows past the end: release the accumulator and go on (warp-uniform)
+                t5::fence_before_sync();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(acce + buf);
+                continue;
+            }
+#pragma unroll 1
+            for (int hl = 0; hl < HB; ++hl) {
                 const int h = hg * HB + hl;
-                if (hl >= HB || h >= heads) break;  // warp-uniform
+                uint32_t r[32];
+                t5::ld_32x32b_x32(tmem + ((uint32_t)(32 * e) << 16) + (uint32_t)(buf * NTILE + hl * HEAD_COLS + p * 32),
+                                  r);
+                t5::wait_ld();
+                if (hl == HB - 1) {  // this warp's last TMEM read of the tile: release the accumulator
+                    t5::fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(acce + buf);
+                }
+                if (h >= heads) break;  // warp-uniform
                 // row `lane` of the block, rounded, into the slot (odd word
                 // counts: conflict-free 4-byte stores)
                 uint32_t* row = reinterpret_cast<uint32_t*>(slot_e) + lane * words;
@@ -365,7 +370,7 @@ project_qkv_kernel(const T* __restrict__ x, const T* __restrict__ w, const float
 #pragma unroll
                 for (int f = 0; f < 16; ++f)
                     if (2 * f < d) {
-                        float x0 = __uint_as_float(r[hl][2 * f]), x1 = __uint_as_float(r[hl][2 * f + 1]);
+                        float x0 = __uint_as_float(r[2 * f]), x1 = __uint_as_float(r[2 * f + 1]);
                         if (biased) {
                             x0 += bs[2 * f];
                             x1 += bs[2 * f + 1];
