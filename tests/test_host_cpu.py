@@ -4,7 +4,6 @@ oracle on the same inputs: PnP-Nystra within the fp32 bar of 1e-4 per unit
 attention within 1e-5, over both landmark poolings, several shapes, ragged
 sizes and edge cases; results independent of the thread count; argument
 checks."""
-import numpy as np
 import pytest
 import torch
 
