@@ -46,6 +46,28 @@ NYSTRA_API int nystra_attention_host(const float* q, const float* k, const float
                                      int heads, int N, int d_h, int m, int iters, int landmarks, int threads);
 
 /*
+ * nystra_pool_bias_host -- the three landmark blocks of n_bias additive score
+ * biases (the reading of nystra.h's nystra_pool_bias): bias [n_bias, N, N]
+ * in, bias_L [n_bias, N, m], bias_U [n_bias, m, N], bias_A [n_bias, m, m]
+ * out, all fp32 host memory, no overlaps; means over each landmark's tokens.
+ * Returns NYSTRA_OK or NYSTRA_EINVAL.
+ */
+NYSTRA_API int nystra_pool_bias_host(const float* bias, int n_bias, int N, int m, int landmarks, float* bias_L,
+                                     float* bias_U, float* bias_A, int threads);
+
+/*
+ * nystra_attention_bias_host -- nystra_attention_host with a pooled score
+ * bias added to the scaled scores of S_L, S_U and S_A before their row
+ * maxima (nystra.h, nystra_attention_bias).  bias_windows = 1: one slice per
+ * head, shared by every window; = n_windows: one per (window, head) unit.
+ * Returns NYSTRA_OK or NYSTRA_EINVAL (also for a bias that overlaps out).
+ */
+NYSTRA_API int nystra_attention_bias_host(const float* q, const float* k, const float* v, float* out,
+                                          int n_windows, int heads, int N, int d_h, int m, int iters,
+                                          int landmarks, const float* bias_L, const float* bias_U,
+                                          const float* bias_A, int bias_windows, int threads);
+
+/*
  * exact_window_attention_host -- exact softmax attention per unit, Eq. (1)
  * with row-max-shifted exponentials (Eq. 2), on the host cores: the CPU
  * computation PnP-Nystra replaces, for comparison.  Arguments and return

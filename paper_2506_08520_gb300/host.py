@@ -38,6 +38,10 @@ def lib() -> ctypes.CDLL:
         L.nystra_attention_host.restype = i
         L.exact_window_attention_host.argtypes = [vp, vp, vp, vp, i, i, i, i, i]
         L.exact_window_attention_host.restype = i
+        L.nystra_pool_bias_host.argtypes = [vp, i, i, i, i, vp, vp, vp, i]
+        L.nystra_pool_bias_host.restype = i
+        L.nystra_attention_bias_host.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i]
+        L.nystra_attention_bias_host.restype = i
         L.nystra_host_threads.restype = i
         _lib = L
     return _lib
@@ -65,6 +69,40 @@ def nystra(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, m: int = 16, iters
                                      iters, binding.LANDMARKS[landmarks], n_threads)
     if rc != binding.NYSTRA_OK:
         raise RuntimeError(f"nystra_attention_host: status {rc}")
+    return out
+
+
+def pool_bias(bias: torch.Tensor, m: int, landmarks: str = "segments", n_threads: int = 0):
+    """The landmark blocks ``(bias_L [n, N, m], bias_U [n, m, N], bias_A [n, m, m])``
+    of float32 CPU score biases ``bias`` ``[n, N, N]`` (per head, or per window
+    and head), for ``nystra_biased``."""
+    if bias.device.type != "cpu" or bias.dtype != torch.float32 or not bias.is_contiguous() or bias.dim() != 3:
+        raise ValueError("bias must be a contiguous float32 CPU tensor [n, N, N]")
+    n, N, _ = bias.shape
+    L = torch.empty(n, N, m)
+    U = torch.empty(n, m, N)
+    A = torch.empty(n, m, m)
+    rc = lib().nystra_pool_bias_host(bias.data_ptr(), n, N, m, binding.LANDMARKS[landmarks], L.data_ptr(),
+                                     U.data_ptr(), A.data_ptr(), n_threads)
+    if rc != binding.NYSTRA_OK:
+        raise RuntimeError(f"nystra_pool_bias_host: status {rc}")
+    return L, U, A
+
+
+def nystra_biased(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, pooled, m: int = 16, iters: int = 6,
+                  landmarks: str = "segments", out: torch.Tensor | None = None, n_threads: int = 0) -> torch.Tensor:
+    """PnP-Nystra with a pooled score bias (``pool_bias``): slices per head
+    (``heads`` slices, shared by every window) or per window and head."""
+    out = torch.empty_like(q) if out is None else out
+    _check(q, k, v, out)
+    nw, h, N, d = q.shape
+    L, U, A = pooled
+    bw = L.shape[0] // h
+    rc = lib().nystra_attention_bias_host(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), nw, h, N, d, m,
+                                          iters, binding.LANDMARKS[landmarks], L.data_ptr(), U.data_ptr(),
+                                          A.data_ptr(), bw, n_threads)
+    if rc != binding.NYSTRA_OK:
+        raise RuntimeError(f"nystra_attention_bias_host: status {rc}")
     return out
 
 

@@ -149,8 +149,10 @@ static void gemm_tn(const float* A, int lda, const float* B, int ldb, float* C, 
         }
 }
 
+/* One unit.  bL, bU, bA: its pooled score-bias blocks (N x m, m x N, m x m;
+ * all null: no bias), added to the scaled scores before the row maxima. */
 static void one_unit(const float* Q, const float* K, const float* V, float* O, int N, int d, int m, int iters,
-                     Scratch* S) {
+                     const float* bL, const float* bU, const float* bA, Scratch* S) {
     const float s = 1.0f / sqrtf((float)d);
     const int dp = (d + 1 + 15) / 16 * 16;  /* columns of [V | 1] padded for full register blocks */
     /* 1. landmarks: sums over each landmark's tokens, then the mean */
@@ -187,6 +189,7 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
         float* row = S->st + (size_t)t * m;
         for (int i = 0; i < m; ++i) {
             row[i] *= s;
+            if (bU) row[i] += bU[(size_t)i * N + t];
             S->mu[i] = row[i] > S->mu[i] ? row[i] : S->mu[i];
         }
     }
@@ -203,7 +206,9 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
     /* 3. A = exp(s Qbar Kbar^T - m_U), row-wise */
     mm(S->qbar, S->kbarT, S->a, m, d, m);
     for (int i = 0; i < m; ++i)
-        for (int j = 0; j < m; ++j) S->a[(size_t)i * m + j] = expf(s * S->a[(size_t)i * m + j] - S->mu[i]);
+        for (int j = 0; j < m; ++j)
+            S->a[(size_t)i * m + j] =
+                expf(s * S->a[(size_t)i * m + j] + (bA ? bA[(size_t)i * m + j] : 0.f) - S->mu[i]);
     /* 4. Z_0 = A^T / (||A||_1 ||A||_inf), then the iteration */
     float n1 = 0.f, ninf = 0.f;
     for (int j = 0; j < m; ++j) {
@@ -242,6 +247,7 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
         float mx = -INFINITY;
         for (int j = 0; j < m; ++j) {
             row[j] *= s;
+            if (bL) row[j] += bL[(size_t)t * m + j];
             mx = row[j] > mx ? row[j] : mx;
         }
         for (int j = 0; j < m; ++j) row[j] = expf(row[j] - mx);
@@ -269,19 +275,113 @@ static int threads_or_default(int threads) {
 
 int nystra_host_threads(void) { return threads_or_default(0); }
 
+/* Landmark of token t: segments of N/m tokens, or b x b patches of the w x w
+ * window (landmark (row / b) * p + col / b). */
+static int landmark_of(int t, int N, int m, int landmarks, int wdt, int pgrid) {
+    if (landmarks == NYSTRA_LANDMARKS_SEGMENTS) return t / (N / m);
+    const int b = wdt / pgrid, row = t / wdt, col = t % wdt;
+    return (row / b) * pgrid + col / b;
+}
+
+static int shape_ok(int N, int m, int landmarks, int* wdt, int* pgrid) {
+    if (N < 1 || N > MAXN || m < 1 || m > N || m > MAXM || N % m != 0) return 0;
+    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return 0;
+    *wdt = *pgrid = 0;
+    if (landmarks == NYSTRA_LANDMARKS_PATCHES) {
+        *wdt = isqrt_exact(N);
+        *pgrid = isqrt_exact(m);
+        if (*wdt < 0 || *pgrid < 0 || *wdt % *pgrid != 0) return 0;
+    }
+    return 1;
+}
+
+static int attention_host(const float* q, const float* k, const float* v, float* out, int n_windows, int heads,
+                          int N, int d_h, int m, int iters, int landmarks, const float* bias_L, const float* bias_U,
+                          const float* bias_A, int bias_windows, int threads);
+
 int nystra_attention_host(const float* q, const float* k, const float* v, float* out, int n_windows, int heads,
                           int N, int d_h, int m, int iters, int landmarks, int threads) {
-    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
-    if (N < 1 || N > MAXN || d_h < 1 || d_h > MAXD) return NYSTRA_EINVAL;
-    if (m < 1 || m > N || m > MAXM || N % m != 0) return NYSTRA_EINVAL;
-    if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
-    if (landmarks != NYSTRA_LANDMARKS_SEGMENTS && landmarks != NYSTRA_LANDMARKS_PATCHES) return NYSTRA_EINVAL;
-    int wdt = 0, pgrid = 0;
-    if (landmarks == NYSTRA_LANDMARKS_PATCHES) {
-        wdt = isqrt_exact(N);
-        pgrid = isqrt_exact(m);
-        if (wdt < 0 || pgrid < 0 || wdt % pgrid != 0) return NYSTRA_EINVAL;
+    return attention_host(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, NULL, NULL, NULL, 0, threads);
+}
+
+int nystra_attention_bias_host(const float* q, const float* k, const float* v, float* out, int n_windows,
+                               int heads, int N, int d_h, int m, int iters, int landmarks, const float* bias_L,
+                               const float* bias_U, const float* bias_A, int bias_windows, int threads) {
+    if (n_windows > 0 && heads > 0) {
+        if (bias_windows != 1 && bias_windows != n_windows) return NYSTRA_EINVAL;
+        if (!bias_L || !bias_U || !bias_A) return NYSTRA_EINVAL;
+        if (N >= 1 && N <= MAXN && m >= 1 && m <= MAXM && d_h >= 1 && d_h <= MAXD && out) {
+            const size_t ob = (size_t)n_windows * heads * N * d_h * sizeof(float);
+            const size_t nm = (size_t)bias_windows * heads * N * m * sizeof(float);
+            const size_t mm2 = (size_t)bias_windows * heads * m * m * sizeof(float);
+            const uintptr_t o = (uintptr_t)out;
+            if ((o < (uintptr_t)bias_L + nm && (uintptr_t)bias_L < o + ob) ||
+                (o < (uintptr_t)bias_U + nm && (uintptr_t)bias_U < o + ob) ||
+                (o < (uintptr_t)bias_A + mm2 && (uintptr_t)bias_A < o + ob))
+                return NYSTRA_EINVAL;
+        }
     }
+    return attention_host(q, k, v, out, n_windows, heads, N, d_h, m, iters, landmarks, bias_L, bias_U, bias_A,
+                          bias_windows, threads);
+}
+
+int nystra_pool_bias_host(const float* bias, int n_bias, int N, int m, int landmarks, float* bias_L, float* bias_U,
+                          float* bias_A, int threads) {
+    int wdt, pgrid;
+    if (n_bias < 0 || !shape_ok(N, m, landmarks, &wdt, &pgrid)) return NYSTRA_EINVAL;
+    if (n_bias == 0) return NYSTRA_OK;
+    if (!bias || !bias_L || !bias_U || !bias_A) return NYSTRA_EINVAL;
+    const size_t in = (size_t)n_bias * N * N * sizeof(float), nm = (size_t)n_bias * N * m * sizeof(float),
+                 mm2 = (size_t)n_bias * m * m * sizeof(float);
+    const void* outs[3] = {bias_L, bias_U, bias_A};
+    const size_t sz[3] = {nm, nm, mm2};
+    for (int i = 0; i < 3; ++i) {
+        const uintptr_t a = (uintptr_t)outs[i];
+        if (a < (uintptr_t)bias + in && (uintptr_t)bias < a + sz[i]) return NYSTRA_EINVAL;
+        for (int j = i + 1; j < 3; ++j) {
+            const uintptr_t b = (uintptr_t)outs[j];
+            if (a < b + sz[j] && b < a + sz[i]) return NYSTRA_EINVAL;
+        }
+    }
+    const int nt = threads_or_default(threads);
+    const float inv = (float)m / (float)N;  /* 1 / (tokens per landmark) */
+#pragma omp parallel for num_threads(nt) schedule(static)
+    for (int u = 0; u < n_bias; ++u) {
+        const float* B = bias + (size_t)u * N * N;
+        float* L = bias_L + (size_t)u * N * m;
+        float* U = bias_U + (size_t)u * m * N;
+        float* A = bias_A + (size_t)u * m * m;
+        memset(L, 0, sizeof(float) * (size_t)N * m);
+        memset(U, 0, sizeof(float) * (size_t)m * N);
+        memset(A, 0, sizeof(float) * (size_t)m * m);
+        /* sums over each landmark's tokens (as keys for L, as queries for U, both for A), then means */
+        for (int s2 = 0; s2 < N; ++s2) {
+            const int i = landmark_of(s2, N, m, landmarks, wdt, pgrid);
+            for (int t = 0; t < N; ++t) {
+                const float b = B[(size_t)s2 * N + t];
+                const int j = landmark_of(t, N, m, landmarks, wdt, pgrid);
+                L[(size_t)s2 * m + j] += b;
+                U[(size_t)i * N + t] += b;
+                A[(size_t)i * m + j] += b;
+            }
+        }
+        for (size_t e = 0; e < (size_t)N * m; ++e) {
+            L[e] *= inv;
+            U[e] *= inv;
+        }
+        for (int e = 0; e < m * m; ++e) A[e] *= inv * inv;
+    }
+    return NYSTRA_OK;
+}
+
+static int attention_host(const float* q, const float* k, const float* v, float* out, int n_windows, int heads,
+                          int N, int d_h, int m, int iters, int landmarks, const float* bias_L, const float* bias_U,
+                          const float* bias_A, int bias_windows, int threads) {
+    if (n_windows < 0 || heads < 0) return NYSTRA_EINVAL;
+    if (d_h < 1 || d_h > MAXD) return NYSTRA_EINVAL;
+    int wdt = 0, pgrid = 0;
+    if (!shape_ok(N, m, landmarks, &wdt, &pgrid)) return NYSTRA_EINVAL;
+    if (iters < 0 || iters > NYSTRA_MAX_ITERS) return NYSTRA_EINVAL;
     const long long units = (long long)n_windows * heads;
     if (units == 0) return NYSTRA_OK;
     if (!q || !k || !v || !out) return NYSTRA_EINVAL;
@@ -296,19 +396,15 @@ int nystra_attention_host(const float* q, const float* k, const float* v, float*
 #pragma omp atomic write
             status = NYSTRA_EINVAL;
         } else {
-            /* landmark of each token: segments of N/m, or b x b patches of the w x w window */
-            for (int t = 0; t < N; ++t) {
-                if (landmarks == NYSTRA_LANDMARKS_SEGMENTS) {
-                    S->seg[t] = t / (N / m);
-                } else {
-                    const int b = wdt / pgrid, row = t / wdt, col = t % wdt;
-                    S->seg[t] = (row / b) * pgrid + col / b;
-                }
-            }
+            for (int t = 0; t < N; ++t) S->seg[t] = landmark_of(t, N, m, landmarks, wdt, pgrid);
 #pragma omp for schedule(static)
             for (long long u = 0; u < units; ++u) {
                 const size_t off = (size_t)u * N * d_h;
-                one_unit(q + off, k + off, v + off, out + off, N, d_h, m, iters, S);
+                /* the unit's bias slice: its head's (shared) or its own (per window) */
+                const long long sl = bias_L ? (bias_windows == 1 ? u % heads : u) : 0;
+                one_unit(q + off, k + off, v + off, out + off, N, d_h, m, iters,
+                         bias_L ? bias_L + (size_t)sl * N * m : NULL, bias_U ? bias_U + (size_t)sl * m * N : NULL,
+                         bias_A ? bias_A + (size_t)sl * m * m : NULL, S);
             }
             free(S);
         }

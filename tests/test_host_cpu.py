@@ -132,3 +132,51 @@ def test_host_library_exports_every_declared_symbol():
     raw = ctypes.CDLL(host.LIB_PATH)
     for name in names:
         assert hasattr(raw, name), f"{name} declared in nystra_host.h but not exported"
+
+
+@pytest.mark.parametrize("N,m,pool,per_window", [(64, 16, "segments", False), (256, 16, "segments", True),
+                                                 (256, 16, "patches", False), (64, 8, "segments", True)])
+def test_host_score_bias_matches_the_oracle(N, m, pool, per_window):
+    # a relative-position bias (one per head, or one per window and head) pooled
+    # into its landmark blocks on the CPU, then PnP-Nystra with it
+    nw, heads, d = 3, 2, 30
+    w = int(round(N ** 0.5))
+    q, k, v = (x.reshape(nw, heads, N, d).contiguous()
+               for x in workloads.random_qkv(nw * heads, N, d, "f32", seed=N + m))
+    b = torch.from_numpy(workloads.relpos_bias(w, heads, seed=7)).float()  # [heads, N, N]
+    if per_window:
+        b = (b[None] + 0.5 * torch.randn(nw, heads, N, N, generator=torch.Generator().manual_seed(3))).reshape(
+            nw * heads, N, N).contiguous()
+    pooled = host.pool_bias(b.contiguous(), m, pool)
+    got = host.nystra_biased(q, k, v, pooled, m, 6, pool)
+    full = b.reshape(-1, heads, N, N) if per_window else b[None]
+    ref = oracle.nystra_attention(q, k, v, m, 6, pool, full.double().numpy())
+    err = per_unit_rel(_units(got).double().numpy(), _units(torch.from_numpy(ref)).numpy())
+    assert err.max() <= 1e-4, f"max rel err {err.max():.3e}"
+
+
+def test_host_bias_pooling_is_the_landmark_mean():
+    # integer biases: the pooled blocks are exact means over each landmark's tokens
+    N, m = 16, 4
+    b = torch.arange(N * N, dtype=torch.float32).reshape(1, N, N) % 7
+    L, U, A = host.pool_bias(b, m)
+    seg = torch.arange(N) // (N // m)
+    for j in range(m):
+        assert torch.allclose(L[0, :, j], b[0][:, seg == j].mean(1))
+        assert torch.allclose(U[0, j, :], b[0][seg == j, :].mean(0))
+        for i in range(m):
+            assert torch.allclose(A[0, i, j], b[0][seg == i][:, seg == j].mean())
+
+
+def test_host_bias_argument_validation():
+    L = host.lib()
+    P = 1 << 20
+    inv = binding.NYSTRA_EINVAL
+    f = L.nystra_attention_bias_host
+    assert f(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 16, 6, 0, 8 * P, 9 * P, 10 * P, 3, 0) == inv   # bias windows
+    assert f(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 16, 6, 0, 0, 9 * P, 10 * P, 1, 0) == inv       # missing block
+    assert f(P, 2 * P, 3 * P, 64 * P, 4, 2, 64, 30, 16, 6, 0, 64 * P, 9 * P, 10 * P, 1, 0) == inv  # overlaps out
+    g = L.nystra_pool_bias_host
+    assert g(P, 1, 64, 15, 0, 2 * P, 3 * P, 4 * P, 0) == inv     # m does not divide N
+    assert g(P, 1, 64, 16, 0, P, 3 * P, 4 * P, 0) == inv         # output overlaps the bias
+    assert g(P, 0, 64, 16, 0, 2 * P, 3 * P, 4 * P, 0) == binding.NYSTRA_OK
