@@ -344,7 +344,9 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
                 fence_proxy_async_smem();  // this lane's writes precede the bulk store
                 __syncwarp();
                 if (lane == 0) {
-                    bulk_s2g(out + chunk_off(u0 + tk.k * stride, tk.c), X0, xbytes);
+                    // O is not read again: evict it first, keeping L2 for the Q rows the
+                    // output pass reads a second time
+                    bulk_s2g_hint(out + chunk_off(u0 + tk.k * stride, tk.c), X0, xbytes, drop);
                     bulk_commit();
                     bulk_wait_read_all();
                 }

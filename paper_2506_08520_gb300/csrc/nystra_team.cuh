@@ -225,7 +225,8 @@ nystra_team_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* __
         fence_proxy_async_smem();  // this lane's writes precede the bulk store
         __syncwarp();
         if (lane == 0) {
-            bulk_s2g(out + unit_off(uk), Vs, tile_bytes);
+            // O is not read again: evict it first, keeping L2 for the Q rows read twice
+            bulk_s2g_hint(out + unit_off(uk), Vs, tile_bytes, drop);
             bulk_commit();
             bulk_wait_read_all();
         }

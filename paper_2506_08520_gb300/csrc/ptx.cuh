@@ -118,6 +118,12 @@ __device__ __forceinline__ void bulk_s2g(void* dst, const void* src, uint32_t by
                  "r"(bytes)
                  : "memory");
 }
+// bulk_s2g with an L2 cache policy.
+__device__ __forceinline__ void bulk_s2g_hint(void* dst, const void* src, uint32_t bytes, uint64_t policy) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group.L2::cache_hint [%0], [%1], %2, %3;" ::"l"(dst),
+                 "r"(smem_addr(src)), "r"(bytes), "l"(policy)
+                 : "memory");
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 // Wait until every committed bulk store has finished reading its source.
 __device__ __forceinline__ void bulk_wait_read_all() {
