@@ -44,7 +44,7 @@ MEASURED_TRAFFIC = {
         "src_hash": "1b521d4f6ce92163", "bytes": 995_407_360 + 273_398_784},
     "sr720p-w32-m16-bf16": {"files": ["common.cuh", "nystra_stream.cuh", "nystra_tc.cuh", "nystra_tc_n1024.cu",
                                       "ptx.cuh"],
-        "src_hash": "3e140e7c59c01e6c", "bytes": 1_030_307_840 + 284_060_160},
+        "src_hash": "e847d1950a7301d2", "bytes": 1_030_822_656 + 284_172_544},
     "large-w16-m64": {"files": ["common.cuh", "nystra_tc.cuh", "nystra_tc_n256.cu", "nystra_team.cuh", "ptx.cuh"],
         "src_hash": "8e80904b0aac3611", "bytes": 245_142_272},
     "sr720p-w32-m16-bf16-qkv": {"files": ["common.cuh", "nystra_pool.cuh", "nystra_qkv.cuh", "nystra_qkv_stream.cuh",

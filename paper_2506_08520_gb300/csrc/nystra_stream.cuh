@@ -133,7 +133,9 @@ nystra_stream_kernel(const T* __restrict__ q, const T* __restrict__ k, const T* 
     uint64_t* barC = barF + 2;           // C[b]: the core's Y^T is ready
 
     const long long stride = (long long)gridDim.x * Lay::TEAMS;
-    const long long u0 = (long long)blockIdx.x * Lay::TEAMS + team;
+    // team-major numbering: when the units do not divide evenly, the teams with one unit more
+    // sit on different SMs (one per SM) instead of filling the first SMs' every team
+    const long long u0 = (long long)team * gridDim.x + blockIdx.x;
     const int count = u0 < n_units ? (int)((n_units - u0 + stride - 1) / stride) : 0;  // units of this team
 
     if (threadIdx.x == 0) {
