@@ -17,7 +17,8 @@
  *           per unit as G_L^n (Z (G_U^n [V | 1])) with the landmark pooling
  *           and pseudo-inverse iteration of nystra.h (segments or square
  *           patches; Z_0 = A^T/(||A||_1 ||A||_inf), `iters` third-order
- *           steps), all in fp32.
+ *           steps), all in fp32 (exponentials: nystra_host_exp's, within a
+ *           few ulp of exp).
  *  Threads  `threads` OpenMP threads (<= 0: the OpenMP default, normally
  *           every core).  Each unit is computed by one thread in a fixed
  *           order, so results do not depend on the thread count.
@@ -75,6 +76,15 @@ NYSTRA_API int nystra_attention_bias_host(const float* q, const float* k, const 
  */
 NYSTRA_API int exact_window_attention_host(const float* q, const float* k, const float* v, float* out,
                                            int n_windows, int heads, int N, int d_h, int threads);
+
+/*
+ * nystra_host_exp -- test-only: y[i] = exp(x[i]) for i < n, by the
+ * vectorisable exponential every entry point above uses for its softmax
+ * blocks (Cody-Waite range reduction and a degree-7 Taylor polynomial;
+ * arguments are taken as min(x, 88), results below exp(-104) are 0, NaN is
+ * kept).  Host memory, no overlap checks, no return value.
+ */
+NYSTRA_API void nystra_host_exp(const float* x, float* y, int n);
 
 /* Threads the host path uses when `threads` <= 0. */
 NYSTRA_API int nystra_host_threads(void);

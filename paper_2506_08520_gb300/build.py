@@ -79,8 +79,11 @@ def build_host(verbose: bool = False) -> str:
     if os.path.exists(HOST_LIB) and os.path.getmtime(HOST_LIB) >= max(os.path.getmtime(f) for f in deps):
         return HOST_LIB
     tmp = HOST_LIB + f".tmp{os.getpid()}"
-    cmd = [os.environ.get("CC", "gcc"), "-O3", "-std=c11", "-fopenmp", "-fno-math-errno", "-fPIC", "-shared",
-           "-fvisibility=hidden", "-I", INCLUDE, "-o", tmp, HOST_SRC, "-lm"]
+    # -fno-trapping-math lets the softmax loops' selects vectorise; -ffp-contract=fast
+    # lets the compiler fuse multiply-adds where the ISA has them (strict -std=c11
+    # turns that off).  No -ffast-math: the sums are not reassociated.
+    cmd = [os.environ.get("CC", "gcc"), "-O3", "-std=c11", "-fopenmp", "-fno-math-errno", "-fno-trapping-math",
+           "-ffp-contract=fast", "-fPIC", "-shared", "-fvisibility=hidden", "-I", INCLUDE, "-o", tmp, HOST_SRC, "-lm"]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"host library build failed:\n{r.stderr}")

@@ -43,12 +43,23 @@ def lib() -> ctypes.CDLL:
         L.nystra_attention_bias_host.argtypes = [vp, vp, vp, vp, i, i, i, i, i, i, i, vp, vp, vp, i, i]
         L.nystra_attention_bias_host.restype = i
         L.nystra_host_threads.restype = i
+        L.nystra_host_exp.argtypes = [vp, vp, i]
+        L.nystra_host_exp.restype = None
         _lib = L
     return _lib
 
 
 def threads() -> int:
     return lib().nystra_host_threads()
+
+
+def exp(x: torch.Tensor) -> torch.Tensor:
+    """The CPU path's exponential on a contiguous float32 CPU tensor (test-only)."""
+    if x.device.type != "cpu" or x.dtype != torch.float32 or not x.is_contiguous():
+        raise ValueError("exp takes a contiguous float32 CPU tensor")
+    y = torch.empty_like(x)
+    lib().nystra_host_exp(x.data_ptr(), y.data_ptr(), x.numel())
+    return y
 
 
 def _check(q, k, v, out):

@@ -43,10 +43,60 @@ static int overlaps(const void* a, const void* b, size_t bytes) {
     return x < y + bytes && y < x + bytes;
 }
 
+/* exp(x) for x <= 88, written so that a loop of calls vectorises (glibc's
+ * scalar expf does not).  Cody-Waite range reduction (W. J. Cody and W. Waite,
+ * Software Manual for the Elementary Functions, 1980): x = k ln 2 + r with k
+ * the nearest integer to x / ln 2, so |r| <= ln 2 / 2, and ln 2 split into a
+ * 9-bit part whose products with k are exact plus a correction.  exp(r) is
+ * its Taylor series to degree 7 (truncation below 1e-8 relative) in Horner
+ * form, and 2^k is applied as two exact powers of two, so results in the
+ * subnormal range round once.  Arguments below -104 give 0 (exp(-104) is
+ * below half the smallest subnormal); a NaN is returned as it is.  Max error
+ * a few ulp (tested against float64 exp). */
+static inline float exp_cw(float x) {
+    const float xc = x > -104.f ? (x < 88.f ? x : 88.f) : -104.f;
+    const float shifter = 12582912.f;  /* 1.5 * 2^23: adding it rounds to an integer */
+    const float kf = (xc * 1.44269504088896341f + shifter) - shifter;
+    const float r = (xc - kf * 0.693359375f) - kf * -2.12194440054690583e-4f;
+    float p = 1.f / 5040.f;
+    p = p * r + 1.f / 720.f;
+    p = p * r + 1.f / 120.f;
+    p = p * r + 1.f / 24.f;
+    p = p * r + 1.f / 6.f;
+    p = p * r + 0.5f;
+    p = p * r + 1.f;
+    p = p * r + 1.f;
+    const int32_t k = (int32_t)kf, k1 = k / 2, k2 = k - k1;  /* both in [-75, 64] */
+    union { int32_t i; float f; } s1, s2;
+    s1.i = (k1 + 127) * (1 << 23);
+    s2.i = (k2 + 127) * (1 << 23);
+    const float y = p * s1.f * s2.f;
+    return x == x ? y : x;
+}
+
+/* max(x[0..n)) (NaNs skipped), as eight running maxima compared elementwise:
+ * the loop vectorises, and the maximum does not depend on the order. */
+static inline float row_max(const float* x, int n) {
+    float acc[8];
+    for (int b = 0; b < 8; ++b) acc[b] = -INFINITY;
+    int j = 0;
+    for (; j + 8 <= n; j += 8)
+        for (int b = 0; b < 8; ++b) acc[b] = x[j + b] > acc[b] ? x[j + b] : acc[b];
+    float mx = acc[0];
+    for (int b = 1; b < 8; ++b) mx = acc[b] > mx ? acc[b] : mx;
+    for (; j < n; ++j) mx = x[j] > mx ? x[j] : mx;
+    return mx;
+}
+
+void nystra_host_exp(const float* x, float* y, int n) {
+    if (!x || !y) return;
+    for (int i = 0; i < n; ++i) y[i] = exp_cw(x[i]);
+}
+
 /* Per-thread scratch of one unit. */
 typedef struct {
     float qbar[MAXM * MAXD], kbar[MAXM * MAXD];
-    float qbarT[MAXD * MAXM], kbarT[MAXD * MAXM];
+    float qbarT[MAXD * MAXM], kbarT[MAXD * MAXM], kbarTs[MAXD * MAXM];  /* qbar: scaled by s */
     float st[MAXN * MAXM];            /* S_U^T, then G_U^n transposed (N x m) */
     float vp[MAXN * MAXDP];           /* [V | 1 | 0]: d + 1 columns padded to DP, a multiple of 16 */
     float w[MAXM * MAXDP];            /* W = G_U^n [V | 1] (padded columns: zero) */
@@ -172,30 +222,32 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
             kb[c] += kt[c];
         }
     }
+    /* the means; s is folded into Qbar (the scores of S_U and A) and into a
+     * copy of Kbar^T (the scores of S_L), so no pass scales a score block */
     for (int j = 0; j < m; ++j) {
         const float inv = 1.0f / (float)cnt[j];
         for (int c = 0; c < d; ++c) {
             S->qbar[(size_t)j * d + c] *= inv;
             S->kbar[(size_t)j * d + c] *= inv;
+            S->qbar[(size_t)j * d + c] *= s;
             S->qbarT[(size_t)c * m + j] = S->qbar[(size_t)j * d + c];
             S->kbarT[(size_t)c * m + j] = S->kbar[(size_t)j * d + c];
+            S->kbarTs[(size_t)c * m + j] = S->kbar[(size_t)j * d + c] * s;
         }
     }
-    /* 2. S_U^T = K Qbar^T (N x m, scaled by s), the maxima over all N keys,
+    /* 2. S_U^T = K (s Qbar)^T (N x m), the maxima over all N keys,
      *    G_U^n, and W = G_U^n [V | 1] (the ones column: the row sums) */
     gemm_nn(K, d, S->qbarT, m, S->st, m, N, d, m, 0);
     for (int i = 0; i < m; ++i) S->mu[i] = -INFINITY;
     for (int t = 0; t < N; ++t) {
         float* row = S->st + (size_t)t * m;
-        for (int i = 0; i < m; ++i) {
-            row[i] *= s;
-            if (bU) row[i] += bU[(size_t)i * N + t];
-            S->mu[i] = row[i] > S->mu[i] ? row[i] : S->mu[i];
-        }
+        if (bU)
+            for (int i = 0; i < m; ++i) row[i] += bU[(size_t)i * N + t];
+        for (int i = 0; i < m; ++i) S->mu[i] = row[i] > S->mu[i] ? row[i] : S->mu[i];
     }
     for (int t = 0; t < N; ++t) {
         float* row = S->st + (size_t)t * m;
-        for (int i = 0; i < m; ++i) row[i] = expf(row[i] - S->mu[i]);
+        for (int i = 0; i < m; ++i) row[i] = exp_cw(row[i] - S->mu[i]);
         float* vr = S->vp + (size_t)t * dp;
         const float* vt = V + (size_t)t * d;
         for (int c = 0; c < d; ++c) vr[c] = vt[c];
@@ -203,12 +255,12 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
         for (int c = d + 1; c < dp; ++c) vr[c] = 0.f;
     }
     gemm_tn(S->st, m, S->vp, dp, S->w, m, N, dp);
-    /* 3. A = exp(s Qbar Kbar^T - m_U), row-wise */
+    /* 3. A = exp((s Qbar) Kbar^T - m_U), row-wise */
     mm(S->qbar, S->kbarT, S->a, m, d, m);
     for (int i = 0; i < m; ++i)
         for (int j = 0; j < m; ++j)
             S->a[(size_t)i * m + j] =
-                expf(s * S->a[(size_t)i * m + j] + (bA ? bA[(size_t)i * m + j] : 0.f) - S->mu[i]);
+                exp_cw(S->a[(size_t)i * m + j] + (bA ? bA[(size_t)i * m + j] : 0.f) - S->mu[i]);
     /* 4. Z_0 = A^T / (||A||_1 ||A||_inf), then the iteration */
     float n1 = 0.f, ninf = 0.f;
     for (int j = 0; j < m; ++j) {
@@ -239,18 +291,15 @@ static void one_unit(const float* Q, const float* K, const float* V, float* O, i
     }
     /* 5. Y = Z W */
     mm(S->z, S->w, S->y, m, m, dp);
-    /* 6. outputs: S_L = Q Kbar^T (N x m, into st), G_L^n row by row, then
+    /* 6. outputs: S_L = Q (s Kbar)^T (N x m, into st), G_L^n row by row, then
      *    (G_L^n Y) into st's room after it, divided by its last column */
-    gemm_nn(Q, d, S->kbarT, m, S->st, m, N, d, m, 0);
+    gemm_nn(Q, d, S->kbarTs, m, S->st, m, N, d, m, 0);
     for (int t = 0; t < N; ++t) {
         float* row = S->st + (size_t)t * m;
-        float mx = -INFINITY;
-        for (int j = 0; j < m; ++j) {
-            row[j] *= s;
-            if (bL) row[j] += bL[(size_t)t * m + j];
-            mx = row[j] > mx ? row[j] : mx;
-        }
-        for (int j = 0; j < m; ++j) row[j] = expf(row[j] - mx);
+        if (bL)
+            for (int j = 0; j < m; ++j) row[j] += bL[(size_t)t * m + j];
+        const float mx = row_max(row, m);
+        for (int j = 0; j < m; ++j) row[j] = exp_cw(row[j] - mx);
     }
     float* num = S->num;
     for (int t0 = 0; t0 < N; t0 += NBLK) {
@@ -427,7 +476,7 @@ int exact_window_attention_host(const float* q, const float* k, const float* v, 
     const int dp = (d_h + 1 + 15) / 16 * 16;  /* [V | 1] padded for full register blocks */
 #pragma omp parallel num_threads(nt)
     {
-        /* per thread: K^T (d x N), [V | 1 | 0] (N x dp), scores and numerators of a block of queries */
+        /* per thread: s K^T (d x N), [V | 1 | 0] (N x dp), scores and numerators of a block of queries */
         float* kT = (float*)malloc(sizeof(float) * (size_t)MAXD * MAXN);
         float* vp = (float*)malloc(sizeof(float) * (size_t)MAXN * MAXDP);
         float* p = (float*)malloc(sizeof(float) * (size_t)NBLK * MAXN);
@@ -443,7 +492,7 @@ int exact_window_attention_host(const float* q, const float* k, const float* v, 
                 float* O = out + off;
                 for (int t = 0; t < N; ++t) {
                     for (int c = 0; c < d_h; ++c) {
-                        kT[(size_t)c * N + t] = K[(size_t)t * d_h + c];
+                        kT[(size_t)c * N + t] = K[(size_t)t * d_h + c] * s;
                         vp[(size_t)t * dp + c] = V[(size_t)t * d_h + c];
                     }
                     vp[(size_t)t * dp + d_h] = 1.f;  /* the ones column: the softmax denominators */
@@ -451,15 +500,11 @@ int exact_window_attention_host(const float* q, const float* k, const float* v, 
                 }
                 for (int i0 = 0; i0 < N; i0 += NBLK) {
                     const int nb = N - i0 < NBLK ? N - i0 : NBLK;
-                    gemm_nn(Q + (size_t)i0 * d_h, d_h, kT, N, p, N, nb, d_h, N, 0);  /* scores Q K^T */
+                    gemm_nn(Q + (size_t)i0 * d_h, d_h, kT, N, p, N, nb, d_h, N, 0);  /* scores Q (s K)^T */
                     for (int i = 0; i < nb; ++i) {
                         float* pr = p + (size_t)i * N;
-                        float mx = -INFINITY;
-                        for (int t = 0; t < N; ++t) {
-                            pr[t] *= s;
-                            mx = pr[t] > mx ? pr[t] : mx;
-                        }
-                        for (int t = 0; t < N; ++t) pr[t] = expf(pr[t] - mx);
+                        const float mx = row_max(pr, N);
+                        for (int t = 0; t < N; ++t) pr[t] = exp_cw(pr[t] - mx);
                     }
                     gemm_nn(p, N, vp, dp, num, dp, nb, N, dp, 0);  /* exp(scores) [V | 1] */
                     for (int i = 0; i < nb; ++i) {

@@ -121,6 +121,30 @@ def test_host_argument_validation():
         host.nystra(*(torch.zeros(1, 1, 64, 30, dtype=torch.bfloat16) for _ in range(3)))
 
 
+def test_host_exp_is_within_two_ulp_of_exp():
+    # the CPU path's own exponential (Cody-Waite reduction, degree-7 Taylor
+    # polynomial) against float64 exp rounded to float32, over the softmax's
+    # argument range (x <= 0: scores minus their row maximum) into the
+    # subnormal results, and a little above 0
+    import numpy as np
+    x = np.concatenate([np.linspace(-104.0, 2.0, 2_000_003), -np.logspace(-8, 0, 10_001),
+                        np.linspace(-1e-3, 1e-3, 10_001)]).astype(np.float32)
+    y = host.exp(torch.from_numpy(x)).numpy()
+    ref = np.exp(x.astype(np.float64))
+    ref32 = ref.astype(np.float32)
+    ulp = np.spacing(ref32).astype(np.float64)  # float32 spacing (2^-149 in the subnormal range)
+    err = np.abs(y.astype(np.float64) - ref) / ulp
+    assert err.max() <= 2.0, (float(err.max()), float(x[err.argmax()]))
+    # exact and special values
+    sp = torch.tensor([0.0, -0.0, float("-inf"), -105.0, -1e30, float("nan"), -103.9], dtype=torch.float32)
+    ys = host.exp(sp)
+    assert ys[0] == 1.0 and ys[1] == 1.0
+    assert ys[2] == 0.0 and ys[3] == 0.0 and ys[4] == 0.0
+    assert torch.isnan(ys[5])
+    assert 0.0 < ys[6] < 1e-44  # a subnormal result, not flushed
+    assert host.exp(torch.zeros(0)).numel() == 0
+
+
 def test_host_library_exports_every_declared_symbol():
     import ctypes
     import os
