@@ -75,7 +75,8 @@ def build(verbose: bool = False, extra: list[str] | None = None) -> str:
 
 def build_host(verbose: bool = False) -> str:
     """Compile the multi-core CPU path into ``libnystra_host.so``."""
-    deps = [HOST_SRC, os.path.join(INCLUDE, "nystra_host.h"), os.path.join(INCLUDE, "nystra.h")]
+    deps = [HOST_SRC, os.path.join(INCLUDE, "nystra_host.h"), os.path.join(INCLUDE, "nystra.h"),
+            os.path.abspath(__file__)]  # the flags below
     if os.path.exists(HOST_LIB) and os.path.getmtime(HOST_LIB) >= max(os.path.getmtime(f) for f in deps):
         return HOST_LIB
     tmp = HOST_LIB + f".tmp{os.getpid()}"
